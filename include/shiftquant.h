@@ -1,0 +1,186 @@
+/*
+ * shiftquant.h -- C ABI of the GB300 (sm_103a) ShiftQuant library, libshiftquant.so.
+ *
+ * ShiftQuant is the quantizer of "Towards Accurate and Efficient Sub-8-Bit Integer
+ * Training" (arXiv 2411.10948).  One quantized linear layer Y = X W runs as
+ *
+ *   forward          Y  = X  W      X: ShiftQuant over its channels (the inner dim),
+ *                                   W: per-out-channel                     (Sec. 5.1)
+ *   loss propagation dX = dY W^T    dY: ShiftQuant over its channels (the inner dim),
+ *                                   W: per-in-channel                       (Eq. 4)
+ *   weight gradient  dW = X^T dY    both operands reuse their ShiftQuant codes; the
+ *                                   inner dim is the token axis
+ *
+ * and each ShiftQuant tensor goes through: a range pass (per-channel max|x|, Sec. 3.1),
+ * the power-of-two grouping (Eq. 3: channel c gets exponent e_c, its group, with
+ * tau_0 2^-(e_c+1) < r_c <= tau_0 2^-e_c), and quantization with step
+ * s 2^-e_c, s = tau_0 / Q, Q = 2^(b-1) - 1 (App. D).  The contraction applies the
+ * group shift to every product before accumulation (ShiftMM, Sec. 3.2 and the
+ * left-shift form of App. D), then one dequantizing multiply.
+ *
+ * Conventions for every entry point
+ *   - Every pointer is a DEVICE pointer unless the argument says otherwise.  The caller
+ *     owns every buffer; the library never allocates device memory and never
+ *     synchronises.  Calls are asynchronous and ordered on `stream` (a cudaStream_t
+ *     passed as void*; NULL is the legacy default stream).
+ *   - Matrices are row-major with an explicit leading dimension `ld*` in ELEMENTS.
+ *   - Host-detectable errors (bad sizes, NULL pointers, alignment, unsupported
+ *     bit/group combinations) return a negative sq_status before anything is launched;
+ *     shiftquant_last_error() then holds a message (per host thread).
+ *   - Device-detected conditions are OR-ed into the caller's int32 `dev_status` word
+ *     (SQ_DEV_* bits), which the caller zeroes and reads after synchronising.
+ *   - Codes are the signed integers q, |q| <= Q, stored in the operand format of the
+ *     float tensor-core MMA that multiplies them exactly (sm_103a has no integer MMA):
+ *     one byte FP8 E4M3 or two bytes BF16, see shiftquant_code_type().  Every stored
+ *     value is an integer (times a power of two for weight codes) and is exact.
+ */
+#ifndef SHIFTQUANT_H
+#define SHIFTQUANT_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef int sq_status;
+#define SQ_OK 0
+#define SQ_EINVAL (-1)        /* bad size, NULL pointer, bad enum value */
+#define SQ_EALIGN (-2)        /* pointer or leading dimension breaks a 16-byte rule */
+#define SQ_EUNSUPPORTED (-3)  /* bit/group/size combination outside the exact range */
+#define SQ_ECUDA (-4)         /* a CUDA runtime call failed (message has the name) */
+
+/* bits OR-ed into *dev_status by the kernels */
+#define SQ_DEV_NONFINITE 1    /* a NaN or Inf was met in the range pass */
+#define SQ_DEV_TIMEOUT 2      /* a pipeline wait gave up (about 1 s); outputs invalid */
+
+typedef enum { SQ_ROUND_NEAREST_EVEN = 0, SQ_ROUND_STOCHASTIC = 1 } sq_round;
+
+/* Granularity of a quantizer call.
+ *   SQ_GRAN_SHIFT   ShiftQuant over the columns (the channel axis) of an activation or
+ *                   gradient [rows = tokens, cols = channels].
+ *   SQ_GRAN_PER_COL one scale per column: a weight W [K, N] in the forward GEMM
+ *                   (per-out-channel, Sec. 5.1).
+ *   SQ_GRAN_PER_ROW one scale per row: a weight W [K, N] in the loss-propagation GEMM
+ *                   (per-in-channel, Sec. 5.1). */
+typedef enum { SQ_GRAN_SHIFT = 0, SQ_GRAN_PER_COL = 1, SQ_GRAN_PER_ROW = 2 } sq_gran;
+
+typedef enum { SQ_CODE_E4M3 = 0, SQ_CODE_BF16 = 1 } sq_code_type;
+
+/* Storage type of the codes for `bits` in [2, 8] and `n_groups` (N_G) in [1, 8]:
+ * FP8 E4M3 when Q <= 15 and the largest shifted weight code Q 2^(N_G-1) <= 448 (the
+ * exactly representable integers of E4M3), else BF16.  Returns a negative sq_status
+ * for out-of-range arguments. */
+int shiftquant_code_type(int bits, int n_groups);
+
+/* Bytes per stored code (1 or 2), or a negative sq_status. */
+int shiftquant_code_bytes(int bits, int n_groups);
+
+/* Range pass and grouping (Sec. 3.1, Eq. 3).
+ *   x [rows, ld] fp32.
+ *   gran == SQ_GRAN_SHIFT: range_out[cols] = max_r |x[r, c]|, *tau0_out = max_c of it
+ *     (r_max of Eq. 1), exp_out[cols] = e_c = min(n_groups-1, floor(log2(tau0/r_c)))
+ *     computed exactly (a zero channel gets n_groups-1).
+ *   gran == SQ_GRAN_PER_COL: range_out[cols] only; tau0_out and exp_out may be NULL.
+ *   gran == SQ_GRAN_PER_ROW: range_out[rows] = max_c |x[r, c]|; the others may be NULL.
+ *   A NaN/Inf anywhere sets SQ_DEV_NONFINITE; tau0 is then NaN or Inf and every e_c 0.
+ *   rows or cols == 0 is allowed (tau0 = 0). */
+sq_status shiftquant_calibrate(const float *x, int64_t rows, int64_t cols, int64_t ld,
+                               int gran, int n_groups, float *range_out, float *tau0_out,
+                               uint8_t *exp_out, int32_t *dev_status, void *stream);
+
+/* Quantization (App. D; stochastic rounding of App. B).
+ *   x [rows, ld] fp32, bits in [2, 8], Q = 2^(bits-1) - 1.
+ *   gran == SQ_GRAN_SHIFT: range_or_tau0 -> the device scalar tau_0 and exp[cols] from
+ *     shiftquant_calibrate; q[r, c] = round(x 2^e_c Q / tau_0); *scale_out = tau_0 / Q.
+ *     fold_exp must be NULL.
+ *   gran == SQ_GRAN_PER_COL: range_or_tau0 -> range[cols]; q = round(x Q / range[c]);
+ *     scale_out[cols] = range[c] / Q.  fold_exp, if not NULL, is indexed by ROW.
+ *   gran == SQ_GRAN_PER_ROW: range_or_tau0 -> range[rows]; scale_out[rows].
+ *     fold_exp, if not NULL, is indexed by COLUMN.
+ *   fold_exp: the group exponents of the OTHER operand along this weight's GEMM inner
+ *     index; the stored value becomes q 2^(n_groups-1-fold_exp[i]), which is how the
+ *     ShiftMM shift of Eq. 4 enters the contraction at no cost.
+ *   mode: SQ_ROUND_NEAREST_EVEN (ties to even) or SQ_ROUND_STOCHASTIC: up with
+ *     probability frac(v) using u = (SplitMix64(seed + (idx+1) 0x9E3779B97F4A7C15) >> 40)
+ *     2^-24, idx = r * cols + c.
+ *   Outputs (codes in the type of shiftquant_code_type(bits, n_groups)):
+ *     codes [rows, ld_codes] (may be NULL), codes_t [cols, ld_t], the transpose (may be
+ *     NULL); at least one must be given.  tau_0 == 0 (or Q/tau_0 overflowing) gives
+ *     all-zero codes and a zero scale; likewise per channel. */
+sq_status shiftquant_quantize(const float *x, int64_t rows, int64_t cols, int64_t ld,
+                              int gran, int bits, int n_groups, const float *range_or_tau0,
+                              const uint8_t *exp, const uint8_t *fold_exp, int mode,
+                              uint64_t seed, void *codes, int64_t ld_codes, void *codes_t,
+                              int64_t ld_t, float *scale_out, void *stream);
+
+/* Forward GEMM Y[M, N] = X[M, K] W[K, N] on quantized operands (Eq. 4 with the roles of
+ * Sec. 5.1):
+ *   a_codes [M, lda]: ShiftQuant codes of X (SQ_GRAN_SHIFT, unshifted), a_scale: device
+ *     scalar s_X.
+ *   b_codes [N, ldb]: per-out-channel codes of W stored TRANSPOSED (codes_t of a
+ *     SQ_GRAN_PER_COL call with fold_exp = X's exponents), b_scale[N] = s_W.
+ *   Result: T[m, n] = sum_k q_X[m, k] q_W[k, n] 2^(G-1-e_k) exactly (int32, see the
+ *     limits below), Y = float(T) * (s_X 2^-(G-1) * s_W[n]).
+ *   acc_out [M, ld_acc] int64 (may be NULL): T itself, for exactness checks.
+ *   workspace: optional int32 scratch of shiftquant_gemm_workspace_bytes() bytes; with
+ *     it, a GEMM with too few output tiles splits K across SMs; NULL never splits.
+ *   Alignment: lda * code_bytes and ldb * code_bytes multiples of 16, code pointers
+ *     16-byte aligned (the operands are read by TMA).
+ *   Limits: max|q_X| max|q_W| 2^(G-1) K < 2^31 (the exact int32 range); larger K returns
+ *     SQ_EUNSUPPORTED.  M, N or K == 0 is allowed. */
+sq_status shiftquant_gemm_fwd(const void *a_codes, int64_t lda, const float *a_scale,
+                              const void *b_codes, int64_t ldb, const float *b_scale,
+                              int64_t M, int64_t N, int64_t K, int bits, int n_groups,
+                              float *y, int64_t ldy, int64_t *acc_out, int64_t ld_acc,
+                              void *workspace, size_t workspace_bytes, int32_t *dev_status,
+                              void *stream);
+
+/* Loss-propagation GEMM dX[M, K] = dY[M, N] W^T (Eq. 4 as printed):
+ *   a_codes [M, lda]: ShiftQuant codes of dY (inner dim N), a_scale: s_dY.
+ *   b_codes [K, ldb]: per-in-channel codes of W [K, N] in their natural layout (codes of
+ *     a SQ_GRAN_PER_ROW call with fold_exp = dY's exponents), b_scale[K].
+ *   In the argument list below the GEMM is written as out[M, N_out] = a [M, K_in] b^T with
+ *   N_out = K (W's in-channels) and K_in = N (dY's channels); everything else is as for
+ *   shiftquant_gemm_fwd. */
+sq_status shiftquant_gemm_dgrad(const void *a_codes, int64_t lda, const float *a_scale,
+                                const void *b_codes, int64_t ldb, const float *b_scale,
+                                int64_t M, int64_t N_out, int64_t K_in, int bits,
+                                int n_groups, float *dx, int64_t ldx, int64_t *acc_out,
+                                int64_t ld_acc, void *workspace, size_t workspace_bytes,
+                                int32_t *dev_status, void *stream);
+
+/* Weight-gradient GEMM dW[Ci, Co] = X^T dY over T tokens:
+ *   xt_codes [Ci, ldx]: the transposed ShiftQuant codes of X (codes_t), x_scale s_X,
+ *     x_exp[Ci] its group exponents.
+ *   gt_codes [Co, ldg]: the transposed ShiftQuant codes of dY, g_scale, g_exp[Co].
+ *   Both channel axes are outer dims here, so each group shift applies to the whole
+ *   inner sum: T[i, j] = (sum_t q_X[t, i] q_dY[t, j]) 2^((G-1-eX_i) + (G-1-eY_j)) and
+ *   dW = float(sum) * (s_X s_dY) 2^-(eX_i + eY_j).  acc_out receives T (int64).
+ *   Limits: max|q_X| max|q_dY| T < 2^31. */
+sq_status shiftquant_gemm_wgrad(const void *xt_codes, int64_t ldx, const float *x_scale,
+                                const uint8_t *x_exp, const void *gt_codes, int64_t ldg,
+                                const float *g_scale, const uint8_t *g_exp, int64_t Ci,
+                                int64_t Co, int64_t T, int bits, int n_groups, float *dw,
+                                int64_t ld_dw, int64_t *acc_out, int64_t ld_acc,
+                                void *workspace, size_t workspace_bytes,
+                                int32_t *dev_status, void *stream);
+
+/* Bytes of int32 scratch that lets a GEMM of this shape split its inner dimension across
+ * SMs on the current device (0 when it would not split).  which: 0 fwd, 1 dgrad,
+ * 2 wgrad; M, N are the output dims and K the inner dim. */
+size_t shiftquant_gemm_workspace_bytes(int which, int64_t M, int64_t N, int64_t K,
+                                       int bits, int n_groups);
+
+/* Static description of a status code. */
+const char *shiftquant_status_string(sq_status status);
+
+/* Message of the last host-side error on this thread ("" if none). */
+const char *shiftquant_last_error(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* SHIFTQUANT_H */

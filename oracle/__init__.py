@@ -50,6 +50,8 @@ def _load():
         lib = ctypes.CDLL(build())
         i64, i32, u64, f32 = ctypes.c_int64, ctypes.c_int, ctypes.c_uint64, ctypes.c_float
         vp = ctypes.c_void_p
+        lib.sqo_max_threads.argtypes = []
+        lib.sqo_max_threads.restype = i32
         lib.sqo_hash.argtypes = [u64, u64]
         lib.sqo_hash.restype = u64
         lib.sqo_range_cols.argtypes = [vp, i64, i64, i64, vp]
@@ -87,6 +89,11 @@ def _rows(rows):
         return None, 0
     r = np.ascontiguousarray(rows, dtype=np.int64)
     return r, int(r.size)
+
+
+def max_threads() -> int:
+    """Threads the oracle's OpenMP loops use."""
+    return int(_load().sqo_max_threads())
 
 
 # ---------------------------------------------------------------- hash (SR draws)

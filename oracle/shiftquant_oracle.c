@@ -36,12 +36,24 @@
  *       A NaN or Inf in the input sets the non-finite status; exponents are then 0.
  */
 #include <math.h>
+#ifdef _OPENMP
+#include <omp.h>
+#endif
 #include <stdint.h>
 #include <stdlib.h>
 #include <string.h>
 
 #define SQO_OK 0
 #define SQO_NONFINITE 1
+
+/* threads the OpenMP loops of this file use (reported beside oracle timings) */
+int sqo_max_threads(void) {
+#ifdef _OPENMP
+    return omp_get_max_threads();
+#else
+    return 1;
+#endif
+}
 
 /* ---------------------------------------------------------------- R6: hash */
 /* SplitMix64 output function applied to the (idx+1)-th state of a generator seeded

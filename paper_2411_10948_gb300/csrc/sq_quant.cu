@@ -1,0 +1,571 @@
+// ShiftQuant quantizer kernels for sm_103a and their C entry points.
+//
+//   range pass  (Sec. 3.1)   per-column max|x| with 128-bit loads and an atomic max on the
+//                            bit pattern of the non-negative float; per-row max for the
+//                            per-in-channel weight role
+//   grouping    (Eq. 3)      tau_0 = max_c r_c, e_c = the largest e <= N_G-1 with
+//                            r_c 2^e <= tau_0, i.e. floor(log2(tau_0 / r_c)) clipped
+//   quantize    (App. D/B)   q = round(x 2^e_c Q / tau_0) with round-to-nearest-even or
+//                            stochastic rounding on a counter-based SplitMix64 draw;
+//                            optional shift of weight codes by 2^(N_G-1-e) (ShiftMM)
+//
+// All three are HBM-bound streaming passes.  The quantizer writes the codes directly in
+// the operand format of the tensor-core GEMM (E4M3 or BF16, exact integers) and, in the
+// same pass, the transposed copy the weight-gradient GEMM reads, staged through shared
+// memory so both writes stay coalesced.
+#include <cuda_fp8.h>
+#include <cuda_runtime.h>
+
+#include <cstdarg>
+#include <cstdio>
+
+#include "sq_device.cuh"
+#include "sq_host.h"
+
+namespace sq {
+
+static thread_local char g_last_error[512];
+
+int fail(int status, const char* fmt, ...) {
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(g_last_error, sizeof g_last_error, fmt, ap);
+  va_end(ap);
+  return status;
+}
+
+static void clear_error() { g_last_error[0] = 0; }
+
+static int num_sms() {
+  int dev = 0, n = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return 148;
+  if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 148;
+  return n > 0 ? n : 148;
+}
+
+// ===================================================================== range pass
+constexpr int kColTx = 32;  // threads along columns, 4 columns each: 128 columns per block
+constexpr int kColTy = 8;   // threads along rows
+
+__device__ __forceinline__ uint32_t abs_bits(float v) { return __float_as_uint(v) & 0x7FFFFFFFu; }
+
+// range_bits[c] = max over this block's rows of |x[r, c]| as an ordered bit pattern
+// (for non-negative floats, larger value <=> larger unsigned pattern; NaN sorts above Inf).
+__global__ void __launch_bounds__(kColTx* kColTy)
+    colmax_kernel(const float* __restrict__ x, int64_t R, int64_t C, int64_t ld,
+                  int64_t rows_per_block, int vec, unsigned* __restrict__ range_bits,
+                  int* __restrict__ status) {
+  __shared__ unsigned red[kColTy][kColTx * 4];
+  const int tx = threadIdx.x, ty = threadIdx.y;
+  const int64_t c0 = (static_cast<int64_t>(blockIdx.x) * kColTx + tx) * 4;
+  const int64_t rb = static_cast<int64_t>(blockIdx.y) * rows_per_block;
+  const int64_t re = min(R, rb + rows_per_block);
+  unsigned m0 = 0, m1 = 0, m2 = 0, m3 = 0;
+  if (vec && c0 + 3 < C) {
+    const float* base = x + c0;
+    int64_t r = rb + ty;
+#pragma unroll 1
+    for (; r + 3 * kColTy < re; r += 4 * kColTy) {
+      float4 v[4];
+#pragma unroll
+      for (int u = 0; u < 4; ++u)
+        v[u] = __ldg(reinterpret_cast<const float4*>(base + (r + u * kColTy) * ld));
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        m0 = max(m0, abs_bits(v[u].x));
+        m1 = max(m1, abs_bits(v[u].y));
+        m2 = max(m2, abs_bits(v[u].z));
+        m3 = max(m3, abs_bits(v[u].w));
+      }
+    }
+#pragma unroll 1
+    for (; r < re; r += kColTy) {
+      const float4 v = __ldg(reinterpret_cast<const float4*>(base + r * ld));
+      m0 = max(m0, abs_bits(v.x));
+      m1 = max(m1, abs_bits(v.y));
+      m2 = max(m2, abs_bits(v.z));
+      m3 = max(m3, abs_bits(v.w));
+    }
+  } else {
+#pragma unroll 1
+    for (int64_t r = rb + ty; r < re; r += kColTy) {
+      const float* row = x + r * ld;
+      if (c0 + 0 < C) m0 = max(m0, abs_bits(__ldg(row + c0 + 0)));
+      if (c0 + 1 < C) m1 = max(m1, abs_bits(__ldg(row + c0 + 1)));
+      if (c0 + 2 < C) m2 = max(m2, abs_bits(__ldg(row + c0 + 2)));
+      if (c0 + 3 < C) m3 = max(m3, abs_bits(__ldg(row + c0 + 3)));
+    }
+  }
+  red[ty][tx * 4 + 0] = m0;
+  red[ty][tx * 4 + 1] = m1;
+  red[ty][tx * 4 + 2] = m2;
+  red[ty][tx * 4 + 3] = m3;
+  __syncthreads();
+  if (ty == 0) {
+    bool bad = false;
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      unsigned m = 0;
+#pragma unroll
+      for (int y = 0; y < kColTy; ++y) m = max(m, red[y][tx * 4 + i]);
+      if (c0 + i < C && m != 0) {
+        atomicMax(range_bits + c0 + i, m);
+        bad |= m >= 0x7F800000u;
+      }
+    }
+    if (bad) atomicOr(status, kDevNonFinite);
+  }
+}
+
+// one warp per row: range[r] = max_c |x[r, c]|
+__global__ void __launch_bounds__(256)
+    rowmax_kernel(const float* __restrict__ x, int64_t R, int64_t C, int64_t ld, int vec,
+                  float* __restrict__ range, int* __restrict__ status) {
+  const int lane = threadIdx.x & 31;
+  const int64_t r = static_cast<int64_t>(blockIdx.x) * (blockDim.x / 32) + (threadIdx.x >> 5);
+  if (r >= R) return;
+  const float* row = x + r * ld;
+  unsigned m = 0;
+  int64_t c = 0;
+  if (vec) {
+    const int64_t c4 = C & ~int64_t(3);
+#pragma unroll 4
+    for (int64_t cc = lane * 4; cc < c4; cc += 128) {
+      const float4 v = __ldg(reinterpret_cast<const float4*>(row + cc));
+      m = max(max(m, abs_bits(v.x)), max(abs_bits(v.y), max(abs_bits(v.z), abs_bits(v.w))));
+    }
+    c = c4;
+  }
+  for (int64_t cc = c + lane; cc < C; cc += 32) m = max(m, abs_bits(__ldg(row + cc)));
+  m = __reduce_max_sync(0xFFFFFFFFu, m);
+  if (lane == 0) {
+    range[r] = __uint_as_float(m);
+    if (m >= 0x7F800000u) atomicOr(status, kDevNonFinite);
+  }
+}
+
+// tau_0 and the exponents.  e_c = max{e in [0, G-1] : r_c 2^e <= tau_0}; the product by
+// 2^e is exact (no rounding) for every finite r_c <= tau_0, so the comparison is exact.
+__global__ void __launch_bounds__(1024)
+    group_kernel(const unsigned* __restrict__ range_bits, int64_t C, int G,
+                 float* __restrict__ tau0_out, uint8_t* __restrict__ exp_out,
+                 int* __restrict__ status) {
+  __shared__ unsigned warp_max[32];
+  __shared__ unsigned tau_bits_s;
+  unsigned m = 0;
+  for (int64_t c = threadIdx.x; c < C; c += blockDim.x) m = max(m, range_bits[c]);
+  m = __reduce_max_sync(0xFFFFFFFFu, m);
+  if ((threadIdx.x & 31) == 0) warp_max[threadIdx.x >> 5] = m;
+  __syncthreads();
+  if (threadIdx.x < 32) {
+    unsigned v = threadIdx.x < (blockDim.x >> 5) ? warp_max[threadIdx.x] : 0u;
+    v = __reduce_max_sync(0xFFFFFFFFu, v);
+    if (threadIdx.x == 0) tau_bits_s = v;
+  }
+  __syncthreads();
+  const unsigned tb = tau_bits_s;
+  const float tau = __uint_as_float(tb);
+  const bool nonfinite = tb >= 0x7F800000u;
+  if (threadIdx.x == 0) {
+    *tau0_out = tau;
+    if (nonfinite) atomicOr(status, kDevNonFinite);
+  }
+  for (int64_t c = threadIdx.x; c < C; c += blockDim.x) {
+    const float r = __uint_as_float(range_bits[c]);
+    int e = 0;
+    if (!nonfinite) {
+      if (r == 0.0f) {
+        e = G - 1;
+      } else {
+#pragma unroll 1
+        for (int k = 1; k < G; ++k) {
+          const float scaled = __fmul_rn(r, __int_as_float((127 + k) << 23));  // r 2^k
+          if (scaled <= tau) e = k;
+          else break;
+        }
+      }
+    }
+    exp_out[c] = static_cast<uint8_t>(e);
+  }
+}
+
+// ======================================================================= quantize
+struct QuantArgs {
+  const float* x;
+  int64_t R, C, ld;
+  int gran, Q, G, mode;
+  uint64_t seed;
+  const float* rt;        // &tau_0 (SHIFT) or range[] (PER_COL / PER_ROW)
+  const uint8_t* exp;     // SHIFT: e_c
+  const uint8_t* fold;    // optional: exponents of the other GEMM operand
+  void* codes;
+  int64_t ldc;
+  void* codes_t;
+  int64_t ldt;
+  float* scale_out;
+  int vec_in, vec_out, vec_t;
+};
+
+// SplitMix64 (Steele, Lea, Flood 2014): the (idx+1)-th output of the generator whose
+// state starts at `seed`.
+__device__ __forceinline__ uint64_t splitmix64_at(uint64_t seed, uint64_t idx) {
+  uint64_t z = seed + (idx + 1ull) * 0x9E3779B97F4A7C15ull;
+  z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
+  z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+  return z ^ (z >> 31);
+}
+
+__device__ __forceinline__ float pow2f(int k) { return __int_as_float((127 + k) << 23); }
+
+template <typename CodeT>
+__device__ __forceinline__ CodeT encode_code(float v);
+
+template <>
+__device__ __forceinline__ uint16_t encode_code<uint16_t>(float v) {
+  // v is an integer with at most 8 significant bits: the top half of its binary32
+  // pattern is its exact BF16 pattern
+  return static_cast<uint16_t>(__float_as_uint(v) >> 16);
+}
+
+template <>
+__device__ __forceinline__ uint8_t encode_code<uint8_t>(float v) {
+  return static_cast<uint8_t>(__nv_cvt_float_to_fp8(v, __NV_SATFINITE, __NV_E4M3));
+}
+
+constexpr int kQT = 64;  // quantize tile: 64 rows x 64 columns, 256 threads
+
+template <typename CodeT>
+__global__ void __launch_bounds__(256) quantize_kernel(const QuantArgs a) {
+  constexpr int kPad = 16 / sizeof(CodeT);
+  __shared__ __align__(16) CodeT tile_t[kQT][kQT + kPad];  // [column][row]
+  const int tid = threadIdx.x;
+  const int cq = tid & 15;
+  const int rq = tid >> 4;
+  const int64_t r0 = static_cast<int64_t>(blockIdx.y) * kQT;
+  const int64_t c0 = static_cast<int64_t>(blockIdx.x) * kQT;
+  const int64_t cb = c0 + cq * 4;
+  const float Qf = static_cast<float>(a.Q);
+
+  // per-column multipliers: 2^e_c (SHIFT) or Q / range_c (PER_COL)
+  float colmul[4];
+  bool colzero[4];
+  int colfold[4];
+  float invS = 0.0f;
+  bool zero_all = false;
+  if (a.gran == SQ_GRAN_SHIFT) {
+    const float tau = __ldg(a.rt);
+    invS = __fdiv_rn(Qf, tau);
+    zero_all = !(tau > 0.0f) || !isfinite(tau) || !isfinite(invS);
+  }
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const int64_t c = cb + i;
+    colmul[i] = 1.0f;
+    colzero[i] = false;
+    colfold[i] = 0;
+    if (c < a.C) {
+      if (a.gran == SQ_GRAN_SHIFT) {
+        colmul[i] = pow2f(__ldg(a.exp + c));
+      } else if (a.gran == SQ_GRAN_PER_COL) {
+        const float rg = __ldg(a.rt + c);
+        colmul[i] = __fdiv_rn(Qf, rg);
+        colzero[i] = !(rg > 0.0f) || !isfinite(rg) || !isfinite(colmul[i]);
+      }
+      if (a.gran == SQ_GRAN_PER_ROW && a.fold) colfold[i] = a.G - 1 - __ldg(a.fold + c);
+    }
+  }
+
+#pragma unroll 1
+  for (int pass = 0; pass < 4; ++pass) {
+    const int lr = rq + 16 * pass;
+    const int64_t r = r0 + lr;
+    float xv[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+    float rowmul = 1.0f;
+    bool rowzero = false;
+    int rowfold = 0;
+    if (r < a.R) {
+      const float* row = a.x + r * a.ld;
+      if (a.vec_in && cb + 3 < a.C) {
+        const float4 v = __ldg(reinterpret_cast<const float4*>(row + cb));
+        xv[0] = v.x;
+        xv[1] = v.y;
+        xv[2] = v.z;
+        xv[3] = v.w;
+      } else {
+#pragma unroll
+        for (int i = 0; i < 4; ++i)
+          if (cb + i < a.C) xv[i] = __ldg(row + cb + i);
+      }
+      if (a.gran == SQ_GRAN_PER_ROW) {
+        const float rg = __ldg(a.rt + r);
+        rowmul = __fdiv_rn(Qf, rg);
+        rowzero = !(rg > 0.0f) || !isfinite(rg) || !isfinite(rowmul);
+      }
+      if (a.gran == SQ_GRAN_PER_COL && a.fold) rowfold = a.G - 1 - __ldg(a.fold + r);
+    }
+    CodeT out[4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const int64_t c = cb + i;
+      float v;
+      bool z;
+      if (a.gran == SQ_GRAN_SHIFT) {
+        v = __fmul_rn(__fmul_rn(xv[i], colmul[i]), invS);  // x 2^e exactly, then * Q/tau
+        z = zero_all;
+      } else if (a.gran == SQ_GRAN_PER_COL) {
+        v = __fmul_rn(xv[i], colmul[i]);
+        z = colzero[i];
+      } else {
+        v = __fmul_rn(xv[i], rowmul);
+        z = rowzero;
+      }
+      float q = 0.0f;
+      if (!z && r < a.R && c < a.C) {
+        if (a.mode == SQ_ROUND_NEAREST_EVEN) {
+          q = rintf(v);
+        } else {
+          const float l = floorf(v);
+          const float frac = __fsub_rn(v, l);
+          const uint64_t h = splitmix64_at(a.seed, static_cast<uint64_t>(r * a.C + c));
+          const float u = __fmul_rn(static_cast<float>(static_cast<uint32_t>(h >> 40)),
+                                    5.9604644775390625e-08f);  // * 2^-24, exact
+          q = (u < frac) ? __fadd_rn(l, 1.0f) : l;
+        }
+        q = fminf(fmaxf(q, -Qf), Qf);
+      }
+      const int f = (a.gran == SQ_GRAN_PER_ROW) ? colfold[i] : rowfold;
+      const float val = __fadd_rn(__fmul_rn(q, pow2f(f)), 0.0f);  // +0 for a zero code
+      out[i] = encode_code<CodeT>(val);
+      tile_t[cq * 4 + i][lr] = out[i];
+    }
+    if (a.codes && r < a.R) {
+      CodeT* dst = static_cast<CodeT*>(a.codes) + r * a.ldc + cb;
+      if (a.vec_out && cb + 3 < a.C) {
+        if constexpr (sizeof(CodeT) == 2) {
+          uint2 w;
+          w.x = static_cast<uint32_t>(out[0]) | (static_cast<uint32_t>(out[1]) << 16);
+          w.y = static_cast<uint32_t>(out[2]) | (static_cast<uint32_t>(out[3]) << 16);
+          *reinterpret_cast<uint2*>(dst) = w;
+        } else {
+          const uint32_t w = static_cast<uint32_t>(out[0]) | (static_cast<uint32_t>(out[1]) << 8) |
+                             (static_cast<uint32_t>(out[2]) << 16) |
+                             (static_cast<uint32_t>(out[3]) << 24);
+          *reinterpret_cast<uint32_t*>(dst) = w;
+        }
+      } else {
+#pragma unroll
+        for (int i = 0; i < 4; ++i)
+          if (cb + i < a.C) dst[i] = out[i];
+      }
+    }
+  }
+
+  if (a.codes_t) {
+    __syncthreads();
+    constexpr int E = 16 / sizeof(CodeT);  // codes per 16-byte chunk
+    constexpr int CPR = kQT / E;           // chunks per transposed row
+    CodeT* ct = static_cast<CodeT*>(a.codes_t);
+#pragma unroll 1
+    for (int idx = tid; idx < kQT * CPR; idx += 256) {
+      const int lc = idx / CPR, ch = idx % CPR;
+      const int64_t c = c0 + lc;
+      const int64_t rs = r0 + ch * E;
+      if (c >= a.C || rs >= a.R) continue;
+      CodeT* dst = ct + c * a.ldt + rs;
+      if (a.vec_t && rs + E <= a.R) {
+        *reinterpret_cast<uint4*>(dst) = *reinterpret_cast<const uint4*>(&tile_t[lc][ch * E]);
+      } else {
+        for (int e = 0; e < E && rs + e < a.R; ++e) dst[e] = tile_t[lc][ch * E + e];
+      }
+    }
+  }
+
+  // scales: s = tau_0 / Q, or range / Q per channel (0 for an all-zero channel)
+  if (a.gran == SQ_GRAN_SHIFT) {
+    if (blockIdx.x == 0 && blockIdx.y == 0 && tid == 0) {
+      const float tau = __ldg(a.rt);
+      *a.scale_out = zero_all ? 0.0f : __fdiv_rn(tau, Qf);
+    }
+  } else if (a.gran == SQ_GRAN_PER_COL) {
+    if (blockIdx.y == 0 && rq == 0) {
+#pragma unroll
+      for (int i = 0; i < 4; ++i)
+        if (cb + i < a.C) a.scale_out[cb + i] = colzero[i] ? 0.0f : __fdiv_rn(__ldg(a.rt + cb + i), Qf);
+    }
+  } else {
+    if (blockIdx.x == 0 && cq == 0) {
+#pragma unroll 1
+      for (int pass = 0; pass < 4; ++pass) {
+        const int64_t r = r0 + rq + 16 * pass;
+        if (r < a.R) {
+          const float rg = __ldg(a.rt + r);
+          const float inv = __fdiv_rn(Qf, rg);
+          const bool z = !(rg > 0.0f) || !isfinite(rg) || !isfinite(inv);
+          a.scale_out[r] = z ? 0.0f : __fdiv_rn(rg, Qf);
+        }
+      }
+    }
+  }
+}
+
+}  // namespace sq
+
+using namespace sq;
+
+// ===================================================================== C entry points
+extern "C" int shiftquant_code_type(int bits, int n_groups) {
+  if (!bits_ok(bits) || !groups_ok(n_groups))
+    return fail(SQ_EINVAL, "bits must be in [2, 8] and n_groups in [1, 8] (got %d, %d)", bits,
+                n_groups);
+  return code_type(bits, n_groups);
+}
+
+extern "C" int shiftquant_code_bytes(int bits, int n_groups) {
+  const int t = shiftquant_code_type(bits, n_groups);
+  return t < 0 ? t : code_bytes(t);
+}
+
+extern "C" const char* shiftquant_status_string(sq_status s) {
+  switch (s) {
+    case SQ_OK: return "ok";
+    case SQ_EINVAL: return "invalid argument";
+    case SQ_EALIGN: return "alignment";
+    case SQ_EUNSUPPORTED: return "unsupported combination";
+    case SQ_ECUDA: return "CUDA error";
+    default: return "unknown status";
+  }
+}
+
+extern "C" const char* shiftquant_last_error(void) { return g_last_error; }
+
+extern "C" sq_status shiftquant_calibrate(const float* x, int64_t rows, int64_t cols,
+                                          int64_t ld, int gran, int n_groups,
+                                          float* range_out, float* tau0_out, uint8_t* exp_out,
+                                          int32_t* dev_status, void* stream) {
+  clear_error();
+  if (rows < 0 || cols < 0) return fail(SQ_EINVAL, "calibrate: negative size");
+  if (gran < SQ_GRAN_SHIFT || gran > SQ_GRAN_PER_ROW) return fail(SQ_EINVAL, "calibrate: bad gran %d", gran);
+  if (gran == SQ_GRAN_SHIFT && !groups_ok(n_groups))
+    return fail(SQ_EINVAL, "calibrate: n_groups must be in [1, 8]");
+  if (rows > 0 && cols > 0 && (x == nullptr || ld < cols))
+    return fail(SQ_EINVAL, "calibrate: x is NULL or ld < cols");
+  const int64_t channels = gran == SQ_GRAN_PER_ROW ? rows : cols;
+  if (dev_status == nullptr || (channels > 0 && range_out == nullptr))
+    return fail(SQ_EINVAL, "calibrate: range_out and dev_status are required");
+  if (gran == SQ_GRAN_SHIFT && (tau0_out == nullptr || (cols > 0 && exp_out == nullptr)))
+    return fail(SQ_EINVAL, "calibrate: SHIFT needs tau0_out and exp_out");
+  cudaStream_t s = as_stream(stream);
+  cudaError_t err;
+  if (gran == SQ_GRAN_PER_ROW) {
+    if (rows == 0) return SQ_OK;
+    if (cols == 0) {
+      err = cudaMemsetAsync(range_out, 0, sizeof(float) * rows, s);
+      return err == cudaSuccess ? SQ_OK : cuda_fail(err, "cudaMemsetAsync");
+    }
+    const int vec = (ld % 4 == 0) && aligned16(x);
+    const int per_block = 8;
+    const int64_t blocks = (rows + per_block - 1) / per_block;
+    rowmax_kernel<<<static_cast<unsigned>(blocks), per_block * 32, 0, s>>>(x, rows, cols, ld, vec,
+                                                                           range_out, dev_status);
+    err = cudaGetLastError();
+    return err == cudaSuccess ? SQ_OK : cuda_fail(err, "rowmax_kernel launch");
+  }
+  if (cols > 0) {
+    err = cudaMemsetAsync(range_out, 0, sizeof(float) * cols, s);
+    if (err != cudaSuccess) return cuda_fail(err, "cudaMemsetAsync");
+  }
+  if (rows > 0 && cols > 0) {
+    const int64_t cblocks = (cols + kColTx * 4 - 1) / (kColTx * 4);
+    const int64_t target = static_cast<int64_t>(num_sms()) * 8;
+    int64_t rblocks = (target + cblocks - 1) / cblocks;
+    const int64_t max_rblocks = (rows + 31) / 32;
+    if (rblocks > max_rblocks) rblocks = max_rblocks;
+    if (rblocks > 65535) rblocks = 65535;
+    if (rblocks < 1) rblocks = 1;
+    const int64_t rpb = (rows + rblocks - 1) / rblocks;
+    rblocks = (rows + rpb - 1) / rpb;
+    const int vec = (ld % 4 == 0) && aligned16(x);
+    dim3 grid(static_cast<unsigned>(cblocks), static_cast<unsigned>(rblocks));
+    colmax_kernel<<<grid, dim3(kColTx, kColTy), 0, s>>>(
+        x, rows, cols, ld, rpb, vec, reinterpret_cast<unsigned*>(range_out), dev_status);
+    err = cudaGetLastError();
+    if (err != cudaSuccess) return cuda_fail(err, "colmax_kernel launch");
+  }
+  if (gran == SQ_GRAN_SHIFT) {
+    group_kernel<<<1, 1024, 0, s>>>(reinterpret_cast<const unsigned*>(range_out), cols, n_groups,
+                                    tau0_out, exp_out, dev_status);
+    err = cudaGetLastError();
+    if (err != cudaSuccess) return cuda_fail(err, "group_kernel launch");
+  }
+  return SQ_OK;
+}
+
+extern "C" sq_status shiftquant_quantize(const float* x, int64_t rows, int64_t cols, int64_t ld,
+                                         int gran, int bits, int n_groups,
+                                         const float* range_or_tau0, const uint8_t* exp,
+                                         const uint8_t* fold_exp, int mode, uint64_t seed,
+                                         void* codes, int64_t ld_codes, void* codes_t,
+                                         int64_t ld_t, float* scale_out, void* stream) {
+  clear_error();
+  if (!bits_ok(bits) || !groups_ok(n_groups))
+    return fail(SQ_EINVAL, "quantize: bits must be in [2, 8] and n_groups in [1, 8]");
+  if (rows < 0 || cols < 0) return fail(SQ_EINVAL, "quantize: negative size");
+  if (gran < SQ_GRAN_SHIFT || gran > SQ_GRAN_PER_ROW) return fail(SQ_EINVAL, "quantize: bad gran");
+  if (mode != SQ_ROUND_NEAREST_EVEN && mode != SQ_ROUND_STOCHASTIC)
+    return fail(SQ_EINVAL, "quantize: bad rounding mode");
+  if (gran == SQ_GRAN_SHIFT && fold_exp != nullptr)
+    return fail(SQ_EINVAL, "quantize: SHIFT takes no fold_exp");
+  cudaStream_t s = as_stream(stream);
+  const int type = code_type(bits, n_groups);
+  const int cbytes = code_bytes(type);
+  if (rows == 0 || cols == 0) {
+    // every range is 0: scales are 0 and there is no code to write
+    const int64_t n = gran == SQ_GRAN_SHIFT ? 1 : (gran == SQ_GRAN_PER_COL ? cols : rows);
+    if (n == 0) return SQ_OK;
+    if (scale_out == nullptr) return fail(SQ_EINVAL, "quantize: scale_out is required");
+    cudaError_t err = cudaMemsetAsync(scale_out, 0, sizeof(float) * n, s);
+    return err == cudaSuccess ? SQ_OK : cuda_fail(err, "cudaMemsetAsync");
+  }
+  if (range_or_tau0 == nullptr || scale_out == nullptr)
+    return fail(SQ_EINVAL, "quantize: range_or_tau0 and scale_out are required");
+  if (gran == SQ_GRAN_SHIFT && exp == nullptr)
+    return fail(SQ_EINVAL, "quantize: SHIFT needs exp");
+  if (codes == nullptr && codes_t == nullptr)
+    return fail(SQ_EINVAL, "quantize: at least one of codes / codes_t is required");
+  if (codes && ld_codes < cols) return fail(SQ_EINVAL, "quantize: ld_codes < cols");
+  if (codes_t && ld_t < rows) return fail(SQ_EINVAL, "quantize: ld_t < rows");
+  if (x == nullptr || ld < cols) return fail(SQ_EINVAL, "quantize: x is NULL or ld < cols");
+  QuantArgs a;
+  a.x = x;
+  a.R = rows;
+  a.C = cols;
+  a.ld = ld;
+  a.gran = gran;
+  a.Q = q_of_bits(bits);
+  a.G = n_groups;
+  a.mode = mode;
+  a.seed = seed;
+  a.rt = range_or_tau0;
+  a.exp = exp;
+  a.fold = fold_exp;
+  a.codes = codes;
+  a.ldc = ld_codes;
+  a.codes_t = codes_t;
+  a.ldt = ld_t;
+  a.scale_out = scale_out;
+  a.vec_in = (ld % 4 == 0) && aligned16(x);
+  a.vec_out = codes != nullptr && ((ld_codes * cbytes) % (4 * cbytes) == 0) &&
+              (reinterpret_cast<uintptr_t>(codes) % (4 * cbytes) == 0);
+  a.vec_t = codes_t != nullptr && ((ld_t * cbytes) % 16 == 0) && aligned16(codes_t);
+  const int64_t gx = (cols + kQT - 1) / kQT, gy = (rows + kQT - 1) / kQT;
+  if (gx > 0x7FFFFFFF || gy > 65535)
+    return fail(SQ_EUNSUPPORTED, "quantize: tensor too large for one launch (%lld x %lld)",
+                static_cast<long long>(rows), static_cast<long long>(cols));
+  dim3 grid(static_cast<unsigned>(gx), static_cast<unsigned>(gy));
+  if (type == SQ_CODE_E4M3)
+    quantize_kernel<uint8_t><<<grid, 256, 0, s>>>(a);
+  else
+    quantize_kernel<uint16_t><<<grid, 256, 0, s>>>(a);
+  const cudaError_t err = cudaGetLastError();
+  return err == cudaSuccess ? SQ_OK : cuda_fail(err, "quantize_kernel launch");
+}

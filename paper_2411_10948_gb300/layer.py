@@ -1,0 +1,158 @@
+"""One ShiftQuant-quantized linear layer Y = X W on the GPU: the buffers it needs and the
+sequence of C-ABI calls for its three training GEMMs, with the operand roles of the
+paper's setup (Sec. 5.1): ShiftQuant on activations and gradients, per-out-channel
+weights in the forward GEMM, per-in-channel weights in loss propagation.
+
+torch only allocates device memory here; every arithmetic step is a libshiftquant call.
+"""
+from __future__ import annotations
+
+from dataclasses import dataclass
+
+import torch
+
+from . import native as N
+
+
+def round_up(n: int, m: int) -> int:
+    return (n + m - 1) // m * m
+
+
+def code_ld(cols: int, bits: int, n_groups: int) -> int:
+    """Leading dimension (elements) that keeps every code row 16-byte aligned for TMA."""
+    return max(round_up(cols, 16 // N.shiftquant_code_bytes(bits, n_groups)), 16)
+
+
+def empty_codes(rows: int, cols: int, bits: int, n_groups: int, device) -> torch.Tensor:
+    """[rows, cols] view of a code buffer whose rows are padded to a 16-byte multiple."""
+    ld = code_ld(cols, bits, n_groups)
+    buf = torch.zeros((max(rows, 1), ld), dtype=N.code_dtype(bits, n_groups), device=device)
+    return buf[:rows, :cols]
+
+
+@dataclass
+class ShiftTensor:
+    """A ShiftQuant-quantized [R, C] tensor: codes (and their transpose), group exponents,
+    the channel ranges, tau_0 and the tensor scale s = tau_0 / Q."""
+    codes: torch.Tensor
+    codes_t: torch.Tensor | None
+    exp: torch.Tensor
+    range: torch.Tensor
+    tau0: torch.Tensor
+    scale: torch.Tensor
+
+    @staticmethod
+    def alloc(R, C, bits, n_groups, device, transposed=True) -> "ShiftTensor":
+        return ShiftTensor(
+            codes=empty_codes(R, C, bits, n_groups, device),
+            codes_t=empty_codes(C, R, bits, n_groups, device) if transposed else None,
+            exp=torch.zeros(max(C, 1), dtype=torch.uint8, device=device)[:C],
+            range=torch.zeros(max(C, 1), dtype=torch.float32, device=device)[:C],
+            tau0=torch.zeros(1, dtype=torch.float32, device=device),
+            scale=torch.zeros(1, dtype=torch.float32, device=device))
+
+
+@dataclass
+class ChannelTensor:
+    """A per-channel quantized weight in the layout one GEMM reads, with its scales."""
+    codes: torch.Tensor
+    range: torch.Tensor
+    scale: torch.Tensor
+
+
+def shift_quantize(x, q: ShiftTensor, bits, n_groups, mode, seed, status, stream=None):
+    """Range pass, grouping and quantization of x [R, C] into q (three launches)."""
+    N.shiftquant_calibrate(x, N.SQ_GRAN_SHIFT, n_groups, q.range, q.tau0, q.exp, status, stream)
+    N.shiftquant_quantize(x, N.SQ_GRAN_SHIFT, bits, n_groups, q.tau0, q.exp, None, mode, seed,
+                          q.codes, q.codes_t, q.scale, stream)
+
+
+def weight_quantize_fwd(w, out: ChannelTensor, fold_exp, bits, n_groups, status, stream=None):
+    """W [K, N] per-out-channel, written transposed [N, K] with 2^(G-1-e_k) folded in."""
+    N.shiftquant_calibrate(w, N.SQ_GRAN_PER_COL, n_groups, out.range, None, None, status, stream)
+    N.shiftquant_quantize(w, N.SQ_GRAN_PER_COL, bits, n_groups, out.range, None, fold_exp,
+                          N.SQ_ROUND_NEAREST_EVEN, 0, None, out.codes, out.scale, stream)
+
+
+def weight_quantize_dgrad(w, out: ChannelTensor, fold_exp, bits, n_groups, status, stream=None):
+    """W [K, N] per-in-channel, natural layout, 2^(G-1-e_j) of dY's channel j folded in."""
+    N.shiftquant_calibrate(w, N.SQ_GRAN_PER_ROW, n_groups, out.range, None, None, status, stream)
+    N.shiftquant_quantize(w, N.SQ_GRAN_PER_ROW, bits, n_groups, out.range, None, fold_exp,
+                          N.SQ_ROUND_NEAREST_EVEN, 0, out.codes, None, out.scale, stream)
+
+
+class QuantLinear:
+    """Buffers and calls of one quantized linear layer: X [M, K], W [K, N], dY [M, N]."""
+
+    def __init__(self, M, K, N_, bits, n_groups, device="cuda", with_acc=False,
+                 use_workspace=True):
+        self.M, self.K, self.N, self.bits, self.G = M, K, N_, bits, n_groups
+        dev = torch.device(device)
+        self.status = torch.zeros(1, dtype=torch.int32, device=dev)
+        self.x = ShiftTensor.alloc(M, K, bits, n_groups, dev)
+        self.g = ShiftTensor.alloc(M, N_, bits, n_groups, dev)
+        self.wf = ChannelTensor(empty_codes(N_, K, bits, n_groups, dev),
+                                torch.zeros(N_, dtype=torch.float32, device=dev),
+                                torch.zeros(N_, dtype=torch.float32, device=dev))
+        self.wd = ChannelTensor(empty_codes(K, N_, bits, n_groups, dev),
+                                torch.zeros(K, dtype=torch.float32, device=dev),
+                                torch.zeros(K, dtype=torch.float32, device=dev))
+        self.y = torch.zeros((M, N_), dtype=torch.float32, device=dev)
+        self.dx = torch.zeros((M, K), dtype=torch.float32, device=dev)
+        self.dw = torch.zeros((K, N_), dtype=torch.float32, device=dev)
+        self.acc = None
+        if with_acc:
+            self.acc = {"fwd": torch.zeros((M, N_), dtype=torch.int64, device=dev),
+                        "dgrad": torch.zeros((M, K), dtype=torch.int64, device=dev),
+                        "wgrad": torch.zeros((K, N_), dtype=torch.int64, device=dev)}
+        self.ws = None
+        if use_workspace:
+            need = max(N.shiftquant_gemm_workspace_bytes(0, M, N_, K, bits, n_groups),
+                       N.shiftquant_gemm_workspace_bytes(1, M, K, N_, bits, n_groups),
+                       N.shiftquant_gemm_workspace_bytes(2, K, N_, M, bits, n_groups))
+            if need:
+                self.ws = torch.zeros(need // 4, dtype=torch.int32, device=dev)
+
+    # --- the hot path, step by step --------------------------------------------------
+    def quantize_activation(self, x, stream=None):
+        shift_quantize(x, self.x, self.bits, self.G, N.SQ_ROUND_NEAREST_EVEN, 0, self.status,
+                       stream)
+
+    def quantize_gradient(self, dy, seed, stream=None):
+        shift_quantize(dy, self.g, self.bits, self.G, N.SQ_ROUND_STOCHASTIC, seed, self.status,
+                       stream)
+
+    def quantize_weights(self, w, stream=None):
+        weight_quantize_fwd(w, self.wf, self.x.exp, self.bits, self.G, self.status, stream)
+        weight_quantize_dgrad(w, self.wd, self.g.exp, self.bits, self.G, self.status, stream)
+
+    def forward(self, stream=None):
+        N.shiftquant_gemm_fwd(self.x.codes, self.x.scale, self.wf.codes, self.wf.scale, self.M,
+                              self.N, self.K, self.bits, self.G, self.y,
+                              self.acc["fwd"] if self.acc else None, self.ws, self.status,
+                              stream)
+
+    def dgrad(self, stream=None):
+        N.shiftquant_gemm_dgrad(self.g.codes, self.g.scale, self.wd.codes, self.wd.scale, self.M,
+                                self.K, self.N, self.bits, self.G, self.dx,
+                                self.acc["dgrad"] if self.acc else None, self.ws, self.status,
+                                stream)
+
+    def wgrad(self, stream=None):
+        N.shiftquant_gemm_wgrad(self.x.codes_t, self.x.scale, self.x.exp, self.g.codes_t,
+                                self.g.scale, self.g.exp, self.K, self.N, self.M, self.bits,
+                                self.G, self.dw, self.acc["wgrad"] if self.acc else None,
+                                self.ws, self.status, stream)
+
+    def step(self, x, w, dy, seed, stream=None):
+        """One training step of the layer: every quantizer pass and all three GEMMs."""
+        self.quantize_activation(x, stream)
+        self.quantize_gradient(dy, seed, stream)
+        self.quantize_weights(w, stream)
+        self.forward(stream)
+        self.dgrad(stream)
+        self.wgrad(stream)
+
+    @property
+    def gemm_ops(self) -> int:
+        return 3 * 2 * self.M * self.N * self.K

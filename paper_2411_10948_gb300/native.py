@@ -1,0 +1,184 @@
+"""ctypes binding of libshiftquant.so: one Python function per C entry point, same names,
+argument marshalling only (tensor -> data pointer, current stream -> cudaStream_t).
+
+Every computation runs in the CUDA library.  If the library is missing the import of a
+function raises: there is no CPU fallback.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+import torch
+
+from . import build as _build
+
+SQ_OK = 0
+SQ_EINVAL = -1
+SQ_EALIGN = -2
+SQ_EUNSUPPORTED = -3
+SQ_ECUDA = -4
+SQ_DEV_NONFINITE = 1
+SQ_DEV_TIMEOUT = 2
+SQ_ROUND_NEAREST_EVEN = 0
+SQ_ROUND_STOCHASTIC = 1
+SQ_GRAN_SHIFT = 0
+SQ_GRAN_PER_COL = 1
+SQ_GRAN_PER_ROW = 2
+SQ_CODE_E4M3 = 0
+SQ_CODE_BF16 = 1
+
+# every symbol declared in include/shiftquant.h
+EXPORTS = (
+    "shiftquant_code_type", "shiftquant_code_bytes", "shiftquant_calibrate",
+    "shiftquant_quantize", "shiftquant_gemm_fwd", "shiftquant_gemm_dgrad",
+    "shiftquant_gemm_wgrad", "shiftquant_gemm_workspace_bytes", "shiftquant_status_string",
+    "shiftquant_last_error",
+)
+
+_lib = None
+
+
+class ShiftQuantError(RuntimeError):
+    def __init__(self, status: int, message: str):
+        super().__init__(f"{message} (status {status})")
+        self.status = status
+
+
+def library_path() -> str:
+    return _build.LIB
+
+
+def load(path: str | None = None) -> ctypes.CDLL:
+    """Load libshiftquant.so (built in-tree by build.build_library)."""
+    global _lib
+    if _lib is not None and path is None:
+        return _lib
+    p = path or _build.LIB
+    if not os.path.exists(p):
+        raise ImportError(f"libshiftquant.so is not built ({p}); run "
+                          "`python -c 'import __graft_entry__ as g; g.build()'`")
+    lib = ctypes.CDLL(p)
+    i32, i64, u64, vp, sz = (ctypes.c_int, ctypes.c_int64, ctypes.c_uint64, ctypes.c_void_p,
+                             ctypes.c_size_t)
+    lib.shiftquant_code_type.argtypes = [i32, i32]
+    lib.shiftquant_code_type.restype = i32
+    lib.shiftquant_code_bytes.argtypes = [i32, i32]
+    lib.shiftquant_code_bytes.restype = i32
+    lib.shiftquant_calibrate.argtypes = [vp, i64, i64, i64, i32, i32, vp, vp, vp, vp, vp]
+    lib.shiftquant_calibrate.restype = i32
+    lib.shiftquant_quantize.argtypes = [vp, i64, i64, i64, i32, i32, i32, vp, vp, vp, i32, u64,
+                                        vp, i64, vp, i64, vp, vp]
+    lib.shiftquant_quantize.restype = i32
+    gemm = [vp, i64, vp, vp, i64, vp, i64, i64, i64, i32, i32, vp, i64, vp, i64, vp, sz, vp, vp]
+    lib.shiftquant_gemm_fwd.argtypes = gemm
+    lib.shiftquant_gemm_fwd.restype = i32
+    lib.shiftquant_gemm_dgrad.argtypes = gemm
+    lib.shiftquant_gemm_dgrad.restype = i32
+    lib.shiftquant_gemm_wgrad.argtypes = [vp, i64, vp, vp, vp, i64, vp, vp, i64, i64, i64, i32,
+                                          i32, vp, i64, vp, i64, vp, sz, vp, vp]
+    lib.shiftquant_gemm_wgrad.restype = i32
+    lib.shiftquant_gemm_workspace_bytes.argtypes = [i32, i64, i64, i64, i32, i32]
+    lib.shiftquant_gemm_workspace_bytes.restype = sz
+    lib.shiftquant_status_string.argtypes = [i32]
+    lib.shiftquant_status_string.restype = ctypes.c_char_p
+    lib.shiftquant_last_error.argtypes = []
+    lib.shiftquant_last_error.restype = ctypes.c_char_p
+    if path is None:
+        _lib = lib
+    return lib
+
+
+def _check(status: int) -> None:
+    if status != SQ_OK:
+        lib = load()
+        msg = lib.shiftquant_last_error().decode() or lib.shiftquant_status_string(status).decode()
+        raise ShiftQuantError(status, msg)
+
+
+def _ptr(t):
+    if t is None:
+        return None
+    return ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream=None):
+    s = stream if stream is not None else torch.cuda.current_stream()
+    return ctypes.c_void_p(s.cuda_stream)
+
+
+def _ld(t) -> int:
+    assert t.dim() == 2 and t.stride(1) == 1, "matrices must be row-major with unit column stride"
+    return t.stride(0)
+
+
+# ------------------------------------------------------------------ entry points
+def shiftquant_code_type(bits: int, n_groups: int) -> int:
+    r = load().shiftquant_code_type(bits, n_groups)
+    if r < 0:
+        _check(r)
+    return r
+
+
+def shiftquant_code_bytes(bits: int, n_groups: int) -> int:
+    r = load().shiftquant_code_bytes(bits, n_groups)
+    if r < 0:
+        _check(r)
+    return r
+
+
+def code_dtype(bits: int, n_groups: int) -> torch.dtype:
+    """torch dtype of the code storage: uint8 bytes holding E4M3, or bfloat16."""
+    return torch.uint8 if shiftquant_code_type(bits, n_groups) == SQ_CODE_E4M3 else torch.bfloat16
+
+
+def shiftquant_calibrate(x, gran, n_groups, range_out, tau0_out, exp_out, dev_status,
+                         stream=None) -> None:
+    _check(load().shiftquant_calibrate(_ptr(x), x.shape[0], x.shape[1], _ld(x), gran, n_groups,
+                                       _ptr(range_out), _ptr(tau0_out), _ptr(exp_out),
+                                       _ptr(dev_status), _stream(stream)))
+
+
+def shiftquant_quantize(x, gran, bits, n_groups, range_or_tau0, exp, fold_exp, mode, seed,
+                        codes, codes_t, scale_out, stream=None) -> None:
+    _check(load().shiftquant_quantize(
+        _ptr(x), x.shape[0], x.shape[1], _ld(x), gran, bits, n_groups, _ptr(range_or_tau0),
+        _ptr(exp), _ptr(fold_exp), mode, seed & (2**64 - 1), _ptr(codes),
+        _ld(codes) if codes is not None else 0, _ptr(codes_t),
+        _ld(codes_t) if codes_t is not None else 0, _ptr(scale_out), _stream(stream)))
+
+
+def _gemm(fn, a, a_scale, b, b_scale, M, N, K, bits, n_groups, y, acc, workspace, dev_status,
+          stream):
+    _check(fn(_ptr(a), _ld(a), _ptr(a_scale), _ptr(b), _ld(b), _ptr(b_scale), M, N, K, bits,
+              n_groups, _ptr(y), _ld(y), _ptr(acc), _ld(acc) if acc is not None else 0,
+              _ptr(workspace), workspace.numel() * workspace.element_size()
+              if workspace is not None else 0, _ptr(dev_status), _stream(stream)))
+
+
+def shiftquant_gemm_fwd(a_codes, a_scale, b_codes, b_scale, M, N, K, bits, n_groups, y,
+                        acc=None, workspace=None, dev_status=None, stream=None) -> None:
+    _gemm(load().shiftquant_gemm_fwd, a_codes, a_scale, b_codes, b_scale, M, N, K, bits,
+          n_groups, y, acc, workspace, dev_status, stream)
+
+
+def shiftquant_gemm_dgrad(a_codes, a_scale, b_codes, b_scale, M, N_out, K_in, bits, n_groups,
+                          dx, acc=None, workspace=None, dev_status=None, stream=None) -> None:
+    _gemm(load().shiftquant_gemm_dgrad, a_codes, a_scale, b_codes, b_scale, M, N_out, K_in,
+          bits, n_groups, dx, acc, workspace, dev_status, stream)
+
+
+def shiftquant_gemm_wgrad(xt_codes, x_scale, x_exp, gt_codes, g_scale, g_exp, Ci, Co, T, bits,
+                          n_groups, dw, acc=None, workspace=None, dev_status=None,
+                          stream=None) -> None:
+    _check(load().shiftquant_gemm_wgrad(
+        _ptr(xt_codes), _ld(xt_codes), _ptr(x_scale), _ptr(x_exp), _ptr(gt_codes), _ld(gt_codes),
+        _ptr(g_scale), _ptr(g_exp), Ci, Co, T, bits, n_groups, _ptr(dw), _ld(dw), _ptr(acc),
+        _ld(acc) if acc is not None else 0, _ptr(workspace),
+        workspace.numel() * workspace.element_size() if workspace is not None else 0,
+        _ptr(dev_status), _stream(stream)))
+
+
+def shiftquant_gemm_workspace_bytes(which: int, M: int, N: int, K: int, bits: int,
+                                    n_groups: int) -> int:
+    return int(load().shiftquant_gemm_workspace_bytes(which, M, N, K, bits, n_groups))

@@ -1,0 +1,140 @@
+"""The C ABI library builds for sm_103a, loads, exports every declared symbol and rejects
+bad arguments on the host before launching anything (no GPU needed)."""
+import ctypes
+import os
+import re
+import subprocess
+
+import pytest
+
+from paper_2411_10948_gb300 import build, native
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "shiftquant.h")
+
+
+@pytest.fixture(scope="module")
+def lib():
+    build.build_library()
+    return native.load()
+
+
+def declared_functions():
+    src = open(HEADER).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(shiftquant_\w+)\s*\(", src)))
+
+
+def test_header_declares_the_boundary():
+    names = declared_functions()
+    for n in ("shiftquant_calibrate", "shiftquant_quantize", "shiftquant_gemm_fwd",
+              "shiftquant_gemm_dgrad", "shiftquant_gemm_wgrad"):
+        assert n in names
+    assert set(names) == set(native.EXPORTS)
+
+
+def test_library_exports_every_declared_symbol(lib):
+    for name in declared_functions():
+        assert hasattr(lib, name), name
+    out = subprocess.run(["nm", "-D", "--defined-only", build.LIB], capture_output=True,
+                         text=True).stdout
+    exported = set(re.findall(r"\bT (shiftquant_\w+)", out))
+    assert set(declared_functions()) <= exported
+
+
+def test_header_compiles_as_plain_c(tmp_path):
+    src = tmp_path / "t.c"
+    src.write_text('#include "shiftquant.h"\nint main(void){return SQ_OK;}\n')
+    subprocess.check_call(["gcc", "-std=c99", "-Wall", "-Werror", "-I", os.path.dirname(HEADER),
+                           "-c", str(src), "-o", str(tmp_path / "t.o")])
+
+
+def test_code_type_rules(lib):
+    # E4M3 holds |q| <= 15 and the shifted weight codes up to 448, else BF16
+    assert native.shiftquant_code_type(4, 4) == native.SQ_CODE_E4M3      # 7 * 8 = 56
+    assert native.shiftquant_code_type(4, 7) == native.SQ_CODE_E4M3      # 7 * 64 = 448
+    assert native.shiftquant_code_type(4, 8) == native.SQ_CODE_BF16      # 7 * 128 > 448
+    assert native.shiftquant_code_type(5, 5) == native.SQ_CODE_E4M3      # 15 * 16 = 240
+    assert native.shiftquant_code_type(5, 6) == native.SQ_CODE_BF16      # 15 * 32 = 480
+    assert native.shiftquant_code_type(6, 4) == native.SQ_CODE_BF16
+    assert native.shiftquant_code_type(8, 1) == native.SQ_CODE_BF16
+    assert native.shiftquant_code_bytes(4, 4) == 1
+    assert native.shiftquant_code_bytes(8, 4) == 2
+    for bad in ((1, 4), (9, 4), (4, 0), (4, 9)):
+        assert lib.shiftquant_code_type(*bad) == native.SQ_EINVAL
+    assert "bits" in lib.shiftquant_last_error().decode()
+
+
+def test_host_validation_rejects_before_launch(lib):
+    st = ctypes.c_void_p(16)   # never dereferenced: every call below fails validation first
+    # negative sizes
+    assert lib.shiftquant_calibrate(st, -1, 4, 4, 0, 4, st, st, st, st, None) == native.SQ_EINVAL
+    # bad granularity and missing outputs
+    assert lib.shiftquant_calibrate(st, 4, 4, 4, 7, 4, st, st, st, st, None) == native.SQ_EINVAL
+    assert lib.shiftquant_calibrate(st, 4, 4, 4, 0, 4, st, None, st, st, None) == native.SQ_EINVAL
+    # ld < cols
+    assert lib.shiftquant_calibrate(st, 4, 8, 4, 0, 4, st, st, st, st, None) == native.SQ_EINVAL
+    # quantize: bits, rounding mode, SHIFT with fold_exp, no outputs
+    args = dict(x=st, rows=4, cols=4, ld=4, gran=0, bits=4, g=4, rt=st, exp=st, fold=None,
+                mode=0, seed=0, codes=st, ldc=16, codes_t=None, ldt=0, scale=st, s=None)
+
+    def q(**kw):
+        a = dict(args, **kw)
+        return lib.shiftquant_quantize(a["x"], a["rows"], a["cols"], a["ld"], a["gran"],
+                                       a["bits"], a["g"], a["rt"], a["exp"], a["fold"], a["mode"],
+                                       a["seed"], a["codes"], a["ldc"], a["codes_t"], a["ldt"],
+                                       a["scale"], a["s"])
+    assert q(bits=9) == native.SQ_EINVAL
+    assert q(mode=5) == native.SQ_EINVAL
+    assert q(fold=st) == native.SQ_EINVAL
+    assert q(codes=None) == native.SQ_EINVAL
+    assert q(ldc=2) == native.SQ_EINVAL
+    # gemm: misaligned operand and leading dimension (TMA needs 16-byte rows)
+    a16, a_odd = ctypes.c_void_p(256), ctypes.c_void_p(257)
+    g = lib.shiftquant_gemm_fwd
+    assert g(a_odd, 64, st, a16, 64, st, 8, 8, 64, 4, 4, st, 8, None, 0, None, 0, st,
+             None) == native.SQ_EALIGN
+    assert g(a16, 65, st, a16, 80, st, 8, 8, 64, 4, 4, st, 8, None, 0, None, 0, st,
+             None) == native.SQ_EALIGN
+    # gemm: missing status word, negative sizes, bad bits
+    assert g(a16, 64, st, a16, 64, st, 8, 8, 64, 4, 4, st, 8, None, 0, None, 0, None,
+             None) == native.SQ_EINVAL
+    assert g(a16, 64, st, a16, 64, st, -8, 8, 64, 4, 4, st, 8, None, 0, None, 0, st,
+             None) == native.SQ_EINVAL
+    assert g(a16, 64, st, a16, 64, st, 8, 8, 64, 1, 4, st, 8, None, 0, None, 0, st,
+             None) == native.SQ_EINVAL
+
+
+def test_exact_range_limits_reject_oversized_inner_dims(lib):
+    st = ctypes.c_void_p(16)
+    a16 = ctypes.c_void_p(256)
+    g = lib.shiftquant_gemm_fwd
+    # 8-bit, N_G = 4: max |T| = 127 * 127 * 8 * K must stay below 2^31 -> K <= 16642
+    r = g(a16, 20000, st, a16, 20000, st, 8, 8, 20000, 8, 4, st, 8, None, 0, None, 0, st, None)
+    assert r == native.SQ_EUNSUPPORTED
+    assert "exact" in lib.shiftquant_last_error().decode()
+
+
+@pytest.mark.skipif(__import__("torch").cuda.is_available(),
+                    reason="passes fake device pointers; only meaningful without a device")
+def test_empty_shapes_accept_null_pointers_of_empty_buffers(lib):
+    # torch hands NULL data pointers for empty tensors: an empty shape must never be
+    # rejected for them (without a device the call ends in SQ_ECUDA or SQ_OK instead)
+    fake = ctypes.c_void_p(4096)
+    for R, C in ((0, 5), (5, 0), (0, 0)):
+        rng = fake if C else None
+        ex = fake if C else None
+        r = lib.shiftquant_calibrate(None, R, C, max(C, 1), 0, 4, rng, fake, ex, fake, None)
+        assert r != native.SQ_EINVAL, (R, C, lib.shiftquant_last_error())
+        r = lib.shiftquant_quantize(None, R, C, max(C, 1), 0, 4, 4, fake, ex, None, 0, 0,
+                                    fake if R and C else None, 16, None, 0, fake, None)
+        assert r != native.SQ_EINVAL, (R, C, lib.shiftquant_last_error())
+        for gran in (1, 2):
+            ch = C if gran == 1 else R
+            r = lib.shiftquant_calibrate(None, R, C, max(C, 1), gran, 4,
+                                         fake if ch else None, None, None, fake, None)
+            assert r != native.SQ_EINVAL, (gran, R, C, lib.shiftquant_last_error())
+            r = lib.shiftquant_quantize(None, R, C, max(C, 1), gran, 4, 4,
+                                        fake if ch else None, None, None, 0, 0, None, 0, None,
+                                        0, fake if ch else None, None)
+            assert r != native.SQ_EINVAL, (gran, R, C, lib.shiftquant_last_error())

@@ -1,0 +1,176 @@
+"""GPU parity of the three ShiftMM GEMMs against the oracle: integer accumulators bit-exact,
+fp32 outputs within 1e-6 relative; plus worst-case magnitudes that push every chunk of
+the exact FP32 accumulation to its bound, split-K against unsplit, and empty shapes."""
+import numpy as np
+import pytest
+import torch
+
+import oracle as O
+from paper_2411_10948_gb300 import layer as L
+from paper_2411_10948_gb300 import native as N
+from parity_util import assert_close_f32, compare_shift, decode, f32_bits, folded, oracle_layer, \
+    to_gpu
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    from paper_2411_10948_gb300 import build
+    build.build_library()
+    N.load()
+
+
+def layer_inputs(rng, M, K, Nn):
+    sx = np.exp(rng.normal(0, 1.0, K)).astype(np.float32)
+    sx[rng.random(K) < 0.02] *= 50
+    x = (rng.standard_normal((M, K)) * sx).astype(np.float32)
+    w = (rng.standard_normal((K, Nn)) * 0.02).astype(np.float32)
+    sg = np.exp(rng.normal(0, 2.0, Nn)).astype(np.float32)
+    sg[rng.random(Nn) < 0.01] *= 1000
+    dy = (rng.laplace(0, 1, (M, Nn)) * sg).astype(np.float32)
+    return x, w, dy
+
+
+def run_and_compare(x, w, dy, bits, G, seed=11, use_workspace=True):
+    M, K = x.shape
+    Nn = w.shape[1]
+    lay = L.QuantLinear(M, K, Nn, bits, G, "cuda", with_acc=True, use_workspace=use_workspace)
+    lay.step(to_gpu(x), to_gpu(w), to_gpu(dy), seed)
+    torch.cuda.synchronize()
+    assert lay.status.item() == 0
+    o = oracle_layer(x, w, dy, bits, G, seed)
+    compare_shift(lay.x, o["x"], "X")
+    compare_shift(lay.g, o["g"], "dY")
+    np.testing.assert_array_equal(decode(lay.wf.codes), folded(o["wf"]["codes"], o["x"]["exp"], G, 0).T)
+    np.testing.assert_array_equal(decode(lay.wd.codes), folded(o["wd"]["codes"], o["g"]["exp"], G, 1))
+    np.testing.assert_array_equal(lay.acc["fwd"].cpu().numpy(), o["T_fwd"], err_msg="T fwd")
+    np.testing.assert_array_equal(lay.acc["dgrad"].cpu().numpy(), o["T_dgrad"], err_msg="T dgrad")
+    np.testing.assert_array_equal(lay.acc["wgrad"].cpu().numpy(), o["T_wgrad"], err_msg="T wgrad")
+    assert_close_f32(lay.y.cpu().numpy(), o["y"], "Y")
+    assert_close_f32(lay.dx.cpu().numpy(), o["dx"], "dX")
+    assert_close_f32(lay.dw.cpu().numpy(), o["dw"], "dW")
+    return lay
+
+
+@pytest.mark.parametrize("M,K,Nn", [(1, 1, 1), (5, 3, 7), (128, 128, 256), (130, 70, 300),
+                                    (257, 520, 260), (300, 1000, 513)])
+@pytest.mark.parametrize("bits", [4, 6, 8])
+def test_layer_chain_matches_oracle(M, K, Nn, bits):
+    rng = np.random.default_rng(M * 7 + K * 3 + Nn + bits)
+    run_and_compare(*layer_inputs(rng, M, K, Nn), bits, 4)
+
+
+@pytest.mark.parametrize("bits,G", [(6, 4), (8, 4), (8, 5), (4, 7), (5, 5), (3, 8)])
+def test_multi_chunk_inner_dims(bits, G):
+    # K long enough that the exact-FP32 chunking splits the K loop several times
+    rng = np.random.default_rng(bits * 13 + G)
+    run_and_compare(*layer_inputs(rng, 200, 5000, 300), bits, G)
+
+
+def test_split_k_equals_unsplit():
+    rng = np.random.default_rng(99)
+    x, w, dy = layer_inputs(rng, 4096, 64, 96)      # wgrad: 1 output tile, K = 4096 tokens
+    a = run_and_compare(x, w, dy, 6, 4, use_workspace=True)
+    assert a.ws is not None, "expected the wgrad to split K across SMs"
+    b = run_and_compare(x, w, dy, 6, 4, use_workspace=False)
+    np.testing.assert_array_equal(a.dw.cpu().numpy(), b.dw.cpu().numpy())
+
+
+def _encode(vals: np.ndarray, bits: int, G: int) -> torch.Tensor:
+    """Code tensor (padded rows) holding the given integers in the library's storage type."""
+    R, C = vals.shape
+    t = L.empty_codes(R, C, bits, G, "cuda")
+    v = torch.from_numpy(vals.astype(np.float32)).cuda()
+    if t.dtype == torch.uint8:
+        t.copy_(v.to(torch.float8_e4m3fn).view(torch.uint8))
+    else:
+        t.copy_(v.to(torch.bfloat16))
+    assert (decode(t) == vals).all()
+    return t
+
+
+@pytest.mark.parametrize("bits,G,K", [(4, 4, 50000), (6, 4, 6628), (8, 4, 1000), (8, 5, 700),
+                                      (6, 8, 3000)])
+def test_worst_case_magnitudes_stay_exact(bits, G, K):
+    # every product at (or one step below) the largest magnitude, same sign within a row,
+    # with odd products mixed in: partial sums reach the chunk bound and an accumulator
+    # that dropped low-order bits would lose the odd terms
+    Q = 2 ** (bits - 1) - 1
+    M, Nn = 130, 260
+    rng = np.random.default_rng(K)
+    A = np.full((M, K), Q, np.int64)
+    A[1::2] *= -1                                   # alternate row signs
+    A[5] = rng.integers(-Q, Q + 1, K)               # one random row
+    kk = np.arange(K)[None, :]
+    nn = np.arange(Nn)[:, None]
+    B = np.where((kk + nn) % 3 == 0, Q, Q << (G - 1)).astype(np.int64)
+    B[7] = rng.integers(-Q, Q + 1, K) << rng.integers(0, G, K)
+    a, b = _encode(A, bits, G), _encode(B, bits, G)
+    one = torch.ones(1, device="cuda")
+    ones = torch.ones(Nn, device="cuda")
+    y = torch.zeros((M, Nn), device="cuda")
+    acc = torch.zeros((M, Nn), dtype=torch.int64, device="cuda")
+    st = torch.zeros(1, dtype=torch.int32, device="cuda")
+    N.shiftquant_gemm_fwd(a, one, b, ones, M, Nn, K, bits, G, y, acc, None, st)
+    torch.cuda.synchronize()
+    assert st.item() == 0
+    T = A @ B.T
+    np.testing.assert_array_equal(acc.cpu().numpy(), T)
+    assert_close_f32(y.cpu().numpy(), T.astype(np.float64) * 2.0 ** -(G - 1), "Y")
+
+
+@pytest.mark.parametrize("bits,T", [(8, 4000), (6, 20000), (4, 9000)])
+def test_worst_case_wgrad(bits, T):
+    Q = 2 ** (bits - 1) - 1
+    G = 4
+    Ci, Co = 140, 270
+    rng = np.random.default_rng(T)
+    X = np.full((Ci, T), Q, np.int64)
+    X[::3] = rng.integers(-Q, Q + 1, (len(X[::3]), T))
+    Y = np.full((Co, T), Q, np.int64)
+    Y[:, ::5] = 1
+    ex = rng.integers(0, G, Ci).astype(np.uint8)
+    ey = rng.integers(0, G, Co).astype(np.uint8)
+    a, b = _encode(X, bits, G), _encode(Y, bits, G)
+    one = torch.ones(1, device="cuda")
+    dw = torch.zeros((Ci, Co), device="cuda")
+    acc = torch.zeros((Ci, Co), dtype=torch.int64, device="cuda")
+    st = torch.zeros(1, dtype=torch.int32, device="cuda")
+    N.shiftquant_gemm_wgrad(a, one, torch.from_numpy(ex).cuda(), b, one,
+                            torch.from_numpy(ey).cuda(), Ci, Co, T, bits, G, dw, acc, None, st)
+    torch.cuda.synchronize()
+    assert st.item() == 0
+    raw = X @ Y.T
+    sh = (2 * (G - 1) - ex.astype(np.int64)[:, None] - ey.astype(np.int64)[None, :])
+    np.testing.assert_array_equal(acc.cpu().numpy(), raw << sh)
+    assert_close_f32(dw.cpu().numpy(), raw * 2.0 ** -(ex[:, None] + ey[None, :]).astype(np.float64),
+                     "dW")
+
+
+def test_empty_and_zero_inner_dims():
+    st = torch.zeros(1, dtype=torch.int32, device="cuda")
+    one = torch.ones(1, device="cuda")
+    codes = L.empty_codes(8, 16, 4, 4, "cuda")
+    y = torch.full((8, 8), 5.0, device="cuda")
+    acc = torch.full((8, 8), 5, dtype=torch.int64, device="cuda")
+    # K = 0: T = 0, Y = 0
+    N.shiftquant_gemm_fwd(codes[:, :0], one, codes[:, :0], torch.ones(8, device="cuda"), 8, 8, 0,
+                          4, 4, y, acc, None, st)
+    torch.cuda.synchronize()
+    assert (y == 0).all() and (acc == 0).all() and st.item() == 0
+    # M = 0 / N = 0: nothing happens
+    N.shiftquant_gemm_fwd(codes, one, codes, torch.ones(8, device="cuda"), 0, 8, 16, 4, 4,
+                          y[:0], None, None, st)
+    N.shiftquant_gemm_dgrad(codes, one, codes, torch.ones(8, device="cuda"), 8, 0, 16, 4, 4,
+                            y[:, :0], None, None, st)
+    torch.cuda.synchronize()
+    assert st.item() == 0
+
+
+def test_zero_gradient_gives_zero_outputs():
+    rng = np.random.default_rng(1)
+    x, w, dy = layer_inputs(rng, 100, 64, 80)
+    dy[:] = 0
+    lay = run_and_compare(x, w, dy, 4, 4)
+    assert (lay.dx == 0).all() and (lay.dw == 0).all()
