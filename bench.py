@@ -1,0 +1,491 @@
+#!/usr/bin/env python3
+"""Throughput of the ShiftQuant training hot path on GB300.
+
+One step = for every linear layer of the workload: the range pass, grouping and
+quantization of the activation X (round to nearest) and of the gradient dY (stochastic),
+the per-out-channel and per-in-channel quantization of W with the ShiftMM shift folded
+in, and the three integer GEMMs (forward, loss propagation, weight gradient) with their
+dequantizing epilogues.  Inputs are resident in HBM when the timed region starts; L2 is
+flushed (a 256 MiB write) before every timed step, outside the timed interval.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+                  [--workload conv3x3|wgrad_small|vit_mlp|large_linear|large_linear_8bit|vit_block]
+
+Prints one JSON line (rank 0).  --impl reference times the plain CPU oracle of the
+same definitions on the host cores instead (a bounded sample of the same workload).
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import re
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "ShiftQuant GEMM TOPS & % dense-INT8 peak; quantizer GB/s & % HBM peak"
+UNIT = "TOPS"
+DEFAULT_WORKLOAD = "conv3x3"
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+FP8_OVER_BF16 = 2.0    # nominal dense ratio (4.5 vs 2.25 PFLOP/s)
+L2_FLUSH_BYTES = 256 << 20
+
+
+def parse_args():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", default=DEFAULT_WORKLOAD)
+    ap.add_argument("--seed", type=int, default=0)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    return ap.parse_args()
+
+
+def load_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        d = json.load(open(p))
+        return {k: float(d[k]) for k in FALLBACK_PEAKS}, "measured"
+    except Exception:
+        return dict(FALLBACK_PEAKS), "fallback"
+
+
+# ----------------------------------------------------------------- clocks sampler
+class ClockSampler:
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+    NAMES = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        try:
+            fd, self.path = tempfile.mkstemp(suffix=".csv")
+            os.close(fd)
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.index}", f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+            time.sleep(0.3)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        rows = []
+        for line in open(self.path):
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 8:
+                continue
+            try:
+                rows.append((float(parts[0]), float(parts[1]), parts[4:8]))
+            except ValueError:
+                continue
+        os.unlink(self.path)
+        if not rows:
+            return None
+        mx = max(r[1] for r in rows)
+        load = [r[0] for r in rows]
+        reasons = sorted({n for r in rows for n, v in zip(self.NAMES, r[2]) if v.lower() == "active"})
+        return {"sm_mhz": statistics.median(load), "sm_max_mhz": mx, "reasons": reasons,
+                "samples": len(rows)}
+
+
+# --------------------------------------------------------------- our CUDA path
+class Step:
+    """All buffers and calls of one workload step (every layer)."""
+
+    def __init__(self, wl, seed, device):
+        import torch
+        from paper_2411_10948_gb300 import layer as L
+        from paper_2411_10948_gb300 import native as N
+        from paper_2411_10948_gb300 import workloads as W
+        self.torch, self.N, self.L = torch, N, L
+        self.wl = wl
+        self.layers, self.inputs = [], []
+        for i, spec in enumerate(wl.layers):
+            self.inputs.append(W.torch_layer_inputs(spec, seed, i, device))
+            self.layers.append(L.QuantLinear(spec.M, spec.K, spec.N, spec.bits, spec.n_groups,
+                                             device, with_acc=False, use_workspace=True))
+        self.specs = list(wl.layers)
+
+    # (name, callable) for every library call of one step, in order
+    def calls(self, step_idx):
+        out = []
+        N, L = self.N, self.L
+        for lay, (x, w, dy) in zip(self.layers, self.inputs):
+            b, G, st = lay.bits, lay.G, lay.status
+            seed = 0x5EED + step_idx
+            out += [
+                ("calibrate", lambda lay=lay, x=x: N.shiftquant_calibrate(
+                    x, N.SQ_GRAN_SHIFT, lay.G, lay.x.range, lay.x.tau0, lay.x.exp, lay.status)),
+                ("quantize", lambda lay=lay, x=x: N.shiftquant_quantize(
+                    x, N.SQ_GRAN_SHIFT, lay.bits, lay.G, lay.x.tau0, lay.x.exp, None,
+                    N.SQ_ROUND_NEAREST_EVEN, 0, lay.x.codes, lay.x.codes_t, lay.x.scale)),
+                ("calibrate", lambda lay=lay, dy=dy: N.shiftquant_calibrate(
+                    dy, N.SQ_GRAN_SHIFT, lay.G, lay.g.range, lay.g.tau0, lay.g.exp, lay.status)),
+                ("quantize", lambda lay=lay, dy=dy, seed=seed: N.shiftquant_quantize(
+                    dy, N.SQ_GRAN_SHIFT, lay.bits, lay.G, lay.g.tau0, lay.g.exp, None,
+                    N.SQ_ROUND_STOCHASTIC, seed, lay.g.codes, lay.g.codes_t, lay.g.scale)),
+                ("calibrate", lambda lay=lay, w=w: N.shiftquant_calibrate(
+                    w, N.SQ_GRAN_PER_COL, lay.G, lay.wf.range, None, None, lay.status)),
+                ("quantize", lambda lay=lay, w=w: N.shiftquant_quantize(
+                    w, N.SQ_GRAN_PER_COL, lay.bits, lay.G, lay.wf.range, None, lay.x.exp,
+                    N.SQ_ROUND_NEAREST_EVEN, 0, None, lay.wf.codes, lay.wf.scale)),
+                ("calibrate", lambda lay=lay, w=w: N.shiftquant_calibrate(
+                    w, N.SQ_GRAN_PER_ROW, lay.G, lay.wd.range, None, None, lay.status)),
+                ("quantize", lambda lay=lay, w=w: N.shiftquant_quantize(
+                    w, N.SQ_GRAN_PER_ROW, lay.bits, lay.G, lay.wd.range, None, lay.g.exp,
+                    N.SQ_ROUND_NEAREST_EVEN, 0, lay.wd.codes, None, lay.wd.scale)),
+                ("gemm", lay.forward),
+                ("gemm", lay.dgrad),
+                ("gemm", lay.wgrad),
+            ]
+        return out
+
+    def launches_per_step(self) -> int:
+        n = 0
+        N = self.N
+        for lay in self.layers:
+            n += 2 + 1 + 2 + 1          # calibrate SHIFT (range + grouping) + quantize, X and dY
+            n += 1 + 1 + 1 + 1          # weights: range + quantize, both roles
+            n += 3                      # the three GEMM kernels
+            if lay.ws is not None:
+                for which, (M, Nn, K) in enumerate(((lay.M, lay.N, lay.K), (lay.M, lay.K, lay.N),
+                                                    (lay.K, lay.N, lay.M))):
+                    if N.shiftquant_gemm_workspace_bytes(which, M, Nn, K, lay.bits, lay.G):
+                        n += 1          # split-K finalize
+        return n
+
+    def gemm_ops(self) -> int:
+        return sum(l.gemm_ops for l in self.layers)
+
+    def gemm_flops_per_launch(self):
+        return [2 * l.M * l.N * l.K for l in self.layers for _ in range(3)]
+
+    def quantizer_bytes(self) -> int:
+        """Algorithmic HBM bytes of the quantizer passes of one step."""
+        tot = 0
+        for s, lay in zip(self.specs, self.layers):
+            cb = self.N.shiftquant_code_bytes(s.bits, s.n_groups)
+            for R, C in ((s.M, s.K), (s.M, s.N)):        # X and dY: range read, read, 2 writes
+                tot += 4 * R * C + 4 * R * C + 2 * cb * R * C
+            tot += 2 * (4 * s.K * s.N + 4 * s.K * s.N + cb * s.K * s.N)   # W, two roles
+        return tot
+
+    def status_ok(self) -> bool:
+        return all(int(l.status.item()) == 0 for l in self.layers)
+
+
+def kernel_source_hash() -> str:
+    h = hashlib.sha256()
+    for f in ("sq_gemm.cu", "sq_device.cuh"):
+        h.update(open(os.path.join(ROOT, "paper_2411_10948_gb300", "csrc", f), "rb").read())
+    return h.hexdigest()[:16]
+
+
+def profiled_traffic(workload: str):
+    """DRAM bytes per launch of the GEMM kernel from the committed ncu summary, or None when
+    the kernel source changed after the capture."""
+    p = os.path.join(ROOT, "profiles", f"shiftmm_{workload}.md")
+    if not os.path.exists(p):
+        return None
+    txt = open(p).read()
+    m = re.search(r"kernel_source_sha256_16:\s*([0-9a-f]+)", txt)
+    t = re.search(r"dram_bytes_per_launch:\s*([0-9.eE+]+)", txt)
+    if not m or not t or m.group(1) != kernel_source_hash():
+        return None
+    return float(t.group(1))
+
+
+def run_ours(args, rank, world, local_rank):
+    import torch
+    from paper_2411_10948_gb300 import build, native
+    from paper_2411_10948_gb300 import layer as L
+    from paper_2411_10948_gb300 import workloads as W
+    build.build_library()
+    native.load()
+    dev = torch.device("cuda", local_rank)
+    torch.cuda.set_device(dev)
+    wl = W.workload(args.workload)
+    st = Step(wl, args.seed + 1000 * rank, dev)
+    flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
+    stream = torch.cuda.current_stream()
+
+    def run_step(i, events=None):
+        for j, (name, fn) in enumerate(st.calls(i)):
+            fn()
+            if events is not None:
+                events[j + 1].record(stream)
+
+    for i in range(args.warmup):
+        flush.zero_()
+        run_step(i)
+    torch.cuda.synchronize()
+    assert st.status_ok(), "device status set during warm-up"
+
+    # the timed step is the whole call sequence captured in one CUDA graph
+    graph = L.CapturedStep(lambda: run_step(args.warmup))
+    for i in range(args.warmup):
+        flush.zero_()
+        graph.replay()
+    torch.cuda.synchronize()
+
+    sampler = ClockSampler(local_rank)
+    sampler.start()
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    pairs = []
+    for i in range(args.steps):
+        flush.zero_()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        graph.replay()
+        b.record(stream)
+        pairs.append((a, b))
+    torch.cuda.synchronize()
+    if world > 1:
+        torch.distributed.barrier()
+    step_ms = [a.elapsed_time(b) for a, b in pairs]
+    ok = st.status_ok()
+
+    # per-call breakdown: the same calls un-graphed, queued behind a sleep kernel so the
+    # GPU never waits on the host; events between consecutive calls
+    names = [n for n, _ in st.calls(0)]
+    ncalls = len(names)
+    kind_ms = {"calibrate": 0.0, "quantize": 0.0, "gemm": 0.0}
+    call_ms = [0.0] * ncalls
+    gemm_launch_ms = []
+    for i in range(args.steps):
+        flush.zero_()
+        torch.cuda._sleep(20_000_000)
+        ev = [torch.cuda.Event(enable_timing=True) for _ in range(ncalls + 1)]
+        ev[0].record(stream)
+        run_step(args.warmup + i, ev)
+        torch.cuda.synchronize()
+        for j, n in enumerate(names):
+            d = ev[j].elapsed_time(ev[j + 1])
+            kind_ms[n] += d
+            call_ms[j] += d
+            if n == "gemm":
+                gemm_launch_ms.append(d)
+    total_ms = sum(step_ms)
+    t = torch.tensor([total_ms], dtype=torch.float64, device=dev)
+    if world > 1:
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+    total_ms = float(t.item())
+    ms_per_step = total_ms / args.steps
+
+    # e2e: host (pinned) -> device inputs, the captured step, device -> host outputs
+    e2e = None
+    if not args.no_e2e:
+        host_in = [[a.cpu().pin_memory() for a in inp] for inp in st.inputs]
+        host_out = [[torch.empty(o.shape, dtype=o.dtype, pin_memory=True) for o in (l.y, l.dx, l.dw)]
+                    for l in st.layers]
+        h2d = sum(a.numel() * a.element_size() for inp in host_in for a in inp)
+        d2h = sum(a.numel() * a.element_size() for outs in host_out for a in outs)
+        e_ms = []
+        for i in range(args.warmup + args.steps):
+            flush.zero_()
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record(stream)
+            for dst, src in zip(st.inputs, host_in):
+                for d_, s_ in zip(dst, src):
+                    d_.copy_(s_, non_blocking=True)
+            graph.replay()
+            for lay, outs in zip(st.layers, host_out):
+                for o, h in zip((lay.y, lay.dx, lay.dw), outs):
+                    h.copy_(o, non_blocking=True)
+            b.record(stream)
+            b.synchronize()
+            if i >= args.warmup:
+                e_ms.append(a.elapsed_time(b))
+        et = torch.tensor([sum(e_ms)], dtype=torch.float64, device=dev)
+        if world > 1:
+            torch.distributed.all_reduce(et, op=torch.distributed.ReduceOp.MAX)
+        e2e = {"value": st.gemm_ops() * world * args.steps / (float(et.item()) * 1e-3) / 1e12,
+               "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+               "ms_per_step": float(et.item()) / args.steps}
+    clocks = sampler.stop()
+
+    peaks, peak_src = load_peaks()
+    spec0 = wl.layers[0]
+    fp8 = native.shiftquant_code_type(spec0.bits, spec0.n_groups) == native.SQ_CODE_E4M3
+    tensor_peak = peaks["bf16_tflops"] * (FP8_OVER_BF16 if fp8 else 1.0)
+    flops = st.gemm_flops_per_launch() * args.steps
+    gemm_tflops = sum(flops) / (sum(gemm_launch_ms) * 1e-3) / 1e12
+    q_bytes = st.quantizer_bytes() * args.steps
+    q_ms = kind_ms["calibrate"] + kind_ms["quantize"]
+    q_gbs = q_bytes / (q_ms * 1e-3) / 1e9
+    gemm_roof = {"bound": "tensor", "achieved": gemm_tflops, "peak": tensor_peak,
+                 "unit": "TFLOP/s", "frac": gemm_tflops / tensor_peak,
+                 "traffic": profiled_traffic(args.workload),
+                 "kernel": "shiftmm_kernel<%d>" % (1 if fp8 else 0),
+                 "peak_source": (f"{peak_src} bf16 burst" + (" x 2 (nominal FP8/BF16)" if fp8 else ""))}
+    quant_roof = {"bound": "hbm", "achieved": q_gbs, "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                  "frac": q_gbs / peaks["hbm_gbs"], "kernel": "calibrate + quantize",
+                  "peak_source": f"{peak_src} copy bandwidth"}
+    dominant = gemm_roof if kind_ms["gemm"] >= q_ms else quant_roof
+
+    result = {
+        "metric": METRIC,
+        "value": st.gemm_ops() * world / (ms_per_step * 1e-3) / 1e12,
+        "unit": UNIT,
+        "n_gpus": world,
+        "steps": args.steps,
+        "warmup": args.warmup,
+        "ms_per_step": ms_per_step,
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "e4m3" if fp8 else "bf16",
+        "data": "synthetic",
+        "config": {"workload": args.workload, "description": wl.description,
+                   "layers": [[s.name, s.M, s.K, s.N] for s in wl.layers],
+                   "bits": spec0.bits, "n_groups": spec0.n_groups,
+                   "l2": "flushed before every timed step (256 MiB write, outside the timed interval)",
+                   "parallelism": f"replica x{world}" if world > 1 else "single GPU"},
+        "roofline": dominant,
+        "gemm": dict(gemm_roof, tops_step=st.gemm_ops() / (ms_per_step * 1e-3) / 1e12,
+                     int8_peak="none: sm_103a has no integer MMA (tcgen05 kind::i8 does not "
+                               "assemble); exact integers run on the E4M3/BF16 tensor cores"),
+        "quantizer": dict(quant_roof, bytes_per_step=st.quantizer_bytes(),
+                          nominal_hbm_gbs=7900.0, frac_nominal=q_gbs / 7900.0),
+        "breakdown_ms_per_step": {k: v / args.steps for k, v in kind_ms.items()},
+        "calls_ms_per_step": [[f"{n}", round(v / args.steps, 5)] for n, v in zip(names, call_ms)],
+        "timing": "CUDA events around one CUDA-graph replay of the whole step; breakdown from "
+                  "un-graphed calls queued behind a sleep kernel",
+        "gpu_launches": st.launches_per_step() * args.steps,
+        "clocks": clocks,
+        "status_ok": ok,
+    }
+    if e2e is not None:
+        result["e2e"] = e2e
+    return result, st
+
+
+def oracle_sample_step(wl, rows_per_layer, seed):
+    """One bounded oracle step: the quantizer chain and the three GEMMs on the first rows."""
+    import oracle as O
+    from paper_2411_10948_gb300 import workloads as W
+    data = [W.np_layer_inputs(s, seed, i, rows=r) for i, (s, r) in
+            enumerate(zip(wl.layers, rows_per_layer))]
+
+    def run(step_idx):
+        t0 = time.perf_counter()
+        for s, (x, w, dy) in zip(wl.layers, data):
+            G = s.n_groups
+            ox = O.shiftquant_tensor(x, s.bits, G, 0)
+            og = O.shiftquant_tensor(dy, s.bits, G, 1, 0x5EED + step_idx)
+            wf = O.channel_tensor(w, s.bits, 0)
+            wd = O.channel_tensor(w, s.bits, 1)
+            T = O.gemm_fwd(ox["codes"], ox["exp"], wf["codes"], G)
+            O.dequant(T, ox["scale"], 1.0, G - 1, wf["scale"])
+            T = O.gemm_dgrad(og["codes"], og["exp"], wd["codes"], G)
+            O.dequant(T, og["scale"], 1.0, G - 1, wd["scale"])
+            T = O.gemm_wgrad(ox["codes"], ox["exp"], og["codes"], og["exp"], G)
+            O.dequant(T, ox["scale"], og["scale"], 2 * (G - 1))
+        return time.perf_counter() - t0
+    ops = sum(3 * 2 * r * s.N * s.K for s, r in zip(wl.layers, rows_per_layer))
+    return run, ops
+
+
+def choose_rows(wl, target_s, seed):
+    """Rows per layer so that one oracle step takes about target_s seconds."""
+    probe = [min(s.M, 256) for s in wl.layers]
+    run, ops = oracle_sample_step(wl, probe, seed)
+    run(0)
+    dt = max(run(0), 1e-3)
+    scale = target_s / dt
+    return [max(1, min(s.M, int(p * scale))) for s, p in zip(wl.layers, probe)]
+
+
+def cpu_baseline(wl, seed, target_s=12.0):
+    import oracle as O
+    rows = choose_rows(wl, target_s, seed)
+    run, ops = oracle_sample_step(wl, rows, seed)
+    dt = run(0)
+    return {"value": ops / dt / 1e12, "unit": UNIT, "cores": O.max_threads(), "kind": "oracle",
+            "sample": (f"first {rows} token rows of the {[s.M for s in wl.layers]} of each layer: "
+                       "range+grouping+quantization of X, dY and W (both roles) and the three "
+                       f"GEMMs over those rows, one step, {dt:.1f} s"),
+            "seconds": dt}
+
+
+def run_reference(args):
+    import oracle as O
+    from paper_2411_10948_gb300 import workloads as W
+    O.build()
+    wl = W.workload(args.workload)
+    rows = choose_rows(wl, 4.0, args.seed)
+    run, ops = oracle_sample_step(wl, rows, args.seed)
+    for i in range(args.warmup):
+        run(i)
+    times = [run(args.warmup + i) for i in range(args.steps)]
+    total = sum(times)
+    value = ops * args.steps / total / 1e12
+    sample = (f"first {rows} token rows of the {[s.M for s in wl.layers]} of each layer per step: "
+              "range+grouping+quantization of X, dY and W and the three GEMMs over those rows")
+    return {
+        "impl": "reference",
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": total / args.steps * 1e3,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "int64",
+        "data": "synthetic",
+        "config": {"workload": args.workload, "description": wl.description,
+                   "layers": [[s.name, s.M, s.K, s.N] for s in wl.layers]},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": O.max_threads(), "kind": "oracle",
+                         "sample": sample},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+
+
+def main():
+    args = parse_args()
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+    if args.impl == "reference":
+        if rank == 0:
+            print(json.dumps(run_reference(args)), flush=True)
+        return
+    if world > 1:
+        import torch
+        import torch.distributed as dist
+        torch.cuda.set_device(local_rank)
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local_rank))
+    result, _ = run_ours(args, rank, world, local_rank)
+    if rank == 0:
+        if world == 1 and not args.no_cpu_baseline:
+            from paper_2411_10948_gb300 import workloads as W
+            result["cpu_baseline"] = cpu_baseline(W.workload(args.workload), args.seed)
+        print(json.dumps(result), flush=True)
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -156,3 +156,25 @@ class QuantLinear:
     @property
     def gemm_ops(self) -> int:
         return 3 * 2 * self.M * self.N * self.K
+
+
+class CapturedStep:
+    """A sequence of library calls captured once into a CUDA graph and replayed with one
+    launch, so a step of many short kernels pays no per-call CPU cost.  Buffers are the
+    ones the calls referenced at capture time: refill them in place between replays.
+    Every kernel runs again on each replay; scalar arguments (such as the SR seed) keep
+    their captured values."""
+
+    def __init__(self, fn, warmup: int = 1):
+        s = torch.cuda.Stream()
+        s.wait_stream(torch.cuda.current_stream())
+        with torch.cuda.stream(s):
+            for _ in range(warmup):
+                fn()
+        torch.cuda.current_stream().wait_stream(s)
+        self.graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(self.graph):
+            fn()
+
+    def replay(self) -> None:
+        self.graph.replay()
