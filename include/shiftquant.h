@@ -167,6 +167,30 @@ sq_status shiftquant_gemm_wgrad(const void *xt_codes, int64_t ldx, const float *
                                 void *workspace, size_t workspace_bytes,
                                 int32_t *dev_status, void *stream);
 
+/* Weight-gradient GEMM for callers that cannot allocate device memory -- for instance a
+ * plug-in running inside a host framework that owns every device allocation, or a
+ * deployment whose device memory is fixed when the library is loaded.  The paper has no
+ * counterpart: this is an allocation strategy, not part of the method.
+ *   Arguments, results and limits are those of shiftquant_gemm_wgrad, minus the workspace.
+ *   Scratch: instead of a caller workspace, the split-K int32 partial sums live in a 4 MiB
+ *     array inside the library (`static __device__`, held by every GPU that loads the
+ *     library until the process exits).  Ci * Co must not exceed 1048576; larger outputs
+ *     return SQ_EUNSUPPORTED before anything is launched.
+ *   Nothing is allocated: no cudaMalloc, no cudaFree, no allocating library routine.
+ *   The first call on each device looks up the array's device address
+ *     (cudaGetSymbolAddress) with that device current; make that first call before any
+ *     stream capture begins.
+ *   All calls on a device share the one array, and it keeps the last call's contents
+ *     (each call clears the part it uses before use).  Two calls whose work overlaps on
+ *     the GPU -- on different streams, or from different host threads -- race on it and
+ *     give wrong results: order them on one stream. */
+sq_status shiftquant_gemm_wgrad_static(const void *xt_codes, int64_t ldx, const float *x_scale,
+                                       const uint8_t *x_exp, const void *gt_codes, int64_t ldg,
+                                       const float *g_scale, const uint8_t *g_exp, int64_t Ci,
+                                       int64_t Co, int64_t T, int bits, int n_groups,
+                                       float *dw, int64_t ld_dw, int64_t *acc_out,
+                                       int64_t ld_acc, int32_t *dev_status, void *stream);
+
 /* Bytes of int32 scratch that lets a GEMM of this shape split its inner dimension across
  * SMs on the current device (0 when it would not split).  which: 0 fwd, 1 dgrad,
  * 2 wgrad; M, N are the output dims and K the inner dim. */

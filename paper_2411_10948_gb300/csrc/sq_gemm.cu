@@ -551,6 +551,35 @@ static int run_gemm(int which, const void* a_codes, int64_t lda, const void* b_c
   return SQ_OK;
 }
 
+
+// ----------------------------------------------- allocation-free weight gradient
+// Scratch for callers that cannot allocate device memory themselves: a fixed array in
+// the library's own device image, present on every GPU that loads the library until the
+// process exits.  It serves as the split-K int32 workspace of
+// shiftquant_gemm_wgrad_static().
+constexpr size_t kStaticScratchBytes = size_t(4) << 20;  // 4 MiB: Ci * Co <= 1048576
+static __device__ __align__(256) int g_wgrad_scratch[kStaticScratchBytes / sizeof(int)];
+
+// Device address of g_wgrad_scratch on the current device.  In host code the array's
+// name only stands in for the symbol, so the address is looked up once per device with
+// that device current and cached.
+static int static_scratch_address(void** out) {
+  static void* addr[64] = {};
+  static std::mutex mu;
+  int dev = 0;
+  cudaError_t err = cudaGetDevice(&dev);
+  if (err != cudaSuccess) return cuda_fail(err, "cudaGetDevice");
+  if (dev < 0 || dev >= 64) return fail(SQ_EUNSUPPORTED, "device index %d beyond 63", dev);
+  std::lock_guard<std::mutex> lock(mu);
+  if (addr[dev] == nullptr) {
+    void* p = nullptr;
+    err = cudaGetSymbolAddress(&p, g_wgrad_scratch);
+    if (err != cudaSuccess) return cuda_fail(err, "cudaGetSymbolAddress");
+    addr[dev] = p;
+  }
+  *out = addr[dev];
+  return SQ_OK;
+}
 }  // namespace sq
 
 using namespace sq;
@@ -602,4 +631,27 @@ extern "C" size_t shiftquant_gemm_workspace_bytes(int which, int64_t M, int64_t 
   Plan pl;
   if (make_plan(which, M, N, K, bits, n_groups, sms, true, &pl) != SQ_OK) return 0;
   return pl.splits > 1 ? static_cast<size_t>(M) * N * sizeof(int) : 0;
+}
+
+extern "C" sq_status shiftquant_gemm_wgrad_static(
+    const void* xt_codes, int64_t ldx, const float* x_scale, const uint8_t* x_exp,
+    const void* gt_codes, int64_t ldg, const float* g_scale, const uint8_t* g_exp, int64_t Ci,
+    int64_t Co, int64_t T, int bits, int n_groups, float* dw, int64_t ld_dw, int64_t* acc_out,
+    int64_t ld_acc, int32_t* dev_status, void* stream) {
+  fail(SQ_OK, "");
+  if (Ci > 0 && Co > 0 &&
+      static_cast<uint64_t>(Ci) * static_cast<uint64_t>(Co) * sizeof(int) > kStaticScratchBytes)
+    return fail(SQ_EUNSUPPORTED,
+                "gemm_wgrad_static: Ci * Co = %lld exceeds the %zu int32 entries of the "
+                "library's static scratch; use shiftquant_gemm_wgrad with a caller workspace",
+                static_cast<long long>(Ci) * static_cast<long long>(Co),
+                kStaticScratchBytes / sizeof(int));
+  void* scratch = nullptr;
+  if (Ci > 0 && Co > 0 && T > 0) {
+    const int st = static_scratch_address(&scratch);
+    if (st != SQ_OK) return st;
+  }
+  return run_gemm(2, xt_codes, ldx, gt_codes, ldg, Ci, Co, T, bits, n_groups, x_scale, g_scale,
+                  x_exp, g_exp, dw, ld_dw, acc_out, ld_acc, scratch,
+                  scratch ? kStaticScratchBytes : 0, dev_status, stream);
 }

@@ -32,7 +32,8 @@ SQ_CODE_BF16 = 1
 EXPORTS = (
     "shiftquant_code_type", "shiftquant_code_bytes", "shiftquant_calibrate",
     "shiftquant_quantize", "shiftquant_gemm_fwd", "shiftquant_gemm_dgrad",
-    "shiftquant_gemm_wgrad", "shiftquant_gemm_workspace_bytes", "shiftquant_status_string",
+    "shiftquant_gemm_wgrad", "shiftquant_gemm_wgrad_static", "shiftquant_gemm_workspace_bytes",
+    "shiftquant_status_string",
     "shiftquant_last_error",
 )
 
@@ -78,6 +79,9 @@ def load(path: str | None = None) -> ctypes.CDLL:
     lib.shiftquant_gemm_wgrad.argtypes = [vp, i64, vp, vp, vp, i64, vp, vp, i64, i64, i64, i32,
                                           i32, vp, i64, vp, i64, vp, sz, vp, vp]
     lib.shiftquant_gemm_wgrad.restype = i32
+    lib.shiftquant_gemm_wgrad_static.argtypes = [vp, i64, vp, vp, vp, i64, vp, vp, i64, i64, i64,
+                                                 i32, i32, vp, i64, vp, i64, vp, vp]
+    lib.shiftquant_gemm_wgrad_static.restype = i32
     lib.shiftquant_gemm_workspace_bytes.argtypes = [i32, i64, i64, i64, i32, i32]
     lib.shiftquant_gemm_workspace_bytes.restype = sz
     lib.shiftquant_status_string.argtypes = [i32]
@@ -177,6 +181,16 @@ def shiftquant_gemm_wgrad(xt_codes, x_scale, x_exp, gt_codes, g_scale, g_exp, Ci
         _ld(acc) if acc is not None else 0, _ptr(workspace),
         workspace.numel() * workspace.element_size() if workspace is not None else 0,
         _ptr(dev_status), _stream(stream)))
+
+
+def shiftquant_gemm_wgrad_static(xt_codes, x_scale, x_exp, gt_codes, g_scale, g_exp, Ci, Co, T,
+                                 bits, n_groups, dw, acc=None, dev_status=None,
+                                 stream=None) -> None:
+    """Weight gradient with the library's own static split-K scratch (no allocation)."""
+    _check(load().shiftquant_gemm_wgrad_static(
+        _ptr(xt_codes), _ld(xt_codes), _ptr(x_scale), _ptr(x_exp), _ptr(gt_codes), _ld(gt_codes),
+        _ptr(g_scale), _ptr(g_exp), Ci, Co, T, bits, n_groups, _ptr(dw), _ld(dw), _ptr(acc),
+        _ld(acc) if acc is not None else 0, _ptr(dev_status), _stream(stream)))
 
 
 def shiftquant_gemm_workspace_bytes(which: int, M: int, N: int, K: int, bits: int,
