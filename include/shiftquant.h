@@ -54,6 +54,7 @@ typedef int sq_status;
 /* bits OR-ed into *dev_status by the kernels */
 #define SQ_DEV_NONFINITE 1    /* a NaN or Inf was met in the range pass */
 #define SQ_DEV_TIMEOUT 2      /* a pipeline wait gave up (about 1 s); outputs invalid */
+#define SQ_DEV_INTERNAL 4     /* a kernel precondition failed (shared-memory alignment) */
 
 typedef enum { SQ_ROUND_NEAREST_EVEN = 0, SQ_ROUND_STOCHASTIC = 1 } sq_round;
 

@@ -25,6 +25,7 @@
 #include <cuda_runtime.h>
 #include <cudaTypedefs.h>
 
+#include <cstring>
 #include <mutex>
 
 #include "sq_device.cuh"
@@ -44,14 +45,24 @@ constexpr int kEpiWarp0 = 4;
 constexpr int kNumEpiWarps = 8;
 constexpr uint32_t kTmemCols = 2 * kBN;       // two FP32 accumulator buffers
 constexpr int64_t kExactSum = int64_t(1) << 24;  // every partial sum of a chunk stays within this
-constexpr size_t kSmemBytes = 1024 + size_t(kStages) * kStageBytes + 256;
+// shared memory: the operand ring, one 32 x 32 output box per epilogue warp (staging for
+// TMA stores), two per-tile column-factor tables, then the barriers
+constexpr int kOutBox = 32;
+constexpr int kOutStageBytes = kOutBox * kOutBox * 4;
+constexpr int kOutOffset = kStages * kStageBytes;
+constexpr int kFacOffset = kOutOffset + kNumEpiWarps * kOutStageBytes;
+constexpr int kBarOffset = kFacOffset + 2 * kBN * 4;
+constexpr int kNumBars = 2 * kStages + 2 + 2 + 2 + 1;   // full, empty, tfull, tempty, fac, drain
+constexpr size_t kSmemBytes = kBarOffset + kNumBars * 8 + 16;
+static_assert(kSmemBytes <= 232448, "shared memory beyond the 227 KB per-CTA limit");
+static_assert(kOutOffset % 1024 == 0 && kOutStageBytes % 1024 == 0, "swizzle atoms need 1 KB");
 
 struct GemmParams {
   int M, N, K;
   int m_tiles, n_tiles, splits, kb_total, kb_per_split, chunk_kb;
   int mode;  // 0: per-column scale (forward, loss propagation); 1: row/column shifts (wgrad)
   int G;
-  int vec_y;
+  int use_tma_y;  // outputs leave through TMA stores (else plain stores)
   const float* a_scale;
   const float* b_scale;
   const uint8_t* row_exp;
@@ -107,16 +118,21 @@ __device__ __forceinline__ Unit decode_unit(const GemmParams& p, int u) {
 template <int kF8>
 __global__ void __launch_bounds__(kThreads, 1)
     shiftmm_kernel(const __grid_constant__ CUtensorMap tma_a,
-                   const __grid_constant__ CUtensorMap tma_b, const GemmParams p) {
-  extern __shared__ uint8_t smem_raw[];
-  uint8_t* smem = reinterpret_cast<uint8_t*>(
-      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
-  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + kStages * kStageBytes);
+                   const __grid_constant__ CUtensorMap tma_b,
+                   const __grid_constant__ CUtensorMap tma_y,
+                   const __grid_constant__ CUtensorMap tma_ws, const GemmParams p) {
+  extern __shared__ __align__(1024) uint8_t smem[];
+  if ((smem_u32(smem) & 1023u) != 0) {  // the swizzled layouts need 1 KB alignment
+    if (threadIdx.x == 0) atomicOr(p.status, kDevInternal);
+    return;
+  }
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + kBarOffset);
   uint64_t* full = bars;
   uint64_t* empty = bars + kStages;
   uint64_t* tfull = bars + 2 * kStages;
   uint64_t* tempty = tfull + 2;
-  uint64_t* drain = tempty + 2;
+  uint64_t* facbar = tempty + 2;
+  uint64_t* drain = facbar + 2;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
@@ -131,6 +147,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (int b = 0; b < 2; ++b) {
       mbar_init(&tfull[b], 1);
       mbar_init(&tempty[b], kNumEpiWarps);
+      mbar_init(&facbar[b], kNumEpiWarps);
     }
     mbar_init(drain, 1);
     *abort_flag = 0;
@@ -237,15 +254,37 @@ __global__ void __launch_bounds__(kThreads, 1)
     mbar_wait(drain, 0, nullptr);
   } else if (warp >= kEpiWarp0) {
     // --------------------------------------------------------------- epilogue
-    const int q = warp & 3;                     // TMEM lanes 32q .. 32q+31 (output rows)
-    const int h = (warp - kEpiWarp0) >> 2;      // column half of the 256-wide tile
+    const int q = warp & 3;                       // TMEM lanes 32q .. 32q+31 (output rows)
+    const int h = (warp - kEpiWarp0) >> 2;        // column half of the 256-wide tile
+    const int et = threadIdx.x - kEpiWarp0 * 32;  // 0 .. 255: one tile column each
+    const uint32_t stage_out = smem_u32(smem + kOutOffset + (warp - kEpiWarp0) * kOutStageBytes);
+    float* fac_tab = reinterpret_cast<float*>(smem + kFacOffset);
     const float a_fac = epilogue_a_factor(p);
+    const bool via_tma = p.ws != nullptr || p.use_tma_y;
     uint32_t c = 0;
     bool ok = true;
-    for (int u = blockIdx.x; u < units && ok; u += gridDim.x) {
+    int it = 0;
+    for (int u = blockIdx.x; u < units && ok; u += gridDim.x, ++it) {
       const Unit w = decode_unit(p, u);
       const int nch = (w.kb1 - w.kb0 + p.chunk_kb - 1) / p.chunk_kb;
-      int32_t acc[128];
+      const int64_t m0 = static_cast<int64_t>(w.mb) * kBM;
+      const int64_t n0 = static_cast<int64_t>(w.nb) * kBN;
+      // the dequantizing factor of each of the tile's 256 columns, computed once per tile
+      // while the tensor core works: s_A 2^-(G-1) s_B[n] (forward, loss propagation) or
+      // s_X s_dY 2^-eY_n (weight gradient; the row's 2^-eX_m is applied separately)
+      float* fac = fac_tab + (it & 1) * kBN;
+      {
+        const int64_t col = n0 + et;
+        float f = 0.0f;
+        if (col < p.N)
+          f = p.mode == 0 ? __fmul_rn(a_fac, __ldg(p.b_scale + col))
+                          : __fmul_rn(a_fac, pow2_neg(__ldg(p.col_exp + col)));
+        fac[et] = f;
+      }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&facbar[it & 1]);
+
+      uint32_t acc[128];  // one chunk: the FP32 pattern of an exact integer; several: int32
       for (int ch = 0; ch < nch; ++ch) {
         const uint32_t b = c & 1u, tph = (c >> 1) & 1u;
         const bool mine = mbar_wait(&tfull[b], tph, abort_flag);
@@ -256,55 +295,94 @@ __global__ void __launch_bounds__(kThreads, 1)
         tc_fence_after();
         const uint32_t taddr = tmem_base + (static_cast<uint32_t>(q * 32) << 16) + b * kBN + h * 128;
 #pragma unroll
-        for (int j = 0; j < 4; ++j) {
-          uint32_t v[32];
-          tmem_ld_32x32b_x32(taddr + j * 32, v);
+        for (int j = 0; j < 8; ++j) {
+          uint32_t v[16];
+          tmem_ld_32x32b_x16(taddr + j * 16, v);
           tmem_ld_wait();
 #pragma unroll
-          for (int i = 0; i < 32; ++i) {
-            // the FP32 value is an integer of magnitude <= 2^24: the conversion is exact
-            const int32_t t = __float2int_rn(__uint_as_float(v[i]));
-            acc[j * 32 + i] = (ch == 0) ? t : acc[j * 32 + i] + t;
+          for (int i = 0; i < 16; ++i) {
+            if (nch == 1) {
+              acc[j * 16 + i] = v[i];
+            } else {
+              // the FP32 value is an integer of magnitude <= 2^24: the conversion is exact
+              const int32_t t = __float2int_rn(__uint_as_float(v[i]));
+              acc[j * 16 + i] =
+                  static_cast<uint32_t>(ch == 0 ? t : static_cast<int32_t>(acc[j * 16 + i]) + t);
+            }
           }
         }
         tc_fence_before();
         __syncwarp();
-        if (lane == 0) mbar_arrive(&tempty[b]);
+        if (lane == 0) mbar_arrive(&tempty[b]);  // TMEM buffer b may take the next chunk
         ++c;
       }
       if (!ok) break;
-      const int64_t row = static_cast<int64_t>(w.mb) * kBM + q * 32 + lane;
-      const int64_t col0 = static_cast<int64_t>(w.nb) * kBN + h * 128;
-      if (row < p.M) {
-        if (p.ws) {
-          int* wrow = p.ws + row * p.N;
+      if (!__all_sync(0xFFFFFFFFu, mbar_wait(&facbar[it & 1], (it >> 1) & 1, abort_flag))) {
+        ok = false;
+        break;
+      }
+      const bool single = nch == 1;
+      const int64_t row0 = m0 + q * 32;
+      const int64_t row = row0 + lane;
+      const bool row_ok = row < p.M;
+      const int er = (p.mode == 1 && row_ok) ? __ldg(p.row_exp + row) : 0;
+      const float rfac = pow2_neg(er);
 #pragma unroll
-          for (int j = 0; j < 128; ++j)
-            if (col0 + j < p.N && acc[j] != 0) atomicAdd(wrow + col0 + j, acc[j]);
-        } else {
+      for (int s = 0; s < 4; ++s) {
+        const int64_t col0 = n0 + h * 128 + s * 32;
+        if (row0 >= p.M || col0 >= p.N) continue;  // warp-uniform: nothing of this box exists
+        const float* f = fac + h * 128 + s * 32;
+        if (via_tma) {
+          // stage the 32 x 32 box (lane = row, 128-byte swizzle) and hand it to TMA, which
+          // clips rows and columns outside the output
+          if (lane == 0) bulk_wait_read<0>();
+          __syncwarp();
+#pragma unroll
+          for (int k = 0; k < 8; ++k) {
+            uint32_t o[4];
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+              const uint32_t a = acc[s * 32 + k * 4 + e];
+              if (p.ws != nullptr) {
+                o[e] = single ? static_cast<uint32_t>(__float2int_rn(__uint_as_float(a))) : a;
+              } else {
+                const float val = single ? __uint_as_float(a) : __int2float_rn(static_cast<int32_t>(a));
+                o[e] = __float_as_uint(__fmul_rn(__fmul_rn(val, rfac), f[k * 4 + e]));
+              }
+            }
+            st_shared_v4(stage_out + lane * 128 + ((k ^ (lane & 7)) << 4), o[0], o[1], o[2], o[3]);
+          }
+          fence_proxy_async_smem();
+          __syncwarp();
+          if (lane == 0) {
+            if (p.ws != nullptr)
+              tma_reduce_add_2d(&tma_ws, stage_out, static_cast<int32_t>(col0), static_cast<int32_t>(row0));
+            else
+              tma_store_2d(&tma_y, stage_out, static_cast<int32_t>(col0), static_cast<int32_t>(row0));
+            bulk_commit();
+          }
+        } else if (row_ok) {
           float* yrow = p.y + row * p.ldy;
 #pragma unroll
-          for (int j = 0; j < 128; j += 4) {
-            const int64_t col = col0 + j;
-            float o[4];
-            long long t64[4];
-#pragma unroll
-            for (int i = 0; i < 4; ++i) {
-              o[i] = 0.0f;
-              t64[i] = 0;
-              if (col + i < p.N) epilogue_value(p, row, col + i, acc[j + i], a_fac, &o[i], &t64[i]);
+          for (int e = 0; e < 32; ++e) {
+            if (col0 + e < p.N) {
+              const uint32_t a = acc[s * 32 + e];
+              const float val = single ? __uint_as_float(a) : __int2float_rn(static_cast<int32_t>(a));
+              yrow[col0 + e] = __fmul_rn(__fmul_rn(val, rfac), f[e]);
             }
-            if (p.vec_y && col + 3 < p.N) {
-              *reinterpret_cast<float4*>(yrow + col) = make_float4(o[0], o[1], o[2], o[3]);
-            } else {
+          }
+        }
+        if (p.acc != nullptr && p.ws == nullptr && row_ok) {
+          // exactness-check output: the canonical integer T of every element
+          long long* arow = p.acc + row * p.ld_acc;
 #pragma unroll
-              for (int i = 0; i < 4; ++i)
-                if (col + i < p.N) yrow[col + i] = o[i];
-            }
-            if (p.acc) {
-#pragma unroll
-              for (int i = 0; i < 4; ++i)
-                if (col + i < p.N) p.acc[row * p.ld_acc + col + i] = t64[i];
+          for (int e = 0; e < 32; ++e) {
+            const int64_t col = col0 + e;
+            if (col < p.N) {
+              const uint32_t a = acc[s * 32 + e];
+              const long long t = single ? static_cast<long long>(__float2int_rn(__uint_as_float(a)))
+                                         : static_cast<long long>(static_cast<int32_t>(a));
+              arow[col] = p.mode == 0 ? t : t << (2 * (p.G - 1) - er - __ldg(p.col_exp + col));
             }
           }
         }
@@ -314,6 +392,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       atomicOr(p.status, kDevTimeout);
       *abort_flag = 1;
     }
+    if (lane == 0) bulk_wait<0>();  // every store has completed before the CTA exits
   }
 
   __syncthreads();
@@ -370,6 +449,23 @@ static int make_operand_map(CUtensorMap* map, const void* base, int64_t rows, in
                         CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
                         CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   if (r != CUDA_SUCCESS) return fail(SQ_ECUDA, "cuTensorMapEncodeTiled failed (%d)", static_cast<int>(r));
+  return SQ_OK;
+}
+
+// fp32 output or int32 split-K workspace [rows, cols] (leading dimension ld elements):
+// 32 x 32 boxes with 128-byte swizzle, matching the epilogue's staging layout
+static int make_output_map(CUtensorMap* map, void* base, int64_t rows, int64_t cols, int64_t ld,
+                           CUtensorMapDataType dt) {
+  auto fn = encode_fn();
+  if (!fn) return fail(SQ_ECUDA, "cuTensorMapEncodeTiled is not available from the driver");
+  cuuint64_t gdim[2] = {static_cast<cuuint64_t>(cols), static_cast<cuuint64_t>(rows)};
+  cuuint64_t gstride[1] = {static_cast<cuuint64_t>(ld * 4)};
+  cuuint32_t box[2] = {static_cast<cuuint32_t>(kOutBox), static_cast<cuuint32_t>(kOutBox)};
+  cuuint32_t estride[2] = {1, 1};
+  const CUresult r = fn(map, dt, 2, base, gdim, gstride, box, estride,
+                        CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                        CU_TENSOR_MAP_L2_PROMOTION_NONE, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) return fail(SQ_ECUDA, "cuTensorMapEncodeTiled (output) failed (%d)", static_cast<int>(r));
   return SQ_OK;
 }
 
@@ -488,8 +584,10 @@ static int run_gemm(int which, const void* a_codes, int64_t lda, const void* b_c
   st = make_plan(which, M, N, K, bits, G, sms, true, &pl);
   if (st != SQ_OK) return st;
   if (pl.splits > 1) {
+    // split-K partials are added by TMA into a [M, N] int32 workspace with N-element rows,
+    // whose rows must stay 16-byte aligned
     const size_t need = static_cast<size_t>(M) * N * sizeof(int);
-    if (workspace == nullptr || workspace_bytes < need || !aligned16(workspace)) {
+    if (workspace == nullptr || workspace_bytes < need || !aligned16(workspace) || N % 4 != 0) {
       st = make_plan(which, M, N, K, bits, G, sms, false, &pl);
       if (st != SQ_OK) return st;
     }
@@ -512,7 +610,7 @@ static int run_gemm(int which, const void* a_codes, int64_t lda, const void* b_c
   p.chunk_kb = pl.chunk_kb;
   p.mode = which == 2 ? 1 : 0;
   p.G = G;
-  p.vec_y = (ldy % 4 == 0) && aligned16(y);
+  p.use_tma_y = (ldy % 4 == 0) && aligned16(y);
   p.a_scale = a_scale;
   p.b_scale = b_scale;
   p.row_exp = row_exp;
@@ -524,6 +622,16 @@ static int run_gemm(int which, const void* a_codes, int64_t lda, const void* b_c
   p.ws = pl.splits > 1 ? static_cast<int*>(workspace) : nullptr;
   p.status = dev_status;
 
+  CUtensorMap my, mw;
+  memset(&my, 0, sizeof(my));
+  memset(&mw, 0, sizeof(mw));
+  if (p.ws) {
+    st = make_output_map(&mw, p.ws, M, N, N, CU_TENSOR_MAP_DATA_TYPE_INT32);
+    if (st != SQ_OK) return st;
+  } else if (p.use_tma_y) {
+    st = make_output_map(&my, y, M, N, ldy, CU_TENSOR_MAP_DATA_TYPE_FLOAT32);
+    if (st != SQ_OK) return st;
+  }
   cudaError_t err;
   if (p.ws) {
     err = cudaMemsetAsync(p.ws, 0, static_cast<size_t>(M) * N * sizeof(int), s);
@@ -533,10 +641,10 @@ static int run_gemm(int which, const void* a_codes, int64_t lda, const void* b_c
   const int grid = units < sms ? units : sms;
   if (eb == 1) {
     if ((st = configure_kernel<1>(dev)) != SQ_OK) return st;
-    shiftmm_kernel<1><<<grid, kThreads, kSmemBytes, s>>>(ma, mb, p);
+    shiftmm_kernel<1><<<grid, kThreads, kSmemBytes, s>>>(ma, mb, my, mw, p);
   } else {
     if ((st = configure_kernel<0>(dev)) != SQ_OK) return st;
-    shiftmm_kernel<0><<<grid, kThreads, kSmemBytes, s>>>(ma, mb, p);
+    shiftmm_kernel<0><<<grid, kThreads, kSmemBytes, s>>>(ma, mb, my, mw, p);
   }
   err = cudaGetLastError();
   if (err != cudaSuccess) return cuda_fail(err, "shiftmm_kernel launch");

@@ -20,6 +20,7 @@ SQ_EUNSUPPORTED = -3
 SQ_ECUDA = -4
 SQ_DEV_NONFINITE = 1
 SQ_DEV_TIMEOUT = 2
+SQ_DEV_INTERNAL = 4
 SQ_ROUND_NEAREST_EVEN = 0
 SQ_ROUND_STOCHASTIC = 1
 SQ_GRAN_SHIFT = 0
