@@ -65,13 +65,13 @@ __global__ void __launch_bounds__(kColTx* kColTy)
     const float* base = x + c0;
     int64_t r = rb + ty;
 #pragma unroll 1
-    for (; r + 3 * kColTy < re; r += 4 * kColTy) {
-      float4 v[4];
+    for (; r + 7 * kColTy < re; r += 8 * kColTy) {
+      float4 v[8];  // eight rows in flight per thread
 #pragma unroll
-      for (int u = 0; u < 4; ++u)
+      for (int u = 0; u < 8; ++u)
         v[u] = __ldg(reinterpret_cast<const float4*>(base + (r + u * kColTy) * ld));
 #pragma unroll
-      for (int u = 0; u < 4; ++u) {
+      for (int u = 0; u < 8; ++u) {
         m0 = max(m0, abs_bits(v[u].x));
         m1 = max(m1, abs_bits(v[u].y));
         m2 = max(m2, abs_bits(v[u].z));
@@ -232,115 +232,151 @@ __device__ __forceinline__ uint8_t encode_code<uint8_t>(float v) {
   return static_cast<uint8_t>(__nv_cvt_float_to_fp8(v, __NV_SATFINITE, __NV_E4M3));
 }
 
-constexpr int kQT = 64;  // quantize tile: 64 rows x 64 columns, 256 threads
+// quantize tile: 64 rows x 128 columns, 256 threads.  Lane l owns columns 4l .. 4l+3 of
+// the tile and warp w the eight rows 8w .. 8w+7: every load instruction of a warp reads 512
+// contiguous bytes of one row, and all eight loads of a thread are in flight together.
+// For the transposed copy each thread packs, per column, its eight codes (rows 8w..8w+7)
+// into one chunk; chunk w of tile column c sits at slot c*8 + (w ^ ((c >> 2) & 7)) of the
+// shared staging area, so the chunk stores of a warp and the row reads that follow both
+// touch every bank equally.
+constexpr int kQR = 64;
+constexpr int kQC = 128;
+constexpr int kQRowsPerWarp = kQR / 8;
 
-template <typename CodeT>
-__global__ void __launch_bounds__(256) quantize_kernel(const QuantArgs a) {
-  constexpr int kPad = 16 / sizeof(CodeT);
-  __shared__ __align__(16) CodeT tile_t[kQT][kQT + kPad];  // [column][row]
+__device__ __forceinline__ int chunk_slot(int col, int chunk) {
+  return col * 8 + (chunk ^ ((col >> 2) & 7));
+}
+
+// One 64 x 128 tile.  GRAN: SQ_GRAN_*; MODE: SQ_ROUND_*; FOLD: weight codes carry the
+// ShiftMM shift 2^(G-1-fold[i]); FULL: the tile lies inside the tensor and every access
+// is vector-aligned, so no element needs a bounds check.
+template <typename CodeT, int GRAN, int MODE, bool FOLD, bool FULL>
+__device__ __forceinline__ void quantize_tile(const QuantArgs& a, uint8_t* tile_t) {
+  constexpr int kChunkBytes = 8 * sizeof(CodeT);  // eight codes of one column
+  constexpr int kWords = kChunkBytes / 4;         // 32-bit words per packed column chunk
+  constexpr int kPerWord = 4 / sizeof(CodeT);
   const int tid = threadIdx.x;
-  const int cq = tid & 15;
-  const int rq = tid >> 4;
-  const int64_t r0 = static_cast<int64_t>(blockIdx.y) * kQT;
-  const int64_t c0 = static_cast<int64_t>(blockIdx.x) * kQT;
-  const int64_t cb = c0 + cq * 4;
+  const int lane = tid & 31;
+  const int wq = tid >> 5;
+  const int64_t r0 = static_cast<int64_t>(blockIdx.y) * kQR;
+  const int64_t c0 = static_cast<int64_t>(blockIdx.x) * kQC;
+  const int64_t cb = c0 + lane * 4;
   const float Qf = static_cast<float>(a.Q);
 
-  // per-column multipliers: 2^e_c (SHIFT) or Q / range_c (PER_COL)
+  // all eight input rows of this thread first, so their loads overlap
+  float4 xin[kQRowsPerWarp];
+#pragma unroll
+  for (int i = 0; i < kQRowsPerWarp; ++i) {
+    const int64_t r = r0 + wq * 8 + i;
+    const float* row = a.x + r * a.ld;
+    if (FULL) {
+      xin[i] = __ldg(reinterpret_cast<const float4*>(row + cb));
+    } else {
+      xin[i] = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+      if (r < a.R) {
+        if (a.vec_in && cb + 3 < a.C) {
+          xin[i] = __ldg(reinterpret_cast<const float4*>(row + cb));
+        } else {
+          if (cb + 0 < a.C) xin[i].x = __ldg(row + cb + 0);
+          if (cb + 1 < a.C) xin[i].y = __ldg(row + cb + 1);
+          if (cb + 2 < a.C) xin[i].z = __ldg(row + cb + 2);
+          if (cb + 3 < a.C) xin[i].w = __ldg(row + cb + 3);
+        }
+      }
+    }
+  }
+
+  // per-column multipliers: 2^e_c (SHIFT) or Q / range_c (PER_COL); per-column shifts
   float colmul[4];
   bool colzero[4];
   int colfold[4];
   float invS = 0.0f;
   bool zero_all = false;
-  if (a.gran == SQ_GRAN_SHIFT) {
+  if (GRAN == SQ_GRAN_SHIFT) {
     const float tau = __ldg(a.rt);
     invS = __fdiv_rn(Qf, tau);
     zero_all = !(tau > 0.0f) || !isfinite(tau) || !isfinite(invS);
   }
 #pragma unroll
-  for (int i = 0; i < 4; ++i) {
-    const int64_t c = cb + i;
-    colmul[i] = 1.0f;
-    colzero[i] = false;
-    colfold[i] = 0;
-    if (c < a.C) {
-      if (a.gran == SQ_GRAN_SHIFT) {
-        colmul[i] = pow2f(__ldg(a.exp + c));
-      } else if (a.gran == SQ_GRAN_PER_COL) {
+  for (int j = 0; j < 4; ++j) {
+    const int64_t c = cb + j;
+    colmul[j] = 1.0f;
+    colzero[j] = false;
+    colfold[j] = 0;
+    if (FULL || c < a.C) {
+      if (GRAN == SQ_GRAN_SHIFT) {
+        colmul[j] = pow2f(__ldg(a.exp + c));
+      } else if (GRAN == SQ_GRAN_PER_COL) {
         const float rg = __ldg(a.rt + c);
-        colmul[i] = __fdiv_rn(Qf, rg);
-        colzero[i] = !(rg > 0.0f) || !isfinite(rg) || !isfinite(colmul[i]);
+        colmul[j] = __fdiv_rn(Qf, rg);
+        colzero[j] = !(rg > 0.0f) || !isfinite(rg) || !isfinite(colmul[j]);
       }
-      if (a.gran == SQ_GRAN_PER_ROW && a.fold) colfold[i] = a.G - 1 - __ldg(a.fold + c);
+      if (GRAN == SQ_GRAN_PER_ROW && FOLD) colfold[j] = a.G - 1 - __ldg(a.fold + c);
     }
   }
 
-#pragma unroll 1
-  for (int pass = 0; pass < 4; ++pass) {
-    const int lr = rq + 16 * pass;
-    const int64_t r = r0 + lr;
-    float xv[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+  uint32_t packed[4][kWords];
+#pragma unroll
+  for (int j = 0; j < 4; ++j)
+#pragma unroll
+    for (int k = 0; k < kWords; ++k) packed[j][k] = 0u;
+
+#pragma unroll
+  for (int i = 0; i < kQRowsPerWarp; ++i) {
+    const int64_t r = r0 + wq * 8 + i;
+    const bool row_in = FULL || r < a.R;
     float rowmul = 1.0f;
     bool rowzero = false;
     int rowfold = 0;
-    if (r < a.R) {
-      const float* row = a.x + r * a.ld;
-      if (a.vec_in && cb + 3 < a.C) {
-        const float4 v = __ldg(reinterpret_cast<const float4*>(row + cb));
-        xv[0] = v.x;
-        xv[1] = v.y;
-        xv[2] = v.z;
-        xv[3] = v.w;
-      } else {
-#pragma unroll
-        for (int i = 0; i < 4; ++i)
-          if (cb + i < a.C) xv[i] = __ldg(row + cb + i);
-      }
-      if (a.gran == SQ_GRAN_PER_ROW) {
+    if (row_in) {
+      if (GRAN == SQ_GRAN_PER_ROW) {
         const float rg = __ldg(a.rt + r);
         rowmul = __fdiv_rn(Qf, rg);
         rowzero = !(rg > 0.0f) || !isfinite(rg) || !isfinite(rowmul);
       }
-      if (a.gran == SQ_GRAN_PER_COL && a.fold) rowfold = a.G - 1 - __ldg(a.fold + r);
+      if (GRAN == SQ_GRAN_PER_COL && FOLD) rowfold = a.G - 1 - __ldg(a.fold + r);
     }
+    const float xv[4] = {xin[i].x, xin[i].y, xin[i].z, xin[i].w};
     CodeT out[4];
 #pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      const int64_t c = cb + i;
+    for (int j = 0; j < 4; ++j) {
       float v;
       bool z;
-      if (a.gran == SQ_GRAN_SHIFT) {
-        v = __fmul_rn(__fmul_rn(xv[i], colmul[i]), invS);  // x 2^e exactly, then * Q/tau
+      if (GRAN == SQ_GRAN_SHIFT) {
+        v = __fmul_rn(__fmul_rn(xv[j], colmul[j]), invS);  // x 2^e exactly, then * Q/tau
         z = zero_all;
-      } else if (a.gran == SQ_GRAN_PER_COL) {
-        v = __fmul_rn(xv[i], colmul[i]);
-        z = colzero[i];
+      } else if (GRAN == SQ_GRAN_PER_COL) {
+        v = __fmul_rn(xv[j], colmul[j]);
+        z = colzero[j];
       } else {
-        v = __fmul_rn(xv[i], rowmul);
+        v = __fmul_rn(xv[j], rowmul);
         z = rowzero;
       }
-      float q = 0.0f;
-      if (!z && r < a.R && c < a.C) {
-        if (a.mode == SQ_ROUND_NEAREST_EVEN) {
-          q = rintf(v);
-        } else {
-          const float l = floorf(v);
-          const float frac = __fsub_rn(v, l);
-          const uint64_t h = splitmix64_at(a.seed, static_cast<uint64_t>(r * a.C + c));
-          const float u = __fmul_rn(static_cast<float>(static_cast<uint32_t>(h >> 40)),
-                                    5.9604644775390625e-08f);  // * 2^-24, exact
-          q = (u < frac) ? __fadd_rn(l, 1.0f) : l;
-        }
+      if (!FULL) z = z || !row_in || cb + j >= a.C;
+      float q;
+      if (MODE == SQ_ROUND_NEAREST_EVEN) {
+        // |x| <= range gives |v| <= Q (1 + 2^-23), so rint never leaves [-Q, Q]
+        q = rintf(v);
+      } else {
+        const float l = floorf(v);
+        const float frac = __fsub_rn(v, l);
+        const uint64_t hsh = splitmix64_at(a.seed, static_cast<uint64_t>(r * a.C + cb + j));
+        const float u = __fmul_rn(static_cast<float>(static_cast<uint32_t>(hsh >> 40)),
+                                  5.9604644775390625e-08f);  // * 2^-24, exact
+        q = (u < frac) ? __fadd_rn(l, 1.0f) : l;
         q = fminf(fmaxf(q, -Qf), Qf);
       }
-      const int f = (a.gran == SQ_GRAN_PER_ROW) ? colfold[i] : rowfold;
-      const float val = __fadd_rn(__fmul_rn(q, pow2f(f)), 0.0f);  // +0 for a zero code
-      out[i] = encode_code<CodeT>(val);
-      tile_t[cq * 4 + i][lr] = out[i];
+      if (z) q = 0.0f;
+      if (FOLD) {
+        const int f = (GRAN == SQ_GRAN_PER_ROW) ? colfold[j] : rowfold;
+        q = __fmul_rn(q, pow2f(f));
+      }
+      out[j] = encode_code<CodeT>(__fadd_rn(q, 0.0f));  // +0 for a zero code
+      packed[j][i / kPerWord] |= static_cast<uint32_t>(out[j]) << (8 * sizeof(CodeT) * (i % kPerWord));
     }
-    if (a.codes && r < a.R) {
+    if (a.codes && row_in) {
       CodeT* dst = static_cast<CodeT*>(a.codes) + r * a.ldc + cb;
-      if (a.vec_out && cb + 3 < a.C) {
+      if (FULL || (a.vec_out && cb + 3 < a.C)) {
         if constexpr (sizeof(CodeT) == 2) {
           uint2 w;
           w.x = static_cast<uint32_t>(out[0]) | (static_cast<uint32_t>(out[1]) << 16);
@@ -354,56 +390,120 @@ __global__ void __launch_bounds__(256) quantize_kernel(const QuantArgs a) {
         }
       } else {
 #pragma unroll
-        for (int i = 0; i < 4; ++i)
-          if (cb + i < a.C) dst[i] = out[i];
+        for (int j = 0; j < 4; ++j)
+          if (cb + j < a.C) dst[j] = out[j];
       }
     }
   }
 
   if (a.codes_t) {
+    const uint32_t base = smem_u32(tile_t);
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const uint32_t dst = base + chunk_slot(lane * 4 + j, wq) * kChunkBytes;
+      if constexpr (kWords == 4)
+        asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(dst), "r"(packed[j][0]),
+                     "r"(packed[j][1]), "r"(packed[j][2]), "r"(packed[j][3]) : "memory");
+      else
+        asm volatile("st.shared.v2.b32 [%0], {%1, %2};" ::"r"(dst), "r"(packed[j][0]),
+                     "r"(packed[j][1]) : "memory");
+    }
     __syncthreads();
-    constexpr int E = 16 / sizeof(CodeT);  // codes per 16-byte chunk
-    constexpr int CPR = kQT / E;           // chunks per transposed row
-    CodeT* ct = static_cast<CodeT*>(a.codes_t);
-#pragma unroll 1
-    for (int idx = tid; idx < kQT * CPR; idx += 256) {
-      const int lc = idx / CPR, ch = idx % CPR;
+    // each transposed row (one tile column) holds 64 codes = 8 chunks; 16-byte stores
+    constexpr int kChunksPerStore = 16 / kChunkBytes;            // 1 (BF16) or 2 (E4M3)
+    constexpr int kStoresPerRow = 8 / kChunksPerStore;
+    constexpr int E = 16 / sizeof(CodeT);                         // codes per 16-byte store
+    uint8_t* ct = static_cast<uint8_t*>(a.codes_t);
+#pragma unroll
+    for (int idx = tid; idx < kQC * kStoresPerRow; idx += 256) {
+      const int lc = idx / kStoresPerRow, st = idx % kStoresPerRow;
       const int64_t c = c0 + lc;
-      const int64_t rs = r0 + ch * E;
-      if (c >= a.C || rs >= a.R) continue;
-      CodeT* dst = ct + c * a.ldt + rs;
-      if (a.vec_t && rs + E <= a.R) {
-        *reinterpret_cast<uint4*>(dst) = *reinterpret_cast<const uint4*>(&tile_t[lc][ch * E]);
+      const int64_t rs = r0 + st * E;
+      if (!FULL && (c >= a.C || rs >= a.R)) continue;
+      uint4 v;
+      if constexpr (kChunksPerStore == 1) {
+        v = *reinterpret_cast<const uint4*>(tile_t + chunk_slot(lc, st) * kChunkBytes);
       } else {
-        for (int e = 0; e < E && rs + e < a.R; ++e) dst[e] = tile_t[lc][ch * E + e];
+        const uint2 lo = *reinterpret_cast<const uint2*>(tile_t + chunk_slot(lc, 2 * st) * kChunkBytes);
+        const uint2 hi = *reinterpret_cast<const uint2*>(tile_t + chunk_slot(lc, 2 * st + 1) * kChunkBytes);
+        v = make_uint4(lo.x, lo.y, hi.x, hi.y);
+      }
+      uint8_t* dst = ct + (c * a.ldt + rs) * static_cast<int64_t>(sizeof(CodeT));
+      if (FULL || (a.vec_t && rs + E <= a.R)) {
+        *reinterpret_cast<uint4*>(dst) = v;
+      } else {
+        const uint8_t* vb = reinterpret_cast<const uint8_t*>(&v);
+        for (int e = 0; e < E && rs + e < a.R; ++e)
+          for (int b = 0; b < static_cast<int>(sizeof(CodeT)); ++b)
+            dst[e * sizeof(CodeT) + b] = vb[e * sizeof(CodeT) + b];
       }
     }
   }
 
   // scales: s = tau_0 / Q, or range / Q per channel (0 for an all-zero channel)
-  if (a.gran == SQ_GRAN_SHIFT) {
+  if (GRAN == SQ_GRAN_SHIFT) {
     if (blockIdx.x == 0 && blockIdx.y == 0 && tid == 0) {
       const float tau = __ldg(a.rt);
       *a.scale_out = zero_all ? 0.0f : __fdiv_rn(tau, Qf);
     }
-  } else if (a.gran == SQ_GRAN_PER_COL) {
-    if (blockIdx.y == 0 && rq == 0) {
+  } else if (GRAN == SQ_GRAN_PER_COL) {
+    if (blockIdx.y == 0 && wq == 0) {
 #pragma unroll
-      for (int i = 0; i < 4; ++i)
-        if (cb + i < a.C) a.scale_out[cb + i] = colzero[i] ? 0.0f : __fdiv_rn(__ldg(a.rt + cb + i), Qf);
+      for (int j = 0; j < 4; ++j)
+        if (FULL || cb + j < a.C)
+          a.scale_out[cb + j] = colzero[j] ? 0.0f : __fdiv_rn(__ldg(a.rt + cb + j), Qf);
     }
   } else {
-    if (blockIdx.x == 0 && cq == 0) {
-#pragma unroll 1
-      for (int pass = 0; pass < 4; ++pass) {
-        const int64_t r = r0 + rq + 16 * pass;
-        if (r < a.R) {
+    if (blockIdx.x == 0 && lane == 0) {
+#pragma unroll
+      for (int i = 0; i < kQRowsPerWarp; ++i) {
+        const int64_t r = r0 + wq * 8 + i;
+        if (FULL || r < a.R) {
           const float rg = __ldg(a.rt + r);
           const float inv = __fdiv_rn(Qf, rg);
           const bool z = !(rg > 0.0f) || !isfinite(rg) || !isfinite(inv);
           a.scale_out[r] = z ? 0.0f : __fdiv_rn(rg, Qf);
         }
       }
+    }
+  }
+}
+
+template <typename CodeT, int GRAN, int MODE, bool FOLD>
+__global__ void __launch_bounds__(256) quantize_kernel(const QuantArgs a) {
+  __shared__ __align__(16) uint8_t tile_t[kQC * 8 * 8 * sizeof(CodeT)];
+  const bool full = (static_cast<int64_t>(blockIdx.y) + 1) * kQR <= a.R &&
+                    (static_cast<int64_t>(blockIdx.x) + 1) * kQC <= a.C && a.vec_in &&
+                    (a.codes == nullptr || a.vec_out) && (a.codes_t == nullptr || a.vec_t);
+  if (full)
+    quantize_tile<CodeT, GRAN, MODE, FOLD, true>(a, tile_t);
+  else
+    quantize_tile<CodeT, GRAN, MODE, FOLD, false>(a, tile_t);
+}
+
+template <typename CodeT>
+static void launch_quantize(const QuantArgs& a, dim3 grid, cudaStream_t s) {
+  const bool fold = a.fold != nullptr;
+  if (a.gran == SQ_GRAN_SHIFT) {
+    if (a.mode == SQ_ROUND_NEAREST_EVEN)
+      quantize_kernel<CodeT, SQ_GRAN_SHIFT, SQ_ROUND_NEAREST_EVEN, false><<<grid, 256, 0, s>>>(a);
+    else
+      quantize_kernel<CodeT, SQ_GRAN_SHIFT, SQ_ROUND_STOCHASTIC, false><<<grid, 256, 0, s>>>(a);
+  } else if (a.gran == SQ_GRAN_PER_COL) {
+    if (a.mode == SQ_ROUND_NEAREST_EVEN) {
+      if (fold) quantize_kernel<CodeT, SQ_GRAN_PER_COL, SQ_ROUND_NEAREST_EVEN, true><<<grid, 256, 0, s>>>(a);
+      else quantize_kernel<CodeT, SQ_GRAN_PER_COL, SQ_ROUND_NEAREST_EVEN, false><<<grid, 256, 0, s>>>(a);
+    } else {
+      if (fold) quantize_kernel<CodeT, SQ_GRAN_PER_COL, SQ_ROUND_STOCHASTIC, true><<<grid, 256, 0, s>>>(a);
+      else quantize_kernel<CodeT, SQ_GRAN_PER_COL, SQ_ROUND_STOCHASTIC, false><<<grid, 256, 0, s>>>(a);
+    }
+  } else {
+    if (a.mode == SQ_ROUND_NEAREST_EVEN) {
+      if (fold) quantize_kernel<CodeT, SQ_GRAN_PER_ROW, SQ_ROUND_NEAREST_EVEN, true><<<grid, 256, 0, s>>>(a);
+      else quantize_kernel<CodeT, SQ_GRAN_PER_ROW, SQ_ROUND_NEAREST_EVEN, false><<<grid, 256, 0, s>>>(a);
+    } else {
+      if (fold) quantize_kernel<CodeT, SQ_GRAN_PER_ROW, SQ_ROUND_STOCHASTIC, true><<<grid, 256, 0, s>>>(a);
+      else quantize_kernel<CodeT, SQ_GRAN_PER_ROW, SQ_ROUND_STOCHASTIC, false><<<grid, 256, 0, s>>>(a);
     }
   }
 }
@@ -476,8 +576,13 @@ extern "C" sq_status shiftquant_calibrate(const float* x, int64_t rows, int64_t 
   }
   if (rows > 0 && cols > 0) {
     const int64_t cblocks = (cols + kColTx * 4 - 1) / (kColTx * 4);
-    const int64_t target = static_cast<int64_t>(num_sms()) * 8;
-    int64_t rblocks = (target + cblocks - 1) / cblocks;
+    // one full wave of resident blocks, each streaming a band of rows
+    int per_sm = 0;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, colmax_kernel, kColTx * kColTy, 0) !=
+            cudaSuccess || per_sm < 1)
+      per_sm = 4;
+    const int64_t target = static_cast<int64_t>(num_sms()) * per_sm;
+    int64_t rblocks = target / cblocks;  // rounded down: a partial second wave costs a whole one
     const int64_t max_rblocks = (rows + 31) / 32;
     if (rblocks > max_rblocks) rblocks = max_rblocks;
     if (rblocks > 65535) rblocks = 65535;
@@ -557,15 +662,15 @@ extern "C" sq_status shiftquant_quantize(const float* x, int64_t rows, int64_t c
   a.vec_out = codes != nullptr && ((ld_codes * cbytes) % (4 * cbytes) == 0) &&
               (reinterpret_cast<uintptr_t>(codes) % (4 * cbytes) == 0);
   a.vec_t = codes_t != nullptr && ((ld_t * cbytes) % 16 == 0) && aligned16(codes_t);
-  const int64_t gx = (cols + kQT - 1) / kQT, gy = (rows + kQT - 1) / kQT;
+  const int64_t gx = (cols + kQC - 1) / kQC, gy = (rows + kQR - 1) / kQR;
   if (gx > 0x7FFFFFFF || gy > 65535)
     return fail(SQ_EUNSUPPORTED, "quantize: tensor too large for one launch (%lld x %lld)",
                 static_cast<long long>(rows), static_cast<long long>(cols));
   dim3 grid(static_cast<unsigned>(gx), static_cast<unsigned>(gy));
   if (type == SQ_CODE_E4M3)
-    quantize_kernel<uint8_t><<<grid, 256, 0, s>>>(a);
+    launch_quantize<uint8_t>(a, grid, s);
   else
-    quantize_kernel<uint16_t><<<grid, 256, 0, s>>>(a);
+    launch_quantize<uint16_t>(a, grid, s);
   const cudaError_t err = cudaGetLastError();
   return err == cudaSuccess ? SQ_OK : cuda_fail(err, "quantize_kernel launch");
 }
