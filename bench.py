@@ -172,11 +172,7 @@ class Step:
             n += 2 + 1 + 2 + 1          # calibrate SHIFT (range + grouping) + quantize, X and dY
             n += 1 + 1 + 1 + 1          # weights: range + quantize, both roles
             n += 3                      # the three GEMM kernels
-            if lay.ws is not None:
-                for which, (M, Nn, K) in enumerate(((lay.M, lay.N, lay.K), (lay.M, lay.K, lay.N),
-                                                    (lay.K, lay.N, lay.M))):
-                    if N.shiftquant_gemm_workspace_bytes(which, M, Nn, K, lay.bits, lay.G):
-                        n += 1          # split-K finalize
+            n += sum(ws is not None for ws in (lay.ws_fwd, lay.ws_dgrad, lay.ws_wgrad))  # finalize
         return n
 
     def gemm_ops(self) -> int:
@@ -253,8 +249,15 @@ def run_ours(args, rank, world, local_rank):
     torch.cuda.synchronize()
     assert st.status_ok(), "device status set during warm-up"
 
-    # the timed step is the whole call sequence captured in one CUDA graph
-    graph = L.CapturedStep(lambda: run_step(args.warmup))
+    # the timed step is the whole step captured in one CUDA graph; each layer's activation
+    # chain, gradient chain and weight-gradient GEMM run on their own streams inside it
+    streams = [[torch.cuda.Stream(device=dev) for _ in range(3)] for _ in st.layers]
+
+    def run_step_concurrent(i):
+        for lay, (x, w, dy), ss in zip(st.layers, st.inputs, streams):
+            lay.step_concurrent(x, w, dy, 0x5EED + i, ss)
+
+    graph = L.CapturedStep(lambda: run_step_concurrent(args.warmup))
     for i in range(args.warmup):
         flush_l2()
         graph.replay()
@@ -384,8 +387,10 @@ def run_ours(args, rank, world, local_rank):
                           nominal_hbm_gbs=7900.0, frac_nominal=q_gbs / 7900.0),
         "breakdown_ms_per_step": {k: v / args.steps for k, v in kind_ms.items()},
         "calls_ms_per_step": [[f"{n}", round(v / args.steps, 5)] for n, v in zip(names, call_ms)],
-        "timing": "CUDA events around one CUDA-graph replay of the whole step; breakdown from "
-                  "un-graphed calls queued behind a sleep kernel",
+        "timing": "CUDA events around one CUDA-graph replay of the whole step (per layer: "
+                  "activation chain + forward GEMM, gradient chain + loss-propagation GEMM, "
+                  "then the weight-gradient GEMM, on three streams); breakdown from un-graphed "
+                  "serial calls queued behind a sleep kernel",
         "gpu_launches": st.launches_per_step() * args.steps,
         "clocks": clocks,
         "status_ok": ok,

@@ -36,7 +36,7 @@ namespace sq {
 constexpr int kBM = 128;
 constexpr int kBN = 256;
 constexpr int kBKBytes = 128;                 // one 128-byte swizzle row of K per stage
-constexpr int kStages = 4;
+constexpr int kStages = 3;
 constexpr int kABytes = kBM * kBKBytes;       // 16 KB
 constexpr int kBBytes = kBN * kBKBytes;       // 32 KB
 constexpr int kStageBytes = kABytes + kBBytes;
@@ -45,12 +45,12 @@ constexpr int kEpiWarp0 = 4;
 constexpr int kNumEpiWarps = 8;
 constexpr uint32_t kTmemCols = 2 * kBN;       // two FP32 accumulator buffers
 constexpr int64_t kExactSum = int64_t(1) << 24;  // every partial sum of a chunk stays within this
-// shared memory: the operand ring, one 32 x 32 output box per epilogue warp (staging for
-// TMA stores), two per-tile column-factor tables, then the barriers
+// shared memory: the operand ring, two 32 x 32 output boxes per epilogue warp (staging for
+// TMA stores, double-buffered), two per-tile column-factor tables, then the barriers
 constexpr int kOutBox = 32;
 constexpr int kOutStageBytes = kOutBox * kOutBox * 4;
 constexpr int kOutOffset = kStages * kStageBytes;
-constexpr int kFacOffset = kOutOffset + kNumEpiWarps * kOutStageBytes;
+constexpr int kFacOffset = kOutOffset + kNumEpiWarps * 2 * kOutStageBytes;
 constexpr int kBarOffset = kFacOffset + 2 * kBN * 4;
 constexpr int kNumBars = 2 * kStages + 2 + 2 + 2 + 1;   // full, empty, tfull, tempty, fac, drain
 constexpr size_t kSmemBytes = kBarOffset + kNumBars * 8 + 16;
@@ -99,23 +99,129 @@ __device__ __forceinline__ float epilogue_a_factor(const GemmParams& p) {
                      : __fmul_rn(__ldg(p.a_scale), __ldg(p.b_scale));
 }
 
+// value of box element (rr, cc) in a staging buffer written with 128-byte swizzle
+__device__ __forceinline__ uint32_t staged(uint32_t buf, int rr, int cc) {
+  uint32_t v;
+  asm volatile("ld.shared.b32 %0, [%1];"
+               : "=r"(v)
+               : "r"(buf + rr * 128 + ((((cc >> 2) ^ (rr & 7))) << 4) + (cc & 3) * 4));
+  return v;
+}
+
+// plain stores of a staged fp32 box (lane = column, one row per step: coalesced)
+__device__ __noinline__ void write_y_box(float* y, int64_t ldy, int64_t M, int64_t N, uint32_t buf,
+                                         int64_t row0, int64_t col0, int lane) {
+  const int64_t col = col0 + lane;
+  for (int rr = 0; rr < 32; ++rr) {
+    const int64_t row = row0 + rr;
+    if (row < M && col < N) y[row * ldy + col] = __uint_as_float(staged(buf, rr, lane));
+  }
+}
+
+// the canonical integers T of a staged int32 box as int64 (exactness-check output);
+// row_exp / col_exp are null for the forward and loss-propagation GEMMs
+__device__ __noinline__ void write_acc_box(long long* acc, int64_t ld_acc, int64_t M, int64_t N,
+                                           const uint8_t* row_exp, const uint8_t* col_exp, int G,
+                                           uint32_t buf, int64_t row0, int64_t col0, int lane) {
+  const int64_t col = col0 + lane;
+  if (col >= N) return;
+  const int ec = col_exp ? __ldg(col_exp + col) : 0;
+  for (int rr = 0; rr < 32; ++rr) {
+    const int64_t row = row0 + rr;
+    if (row >= M) break;
+    const long long t = static_cast<int32_t>(staged(buf, rr, lane));
+    acc[row * ld_acc + col] = row_exp ? t << (2 * (G - 1) - __ldg(row_exp + row) - ec) : t;
+  }
+}
+
+// One 32 x 32 output box of an epilogue warp: lane = row, vals = the lane's 32 columns as
+// exact integers (FP32 patterns when `as_float`, else int32).  Stages the box in shared
+// memory and hands it to TMA (store of the dequantized fp32 values, or int32 reduce-add
+// into the split-K workspace); writes the exactness-check integers when asked.
+__device__ __forceinline__ void emit_box(const GemmParams& p, const CUtensorMap* tma_y,
+                                         const CUtensorMap* tma_ws, const uint32_t (&vals)[32],
+                                         bool as_float, const float* f, float rfac, uint32_t buf,
+                                         int64_t row0, int64_t col0, int lane, bool via_tma) {
+  if (lane == 0) bulk_wait_read<1>();
+  __syncwarp();
+  if (p.acc != nullptr && p.ws == nullptr) {
+#pragma unroll
+    for (int k = 0; k < 8; ++k) {
+      uint32_t o[4];
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const uint32_t a = vals[k * 4 + e];
+        o[e] = as_float ? static_cast<uint32_t>(__float2int_rn(__uint_as_float(a))) : a;
+      }
+      st_shared_v4(buf + lane * 128 + ((k ^ (lane & 7)) << 4), o[0], o[1], o[2], o[3]);
+    }
+    __syncwarp();
+    write_acc_box(p.acc, p.ld_acc, p.M, p.N, p.mode == 1 ? p.row_exp : nullptr,
+                  p.mode == 1 ? p.col_exp : nullptr, p.G, buf, row0, col0, lane);
+    __syncwarp();
+  }
+#pragma unroll
+  for (int k = 0; k < 8; ++k) {
+    uint32_t o[4];
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      const uint32_t a = vals[k * 4 + e];
+      if (p.ws != nullptr) {
+        o[e] = as_float ? static_cast<uint32_t>(__float2int_rn(__uint_as_float(a))) : a;
+      } else {
+        const float val = as_float ? __uint_as_float(a) : __int2float_rn(static_cast<int32_t>(a));
+        o[e] = __float_as_uint(__fmul_rn(__fmul_rn(val, rfac), f[k * 4 + e]));
+      }
+    }
+    st_shared_v4(buf + lane * 128 + ((k ^ (lane & 7)) << 4), o[0], o[1], o[2], o[3]);
+  }
+  if (via_tma) {
+    fence_proxy_async_smem();
+    __syncwarp();
+    if (lane == 0) {
+      if (p.ws != nullptr)
+        tma_reduce_add_2d(tma_ws, buf, static_cast<int32_t>(col0), static_cast<int32_t>(row0));
+      else
+        tma_store_2d(tma_y, buf, static_cast<int32_t>(col0), static_cast<int32_t>(row0));
+      bulk_commit();
+    }
+  } else {
+    __syncwarp();
+    write_y_box(p.y, p.ldy, p.M, p.N, buf, row0, col0, lane);  // outputs TMA cannot address
+    __syncwarp();
+  }
+}
+
 struct Unit {
   int mb, nb, kb0, kb1;
 };
+
+// Work unit u -> (tile, K split).  Tiles go in groups of kGroupM row tiles: inside a group
+// the row tile changes fastest, then the column tile.  The CTAs running at one time then
+// cover a compact block of the output, so the A rows of a group stay in L2 while every
+// column tile of B passes by, and neither operand is streamed from HBM more than once
+// per group.
+constexpr int kGroupM = 16;
 
 __device__ __forceinline__ Unit decode_unit(const GemmParams& p, int u) {
   const int tiles = p.m_tiles * p.n_tiles;
   const int split = u / tiles;
   const int t = u - split * tiles;
+  const int per_group = kGroupM * p.n_tiles;
+  const int g = t / per_group;
+  const int gm = min(kGroupM, p.m_tiles - g * kGroupM);  // row tiles in this group
+  const int in = t - g * per_group;
   Unit r;
-  r.mb = t % p.m_tiles;
-  r.nb = t / p.m_tiles;
+  r.mb = g * kGroupM + in % gm;
+  r.nb = in / gm;
   r.kb0 = split * p.kb_per_split;
   r.kb1 = min(p.kb_total, r.kb0 + p.kb_per_split);
   return r;
 }
 
-template <int kF8>
+// kMulti: the K loop of a tile spans several exact chunks, whose int32 sums the epilogue
+// keeps in registers; otherwise every output streams from TMEM once.
+template <int kF8, bool kMulti>
 __global__ void __launch_bounds__(kThreads, 1)
     shiftmm_kernel(const __grid_constant__ CUtensorMap tma_a,
                    const __grid_constant__ CUtensorMap tma_b,
@@ -257,7 +363,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int q = warp & 3;                       // TMEM lanes 32q .. 32q+31 (output rows)
     const int h = (warp - kEpiWarp0) >> 2;        // column half of the 256-wide tile
     const int et = threadIdx.x - kEpiWarp0 * 32;  // 0 .. 255: one tile column each
-    const uint32_t stage_out = smem_u32(smem + kOutOffset + (warp - kEpiWarp0) * kOutStageBytes);
+    const uint32_t stage_out0 =
+        smem_u32(smem + kOutOffset + (warp - kEpiWarp0) * 2 * kOutStageBytes);
+    uint32_t nbox = 0;  // boxes this warp has handed to TMA: selects the staging buffer
     float* fac_tab = reinterpret_cast<float*>(smem + kFacOffset);
     const float a_fac = epilogue_a_factor(p);
     const bool via_tma = p.ws != nullptr || p.use_tma_y;
@@ -284,107 +392,82 @@ __global__ void __launch_bounds__(kThreads, 1)
       __syncwarp();
       if (lane == 0) mbar_arrive(&facbar[it & 1]);
 
-      uint32_t acc[128];  // one chunk: the FP32 pattern of an exact integer; several: int32
-      for (int ch = 0; ch < nch; ++ch) {
+      const int64_t row0 = m0 + q * 32;
+      const int64_t row = row0 + lane;
+      const bool row_ok = row < p.M;
+      const float rfac = pow2_neg((p.mode == 1 && row_ok) ? __ldg(p.row_exp + row) : 0);
+      if constexpr (!kMulti) {
+        // one exact chunk: each TMEM value is already the integer T (as FP32)
         const uint32_t b = c & 1u, tph = (c >> 1) & 1u;
-        const bool mine = mbar_wait(&tfull[b], tph, abort_flag);
-        if (!__all_sync(0xFFFFFFFFu, mine)) {
+        if (!__all_sync(0xFFFFFFFFu, mbar_wait(&tfull[b], tph, abort_flag)) ||
+            !__all_sync(0xFFFFFFFFu, mbar_wait(&facbar[it & 1], (it >> 1) & 1, abort_flag))) {
           ok = false;
           break;
         }
         tc_fence_after();
         const uint32_t taddr = tmem_base + (static_cast<uint32_t>(q * 32) << 16) + b * kBN + h * 128;
-#pragma unroll
-        for (int j = 0; j < 8; ++j) {
-          uint32_t v[16];
-          tmem_ld_32x32b_x16(taddr + j * 16, v);
+#pragma unroll 1
+        for (int s = 0; s < 4; ++s) {
+          uint32_t v[32];
+          tmem_ld_32x32b_x32(taddr + s * 32, v);
           tmem_ld_wait();
+          if (s == 3) {
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&tempty[b]);  // TMEM buffer b may take the next tile
+          }
+          const int64_t col0 = n0 + h * 128 + s * 32;
+          if (row0 >= p.M || col0 >= p.N) continue;  // warp-uniform: nothing of this box exists
+          const uint32_t buf = stage_out0 + (nbox & 1u) * kOutStageBytes;
+          ++nbox;
+          emit_box(p, &tma_y, &tma_ws, v, true, fac + h * 128 + s * 32, rfac, buf, row0, col0,
+                   lane, via_tma);
+        }
+        ++c;
+      } else {
+        uint32_t acc[128];  // int32 sums of the chunks
+        for (int ch = 0; ch < nch; ++ch) {
+          const uint32_t b = c & 1u, tph = (c >> 1) & 1u;
+          if (!__all_sync(0xFFFFFFFFu, mbar_wait(&tfull[b], tph, abort_flag))) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t taddr = tmem_base + (static_cast<uint32_t>(q * 32) << 16) + b * kBN + h * 128;
 #pragma unroll
-          for (int i = 0; i < 16; ++i) {
-            if (nch == 1) {
-              acc[j * 16 + i] = v[i];
-            } else {
+          for (int j = 0; j < 8; ++j) {
+            uint32_t v[16];
+            tmem_ld_32x32b_x16(taddr + j * 16, v);
+            tmem_ld_wait();
+#pragma unroll
+            for (int i = 0; i < 16; ++i) {
               // the FP32 value is an integer of magnitude <= 2^24: the conversion is exact
               const int32_t t = __float2int_rn(__uint_as_float(v[i]));
               acc[j * 16 + i] =
                   static_cast<uint32_t>(ch == 0 ? t : static_cast<int32_t>(acc[j * 16 + i]) + t);
             }
           }
-        }
-        tc_fence_before();
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&tempty[b]);  // TMEM buffer b may take the next chunk
-        ++c;
-      }
-      if (!ok) break;
-      if (!__all_sync(0xFFFFFFFFu, mbar_wait(&facbar[it & 1], (it >> 1) & 1, abort_flag))) {
-        ok = false;
-        break;
-      }
-      const bool single = nch == 1;
-      const int64_t row0 = m0 + q * 32;
-      const int64_t row = row0 + lane;
-      const bool row_ok = row < p.M;
-      const int er = (p.mode == 1 && row_ok) ? __ldg(p.row_exp + row) : 0;
-      const float rfac = pow2_neg(er);
-#pragma unroll
-      for (int s = 0; s < 4; ++s) {
-        const int64_t col0 = n0 + h * 128 + s * 32;
-        if (row0 >= p.M || col0 >= p.N) continue;  // warp-uniform: nothing of this box exists
-        const float* f = fac + h * 128 + s * 32;
-        if (via_tma) {
-          // stage the 32 x 32 box (lane = row, 128-byte swizzle) and hand it to TMA, which
-          // clips rows and columns outside the output
-          if (lane == 0) bulk_wait_read<0>();
+          tc_fence_before();
           __syncwarp();
-#pragma unroll
-          for (int k = 0; k < 8; ++k) {
-            uint32_t o[4];
-#pragma unroll
-            for (int e = 0; e < 4; ++e) {
-              const uint32_t a = acc[s * 32 + k * 4 + e];
-              if (p.ws != nullptr) {
-                o[e] = single ? static_cast<uint32_t>(__float2int_rn(__uint_as_float(a))) : a;
-              } else {
-                const float val = single ? __uint_as_float(a) : __int2float_rn(static_cast<int32_t>(a));
-                o[e] = __float_as_uint(__fmul_rn(__fmul_rn(val, rfac), f[k * 4 + e]));
-              }
-            }
-            st_shared_v4(stage_out + lane * 128 + ((k ^ (lane & 7)) << 4), o[0], o[1], o[2], o[3]);
-          }
-          fence_proxy_async_smem();
-          __syncwarp();
-          if (lane == 0) {
-            if (p.ws != nullptr)
-              tma_reduce_add_2d(&tma_ws, stage_out, static_cast<int32_t>(col0), static_cast<int32_t>(row0));
-            else
-              tma_store_2d(&tma_y, stage_out, static_cast<int32_t>(col0), static_cast<int32_t>(row0));
-            bulk_commit();
-          }
-        } else if (row_ok) {
-          float* yrow = p.y + row * p.ldy;
-#pragma unroll
-          for (int e = 0; e < 32; ++e) {
-            if (col0 + e < p.N) {
-              const uint32_t a = acc[s * 32 + e];
-              const float val = single ? __uint_as_float(a) : __int2float_rn(static_cast<int32_t>(a));
-              yrow[col0 + e] = __fmul_rn(__fmul_rn(val, rfac), f[e]);
-            }
-          }
+          if (lane == 0) mbar_arrive(&tempty[b]);  // TMEM buffer b may take the next chunk
+          ++c;
         }
-        if (p.acc != nullptr && p.ws == nullptr && row_ok) {
-          // exactness-check output: the canonical integer T of every element
-          long long* arow = p.acc + row * p.ld_acc;
+        if (!ok) break;
+        if (!__all_sync(0xFFFFFFFFu, mbar_wait(&facbar[it & 1], (it >> 1) & 1, abort_flag))) {
+          ok = false;
+          break;
+        }
 #pragma unroll
-          for (int e = 0; e < 32; ++e) {
-            const int64_t col = col0 + e;
-            if (col < p.N) {
-              const uint32_t a = acc[s * 32 + e];
-              const long long t = single ? static_cast<long long>(__float2int_rn(__uint_as_float(a)))
-                                         : static_cast<long long>(static_cast<int32_t>(a));
-              arow[col] = p.mode == 0 ? t : t << (2 * (p.G - 1) - er - __ldg(p.col_exp + col));
-            }
-          }
+        for (int s = 0; s < 4; ++s) {
+          const int64_t col0 = n0 + h * 128 + s * 32;
+          if (row0 >= p.M || col0 >= p.N) continue;
+          uint32_t v[32];
+#pragma unroll
+          for (int i = 0; i < 32; ++i) v[i] = acc[s * 32 + i];
+          const uint32_t buf = stage_out0 + (nbox & 1u) * kOutStageBytes;
+          ++nbox;
+          emit_box(p, &tma_y, &tma_ws, v, false, fac + h * 128 + s * 32, rfac, buf, row0, col0,
+                   lane, via_tma);
         }
       }
     }
@@ -392,7 +475,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       atomicOr(p.status, kDevTimeout);
       *abort_flag = 1;
     }
-    if (lane == 0) bulk_wait<0>();  // every store has completed before the CTA exits
+    if (lane == 0) bulk_wait_read<0>();  // no store still reads shared memory at exit
   }
 
   __syncthreads();
@@ -530,11 +613,11 @@ static int make_plan(int which, int64_t M, int64_t N, int64_t K, int bits, int G
   return SQ_OK;
 }
 
-template <int kF8>
+template <int kF8, bool kMulti>
 static int configure_kernel(int dev) {
   static bool done[64] = {};
   if (dev >= 0 && dev < 64 && done[dev]) return SQ_OK;
-  const cudaError_t err = cudaFuncSetAttribute(shiftmm_kernel<kF8>,
+  const cudaError_t err = cudaFuncSetAttribute(shiftmm_kernel<kF8, kMulti>,
                                                cudaFuncAttributeMaxDynamicSharedMemorySize,
                                                static_cast<int>(kSmemBytes));
   if (err != cudaSuccess) return cuda_fail(err, "cudaFuncSetAttribute");
@@ -639,12 +722,23 @@ static int run_gemm(int which, const void* a_codes, int64_t lda, const void* b_c
   }
   const int units = pl.m_tiles * pl.n_tiles * pl.splits;
   const int grid = units < sms ? units : sms;
+  const bool multi = pl.kb_per_split > pl.chunk_kb;  // some unit spans several exact chunks
   if (eb == 1) {
-    if ((st = configure_kernel<1>(dev)) != SQ_OK) return st;
-    shiftmm_kernel<1><<<grid, kThreads, kSmemBytes, s>>>(ma, mb, my, mw, p);
+    if (multi) {
+      if ((st = configure_kernel<1, true>(dev)) != SQ_OK) return st;
+      shiftmm_kernel<1, true><<<grid, kThreads, kSmemBytes, s>>>(ma, mb, my, mw, p);
+    } else {
+      if ((st = configure_kernel<1, false>(dev)) != SQ_OK) return st;
+      shiftmm_kernel<1, false><<<grid, kThreads, kSmemBytes, s>>>(ma, mb, my, mw, p);
+    }
   } else {
-    if ((st = configure_kernel<0>(dev)) != SQ_OK) return st;
-    shiftmm_kernel<0><<<grid, kThreads, kSmemBytes, s>>>(ma, mb, my, mw, p);
+    if (multi) {
+      if ((st = configure_kernel<0, true>(dev)) != SQ_OK) return st;
+      shiftmm_kernel<0, true><<<grid, kThreads, kSmemBytes, s>>>(ma, mb, my, mw, p);
+    } else {
+      if ((st = configure_kernel<0, false>(dev)) != SQ_OK) return st;
+      shiftmm_kernel<0, false><<<grid, kThreads, kSmemBytes, s>>>(ma, mb, my, mw, p);
+    }
   }
   err = cudaGetLastError();
   if (err != cudaSuccess) return cuda_fail(err, "shiftmm_kernel launch");

@@ -105,13 +105,17 @@ class QuantLinear:
             self.acc = {"fwd": torch.zeros((M, N_), dtype=torch.int64, device=dev),
                         "dgrad": torch.zeros((M, K), dtype=torch.int64, device=dev),
                         "wgrad": torch.zeros((K, N_), dtype=torch.int64, device=dev)}
-        self.ws = None
+        # one split-K workspace per GEMM, so the three may run concurrently
+        self.ws_fwd = self.ws_dgrad = self.ws_wgrad = None
         if use_workspace:
-            need = max(N.shiftquant_gemm_workspace_bytes(0, M, N_, K, bits, n_groups),
-                       N.shiftquant_gemm_workspace_bytes(1, M, K, N_, bits, n_groups),
-                       N.shiftquant_gemm_workspace_bytes(2, K, N_, M, bits, n_groups))
-            if need:
-                self.ws = torch.zeros(need // 4, dtype=torch.int32, device=dev)
+            def ws(which, m, n, k):
+                need = N.shiftquant_gemm_workspace_bytes(which, m, n, k, bits, n_groups)
+                return torch.zeros(need // 4, dtype=torch.int32, device=dev) if need else None
+            self.ws_fwd = ws(0, M, N_, K)
+            self.ws_dgrad = ws(1, M, K, N_)
+            self.ws_wgrad = ws(2, K, N_, M)
+        self.ws = self.ws_fwd if self.ws_fwd is not None else (
+            self.ws_dgrad if self.ws_dgrad is not None else self.ws_wgrad)
 
     # --- the hot path, step by step --------------------------------------------------
     def quantize_activation(self, x, stream=None):
@@ -129,20 +133,20 @@ class QuantLinear:
     def forward(self, stream=None):
         N.shiftquant_gemm_fwd(self.x.codes, self.x.scale, self.wf.codes, self.wf.scale, self.M,
                               self.N, self.K, self.bits, self.G, self.y,
-                              self.acc["fwd"] if self.acc else None, self.ws, self.status,
+                              self.acc["fwd"] if self.acc else None, self.ws_fwd, self.status,
                               stream)
 
     def dgrad(self, stream=None):
         N.shiftquant_gemm_dgrad(self.g.codes, self.g.scale, self.wd.codes, self.wd.scale, self.M,
                                 self.K, self.N, self.bits, self.G, self.dx,
-                                self.acc["dgrad"] if self.acc else None, self.ws, self.status,
-                                stream)
+                                self.acc["dgrad"] if self.acc else None, self.ws_dgrad,
+                                self.status, stream)
 
     def wgrad(self, stream=None):
         N.shiftquant_gemm_wgrad(self.x.codes_t, self.x.scale, self.x.exp, self.g.codes_t,
                                 self.g.scale, self.g.exp, self.K, self.N, self.M, self.bits,
                                 self.G, self.dw, self.acc["wgrad"] if self.acc else None,
-                                self.ws, self.status, stream)
+                                self.ws_wgrad, self.status, stream)
 
     def step(self, x, w, dy, seed, stream=None):
         """One training step of the layer: every quantizer pass and all three GEMMs."""
@@ -152,6 +156,34 @@ class QuantLinear:
         self.forward(stream)
         self.dgrad(stream)
         self.wgrad(stream)
+
+    def step_concurrent(self, x, w, dy, seed, streams):
+        """The same step with its independent chains on three streams (forked from and joined
+        back to the current stream): activation chain and forward GEMM, gradient chain and
+        loss-propagation GEMM, then the weight-gradient GEMM once both code sets exist.
+        Capturable in a CUDA graph, which then runs the chains concurrently."""
+        main = torch.cuda.current_stream()
+        s_x, s_g, s_w = streams
+        for s in streams:
+            s.wait_stream(main)
+        with torch.cuda.stream(s_x):
+            self.quantize_activation(x, s_x)
+            x_done = torch.cuda.Event()
+            x_done.record(s_x)
+            weight_quantize_fwd(w, self.wf, self.x.exp, self.bits, self.G, self.status, s_x)
+            self.forward(s_x)
+        with torch.cuda.stream(s_g):
+            self.quantize_gradient(dy, seed, s_g)
+            g_done = torch.cuda.Event()
+            g_done.record(s_g)
+            weight_quantize_dgrad(w, self.wd, self.g.exp, self.bits, self.G, self.status, s_g)
+            self.dgrad(s_g)
+        with torch.cuda.stream(s_w):
+            s_w.wait_event(x_done)
+            s_w.wait_event(g_done)
+            self.wgrad(s_w)
+        for s in streams:
+            main.wait_stream(s)
 
     @property
     def gemm_ops(self) -> int:

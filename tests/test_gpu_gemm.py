@@ -174,3 +174,24 @@ def test_zero_gradient_gives_zero_outputs():
     dy[:] = 0
     lay = run_and_compare(x, w, dy, 4, 4)
     assert (lay.dx == 0).all() and (lay.dw == 0).all()
+
+
+def test_concurrent_step_equals_serial_step():
+    # the three-stream step (as captured in the benchmark's CUDA graph) computes exactly
+    # what the serial step computes
+    rng = np.random.default_rng(77)
+    x, w, dy = layer_inputs(rng, 4096, 320, 192)
+    ser = L.QuantLinear(4096, 320, 192, 4, 4, "cuda", with_acc=True)
+    con = L.QuantLinear(4096, 320, 192, 4, 4, "cuda", with_acc=True)
+    xg, wg, dyg = to_gpu(x), to_gpu(w), to_gpu(dy)
+    ser.step(xg, wg, dyg, 5)
+    streams = [torch.cuda.Stream() for _ in range(3)]
+    graph = L.CapturedStep(lambda: con.step_concurrent(xg, wg, dyg, 5, streams))
+    graph.replay()
+    graph.replay()
+    torch.cuda.synchronize()
+    assert ser.status.item() == 0 and con.status.item() == 0
+    for k in ("fwd", "dgrad", "wgrad"):
+        np.testing.assert_array_equal(ser.acc[k].cpu().numpy(), con.acc[k].cpu().numpy())
+    for a, b in ((ser.y, con.y), (ser.dx, con.dx), (ser.dw, con.dw)):
+        np.testing.assert_array_equal(a.cpu().numpy(), b.cpu().numpy())
