@@ -169,8 +169,9 @@ class Step:
         n = 0
         N = self.N
         for lay in self.layers:
-            n += 2 + 1 + 2 + 1          # calibrate SHIFT (range + grouping) + quantize, X and dY
-            n += 1 + 1 + 1 + 1          # weights: range + quantize, both roles
+            n += 2 + 1 + 2 + 1          # X and dY: range init + range/grouping, quantize
+            n += 2 + 1 + 1 + 1          # weights: range init + range, quantize (out-channel);
+                                        # row range, quantize (in-channel)
             n += 3                      # the three GEMM kernels
             n += sum(ws is not None for ws in (lay.ws_fwd, lay.ws_dgrad, lay.ws_wgrad))  # finalize
         return n
@@ -250,8 +251,9 @@ def run_ours(args, rank, world, local_rank):
     assert st.status_ok(), "device status set during warm-up"
 
     # the timed step is the whole step captured in one CUDA graph; each layer's activation
-    # chain, gradient chain and weight-gradient GEMM run on their own streams inside it
-    streams = [[torch.cuda.Stream(device=dev) for _ in range(3)] for _ in st.layers]
+    # chain, gradient chain, two weight roles and weight-gradient GEMM run on their own
+    # streams inside it
+    streams = [[torch.cuda.Stream(device=dev) for _ in range(5)] for _ in st.layers]
 
     def run_step_concurrent(i):
         for lay, (x, w, dy), ss in zip(st.layers, st.inputs, streams):
@@ -387,10 +389,10 @@ def run_ours(args, rank, world, local_rank):
                           nominal_hbm_gbs=7900.0, frac_nominal=q_gbs / 7900.0),
         "breakdown_ms_per_step": {k: v / args.steps for k, v in kind_ms.items()},
         "calls_ms_per_step": [[f"{n}", round(v / args.steps, 5)] for n, v in zip(names, call_ms)],
-        "timing": "CUDA events around one CUDA-graph replay of the whole step (per layer: "
-                  "activation chain + forward GEMM, gradient chain + loss-propagation GEMM, "
-                  "then the weight-gradient GEMM, on three streams); breakdown from un-graphed "
-                  "serial calls queued behind a sleep kernel",
+        "timing": "CUDA events around one CUDA-graph replay of the whole step (per layer five "
+                  "streams: activation chain, gradient chain, forward weights + GEMM, "
+                  "loss-propagation weights + GEMM, weight-gradient GEMM); breakdown from "
+                  "un-graphed serial calls queued behind a sleep kernel",
         "gpu_launches": st.launches_per_step() * args.steps,
         "clocks": clocks,
         "status_ok": ok,

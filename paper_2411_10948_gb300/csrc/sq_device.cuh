@@ -27,6 +27,17 @@ __device__ __forceinline__ uint64_t globaltimer_ns() {
   return t;
 }
 
+// 16-byte streaming load (read-only path, no L1 allocation, 256-byte L2 prefetch).  The
+// asm is volatile so a run of these stays in program order: all of them are issued before
+// the first result is used, whatever register budget the compiler aims for.
+__device__ __forceinline__ float4 ld_stream_v4(const float* p) {
+  float4 v;
+  asm volatile("ld.global.nc.L1::no_allocate.L2::256B.v4.f32 {%0, %1, %2, %3}, [%4];"
+               : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
+               : "l"(p));
+  return v;
+}
+
 // ------------------------------------------------------------------ mbarrier
 __device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
   asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count)

@@ -36,13 +36,6 @@ int fail(int status, const char* fmt, ...) {
 
 static void clear_error() { g_last_error[0] = 0; }
 
-static int num_sms() {
-  int dev = 0, n = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess) return 148;
-  if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 148;
-  return n > 0 ? n : 148;
-}
-
 // ===================================================================== range pass
 constexpr int kColTx = 32;  // threads along columns, 4 columns each: 128 columns per block
 constexpr int kColTy = 8;   // threads along rows
@@ -51,49 +44,96 @@ __device__ __forceinline__ uint32_t abs_bits(float v) { return __float_as_uint(v
 
 // range_bits[c] = max over this block's rows of |x[r, c]| as an ordered bit pattern
 // (for non-negative floats, larger value <=> larger unsigned pattern; NaN sorts above Inf).
-__global__ void __launch_bounds__(kColTx* kColTy)
-    colmax_kernel(const float* __restrict__ x, int64_t R, int64_t C, int64_t ld,
-                  int64_t rows_per_block, int vec, unsigned* __restrict__ range_bits,
-                  int* __restrict__ status) {
-  __shared__ unsigned red[kColTy][kColTx * 4];
-  const int tx = threadIdx.x, ty = threadIdx.y;
-  const int64_t c0 = (static_cast<int64_t>(blockIdx.x) * kColTx + tx) * 4;
-  const int64_t rb = static_cast<int64_t>(blockIdx.y) * rows_per_block;
-  const int64_t re = min(R, rb + rows_per_block);
-  unsigned m0 = 0, m1 = 0, m2 = 0, m3 = 0;
-  if (vec && c0 + 3 < C) {
-    const float* base = x + c0;
-    int64_t r = rb + ty;
+// exponent of one channel: max{e in [0, G-1] : r 2^e <= tau}; the product by 2^e is exact
+// (no rounding) for every finite r <= tau, so the comparison is exact
+__device__ __forceinline__ int group_exponent(float r, float tau, int G) {
+  if (r == 0.0f) return G - 1;
+  int e = 0;
 #pragma unroll 1
-    for (; r + 7 * kColTy < re; r += 8 * kColTy) {
-      float4 v[8];  // eight rows in flight per thread
-#pragma unroll
-      for (int u = 0; u < 8; ++u)
-        v[u] = __ldg(reinterpret_cast<const float4*>(base + (r + u * kColTy) * ld));
+  for (int k = 1; k < G; ++k) {
+    const float scaled = __fmul_rn(r, __int_as_float((127 + k) << 23));  // r 2^k
+    if (scaled <= tau) e = k;
+    else break;
+  }
+  return e;
+}
+
+// zero the range accumulators (and the completion counter of the grouping step)
+__global__ void __launch_bounds__(256)
+    calib_init_kernel(unsigned* __restrict__ range_bits, int64_t C, unsigned* __restrict__ counter) {
+  for (int64_t c = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; c < C;
+       c += static_cast<int64_t>(gridDim.x) * blockDim.x)
+    range_bits[c] = 0u;
+  if (counter != nullptr && blockIdx.x == 0 && threadIdx.x == 0) *counter = 0u;
+}
+
+// Range pass: one wave of blocks, block (x, y) owning 128 columns and the 64-row tiles
+// y, y + gridDim.y, ... (so the blocks resident at one time read a contiguous band of whole
+// rows: long DRAM bursts).  Warp w reads rows 8w .. 8w+7 of a tile with all eight 16-byte
+// loads in flight; lane l owns columns 4l .. 4l+3.  The block's per-column maxima go to
+// range_bits with one atomic max each, on the ordered bit pattern of the non-negative
+// floats (NaN sorts above Inf).
+// G > 0: the block that finishes last also performs the grouping (Eq. 3): tau_0 and the
+// exponents.  Until then tau0_out holds the count of finished blocks.
+constexpr int kRangeRows = 64;
+
+__global__ void __launch_bounds__(kColTx* kColTy)
+    colmax_kernel(const float* __restrict__ x, int64_t R, int64_t C, int64_t ld, int vec,
+                  unsigned* __restrict__ range_bits, int* __restrict__ status, int G,
+                  float* __restrict__ tau0_out, uint8_t* __restrict__ exp_out) {
+  __shared__ unsigned red[kColTy][kColTx * 4];
+  __shared__ unsigned last_block;
+  const int tx = threadIdx.x, ty = threadIdx.y;   // tx: lane (columns), ty: warp (rows)
+  const int64_t c0 = (static_cast<int64_t>(blockIdx.x) * kColTx + tx) * 4;
+  unsigned m0 = 0, m1 = 0, m2 = 0, m3 = 0;
+  // grid-stride over row tiles: the blocks resident together cover consecutive row tiles
+  if (vec && c0 + 3 < C) {
+    // software-pipelined: the next tile's eight loads leave before this tile is reduced.
+    // Rows past the end re-read the last row, which leaves a maximum unchanged.
+    auto load_tile = [&](int64_t t, float4 (&v)[8]) {
+      const int64_t r0 = t * kRangeRows + ty * 8;
 #pragma unroll
       for (int u = 0; u < 8; ++u) {
-        m0 = max(m0, abs_bits(v[u].x));
-        m1 = max(m1, abs_bits(v[u].y));
-        m2 = max(m2, abs_bits(v[u].z));
-        m3 = max(m3, abs_bits(v[u].w));
+        const int64_t r = min(r0 + u, R - 1);
+        v[u] = ld_stream_v4(x + r * ld + c0);
       }
-    }
+    };
+    float4 cur[8], nxt[8];
+    int64_t t = blockIdx.y;
+    if (t * kRangeRows < R) {
+      load_tile(t, cur);
 #pragma unroll 1
-    for (; r < re; r += kColTy) {
-      const float4 v = __ldg(reinterpret_cast<const float4*>(base + r * ld));
-      m0 = max(m0, abs_bits(v.x));
-      m1 = max(m1, abs_bits(v.y));
-      m2 = max(m2, abs_bits(v.z));
-      m3 = max(m3, abs_bits(v.w));
+      while (true) {
+        const int64_t tn = t + gridDim.y;
+        const bool more = tn * kRangeRows < R;
+        if (more) load_tile(tn, nxt);
+#pragma unroll
+        for (int u = 0; u < 8; ++u) {
+          m0 = max(m0, abs_bits(cur[u].x));
+          m1 = max(m1, abs_bits(cur[u].y));
+          m2 = max(m2, abs_bits(cur[u].z));
+          m3 = max(m3, abs_bits(cur[u].w));
+        }
+        if (!more) break;
+#pragma unroll
+        for (int u = 0; u < 8; ++u) cur[u] = nxt[u];
+        t = tn;
+      }
     }
   } else {
 #pragma unroll 1
-    for (int64_t r = rb + ty; r < re; r += kColTy) {
-      const float* row = x + r * ld;
-      if (c0 + 0 < C) m0 = max(m0, abs_bits(__ldg(row + c0 + 0)));
-      if (c0 + 1 < C) m1 = max(m1, abs_bits(__ldg(row + c0 + 1)));
-      if (c0 + 2 < C) m2 = max(m2, abs_bits(__ldg(row + c0 + 2)));
-      if (c0 + 3 < C) m3 = max(m3, abs_bits(__ldg(row + c0 + 3)));
+    for (int64_t t = blockIdx.y; t * kRangeRows < R; t += gridDim.y) {
+      const int64_t r0 = t * kRangeRows + ty * 8;
+#pragma unroll 1
+      for (int u = 0; u < 8; ++u) {
+        const int64_t r = r0 + u;
+        if (r >= R) break;
+        const float* row = x + r * ld;
+        if (c0 + 0 < C) m0 = max(m0, abs_bits(__ldg(row + c0 + 0)));
+        if (c0 + 1 < C) m1 = max(m1, abs_bits(__ldg(row + c0 + 1)));
+        if (c0 + 2 < C) m2 = max(m2, abs_bits(__ldg(row + c0 + 2)));
+        if (c0 + 3 < C) m3 = max(m3, abs_bits(__ldg(row + c0 + 3)));
+      }
     }
   }
   red[ty][tx * 4 + 0] = m0;
@@ -114,6 +154,40 @@ __global__ void __launch_bounds__(kColTx* kColTy)
       }
     }
     if (bad) atomicOr(status, kDevNonFinite);
+  }
+  if (G == 0) return;
+  // grouping by the last block to finish (the classic fence-then-count pattern)
+  __threadfence();
+  __syncthreads();
+  const int tid = ty * kColTx + tx;
+  if (tid == 0) {
+    const unsigned total = gridDim.x * gridDim.y;
+    last_block = atomicAdd(reinterpret_cast<unsigned*>(tau0_out), 1u) == total - 1u;
+  }
+  __syncthreads();
+  if (!last_block) return;
+  __threadfence();
+  unsigned m = 0;
+  for (int64_t c = tid; c < C; c += kColTx * kColTy) m = max(m, __ldcg(range_bits + c));
+  m = __reduce_max_sync(0xFFFFFFFFu, m);
+  unsigned* wmax = &red[0][0];
+  if ((tid & 31) == 0) wmax[tid >> 5] = m;
+  __syncthreads();
+  if (tid < 32) {
+    unsigned v = tid < (kColTx * kColTy) / 32 ? wmax[tid] : 0u;
+    v = __reduce_max_sync(0xFFFFFFFFu, v);
+    if (tid == 0) wmax[32] = v;
+  }
+  __syncthreads();
+  const unsigned tb = wmax[32];
+  const float tau = __uint_as_float(tb);
+  const bool nonfinite = tb >= 0x7F800000u;
+  for (int64_t c = tid; c < C; c += kColTx * kColTy)
+    exp_out[c] = static_cast<uint8_t>(nonfinite ? 0 : group_exponent(__uint_as_float(__ldcg(range_bits + c)), tau, G));
+  __syncthreads();
+  if (tid == 0) {
+    *tau0_out = tau;  // replaces the block counter
+    if (nonfinite) atomicOr(status, kDevNonFinite);
   }
 }
 
@@ -141,51 +215,6 @@ __global__ void __launch_bounds__(256)
   if (lane == 0) {
     range[r] = __uint_as_float(m);
     if (m >= 0x7F800000u) atomicOr(status, kDevNonFinite);
-  }
-}
-
-// tau_0 and the exponents.  e_c = max{e in [0, G-1] : r_c 2^e <= tau_0}; the product by
-// 2^e is exact (no rounding) for every finite r_c <= tau_0, so the comparison is exact.
-__global__ void __launch_bounds__(1024)
-    group_kernel(const unsigned* __restrict__ range_bits, int64_t C, int G,
-                 float* __restrict__ tau0_out, uint8_t* __restrict__ exp_out,
-                 int* __restrict__ status) {
-  __shared__ unsigned warp_max[32];
-  __shared__ unsigned tau_bits_s;
-  unsigned m = 0;
-  for (int64_t c = threadIdx.x; c < C; c += blockDim.x) m = max(m, range_bits[c]);
-  m = __reduce_max_sync(0xFFFFFFFFu, m);
-  if ((threadIdx.x & 31) == 0) warp_max[threadIdx.x >> 5] = m;
-  __syncthreads();
-  if (threadIdx.x < 32) {
-    unsigned v = threadIdx.x < (blockDim.x >> 5) ? warp_max[threadIdx.x] : 0u;
-    v = __reduce_max_sync(0xFFFFFFFFu, v);
-    if (threadIdx.x == 0) tau_bits_s = v;
-  }
-  __syncthreads();
-  const unsigned tb = tau_bits_s;
-  const float tau = __uint_as_float(tb);
-  const bool nonfinite = tb >= 0x7F800000u;
-  if (threadIdx.x == 0) {
-    *tau0_out = tau;
-    if (nonfinite) atomicOr(status, kDevNonFinite);
-  }
-  for (int64_t c = threadIdx.x; c < C; c += blockDim.x) {
-    const float r = __uint_as_float(range_bits[c]);
-    int e = 0;
-    if (!nonfinite) {
-      if (r == 0.0f) {
-        e = G - 1;
-      } else {
-#pragma unroll 1
-        for (int k = 1; k < G; ++k) {
-          const float scaled = __fmul_rn(r, __int_as_float((127 + k) << 23));  // r 2^k
-          if (scaled <= tau) e = k;
-          else break;
-        }
-      }
-    }
-    exp_out[c] = static_cast<uint8_t>(e);
   }
 }
 
@@ -270,7 +299,7 @@ __device__ __forceinline__ void quantize_tile(const QuantArgs& a, uint8_t* tile_
     const int64_t r = r0 + wq * 8 + i;
     const float* row = a.x + r * a.ld;
     if (FULL) {
-      xin[i] = __ldg(reinterpret_cast<const float4*>(row + cb));
+      xin[i] = ld_stream_v4(row + cb);
     } else {
       xin[i] = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
       if (r < a.R) {
@@ -570,39 +599,49 @@ extern "C" sq_status shiftquant_calibrate(const float* x, int64_t rows, int64_t 
     err = cudaGetLastError();
     return err == cudaSuccess ? SQ_OK : cuda_fail(err, "rowmax_kernel launch");
   }
-  if (cols > 0) {
-    err = cudaMemsetAsync(range_out, 0, sizeof(float) * cols, s);
-    if (err != cudaSuccess) return cuda_fail(err, "cudaMemsetAsync");
+  const bool shift = gran == SQ_GRAN_SHIFT;
+  if (rows == 0 || cols == 0) {
+    // every range is 0: tau_0 = 0 and every channel in the last group
+    if (cols > 0) {
+      err = cudaMemsetAsync(range_out, 0, sizeof(float) * cols, s);
+      if (err == cudaSuccess && shift) err = cudaMemsetAsync(exp_out, n_groups - 1, cols, s);
+      if (err != cudaSuccess) return cuda_fail(err, "cudaMemsetAsync");
+    }
+    if (shift) {
+      err = cudaMemsetAsync(tau0_out, 0, sizeof(float), s);
+      if (err != cudaSuccess) return cuda_fail(err, "cudaMemsetAsync");
+    }
+    return SQ_OK;
   }
-  if (rows > 0 && cols > 0) {
-    const int64_t cblocks = (cols + kColTx * 4 - 1) / (kColTx * 4);
-    // one full wave of resident blocks, each streaming a band of rows
-    int per_sm = 0;
-    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, colmax_kernel, kColTx * kColTy, 0) !=
-            cudaSuccess || per_sm < 1)
-      per_sm = 4;
-    const int64_t target = static_cast<int64_t>(num_sms()) * per_sm;
-    int64_t rblocks = target / cblocks;  // rounded down: a partial second wave costs a whole one
-    const int64_t max_rblocks = (rows + 31) / 32;
-    if (rblocks > max_rblocks) rblocks = max_rblocks;
-    if (rblocks > 65535) rblocks = 65535;
-    if (rblocks < 1) rblocks = 1;
-    const int64_t rpb = (rows + rblocks - 1) / rblocks;
-    rblocks = (rows + rpb - 1) / rpb;
-    const int vec = (ld % 4 == 0) && aligned16(x);
-    dim3 grid(static_cast<unsigned>(cblocks), static_cast<unsigned>(rblocks));
-    colmax_kernel<<<grid, dim3(kColTx, kColTy), 0, s>>>(
-        x, rows, cols, ld, rpb, vec, reinterpret_cast<unsigned*>(range_out), dev_status);
+  {
+    const int64_t iblocks = (cols + 255) / 256;
+    calib_init_kernel<<<static_cast<unsigned>(iblocks < 1024 ? iblocks : 1024), 256, 0, s>>>(
+        reinterpret_cast<unsigned*>(range_out), cols,
+        shift ? reinterpret_cast<unsigned*>(tau0_out) : nullptr);
     err = cudaGetLastError();
-    if (err != cudaSuccess) return cuda_fail(err, "colmax_kernel launch");
+    if (err != cudaSuccess) return cuda_fail(err, "calib_init_kernel launch");
   }
-  if (gran == SQ_GRAN_SHIFT) {
-    group_kernel<<<1, 1024, 0, s>>>(reinterpret_cast<const unsigned*>(range_out), cols, n_groups,
-                                    tau0_out, exp_out, dev_status);
-    err = cudaGetLastError();
-    if (err != cudaSuccess) return cuda_fail(err, "group_kernel launch");
-  }
-  return SQ_OK;
+  const int64_t cblocks = (cols + kColTx * 4 - 1) / (kColTx * 4);
+  const int64_t tiles = (rows + kRangeRows - 1) / kRangeRows;
+  // one wave of resident blocks (never a partial second wave)
+  int per_sm = 0, dev = 0, sms = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || sms < 1)
+    sms = 148;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, colmax_kernel, kColTx * kColTy, 0) !=
+          cudaSuccess || per_sm < 1)
+    per_sm = 4;
+  int64_t rblocks = static_cast<int64_t>(sms) * per_sm / cblocks;
+  if (rblocks > tiles) rblocks = tiles;
+  if (rblocks > 65535) rblocks = 65535;
+  if (rblocks < 1) rblocks = 1;
+  const int vec = (ld % 4 == 0) && aligned16(x);
+  dim3 grid(static_cast<unsigned>(cblocks), static_cast<unsigned>(rblocks));
+  colmax_kernel<<<grid, dim3(kColTx, kColTy), 0, s>>>(
+      x, rows, cols, ld, vec, reinterpret_cast<unsigned*>(range_out), dev_status,
+      shift ? n_groups : 0, tau0_out, exp_out);
+  err = cudaGetLastError();
+  return err == cudaSuccess ? SQ_OK : cuda_fail(err, "colmax_kernel launch");
 }
 
 extern "C" sq_status shiftquant_quantize(const float* x, int64_t rows, int64_t cols, int64_t ld,

@@ -158,29 +158,44 @@ class QuantLinear:
         self.wgrad(stream)
 
     def step_concurrent(self, x, w, dy, seed, streams):
-        """The same step with its independent chains on three streams (forked from and joined
-        back to the current stream): activation chain and forward GEMM, gradient chain and
-        loss-propagation GEMM, then the weight-gradient GEMM once both code sets exist.
-        Capturable in a CUDA graph, which then runs the chains concurrently."""
+        """The same step on five streams forked from (and joined back to) the current one:
+        the activation chain, the gradient chain, each weight role (its range pass right
+        away, its quantization once the other operand's exponents exist, then its GEMM once
+        the codes exist) and the weight-gradient GEMM once both code sets exist.
+        Capturable in a CUDA graph, which then runs the independent work concurrently."""
         main = torch.cuda.current_stream()
-        s_x, s_g, s_w = streams
+        s_x, s_g, s_wf, s_wd, s_w = streams
         for s in streams:
             s.wait_stream(main)
-        with torch.cuda.stream(s_x):
-            self.quantize_activation(x, s_x)
-            x_done = torch.cuda.Event()
-            x_done.record(s_x)
-            weight_quantize_fwd(w, self.wf, self.x.exp, self.bits, self.G, self.status, s_x)
-            self.forward(s_x)
-        with torch.cuda.stream(s_g):
-            self.quantize_gradient(dy, seed, s_g)
-            g_done = torch.cuda.Event()
-            g_done.record(s_g)
-            weight_quantize_dgrad(w, self.wd, self.g.exp, self.bits, self.G, self.status, s_g)
-            self.dgrad(s_g)
+        ev = {k: torch.cuda.Event() for k in ("x_cal", "x_q", "g_cal", "g_q")}
+        b, G, st = self.bits, self.G, self.status
+        for s_, q, t, mode, sd, cal, qd in ((s_x, self.x, x, N.SQ_ROUND_NEAREST_EVEN, 0, "x_cal", "x_q"),
+                                           (s_g, self.g, dy, N.SQ_ROUND_STOCHASTIC, seed, "g_cal", "g_q")):
+            with torch.cuda.stream(s_):
+                N.shiftquant_calibrate(t, N.SQ_GRAN_SHIFT, G, q.range, q.tau0, q.exp, st, s_)
+                ev[cal].record(s_)
+                N.shiftquant_quantize(t, N.SQ_GRAN_SHIFT, b, G, q.tau0, q.exp, None, mode, sd,
+                                      q.codes, q.codes_t, q.scale, s_)
+                ev[qd].record(s_)
+        with torch.cuda.stream(s_wf):
+            N.shiftquant_calibrate(w, N.SQ_GRAN_PER_COL, G, self.wf.range, None, None, st, s_wf)
+            s_wf.wait_event(ev["x_cal"])
+            N.shiftquant_quantize(w, N.SQ_GRAN_PER_COL, b, G, self.wf.range, None, self.x.exp,
+                                  N.SQ_ROUND_NEAREST_EVEN, 0, None, self.wf.codes, self.wf.scale,
+                                  s_wf)
+            s_wf.wait_event(ev["x_q"])
+            self.forward(s_wf)
+        with torch.cuda.stream(s_wd):
+            N.shiftquant_calibrate(w, N.SQ_GRAN_PER_ROW, G, self.wd.range, None, None, st, s_wd)
+            s_wd.wait_event(ev["g_cal"])
+            N.shiftquant_quantize(w, N.SQ_GRAN_PER_ROW, b, G, self.wd.range, None, self.g.exp,
+                                  N.SQ_ROUND_NEAREST_EVEN, 0, self.wd.codes, None, self.wd.scale,
+                                  s_wd)
+            s_wd.wait_event(ev["g_q"])
+            self.dgrad(s_wd)
         with torch.cuda.stream(s_w):
-            s_w.wait_event(x_done)
-            s_w.wait_event(g_done)
+            s_w.wait_event(ev["x_q"])
+            s_w.wait_event(ev["g_q"])
             self.wgrad(s_w)
         for s in streams:
             main.wait_stream(s)

@@ -177,7 +177,7 @@ def test_zero_gradient_gives_zero_outputs():
 
 
 def test_concurrent_step_equals_serial_step():
-    # the three-stream step (as captured in the benchmark's CUDA graph) computes exactly
+    # the five-stream step (as captured in the benchmark's CUDA graph) computes exactly
     # what the serial step computes
     rng = np.random.default_rng(77)
     x, w, dy = layer_inputs(rng, 4096, 320, 192)
@@ -185,7 +185,7 @@ def test_concurrent_step_equals_serial_step():
     con = L.QuantLinear(4096, 320, 192, 4, 4, "cuda", with_acc=True)
     xg, wg, dyg = to_gpu(x), to_gpu(w), to_gpu(dy)
     ser.step(xg, wg, dyg, 5)
-    streams = [torch.cuda.Stream() for _ in range(3)]
+    streams = [torch.cuda.Stream() for _ in range(5)]
     graph = L.CapturedStep(lambda: con.step_concurrent(xg, wg, dyg, 5, streams))
     graph.replay()
     graph.replay()
