@@ -159,9 +159,7 @@ class Step:
                 ("quantize", lambda lay=lay, w=w: N.shiftquant_quantize(
                     w, N.SQ_GRAN_PER_ROW, lay.bits, lay.G, lay.wd.range, None, lay.g.exp,
                     N.SQ_ROUND_NEAREST_EVEN, 0, lay.wd.codes, None, lay.wd.scale)),
-                ("gemm", lay.forward),
-                ("gemm", lay.dgrad),
-                ("gemm", lay.wgrad),
+                ("gemm", lay.gemms),   # forward, loss propagation, weight gradient: one launch
             ]
         return out
 
@@ -172,7 +170,7 @@ class Step:
             n += 2 + 1 + 2 + 1          # X and dY: range init + range/grouping, quantize
             n += 2 + 1 + 1 + 1          # weights: range init + range, quantize (out-channel);
                                         # row range, quantize (in-channel)
-            n += 3                      # the three GEMM kernels
+            n += 1                      # the three GEMMs: one launch
             n += sum(ws is not None for ws in (lay.ws_fwd, lay.ws_dgrad, lay.ws_wgrad))  # finalize
         return n
 
@@ -180,7 +178,7 @@ class Step:
         return sum(l.gemm_ops for l in self.layers)
 
     def gemm_flops_per_launch(self):
-        return [2 * l.M * l.N * l.K for l in self.layers for _ in range(3)]
+        return [3 * 2 * l.M * l.N * l.K for l in self.layers]
 
     def quantizer_bytes(self) -> int:
         """Algorithmic HBM bytes of the quantizer passes of one step."""
@@ -250,10 +248,10 @@ def run_ours(args, rank, world, local_rank):
     torch.cuda.synchronize()
     assert st.status_ok(), "device status set during warm-up"
 
-    # the timed step is the whole step captured in one CUDA graph; each layer's activation
-    # chain, gradient chain, two weight roles and weight-gradient GEMM run on their own
-    # streams inside it
-    streams = [[torch.cuda.Stream(device=dev) for _ in range(5)] for _ in st.layers]
+    # the timed step is the whole step captured in one CUDA graph: per layer, the activation
+    # chain, the gradient chain and the two weight roles on their own streams, then the
+    # layer's three GEMMs as one launch
+    streams = [[torch.cuda.Stream(device=dev) for _ in range(4)] for _ in st.layers]
 
     def run_step_concurrent(i):
         for lay, (x, w, dy), ss in zip(st.layers, st.inputs, streams):
@@ -355,7 +353,8 @@ def run_ours(args, rank, world, local_rank):
     gemm_roof = {"bound": "tensor", "achieved": gemm_tflops, "peak": tensor_peak,
                  "unit": "TFLOP/s", "frac": gemm_tflops / tensor_peak,
                  "traffic": profiled_traffic(args.workload),
-                 "kernel": "shiftmm_kernel<%d>" % (1 if fp8 else 0),
+                 "kernel": "shiftmm_kernel<%d, *> (one launch = forward + loss propagation + "
+                           "weight gradient of a layer)" % (1 if fp8 else 0),
                  "peak_source": (f"{peak_src} bf16 burst" + (" x 2 (nominal FP8/BF16)" if fp8 else ""))}
     quant_roof = {"bound": "hbm", "achieved": q_gbs, "peak": peaks["hbm_gbs"], "unit": "GB/s",
                   "frac": q_gbs / peaks["hbm_gbs"], "kernel": "calibrate + quantize",
@@ -389,10 +388,10 @@ def run_ours(args, rank, world, local_rank):
                           nominal_hbm_gbs=7900.0, frac_nominal=q_gbs / 7900.0),
         "breakdown_ms_per_step": {k: v / args.steps for k, v in kind_ms.items()},
         "calls_ms_per_step": [[f"{n}", round(v / args.steps, 5)] for n, v in zip(names, call_ms)],
-        "timing": "CUDA events around one CUDA-graph replay of the whole step (per layer five "
-                  "streams: activation chain, gradient chain, forward weights + GEMM, "
-                  "loss-propagation weights + GEMM, weight-gradient GEMM); breakdown from "
-                  "un-graphed serial calls queued behind a sleep kernel",
+        "timing": "CUDA events around one CUDA-graph replay of the whole step (per layer: "
+                  "activation chain, gradient chain and both weight roles on four streams, "
+                  "then the three GEMMs as one launch); breakdown from un-graphed serial "
+                  "calls (one launch per GEMM) queued behind a sleep kernel",
         "gpu_launches": st.launches_per_step() * args.steps,
         "clocks": clocks,
         "status_ok": ok,

@@ -168,6 +168,49 @@ sq_status shiftquant_gemm_wgrad(const void *xt_codes, int64_t ldx, const float *
                                 void *workspace, size_t workspace_bytes,
                                 int32_t *dev_status, void *stream);
 
+/* The three GEMMs of one quantized linear layer in ONE persistent launch.  They are
+ * independent (each reads only codes produced before the call), so their output tiles share
+ * the SMs: the work units of all three form one list, the GEMM with the longest K loop per
+ * unit first.  Semantics, layouts and limits of every part are those of
+ * shiftquant_gemm_fwd / _dgrad / _wgrad with these operands (X [M, K], W [K, N],
+ * dY [M, N]; all codes with the same bits and n_groups):
+ *   forward            y [M, N]  from x_codes [M, K] and wf_codes [N, K] (per-out-channel W
+ *                      codes, transposed, X's shifts folded in), scales x_scale, wf_scale[N]
+ *   loss propagation   dx [M, K] from g_codes [M, N] and wd_codes [K, N] (per-in-channel W
+ *                      codes, dY's shifts folded in), scales g_scale, wd_scale[K]
+ *   weight gradient    dw [K, N] from xt_codes [K, M] and gt_codes [N, M] with the exponents
+ *                      x_exp[K], g_exp[N] and the scales x_scale, g_scale
+ * acc_* are the optional int64 exactness-check outputs.  The struct lives in host memory and
+ * is read during the call only. */
+typedef struct {
+  const void *x_codes;  int64_t ld_x;
+  const void *xt_codes; int64_t ld_xt;
+  const float *x_scale; const uint8_t *x_exp;
+  const void *g_codes;  int64_t ld_g;
+  const void *gt_codes; int64_t ld_gt;
+  const float *g_scale; const uint8_t *g_exp;
+  const void *wf_codes; int64_t ld_wf; const float *wf_scale;
+  const void *wd_codes; int64_t ld_wd; const float *wd_scale;
+  int64_t M, K, N;
+  int bits, n_groups;
+  float *y;  int64_t ld_y;
+  float *dx; int64_t ld_dx;
+  float *dw; int64_t ld_dw;
+  int64_t *acc_y;  int64_t ld_acc_y;
+  int64_t *acc_dx; int64_t ld_acc_dx;
+  int64_t *acc_dw; int64_t ld_acc_dw;
+} sq_layer_gemms;
+
+/* workspace: optional int32 scratch of shiftquant_gemm_layer_workspace_bytes() bytes; each
+ * GEMM with too few output tiles for the SMs splits its K loop into its own region of it. */
+sq_status shiftquant_gemm_layer(const sq_layer_gemms *args, void *workspace,
+                                size_t workspace_bytes, int32_t *dev_status, void *stream);
+
+/* Bytes of workspace that let shiftquant_gemm_layer split every GEMM that would benefit
+ * (0 when none would) on the current device. */
+size_t shiftquant_gemm_layer_workspace_bytes(int64_t M, int64_t K, int64_t N, int bits,
+                                             int n_groups);
+
 /* Weight-gradient GEMM for callers that cannot allocate device memory -- for instance a
  * plug-in running inside a host framework that owns every device allocation, or a
  * deployment whose device memory is fixed when the library is loaded.  The paper has no

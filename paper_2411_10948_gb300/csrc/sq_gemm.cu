@@ -36,7 +36,6 @@ namespace sq {
 constexpr int kBM = 128;
 constexpr int kBN = 256;
 constexpr int kBKBytes = 128;                 // one 128-byte swizzle row of K per stage
-constexpr int kStages = 3;
 constexpr int kABytes = kBM * kBKBytes;       // 16 KB
 constexpr int kBBytes = kBN * kBKBytes;       // 32 KB
 constexpr int kStageBytes = kABytes + kBBytes;
@@ -45,24 +44,33 @@ constexpr int kEpiWarp0 = 4;
 constexpr int kNumEpiWarps = 8;
 constexpr uint32_t kTmemCols = 2 * kBN;       // two FP32 accumulator buffers
 constexpr int64_t kExactSum = int64_t(1) << 24;  // every partial sum of a chunk stays within this
-// shared memory: the operand ring, two 32 x 32 output boxes per epilogue warp (staging for
-// TMA stores, double-buffered), two per-tile column-factor tables, then the barriers
+// Shared memory of a CTA, in two layouts.  Plain-store mode: a 4-stage operand ring and one
+// 32 x 32 output staging box per epilogue warp (the box turns the lane-per-row TMEM layout
+// into row-contiguous stores).  TMA-store mode, for launches whose outputs outweigh their
+// operands: a 3-stage ring and two staging boxes per warp, so one box is written while TMA
+// stores the other.  Then two per-tile column-factor tables and the barriers.
 constexpr int kOutBox = 32;
 constexpr int kOutStageBytes = kOutBox * kOutBox * 4;
-constexpr int kOutOffset = kStages * kStageBytes;
-constexpr int kFacOffset = kOutOffset + kNumEpiWarps * 2 * kOutStageBytes;
-constexpr int kBarOffset = kFacOffset + 2 * kBN * 4;
-constexpr int kNumBars = 2 * kStages + 2 + 2 + 2 + 1;   // full, empty, tfull, tempty, fac, drain
-constexpr size_t kSmemBytes = kBarOffset + kNumBars * 8 + 16;
-static_assert(kSmemBytes <= 232448, "shared memory beyond the 227 KB per-CTA limit");
-static_assert(kOutOffset % 1024 == 0 && kOutStageBytes % 1024 == 0, "swizzle atoms need 1 KB");
+
+template <bool kTmaSt>
+struct Smem {
+  static constexpr int stages = kTmaSt ? 3 : 4;
+  static constexpr int out_bufs = kTmaSt ? 2 : 1;
+  static constexpr int out_offset = stages * kStageBytes;
+  static constexpr int fac_offset = out_offset + kNumEpiWarps * out_bufs * kOutStageBytes;
+  static constexpr int bar_offset = fac_offset + 2 * kBN * 4;
+  static constexpr int num_bars = 2 * stages + 2 + 2 + 2 + 1;  // full, empty, tfull, tempty, fac, drain
+  static constexpr size_t bytes = bar_offset + num_bars * 8 + 16;
+  static_assert(bytes <= 232448, "shared memory beyond the 227 KB per-CTA limit");
+  static_assert(out_offset % 1024 == 0 && kOutStageBytes % 1024 == 0, "swizzle atoms need 1 KB");
+};
 
 struct GemmParams {
   int M, N, K;
   int m_tiles, n_tiles, splits, kb_total, kb_per_split, chunk_kb;
   int mode;  // 0: per-column scale (forward, loss propagation); 1: row/column shifts (wgrad)
   int G;
-  int use_tma_y;  // outputs leave through TMA stores (else plain stores)
+  int vec_y;  // output rows 16-byte aligned: 16-byte stores
   const float* a_scale;
   const float* b_scale;
   const uint8_t* row_exp;
@@ -72,6 +80,22 @@ struct GemmParams {
   long long* acc;
   int64_t ld_acc;
   int* ws;  // split-K int32 partial sums [M, N], or null
+  int* status;
+};
+
+// Up to three GEMMs run by one persistent launch (the three GEMMs of a layer are
+// independent).  Work units of all of them form one list, GEMM by GEMM in the order given
+// (the host puts the GEMM with the longest K loop per unit first); CTA i takes units
+// i, i + gridDim.x, ...
+constexpr int kMaxBatch = 3;
+struct GemmBatch {
+  CUtensorMap a[kMaxBatch];
+  CUtensorMap b[kMaxBatch];
+  CUtensorMap y[kMaxBatch];   // fp32 output maps (TMA-store mode, aligned outputs)
+  CUtensorMap ws[kMaxBatch];  // split-K workspace maps (unused when a GEMM does not split)
+  GemmParams p[kMaxBatch];
+  int unit_end[kMaxBatch];  // cumulative unit counts
+  int count;
   int* status;
 };
 
@@ -108,16 +132,6 @@ __device__ __forceinline__ uint32_t staged(uint32_t buf, int rr, int cc) {
   return v;
 }
 
-// plain stores of a staged fp32 box (lane = column, one row per step: coalesced)
-__device__ __noinline__ void write_y_box(float* y, int64_t ldy, int64_t M, int64_t N, uint32_t buf,
-                                         int64_t row0, int64_t col0, int lane) {
-  const int64_t col = col0 + lane;
-  for (int rr = 0; rr < 32; ++rr) {
-    const int64_t row = row0 + rr;
-    if (row < M && col < N) y[row * ldy + col] = __uint_as_float(staged(buf, rr, lane));
-  }
-}
-
 // the canonical integers T of a staged int32 box as int64 (exactness-check output);
 // row_exp / col_exp are null for the forward and loss-propagation GEMMs
 __device__ __noinline__ void write_acc_box(long long* acc, int64_t ld_acc, int64_t M, int64_t N,
@@ -135,14 +149,22 @@ __device__ __noinline__ void write_acc_box(long long* acc, int64_t ld_acc, int64
 }
 
 // One 32 x 32 output box of an epilogue warp: lane = row, vals = the lane's 32 columns as
-// exact integers (FP32 patterns when `as_float`, else int32).  Stages the box in shared
-// memory and hands it to TMA (store of the dequantized fp32 values, or int32 reduce-add
-// into the split-K workspace); writes the exactness-check integers when asked.
+// exact integers (FP32 patterns when `as_float`, else int32).  The box is staged in shared
+// memory (128-byte swizzle) and leaves either as dequantized fp32 values through
+// row-contiguous 16-byte stores (eight lanes per 128-byte row, four rows per instruction),
+// or as int32 partial sums through a TMA reduce-add into the split-K workspace.  The
+// exactness-check integers are written when asked.
+template <bool kTmaSt>
 __device__ __forceinline__ void emit_box(const GemmParams& p, const CUtensorMap* tma_y,
                                          const CUtensorMap* tma_ws, const uint32_t (&vals)[32],
                                          bool as_float, const float* f, float rfac, uint32_t buf,
-                                         int64_t row0, int64_t col0, int lane, bool via_tma) {
-  if (lane == 0) bulk_wait_read<1>();
+                                         int64_t row0, int64_t col0, int lane) {
+  const bool tma_out = p.ws != nullptr || (kTmaSt && p.vec_y);
+  if (tma_out && lane == 0) {
+    // in TMA-store mode the box two stores back used this buffer; otherwise the last one
+    if (kTmaSt) bulk_wait_read<1>();
+    else bulk_wait_read<0>();
+  }
   __syncwarp();
   if (p.acc != nullptr && p.ws == nullptr) {
 #pragma unroll
@@ -175,7 +197,7 @@ __device__ __forceinline__ void emit_box(const GemmParams& p, const CUtensorMap*
     }
     st_shared_v4(buf + lane * 128 + ((k ^ (lane & 7)) << 4), o[0], o[1], o[2], o[3]);
   }
-  if (via_tma) {
+  if (tma_out) {
     fence_proxy_async_smem();
     __syncwarp();
     if (lane == 0) {
@@ -185,11 +207,33 @@ __device__ __forceinline__ void emit_box(const GemmParams& p, const CUtensorMap*
         tma_store_2d(tma_y, buf, static_cast<int32_t>(col0), static_cast<int32_t>(row0));
       bulk_commit();
     }
-  } else {
-    __syncwarp();
-    write_y_box(p.y, p.ldy, p.M, p.N, buf, row0, col0, lane);  // outputs TMA cannot address
-    __syncwarp();
+    return;
   }
+  __syncwarp();
+  const int lr = lane >> 3;         // row within a group of four
+  const int lc = lane & 7;          // 16-byte chunk within the 128-byte row
+  const int64_t col = col0 + lc * 4;
+#pragma unroll
+  for (int i = 0; i < 8; ++i) {
+    const int rr = i * 4 + lr;
+    const int64_t row = row0 + rr;
+    uint32_t v0, v1, v2, v3;
+    asm volatile("ld.shared.v4.b32 {%0, %1, %2, %3}, [%4];"
+                 : "=r"(v0), "=r"(v1), "=r"(v2), "=r"(v3)
+                 : "r"(buf + rr * 128 + ((lc ^ (rr & 7)) << 4)));
+    if (row < p.M) {
+      float* dst = p.y + row * p.ldy + col;
+      if (p.vec_y && col + 3 < p.N) {
+        *reinterpret_cast<uint4*>(dst) = make_uint4(v0, v1, v2, v3);
+      } else {
+        if (col + 0 < p.N) dst[0] = __uint_as_float(v0);
+        if (col + 1 < p.N) dst[1] = __uint_as_float(v1);
+        if (col + 2 < p.N) dst[2] = __uint_as_float(v2);
+        if (col + 3 < p.N) dst[3] = __uint_as_float(v3);
+      }
+    }
+  }
+  __syncwarp();  // the staging box is free for the next one
 }
 
 struct Unit {
@@ -221,18 +265,26 @@ __device__ __forceinline__ Unit decode_unit(const GemmParams& p, int u) {
 
 // kMulti: the K loop of a tile spans several exact chunks, whose int32 sums the epilogue
 // keeps in registers; otherwise every output streams from TMEM once.
-template <int kF8, bool kMulti>
+// the GEMM of global unit u, and u's index inside that GEMM
+__device__ __forceinline__ int batch_member(const GemmBatch& bt, int u, int* local) {
+  int g = 0;
+  while (g + 1 < bt.count && u >= bt.unit_end[g]) ++g;
+  *local = u - (g ? bt.unit_end[g - 1] : 0);
+  return g;
+}
+
+// kTmaSt: shared-memory layout and output path (Smem<kTmaSt>)
+template <int kF8, bool kMulti, bool kTmaSt>
 __global__ void __launch_bounds__(kThreads, 1)
-    shiftmm_kernel(const __grid_constant__ CUtensorMap tma_a,
-                   const __grid_constant__ CUtensorMap tma_b,
-                   const __grid_constant__ CUtensorMap tma_y,
-                   const __grid_constant__ CUtensorMap tma_ws, const GemmParams p) {
+    shiftmm_kernel(const __grid_constant__ GemmBatch bt) {
+  using L = Smem<kTmaSt>;
+  constexpr int kStages = L::stages;
   extern __shared__ __align__(1024) uint8_t smem[];
   if ((smem_u32(smem) & 1023u) != 0) {  // the swizzled layouts need 1 KB alignment
-    if (threadIdx.x == 0) atomicOr(p.status, kDevInternal);
+    if (threadIdx.x == 0) atomicOr(bt.status, kDevInternal);
     return;
   }
-  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + kBarOffset);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + L::bar_offset);
   uint64_t* full = bars;
   uint64_t* empty = bars + kStages;
   uint64_t* tfull = bars + 2 * kStages;
@@ -260,8 +312,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     fence_mbar_init();
   }
   if (warp == 0 && lane == 0) {
-    tma_prefetch_desc(&tma_a);
-    tma_prefetch_desc(&tma_b);
+    for (int g = 0; g < bt.count; ++g) {
+      tma_prefetch_desc(&bt.a[g]);
+      tma_prefetch_desc(&bt.b[g]);
+    }
   }
   if (warp == 1) {
     tmem_alloc(smem_u32(tmem_slot), kTmemCols);
@@ -271,7 +325,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
-  const int units = p.m_tiles * p.n_tiles * p.splits;
+  const int units = bt.unit_end[bt.count - 1];
   constexpr int kBKElems = kF8 ? kBKBytes : kBKBytes / 2;
 
   if (warp == 0 && lane == 0) {
@@ -281,7 +335,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     long long issued = 0;
     bool ok = true;
     for (int u = blockIdx.x; u < units && ok; u += gridDim.x) {
-      const Unit w = decode_unit(p, u);
+      int lu;
+      const int g = batch_member(bt, u, &lu);
+      const Unit w = decode_unit(bt.p[g], lu);
       for (int kb = w.kb0; kb < w.kb1; ++kb) {
         if (!mbar_wait(&empty[s], ph ^ 1u, abort_flag)) {
           ok = false;
@@ -289,8 +345,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         const uint32_t sa = smem_u32(smem + s * kStageBytes);
         mbar_arrive_expect_tx(&full[s], kStageBytes);
-        tma_load_2d(sa, &tma_a, smem_u32(&full[s]), kb * kBKElems, w.mb * kBM);
-        tma_load_2d(sa + kABytes, &tma_b, smem_u32(&full[s]), kb * kBKElems, w.nb * kBN);
+        tma_load_2d(sa, &bt.a[g], smem_u32(&full[s]), kb * kBKElems, w.mb * kBM);
+        tma_load_2d(sa + kABytes, &bt.b[g], smem_u32(&full[s]), kb * kBKElems, w.nb * kBN);
         ++issued;
         if (++s == kStages) {
           s = 0;
@@ -299,7 +355,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
     }
     if (!ok) {
-      atomicOr(p.status, kDevTimeout);
+      atomicOr(bt.status, kDevTimeout);
       *abort_flag = 1;
     }
     // every issued copy must have landed before the CTA may exit
@@ -313,9 +369,12 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint32_t c = 0;
     bool ok = true;
     for (int u = blockIdx.x; u < units && ok; u += gridDim.x) {
-      const Unit w = decode_unit(p, u);
-      for (int kc = w.kb0; kc < w.kb1 && ok; kc += p.chunk_kb) {
-        const int kce = min(w.kb1, kc + p.chunk_kb);
+      int lu;
+      const int g = batch_member(bt, u, &lu);
+      const int chunk_kb = bt.p[g].chunk_kb;
+      const Unit w = decode_unit(bt.p[g], lu);
+      for (int kc = w.kb0; kc < w.kb1 && ok; kc += chunk_kb) {
+        const int kce = min(w.kb1, kc + chunk_kb);
         const uint32_t b = c & 1u, tph = (c >> 1) & 1u;
         if (!mbar_wait(&tempty[b], tph ^ 1u, abort_flag)) {
           ok = false;
@@ -353,7 +412,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
     }
     if (!ok) {
-      atomicOr(p.status, kDevTimeout);
+      atomicOr(bt.status, kDevTimeout);
       *abort_flag = 1;
     }
     tc_commit(smem_u32(drain));
@@ -364,16 +423,20 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int h = (warp - kEpiWarp0) >> 2;        // column half of the 256-wide tile
     const int et = threadIdx.x - kEpiWarp0 * 32;  // 0 .. 255: one tile column each
     const uint32_t stage_out0 =
-        smem_u32(smem + kOutOffset + (warp - kEpiWarp0) * 2 * kOutStageBytes);
-    uint32_t nbox = 0;  // boxes this warp has handed to TMA: selects the staging buffer
-    float* fac_tab = reinterpret_cast<float*>(smem + kFacOffset);
-    const float a_fac = epilogue_a_factor(p);
-    const bool via_tma = p.ws != nullptr || p.use_tma_y;
+        smem_u32(smem + L::out_offset + (warp - kEpiWarp0) * L::out_bufs * kOutStageBytes);
+    uint32_t nbox = 0;  // boxes emitted: alternates the staging buffers in TMA-store mode
+    float* fac_tab = reinterpret_cast<float*>(smem + L::fac_offset);
     uint32_t c = 0;
     bool ok = true;
     int it = 0;
     for (int u = blockIdx.x; u < units && ok; u += gridDim.x, ++it) {
-      const Unit w = decode_unit(p, u);
+      int lu;
+      const int g = batch_member(bt, u, &lu);
+      const GemmParams& p = bt.p[g];
+      const CUtensorMap* tma_y = &bt.y[g];
+      const CUtensorMap* tma_ws = &bt.ws[g];
+      const float a_fac = epilogue_a_factor(p);
+      const Unit w = decode_unit(p, lu);
       const int nch = (w.kb1 - w.kb0 + p.chunk_kb - 1) / p.chunk_kb;
       const int64_t m0 = static_cast<int64_t>(w.mb) * kBM;
       const int64_t n0 = static_cast<int64_t>(w.nb) * kBN;
@@ -418,10 +481,9 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
           const int64_t col0 = n0 + h * 128 + s * 32;
           if (row0 >= p.M || col0 >= p.N) continue;  // warp-uniform: nothing of this box exists
-          const uint32_t buf = stage_out0 + (nbox & 1u) * kOutStageBytes;
-          ++nbox;
-          emit_box(p, &tma_y, &tma_ws, v, true, fac + h * 128 + s * 32, rfac, buf, row0, col0,
-                   lane, via_tma);
+          const uint32_t buf = stage_out0 + (nbox++ % L::out_bufs) * kOutStageBytes;
+          emit_box<kTmaSt>(p, tma_y, tma_ws, v, true, fac + h * 128 + s * 32, rfac, buf, row0,
+                           col0, lane);
         }
         ++c;
       } else {
@@ -464,15 +526,14 @@ __global__ void __launch_bounds__(kThreads, 1)
           uint32_t v[32];
 #pragma unroll
           for (int i = 0; i < 32; ++i) v[i] = acc[s * 32 + i];
-          const uint32_t buf = stage_out0 + (nbox & 1u) * kOutStageBytes;
-          ++nbox;
-          emit_box(p, &tma_y, &tma_ws, v, false, fac + h * 128 + s * 32, rfac, buf, row0, col0,
-                   lane, via_tma);
+          const uint32_t buf = stage_out0 + (nbox++ % L::out_bufs) * kOutStageBytes;
+          emit_box<kTmaSt>(p, tma_y, tma_ws, v, false, fac + h * 128 + s * 32, rfac, buf, row0,
+                           col0, lane);
         }
       }
     }
     if (!ok) {
-      atomicOr(p.status, kDevTimeout);
+      atomicOr(bt.status, kDevTimeout);
       *abort_flag = 1;
     }
     if (lane == 0) bulk_wait_read<0>();  // no store still reads shared memory at exit
@@ -613,15 +674,222 @@ static int make_plan(int which, int64_t M, int64_t N, int64_t K, int bits, int G
   return SQ_OK;
 }
 
-template <int kF8, bool kMulti>
+template <int kF8, bool kMulti, bool kTmaSt>
 static int configure_kernel(int dev) {
   static bool done[64] = {};
   if (dev >= 0 && dev < 64 && done[dev]) return SQ_OK;
-  const cudaError_t err = cudaFuncSetAttribute(shiftmm_kernel<kF8, kMulti>,
+  const cudaError_t err = cudaFuncSetAttribute(shiftmm_kernel<kF8, kMulti, kTmaSt>,
                                                cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                               static_cast<int>(kSmemBytes));
+                                               static_cast<int>(Smem<kTmaSt>::bytes));
   if (err != cudaSuccess) return cuda_fail(err, "cudaFuncSetAttribute");
   if (dev >= 0 && dev < 64) done[dev] = true;
+  return SQ_OK;
+}
+
+// One GEMM of a launch: out[M, N] = A[M, K] B[N, K]^T with the operand roles of `which`
+// (0 forward, 1 loss propagation, 2 weight gradient).
+struct GemmJob {
+  int which;
+  const void* a;
+  int64_t lda;
+  const void* b;
+  int64_t ldb;
+  int64_t M, N, K;
+  const float* a_scale;
+  const float* b_scale;
+  const uint8_t* row_exp;
+  const uint8_t* col_exp;
+  float* y;
+  int64_t ldy;
+  int64_t* acc;
+  int64_t ld_acc;
+  void* ws;
+  size_t ws_bytes;
+};
+
+static const char* job_name(int which) {
+  static const char* names[3] = {"gemm_fwd", "gemm_dgrad", "gemm_wgrad"};
+  return names[which];
+}
+
+// Argument checks of one GEMM; *launch is false when there is nothing for the kernel to do
+// (an empty output, or K == 0 whose zero result is written here with memsets).
+static int check_job(const GemmJob& j, int bits, int G, int32_t* dev_status, cudaStream_t s,
+                     bool* launch) {
+  const char* nm = job_name(j.which);
+  *launch = false;
+  if (!bits_ok(bits) || !groups_ok(G))
+    return fail(SQ_EINVAL, "%s: bits must be in [2, 8] and n_groups in [1, 8]", nm);
+  if (j.M < 0 || j.N < 0 || j.K < 0) return fail(SQ_EINVAL, "%s: negative size", nm);
+  if (j.M > INT32_MAX || j.N > INT32_MAX || j.K > INT32_MAX)
+    return fail(SQ_EUNSUPPORTED, "%s: dimensions beyond 2^31", nm);
+  if (dev_status == nullptr) return fail(SQ_EINVAL, "%s: dev_status is required", nm);
+  if (j.M == 0 || j.N == 0) return SQ_OK;
+  if (j.y == nullptr || j.ldy < j.N) return fail(SQ_EINVAL, "%s: output is NULL or its ld < N", nm);
+  if (j.acc != nullptr && j.ld_acc < j.N) return fail(SQ_EINVAL, "%s: ld_acc < N", nm);
+  if (j.a_scale == nullptr || j.b_scale == nullptr)
+    return fail(SQ_EINVAL, "%s: scales are required", nm);
+  if (j.which == 2 && (j.row_exp == nullptr || j.col_exp == nullptr))
+    return fail(SQ_EINVAL, "%s: exponents are required", nm);
+  if (j.K == 0) {
+    // an empty inner sum: T = 0 everywhere
+    cudaError_t err = cudaMemset2DAsync(j.y, j.ldy * sizeof(float), 0, j.N * sizeof(float), j.M, s);
+    if (err == cudaSuccess && j.acc)
+      err = cudaMemset2DAsync(j.acc, j.ld_acc * sizeof(int64_t), 0, j.N * sizeof(int64_t), j.M, s);
+    return err == cudaSuccess ? SQ_OK : cuda_fail(err, "cudaMemset2DAsync");
+  }
+  if (j.a == nullptr || j.b == nullptr) return fail(SQ_EINVAL, "%s: codes are NULL", nm);
+  if (j.lda < j.K || j.ldb < j.K) return fail(SQ_EINVAL, "%s: operand ld smaller than K", nm);
+  const int eb = code_bytes(code_type(bits, G));
+  if (!aligned16(j.a) || !aligned16(j.b) || (j.lda * eb) % 16 != 0 || (j.ldb * eb) % 16 != 0)
+    return fail(SQ_EALIGN, "%s: operand pointers must be 16-byte aligned and ld * %d bytes a "
+                "multiple of 16", nm, eb);
+  const int st = check_exact_range(j.which, j.K, bits, G);
+  if (st != SQ_OK) return st;
+  *launch = true;
+  return SQ_OK;
+}
+
+// Plan of one checked GEMM and its slot in the batch: tiles, K splits (only with a
+// workspace large enough for the [M, N] int32 partial sums), tensor maps, parameters.
+static int prepare_job(const GemmJob& j, int bits, int G, int sms, int32_t* dev_status,
+                       GemmBatch* bt, int g, Plan* pl) {
+  int st = make_plan(j.which, j.M, j.N, j.K, bits, G, sms, true, pl);
+  if (st != SQ_OK) return st;
+  if (pl->splits > 1) {
+    // split-K partials are added by TMA into a [M, N] int32 workspace with N-element rows,
+    // whose rows must stay 16-byte aligned
+    const size_t need = static_cast<size_t>(j.M) * j.N * sizeof(int);
+    if (j.ws == nullptr || j.ws_bytes < need || !aligned16(j.ws) || j.N % 4 != 0) {
+      st = make_plan(j.which, j.M, j.N, j.K, bits, G, sms, false, pl);
+      if (st != SQ_OK) return st;
+    }
+  }
+  const int eb = pl->elem_bytes;
+  if ((st = make_operand_map(&bt->a[g], j.a, j.M, j.K, j.lda, eb, kBM)) != SQ_OK) return st;
+  if ((st = make_operand_map(&bt->b[g], j.b, j.N, j.K, j.ldb, eb, kBN)) != SQ_OK) return st;
+  GemmParams& p = bt->p[g];
+  p.M = static_cast<int>(j.M);
+  p.N = static_cast<int>(j.N);
+  p.K = static_cast<int>(j.K);
+  p.m_tiles = pl->m_tiles;
+  p.n_tiles = pl->n_tiles;
+  p.splits = pl->splits;
+  p.kb_total = pl->kb_total;
+  p.kb_per_split = pl->kb_per_split;
+  p.chunk_kb = pl->chunk_kb;
+  p.mode = j.which == 2 ? 1 : 0;
+  p.G = G;
+  p.vec_y = (j.ldy % 4 == 0) && aligned16(j.y);
+  p.a_scale = j.a_scale;
+  p.b_scale = j.b_scale;
+  p.row_exp = j.row_exp;
+  p.col_exp = j.col_exp;
+  p.y = j.y;
+  p.ldy = j.ldy;
+  p.acc = reinterpret_cast<long long*>(j.acc);
+  p.ld_acc = j.ld_acc;
+  p.ws = pl->splits > 1 ? static_cast<int*>(j.ws) : nullptr;
+  p.status = dev_status;
+  memset(&bt->y[g], 0, sizeof(CUtensorMap));
+  memset(&bt->ws[g], 0, sizeof(CUtensorMap));
+  if (p.ws)
+    st = make_output_map(&bt->ws[g], p.ws, j.M, j.N, j.N, CU_TENSOR_MAP_DATA_TYPE_INT32);
+  else if (p.vec_y)
+    st = make_output_map(&bt->y[g], j.y, j.M, j.N, j.ldy, CU_TENSOR_MAP_DATA_TYPE_FLOAT32);
+  return st;
+}
+
+template <int kF8, bool kMulti, bool kTmaSt>
+static int launch_kernel(const GemmBatch& bt, int grid, int dev, cudaStream_t s) {
+  const int st = configure_kernel<kF8, kMulti, kTmaSt>(dev);
+  if (st != SQ_OK) return st;
+  shiftmm_kernel<kF8, kMulti, kTmaSt><<<grid, kThreads, Smem<kTmaSt>::bytes, s>>>(bt);
+  const cudaError_t err = cudaGetLastError();
+  return err == cudaSuccess ? SQ_OK : cuda_fail(err, "shiftmm_kernel launch");
+}
+
+template <int kF8>
+static int launch_variant(const GemmBatch& bt, int grid, int dev, cudaStream_t s, bool multi,
+                          bool tma_st) {
+  if (multi)
+    return tma_st ? launch_kernel<kF8, true, true>(bt, grid, dev, s)
+                  : launch_kernel<kF8, true, false>(bt, grid, dev, s);
+  return tma_st ? launch_kernel<kF8, false, true>(bt, grid, dev, s)
+                : launch_kernel<kF8, false, false>(bt, grid, dev, s);
+}
+
+// Checks, plans and launches up to kMaxBatch GEMMs (all with the same bits / n_groups) as
+// one persistent kernel; split-K partial sums are zeroed before and finalized after it.
+static int run_jobs(GemmJob* jobs, int njobs, int bits, int G, int32_t* dev_status, void* stream) {
+  cudaStream_t s = as_stream(stream);
+  int live[kMaxBatch];
+  int nlive = 0;
+  for (int i = 0; i < njobs; ++i) {
+    bool launch = false;
+    const int st = check_job(jobs[i], bits, G, dev_status, s, &launch);
+    if (st != SQ_OK) return st;
+    if (launch) live[nlive++] = i;
+  }
+  if (nlive == 0) return SQ_OK;
+  int dev = 0;
+  const int sms = device_sms(&dev);
+  if (sms <= 0) return fail(SQ_ECUDA, "%s: no current CUDA device", job_name(jobs[live[0]].which));
+  GemmBatch bt;
+  memset(&bt, 0, sizeof(bt));
+  Plan plans[kMaxBatch];
+  for (int g = 0; g < nlive; ++g) {
+    const int st = prepare_job(jobs[live[g]], bits, G, sms, dev_status, &bt, g, &plans[g]);
+    if (st != SQ_OK) return st;
+  }
+  // longest K loop per unit first: the short units then fill in behind the long ones
+  for (int a = 0; a < nlive; ++a)
+    for (int b = a + 1; b < nlive; ++b)
+      if (plans[b].kb_per_split > plans[a].kb_per_split) {
+        const GemmParams tp = bt.p[a]; bt.p[a] = bt.p[b]; bt.p[b] = tp;
+        const Plan tl = plans[a]; plans[a] = plans[b]; plans[b] = tl;
+        CUtensorMap t;
+        t = bt.a[a]; bt.a[a] = bt.a[b]; bt.a[b] = t;
+        t = bt.b[a]; bt.b[a] = bt.b[b]; bt.b[b] = t;
+        t = bt.y[a]; bt.y[a] = bt.y[b]; bt.y[b] = t;
+        t = bt.ws[a]; bt.ws[a] = bt.ws[b]; bt.ws[b] = t;
+      }
+  int units = 0;
+  bool multi = false;
+  for (int g = 0; g < nlive; ++g) {
+    units += plans[g].m_tiles * plans[g].n_tiles * plans[g].splits;
+    bt.unit_end[g] = units;
+    multi |= plans[g].kb_per_split > plans[g].chunk_kb;  // a unit spans several exact chunks
+  }
+  bt.count = nlive;
+  bt.status = dev_status;
+  cudaError_t err;
+  for (int g = 0; g < nlive; ++g)
+    if (bt.p[g].ws) {
+      err = cudaMemsetAsync(bt.p[g].ws, 0, static_cast<size_t>(bt.p[g].M) * bt.p[g].N * sizeof(int), s);
+      if (err != cudaSuccess) return cuda_fail(err, "cudaMemsetAsync");
+    }
+  // TMA-store mode when the outputs written are a large share of the operand tiles read
+  double out_bytes = 0.0, in_bytes = 0.0;
+  for (int g = 0; g < nlive; ++g) {
+    if (!bt.p[g].ws) out_bytes += 4.0 * bt.p[g].M * bt.p[g].N;
+    in_bytes += static_cast<double>(kStageBytes) * plans[g].m_tiles * plans[g].n_tiles *
+                plans[g].splits * plans[g].kb_per_split;
+  }
+  const bool tma_st = out_bytes > 0.2 * in_bytes;
+  const int grid = units < sms ? units : sms;
+  const int st = plans[0].elem_bytes == 1 ? launch_variant<1>(bt, grid, dev, s, multi, tma_st)
+                                          : launch_variant<0>(bt, grid, dev, s, multi, tma_st);
+  if (st != SQ_OK) return st;
+  for (int g = 0; g < nlive; ++g) {
+    if (!bt.p[g].ws) continue;
+    const int64_t total = static_cast<int64_t>(bt.p[g].M) * bt.p[g].N;
+    int64_t blocks = (total + 255) / 256;
+    if (blocks > static_cast<int64_t>(sms) * 16) blocks = static_cast<int64_t>(sms) * 16;
+    splitk_finalize_kernel<<<static_cast<unsigned>(blocks), 256, 0, s>>>(bt.p[g]);
+    err = cudaGetLastError();
+    if (err != cudaSuccess) return cuda_fail(err, "splitk_finalize_kernel launch");
+  }
   return SQ_OK;
 }
 
@@ -630,129 +898,34 @@ static int run_gemm(int which, const void* a_codes, int64_t lda, const void* b_c
                     const float* b_scale, const uint8_t* row_exp, const uint8_t* col_exp,
                     float* y, int64_t ldy, int64_t* acc_out, int64_t ld_acc, void* workspace,
                     size_t workspace_bytes, int32_t* dev_status, void* stream) {
-  static const char* names[3] = {"gemm_fwd", "gemm_dgrad", "gemm_wgrad"};
-  const char* nm = names[which];
-  if (!bits_ok(bits) || !groups_ok(G))
-    return fail(SQ_EINVAL, "%s: bits must be in [2, 8] and n_groups in [1, 8]", nm);
-  if (M < 0 || N < 0 || K < 0) return fail(SQ_EINVAL, "%s: negative size", nm);
-  if (M > INT32_MAX || N > INT32_MAX || K > INT32_MAX)
-    return fail(SQ_EUNSUPPORTED, "%s: dimensions beyond 2^31", nm);
-  if (dev_status == nullptr) return fail(SQ_EINVAL, "%s: dev_status is required", nm);
-  if (M == 0 || N == 0) return SQ_OK;
-  if (y == nullptr || ldy < N) return fail(SQ_EINVAL, "%s: output is NULL or its ld < N", nm);
-  if (acc_out != nullptr && ld_acc < N) return fail(SQ_EINVAL, "%s: ld_acc < N", nm);
-  if (a_scale == nullptr || b_scale == nullptr) return fail(SQ_EINVAL, "%s: scales are required", nm);
-  if (which == 2 && (row_exp == nullptr || col_exp == nullptr))
-    return fail(SQ_EINVAL, "%s: exponents are required", nm);
-  cudaStream_t s = as_stream(stream);
-  if (K == 0) {
-    // an empty inner sum: T = 0 everywhere
-    cudaError_t err = cudaMemset2DAsync(y, ldy * sizeof(float), 0, N * sizeof(float), M, s);
-    if (err == cudaSuccess && acc_out)
-      err = cudaMemset2DAsync(acc_out, ld_acc * sizeof(int64_t), 0, N * sizeof(int64_t), M, s);
-    return err == cudaSuccess ? SQ_OK : cuda_fail(err, "cudaMemset2DAsync");
-  }
-  if (a_codes == nullptr || b_codes == nullptr) return fail(SQ_EINVAL, "%s: codes are NULL", nm);
-  if (lda < K || ldb < K) return fail(SQ_EINVAL, "%s: operand ld smaller than K", nm);
-  const int eb = code_bytes(code_type(bits, G));
-  if (!aligned16(a_codes) || !aligned16(b_codes) || (lda * eb) % 16 != 0 || (ldb * eb) % 16 != 0)
-    return fail(SQ_EALIGN, "%s: operand pointers must be 16-byte aligned and ld * %d bytes a "
-                "multiple of 16", nm, eb);
-  int st = check_exact_range(which, K, bits, G);
-  if (st != SQ_OK) return st;
-  int dev = 0;
-  const int sms = device_sms(&dev);
-  if (sms <= 0) return fail(SQ_ECUDA, "%s: no current CUDA device", nm);
-  Plan pl;
-  st = make_plan(which, M, N, K, bits, G, sms, true, &pl);
-  if (st != SQ_OK) return st;
-  if (pl.splits > 1) {
-    // split-K partials are added by TMA into a [M, N] int32 workspace with N-element rows,
-    // whose rows must stay 16-byte aligned
-    const size_t need = static_cast<size_t>(M) * N * sizeof(int);
-    if (workspace == nullptr || workspace_bytes < need || !aligned16(workspace) || N % 4 != 0) {
-      st = make_plan(which, M, N, K, bits, G, sms, false, &pl);
-      if (st != SQ_OK) return st;
-    }
-  }
-  CUtensorMap ma, mb;
-  st = make_operand_map(&ma, a_codes, M, K, lda, eb, kBM);
-  if (st != SQ_OK) return st;
-  st = make_operand_map(&mb, b_codes, N, K, ldb, eb, kBN);
-  if (st != SQ_OK) return st;
-
-  GemmParams p;
-  p.M = static_cast<int>(M);
-  p.N = static_cast<int>(N);
-  p.K = static_cast<int>(K);
-  p.m_tiles = pl.m_tiles;
-  p.n_tiles = pl.n_tiles;
-  p.splits = pl.splits;
-  p.kb_total = pl.kb_total;
-  p.kb_per_split = pl.kb_per_split;
-  p.chunk_kb = pl.chunk_kb;
-  p.mode = which == 2 ? 1 : 0;
-  p.G = G;
-  p.use_tma_y = (ldy % 4 == 0) && aligned16(y);
-  p.a_scale = a_scale;
-  p.b_scale = b_scale;
-  p.row_exp = row_exp;
-  p.col_exp = col_exp;
-  p.y = y;
-  p.ldy = ldy;
-  p.acc = reinterpret_cast<long long*>(acc_out);
-  p.ld_acc = ld_acc;
-  p.ws = pl.splits > 1 ? static_cast<int*>(workspace) : nullptr;
-  p.status = dev_status;
-
-  CUtensorMap my, mw;
-  memset(&my, 0, sizeof(my));
-  memset(&mw, 0, sizeof(mw));
-  if (p.ws) {
-    st = make_output_map(&mw, p.ws, M, N, N, CU_TENSOR_MAP_DATA_TYPE_INT32);
-    if (st != SQ_OK) return st;
-  } else if (p.use_tma_y) {
-    st = make_output_map(&my, y, M, N, ldy, CU_TENSOR_MAP_DATA_TYPE_FLOAT32);
-    if (st != SQ_OK) return st;
-  }
-  cudaError_t err;
-  if (p.ws) {
-    err = cudaMemsetAsync(p.ws, 0, static_cast<size_t>(M) * N * sizeof(int), s);
-    if (err != cudaSuccess) return cuda_fail(err, "cudaMemsetAsync");
-  }
-  const int units = pl.m_tiles * pl.n_tiles * pl.splits;
-  const int grid = units < sms ? units : sms;
-  const bool multi = pl.kb_per_split > pl.chunk_kb;  // some unit spans several exact chunks
-  if (eb == 1) {
-    if (multi) {
-      if ((st = configure_kernel<1, true>(dev)) != SQ_OK) return st;
-      shiftmm_kernel<1, true><<<grid, kThreads, kSmemBytes, s>>>(ma, mb, my, mw, p);
-    } else {
-      if ((st = configure_kernel<1, false>(dev)) != SQ_OK) return st;
-      shiftmm_kernel<1, false><<<grid, kThreads, kSmemBytes, s>>>(ma, mb, my, mw, p);
-    }
-  } else {
-    if (multi) {
-      if ((st = configure_kernel<0, true>(dev)) != SQ_OK) return st;
-      shiftmm_kernel<0, true><<<grid, kThreads, kSmemBytes, s>>>(ma, mb, my, mw, p);
-    } else {
-      if ((st = configure_kernel<0, false>(dev)) != SQ_OK) return st;
-      shiftmm_kernel<0, false><<<grid, kThreads, kSmemBytes, s>>>(ma, mb, my, mw, p);
-    }
-  }
-  err = cudaGetLastError();
-  if (err != cudaSuccess) return cuda_fail(err, "shiftmm_kernel launch");
-  if (p.ws) {
-    const int64_t total = static_cast<int64_t>(M) * N;
-    int64_t blocks = (total + 255) / 256;
-    if (blocks > static_cast<int64_t>(sms) * 16) blocks = static_cast<int64_t>(sms) * 16;
-    splitk_finalize_kernel<<<static_cast<unsigned>(blocks), 256, 0, s>>>(p);
-    err = cudaGetLastError();
-    if (err != cudaSuccess) return cuda_fail(err, "splitk_finalize_kernel launch");
-  }
-  return SQ_OK;
+  GemmJob j{which, a_codes, lda, b_codes, ldb, M, N, K, a_scale, b_scale, row_exp, col_exp,
+            y, ldy, acc_out, ld_acc, workspace, workspace_bytes};
+  return run_jobs(&j, 1, bits, G, dev_status, stream);
 }
 
+// The three GEMMs of a layer as jobs, workspace regions assigned to those that split.
+static void layer_jobs(const sq_layer_gemms* a, GemmJob jobs[3]) {
+  jobs[0] = GemmJob{0, a->x_codes, a->ld_x, a->wf_codes, a->ld_wf, a->M, a->N, a->K, a->x_scale,
+                    a->wf_scale, nullptr, nullptr, a->y, a->ld_y, a->acc_y, a->ld_acc_y, nullptr, 0};
+  jobs[1] = GemmJob{1, a->g_codes, a->ld_g, a->wd_codes, a->ld_wd, a->M, a->K, a->N, a->g_scale,
+                    a->wd_scale, nullptr, nullptr, a->dx, a->ld_dx, a->acc_dx, a->ld_acc_dx, nullptr, 0};
+  jobs[2] = GemmJob{2, a->xt_codes, a->ld_xt, a->gt_codes, a->ld_gt, a->K, a->N, a->M, a->x_scale,
+                    a->g_scale, a->x_exp, a->g_exp, a->dw, a->ld_dw, a->acc_dw, a->ld_acc_dw,
+                    nullptr, 0};
+}
+
+// Bytes each GEMM of the layer would use for split-K partial sums (0: it would not split),
+// each rounded up to 256 bytes.
+static void layer_ws_need(const GemmJob jobs[3], int bits, int G, int sms, size_t need[3]) {
+  for (int i = 0; i < 3; ++i) {
+    need[i] = 0;
+    const GemmJob& j = jobs[i];
+    if (j.M <= 0 || j.N <= 0 || j.K <= 0 || j.N % 4 != 0) continue;
+    Plan pl;
+    if (make_plan(j.which, j.M, j.N, j.K, bits, G, sms, true, &pl) != SQ_OK) continue;
+    if (pl.splits > 1) need[i] = (static_cast<size_t>(j.M) * j.N * sizeof(int) + 255) & ~size_t(255);
+  }
+}
 
 // ----------------------------------------------- allocation-free weight gradient
 // Scratch for callers that cannot allocate device memory themselves: a fixed array in
@@ -856,4 +1029,47 @@ extern "C" sq_status shiftquant_gemm_wgrad_static(
   return run_gemm(2, xt_codes, ldx, gt_codes, ldg, Ci, Co, T, bits, n_groups, x_scale, g_scale,
                   x_exp, g_exp, dw, ld_dw, acc_out, ld_acc, scratch,
                   scratch ? kStaticScratchBytes : 0, dev_status, stream);
+}
+
+extern "C" sq_status shiftquant_gemm_layer(const sq_layer_gemms* args, void* workspace,
+                                           size_t workspace_bytes, int32_t* dev_status,
+                                           void* stream) {
+  fail(SQ_OK, "");
+  if (args == nullptr) return fail(SQ_EINVAL, "gemm_layer: args is NULL");
+  if (!bits_ok(args->bits) || !groups_ok(args->n_groups))
+    return fail(SQ_EINVAL, "gemm_layer: bits must be in [2, 8] and n_groups in [1, 8]");
+  GemmJob jobs[3];
+  layer_jobs(args, jobs);
+  if (workspace != nullptr && workspace_bytes > 0) {
+    const int sms = device_sms(nullptr);
+    if (sms > 0) {
+      size_t need[3];
+      layer_ws_need(jobs, args->bits, args->n_groups, sms, need);
+      size_t off = 0;
+      for (int i = 0; i < 3; ++i) {
+        if (need[i] == 0 || off + need[i] > workspace_bytes) continue;
+        jobs[i].ws = static_cast<char*>(workspace) + off;
+        jobs[i].ws_bytes = need[i];
+        off += need[i];
+      }
+    }
+  }
+  return run_jobs(jobs, 3, args->bits, args->n_groups, dev_status, stream);
+}
+
+extern "C" size_t shiftquant_gemm_layer_workspace_bytes(int64_t M, int64_t K, int64_t N, int bits,
+                                                        int n_groups) {
+  if (!bits_ok(bits) || !groups_ok(n_groups)) return 0;
+  const int sms = device_sms(nullptr);
+  if (sms <= 0) return 0;
+  sq_layer_gemms a;
+  memset(&a, 0, sizeof(a));
+  a.M = M;
+  a.K = K;
+  a.N = N;
+  GemmJob jobs[3];
+  layer_jobs(&a, jobs);
+  size_t need[3];
+  layer_ws_need(jobs, bits, n_groups, sms, need);
+  return need[0] + need[1] + need[2];
 }

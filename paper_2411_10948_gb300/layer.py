@@ -116,6 +116,11 @@ class QuantLinear:
             self.ws_wgrad = ws(2, K, N_, M)
         self.ws = self.ws_fwd if self.ws_fwd is not None else (
             self.ws_dgrad if self.ws_dgrad is not None else self.ws_wgrad)
+        self.ws_layer = None
+        if use_workspace:
+            need = N.shiftquant_gemm_layer_workspace_bytes(M, K, N_, bits, n_groups)
+            if need:
+                self.ws_layer = torch.zeros(need // 4, dtype=torch.int32, device=dev)
 
     # --- the hot path, step by step --------------------------------------------------
     def quantize_activation(self, x, stream=None):
@@ -148,6 +153,16 @@ class QuantLinear:
                                 self.G, self.dw, self.acc["wgrad"] if self.acc else None,
                                 self.ws_wgrad, self.status, stream)
 
+    def gemms(self, stream=None):
+        """The three GEMMs in one persistent launch (shiftquant_gemm_layer)."""
+        acc = self.acc or {}
+        N.shiftquant_gemm_layer(self.x.codes, self.x.codes_t, self.x.scale, self.x.exp,
+                                self.g.codes, self.g.codes_t, self.g.scale, self.g.exp,
+                                self.wf.codes, self.wf.scale, self.wd.codes, self.wd.scale,
+                                self.M, self.K, self.N, self.bits, self.G, self.y, self.dx,
+                                self.dw, acc.get("fwd"), acc.get("dgrad"), acc.get("wgrad"),
+                                self.ws_layer, self.status, stream)
+
     def step(self, x, w, dy, seed, stream=None):
         """One training step of the layer: every quantizer pass and all three GEMMs."""
         self.quantize_activation(x, stream)
@@ -158,47 +173,39 @@ class QuantLinear:
         self.wgrad(stream)
 
     def step_concurrent(self, x, w, dy, seed, streams):
-        """The same step on five streams forked from (and joined back to) the current one:
-        the activation chain, the gradient chain, each weight role (its range pass right
-        away, its quantization once the other operand's exponents exist, then its GEMM once
-        the codes exist) and the weight-gradient GEMM once both code sets exist.
+        """The same step with its independent quantizer work on four streams forked from the
+        current one -- the activation chain, the gradient chain and each weight role (its
+        range pass right away, its quantization once the other operand's exponents exist) --
+        joined back before the three GEMMs run as one launch on the current stream.
         Capturable in a CUDA graph, which then runs the independent work concurrently."""
         main = torch.cuda.current_stream()
-        s_x, s_g, s_wf, s_wd, s_w = streams
-        for s in streams:
+        s_x, s_g, s_wf, s_wd = streams[:4]
+        for s in (s_x, s_g, s_wf, s_wd):
             s.wait_stream(main)
-        ev = {k: torch.cuda.Event() for k in ("x_cal", "x_q", "g_cal", "g_q")}
+        ev = {k: torch.cuda.Event() for k in ("x_cal", "g_cal")}
         b, G, st = self.bits, self.G, self.status
-        for s_, q, t, mode, sd, cal, qd in ((s_x, self.x, x, N.SQ_ROUND_NEAREST_EVEN, 0, "x_cal", "x_q"),
-                                           (s_g, self.g, dy, N.SQ_ROUND_STOCHASTIC, seed, "g_cal", "g_q")):
+        for s_, q, t, mode, sd, cal in ((s_x, self.x, x, N.SQ_ROUND_NEAREST_EVEN, 0, "x_cal"),
+                                        (s_g, self.g, dy, N.SQ_ROUND_STOCHASTIC, seed, "g_cal")):
             with torch.cuda.stream(s_):
                 N.shiftquant_calibrate(t, N.SQ_GRAN_SHIFT, G, q.range, q.tau0, q.exp, st, s_)
                 ev[cal].record(s_)
                 N.shiftquant_quantize(t, N.SQ_GRAN_SHIFT, b, G, q.tau0, q.exp, None, mode, sd,
                                       q.codes, q.codes_t, q.scale, s_)
-                ev[qd].record(s_)
         with torch.cuda.stream(s_wf):
             N.shiftquant_calibrate(w, N.SQ_GRAN_PER_COL, G, self.wf.range, None, None, st, s_wf)
             s_wf.wait_event(ev["x_cal"])
             N.shiftquant_quantize(w, N.SQ_GRAN_PER_COL, b, G, self.wf.range, None, self.x.exp,
                                   N.SQ_ROUND_NEAREST_EVEN, 0, None, self.wf.codes, self.wf.scale,
                                   s_wf)
-            s_wf.wait_event(ev["x_q"])
-            self.forward(s_wf)
         with torch.cuda.stream(s_wd):
             N.shiftquant_calibrate(w, N.SQ_GRAN_PER_ROW, G, self.wd.range, None, None, st, s_wd)
             s_wd.wait_event(ev["g_cal"])
             N.shiftquant_quantize(w, N.SQ_GRAN_PER_ROW, b, G, self.wd.range, None, self.g.exp,
                                   N.SQ_ROUND_NEAREST_EVEN, 0, self.wd.codes, None, self.wd.scale,
                                   s_wd)
-            s_wd.wait_event(ev["g_q"])
-            self.dgrad(s_wd)
-        with torch.cuda.stream(s_w):
-            s_w.wait_event(ev["x_q"])
-            s_w.wait_event(ev["g_q"])
-            self.wgrad(s_w)
-        for s in streams:
+        for s in (s_x, s_g, s_wf, s_wd):
             main.wait_stream(s)
+        self.gemms(main)
 
     @property
     def gemm_ops(self) -> int:

@@ -34,11 +34,33 @@ EXPORTS = (
     "shiftquant_code_type", "shiftquant_code_bytes", "shiftquant_calibrate",
     "shiftquant_quantize", "shiftquant_gemm_fwd", "shiftquant_gemm_dgrad",
     "shiftquant_gemm_wgrad", "shiftquant_gemm_wgrad_static", "shiftquant_gemm_workspace_bytes",
-    "shiftquant_status_string",
+    "shiftquant_gemm_layer", "shiftquant_gemm_layer_workspace_bytes", "shiftquant_status_string",
     "shiftquant_last_error",
 )
 
 _lib = None
+
+
+class SqLayerGemms(ctypes.Structure):
+    """Mirror of the C struct sq_layer_gemms (include/shiftquant.h)."""
+    _fields_ = [
+        ("x_codes", ctypes.c_void_p), ("ld_x", ctypes.c_int64),
+        ("xt_codes", ctypes.c_void_p), ("ld_xt", ctypes.c_int64),
+        ("x_scale", ctypes.c_void_p), ("x_exp", ctypes.c_void_p),
+        ("g_codes", ctypes.c_void_p), ("ld_g", ctypes.c_int64),
+        ("gt_codes", ctypes.c_void_p), ("ld_gt", ctypes.c_int64),
+        ("g_scale", ctypes.c_void_p), ("g_exp", ctypes.c_void_p),
+        ("wf_codes", ctypes.c_void_p), ("ld_wf", ctypes.c_int64), ("wf_scale", ctypes.c_void_p),
+        ("wd_codes", ctypes.c_void_p), ("ld_wd", ctypes.c_int64), ("wd_scale", ctypes.c_void_p),
+        ("M", ctypes.c_int64), ("K", ctypes.c_int64), ("N", ctypes.c_int64),
+        ("bits", ctypes.c_int), ("n_groups", ctypes.c_int),
+        ("y", ctypes.c_void_p), ("ld_y", ctypes.c_int64),
+        ("dx", ctypes.c_void_p), ("ld_dx", ctypes.c_int64),
+        ("dw", ctypes.c_void_p), ("ld_dw", ctypes.c_int64),
+        ("acc_y", ctypes.c_void_p), ("ld_acc_y", ctypes.c_int64),
+        ("acc_dx", ctypes.c_void_p), ("ld_acc_dx", ctypes.c_int64),
+        ("acc_dw", ctypes.c_void_p), ("ld_acc_dw", ctypes.c_int64),
+    ]
 
 
 class ShiftQuantError(RuntimeError):
@@ -83,6 +105,10 @@ def load(path: str | None = None) -> ctypes.CDLL:
     lib.shiftquant_gemm_wgrad_static.argtypes = [vp, i64, vp, vp, vp, i64, vp, vp, i64, i64, i64,
                                                  i32, i32, vp, i64, vp, i64, vp, vp]
     lib.shiftquant_gemm_wgrad_static.restype = i32
+    lib.shiftquant_gemm_layer.argtypes = [ctypes.POINTER(SqLayerGemms), vp, sz, vp, vp]
+    lib.shiftquant_gemm_layer.restype = i32
+    lib.shiftquant_gemm_layer_workspace_bytes.argtypes = [i64, i64, i64, i32, i32]
+    lib.shiftquant_gemm_layer_workspace_bytes.restype = sz
     lib.shiftquant_gemm_workspace_bytes.argtypes = [i32, i64, i64, i64, i32, i32]
     lib.shiftquant_gemm_workspace_bytes.restype = sz
     lib.shiftquant_status_string.argtypes = [i32]
@@ -197,3 +223,34 @@ def shiftquant_gemm_wgrad_static(xt_codes, x_scale, x_exp, gt_codes, g_scale, g_
 def shiftquant_gemm_workspace_bytes(which: int, M: int, N: int, K: int, bits: int,
                                     n_groups: int) -> int:
     return int(load().shiftquant_gemm_workspace_bytes(which, M, N, K, bits, n_groups))
+
+
+def _addr(t):
+    return t.data_ptr() if t is not None else None
+
+
+def shiftquant_gemm_layer(x_codes, xt_codes, x_scale, x_exp, g_codes, gt_codes, g_scale, g_exp,
+                          wf_codes, wf_scale, wd_codes, wd_scale, M, K, N, bits, n_groups, y, dx,
+                          dw, acc_y=None, acc_dx=None, acc_dw=None, workspace=None,
+                          dev_status=None, stream=None) -> None:
+    """Forward, loss-propagation and weight-gradient GEMMs of one layer in one launch."""
+    a = SqLayerGemms(
+        x_codes=_addr(x_codes), ld_x=_ld(x_codes), xt_codes=_addr(xt_codes), ld_xt=_ld(xt_codes),
+        x_scale=_addr(x_scale), x_exp=_addr(x_exp),
+        g_codes=_addr(g_codes), ld_g=_ld(g_codes), gt_codes=_addr(gt_codes), ld_gt=_ld(gt_codes),
+        g_scale=_addr(g_scale), g_exp=_addr(g_exp),
+        wf_codes=_addr(wf_codes), ld_wf=_ld(wf_codes), wf_scale=_addr(wf_scale),
+        wd_codes=_addr(wd_codes), ld_wd=_ld(wd_codes), wd_scale=_addr(wd_scale),
+        M=M, K=K, N=N, bits=bits, n_groups=n_groups,
+        y=_addr(y), ld_y=_ld(y), dx=_addr(dx), ld_dx=_ld(dx), dw=_addr(dw), ld_dw=_ld(dw),
+        acc_y=_addr(acc_y), ld_acc_y=_ld(acc_y) if acc_y is not None else 0,
+        acc_dx=_addr(acc_dx), ld_acc_dx=_ld(acc_dx) if acc_dx is not None else 0,
+        acc_dw=_addr(acc_dw), ld_acc_dw=_ld(acc_dw) if acc_dw is not None else 0)
+    _check(load().shiftquant_gemm_layer(
+        ctypes.byref(a), _ptr(workspace),
+        workspace.numel() * workspace.element_size() if workspace is not None else 0,
+        _ptr(dev_status), _stream(stream)))
+
+
+def shiftquant_gemm_layer_workspace_bytes(M: int, K: int, N: int, bits: int, n_groups: int) -> int:
+    return int(load().shiftquant_gemm_layer_workspace_bytes(M, K, N, bits, n_groups))

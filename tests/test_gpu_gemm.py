@@ -32,11 +32,17 @@ def layer_inputs(rng, M, K, Nn):
     return x, w, dy
 
 
-def run_and_compare(x, w, dy, bits, G, seed=11, use_workspace=True):
+def run_and_compare(x, w, dy, bits, G, seed=11, use_workspace=True, fused=False):
     M, K = x.shape
     Nn = w.shape[1]
     lay = L.QuantLinear(M, K, Nn, bits, G, "cuda", with_acc=True, use_workspace=use_workspace)
-    lay.step(to_gpu(x), to_gpu(w), to_gpu(dy), seed)
+    if fused:
+        lay.quantize_activation(to_gpu(x))
+        lay.quantize_gradient(to_gpu(dy), seed)
+        lay.quantize_weights(to_gpu(w))
+        lay.gemms()
+    else:
+        lay.step(to_gpu(x), to_gpu(w), to_gpu(dy), seed)
     torch.cuda.synchronize()
     assert lay.status.item() == 0
     o = oracle_layer(x, w, dy, bits, G, seed)
@@ -195,3 +201,20 @@ def test_concurrent_step_equals_serial_step():
         np.testing.assert_array_equal(ser.acc[k].cpu().numpy(), con.acc[k].cpu().numpy())
     for a, b in ((ser.y, con.y), (ser.dx, con.dx), (ser.dw, con.dw)):
         np.testing.assert_array_equal(a.cpu().numpy(), b.cpu().numpy())
+
+
+@pytest.mark.parametrize("M,K,Nn", [(5, 3, 7), (300, 1000, 513), (4096, 64, 96), (2000, 700, 256)])
+@pytest.mark.parametrize("bits", [4, 6, 8])
+def test_layer_gemms_in_one_launch_match_oracle(M, K, Nn, bits):
+    # shiftquant_gemm_layer: the three GEMMs share one persistent launch (and one workspace)
+    rng = np.random.default_rng(M + K + Nn + bits)
+    run_and_compare(*layer_inputs(rng, M, K, Nn), bits, 4, fused=True)
+
+
+def test_layer_gemms_equal_separate_launches():
+    rng = np.random.default_rng(5)
+    x, w, dy = layer_inputs(rng, 3000, 640, 384)
+    a = run_and_compare(x, w, dy, 6, 4, fused=True)
+    b = run_and_compare(x, w, dy, 6, 4, fused=False)
+    for t, u in ((a.y, b.y), (a.dx, b.dx), (a.dw, b.dw)):
+        np.testing.assert_array_equal(t.cpu().numpy(), u.cpu().numpy())
