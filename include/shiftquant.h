@@ -201,13 +201,17 @@ typedef struct {
   int64_t *acc_dw; int64_t ld_acc_dw;
 } sq_layer_gemms;
 
-/* workspace: optional int32 scratch of shiftquant_gemm_layer_workspace_bytes() bytes; each
- * GEMM with too few output tiles for the SMs splits its K loop into its own region of it. */
+/* workspace: optional int32 scratch of shiftquant_gemm_layer_workspace_bytes() bytes,
+ * 16-byte aligned.  Its first 256 bytes hold the counter through which the CTAs take their
+ * work units as they free up (the units of the three GEMMs differ in length); without a
+ * workspace each CTA strides over the unit list.  After it, each GEMM with too few output
+ * tiles for the SMs splits its K loop into its own region -- into fewer parts than alone,
+ * as the other GEMMs of the launch keep the SMs busy. */
 sq_status shiftquant_gemm_layer(const sq_layer_gemms *args, void *workspace,
                                 size_t workspace_bytes, int32_t *dev_status, void *stream);
 
-/* Bytes of workspace that let shiftquant_gemm_layer split every GEMM that would benefit
- * (0 when none would) on the current device. */
+/* Bytes of workspace that let shiftquant_gemm_layer schedule its units dynamically and
+ * split every GEMM that would benefit on the current device (at least 256). */
 size_t shiftquant_gemm_layer_workspace_bytes(int64_t M, int64_t K, int64_t N, int bits,
                                              int n_groups);
 

@@ -19,6 +19,9 @@
 //   warp 1      TMEM allocation and the MMA issuer (one thread)
 //   warps 4-11  epilogue: tcgen05.ld, int32 accumulation across chunks, dequantizing
 //               multiply, stores (or int32 reductions into a split-K workspace)
+// Work units reach the three roles through a small shared-memory ring that the producer
+// fills: with a scheduling counter the producer takes each next unit from it (units are
+// handed out in list order as CTAs free up), without one it strides over the list.
 // Every wait is bounded (about 1 s); on expiry the kernel records SQ_DEV_TIMEOUT,
 // drains its own copies and MMAs, frees TMEM and returns.
 #include <cuda.h>
@@ -48,8 +51,9 @@ constexpr int64_t kExactSum = int64_t(1) << 24;  // every partial sum of a chunk
 // 32 x 32 output staging box per epilogue warp (the box turns the lane-per-row TMEM layout
 // into row-contiguous stores).  TMA-store mode, for launches whose outputs outweigh their
 // operands: a 3-stage ring and two staging boxes per warp, so one box is written while TMA
-// stores the other.  Then two per-tile column-factor tables and the barriers.
+// stores the other.  Then two per-tile column-factor tables, the barriers and the unit ring.
 constexpr int kOutBox = 32;
+constexpr int kUnitRing = 8;  // work units published by the producer ahead of the consumers
 constexpr int kOutStageBytes = kOutBox * kOutBox * 4;
 
 template <bool kTmaSt>
@@ -59,8 +63,10 @@ struct Smem {
   static constexpr int out_offset = stages * kStageBytes;
   static constexpr int fac_offset = out_offset + kNumEpiWarps * out_bufs * kOutStageBytes;
   static constexpr int bar_offset = fac_offset + 2 * kBN * 4;
-  static constexpr int num_bars = 2 * stages + 2 + 2 + 2 + 1;  // full, empty, tfull, tempty, fac, drain
-  static constexpr size_t bytes = bar_offset + num_bars * 8 + 16;
+  // full, empty, tfull, tempty, fac, drain, unit ring full / empty
+  static constexpr int num_bars = 2 * stages + 2 + 2 + 2 + 1 + 2 * kUnitRing;
+  static constexpr int ring_offset = bar_offset + num_bars * 8 + 16;  // after TMEM slot, flag
+  static constexpr size_t bytes = ring_offset + kUnitRing * 4;
   static_assert(bytes <= 232448, "shared memory beyond the 227 KB per-CTA limit");
   static_assert(out_offset % 1024 == 0 && kOutStageBytes % 1024 == 0, "swizzle atoms need 1 KB");
 };
@@ -85,8 +91,7 @@ struct GemmParams {
 
 // Up to three GEMMs run by one persistent launch (the three GEMMs of a layer are
 // independent).  Work units of all of them form one list, GEMM by GEMM in the order given
-// (the host puts the GEMM with the longest K loop per unit first); CTA i takes units
-// i, i + gridDim.x, ...
+// (the host puts the GEMM with the longest K loop per unit first).
 constexpr int kMaxBatch = 3;
 struct GemmBatch {
   CUtensorMap a[kMaxBatch];
@@ -96,6 +101,7 @@ struct GemmBatch {
   GemmParams p[kMaxBatch];
   int unit_end[kMaxBatch];  // cumulative unit counts
   int count;
+  int* sched;  // unit counter (zero before launch) for dynamic scheduling, or null
   int* status;
 };
 
@@ -149,7 +155,9 @@ __device__ __noinline__ void write_acc_box(long long* acc, int64_t ld_acc, int64
 }
 
 // One 32 x 32 output box of an epilogue warp: lane = row, vals = the lane's 32 columns as
-// exact integers (FP32 patterns when `as_float`, else int32).  The box is staged in shared
+// exact integers (FP32 patterns when `as_float`, else int32); fac = shared-memory address
+// of the box's 32 column factors (16-byte aligned), rfac the row's factor (weight gradient
+// only: the forward and loss-propagation outputs take the column factor alone).  The box is staged in shared
 // memory (128-byte swizzle) and leaves either as dequantized fp32 values through
 // row-contiguous 16-byte stores (eight lanes per 128-byte row, four rows per instruction),
 // or as int32 partial sums through a TMA reduce-add into the split-K workspace.  The
@@ -157,7 +165,7 @@ __device__ __noinline__ void write_acc_box(long long* acc, int64_t ld_acc, int64
 template <bool kTmaSt>
 __device__ __forceinline__ void emit_box(const GemmParams& p, const CUtensorMap* tma_y,
                                          const CUtensorMap* tma_ws, const uint32_t (&vals)[32],
-                                         bool as_float, const float* f, float rfac, uint32_t buf,
+                                         bool as_float, uint32_t fac, float rfac, uint32_t buf,
                                          int64_t row0, int64_t col0, int lane) {
   const bool tma_out = p.ws != nullptr || (kTmaSt && p.vec_y);
   if (tma_out && lane == 0) {
@@ -182,9 +190,12 @@ __device__ __forceinline__ void emit_box(const GemmParams& p, const CUtensorMap*
                   p.mode == 1 ? p.col_exp : nullptr, p.G, buf, row0, col0, lane);
     __syncwarp();
   }
+  const bool row_scaled = p.mode == 1;
 #pragma unroll
   for (int k = 0; k < 8; ++k) {
     uint32_t o[4];
+    const float4 f4 = p.ws != nullptr ? make_float4(0.f, 0.f, 0.f, 0.f) : ld_shared_v4_f32(fac + k * 16);
+    const float f[4] = {f4.x, f4.y, f4.z, f4.w};
 #pragma unroll
     for (int e = 0; e < 4; ++e) {
       const uint32_t a = vals[k * 4 + e];
@@ -192,7 +203,8 @@ __device__ __forceinline__ void emit_box(const GemmParams& p, const CUtensorMap*
         o[e] = as_float ? static_cast<uint32_t>(__float2int_rn(__uint_as_float(a))) : a;
       } else {
         const float val = as_float ? __uint_as_float(a) : __int2float_rn(static_cast<int32_t>(a));
-        o[e] = __float_as_uint(__fmul_rn(__fmul_rn(val, rfac), f[k * 4 + e]));
+        // x * 1 is x exactly, so skipping the row factor of 1 changes no result
+        o[e] = __float_as_uint(__fmul_rn(row_scaled ? __fmul_rn(val, rfac) : val, f[e]));
       }
     }
     st_shared_v4(buf + lane * 128 + ((k ^ (lane & 7)) << 4), o[0], o[1], o[2], o[3]);
@@ -266,6 +278,7 @@ __device__ __forceinline__ Unit decode_unit(const GemmParams& p, int u) {
 // kMulti: the K loop of a tile spans several exact chunks, whose int32 sums the epilogue
 // keeps in registers; otherwise every output streams from TMEM once.
 // the GEMM of global unit u, and u's index inside that GEMM
+// the GEMM of global unit u, and u's index inside that GEMM
 __device__ __forceinline__ int batch_member(const GemmBatch& bt, int u, int* local) {
   int g = 0;
   while (g + 1 < bt.count && u >= bt.unit_end[g]) ++g;
@@ -291,8 +304,11 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint64_t* tempty = tfull + 2;
   uint64_t* facbar = tempty + 2;
   uint64_t* drain = facbar + 2;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
+  uint64_t* ufull = drain + 1;
+  uint64_t* uempty = ufull + kUnitRing;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(uempty + kUnitRing);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+  volatile int* unit_ring = reinterpret_cast<volatile int*>(smem + L::ring_offset);
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -308,6 +324,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&facbar[b], kNumEpiWarps);
     }
     mbar_init(drain, 1);
+    for (int r = 0; r < kUnitRing; ++r) {
+      mbar_init(&ufull[r], 1);
+      mbar_init(&uempty[r], 1 + kNumEpiWarps);  // the MMA thread and every epilogue warp
+    }
     *abort_flag = 0;
     fence_mbar_init();
   }
@@ -334,7 +354,32 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint32_t ph = 0;
     long long issued = 0;
     bool ok = true;
-    for (int u = blockIdx.x; u < units && ok; u += gridDim.x) {
+    int next = blockIdx.x;  // a CTA's first unit is its own index
+    int us = 0;
+    uint32_t uph = 0;
+    while (ok) {
+      // publish the unit (or, past the end, the stop mark) to the MMA and epilogue roles
+      const int u = next;
+      if (!mbar_wait(&uempty[us], uph ^ 1u, abort_flag)) {
+        ok = false;
+        break;
+      }
+      unit_ring[us] = u;
+      mbar_arrive(&ufull[us]);
+      if (++us == kUnitRing) {
+        us = 0;
+        uph ^= 1u;
+      }
+      if (u >= units) break;
+      // Within the last wave of units a CTA takes its next unit only once its epilogue has
+      // started this one, so that no CTA holds several queued units while others run dry.
+      const bool lazy = bt.sched != nullptr && u >= units - static_cast<int>(gridDim.x);
+      const int u_slot = us == 0 ? kUnitRing - 1 : us - 1;
+      const uint32_t u_par = us == 0 ? uph ^ 1u : uph;
+      if (bt.sched == nullptr)
+        next = u + static_cast<int>(gridDim.x);
+      else if (!lazy)
+        next = static_cast<int>(gridDim.x) + atomicAdd(bt.sched, 1);
       int lu;
       const int g = batch_member(bt, u, &lu);
       const Unit w = decode_unit(bt.p[g], lu);
@@ -353,6 +398,13 @@ __global__ void __launch_bounds__(kThreads, 1)
           ph ^= 1u;
         }
       }
+      if (ok && lazy) {
+        if (!mbar_wait(&uempty[u_slot], u_par, abort_flag)) {
+          ok = false;
+          break;
+        }
+        next = static_cast<int>(gridDim.x) + atomicAdd(bt.sched, 1);
+      }
     }
     if (!ok) {
       atomicOr(bt.status, kDevTimeout);
@@ -368,7 +420,20 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint32_t ph = 0;
     uint32_t c = 0;
     bool ok = true;
-    for (int u = blockIdx.x; u < units && ok; u += gridDim.x) {
+    int us = 0;
+    uint32_t uph = 0;
+    while (ok) {
+      if (!mbar_wait(&ufull[us], uph, abort_flag)) {
+        ok = false;
+        break;
+      }
+      const int u = unit_ring[us];
+      mbar_arrive(&uempty[us]);
+      if (++us == kUnitRing) {
+        us = 0;
+        uph ^= 1u;
+      }
+      if (u >= units) break;
       int lu;
       const int g = batch_member(bt, u, &lu);
       const int chunk_kb = bt.p[g].chunk_kb;
@@ -428,8 +493,21 @@ __global__ void __launch_bounds__(kThreads, 1)
     float* fac_tab = reinterpret_cast<float*>(smem + L::fac_offset);
     uint32_t c = 0;
     bool ok = true;
-    int it = 0;
-    for (int u = blockIdx.x; u < units && ok; u += gridDim.x, ++it) {
+    int us = 0;
+    uint32_t uph = 0;
+    for (int it = 0; ok; ++it) {
+      if (!__all_sync(0xFFFFFFFFu, mbar_wait(&ufull[us], uph, abort_flag))) {
+        ok = false;
+        break;
+      }
+      const int u = unit_ring[us];
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&uempty[us]);
+      if (++us == kUnitRing) {
+        us = 0;
+        uph ^= 1u;
+      }
+      if (u >= units) break;
       int lu;
       const int g = batch_member(bt, u, &lu);
       const GemmParams& p = bt.p[g];
@@ -482,7 +560,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           const int64_t col0 = n0 + h * 128 + s * 32;
           if (row0 >= p.M || col0 >= p.N) continue;  // warp-uniform: nothing of this box exists
           const uint32_t buf = stage_out0 + (nbox++ % L::out_bufs) * kOutStageBytes;
-          emit_box<kTmaSt>(p, tma_y, tma_ws, v, true, fac + h * 128 + s * 32, rfac, buf, row0,
+          emit_box<kTmaSt>(p, tma_y, tma_ws, v, true, smem_u32(fac + h * 128 + s * 32), rfac, buf, row0,
                            col0, lane);
         }
         ++c;
@@ -527,7 +605,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
           for (int i = 0; i < 32; ++i) v[i] = acc[s * 32 + i];
           const uint32_t buf = stage_out0 + (nbox++ % L::out_bufs) * kOutStageBytes;
-          emit_box<kTmaSt>(p, tma_y, tma_ws, v, false, fac + h * 128 + s * 32, rfac, buf, row0,
+          emit_box<kTmaSt>(p, tma_y, tma_ws, v, false, smem_u32(fac + h * 128 + s * 32), rfac, buf, row0,
                            col0, lane);
         }
       }
@@ -650,8 +728,9 @@ static int check_exact_range(int which, int64_t K, int bits, int G) {
   return SQ_OK;
 }
 
+// max_splits: 1 never splits K; 0 lets the SM count alone decide
 static int make_plan(int which, int64_t M, int64_t N, int64_t K, int bits, int G, int sms,
-                     bool allow_split, Plan* pl) {
+                     int max_splits, Plan* pl) {
   const int st = check_exact_range(which, K, bits, G);
   if (st != SQ_OK) return st;
   const int64_t P = max_product(which, bits, G);
@@ -664,15 +743,24 @@ static int make_plan(int which, int64_t M, int64_t N, int64_t K, int bits, int G
   pl->kb_total = static_cast<int>((K + bk - 1) / bk);
   const int64_t tiles = static_cast<int64_t>(pl->m_tiles) * pl->n_tiles;
   int splits = 1;
-  if (allow_split && tiles < sms && pl->kb_total >= 4) {
+  if (max_splits != 1 && tiles < sms && pl->kb_total >= 4) {
     splits = static_cast<int>(sms / tiles);
     if (splits > pl->kb_total / 2) splits = pl->kb_total / 2;
+    if (max_splits > 1 && splits > max_splits) splits = max_splits;
     if (splits < 1) splits = 1;
   }
   pl->kb_per_split = (pl->kb_total + splits - 1) / splits;
   pl->splits = (pl->kb_total + pl->kb_per_split - 1) / pl->kb_per_split;
   return SQ_OK;
 }
+
+// Split-K workspace of one GEMM: the int32 partial sums [M, N], zeroed before every launch
+// that uses them, rounded up to 256 bytes.
+static size_t split_ws_bytes(int64_t M, int64_t N) {
+  return (static_cast<size_t>(M) * static_cast<size_t>(N) * sizeof(int) + 255) & ~size_t(255);
+}
+// The layer launch's workspace starts with the unit counter of its dynamic schedule.
+constexpr size_t kSchedBytes = 256;
 
 template <int kF8, bool kMulti, bool kTmaSt>
 static int configure_kernel(int dev) {
@@ -752,16 +840,16 @@ static int check_job(const GemmJob& j, int bits, int G, int32_t* dev_status, cud
 
 // Plan of one checked GEMM and its slot in the batch: tiles, K splits (only with a
 // workspace large enough for the [M, N] int32 partial sums), tensor maps, parameters.
-static int prepare_job(const GemmJob& j, int bits, int G, int sms, int32_t* dev_status,
-                       GemmBatch* bt, int g, Plan* pl) {
-  int st = make_plan(j.which, j.M, j.N, j.K, bits, G, sms, true, pl);
+static int prepare_job(const GemmJob& j, int bits, int G, int sms, int max_splits,
+                       int32_t* dev_status, GemmBatch* bt, int g, Plan* pl) {
+  int st = make_plan(j.which, j.M, j.N, j.K, bits, G, sms, max_splits, pl);
   if (st != SQ_OK) return st;
   if (pl->splits > 1) {
     // split-K partials are added by TMA into a [M, N] int32 workspace with N-element rows,
     // whose rows must stay 16-byte aligned
-    const size_t need = static_cast<size_t>(j.M) * j.N * sizeof(int);
+    const size_t need = split_ws_bytes(j.M, j.N);
     if (j.ws == nullptr || j.ws_bytes < need || !aligned16(j.ws) || j.N % 4 != 0) {
-      st = make_plan(j.which, j.M, j.N, j.K, bits, G, sms, false, pl);
+      st = make_plan(j.which, j.M, j.N, j.K, bits, G, sms, 1, pl);
       if (st != SQ_OK) return st;
     }
   }
@@ -821,7 +909,11 @@ static int launch_variant(const GemmBatch& bt, int grid, int dev, cudaStream_t s
 
 // Checks, plans and launches up to kMaxBatch GEMMs (all with the same bits / n_groups) as
 // one persistent kernel; split-K partial sums are zeroed before and finalized after it.
-static int run_jobs(GemmJob* jobs, int njobs, int bits, int G, int32_t* dev_status, void* stream) {
+// sched (may be null): a unit counter, zeroed here before the launch, through which the
+// CTAs take their units as they free up -- for batches whose units differ in length.
+// Without one each CTA strides over the unit list.
+static int run_jobs(GemmJob* jobs, int njobs, int bits, int G, int32_t* dev_status, void* stream,
+                    int* sched) {
   cudaStream_t s = as_stream(stream);
   int live[kMaxBatch];
   int nlive = 0;
@@ -839,8 +931,34 @@ static int run_jobs(GemmJob* jobs, int njobs, int bits, int G, int32_t* dev_stat
   memset(&bt, 0, sizeof(bt));
   Plan plans[kMaxBatch];
   for (int g = 0; g < nlive; ++g) {
-    const int st = prepare_job(jobs[live[g]], bits, G, sms, dev_status, &bt, g, &plans[g]);
+    const int st = prepare_job(jobs[live[g]], bits, G, sms, 0, dev_status, &bt, g, &plans[g]);
     if (st != SQ_OK) return st;
+  }
+  // Sharing the launch with other GEMMs, a split GEMM needs fewer splits: just enough that
+  // its units stay well inside the launch's expected length.  Every split adds the whole
+  // output once more to the L2 reductions, whose throughput is far below a plain store's.
+  // Unit cost model, in K-block times: the K loop plus about 8 for the epilogue.
+  if (nlive > 1) {
+    constexpr double kEpiKb = 8.0;
+    double work = 0.0;  // the batch's total cost, with every split GEMM at its maximum
+    for (int g = 0; g < nlive; ++g)
+      work += static_cast<double>(plans[g].m_tiles) * plans[g].n_tiles * plans[g].splits *
+              (plans[g].kb_per_split + kEpiKb);
+    for (int g = 0; g < nlive; ++g) {
+      if (plans[g].splits <= 1) continue;
+      const double tiles = static_cast<double>(plans[g].m_tiles) * plans[g].n_tiles;
+      int s = 1;
+      for (; s < plans[g].splits; ++s) {
+        const double kbs = static_cast<double>((plans[g].kb_total + s - 1) / s);
+        const double w = work - tiles * plans[g].splits * (plans[g].kb_per_split + kEpiKb) +
+                         tiles * s * (kbs + kEpiKb);
+        if (kbs + kEpiKb <= 0.8 * w / sms) break;
+      }
+      if (s < plans[g].splits) {
+        const int st = prepare_job(jobs[live[g]], bits, G, sms, s, dev_status, &bt, g, &plans[g]);
+        if (st != SQ_OK) return st;
+      }
+    }
   }
   // longest K loop per unit first: the short units then fill in behind the long ones
   for (int a = 0; a < nlive; ++a)
@@ -863,12 +981,27 @@ static int run_jobs(GemmJob* jobs, int njobs, int bits, int G, int32_t* dev_stat
   }
   bt.count = nlive;
   bt.status = dev_status;
+  bt.sched = sched;
+  // zero the counter and the partial sums, with one memset for the regions that follow the
+  // counter back to back
+  char* zero_from = reinterpret_cast<char*>(sched);
+  char* zero_end = sched ? zero_from + kSchedBytes : nullptr;
   cudaError_t err;
-  for (int g = 0; g < nlive; ++g)
-    if (bt.p[g].ws) {
-      err = cudaMemsetAsync(bt.p[g].ws, 0, static_cast<size_t>(bt.p[g].M) * bt.p[g].N * sizeof(int), s);
-      if (err != cudaSuccess) return cuda_fail(err, "cudaMemsetAsync");
+  for (int g = 0; g < nlive; ++g) {
+    if (!bt.p[g].ws) continue;
+    char* w = reinterpret_cast<char*>(bt.p[g].ws);
+    const size_t b = split_ws_bytes(bt.p[g].M, bt.p[g].N);
+    if (zero_end != nullptr && w == zero_end) {
+      zero_end = w + b;
+      continue;
     }
+    err = cudaMemsetAsync(w, 0, b, s);
+    if (err != cudaSuccess) return cuda_fail(err, "cudaMemsetAsync");
+  }
+  if (zero_from != nullptr) {
+    err = cudaMemsetAsync(zero_from, 0, static_cast<size_t>(zero_end - zero_from), s);
+    if (err != cudaSuccess) return cuda_fail(err, "cudaMemsetAsync");
+  }
   // TMA-store mode when the outputs written are a large share of the operand tiles read
   double out_bytes = 0.0, in_bytes = 0.0;
   for (int g = 0; g < nlive; ++g) {
@@ -900,7 +1033,7 @@ static int run_gemm(int which, const void* a_codes, int64_t lda, const void* b_c
                     size_t workspace_bytes, int32_t* dev_status, void* stream) {
   GemmJob j{which, a_codes, lda, b_codes, ldb, M, N, K, a_scale, b_scale, row_exp, col_exp,
             y, ldy, acc_out, ld_acc, workspace, workspace_bytes};
-  return run_jobs(&j, 1, bits, G, dev_status, stream);
+  return run_jobs(&j, 1, bits, G, dev_status, stream, nullptr);
 }
 
 // The three GEMMs of a layer as jobs, workspace regions assigned to those that split.
@@ -914,16 +1047,16 @@ static void layer_jobs(const sq_layer_gemms* a, GemmJob jobs[3]) {
                     nullptr, 0};
 }
 
-// Bytes each GEMM of the layer would use for split-K partial sums (0: it would not split),
-// each rounded up to 256 bytes.
+// Bytes of split-K workspace each GEMM of the layer would use (0: it would not split),
+// a multiple of 256 bytes.
 static void layer_ws_need(const GemmJob jobs[3], int bits, int G, int sms, size_t need[3]) {
   for (int i = 0; i < 3; ++i) {
     need[i] = 0;
     const GemmJob& j = jobs[i];
     if (j.M <= 0 || j.N <= 0 || j.K <= 0 || j.N % 4 != 0) continue;
     Plan pl;
-    if (make_plan(j.which, j.M, j.N, j.K, bits, G, sms, true, &pl) != SQ_OK) continue;
-    if (pl.splits > 1) need[i] = (static_cast<size_t>(j.M) * j.N * sizeof(int) + 255) & ~size_t(255);
+    if (make_plan(j.which, j.M, j.N, j.K, bits, G, sms, 0, &pl) != SQ_OK) continue;
+    if (pl.splits > 1) need[i] = split_ws_bytes(j.M, j.N);
   }
 }
 
@@ -932,7 +1065,8 @@ static void layer_ws_need(const GemmJob jobs[3], int bits, int G, int sms, size_
 // the library's own device image, present on every GPU that loads the library until the
 // process exits.  It serves as the split-K int32 workspace of
 // shiftquant_gemm_wgrad_static().
-constexpr size_t kStaticScratchBytes = size_t(4) << 20;  // 4 MiB: Ci * Co <= 1048576
+constexpr int64_t kStaticMaxOutputs = int64_t(1) << 20;  // Ci * Co
+constexpr size_t kStaticScratchBytes = size_t(4) << 20;   // the int32 sums of 2^20 outputs
 static __device__ __align__(256) int g_wgrad_scratch[kStaticScratchBytes / sizeof(int)];
 
 // Device address of g_wgrad_scratch on the current device.  In host code the array's
@@ -1004,8 +1138,8 @@ extern "C" size_t shiftquant_gemm_workspace_bytes(int which, int64_t M, int64_t 
   const int sms = device_sms(nullptr);
   if (sms <= 0) return 0;
   Plan pl;
-  if (make_plan(which, M, N, K, bits, n_groups, sms, true, &pl) != SQ_OK) return 0;
-  return pl.splits > 1 ? static_cast<size_t>(M) * N * sizeof(int) : 0;
+  if (make_plan(which, M, N, K, bits, n_groups, sms, 0, &pl) != SQ_OK) return 0;
+  return pl.splits > 1 ? split_ws_bytes(M, N) : 0;
 }
 
 extern "C" sq_status shiftquant_gemm_wgrad_static(
@@ -1014,13 +1148,12 @@ extern "C" sq_status shiftquant_gemm_wgrad_static(
     int64_t Co, int64_t T, int bits, int n_groups, float* dw, int64_t ld_dw, int64_t* acc_out,
     int64_t ld_acc, int32_t* dev_status, void* stream) {
   fail(SQ_OK, "");
-  if (Ci > 0 && Co > 0 &&
-      static_cast<uint64_t>(Ci) * static_cast<uint64_t>(Co) * sizeof(int) > kStaticScratchBytes)
+  if (Ci > 0 && Co > 0 && Ci * Co > kStaticMaxOutputs)
     return fail(SQ_EUNSUPPORTED,
-                "gemm_wgrad_static: Ci * Co = %lld exceeds the %zu int32 entries of the "
-                "library's static scratch; use shiftquant_gemm_wgrad with a caller workspace",
+                "gemm_wgrad_static: Ci * Co = %lld exceeds the %lld outputs of the library's "
+                "static scratch; use shiftquant_gemm_wgrad with a caller workspace",
                 static_cast<long long>(Ci) * static_cast<long long>(Co),
-                kStaticScratchBytes / sizeof(int));
+                static_cast<long long>(kStaticMaxOutputs));
   void* scratch = nullptr;
   if (Ci > 0 && Co > 0 && T > 0) {
     const int st = static_scratch_address(&scratch);
@@ -1040,12 +1173,14 @@ extern "C" sq_status shiftquant_gemm_layer(const sq_layer_gemms* args, void* wor
     return fail(SQ_EINVAL, "gemm_layer: bits must be in [2, 8] and n_groups in [1, 8]");
   GemmJob jobs[3];
   layer_jobs(args, jobs);
-  if (workspace != nullptr && workspace_bytes > 0) {
+  int* sched = nullptr;
+  if (workspace != nullptr && workspace_bytes >= kSchedBytes && aligned16(workspace)) {
+    sched = static_cast<int*>(workspace);
     const int sms = device_sms(nullptr);
     if (sms > 0) {
       size_t need[3];
       layer_ws_need(jobs, args->bits, args->n_groups, sms, need);
-      size_t off = 0;
+      size_t off = kSchedBytes;
       for (int i = 0; i < 3; ++i) {
         if (need[i] == 0 || off + need[i] > workspace_bytes) continue;
         jobs[i].ws = static_cast<char*>(workspace) + off;
@@ -1054,7 +1189,7 @@ extern "C" sq_status shiftquant_gemm_layer(const sq_layer_gemms* args, void* wor
       }
     }
   }
-  return run_jobs(jobs, 3, args->bits, args->n_groups, dev_status, stream);
+  return run_jobs(jobs, 3, args->bits, args->n_groups, dev_status, stream, sched);
 }
 
 extern "C" size_t shiftquant_gemm_layer_workspace_bytes(int64_t M, int64_t K, int64_t N, int bits,
@@ -1071,5 +1206,5 @@ extern "C" size_t shiftquant_gemm_layer_workspace_bytes(int64_t M, int64_t K, in
   layer_jobs(&a, jobs);
   size_t need[3];
   layer_ws_need(jobs, bits, n_groups, sms, need);
-  return need[0] + need[1] + need[2];
+  return kSchedBytes + need[0] + need[1] + need[2];
 }
