@@ -172,8 +172,10 @@ class Step:
             n += 2 + 1 + 2 + 1          # X and dY: range init + range/grouping, quantize
             n += 2 + 1 + 1 + 1          # weights: range init + range, quantize (out-channel);
                                         # row range, quantize (in-channel)
-            n += 1                      # the three GEMMs: one launch
-            n += sum(ws is not None for ws in (lay.ws_fwd, lay.ws_dgrad, lay.ws_wgrad))  # finalize
+            # the three GEMMs: one launch, plus the output pass of each GEMM that splits K
+            n += N.shiftquant_gemm_layer_kernel_launches(
+                lay.M, lay.K, lay.N, lay.bits, lay.G,
+                0 if lay.ws_layer is None else lay.ws_layer.numel() * 4)
         return n
 
     def gemm_ops(self) -> int:
@@ -394,8 +396,8 @@ def run_ours(args, rank, world, local_rank):
     quant_roof = {"bound": "hbm", "achieved": q_gbs, "peak": peaks["hbm_gbs"], "unit": "GB/s",
                   "frac": q_gbs / peaks["hbm_gbs"], "kernel": "calibrate + quantize",
                   "peak_source": f"{peak_src} copy bandwidth"}
-    # the dominant kernel: the kernel class (range pass, quantize, layer GEMM launch) with
-    # the most device time in the step
+    # the dominant kernel: the kernel class (range pass, quantize, layer GEMM launch) of the
+    # single launch with the most device time in the step
     def hbm_roof(nbytes, ms, name):
         gbs = nbytes * args.steps / (ms * 1e-3) / 1e9
         return {"bound": "hbm", "achieved": gbs, "peak": peaks["hbm_gbs"], "unit": "GB/s",
@@ -407,7 +409,10 @@ def run_ours(args, rank, world, local_rank):
                                              "(range pass with grouping)")),
              (kind_ms["quantize"], hbm_roof(st.quantize_bytes(), kind_ms["quantize"],
                                             "quantize_kernel"))]
-    dominant = max(cands, key=lambda c: c[0])[1]
+    longest = {k: max([v for n, v in zip(names, call_ms) if n == k] or [0.0])
+               for k in ("gemm", "calibrate", "quantize")}
+    dominant = max(zip(("gemm", "calibrate", "quantize"), cands),
+                   key=lambda kc: longest[kc[0]])[1][1]
 
     result = {
         "metric": METRIC,

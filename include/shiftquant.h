@@ -215,6 +215,13 @@ sq_status shiftquant_gemm_layer(const sq_layer_gemms *args, void *workspace,
 size_t shiftquant_gemm_layer_workspace_bytes(int64_t M, int64_t K, int64_t N, int bits,
                                              int n_groups);
 
+/* Number of kernels one shiftquant_gemm_layer call with this shape and workspace size
+ * launches on the current device: the GEMM launch, plus one output pass per GEMM that
+ * splits its K loop (0 when every GEMM is empty; memsets are not counted).  -1 for invalid
+ * arguments, a shape beyond the exact range, or no device. */
+int shiftquant_gemm_layer_kernel_launches(int64_t M, int64_t K, int64_t N, int bits,
+                                          int n_groups, size_t workspace_bytes);
+
 /* Weight-gradient GEMM for callers that cannot allocate device memory -- for instance a
  * plug-in running inside a host framework that owns every device allocation, or a
  * deployment whose device memory is fixed when the library is loaded.  The paper has no

@@ -38,6 +38,16 @@ __device__ __forceinline__ float4 ld_stream_v4(const float* p) {
   return v;
 }
 
+// ----------------------------------------------------- programmatic dependent launch
+// Wait until the preceding kernel of the stream has completed and its writes are visible
+// (a no-op for a kernel launched without programmatic stream serialization).
+__device__ __forceinline__ void griddep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+// Let the next kernel of the stream (if launched with programmatic stream serialization)
+// start its launch; it still waits for this grid's completion before reading its results.
+__device__ __forceinline__ void griddep_launch_dependents() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
 // ------------------------------------------------------------------ mbarrier
 __device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
   asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count)

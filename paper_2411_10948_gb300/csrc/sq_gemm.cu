@@ -838,21 +838,50 @@ static int check_job(const GemmJob& j, int bits, int G, int32_t* dev_status, cud
   return SQ_OK;
 }
 
-// Plan of one checked GEMM and its slot in the batch: tiles, K splits (only with a
-// workspace large enough for the [M, N] int32 partial sums), tensor maps, parameters.
-static int prepare_job(const GemmJob& j, int bits, int G, int sms, int max_splits,
-                       int32_t* dev_status, GemmBatch* bt, int g, Plan* pl) {
-  int st = make_plan(j.which, j.M, j.N, j.K, bits, G, sms, max_splits, pl);
-  if (st != SQ_OK) return st;
-  if (pl->splits > 1) {
-    // split-K partials are added by TMA into a [M, N] int32 workspace with N-element rows,
-    // whose rows must stay 16-byte aligned
-    const size_t need = split_ws_bytes(j.M, j.N);
-    if (j.ws == nullptr || j.ws_bytes < need || !aligned16(j.ws) || j.N % 4 != 0) {
-      st = make_plan(j.which, j.M, j.N, j.K, bits, G, sms, 1, pl);
+// Tiles and K splits of one checked GEMM: the SM count decides the splits, up to
+// max_splits, and a split needs a workspace for the [M, N] int32 partial sums (added by TMA
+// into N-element rows, which must stay 16-byte aligned).
+static int plan_job(const GemmJob& j, int bits, int G, int sms, int max_splits, Plan* pl) {
+  const int st = make_plan(j.which, j.M, j.N, j.K, bits, G, sms, max_splits, pl);
+  if (st != SQ_OK || pl->splits <= 1) return st;
+  if (j.ws == nullptr || j.ws_bytes < split_ws_bytes(j.M, j.N) || !aligned16(j.ws) || j.N % 4 != 0)
+    return make_plan(j.which, j.M, j.N, j.K, bits, G, sms, 1, pl);
+  return SQ_OK;
+}
+
+// Sharing the launch with other GEMMs, a split GEMM needs fewer splits: just enough that
+// its units stay well inside the launch's expected length.  Every split adds the whole
+// output once more to the L2 reductions, whose throughput is far below a plain store's.
+// Unit cost model, in K-block times: the K loop plus about 8 for the epilogue.
+static int balance_splits(GemmJob* const* jobs, int n, int bits, int G, int sms, Plan* plans) {
+  if (n <= 1) return SQ_OK;
+  constexpr double kEpiKb = 8.0;
+  double work = 0.0;  // the batch's total cost, with every split GEMM at its maximum
+  for (int g = 0; g < n; ++g)
+    work += static_cast<double>(plans[g].m_tiles) * plans[g].n_tiles * plans[g].splits *
+            (plans[g].kb_per_split + kEpiKb);
+  for (int g = 0; g < n; ++g) {
+    if (plans[g].splits <= 1) continue;
+    const double tiles = static_cast<double>(plans[g].m_tiles) * plans[g].n_tiles;
+    int s = 1;
+    for (; s < plans[g].splits; ++s) {
+      const double kbs = static_cast<double>((plans[g].kb_total + s - 1) / s);
+      const double w = work - tiles * plans[g].splits * (plans[g].kb_per_split + kEpiKb) +
+                       tiles * s * (kbs + kEpiKb);
+      if (kbs + kEpiKb <= 0.8 * w / sms) break;
+    }
+    if (s < plans[g].splits) {
+      const int st = plan_job(*jobs[g], bits, G, sms, s, &plans[g]);
       if (st != SQ_OK) return st;
     }
   }
+  return SQ_OK;
+}
+
+// Slot g of the batch for one planned GEMM: tensor maps and parameters.
+static int prepare_job(const GemmJob& j, const Plan* pl, int G, int32_t* dev_status,
+                       GemmBatch* bt, int g) {
+  int st;
   const int eb = pl->elem_bytes;
   if ((st = make_operand_map(&bt->a[g], j.a, j.M, j.K, j.lda, eb, kBM)) != SQ_OK) return st;
   if ((st = make_operand_map(&bt->b[g], j.b, j.N, j.K, j.ldb, eb, kBN)) != SQ_OK) return st;
@@ -930,36 +959,16 @@ static int run_jobs(GemmJob* jobs, int njobs, int bits, int G, int32_t* dev_stat
   GemmBatch bt;
   memset(&bt, 0, sizeof(bt));
   Plan plans[kMaxBatch];
+  GemmJob* lj[kMaxBatch];
   for (int g = 0; g < nlive; ++g) {
-    const int st = prepare_job(jobs[live[g]], bits, G, sms, 0, dev_status, &bt, g, &plans[g]);
+    lj[g] = &jobs[live[g]];
+    const int st = plan_job(*lj[g], bits, G, sms, 0, &plans[g]);
     if (st != SQ_OK) return st;
   }
-  // Sharing the launch with other GEMMs, a split GEMM needs fewer splits: just enough that
-  // its units stay well inside the launch's expected length.  Every split adds the whole
-  // output once more to the L2 reductions, whose throughput is far below a plain store's.
-  // Unit cost model, in K-block times: the K loop plus about 8 for the epilogue.
-  if (nlive > 1) {
-    constexpr double kEpiKb = 8.0;
-    double work = 0.0;  // the batch's total cost, with every split GEMM at its maximum
-    for (int g = 0; g < nlive; ++g)
-      work += static_cast<double>(plans[g].m_tiles) * plans[g].n_tiles * plans[g].splits *
-              (plans[g].kb_per_split + kEpiKb);
-    for (int g = 0; g < nlive; ++g) {
-      if (plans[g].splits <= 1) continue;
-      const double tiles = static_cast<double>(plans[g].m_tiles) * plans[g].n_tiles;
-      int s = 1;
-      for (; s < plans[g].splits; ++s) {
-        const double kbs = static_cast<double>((plans[g].kb_total + s - 1) / s);
-        const double w = work - tiles * plans[g].splits * (plans[g].kb_per_split + kEpiKb) +
-                         tiles * s * (kbs + kEpiKb);
-        if (kbs + kEpiKb <= 0.8 * w / sms) break;
-      }
-      if (s < plans[g].splits) {
-        const int st = prepare_job(jobs[live[g]], bits, G, sms, s, dev_status, &bt, g, &plans[g]);
-        if (st != SQ_OK) return st;
-      }
-    }
-  }
+  int st = balance_splits(lj, nlive, bits, G, sms, plans);
+  if (st != SQ_OK) return st;
+  for (int g = 0; g < nlive; ++g)
+    if ((st = prepare_job(*lj[g], &plans[g], G, dev_status, &bt, g)) != SQ_OK) return st;
   // longest K loop per unit first: the short units then fill in behind the long ones
   for (int a = 0; a < nlive; ++a)
     for (int b = a + 1; b < nlive; ++b)
@@ -1011,8 +1020,8 @@ static int run_jobs(GemmJob* jobs, int njobs, int bits, int G, int32_t* dev_stat
   }
   const bool tma_st = out_bytes > 0.2 * in_bytes;
   const int grid = units < sms ? units : sms;
-  const int st = plans[0].elem_bytes == 1 ? launch_variant<1>(bt, grid, dev, s, multi, tma_st)
-                                          : launch_variant<0>(bt, grid, dev, s, multi, tma_st);
+  st = plans[0].elem_bytes == 1 ? launch_variant<1>(bt, grid, dev, s, multi, tma_st)
+                                : launch_variant<0>(bt, grid, dev, s, multi, tma_st);
   if (st != SQ_OK) return st;
   for (int g = 0; g < nlive; ++g) {
     if (!bt.p[g].ws) continue;
@@ -1058,6 +1067,26 @@ static void layer_ws_need(const GemmJob jobs[3], int bits, int G, int sms, size_
     if (make_plan(j.which, j.M, j.N, j.K, bits, G, sms, 0, &pl) != SQ_OK) continue;
     if (pl.splits > 1) need[i] = split_ws_bytes(j.M, j.N);
   }
+}
+
+// The layer workspace: the unit counter, then a split-K region for each GEMM that would
+// split, as far as the workspace reaches.  Returns the counter (null without a usable
+// workspace: the launch then strides over its units and splits nothing).
+static int* assign_layer_ws(GemmJob jobs[3], int bits, int G, int sms, void* workspace,
+                            size_t workspace_bytes) {
+  if (workspace == nullptr || workspace_bytes < kSchedBytes || !aligned16(workspace)) return nullptr;
+  if (sms > 0) {
+    size_t need[3];
+    layer_ws_need(jobs, bits, G, sms, need);
+    size_t off = kSchedBytes;
+    for (int i = 0; i < 3; ++i) {
+      if (need[i] == 0 || off + need[i] > workspace_bytes) continue;
+      jobs[i].ws = static_cast<char*>(workspace) + off;
+      jobs[i].ws_bytes = need[i];
+      off += need[i];
+    }
+  }
+  return static_cast<int*>(workspace);
 }
 
 // ----------------------------------------------- allocation-free weight gradient
@@ -1173,22 +1202,8 @@ extern "C" sq_status shiftquant_gemm_layer(const sq_layer_gemms* args, void* wor
     return fail(SQ_EINVAL, "gemm_layer: bits must be in [2, 8] and n_groups in [1, 8]");
   GemmJob jobs[3];
   layer_jobs(args, jobs);
-  int* sched = nullptr;
-  if (workspace != nullptr && workspace_bytes >= kSchedBytes && aligned16(workspace)) {
-    sched = static_cast<int*>(workspace);
-    const int sms = device_sms(nullptr);
-    if (sms > 0) {
-      size_t need[3];
-      layer_ws_need(jobs, args->bits, args->n_groups, sms, need);
-      size_t off = kSchedBytes;
-      for (int i = 0; i < 3; ++i) {
-        if (need[i] == 0 || off + need[i] > workspace_bytes) continue;
-        jobs[i].ws = static_cast<char*>(workspace) + off;
-        jobs[i].ws_bytes = need[i];
-        off += need[i];
-      }
-    }
-  }
+  const int sms = device_sms(nullptr);
+  int* sched = assign_layer_ws(jobs, args->bits, args->n_groups, sms, workspace, workspace_bytes);
   return run_jobs(jobs, 3, args->bits, args->n_groups, dev_status, stream, sched);
 }
 
@@ -1207,4 +1222,35 @@ extern "C" size_t shiftquant_gemm_layer_workspace_bytes(int64_t M, int64_t K, in
   size_t need[3];
   layer_ws_need(jobs, bits, n_groups, sms, need);
   return kSchedBytes + need[0] + need[1] + need[2];
+}
+
+extern "C" int shiftquant_gemm_layer_kernel_launches(int64_t M, int64_t K, int64_t N, int bits,
+                                                     int n_groups, size_t workspace_bytes) {
+  if (!bits_ok(bits) || !groups_ok(n_groups) || M < 0 || K < 0 || N < 0) return -1;
+  const int sms = device_sms(nullptr);
+  if (sms <= 0) return -1;
+  sq_layer_gemms a;
+  memset(&a, 0, sizeof(a));
+  a.M = M;
+  a.K = K;
+  a.N = N;
+  GemmJob jobs[3];
+  layer_jobs(&a, jobs);
+  // the plan looks at the workspace's size and alignment only: a stand-in address serves
+  assign_layer_ws(jobs, bits, n_groups, sms, workspace_bytes ? reinterpret_cast<void*>(4096) : nullptr,
+                  workspace_bytes);
+  Plan plans[kMaxBatch];
+  GemmJob* lj[kMaxBatch];
+  int n = 0;
+  for (int i = 0; i < 3; ++i) {
+    if (jobs[i].M == 0 || jobs[i].N == 0 || jobs[i].K == 0) continue;
+    lj[n] = &jobs[i];
+    if (plan_job(jobs[i], bits, n_groups, sms, 0, &plans[n]) != SQ_OK) return -1;
+    ++n;
+  }
+  if (n == 0) return 0;
+  if (balance_splits(lj, n, bits, n_groups, sms, plans) != SQ_OK) return -1;
+  int launches = 1;
+  for (int g = 0; g < n; ++g) launches += plans[g].splits > 1;
+  return launches;
 }

@@ -58,9 +58,11 @@ __device__ __forceinline__ int group_exponent(float r, float tau, int G) {
   return e;
 }
 
-// zero the range accumulators (and the completion counter of the grouping step)
+// zero the range accumulators (and the completion counter of the grouping step); the range
+// pass that follows may launch at once: it reads x first and these only after its wait
 __global__ void __launch_bounds__(256)
     calib_init_kernel(unsigned* __restrict__ range_bits, int64_t C, unsigned* __restrict__ counter) {
+  griddep_launch_dependents();
   for (int64_t c = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; c < C;
        c += static_cast<int64_t>(gridDim.x) * blockDim.x)
     range_bits[c] = 0u;
@@ -136,6 +138,10 @@ __global__ void __launch_bounds__(kColTx* kColTy)
       }
     }
   }
+  // x has been read: the next kernel (the quantizer) may start launching; the
+  // accumulators below are zeroed by the preceding kernel, which must have completed
+  griddep_launch_dependents();
+  griddep_wait();
   red[ty][tx * 4 + 0] = m0;
   red[ty][tx * 4 + 1] = m1;
   red[ty][tx * 4 + 2] = m2;
@@ -501,6 +507,8 @@ __device__ __forceinline__ void quantize_tile(const QuantArgs& a, uint8_t* tile_
 template <typename CodeT, int GRAN, int MODE, bool FOLD>
 __global__ void __launch_bounds__(256) quantize_kernel(const QuantArgs a) {
   __shared__ __align__(16) uint8_t tile_t[kQC * 8 * 8 * sizeof(CodeT)];
+  // launched early behind the range pass: nothing it wrote (nor x) is read before it is done
+  griddep_wait();
   const bool full = (static_cast<int64_t>(blockIdx.y) + 1) * kQR <= a.R &&
                     (static_cast<int64_t>(blockIdx.x) + 1) * kQC <= a.C && a.vec_in &&
                     (a.codes == nullptr || a.vec_out) && (a.codes_t == nullptr || a.vec_t);
@@ -510,29 +518,49 @@ __global__ void __launch_bounds__(256) quantize_kernel(const QuantArgs a) {
     quantize_tile<CodeT, GRAN, MODE, FOLD, false>(a, tile_t);
 }
 
+// Launch with programmatic stream serialization: the kernel may begin launching while the
+// preceding kernel of the stream finishes, and waits for it (griddep_wait) before reading
+// anything.
+template <typename... Params, typename... Args>
+static cudaError_t launch_pdl(void (*kernel)(Params...), dim3 grid, dim3 block, cudaStream_t s,
+                              Args... args) {
+  cudaLaunchConfig_t cfg;
+  memset(&cfg, 0, sizeof(cfg));
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = 0;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kernel, args...);
+}
+
 template <typename CodeT>
 static void launch_quantize(const QuantArgs& a, dim3 grid, cudaStream_t s) {
   const bool fold = a.fold != nullptr;
   if (a.gran == SQ_GRAN_SHIFT) {
     if (a.mode == SQ_ROUND_NEAREST_EVEN)
-      quantize_kernel<CodeT, SQ_GRAN_SHIFT, SQ_ROUND_NEAREST_EVEN, false><<<grid, 256, 0, s>>>(a);
+      launch_pdl(quantize_kernel<CodeT, SQ_GRAN_SHIFT, SQ_ROUND_NEAREST_EVEN, false>, grid, dim3(256), s, a);
     else
-      quantize_kernel<CodeT, SQ_GRAN_SHIFT, SQ_ROUND_STOCHASTIC, false><<<grid, 256, 0, s>>>(a);
+      launch_pdl(quantize_kernel<CodeT, SQ_GRAN_SHIFT, SQ_ROUND_STOCHASTIC, false>, grid, dim3(256), s, a);
   } else if (a.gran == SQ_GRAN_PER_COL) {
     if (a.mode == SQ_ROUND_NEAREST_EVEN) {
-      if (fold) quantize_kernel<CodeT, SQ_GRAN_PER_COL, SQ_ROUND_NEAREST_EVEN, true><<<grid, 256, 0, s>>>(a);
-      else quantize_kernel<CodeT, SQ_GRAN_PER_COL, SQ_ROUND_NEAREST_EVEN, false><<<grid, 256, 0, s>>>(a);
+      if (fold) launch_pdl(quantize_kernel<CodeT, SQ_GRAN_PER_COL, SQ_ROUND_NEAREST_EVEN, true>, grid, dim3(256), s, a);
+      else launch_pdl(quantize_kernel<CodeT, SQ_GRAN_PER_COL, SQ_ROUND_NEAREST_EVEN, false>, grid, dim3(256), s, a);
     } else {
-      if (fold) quantize_kernel<CodeT, SQ_GRAN_PER_COL, SQ_ROUND_STOCHASTIC, true><<<grid, 256, 0, s>>>(a);
-      else quantize_kernel<CodeT, SQ_GRAN_PER_COL, SQ_ROUND_STOCHASTIC, false><<<grid, 256, 0, s>>>(a);
+      if (fold) launch_pdl(quantize_kernel<CodeT, SQ_GRAN_PER_COL, SQ_ROUND_STOCHASTIC, true>, grid, dim3(256), s, a);
+      else launch_pdl(quantize_kernel<CodeT, SQ_GRAN_PER_COL, SQ_ROUND_STOCHASTIC, false>, grid, dim3(256), s, a);
     }
   } else {
     if (a.mode == SQ_ROUND_NEAREST_EVEN) {
-      if (fold) quantize_kernel<CodeT, SQ_GRAN_PER_ROW, SQ_ROUND_NEAREST_EVEN, true><<<grid, 256, 0, s>>>(a);
-      else quantize_kernel<CodeT, SQ_GRAN_PER_ROW, SQ_ROUND_NEAREST_EVEN, false><<<grid, 256, 0, s>>>(a);
+      if (fold) launch_pdl(quantize_kernel<CodeT, SQ_GRAN_PER_ROW, SQ_ROUND_NEAREST_EVEN, true>, grid, dim3(256), s, a);
+      else launch_pdl(quantize_kernel<CodeT, SQ_GRAN_PER_ROW, SQ_ROUND_NEAREST_EVEN, false>, grid, dim3(256), s, a);
     } else {
-      if (fold) quantize_kernel<CodeT, SQ_GRAN_PER_ROW, SQ_ROUND_STOCHASTIC, true><<<grid, 256, 0, s>>>(a);
-      else quantize_kernel<CodeT, SQ_GRAN_PER_ROW, SQ_ROUND_STOCHASTIC, false><<<grid, 256, 0, s>>>(a);
+      if (fold) launch_pdl(quantize_kernel<CodeT, SQ_GRAN_PER_ROW, SQ_ROUND_STOCHASTIC, true>, grid, dim3(256), s, a);
+      else launch_pdl(quantize_kernel<CodeT, SQ_GRAN_PER_ROW, SQ_ROUND_STOCHASTIC, false>, grid, dim3(256), s, a);
     }
   }
 }
@@ -637,10 +665,10 @@ extern "C" sq_status shiftquant_calibrate(const float* x, int64_t rows, int64_t 
   if (rblocks < 1) rblocks = 1;
   const int vec = (ld % 4 == 0) && aligned16(x);
   dim3 grid(static_cast<unsigned>(cblocks), static_cast<unsigned>(rblocks));
-  colmax_kernel<<<grid, dim3(kColTx, kColTy), 0, s>>>(
-      x, rows, cols, ld, vec, reinterpret_cast<unsigned*>(range_out), dev_status,
-      shift ? n_groups : 0, tau0_out, exp_out);
-  err = cudaGetLastError();
+  err = launch_pdl(colmax_kernel, grid, dim3(kColTx, kColTy), s, x, rows, cols, ld, vec,
+                   reinterpret_cast<unsigned*>(range_out), dev_status, shift ? n_groups : 0,
+                   tau0_out, exp_out);
+  if (err == cudaSuccess) err = cudaGetLastError();
   return err == cudaSuccess ? SQ_OK : cuda_fail(err, "colmax_kernel launch");
 }
 

@@ -34,8 +34,8 @@ EXPORTS = (
     "shiftquant_code_type", "shiftquant_code_bytes", "shiftquant_calibrate",
     "shiftquant_quantize", "shiftquant_gemm_fwd", "shiftquant_gemm_dgrad",
     "shiftquant_gemm_wgrad", "shiftquant_gemm_wgrad_static", "shiftquant_gemm_workspace_bytes",
-    "shiftquant_gemm_layer", "shiftquant_gemm_layer_workspace_bytes", "shiftquant_status_string",
-    "shiftquant_last_error",
+    "shiftquant_gemm_layer", "shiftquant_gemm_layer_workspace_bytes",
+    "shiftquant_gemm_layer_kernel_launches", "shiftquant_status_string", "shiftquant_last_error",
 )
 
 _lib = None
@@ -109,6 +109,8 @@ def load(path: str | None = None) -> ctypes.CDLL:
     lib.shiftquant_gemm_layer.restype = i32
     lib.shiftquant_gemm_layer_workspace_bytes.argtypes = [i64, i64, i64, i32, i32]
     lib.shiftquant_gemm_layer_workspace_bytes.restype = sz
+    lib.shiftquant_gemm_layer_kernel_launches.argtypes = [i64, i64, i64, i32, i32, sz]
+    lib.shiftquant_gemm_layer_kernel_launches.restype = i32
     lib.shiftquant_gemm_workspace_bytes.argtypes = [i32, i64, i64, i64, i32, i32]
     lib.shiftquant_gemm_workspace_bytes.restype = sz
     lib.shiftquant_status_string.argtypes = [i32]
@@ -254,3 +256,9 @@ def shiftquant_gemm_layer(x_codes, xt_codes, x_scale, x_exp, g_codes, gt_codes, 
 
 def shiftquant_gemm_layer_workspace_bytes(M: int, K: int, N: int, bits: int, n_groups: int) -> int:
     return int(load().shiftquant_gemm_layer_workspace_bytes(M, K, N, bits, n_groups))
+
+
+def shiftquant_gemm_layer_kernel_launches(M: int, K: int, N: int, bits: int, n_groups: int,
+                                          workspace_bytes: int) -> int:
+    return int(load().shiftquant_gemm_layer_kernel_launches(M, K, N, bits, n_groups,
+                                                            workspace_bytes))

@@ -218,3 +218,29 @@ def test_layer_gemms_equal_separate_launches():
     b = run_and_compare(x, w, dy, 6, 4, fused=False)
     for t, u in ((a.y, b.y), (a.dx, b.dx), (a.dw, b.dw)):
         np.testing.assert_array_equal(t.cpu().numpy(), u.cpu().numpy())
+
+
+@pytest.mark.parametrize("M,K,Nn,bits", [(12544, 2304, 256, 4), (4096, 64, 96, 6),
+                                         (3000, 640, 384, 6), (12608, 768, 3072, 6)])
+def test_layer_launch_count_query_matches_the_launch(M, K, Nn, bits):
+    # shiftquant_gemm_layer_kernel_launches predicts the kernels one layer call launches (the
+    # GEMM launch and one output pass per split GEMM); count them in a profiler trace
+    from torch.profiler import ProfilerActivity, profile
+    rng = np.random.default_rng(M + Nn)
+    x, w, dy = layer_inputs(rng, M, K, Nn)
+    lay = L.QuantLinear(M, K, Nn, bits, 4, "cuda")
+    lay.quantize_activation(to_gpu(x))
+    lay.quantize_gradient(to_gpu(dy), 3)
+    lay.quantize_weights(to_gpu(w))
+    torch.cuda.synchronize()
+    with profile(activities=[ProfilerActivity.CUDA]) as prof:
+        lay.gemms()
+        torch.cuda.synchronize()
+    names = [e.name for e in prof.events()]
+    ours = [n for n in names if "shiftmm_kernel" in n or "splitk_finalize_kernel" in n]
+    if not ours:
+        pytest.skip("the profiler recorded no kernels on this machine")
+    assert lay.status.item() == 0
+    want = N.shiftquant_gemm_layer_kernel_launches(M, K, Nn, bits, 4, lay.ws_layer.numel() * 4)
+    assert len(ours) == want, ours
+    assert N.shiftquant_gemm_layer_kernel_launches(M, K, Nn, bits, 4, 0) == 1
