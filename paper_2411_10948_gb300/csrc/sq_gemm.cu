@@ -579,12 +579,29 @@ __global__ void __launch_bounds__(kThreads, 1)
             uint32_t v[16];
             tmem_ld_32x32b_x16(taddr + j * 16, v);
             tmem_ld_wait();
+            // Each FP32 value is an integer of magnitude <= 2^24.  Below 2^22, adding
+            // 1.5 * 2^23 lands it in [2^23, 2^24), where the FP32 spacing is 1, so the
+            // integer is the bit pattern minus that of 1.5 * 2^23: an exact conversion on
+            // the FP32 and integer pipes.  The conversion unit (a fraction of their rate,
+            // and the limit of short chunks) takes groups holding a larger value.
+            float vmax = 0.0f;
 #pragma unroll
-            for (int i = 0; i < 16; ++i) {
-              // the FP32 value is an integer of magnitude <= 2^24: the conversion is exact
-              const int32_t t = __float2int_rn(__uint_as_float(v[i]));
-              acc[j * 16 + i] =
-                  static_cast<uint32_t>(ch == 0 ? t : static_cast<int32_t>(acc[j * 16 + i]) + t);
+            for (int i = 0; i < 16; ++i) vmax = fmaxf(vmax, fabsf(__uint_as_float(v[i])));
+            if (__all_sync(0xFFFFFFFFu, vmax < 4194304.0f)) {
+#pragma unroll
+              for (int i = 0; i < 16; ++i) {
+                const int32_t t =
+                    __float_as_int(__fadd_rn(__uint_as_float(v[i]), 12582912.0f)) - 0x4B400000;
+                acc[j * 16 + i] =
+                    static_cast<uint32_t>(ch == 0 ? t : static_cast<int32_t>(acc[j * 16 + i]) + t);
+              }
+            } else {
+#pragma unroll
+              for (int i = 0; i < 16; ++i) {
+                const int32_t t = __float2int_rn(__uint_as_float(v[i]));
+                acc[j * 16 + i] =
+                    static_cast<uint32_t>(ch == 0 ? t : static_cast<int32_t>(acc[j * 16 + i]) + t);
+              }
             }
           }
           tc_fence_before();
