@@ -641,18 +641,33 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 }
 
-// split-K: turn the summed int32 partials into the outputs
+// split-K: turn the summed int32 partials into the outputs, four consecutive outputs of a
+// row per thread (a split GEMM has N % 4 == 0); every load of a thread leaves at once
 __global__ void __launch_bounds__(256) splitk_finalize_kernel(const GemmParams p) {
   const float a_fac = epilogue_a_factor(p);
-  const int64_t total = static_cast<int64_t>(p.M) * p.N;
-  for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < total;
+  const int nq = p.N / 4;
+  const int64_t quads = static_cast<int64_t>(p.M) * nq;
+  for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < quads;
        i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
-    const int64_t row = i / p.N, col = i - row * p.N;
-    float o;
-    long long t;
-    epilogue_value(p, row, col, p.ws[i], a_fac, &o, &t);
-    p.y[row * p.ldy + col] = o;
-    if (p.acc) p.acc[row * p.ld_acc + col] = t;
+    const int64_t row = i / nq;
+    const int64_t col = (i - row * nq) * 4;
+    const int4 t4 = __ldcs(reinterpret_cast<const int4*>(p.ws) + i);
+    const int tv[4] = {t4.x, t4.y, t4.z, t4.w};
+    float o[4];
+    long long t[4];
+#pragma unroll
+    for (int e = 0; e < 4; ++e) epilogue_value(p, row, col + e, tv[e], a_fac, &o[e], &t[e]);
+    float* dst = p.y + row * p.ldy + col;
+    if (p.vec_y) {
+      *reinterpret_cast<float4*>(dst) = make_float4(o[0], o[1], o[2], o[3]);
+    } else {
+#pragma unroll
+      for (int e = 0; e < 4; ++e) dst[e] = o[e];
+    }
+    if (p.acc) {
+#pragma unroll
+      for (int e = 0; e < 4; ++e) p.acc[row * p.ld_acc + col + e] = t[e];
+    }
   }
 }
 
@@ -1042,8 +1057,8 @@ static int run_jobs(GemmJob* jobs, int njobs, int bits, int G, int32_t* dev_stat
   if (st != SQ_OK) return st;
   for (int g = 0; g < nlive; ++g) {
     if (!bt.p[g].ws) continue;
-    const int64_t total = static_cast<int64_t>(bt.p[g].M) * bt.p[g].N;
-    int64_t blocks = (total + 255) / 256;
+    const int64_t quads = static_cast<int64_t>(bt.p[g].M) * (bt.p[g].N / 4);
+    int64_t blocks = (quads + 255) / 256;
     if (blocks > static_cast<int64_t>(sms) * 16) blocks = static_cast<int64_t>(sms) * 16;
     splitk_finalize_kernel<<<static_cast<unsigned>(blocks), 256, 0, s>>>(bt.p[g]);
     err = cudaGetLastError();
