@@ -29,6 +29,8 @@ import sys
 import tempfile
 import time
 
+import numpy as np
+
 ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
@@ -163,6 +165,28 @@ class Step:
                     N.SQ_ROUND_NEAREST_EVEN, 0, lay.wd.codes, None, lay.wd.scale)),
                 ("gemm", lay.gemms),   # forward, loss propagation, weight gradient: one launch
             ]
+        return out
+
+    def call_bytes(self):
+        """(layer, tensor, algorithmic HBM bytes) of each call of calls(), in its order."""
+        out = []
+        for s, lay, gb in zip(self.specs, self.layers, self.gemm_bytes_per_launch()):
+            cb = self.N.shiftquant_code_bytes(s.bits, s.n_groups)
+            MK, MN, KN = s.M * s.K, s.M * s.N, s.K * s.N
+            out += [(s.name, "X", 4 * MK), (s.name, "X", 4 * MK + 2 * cb * MK),
+                    (s.name, "dY", 4 * MN), (s.name, "dY", 4 * MN + 2 * cb * MN),
+                    (s.name, "W per out-channel", 4 * KN), (s.name, "W per out-channel", 4 * KN + cb * KN),
+                    (s.name, "W per in-channel", 4 * KN), (s.name, "W per in-channel", 4 * KN + cb * KN),
+                    (s.name, "GEMMs", gb)]
+        return out
+
+    def group_histograms(self):
+        """Channels per group of every grouped tensor (after the last step)."""
+        out = {}
+        for s, lay in zip(self.specs, self.layers):
+            for t, q in (("X", lay.x), ("dY", lay.g)):
+                e = q.exp.cpu().numpy()
+                out[f"{s.name}:{t}"] = [int(c) for c in np.bincount(e, minlength=s.n_groups)]
         return out
 
     def launches_per_step(self) -> int:
@@ -363,6 +387,17 @@ def run_ours(args, rank, world, local_rank):
                "ms_per_step": float(et.item()) / args.steps}
     clocks = sampler.stop()
 
+    # quantizer throughput per tensor: range pass, quantize pass and both, from the breakdown
+    per_tensor = []
+    cbytes = st.call_bytes()
+    for j in range(0, len(names), 9):
+        for k in range(4):
+            (lname, tname, rb), (_, _, qb) = cbytes[j + 2 * k], cbytes[j + 2 * k + 1]
+            rms, qms = call_ms[j + 2 * k] / args.steps, call_ms[j + 2 * k + 1] / args.steps
+            per_tensor.append({"layer": lname, "tensor": tname,
+                               "range_gbs": round(rb / (rms * 1e-3) / 1e9, 1),
+                               "quantize_gbs": round(qb / (qms * 1e-3) / 1e9, 1),
+                               "both_gbs": round((rb + qb) / ((rms + qms) * 1e-3) / 1e9, 1)})
     peaks, peak_src = load_peaks()
     spec0 = wl.layers[0]
     fp8 = native.shiftquant_code_type(spec0.bits, spec0.n_groups) == native.SQ_CODE_E4M3
@@ -443,6 +478,8 @@ def run_ours(args, rank, world, local_rank):
                           nominal_hbm_gbs=7900.0, frac_nominal=q_gbs / 7900.0),
         "breakdown_ms_per_step": {k: v / args.steps for k, v in kind_ms.items()},
         "calls_ms_per_step": [[f"{n}", round(v / args.steps, 5)] for n, v in zip(names, call_ms)],
+        "quantizer_per_tensor": per_tensor,
+        "group_histograms": st.group_histograms(),
         "timing": "CUDA events around one CUDA-graph replay of the whole step (per layer: "
                   "activation chain, gradient chain and both weight roles on four streams, "
                   "then the three GEMMs as one launch); breakdown from un-graphed serial "
