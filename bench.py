@@ -261,6 +261,22 @@ def profiled_traffic(workload: str):
     return float(t.group(1))
 
 
+def max_over_ranks(value: float, device) -> float:
+    """The maximum of a per-rank float over all ranks (the value itself without a process
+    group): the slowest replica's time is the job's time."""
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([value], dtype=torch.float64, device=device)
+    if dist.is_available() and dist.is_initialized() and dist.get_world_size() > 1:
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_throughput(ops_per_step: int, world: int, steps: int, total_ms: float) -> float:
+    """Whole-job TOPS: every replica runs its own step of ops_per_step operations."""
+    return ops_per_step * world * steps / (total_ms * 1e-3) / 1e12
+
+
 def run_ours(args, rank, world, local_rank):
     import torch
     from paper_2411_10948_gb300 import build, native
@@ -348,11 +364,7 @@ def run_ours(args, rank, world, local_rank):
             call_ms[j] += d
             if n == "gemm":
                 gemm_launch_ms.append(d)
-    total_ms = sum(step_ms)
-    t = torch.tensor([total_ms], dtype=torch.float64, device=dev)
-    if world > 1:
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-    total_ms = float(t.item())
+    total_ms = max_over_ranks(sum(step_ms), dev)
     ms_per_step = total_ms / args.steps
 
     # e2e: host (pinned) -> device inputs, the captured step, device -> host outputs
@@ -379,12 +391,10 @@ def run_ours(args, rank, world, local_rank):
             b.synchronize()
             if i >= args.warmup:
                 e_ms.append(a.elapsed_time(b))
-        et = torch.tensor([sum(e_ms)], dtype=torch.float64, device=dev)
-        if world > 1:
-            torch.distributed.all_reduce(et, op=torch.distributed.ReduceOp.MAX)
-        e2e = {"value": st.gemm_ops() * world * args.steps / (float(et.item()) * 1e-3) / 1e12,
+        e_total = max_over_ranks(sum(e_ms), dev)
+        e2e = {"value": job_throughput(st.gemm_ops(), world, args.steps, e_total),
                "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
-               "ms_per_step": float(et.item()) / args.steps}
+               "ms_per_step": e_total / args.steps}
     clocks = sampler.stop()
 
     # quantizer throughput per tensor: range pass, quantize pass and both, from the breakdown
@@ -451,7 +461,7 @@ def run_ours(args, rank, world, local_rank):
 
     result = {
         "metric": METRIC,
-        "value": st.gemm_ops() * world / (ms_per_step * 1e-3) / 1e12,
+        "value": job_throughput(st.gemm_ops(), world, args.steps, total_ms),
         "unit": UNIT,
         "n_gpus": world,
         "steps": args.steps,
