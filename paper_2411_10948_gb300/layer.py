@@ -172,12 +172,14 @@ class QuantLinear:
         self.dgrad(stream)
         self.wgrad(stream)
 
-    def step_concurrent(self, x, w, dy, seed, streams):
+    def step_concurrent(self, x, w, dy, seed, streams, gemm_events=None):
         """The same step with its independent quantizer work on four streams forked from the
         current one -- the activation chain, the gradient chain and each weight role (its
         range pass right away, its quantization once the other operand's exponents exist) --
         joined back before the three GEMMs run as one launch on the current stream.
-        Capturable in a CUDA graph, which then runs the independent work concurrently."""
+        Capturable in a CUDA graph, which then runs the independent work concurrently.
+        gemm_events: optional (start, end) CUDA events recorded around the GEMM call (for
+        timing inside a captured graph they must be created with external=True)."""
         main = torch.cuda.current_stream()
         s_x, s_g, s_wf, s_wd = streams[:4]
         for s in (s_x, s_g, s_wf, s_wd):
@@ -205,7 +207,11 @@ class QuantLinear:
                                   s_wd)
         for s in (s_x, s_g, s_wf, s_wd):
             main.wait_stream(s)
+        if gemm_events is not None:
+            gemm_events[0].record(main)
         self.gemms(main)
+        if gemm_events is not None:
+            gemm_events[1].record(main)
 
     @property
     def gemm_ops(self) -> int:
