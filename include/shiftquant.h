@@ -199,6 +199,12 @@ typedef struct {
   int64_t *acc_y;  int64_t ld_acc_y;
   int64_t *acc_dx; int64_t ld_acc_dx;
   int64_t *acc_dw; int64_t ld_acc_dw;
+  /* Which GEMMs to run: bit 0 forward, bit 1 loss propagation, bit 2 weight gradient; 0 runs
+   * all three.  Fields of GEMMs left out are not read. */
+  int gemm_mask;
+  /* At most this many CTAs (0: one per SM), for a launch that shares the GPU with work
+   * running beside it on other streams. */
+  int max_ctas;
 } sq_layer_gemms;
 
 /* workspace: optional int32 scratch of shiftquant_gemm_layer_workspace_bytes() bytes,
@@ -215,12 +221,12 @@ sq_status shiftquant_gemm_layer(const sq_layer_gemms *args, void *workspace,
 size_t shiftquant_gemm_layer_workspace_bytes(int64_t M, int64_t K, int64_t N, int bits,
                                              int n_groups);
 
-/* Number of kernels one shiftquant_gemm_layer call with this shape and workspace size
- * launches on the current device: the GEMM launch, plus one output pass per GEMM that
- * splits its K loop (0 when every GEMM is empty; memsets are not counted).  -1 for invalid
- * arguments, a shape beyond the exact range, or no device. */
+/* Number of kernels one shiftquant_gemm_layer call with this shape, workspace size and
+ * gemm_mask launches on the current device: the GEMM launch, plus one output pass per GEMM
+ * that splits its K loop (0 when every GEMM is empty; memsets are not counted).  -1 for
+ * invalid arguments, a shape beyond the exact range, or no device. */
 int shiftquant_gemm_layer_kernel_launches(int64_t M, int64_t K, int64_t N, int bits,
-                                          int n_groups, size_t workspace_bytes);
+                                          int n_groups, size_t workspace_bytes, int gemm_mask);
 
 /* Weight-gradient GEMM for callers that cannot allocate device memory -- for instance a
  * plug-in running inside a host framework that owns every device allocation, or a

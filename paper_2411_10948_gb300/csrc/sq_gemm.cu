@@ -974,7 +974,7 @@ static int launch_variant(const GemmBatch& bt, int grid, int dev, cudaStream_t s
 // CTAs take their units as they free up -- for batches whose units differ in length.
 // Without one each CTA strides over the unit list.
 static int run_jobs(GemmJob* jobs, int njobs, int bits, int G, int32_t* dev_status, void* stream,
-                    int* sched) {
+                    int* sched, int max_ctas = 0) {
   cudaStream_t s = as_stream(stream);
   int live[kMaxBatch];
   int nlive = 0;
@@ -1051,7 +1051,8 @@ static int run_jobs(GemmJob* jobs, int njobs, int bits, int G, int32_t* dev_stat
                 plans[g].splits * plans[g].kb_per_split;
   }
   const bool tma_st = out_bytes > 0.2 * in_bytes;
-  const int grid = units < sms ? units : sms;
+  int grid = units < sms ? units : sms;
+  if (max_ctas > 0 && grid > max_ctas) grid = max_ctas;
   st = plans[0].elem_bytes == 1 ? launch_variant<1>(bt, grid, dev, s, multi, tma_st)
                                 : launch_variant<0>(bt, grid, dev, s, multi, tma_st);
   if (st != SQ_OK) return st;
@@ -1078,7 +1079,7 @@ static int run_gemm(int which, const void* a_codes, int64_t lda, const void* b_c
 }
 
 // The three GEMMs of a layer as jobs, workspace regions assigned to those that split.
-static void layer_jobs(const sq_layer_gemms* a, GemmJob jobs[3]) {
+static void layer_jobs(const sq_layer_gemms* a, GemmJob jobs[3], int mask) {
   jobs[0] = GemmJob{0, a->x_codes, a->ld_x, a->wf_codes, a->ld_wf, a->M, a->N, a->K, a->x_scale,
                     a->wf_scale, nullptr, nullptr, a->y, a->ld_y, a->acc_y, a->ld_acc_y, nullptr, 0};
   jobs[1] = GemmJob{1, a->g_codes, a->ld_g, a->wd_codes, a->ld_wd, a->M, a->K, a->N, a->g_scale,
@@ -1086,6 +1087,9 @@ static void layer_jobs(const sq_layer_gemms* a, GemmJob jobs[3]) {
   jobs[2] = GemmJob{2, a->xt_codes, a->ld_xt, a->gt_codes, a->ld_gt, a->K, a->N, a->M, a->x_scale,
                     a->g_scale, a->x_exp, a->g_exp, a->dw, a->ld_dw, a->acc_dw, a->ld_acc_dw,
                     nullptr, 0};
+  // a GEMM left out of the mask becomes empty: nothing of it is checked or launched
+  for (int i = 0; i < 3; ++i)
+    if (mask != 0 && !(mask & (1 << i))) jobs[i].M = 0;
 }
 
 // Bytes of split-K workspace each GEMM of the layer would use (0: it would not split),
@@ -1232,11 +1236,13 @@ extern "C" sq_status shiftquant_gemm_layer(const sq_layer_gemms* args, void* wor
   if (args == nullptr) return fail(SQ_EINVAL, "gemm_layer: args is NULL");
   if (!bits_ok(args->bits) || !groups_ok(args->n_groups))
     return fail(SQ_EINVAL, "gemm_layer: bits must be in [2, 8] and n_groups in [1, 8]");
+  if (args->gemm_mask < 0 || args->gemm_mask > 7 || args->max_ctas < 0)
+    return fail(SQ_EINVAL, "gemm_layer: gemm_mask must be in [0, 7] and max_ctas >= 0");
   GemmJob jobs[3];
-  layer_jobs(args, jobs);
+  layer_jobs(args, jobs, args->gemm_mask);
   const int sms = device_sms(nullptr);
   int* sched = assign_layer_ws(jobs, args->bits, args->n_groups, sms, workspace, workspace_bytes);
-  return run_jobs(jobs, 3, args->bits, args->n_groups, dev_status, stream, sched);
+  return run_jobs(jobs, 3, args->bits, args->n_groups, dev_status, stream, sched, args->max_ctas);
 }
 
 extern "C" size_t shiftquant_gemm_layer_workspace_bytes(int64_t M, int64_t K, int64_t N, int bits,
@@ -1250,15 +1256,18 @@ extern "C" size_t shiftquant_gemm_layer_workspace_bytes(int64_t M, int64_t K, in
   a.K = K;
   a.N = N;
   GemmJob jobs[3];
-  layer_jobs(&a, jobs);
+  layer_jobs(&a, jobs, 0);
   size_t need[3];
   layer_ws_need(jobs, bits, n_groups, sms, need);
   return kSchedBytes + need[0] + need[1] + need[2];
 }
 
 extern "C" int shiftquant_gemm_layer_kernel_launches(int64_t M, int64_t K, int64_t N, int bits,
-                                                     int n_groups, size_t workspace_bytes) {
-  if (!bits_ok(bits) || !groups_ok(n_groups) || M < 0 || K < 0 || N < 0) return -1;
+                                                     int n_groups, size_t workspace_bytes,
+                                                     int gemm_mask) {
+  if (!bits_ok(bits) || !groups_ok(n_groups) || M < 0 || K < 0 || N < 0 || gemm_mask < 0 ||
+      gemm_mask > 7)
+    return -1;
   const int sms = device_sms(nullptr);
   if (sms <= 0) return -1;
   sq_layer_gemms a;
@@ -1267,7 +1276,7 @@ extern "C" int shiftquant_gemm_layer_kernel_launches(int64_t M, int64_t K, int64
   a.K = K;
   a.N = N;
   GemmJob jobs[3];
-  layer_jobs(&a, jobs);
+  layer_jobs(&a, jobs, gemm_mask);
   // the plan looks at the workspace's size and alignment only: a stand-in address serves
   assign_layer_ws(jobs, bits, n_groups, sms, workspace_bytes ? reinterpret_cast<void*>(4096) : nullptr,
                   workspace_bytes);

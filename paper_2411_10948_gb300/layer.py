@@ -153,15 +153,19 @@ class QuantLinear:
                                 self.G, self.dw, self.acc["wgrad"] if self.acc else None,
                                 self.ws_wgrad, self.status, stream)
 
-    def gemms(self, stream=None):
-        """The three GEMMs in one persistent launch (shiftquant_gemm_layer)."""
+    def gemms(self, stream=None, gemm_mask=0, max_ctas=0, use_workspace=True):
+        """The three GEMMs in one persistent launch (shiftquant_gemm_layer); gemm_mask picks
+        a subset (bit 0 forward, 1 loss propagation, 2 weight gradient), max_ctas caps the
+        CTAs.  A launch running beside another on a different stream must not share its
+        workspace: pass use_workspace=False to one of them."""
         acc = self.acc or {}
         N.shiftquant_gemm_layer(self.x.codes, self.x.codes_t, self.x.scale, self.x.exp,
                                 self.g.codes, self.g.codes_t, self.g.scale, self.g.exp,
                                 self.wf.codes, self.wf.scale, self.wd.codes, self.wd.scale,
                                 self.M, self.K, self.N, self.bits, self.G, self.y, self.dx,
                                 self.dw, acc.get("fwd"), acc.get("dgrad"), acc.get("wgrad"),
-                                self.ws_layer, self.status, stream)
+                                self.ws_layer if use_workspace else None, self.status, stream,
+                                gemm_mask=gemm_mask, max_ctas=max_ctas)
 
     def step(self, x, w, dy, seed, stream=None):
         """One training step of the layer: every quantizer pass and all three GEMMs."""
@@ -172,14 +176,18 @@ class QuantLinear:
         self.dgrad(stream)
         self.wgrad(stream)
 
-    def step_concurrent(self, x, w, dy, seed, streams, gemm_events=None):
+    def step_concurrent(self, x, w, dy, seed, streams, gemm_events=None, dgrad_ctas=0):
         """The same step with its independent quantizer work on four streams forked from the
         current one -- the activation chain, the gradient chain and each weight role (its
         range pass right away, its quantization once the other operand's exponents exist) --
         joined back before the three GEMMs run as one launch on the current stream.
         Capturable in a CUDA graph, which then runs the independent work concurrently.
         gemm_events: optional (start, end) CUDA events recorded around the GEMM call (for
-        timing inside a captured graph they must be created with external=True)."""
+        timing inside a captured graph they must be created with external=True).
+        dgrad_ctas > 0: the loss-propagation GEMM (which needs only dY's and W's codes) runs
+        as its own launch of at most that many CTAs on the gradient stream as soon as its
+        operands exist, beside the activation chain; the forward and weight-gradient GEMMs
+        follow as one launch."""
         main = torch.cuda.current_stream()
         s_x, s_g, s_wf, s_wd = streams[:4]
         for s in (s_x, s_g, s_wf, s_wd):
@@ -205,6 +213,19 @@ class QuantLinear:
             N.shiftquant_quantize(w, N.SQ_GRAN_PER_ROW, b, G, self.wd.range, None, self.g.exp,
                                   N.SQ_ROUND_NEAREST_EVEN, 0, self.wd.codes, None, self.wd.scale,
                                   s_wd)
+        if dgrad_ctas > 0:
+            with torch.cuda.stream(s_g):
+                s_g.wait_stream(s_wd)
+                self.gemms(s_g, gemm_mask=2, max_ctas=dgrad_ctas, use_workspace=False)
+            for s in (s_x, s_wf, s_wd):
+                main.wait_stream(s)
+            if gemm_events is not None:
+                gemm_events[0].record(main)
+            self.gemms(main, gemm_mask=5)
+            if gemm_events is not None:
+                gemm_events[1].record(main)
+            main.wait_stream(s_g)
+            return
         for s in (s_x, s_g, s_wf, s_wd):
             main.wait_stream(s)
         if gemm_events is not None:

@@ -60,6 +60,7 @@ class SqLayerGemms(ctypes.Structure):
         ("acc_y", ctypes.c_void_p), ("ld_acc_y", ctypes.c_int64),
         ("acc_dx", ctypes.c_void_p), ("ld_acc_dx", ctypes.c_int64),
         ("acc_dw", ctypes.c_void_p), ("ld_acc_dw", ctypes.c_int64),
+        ("gemm_mask", ctypes.c_int), ("max_ctas", ctypes.c_int),
     ]
 
 
@@ -109,7 +110,7 @@ def load(path: str | None = None) -> ctypes.CDLL:
     lib.shiftquant_gemm_layer.restype = i32
     lib.shiftquant_gemm_layer_workspace_bytes.argtypes = [i64, i64, i64, i32, i32]
     lib.shiftquant_gemm_layer_workspace_bytes.restype = sz
-    lib.shiftquant_gemm_layer_kernel_launches.argtypes = [i64, i64, i64, i32, i32, sz]
+    lib.shiftquant_gemm_layer_kernel_launches.argtypes = [i64, i64, i64, i32, i32, sz, i32]
     lib.shiftquant_gemm_layer_kernel_launches.restype = i32
     lib.shiftquant_gemm_workspace_bytes.argtypes = [i32, i64, i64, i64, i32, i32]
     lib.shiftquant_gemm_workspace_bytes.restype = sz
@@ -234,8 +235,9 @@ def _addr(t):
 def shiftquant_gemm_layer(x_codes, xt_codes, x_scale, x_exp, g_codes, gt_codes, g_scale, g_exp,
                           wf_codes, wf_scale, wd_codes, wd_scale, M, K, N, bits, n_groups, y, dx,
                           dw, acc_y=None, acc_dx=None, acc_dw=None, workspace=None,
-                          dev_status=None, stream=None) -> None:
-    """Forward, loss-propagation and weight-gradient GEMMs of one layer in one launch."""
+                          dev_status=None, stream=None, gemm_mask=0, max_ctas=0) -> None:
+    """Forward, loss-propagation and weight-gradient GEMMs of one layer in one launch
+    (gemm_mask: bit 0 forward, 1 loss propagation, 2 weight gradient; 0 = all)."""
     a = SqLayerGemms(
         x_codes=_addr(x_codes), ld_x=_ld(x_codes), xt_codes=_addr(xt_codes), ld_xt=_ld(xt_codes),
         x_scale=_addr(x_scale), x_exp=_addr(x_exp),
@@ -247,7 +249,8 @@ def shiftquant_gemm_layer(x_codes, xt_codes, x_scale, x_exp, g_codes, gt_codes, 
         y=_addr(y), ld_y=_ld(y), dx=_addr(dx), ld_dx=_ld(dx), dw=_addr(dw), ld_dw=_ld(dw),
         acc_y=_addr(acc_y), ld_acc_y=_ld(acc_y) if acc_y is not None else 0,
         acc_dx=_addr(acc_dx), ld_acc_dx=_ld(acc_dx) if acc_dx is not None else 0,
-        acc_dw=_addr(acc_dw), ld_acc_dw=_ld(acc_dw) if acc_dw is not None else 0)
+        acc_dw=_addr(acc_dw), ld_acc_dw=_ld(acc_dw) if acc_dw is not None else 0,
+        gemm_mask=gemm_mask, max_ctas=max_ctas)
     _check(load().shiftquant_gemm_layer(
         ctypes.byref(a), _ptr(workspace),
         workspace.numel() * workspace.element_size() if workspace is not None else 0,
@@ -259,6 +262,6 @@ def shiftquant_gemm_layer_workspace_bytes(M: int, K: int, N: int, bits: int, n_g
 
 
 def shiftquant_gemm_layer_kernel_launches(M: int, K: int, N: int, bits: int, n_groups: int,
-                                          workspace_bytes: int) -> int:
+                                          workspace_bytes: int, gemm_mask: int = 0) -> int:
     return int(load().shiftquant_gemm_layer_kernel_launches(M, K, N, bits, n_groups,
-                                                            workspace_bytes))
+                                                            workspace_bytes, gemm_mask))

@@ -138,3 +138,22 @@ def test_empty_shapes_accept_null_pointers_of_empty_buffers(lib):
                                         fake if ch else None, None, None, 0, 0, None, 0, None,
                                         0, fake if ch else None, None)
             assert r != native.SQ_EINVAL, (gran, R, C, lib.shiftquant_last_error())
+
+
+def test_layer_struct_layout_matches_the_binding(tmp_path):
+    # the ctypes mirror of sq_layer_gemms must have the C struct's size and field offsets
+    import ctypes
+    from paper_2411_10948_gb300.native import SqLayerGemms
+    fields = [f for f, _ in SqLayerGemms._fields_]
+    src = tmp_path / "layout.c"
+    src.write_text('#include <stddef.h>\n#include <stdio.h>\n#include "shiftquant.h"\nint main(void) {\n'
+                   '  printf("%zu\\n", sizeof(sq_layer_gemms));\n' +
+                   "".join(f'  printf("%zu\\n", offsetof(sq_layer_gemms, {f}));\n' for f in fields) +
+                   "  return 0;\n}\n")
+    exe = tmp_path / "layout"
+    subprocess.run(["gcc", "-std=c99", "-I", os.path.join(ROOT, "include"), str(src), "-o", str(exe)],
+                   check=True)
+    out = [int(v) for v in subprocess.run([str(exe)], capture_output=True, text=True,
+                                          check=True).stdout.split()]
+    assert out[0] == ctypes.sizeof(SqLayerGemms)
+    assert out[1:] == [getattr(SqLayerGemms, f).offset for f in fields]

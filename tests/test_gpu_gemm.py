@@ -247,3 +247,48 @@ def test_layer_launch_count_query_matches_the_launch(M, K, Nn, bits):
     want = N.shiftquant_gemm_layer_kernel_launches(M, K, Nn, bits, 4, lay.ws_layer.numel() * 4)
     assert len(ours) == want, ours
     assert N.shiftquant_gemm_layer_kernel_launches(M, K, Nn, bits, 4, 0) == 1
+
+
+@pytest.mark.parametrize("mask", [1, 2, 4, 5, 6])
+def test_layer_launch_subsets_match_the_full_launch(mask):
+    # gemm_mask runs a subset of the layer's GEMMs (bit 0 forward, 1 loss propagation,
+    # 2 weight gradient); max_ctas caps the grid: each output equals the full launch's, and
+    # the outputs left out stay untouched
+    rng = np.random.default_rng(40 + mask)
+    x, w, dy = layer_inputs(rng, 2000, 700, 256)
+    full = L.QuantLinear(2000, 700, 256, 4, 4, "cuda")
+    part = L.QuantLinear(2000, 700, 256, 4, 4, "cuda")
+    for lay in (full, part):
+        lay.quantize_activation(to_gpu(x))
+        lay.quantize_gradient(to_gpu(dy), 9)
+        lay.quantize_weights(to_gpu(w))
+    full.gemms()
+    for t in (part.y, part.dx, part.dw):
+        t.fill_(-3.0)
+    part.gemms(gemm_mask=mask, max_ctas=37)
+    torch.cuda.synchronize()
+    assert full.status.item() == 0 and part.status.item() == 0
+    for bit, a, b in ((1, full.y, part.y), (2, full.dx, part.dx), (4, full.dw, part.dw)):
+        if mask & bit:
+            np.testing.assert_array_equal(a.cpu().numpy(), b.cpu().numpy())
+        else:
+            assert (b == -3.0).all()
+
+
+def test_step_with_a_separate_loss_propagation_launch_equals_the_fused_step():
+    rng = np.random.default_rng(41)
+    x, w, dy = layer_inputs(rng, 4096, 320, 192)
+    fused = L.QuantLinear(4096, 320, 192, 6, 4, "cuda", with_acc=True)
+    split = L.QuantLinear(4096, 320, 192, 6, 4, "cuda", with_acc=True)
+    xg, wg, dyg = to_gpu(x), to_gpu(w), to_gpu(dy)
+    streams = [torch.cuda.Stream() for _ in range(5)]
+    g1 = L.CapturedStep(lambda: fused.step_concurrent(xg, wg, dyg, 5, streams))
+    g2 = L.CapturedStep(lambda: split.step_concurrent(xg, wg, dyg, 5, streams, dgrad_ctas=40))
+    g1.replay()
+    g2.replay()
+    torch.cuda.synchronize()
+    assert fused.status.item() == 0 and split.status.item() == 0
+    for k in ("fwd", "dgrad", "wgrad"):
+        np.testing.assert_array_equal(fused.acc[k].cpu().numpy(), split.acc[k].cpu().numpy())
+    for a, b in ((fused.y, split.y), (fused.dx, split.dx), (fused.dw, split.dw)):
+        np.testing.assert_array_equal(a.cpu().numpy(), b.cpu().numpy())
