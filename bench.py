@@ -241,9 +241,13 @@ class Step:
 
 
 def kernel_source_hash() -> str:
+    """Hash of the GEMM kernel's device code (sq_gemm.cu up to its host-side part, and the
+    device helpers): a profile's DRAM traffic stays valid while this is unchanged."""
+    csrc = os.path.join(ROOT, "paper_2411_10948_gb300", "csrc")
+    gemm = open(os.path.join(csrc, "sq_gemm.cu"), "rb").read()
     h = hashlib.sha256()
-    for f in ("sq_gemm.cu", "sq_device.cuh"):
-        h.update(open(os.path.join(ROOT, "paper_2411_10948_gb300", "csrc", f), "rb").read())
+    h.update(gemm.split(b"// " + b"-" * 71 + b" host side")[0])
+    h.update(open(os.path.join(csrc, "sq_device.cuh"), "rb").read())
     return h.hexdigest()[:16]
 
 
