@@ -17,6 +17,8 @@
 //   warp 0      TMA producer: A and B tiles (128-byte rows, 128-byte swizzle) into a
 //               4-stage shared-memory ring
 //   warp 1      TMEM allocation and the MMA issuer (one thread)
+//   warp 2      TMA-store layout: the dequantizing column factors of each tile, ahead of
+//               the epilogue (otherwise the epilogue warps compute them themselves)
 //   warps 4-11  epilogue: tcgen05.ld, int32 accumulation across chunks, dequantizing
 //               multiply, stores (or int32 reductions into a split-K workspace)
 // Work units reach the three roles through a small shared-memory ring that the producer
@@ -45,6 +47,7 @@ constexpr int kStageBytes = kABytes + kBBytes;
 constexpr int kThreads = 384;
 constexpr int kEpiWarp0 = 4;
 constexpr int kNumEpiWarps = 8;
+constexpr int kFacWarp = 2;
 constexpr uint32_t kTmemCols = 2 * kBN;       // two FP32 accumulator buffers
 constexpr int64_t kExactSum = int64_t(1) << 24;  // every partial sum of a chunk stays within this
 // Shared memory of a CTA, in two layouts.  Plain-store mode: a 4-stage operand ring and one
@@ -63,8 +66,8 @@ struct Smem {
   static constexpr int out_offset = stages * kStageBytes;
   static constexpr int fac_offset = out_offset + kNumEpiWarps * out_bufs * kOutStageBytes;
   static constexpr int bar_offset = fac_offset + 2 * kBN * 4;
-  // full, empty, tfull, tempty, fac, drain, unit ring full / empty
-  static constexpr int num_bars = 2 * stages + 2 + 2 + 2 + 1 + 2 * kUnitRing;
+  // full, empty, tfull, tempty, fac, drain, unit ring full / empty, fac free
+  static constexpr int num_bars = 2 * stages + 2 + 2 + 2 + 1 + 2 * kUnitRing + 2;
   static constexpr int ring_offset = bar_offset + num_bars * 8 + 16;  // after TMEM slot, flag
   static constexpr size_t bytes = ring_offset + kUnitRing * 4;
   static_assert(bytes <= 232448, "shared memory beyond the 227 KB per-CTA limit");
@@ -286,6 +289,63 @@ __device__ __forceinline__ int batch_member(const GemmBatch& bt, int u, int* loc
   return g;
 }
 
+// The factor warp: the dequantizing factor of each of a tile's 256 columns, into one of
+// two tables ahead of the epilogue: s_A 2^-(G-1) s_B[n] (forward, loss propagation) or
+// s_X s_dY 2^-eY_n (weight gradient; the row's 2^-eX_m is the epilogue's).  It reads the
+// units from the same ring as the other roles; a table is refilled once every epilogue
+// warp has released it (facfree).  Kept out of line: its registers stay its own.
+__device__ __noinline__ void factor_warp(const GemmBatch& bt, int units, uint64_t* ufull,
+                                         uint64_t* uempty, volatile int* unit_ring,
+                                         uint64_t* facbar, uint64_t* facfree, float* fac_tab,
+                                         volatile int* abort_flag, int lane) {
+  bool ok = true;
+  int us = 0;
+  uint32_t uph = 0;
+  for (int it = 0; ok; ++it) {
+    if (!__all_sync(0xFFFFFFFFu, mbar_wait(&ufull[us], uph, abort_flag))) {
+      ok = false;
+      break;
+    }
+    const int u = unit_ring[us];
+    __syncwarp();
+    if (lane == 0) mbar_arrive(&uempty[us]);
+    if (++us == kUnitRing) {
+      us = 0;
+      uph ^= 1u;
+    }
+    if (u >= units) break;
+    int lu;
+    const int g = batch_member(bt, u, &lu);
+    const GemmParams& p = bt.p[g];
+    const float a_fac = epilogue_a_factor(p);
+    const int64_t n0 = static_cast<int64_t>(decode_unit(p, lu).nb) * kBN;
+    float f[kBN / 32];
+#pragma unroll
+    for (int j = 0; j < kBN / 32; ++j) {
+      const int64_t col = n0 + lane + 32 * j;
+      f[j] = 0.0f;
+      if (col < p.N)
+        f[j] = p.mode == 0 ? __fmul_rn(a_fac, __ldg(p.b_scale + col))
+                           : __fmul_rn(a_fac, pow2_neg(__ldg(p.col_exp + col)));
+    }
+    // table it & 1 last held unit it - 2: wait until the epilogue is done with it
+    if (it >= 2 &&
+        !__all_sync(0xFFFFFFFFu, mbar_wait(&facfree[it & 1], ((it >> 1) & 1) ^ 1u, abort_flag))) {
+      ok = false;
+      break;
+    }
+    float* fac = fac_tab + (it & 1) * kBN;
+#pragma unroll
+    for (int j = 0; j < kBN / 32; ++j) fac[lane + 32 * j] = f[j];
+    __syncwarp();
+    if (lane == 0) mbar_arrive(&facbar[it & 1]);
+  }
+  if (!ok && lane == 0) {
+    atomicOr(bt.status, kDevTimeout);
+    *abort_flag = 1;
+  }
+}
+
 // kTmaSt: shared-memory layout and output path (Smem<kTmaSt>)
 template <int kF8, bool kMulti, bool kTmaSt>
 __global__ void __launch_bounds__(kThreads, 1)
@@ -306,7 +366,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint64_t* drain = facbar + 2;
   uint64_t* ufull = drain + 1;
   uint64_t* uempty = ufull + kUnitRing;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(uempty + kUnitRing);
+  uint64_t* facfree = uempty + kUnitRing;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(facfree + 2);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
   volatile int* unit_ring = reinterpret_cast<volatile int*>(smem + L::ring_offset);
 
@@ -321,12 +382,15 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (int b = 0; b < 2; ++b) {
       mbar_init(&tfull[b], 1);
       mbar_init(&tempty[b], kNumEpiWarps);
-      mbar_init(&facbar[b], kNumEpiWarps);
+      // table b is filled: by the factor warp, or by the epilogue warps' shares
+      mbar_init(&facbar[b], kTmaSt ? 1 : kNumEpiWarps);
+      mbar_init(&facfree[b], kNumEpiWarps);    // every epilogue warp is done with table b
     }
     mbar_init(drain, 1);
     for (int r = 0; r < kUnitRing; ++r) {
       mbar_init(&ufull[r], 1);
-      mbar_init(&uempty[r], 1 + kNumEpiWarps);  // the MMA thread and every epilogue warp
+      // the MMA thread, the factor warp (TMA-store layout) and every epilogue warp
+      mbar_init(&uempty[r], (kTmaSt ? 2 : 1) + kNumEpiWarps);
     }
     *abort_flag = 0;
     fence_mbar_init();
@@ -482,11 +546,14 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     tc_commit(smem_u32(drain));
     mbar_wait(drain, 0, nullptr);
+  } else if (kTmaSt && warp == kFacWarp) {
+    // ---------------------------------------------------------- column factors
+    factor_warp(bt, units, ufull, uempty, unit_ring, facbar, facfree,
+                reinterpret_cast<float*>(smem + L::fac_offset), abort_flag, lane);
   } else if (warp >= kEpiWarp0) {
     // --------------------------------------------------------------- epilogue
     const int q = warp & 3;                       // TMEM lanes 32q .. 32q+31 (output rows)
     const int h = (warp - kEpiWarp0) >> 2;        // column half of the 256-wide tile
-    const int et = threadIdx.x - kEpiWarp0 * 32;  // 0 .. 255: one tile column each
     const uint32_t stage_out0 =
         smem_u32(smem + L::out_offset + (warp - kEpiWarp0) * L::out_bufs * kOutStageBytes);
     uint32_t nbox = 0;  // boxes emitted: alternates the staging buffers in TMA-store mode
@@ -513,25 +580,24 @@ __global__ void __launch_bounds__(kThreads, 1)
       const GemmParams& p = bt.p[g];
       const CUtensorMap* tma_y = &bt.y[g];
       const CUtensorMap* tma_ws = &bt.ws[g];
-      const float a_fac = epilogue_a_factor(p);
       const Unit w = decode_unit(p, lu);
       const int nch = (w.kb1 - w.kb0 + p.chunk_kb - 1) / p.chunk_kb;
       const int64_t m0 = static_cast<int64_t>(w.mb) * kBM;
       const int64_t n0 = static_cast<int64_t>(w.nb) * kBN;
-      // the dequantizing factor of each of the tile's 256 columns, computed once per tile
-      // while the tensor core works: s_A 2^-(G-1) s_B[n] (forward, loss propagation) or
-      // s_X s_dY 2^-eY_n (weight gradient; the row's 2^-eX_m is applied separately)
       float* fac = fac_tab + (it & 1) * kBN;
-      {
+      if constexpr (!kTmaSt) {
+        // this thread's column of the table: written once the warps that read the table
+        // two units ago are past it (facbar of the last unit needed every warp to arrive)
+        const int et = threadIdx.x - kEpiWarp0 * 32;
         const int64_t col = n0 + et;
         float f = 0.0f;
         if (col < p.N)
-          f = p.mode == 0 ? __fmul_rn(a_fac, __ldg(p.b_scale + col))
-                          : __fmul_rn(a_fac, pow2_neg(__ldg(p.col_exp + col)));
+          f = p.mode == 0 ? __fmul_rn(epilogue_a_factor(p), __ldg(p.b_scale + col))
+                          : __fmul_rn(epilogue_a_factor(p), pow2_neg(__ldg(p.col_exp + col)));
         fac[et] = f;
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&facbar[it & 1]);
       }
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&facbar[it & 1]);
 
       const int64_t row0 = m0 + q * 32;
       const int64_t row = row0 + lane;
@@ -562,6 +628,10 @@ __global__ void __launch_bounds__(kThreads, 1)
           const uint32_t buf = stage_out0 + (nbox++ % L::out_bufs) * kOutStageBytes;
           emit_box<kTmaSt>(p, tma_y, tma_ws, v, true, smem_u32(fac + h * 128 + s * 32), rfac, buf, row0,
                            col0, lane);
+        }
+        if constexpr (kTmaSt) {
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&facfree[it & 1]);  // this warp is done with the table
         }
         ++c;
       } else {
@@ -624,6 +694,10 @@ __global__ void __launch_bounds__(kThreads, 1)
           const uint32_t buf = stage_out0 + (nbox++ % L::out_bufs) * kOutStageBytes;
           emit_box<kTmaSt>(p, tma_y, tma_ws, v, false, smem_u32(fac + h * 128 + s * 32), rfac, buf, row0,
                            col0, lane);
+        }
+        if constexpr (kTmaSt) {
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&facfree[it & 1]);  // this warp is done with the table
         }
       }
     }
