@@ -12,13 +12,20 @@
 // The ShiftMM shift 2^(G-1-e_k) of inner index k is already inside the weight codes
 // (the quantizer folds it in), so the tensor core applies it to every product before
 // accumulation at no cost, exactly as ShiftMM prescribes (Sec. 3.2).
+// Chunk length: the worst case assumes the largest shift on every inner index.  Where the
+// inner channels' exponents are given (the layer launch), warp 2 of every CTA bounds the
+// shifts per K block from them at the start, and the chunks take as many K blocks as
+// max|q_A| max|q_B| x (largest per-block shift sum) x blocks <= 2^24 allows; with most
+// channels in the last group (the usual case: tau_0 set by a few outlier channels) an
+// 8-bit chunk grows from 2 K blocks to about 10.
 //
 // One CTA per SM, persistent over output tiles of 128 x 256:
 //   warp 0      TMA producer: A and B tiles (128-byte rows, 128-byte swizzle) into a
 //               4-stage shared-memory ring
 //   warp 1      TMEM allocation and the MMA issuer (one thread)
-//   warp 2      TMA-store layout: the dequantizing column factors of each tile, ahead of
-//               the epilogue (otherwise the epilogue warps compute them themselves)
+//   warp 2      the chunk plan (see above); then, in the TMA-store layout, the
+//               dequantizing column factors of each tile ahead of the epilogue (otherwise
+//               the epilogue warps compute them themselves)
 //   warps 4-11  epilogue: tcgen05.ld, int32 accumulation across chunks, dequantizing
 //               multiply, stores (or int32 reductions into a split-K workspace)
 // Work units reach the three roles through a small shared-memory ring that the producer
@@ -47,7 +54,7 @@ constexpr int kStageBytes = kABytes + kBBytes;
 constexpr int kThreads = 384;
 constexpr int kEpiWarp0 = 4;
 constexpr int kNumEpiWarps = 8;
-constexpr int kFacWarp = 2;
+constexpr int kFacWarp = 2;   // chunk plan, then the column factors
 constexpr uint32_t kTmemCols = 2 * kBN;       // two FP32 accumulator buffers
 constexpr int64_t kExactSum = int64_t(1) << 24;  // every partial sum of a chunk stays within this
 // Shared memory of a CTA, in two layouts.  Plain-store mode: a 4-stage operand ring and one
@@ -66,10 +73,11 @@ struct Smem {
   static constexpr int out_offset = stages * kStageBytes;
   static constexpr int fac_offset = out_offset + kNumEpiWarps * out_bufs * kOutStageBytes;
   static constexpr int bar_offset = fac_offset + 2 * kBN * 4;
-  // full, empty, tfull, tempty, fac, drain, unit ring full / empty, fac free
-  static constexpr int num_bars = 2 * stages + 2 + 2 + 2 + 1 + 2 * kUnitRing + 2;
+  // full, empty, tfull, tempty, fac, drain, unit ring full / empty, fac free, chunk plan
+  static constexpr int num_bars = 2 * stages + 2 + 2 + 2 + 1 + 2 * kUnitRing + 2 + 1;
   static constexpr int ring_offset = bar_offset + num_bars * 8 + 16;  // after TMEM slot, flag
-  static constexpr size_t bytes = ring_offset + kUnitRing * 4;
+  static constexpr int chunk_offset = ring_offset + kUnitRing * 4;  // K blocks per chunk, per GEMM
+  static constexpr size_t bytes = chunk_offset + 4 * 4;
   static_assert(bytes <= 232448, "shared memory beyond the 227 KB per-CTA limit");
   static_assert(out_offset % 1024 == 0 && kOutStageBytes % 1024 == 0, "swizzle atoms need 1 KB");
 };
@@ -105,6 +113,11 @@ struct GemmBatch {
   int unit_end[kMaxBatch];  // cumulative unit counts
   int count;
   int* sched;  // unit counter (zero before launch) for dynamic scheduling, or null
+  // per GEMM: exponents e_k of the inner channels (forward, loss propagation; null:
+  // worst-case chunks) and the bound max|q_A| max|q_B| of an unshifted product
+  const uint8_t* k_exp[kMaxBatch];
+  int raw_prod[kMaxBatch];
+  int planned;  // some GEMM sizes its chunks from exponents (warp 2 plans them)
   int* status;
 };
 
@@ -346,6 +359,73 @@ __device__ __noinline__ void factor_warp(const GemmBatch& bt, int units, uint64_
   }
 }
 
+// The chunk length (K blocks) of every GEMM of the batch, into out[g], by one warp.  With
+// the inner channels' exponents, a K block of channels c contributes products of at most
+// raw_prod x sum_c 2^(G-1-e_c); the chunk takes as many blocks as keep the largest such
+// sum times the block count within 2^24.  Never shorter than the worst-case chunk.
+// block: inner elements per K block (128 bytes of codes: 64 or 128).  The exponents are
+// read 16 at a time, four 16-byte loads of a lane in flight together.
+__device__ __forceinline__ unsigned shift_weight(uint32_t word, int G, int64_t c, int64_t K) {
+  unsigned w = 0;
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const int e = (word >> (8 * i)) & 0xFF;
+    if (c + i < K) w += 1u << (e >= G ? G - 1 : G - 1 - e);  // out of range: the largest shift
+  }
+  return w;
+}
+
+__device__ __noinline__ void plan_chunks(const GemmBatch& bt, volatile int* out, int lane,
+                                         int block) {
+  for (int g = 0; g < bt.count; ++g) {
+    const GemmParams& p = bt.p[g];
+    int chunk = p.chunk_kb;
+    const uint8_t* k_exp = bt.k_exp[g];
+    if (k_exp != nullptr) {
+      const int spb = block / 16;                      // 16-channel segments per block
+      const int64_t nseg = (static_cast<int64_t>(p.K) + 15) / 16;
+      const bool vec = (reinterpret_cast<uintptr_t>(k_exp) & 15) == 0;
+      unsigned wmax = 0;
+      // 32 lanes cover 32 consecutive segments = 32 / spb whole blocks per round
+      for (int64_t s0 = 0; s0 < nseg; s0 += 4 * 32) {
+        unsigned wseg[4];
+#pragma unroll
+        for (int r = 0; r < 4; ++r) {
+          const int64_t sg = s0 + r * 32 + lane;
+          const int64_t c = sg * 16;
+          uint32_t wd[4] = {0u, 0u, 0u, 0u};
+          if (sg < nseg) {
+            if (vec && c + 16 <= p.K) {
+              const uint4 v = __ldg(reinterpret_cast<const uint4*>(k_exp + c));
+              wd[0] = v.x; wd[1] = v.y; wd[2] = v.z; wd[3] = v.w;
+            } else {
+              for (int i = 0; i < 16 && c + i < p.K; ++i)
+                wd[i >> 2] |= static_cast<uint32_t>(__ldg(k_exp + c + i)) << (8 * (i & 3));
+            }
+          }
+          unsigned w = 0;
+#pragma unroll
+          for (int q = 0; q < 4; ++q) w += sg < nseg ? shift_weight(wd[q], p.G, c + 4 * q, p.K) : 0u;
+          wseg[r] = w;
+        }
+#pragma unroll
+        for (int r = 0; r < 4; ++r) {
+          unsigned w = wseg[r];
+          for (int o = 1; o < spb; o <<= 1) w += __shfl_xor_sync(0xFFFFFFFFu, w, o);
+          wmax = max(wmax, w);   // every lane of a block's group holds the block's sum
+        }
+      }
+      wmax = __reduce_max_sync(0xFFFFFFFFu, wmax);
+      if (wmax > 0) {
+        int64_t l = kExactSum / (static_cast<int64_t>(bt.raw_prod[g]) * wmax);
+        if (l > (1 << 20)) l = 1 << 20;
+        if (l > chunk) chunk = static_cast<int>(l);
+      }
+    }
+    if (lane == 0) out[g] = chunk;
+  }
+}
+
 // kTmaSt: shared-memory layout and output path (Smem<kTmaSt>)
 template <int kF8, bool kMulti, bool kTmaSt>
 __global__ void __launch_bounds__(kThreads, 1)
@@ -367,7 +447,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint64_t* ufull = drain + 1;
   uint64_t* uempty = ufull + kUnitRing;
   uint64_t* facfree = uempty + kUnitRing;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(facfree + 2);
+  uint64_t* chunkbar = facfree + 2;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(chunkbar + 1);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
   volatile int* unit_ring = reinterpret_cast<volatile int*>(smem + L::ring_offset);
 
@@ -387,6 +468,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(&facfree[b], kNumEpiWarps);    // every epilogue warp is done with table b
     }
     mbar_init(drain, 1);
+    mbar_init(chunkbar, 1);  // warp 2 has set the chunk length of every GEMM
     for (int r = 0; r < kUnitRing; ++r) {
       mbar_init(&ufull[r], 1);
       // the MMA thread, the factor warp (TMA-store layout) and every epilogue warp
@@ -483,7 +565,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     int s = 0;
     uint32_t ph = 0;
     uint32_t c = 0;
-    bool ok = true;
+    bool ok = !bt.planned || mbar_wait(chunkbar, 0, abort_flag);  // the chunk plan is in
     int us = 0;
     uint32_t uph = 0;
     while (ok) {
@@ -500,7 +582,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (u >= units) break;
       int lu;
       const int g = batch_member(bt, u, &lu);
-      const int chunk_kb = bt.p[g].chunk_kb;
+      const int chunk_kb =
+          bt.planned ? reinterpret_cast<volatile int*>(smem + L::chunk_offset)[g] : bt.p[g].chunk_kb;
       const Unit w = decode_unit(bt.p[g], lu);
       for (int kc = w.kb0; kc < w.kb1 && ok; kc += chunk_kb) {
         const int kce = min(w.kb1, kc + chunk_kb);
@@ -546,10 +629,16 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     tc_commit(smem_u32(drain));
     mbar_wait(drain, 0, nullptr);
-  } else if (kTmaSt && warp == kFacWarp) {
-    // ---------------------------------------------------------- column factors
-    factor_warp(bt, units, ufull, uempty, unit_ring, facbar, facfree,
-                reinterpret_cast<float*>(smem + L::fac_offset), abort_flag, lane);
+  } else if (warp == kFacWarp) {
+    // --------------------------------------------------- chunk plan, column factors
+    if (bt.planned) {
+      plan_chunks(bt, reinterpret_cast<volatile int*>(smem + L::chunk_offset), lane, kBKElems);
+      __syncwarp();
+      if (lane == 0) mbar_arrive(chunkbar);
+    }
+    if constexpr (kTmaSt)
+      factor_warp(bt, units, ufull, uempty, unit_ring, facbar, facfree,
+                  reinterpret_cast<float*>(smem + L::fac_offset), abort_flag, lane);
   } else if (warp >= kEpiWarp0) {
     // --------------------------------------------------------------- epilogue
     const int q = warp & 3;                       // TMEM lanes 32q .. 32q+31 (output rows)
@@ -559,7 +648,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint32_t nbox = 0;  // boxes emitted: alternates the staging buffers in TMA-store mode
     float* fac_tab = reinterpret_cast<float*>(smem + L::fac_offset);
     uint32_t c = 0;
-    bool ok = true;
+    bool ok = !bt.planned || __all_sync(0xFFFFFFFFu, mbar_wait(chunkbar, 0, abort_flag));
     int us = 0;
     uint32_t uph = 0;
     for (int it = 0; ok; ++it) {
@@ -581,7 +670,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       const CUtensorMap* tma_y = &bt.y[g];
       const CUtensorMap* tma_ws = &bt.ws[g];
       const Unit w = decode_unit(p, lu);
-      const int nch = (w.kb1 - w.kb0 + p.chunk_kb - 1) / p.chunk_kb;
+      const int ckb =
+          bt.planned ? reinterpret_cast<volatile int*>(smem + L::chunk_offset)[g] : p.chunk_kb;
+      const int nch = (w.kb1 - w.kb0 + ckb - 1) / ckb;
       const int64_t m0 = static_cast<int64_t>(w.mb) * kBM;
       const int64_t n0 = static_cast<int64_t>(w.nb) * kBN;
       float* fac = fac_tab + (it & 1) * kBN;
@@ -899,6 +990,7 @@ struct GemmJob {
   int64_t ld_acc;
   void* ws;
   size_t ws_bytes;
+  const uint8_t* k_exp;  // exponents of the inner channels (forward, loss propagation), or null
 };
 
 static const char* job_name(int which) {
@@ -985,7 +1077,7 @@ static int balance_splits(GemmJob* const* jobs, int n, int bits, int G, int sms,
 }
 
 // Slot g of the batch for one planned GEMM: tensor maps and parameters.
-static int prepare_job(const GemmJob& j, const Plan* pl, int G, int32_t* dev_status,
+static int prepare_job(const GemmJob& j, const Plan* pl, int bits, int G, int32_t* dev_status,
                        GemmBatch* bt, int g) {
   int st;
   const int eb = pl->elem_bytes;
@@ -1001,6 +1093,10 @@ static int prepare_job(const GemmJob& j, const Plan* pl, int G, int32_t* dev_sta
   p.kb_total = pl->kb_total;
   p.kb_per_split = pl->kb_per_split;
   p.chunk_kb = pl->chunk_kb;
+  // exponent-sized chunks pay where worst-case chunks would split a unit three ways or more
+  // (8-bit); elsewhere the planning only costs time
+  bt->k_exp[g] = (j.which == 2 || pl->kb_per_split <= 2 * pl->chunk_kb) ? nullptr : j.k_exp;
+  bt->raw_prod[g] = q_of_bits(bits) * q_of_bits(bits);
   p.mode = j.which == 2 ? 1 : 0;
   p.G = G;
   p.vec_y = (j.ldy % 4 == 0) && aligned16(j.y);
@@ -1074,7 +1170,7 @@ static int run_jobs(GemmJob* jobs, int njobs, int bits, int G, int32_t* dev_stat
   int st = balance_splits(lj, nlive, bits, G, sms, plans);
   if (st != SQ_OK) return st;
   for (int g = 0; g < nlive; ++g)
-    if ((st = prepare_job(*lj[g], &plans[g], G, dev_status, &bt, g)) != SQ_OK) return st;
+    if ((st = prepare_job(*lj[g], &plans[g], bits, G, dev_status, &bt, g)) != SQ_OK) return st;
   // longest K loop per unit first: the short units then fill in behind the long ones
   for (int a = 0; a < nlive; ++a)
     for (int b = a + 1; b < nlive; ++b)
@@ -1086,6 +1182,8 @@ static int run_jobs(GemmJob* jobs, int njobs, int bits, int G, int32_t* dev_stat
         t = bt.b[a]; bt.b[a] = bt.b[b]; bt.b[b] = t;
         t = bt.y[a]; bt.y[a] = bt.y[b]; bt.y[b] = t;
         t = bt.ws[a]; bt.ws[a] = bt.ws[b]; bt.ws[b] = t;
+        const uint8_t* te = bt.k_exp[a]; bt.k_exp[a] = bt.k_exp[b]; bt.k_exp[b] = te;
+        const int tr = bt.raw_prod[a]; bt.raw_prod[a] = bt.raw_prod[b]; bt.raw_prod[b] = tr;
       }
   int units = 0;
   bool multi = false;
@@ -1097,6 +1195,8 @@ static int run_jobs(GemmJob* jobs, int njobs, int bits, int G, int32_t* dev_stat
   bt.count = nlive;
   bt.status = dev_status;
   bt.sched = sched;
+  bt.planned = 0;
+  for (int g = 0; g < nlive; ++g) bt.planned |= bt.k_exp[g] != nullptr;
   // zero the counter and the partial sums, with one memset for the regions that follow the
   // counter back to back
   char* zero_from = reinterpret_cast<char*>(sched);
@@ -1164,6 +1264,8 @@ static void layer_jobs(const sq_layer_gemms* a, GemmJob jobs[3], int mask) {
   jobs[2] = GemmJob{2, a->xt_codes, a->ld_xt, a->gt_codes, a->ld_gt, a->K, a->N, a->M, a->x_scale,
                     a->g_scale, a->x_exp, a->g_exp, a->dw, a->ld_dw, a->acc_dw, a->ld_acc_dw,
                     nullptr, 0};
+  jobs[0].k_exp = a->x_exp;  // the forward GEMM's inner channels are X's
+  jobs[1].k_exp = a->g_exp;  // loss propagation's are dY's
   // a GEMM left out of the mask becomes empty: nothing of it is checked or launched
   for (int i = 0; i < 3; ++i)
     if (mask != 0 && !(mask & (1 << i))) jobs[i].M = 0;

@@ -232,6 +232,11 @@ def _addr(t):
     return t.data_ptr() if t is not None else None
 
 
+def _ld_opt(t) -> int:
+    """Leading dimension of an optional matrix (0 when absent)."""
+    return _ld(t) if t is not None else 0
+
+
 def shiftquant_gemm_layer(x_codes, xt_codes, x_scale, x_exp, g_codes, gt_codes, g_scale, g_exp,
                           wf_codes, wf_scale, wd_codes, wd_scale, M, K, N, bits, n_groups, y, dx,
                           dw, acc_y=None, acc_dx=None, acc_dw=None, workspace=None,
@@ -239,17 +244,17 @@ def shiftquant_gemm_layer(x_codes, xt_codes, x_scale, x_exp, g_codes, gt_codes, 
     """Forward, loss-propagation and weight-gradient GEMMs of one layer in one launch
     (gemm_mask: bit 0 forward, 1 loss propagation, 2 weight gradient; 0 = all)."""
     a = SqLayerGemms(
-        x_codes=_addr(x_codes), ld_x=_ld(x_codes), xt_codes=_addr(xt_codes), ld_xt=_ld(xt_codes),
-        x_scale=_addr(x_scale), x_exp=_addr(x_exp),
-        g_codes=_addr(g_codes), ld_g=_ld(g_codes), gt_codes=_addr(gt_codes), ld_gt=_ld(gt_codes),
-        g_scale=_addr(g_scale), g_exp=_addr(g_exp),
-        wf_codes=_addr(wf_codes), ld_wf=_ld(wf_codes), wf_scale=_addr(wf_scale),
-        wd_codes=_addr(wd_codes), ld_wd=_ld(wd_codes), wd_scale=_addr(wd_scale),
+        x_codes=_addr(x_codes), ld_x=_ld_opt(x_codes), xt_codes=_addr(xt_codes),
+        ld_xt=_ld_opt(xt_codes), x_scale=_addr(x_scale), x_exp=_addr(x_exp),
+        g_codes=_addr(g_codes), ld_g=_ld_opt(g_codes), gt_codes=_addr(gt_codes),
+        ld_gt=_ld_opt(gt_codes), g_scale=_addr(g_scale), g_exp=_addr(g_exp),
+        wf_codes=_addr(wf_codes), ld_wf=_ld_opt(wf_codes), wf_scale=_addr(wf_scale),
+        wd_codes=_addr(wd_codes), ld_wd=_ld_opt(wd_codes), wd_scale=_addr(wd_scale),
         M=M, K=K, N=N, bits=bits, n_groups=n_groups,
-        y=_addr(y), ld_y=_ld(y), dx=_addr(dx), ld_dx=_ld(dx), dw=_addr(dw), ld_dw=_ld(dw),
-        acc_y=_addr(acc_y), ld_acc_y=_ld(acc_y) if acc_y is not None else 0,
-        acc_dx=_addr(acc_dx), ld_acc_dx=_ld(acc_dx) if acc_dx is not None else 0,
-        acc_dw=_addr(acc_dw), ld_acc_dw=_ld(acc_dw) if acc_dw is not None else 0,
+        y=_addr(y), ld_y=_ld_opt(y), dx=_addr(dx), ld_dx=_ld_opt(dx), dw=_addr(dw),
+        ld_dw=_ld_opt(dw), acc_y=_addr(acc_y), ld_acc_y=_ld_opt(acc_y),
+        acc_dx=_addr(acc_dx), ld_acc_dx=_ld_opt(acc_dx),
+        acc_dw=_addr(acc_dw), ld_acc_dw=_ld_opt(acc_dw),
         gemm_mask=gemm_mask, max_ctas=max_ctas)
     _check(load().shiftquant_gemm_layer(
         ctypes.byref(a), _ptr(workspace),

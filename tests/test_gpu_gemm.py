@@ -292,3 +292,38 @@ def test_step_with_a_separate_loss_propagation_launch_equals_the_fused_step():
         np.testing.assert_array_equal(fused.acc[k].cpu().numpy(), split.acc[k].cpu().numpy())
     for a, b in ((fused.y, split.y), (fused.dx, split.dx), (fused.dw, split.dw)):
         np.testing.assert_array_equal(a.cpu().numpy(), b.cpu().numpy())
+
+
+@pytest.mark.parametrize("bits,G,K", [(8, 4, 5000), (6, 4, 9000), (4, 4, 30000), (8, 3, 3000)])
+def test_layer_chunks_from_exponents_stay_exact(bits, G, K):
+    # The layer launch sizes its exact FP32 chunks from the inner channels' exponents.
+    # Codes at the largest magnitude with one sign per row, a few channels in group 0 (the
+    # largest fold) among many in the last group, and odd products mixed in: every chunk's
+    # partial sums reach the bound, and an off-by-one chunk would round away odd terms.
+    Q = 2 ** (bits - 1) - 1
+    M, Nn = 130, 260
+    rng = np.random.default_rng(K + bits)
+    e = np.full(K, G - 1, np.int64)
+    e[::17] = 0
+    e[5::41] = 1
+    A = np.full((M, K), Q, np.int64)
+    A[1::2] *= -1
+    A[3] = rng.integers(-Q, Q + 1, K)
+    Bq = np.where((np.arange(K)[None, :] + np.arange(Nn)[:, None]) % 3 == 0, Q, Q - 1)
+    Bq[9] = rng.integers(-Q, Q + 1, K)
+    Bf = Bq.astype(np.int64) << (G - 1 - e)[None, :]
+    a, b = _encode(A, bits, G), _encode(Bf, bits, G)
+    xe = torch.from_numpy(e.astype(np.uint8)).cuda()
+    one = torch.ones(1, device="cuda")
+    ones = torch.ones(Nn, device="cuda")
+    y = torch.zeros((M, Nn), device="cuda")
+    acc = torch.zeros((M, Nn), dtype=torch.int64, device="cuda")
+    st = torch.zeros(1, dtype=torch.int32, device="cuda")
+    N.shiftquant_gemm_layer(a, None, one, xe, None, None, None, None, b, ones, None, None,
+                            M, K, Nn, bits, G, y, None, None, acc_y=acc, dev_status=st,
+                            gemm_mask=1)
+    torch.cuda.synchronize()
+    assert st.item() == 0
+    T = A @ Bf.T
+    np.testing.assert_array_equal(acc.cpu().numpy(), T)
+    assert_close_f32(y.cpu().numpy(), T.astype(np.float64) * 2.0 ** -(G - 1), "Y")
