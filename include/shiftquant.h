@@ -181,7 +181,12 @@ sq_status shiftquant_gemm_wgrad(const void *xt_codes, int64_t ldx, const float *
  *   weight gradient    dw [K, N] from xt_codes [K, M] and gt_codes [N, M] with the exponents
  *                      x_exp[K], g_exp[N] and the scales x_scale, g_scale
  * acc_* are the optional int64 exactness-check outputs.  The struct lives in host memory and
- * is read during the call only. */
+ * is read during the call only.
+ * The launch sizes the exact FP32 accumulation chunks of the forward and loss-propagation
+ * GEMMs from x_exp and g_exp (a K block's products are bounded by max|q|^2 times its
+ * channels' shifts): wf_codes and wd_codes must carry exactly the shifts 2^(G-1-e) of those
+ * exponents, as shiftquant_quantize with fold_exp = x_exp / g_exp writes them, and every
+ * code magnitude must be at most Q = 2^(bits-1) - 1. */
 typedef struct {
   const void *x_codes;  int64_t ld_x;
   const void *xt_codes; int64_t ld_xt;
