@@ -23,11 +23,12 @@
 //   warp 0      TMA producer: A and B tiles (128-byte rows, 128-byte swizzle) into a
 //               4-stage shared-memory ring
 //   warp 1      TMEM allocation and the MMA issuer (one thread)
-//   warp 2      the chunk plan (see above); then, in the TMA-store layout, the
-//               dequantizing column factors of each tile ahead of the epilogue (otherwise
-//               the epilogue warps compute them themselves)
+//   warp 2      the chunk plan (see above); then the dequantizing column factors of each
+//               tile, ahead of the epilogue
 //   warps 4-11  epilogue: tcgen05.ld, int32 accumulation across chunks, dequantizing
-//               multiply, stores (or int32 reductions into a split-K workspace)
+//               multiply, TMA stores of 32 x 32 boxes (or int32 TMA reductions into a
+//               split-K workspace; plain stores where the output rows are not 16-byte
+//               aligned)
 // Work units reach the three roles through a small shared-memory ring that the producer
 // fills: with a scheduling counter the producer takes each next unit from it (units are
 // handed out in list order as CTAs free up), without one it strides over the list.
@@ -57,21 +58,22 @@ constexpr int kNumEpiWarps = 8;
 constexpr int kFacWarp = 2;   // chunk plan, then the column factors
 constexpr uint32_t kTmemCols = 2 * kBN;       // two FP32 accumulator buffers
 constexpr int64_t kExactSum = int64_t(1) << 24;  // every partial sum of a chunk stays within this
-// Shared memory of a CTA, in two layouts.  Plain-store mode: a 4-stage operand ring and one
-// 32 x 32 output staging box per epilogue warp (the box turns the lane-per-row TMEM layout
-// into row-contiguous stores).  TMA-store mode, for launches whose outputs outweigh their
-// operands: a 3-stage ring and two staging boxes per warp, so one box is written while TMA
-// stores the other.  Then two per-tile column-factor tables, the barriers and the unit ring.
+// Shared memory of a CTA: a 4-stage operand ring, one 32 x 32 output staging box per
+// epilogue warp (the box turns the lane-per-row TMEM layout into row-contiguous stores, or
+// is the source of a TMA store), two per-tile column-factor tables, the barriers and the
+// unit ring.  Four stages hold about 1.3 us of MMA work at the tensor cores' rate; an
+// operand tile fetched from HBM while other SMs stream outputs takes longer than 1 us to
+// land, so a ring of three stages left the MMA waiting (two staging boxes per warp with
+// three stages measured 8-13% slower on MMA-bound layer launches and no faster on an
+// output-bound one).
 constexpr int kOutBox = 32;
 constexpr int kUnitRing = 8;  // work units published by the producer ahead of the consumers
 constexpr int kOutStageBytes = kOutBox * kOutBox * 4;
 
-template <bool kTmaSt>
 struct Smem {
-  static constexpr int stages = kTmaSt ? 3 : 4;
-  static constexpr int out_bufs = kTmaSt ? 2 : 1;
+  static constexpr int stages = 4;
   static constexpr int out_offset = stages * kStageBytes;
-  static constexpr int fac_offset = out_offset + kNumEpiWarps * out_bufs * kOutStageBytes;
+  static constexpr int fac_offset = out_offset + kNumEpiWarps * kOutStageBytes;
   static constexpr int bar_offset = fac_offset + 2 * kBN * 4;
   // full, empty, tfull, tempty, fac, drain, unit ring full / empty, fac free, chunk plan
   static constexpr int num_bars = 2 * stages + 2 + 2 + 2 + 1 + 2 * kUnitRing + 2 + 1;
@@ -107,7 +109,7 @@ constexpr int kMaxBatch = 3;
 struct GemmBatch {
   CUtensorMap a[kMaxBatch];
   CUtensorMap b[kMaxBatch];
-  CUtensorMap y[kMaxBatch];   // fp32 output maps (TMA-store mode, aligned outputs)
+  CUtensorMap y[kMaxBatch];   // fp32 output maps (outputs with 16-byte aligned rows)
   CUtensorMap ws[kMaxBatch];  // split-K workspace maps (unused when a GEMM does not split)
   GemmParams p[kMaxBatch];
   int unit_end[kMaxBatch];  // cumulative unit counts
@@ -178,16 +180,13 @@ __device__ __noinline__ void write_acc_box(long long* acc, int64_t ld_acc, int64
 // row-contiguous 16-byte stores (eight lanes per 128-byte row, four rows per instruction),
 // or as int32 partial sums through a TMA reduce-add into the split-K workspace.  The
 // exactness-check integers are written when asked.
-template <bool kTmaSt>
 __device__ __forceinline__ void emit_box(const GemmParams& p, const CUtensorMap* tma_y,
                                          const CUtensorMap* tma_ws, const uint32_t (&vals)[32],
                                          bool as_float, uint32_t fac, float rfac, uint32_t buf,
                                          int64_t row0, int64_t col0, int lane) {
-  const bool tma_out = p.ws != nullptr || (kTmaSt && p.vec_y);
+  const bool tma_out = p.ws != nullptr || p.vec_y;
   if (tma_out && lane == 0) {
-    // in TMA-store mode the box two stores back used this buffer; otherwise the last one
-    if (kTmaSt) bulk_wait_read<1>();
-    else bulk_wait_read<0>();
+    bulk_wait_read<0>();  // the last TMA store has read the box
   }
   __syncwarp();
   if (p.acc != nullptr && p.ws == nullptr) {
@@ -426,11 +425,10 @@ __device__ __noinline__ void plan_chunks(const GemmBatch& bt, volatile int* out,
   }
 }
 
-// kTmaSt: shared-memory layout and output path (Smem<kTmaSt>)
-template <int kF8, bool kMulti, bool kTmaSt>
+template <int kF8, bool kMulti>
 __global__ void __launch_bounds__(kThreads, 1)
     shiftmm_kernel(const __grid_constant__ GemmBatch bt) {
-  using L = Smem<kTmaSt>;
+  using L = Smem;
   constexpr int kStages = L::stages;
   extern __shared__ __align__(1024) uint8_t smem[];
   if ((smem_u32(smem) & 1023u) != 0) {  // the swizzled layouts need 1 KB alignment
@@ -463,16 +461,15 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (int b = 0; b < 2; ++b) {
       mbar_init(&tfull[b], 1);
       mbar_init(&tempty[b], kNumEpiWarps);
-      // table b is filled: by the factor warp, or by the epilogue warps' shares
-      mbar_init(&facbar[b], kTmaSt ? 1 : kNumEpiWarps);
+      mbar_init(&facbar[b], 1);                // the factor warp has filled table b
       mbar_init(&facfree[b], kNumEpiWarps);    // every epilogue warp is done with table b
     }
     mbar_init(drain, 1);
     mbar_init(chunkbar, 1);  // warp 2 has set the chunk length of every GEMM
     for (int r = 0; r < kUnitRing; ++r) {
       mbar_init(&ufull[r], 1);
-      // the MMA thread, the factor warp (TMA-store layout) and every epilogue warp
-      mbar_init(&uempty[r], (kTmaSt ? 2 : 1) + kNumEpiWarps);
+      // the MMA thread, the factor warp and every epilogue warp
+      mbar_init(&uempty[r], 2 + kNumEpiWarps);
     }
     *abort_flag = 0;
     fence_mbar_init();
@@ -636,16 +633,14 @@ __global__ void __launch_bounds__(kThreads, 1)
       __syncwarp();
       if (lane == 0) mbar_arrive(chunkbar);
     }
-    if constexpr (kTmaSt)
-      factor_warp(bt, units, ufull, uempty, unit_ring, facbar, facfree,
-                  reinterpret_cast<float*>(smem + L::fac_offset), abort_flag, lane);
+    factor_warp(bt, units, ufull, uempty, unit_ring, facbar, facfree,
+                reinterpret_cast<float*>(smem + L::fac_offset), abort_flag, lane);
   } else if (warp >= kEpiWarp0) {
     // --------------------------------------------------------------- epilogue
     const int q = warp & 3;                       // TMEM lanes 32q .. 32q+31 (output rows)
     const int h = (warp - kEpiWarp0) >> 2;        // column half of the 256-wide tile
     const uint32_t stage_out0 =
-        smem_u32(smem + L::out_offset + (warp - kEpiWarp0) * L::out_bufs * kOutStageBytes);
-    uint32_t nbox = 0;  // boxes emitted: alternates the staging buffers in TMA-store mode
+        smem_u32(smem + L::out_offset + (warp - kEpiWarp0) * kOutStageBytes);
     float* fac_tab = reinterpret_cast<float*>(smem + L::fac_offset);
     uint32_t c = 0;
     bool ok = !bt.planned || __all_sync(0xFFFFFFFFu, mbar_wait(chunkbar, 0, abort_flag));
@@ -676,20 +671,6 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int64_t m0 = static_cast<int64_t>(w.mb) * kBM;
       const int64_t n0 = static_cast<int64_t>(w.nb) * kBN;
       float* fac = fac_tab + (it & 1) * kBN;
-      if constexpr (!kTmaSt) {
-        // this thread's column of the table: written once the warps that read the table
-        // two units ago are past it (facbar of the last unit needed every warp to arrive)
-        const int et = threadIdx.x - kEpiWarp0 * 32;
-        const int64_t col = n0 + et;
-        float f = 0.0f;
-        if (col < p.N)
-          f = p.mode == 0 ? __fmul_rn(epilogue_a_factor(p), __ldg(p.b_scale + col))
-                          : __fmul_rn(epilogue_a_factor(p), pow2_neg(__ldg(p.col_exp + col)));
-        fac[et] = f;
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&facbar[it & 1]);
-      }
-
       const int64_t row0 = m0 + q * 32;
       const int64_t row = row0 + lane;
       const bool row_ok = row < p.M;
@@ -716,14 +697,12 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
           const int64_t col0 = n0 + h * 128 + s * 32;
           if (row0 >= p.M || col0 >= p.N) continue;  // warp-uniform: nothing of this box exists
-          const uint32_t buf = stage_out0 + (nbox++ % L::out_bufs) * kOutStageBytes;
-          emit_box<kTmaSt>(p, tma_y, tma_ws, v, true, smem_u32(fac + h * 128 + s * 32), rfac, buf, row0,
+          const uint32_t buf = stage_out0;
+          emit_box(p, tma_y, tma_ws, v, true, smem_u32(fac + h * 128 + s * 32), rfac, buf, row0,
                            col0, lane);
         }
-        if constexpr (kTmaSt) {
-          __syncwarp();
-          if (lane == 0) mbar_arrive(&facfree[it & 1]);  // this warp is done with the table
-        }
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&facfree[it & 1]);  // this warp is done with the table
         ++c;
       } else {
         uint32_t acc[128];  // int32 sums of the chunks
@@ -782,14 +761,12 @@ __global__ void __launch_bounds__(kThreads, 1)
           uint32_t v[32];
 #pragma unroll
           for (int i = 0; i < 32; ++i) v[i] = acc[s * 32 + i];
-          const uint32_t buf = stage_out0 + (nbox++ % L::out_bufs) * kOutStageBytes;
-          emit_box<kTmaSt>(p, tma_y, tma_ws, v, false, smem_u32(fac + h * 128 + s * 32), rfac, buf, row0,
+          const uint32_t buf = stage_out0;
+          emit_box(p, tma_y, tma_ws, v, false, smem_u32(fac + h * 128 + s * 32), rfac, buf, row0,
                            col0, lane);
         }
-        if constexpr (kTmaSt) {
-          __syncwarp();
-          if (lane == 0) mbar_arrive(&facfree[it & 1]);  // this warp is done with the table
-        }
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&facfree[it & 1]);  // this warp is done with the table
       }
     }
     if (!ok) {
@@ -959,13 +936,13 @@ static size_t split_ws_bytes(int64_t M, int64_t N) {
 // The layer launch's workspace starts with the unit counter of its dynamic schedule.
 constexpr size_t kSchedBytes = 256;
 
-template <int kF8, bool kMulti, bool kTmaSt>
+template <int kF8, bool kMulti>
 static int configure_kernel(int dev) {
   static bool done[64] = {};
   if (dev >= 0 && dev < 64 && done[dev]) return SQ_OK;
-  const cudaError_t err = cudaFuncSetAttribute(shiftmm_kernel<kF8, kMulti, kTmaSt>,
+  const cudaError_t err = cudaFuncSetAttribute(shiftmm_kernel<kF8, kMulti>,
                                                cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                               static_cast<int>(Smem<kTmaSt>::bytes));
+                                               static_cast<int>(Smem::bytes));
   if (err != cudaSuccess) return cuda_fail(err, "cudaFuncSetAttribute");
   if (dev >= 0 && dev < 64) done[dev] = true;
   return SQ_OK;
@@ -1119,23 +1096,18 @@ static int prepare_job(const GemmJob& j, const Plan* pl, int bits, int G, int32_
   return st;
 }
 
-template <int kF8, bool kMulti, bool kTmaSt>
+template <int kF8, bool kMulti>
 static int launch_kernel(const GemmBatch& bt, int grid, int dev, cudaStream_t s) {
-  const int st = configure_kernel<kF8, kMulti, kTmaSt>(dev);
+  const int st = configure_kernel<kF8, kMulti>(dev);
   if (st != SQ_OK) return st;
-  shiftmm_kernel<kF8, kMulti, kTmaSt><<<grid, kThreads, Smem<kTmaSt>::bytes, s>>>(bt);
+  shiftmm_kernel<kF8, kMulti><<<grid, kThreads, Smem::bytes, s>>>(bt);
   const cudaError_t err = cudaGetLastError();
   return err == cudaSuccess ? SQ_OK : cuda_fail(err, "shiftmm_kernel launch");
 }
 
 template <int kF8>
-static int launch_variant(const GemmBatch& bt, int grid, int dev, cudaStream_t s, bool multi,
-                          bool tma_st) {
-  if (multi)
-    return tma_st ? launch_kernel<kF8, true, true>(bt, grid, dev, s)
-                  : launch_kernel<kF8, true, false>(bt, grid, dev, s);
-  return tma_st ? launch_kernel<kF8, false, true>(bt, grid, dev, s)
-                : launch_kernel<kF8, false, false>(bt, grid, dev, s);
+static int launch_variant(const GemmBatch& bt, int grid, int dev, cudaStream_t s, bool multi) {
+  return multi ? launch_kernel<kF8, true>(bt, grid, dev, s) : launch_kernel<kF8, false>(bt, grid, dev, s);
 }
 
 // Checks, plans and launches up to kMaxBatch GEMMs (all with the same bits / n_groups) as
@@ -1217,21 +1189,10 @@ static int run_jobs(GemmJob* jobs, int njobs, int bits, int G, int32_t* dev_stat
     err = cudaMemsetAsync(zero_from, 0, static_cast<size_t>(zero_end - zero_from), s);
     if (err != cudaSuccess) return cuda_fail(err, "cudaMemsetAsync");
   }
-  // TMA-store mode unless the K loops are long: its epilogue leaves a 128 x 256 tile in about
-  // 3.3 us against 8 us for the plain stores, while the fourth operand stage of the plain
-  // layout only pays where the tensor core, not the epilogue, sets the pace.  Output bytes
-  // over operand-tile bytes is 2.67 / K-blocks per unit; 0.05 puts the switch near 50.
-  double out_bytes = 0.0, in_bytes = 0.0;
-  for (int g = 0; g < nlive; ++g) {
-    if (!bt.p[g].ws) out_bytes += 4.0 * bt.p[g].M * bt.p[g].N;
-    in_bytes += static_cast<double>(kStageBytes) * plans[g].m_tiles * plans[g].n_tiles *
-                plans[g].splits * plans[g].kb_per_split;
-  }
-  const bool tma_st = out_bytes > 0.05 * in_bytes;
   int grid = units < sms ? units : sms;
   if (max_ctas > 0 && grid > max_ctas) grid = max_ctas;
-  st = plans[0].elem_bytes == 1 ? launch_variant<1>(bt, grid, dev, s, multi, tma_st)
-                                : launch_variant<0>(bt, grid, dev, s, multi, tma_st);
+  st = plans[0].elem_bytes == 1 ? launch_variant<1>(bt, grid, dev, s, multi)
+                                : launch_variant<0>(bt, grid, dev, s, multi);
   if (st != SQ_OK) return st;
   for (int g = 0; g < nlive; ++g) {
     if (!bt.p[g].ws) continue;
