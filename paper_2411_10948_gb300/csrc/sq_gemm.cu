@@ -46,11 +46,13 @@
 
 namespace sq {
 
-constexpr int kBM = 128;
-constexpr int kBN = 256;
+constexpr int kBM = 128;                      // output rows of a CTA (its TMEM lanes)
+constexpr int kBN = 256;                      // output columns of a tile
+constexpr int kTileM = 2 * kBM;               // output rows of a CTA pair's tile
+constexpr int kBHalf = kBN / 2;               // B rows (output columns) a CTA holds
 constexpr int kBKBytes = 128;                 // one 128-byte swizzle row of K per stage
 constexpr int kABytes = kBM * kBKBytes;       // 16 KB
-constexpr int kBBytes = kBN * kBKBytes;       // 32 KB
+constexpr int kBBytes = kBHalf * kBKBytes;    // 16 KB
 constexpr int kStageBytes = kABytes + kBBytes;
 constexpr int kThreads = 384;
 constexpr int kEpiWarp0 = 4;
@@ -58,20 +60,18 @@ constexpr int kNumEpiWarps = 8;
 constexpr int kFacWarp = 2;   // chunk plan, then the column factors
 constexpr uint32_t kTmemCols = 2 * kBN;       // two FP32 accumulator buffers
 constexpr int64_t kExactSum = int64_t(1) << 24;  // every partial sum of a chunk stays within this
-// Shared memory of a CTA: a 4-stage operand ring, one 32 x 32 output staging box per
-// epilogue warp (the box turns the lane-per-row TMEM layout into row-contiguous stores, or
-// is the source of a TMA store), two per-tile column-factor tables, the barriers and the
-// unit ring.  Four stages hold about 1.3 us of MMA work at the tensor cores' rate; an
-// operand tile fetched from HBM while other SMs stream outputs takes longer than 1 us to
-// land, so a ring of three stages left the MMA waiting (two staging boxes per warp with
-// three stages measured 8-13% slower on MMA-bound layer launches and no faster on an
-// output-bound one).
+// Shared memory of a CTA: a 6-stage operand ring (a stage: 128 rows of A and 128 of B's
+// rows, 32 KB), one 32 x 32 output staging box per epilogue warp (the box turns the
+// lane-per-row TMEM layout into row-contiguous stores, or is the source of a TMA store), two
+// per-tile column-factor tables, the barriers and the unit ring.  Six stages hold about
+// 1.5 us of MMA work at the tensor cores' rate: an operand tile fetched while other SMs
+// stream outputs takes more than 1 us to land.
 constexpr int kOutBox = 32;
 constexpr int kUnitRing = 8;  // work units published by the producer ahead of the consumers
 constexpr int kOutStageBytes = kOutBox * kOutBox * 4;
 
 struct Smem {
-  static constexpr int stages = 4;
+  static constexpr int stages = 6;
   static constexpr int out_offset = stages * kStageBytes;
   static constexpr int fac_offset = out_offset + kNumEpiWarps * kOutStageBytes;
   static constexpr int bar_offset = fac_offset + 2 * kBN * 4;
@@ -121,6 +121,7 @@ struct GemmBatch {
   int raw_prod[kMaxBatch];
   int planned;  // some GEMM sizes its chunks from exponents (warp 2 plans them)
   int* status;
+  int lazy_from;  // with the counter: from this unit on, a pair takes one unit at a time
 };
 
 __device__ __forceinline__ float pow2_neg(int k) { return __int_as_float((127 - k) << 23); }
@@ -272,7 +273,7 @@ struct Unit {
 // cover a compact block of the output, so the A rows of a group stay in L2 while every
 // column tile of B passes by, and neither operand is streamed from HBM more than once
 // per group.
-constexpr int kGroupM = 16;
+constexpr int kGroupM = 8;
 
 __device__ __forceinline__ Unit decode_unit(const GemmParams& p, int u) {
   const int tiles = p.m_tiles * p.n_tiles;
@@ -307,20 +308,21 @@ __device__ __forceinline__ int batch_member(const GemmBatch& bt, int u, int* loc
 // units from the same ring as the other roles; a table is refilled once every epilogue
 // warp has released it (facfree).  Kept out of line: its registers stay its own.
 __device__ __noinline__ void factor_warp(const GemmBatch& bt, int units, uint64_t* ufull,
-                                         uint64_t* uempty, volatile int* unit_ring,
+                                         uint32_t uempty_c, volatile int* unit_ring,
                                          uint64_t* facbar, uint64_t* facfree, float* fac_tab,
-                                         volatile int* abort_flag, int lane) {
+                                         volatile int* abort_flag, uint32_t peer_abort_c,
+                                         int lane) {
   bool ok = true;
   int us = 0;
   uint32_t uph = 0;
   for (int it = 0; ok; ++it) {
-    if (!__all_sync(0xFFFFFFFFu, mbar_wait(&ufull[us], uph, abort_flag))) {
+    if (!__all_sync(0xFFFFFFFFu, mbar_wait_cluster(&ufull[us], uph, abort_flag))) {
       ok = false;
       break;
     }
     const int u = unit_ring[us];
     __syncwarp();
-    if (lane == 0) mbar_arrive(&uempty[us]);
+    if (lane == 0) mbar_arrive_cluster(uempty_c + us * 8);
     if (++us == kUnitRing) {
       us = 0;
       uph ^= 1u;
@@ -355,6 +357,7 @@ __device__ __noinline__ void factor_warp(const GemmBatch& bt, int units, uint64_
   if (!ok && lane == 0) {
     atomicOr(bt.status, kDevTimeout);
     *abort_flag = 1;
+    st_cluster_u32(peer_abort_c, 1);
   }
 }
 
@@ -426,7 +429,7 @@ __device__ __noinline__ void plan_chunks(const GemmBatch& bt, volatile int* out,
 }
 
 template <int kF8, bool kMulti>
-__global__ void __launch_bounds__(kThreads, 1)
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     shiftmm_kernel(const __grid_constant__ GemmBatch bt) {
   using L = Smem;
   constexpr int kStages = L::stages;
@@ -460,7 +463,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(&tfull[b], 1);
-      mbar_init(&tempty[b], kNumEpiWarps);
+      mbar_init(&tempty[b], 2 * kNumEpiWarps);  // the leader's: the epilogue warps of both CTAs
       mbar_init(&facbar[b], 1);                // the factor warp has filled table b
       mbar_init(&facfree[b], kNumEpiWarps);    // every epilogue warp is done with table b
     }
@@ -468,8 +471,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     mbar_init(chunkbar, 1);  // warp 2 has set the chunk length of every GEMM
     for (int r = 0; r < kUnitRing; ++r) {
       mbar_init(&ufull[r], 1);
-      // the MMA thread, the factor warp and every epilogue warp
-      mbar_init(&uempty[r], 2 + kNumEpiWarps);
+      // the leader's: its MMA thread, and the producer (peer) or factor warp and every
+      // epilogue warp of both CTAs
+      mbar_init(&uempty[r], 2 * (2 + kNumEpiWarps));
     }
     *abort_flag = 0;
     fence_mbar_init();
@@ -481,60 +485,92 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   }
   if (warp == 1) {
-    tmem_alloc(smem_u32(tmem_slot), kTmemCols);
-    tmem_relinquish();
+    tmem_alloc_pair(smem_u32(tmem_slot), kTmemCols);
+    tmem_relinquish_pair();
   }
   tc_fence_before();
-  __syncthreads();
+  cluster_sync();  // both CTAs' barriers exist and their TMEM is allocated
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
   const int units = bt.unit_end[bt.count - 1];
   constexpr int kBKElems = kF8 ? kBKBytes : kBKBytes / 2;
+  const uint32_t rank = cluster_ctarank();  // 0: the leader, which issues the MMAs
+  const int pair = static_cast<int>(blockIdx.x >> 1);
+  const int npairs = static_cast<int>(gridDim.x >> 1);
+  // the leader's unit-ring and TMEM release barriers, the peer's ring, the other's flag
+  const uint32_t uempty_c = mapa_shared(smem_u32(uempty), 0);
+  const uint32_t tempty_c = mapa_shared(smem_u32(tempty), 0);
+  const uint32_t full_c = mapa_shared(smem_u32(full), 0);
+  const uint32_t peer_ring_c = mapa_shared(smem_u32(const_cast<int*>(unit_ring)), 1);
+  const uint32_t peer_ufull_c = mapa_shared(smem_u32(ufull), 1);
+  const uint32_t peer_abort_c = mapa_shared(smem_u32(const_cast<int*>(abort_flag)), rank ^ 1u);
 
   if (warp == 0 && lane == 0) {
     // ------------------------------------------------------------ TMA producer
+    // Both CTAs load their halves of every stage: A rows m0 + 128 rank, B rows (output
+    // columns) n0 + 128 rank.  The leader takes the units (from the counter, or striding),
+    // publishes each to both CTAs' rings, and arms each stage's barrier for the bytes of
+    // both halves; the peer's copies count their bytes on that barrier too.
     int s = 0;
     uint32_t ph = 0;
     long long issued = 0;
     bool ok = true;
-    int next = blockIdx.x;  // a CTA's first unit is its own index
+    int next = pair;  // a pair's first unit is its own index
     int us = 0;
     uint32_t uph = 0;
     while (ok) {
-      // publish the unit (or, past the end, the stop mark) to the MMA and epilogue roles
-      const int u = next;
-      if (!mbar_wait(&uempty[us], uph ^ 1u, abort_flag)) {
-        ok = false;
-        break;
+      int u;
+      if (rank == 0) {
+        // publish the unit (or, past the end, the stop mark) to the roles of both CTAs
+        u = next;
+        if (!mbar_wait_cluster(&uempty[us], uph ^ 1u, abort_flag)) {
+          ok = false;
+          break;
+        }
+        unit_ring[us] = u;
+        st_cluster_u32(peer_ring_c + us * 4, static_cast<uint32_t>(u));
+        mbar_arrive(&ufull[us]);
+        mbar_arrive_cluster(peer_ufull_c + us * 8);
+      } else {
+        if (!mbar_wait_cluster(&ufull[us], uph, abort_flag)) {
+          ok = false;
+          break;
+        }
+        u = unit_ring[us];
+        mbar_arrive_cluster(uempty_c + us * 8);
       }
-      unit_ring[us] = u;
-      mbar_arrive(&ufull[us]);
       if (++us == kUnitRing) {
         us = 0;
         uph ^= 1u;
       }
       if (u >= units) break;
-      // Within the last wave of units a CTA takes its next unit only once its epilogue has
-      // started this one, so that no CTA holds several queued units while others run dry.
-      const bool lazy = bt.sched != nullptr && u >= units - static_cast<int>(gridDim.x);
+      // Within the last waves of units a pair takes its next unit only once its epilogues
+      // have started this one, so that no pair holds several queued units while others
+      // run dry.
+      const bool lazy = rank == 0 && bt.sched != nullptr && u >= bt.lazy_from;
       const int u_slot = us == 0 ? kUnitRing - 1 : us - 1;
       const uint32_t u_par = us == 0 ? uph ^ 1u : uph;
-      if (bt.sched == nullptr)
-        next = u + static_cast<int>(gridDim.x);
-      else if (!lazy)
-        next = static_cast<int>(gridDim.x) + atomicAdd(bt.sched, 1);
+      if (rank == 0) {
+        if (bt.sched == nullptr)
+          next = u + npairs;
+        else if (!lazy)
+          next = npairs + atomicAdd(bt.sched, 1);
+      }
       int lu;
       const int g = batch_member(bt, u, &lu);
       const Unit w = decode_unit(bt.p[g], lu);
+      // rows past M (and columns past N) are read as zeros and never stored
+      const int32_t ya = w.mb * kTileM + static_cast<int32_t>(rank) * kBM;
+      const int32_t yb = w.nb * kBN + static_cast<int32_t>(rank) * kBHalf;
       for (int kb = w.kb0; kb < w.kb1; ++kb) {
         if (!mbar_wait(&empty[s], ph ^ 1u, abort_flag)) {
           ok = false;
           break;
         }
         const uint32_t sa = smem_u32(smem + s * kStageBytes);
-        mbar_arrive_expect_tx(&full[s], kStageBytes);
-        tma_load_2d(sa, &bt.a[g], smem_u32(&full[s]), kb * kBKElems, w.mb * kBM);
-        tma_load_2d(sa + kABytes, &bt.b[g], smem_u32(&full[s]), kb * kBKElems, w.nb * kBN);
+        if (rank == 0) mbar_arrive_expect_tx(&full[s], 2 * kStageBytes);
+        tma_load_2d_pair(sa, &bt.a[g], full_c + s * 8, kb * kBKElems, ya);
+        tma_load_2d_pair(sa + kABytes, &bt.b[g], full_c + s * 8, kb * kBKElems, yb);
         ++issued;
         if (++s == kStages) {
           s = 0;
@@ -542,23 +578,34 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       }
       if (ok && lazy) {
-        if (!mbar_wait(&uempty[u_slot], u_par, abort_flag)) {
+        if (!mbar_wait_cluster(&uempty[u_slot], u_par, abort_flag)) {
           ok = false;
           break;
         }
-        next = static_cast<int>(gridDim.x) + atomicAdd(bt.sched, 1);
+        next = npairs + atomicAdd(bt.sched, 1);
       }
     }
     if (!ok) {
       atomicOr(bt.status, kDevTimeout);
       *abort_flag = 1;
+      st_cluster_u32(peer_abort_c, 1);
     }
-    // every issued copy must have landed before the CTA may exit
-    for (long long i = issued > kStages ? issued - kStages : 0; i < issued; ++i)
-      mbar_wait(&full[i % kStages], static_cast<uint32_t>((i / kStages) & 1), nullptr);
-  } else if (warp == 1 && lane == 0) {
-    // ------------------------------------------------------------- MMA issuer
-    constexpr uint32_t idesc = make_idesc(kF8 ? 0u : 1u, kBM, kBN);
+    // Every issued copy must have landed before the CTAs may exit.  The leader's stage
+    // barriers count both CTAs' bytes; after a timeout the peer cannot tell its own copies
+    // apart there and gives them time instead (a copy lands within microseconds).
+    if (rank == 0) {
+      for (long long i = issued > kStages ? issued - kStages : 0; i < issued; ++i)
+        mbar_wait(&full[i % kStages], static_cast<uint32_t>((i / kStages) & 1), nullptr);
+    } else if (!ok) {
+      const uint64_t t0 = globaltimer_ns();
+      while (globaltimer_ns() - t0 < 200000ull) {
+      }
+    }
+  } else if (warp == 1 && lane == 0 && rank == 0) {
+    // ------------------------------------------------- MMA issuer (the leader's)
+    // 256 x 256 pair MMAs; a stage is released in both CTAs, and a finished chunk is
+    // announced to both CTAs' epilogues, by multicast commits.
+    constexpr uint32_t idesc = make_idesc(kF8 ? 0u : 1u, kTileM, kBN);
     int s = 0;
     uint32_t ph = 0;
     uint32_t c = 0;
@@ -585,7 +632,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int kc = w.kb0; kc < w.kb1 && ok; kc += chunk_kb) {
         const int kce = min(w.kb1, kc + chunk_kb);
         const uint32_t b = c & 1u, tph = (c >> 1) & 1u;
-        if (!mbar_wait(&tempty[b], tph ^ 1u, abort_flag)) {
+        if (!mbar_wait_cluster(&tempty[b], tph ^ 1u, abort_flag)) {  // both CTAs' epilogues
           ok = false;
           break;
         }
@@ -609,22 +656,23 @@ __global__ void __launch_bounds__(kThreads, 1)
             else
               tc_mma_f16(d, ad, bd, idesc, accumulate);
           }
-          tc_commit(smem_u32(&empty[s]));  // frees the stage once these MMAs are done
+          tc_commit_pair(smem_u32(&empty[s]), 0x3);  // frees the stage in both CTAs
           if (++s == kStages) {
             s = 0;
             ph ^= 1u;
           }
         }
         if (!ok) break;
-        tc_commit(smem_u32(&tfull[b]));  // chunk complete in TMEM buffer b
+        tc_commit_pair(smem_u32(&tfull[b]), 0x3);  // chunk complete in TMEM buffer b
         ++c;
       }
     }
     if (!ok) {
       atomicOr(bt.status, kDevTimeout);
       *abort_flag = 1;
+      st_cluster_u32(peer_abort_c, 1);
     }
-    tc_commit(smem_u32(drain));
+    tc_commit_pair(smem_u32(drain), 0x1);  // every MMA issued has completed
     mbar_wait(drain, 0, nullptr);
   } else if (warp == kFacWarp) {
     // --------------------------------------------------- chunk plan, column factors
@@ -633,8 +681,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       __syncwarp();
       if (lane == 0) mbar_arrive(chunkbar);
     }
-    factor_warp(bt, units, ufull, uempty, unit_ring, facbar, facfree,
-                reinterpret_cast<float*>(smem + L::fac_offset), abort_flag, lane);
+    factor_warp(bt, units, ufull, uempty_c, unit_ring, facbar, facfree,
+                reinterpret_cast<float*>(smem + L::fac_offset), abort_flag, peer_abort_c, lane);
   } else if (warp >= kEpiWarp0) {
     // --------------------------------------------------------------- epilogue
     const int q = warp & 3;                       // TMEM lanes 32q .. 32q+31 (output rows)
@@ -647,13 +695,13 @@ __global__ void __launch_bounds__(kThreads, 1)
     int us = 0;
     uint32_t uph = 0;
     for (int it = 0; ok; ++it) {
-      if (!__all_sync(0xFFFFFFFFu, mbar_wait(&ufull[us], uph, abort_flag))) {
+      if (!__all_sync(0xFFFFFFFFu, mbar_wait_cluster(&ufull[us], uph, abort_flag))) {
         ok = false;
         break;
       }
       const int u = unit_ring[us];
       __syncwarp();
-      if (lane == 0) mbar_arrive(&uempty[us]);
+      if (lane == 0) mbar_arrive_cluster(uempty_c + us * 8);
       if (++us == kUnitRing) {
         us = 0;
         uph ^= 1u;
@@ -668,7 +716,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int ckb =
           bt.planned ? reinterpret_cast<volatile int*>(smem + L::chunk_offset)[g] : p.chunk_kb;
       const int nch = (w.kb1 - w.kb0 + ckb - 1) / ckb;
-      const int64_t m0 = static_cast<int64_t>(w.mb) * kBM;
+      const int64_t m0 = static_cast<int64_t>(w.mb) * kTileM + rank * kBM;  // this CTA's rows
       const int64_t n0 = static_cast<int64_t>(w.nb) * kBN;
       float* fac = fac_tab + (it & 1) * kBN;
       const int64_t row0 = m0 + q * 32;
@@ -693,7 +741,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (s == 3) {
             tc_fence_before();
             __syncwarp();
-            if (lane == 0) mbar_arrive(&tempty[b]);  // TMEM buffer b may take the next tile
+            if (lane == 0) mbar_arrive_cluster(tempty_c + b * 8);  // buffer b may take the next tile
           }
           const int64_t col0 = n0 + h * 128 + s * 32;
           if (row0 >= p.M || col0 >= p.N) continue;  // warp-uniform: nothing of this box exists
@@ -746,7 +794,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
           tc_fence_before();
           __syncwarp();
-          if (lane == 0) mbar_arrive(&tempty[b]);  // TMEM buffer b may take the next chunk
+          if (lane == 0) mbar_arrive_cluster(tempty_c + b * 8);  // buffer b may take the next chunk
           ++c;
         }
         if (!ok) break;
@@ -772,14 +820,17 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (!ok) {
       atomicOr(bt.status, kDevTimeout);
       *abort_flag = 1;
+      st_cluster_u32(peer_abort_c, 1);
     }
     if (lane == 0) bulk_wait_read<0>();  // no store still reads shared memory at exit
   }
 
-  __syncthreads();
+  // neither CTA leaves while the other may still reach its barriers, shared memory or TMEM
+  tc_fence_before();
+  cluster_sync();
   if (warp == 1) {
     tc_fence_after();
-    tmem_dealloc(tmem_base, kTmemCols);
+    tmem_dealloc_pair(tmem_base, kTmemCols);
   }
 }
 
@@ -903,7 +954,7 @@ static int check_exact_range(int which, int64_t K, int bits, int G) {
 }
 
 // max_splits: 1 never splits K; 0 lets the SM count alone decide
-static int make_plan(int which, int64_t M, int64_t N, int64_t K, int bits, int G, int sms,
+static int make_plan(int which, int64_t M, int64_t N, int64_t K, int bits, int G, int pairs,
                      int max_splits, Plan* pl) {
   const int st = check_exact_range(which, K, bits, G);
   if (st != SQ_OK) return st;
@@ -912,13 +963,13 @@ static int make_plan(int which, int64_t M, int64_t N, int64_t K, int bits, int G
   const int bk = kBKBytes / pl->elem_bytes;
   pl->chunk_kb = static_cast<int>((kExactSum / P) / bk);
   if (pl->chunk_kb > (1 << 20)) pl->chunk_kb = 1 << 20;
-  pl->m_tiles = static_cast<int>((M + kBM - 1) / kBM);
+  pl->m_tiles = static_cast<int>((M + kTileM - 1) / kTileM);
   pl->n_tiles = static_cast<int>((N + kBN - 1) / kBN);
   pl->kb_total = static_cast<int>((K + bk - 1) / bk);
   const int64_t tiles = static_cast<int64_t>(pl->m_tiles) * pl->n_tiles;
   int splits = 1;
-  if (max_splits != 1 && tiles < sms && pl->kb_total >= 4) {
-    splits = static_cast<int>(sms / tiles);
+  if (max_splits != 1 && tiles < pairs && pl->kb_total >= 4) {
+    splits = static_cast<int>(pairs / tiles);
     if (splits > pl->kb_total / 2) splits = pl->kb_total / 2;
     if (max_splits > 1 && splits > max_splits) splits = max_splits;
     if (splits < 1) splits = 1;
@@ -946,6 +997,33 @@ static int configure_kernel(int dev) {
   if (err != cudaSuccess) return cuda_fail(err, "cudaFuncSetAttribute");
   if (dev >= 0 && dev < 64) done[dev] = true;
   return SQ_OK;
+}
+
+// CTA pairs of the GEMM kernel resident at once: one per two SMs, fewer where the GPU's
+// SM groups leave single SMs over.  -1 without a device.
+static int device_pairs(int* dev_out) {
+  static int cached[64] = {};
+  int dev = 0;
+  const int sms = device_sms(&dev);
+  if (sms <= 0) return -1;
+  if (dev_out) *dev_out = dev;
+  if (dev >= 0 && dev < 64 && cached[dev] > 0) return cached[dev];
+  int pairs = sms / 2;
+  if (configure_kernel<1, false>(dev) == SQ_OK) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(2 * pairs);
+    cfg.blockDim = dim3(kThreads);
+    cfg.dynamicSmemBytes = Smem::bytes;
+    int n = 0;
+    if (cudaOccupancyMaxActiveClusters(&n, shiftmm_kernel<1, false>, &cfg) == cudaSuccess && n > 0 &&
+        n < pairs)
+      pairs = n;
+    else
+      cudaGetLastError();  // an unanswered query leaves no error behind
+  }
+  if (pairs < 1) pairs = 1;
+  if (dev >= 0 && dev < 64) cached[dev] = pairs;
+  return pairs;
 }
 
 // One GEMM of a launch: out[M, N] = A[M, K] B[N, K]^T with the operand roles of `which`
@@ -1016,11 +1094,11 @@ static int check_job(const GemmJob& j, int bits, int G, int32_t* dev_status, cud
 // Tiles and K splits of one checked GEMM: the SM count decides the splits, up to
 // max_splits, and a split needs a workspace for the [M, N] int32 partial sums (added by TMA
 // into N-element rows, which must stay 16-byte aligned).
-static int plan_job(const GemmJob& j, int bits, int G, int sms, int max_splits, Plan* pl) {
-  const int st = make_plan(j.which, j.M, j.N, j.K, bits, G, sms, max_splits, pl);
+static int plan_job(const GemmJob& j, int bits, int G, int pairs, int max_splits, Plan* pl) {
+  const int st = make_plan(j.which, j.M, j.N, j.K, bits, G, pairs, max_splits, pl);
   if (st != SQ_OK || pl->splits <= 1) return st;
   if (j.ws == nullptr || j.ws_bytes < split_ws_bytes(j.M, j.N) || !aligned16(j.ws) || j.N % 4 != 0)
-    return make_plan(j.which, j.M, j.N, j.K, bits, G, sms, 1, pl);
+    return make_plan(j.which, j.M, j.N, j.K, bits, G, pairs, 1, pl);
   return SQ_OK;
 }
 
@@ -1028,7 +1106,7 @@ static int plan_job(const GemmJob& j, int bits, int G, int sms, int max_splits, 
 // its units stay well inside the launch's expected length.  Every split adds the whole
 // output once more to the L2 reductions, whose throughput is far below a plain store's.
 // Unit cost model, in K-block times: the K loop plus about 8 for the epilogue.
-static int balance_splits(GemmJob* const* jobs, int n, int bits, int G, int sms, Plan* plans) {
+static int balance_splits(GemmJob* const* jobs, int n, int bits, int G, int pairs, Plan* plans) {
   if (n <= 1) return SQ_OK;
   constexpr double kEpiKb = 8.0;
   double work = 0.0;  // the batch's total cost, with every split GEMM at its maximum
@@ -1043,10 +1121,10 @@ static int balance_splits(GemmJob* const* jobs, int n, int bits, int G, int sms,
       const double kbs = static_cast<double>((plans[g].kb_total + s - 1) / s);
       const double w = work - tiles * plans[g].splits * (plans[g].kb_per_split + kEpiKb) +
                        tiles * s * (kbs + kEpiKb);
-      if (kbs + kEpiKb <= 0.8 * w / sms) break;
+      if (kbs + kEpiKb <= 0.8 * w / pairs) break;
     }
     if (s < plans[g].splits) {
-      const int st = plan_job(*jobs[g], bits, G, sms, s, &plans[g]);
+      const int st = plan_job(*jobs[g], bits, G, pairs, s, &plans[g]);
       if (st != SQ_OK) return st;
     }
   }
@@ -1059,7 +1137,7 @@ static int prepare_job(const GemmJob& j, const Plan* pl, int bits, int G, int32_
   int st;
   const int eb = pl->elem_bytes;
   if ((st = make_operand_map(&bt->a[g], j.a, j.M, j.K, j.lda, eb, kBM)) != SQ_OK) return st;
-  if ((st = make_operand_map(&bt->b[g], j.b, j.N, j.K, j.ldb, eb, kBN)) != SQ_OK) return st;
+  if ((st = make_operand_map(&bt->b[g], j.b, j.N, j.K, j.ldb, eb, kBHalf)) != SQ_OK) return st;
   GemmParams& p = bt->p[g];
   p.M = static_cast<int>(j.M);
   p.N = static_cast<int>(j.N);
@@ -1128,18 +1206,18 @@ static int run_jobs(GemmJob* jobs, int njobs, int bits, int G, int32_t* dev_stat
   }
   if (nlive == 0) return SQ_OK;
   int dev = 0;
-  const int sms = device_sms(&dev);
-  if (sms <= 0) return fail(SQ_ECUDA, "%s: no current CUDA device", job_name(jobs[live[0]].which));
+  const int pairs = device_pairs(&dev);
+  if (pairs <= 0) return fail(SQ_ECUDA, "%s: no current CUDA device", job_name(jobs[live[0]].which));
   GemmBatch bt;
   memset(&bt, 0, sizeof(bt));
   Plan plans[kMaxBatch];
   GemmJob* lj[kMaxBatch];
   for (int g = 0; g < nlive; ++g) {
     lj[g] = &jobs[live[g]];
-    const int st = plan_job(*lj[g], bits, G, sms, 0, &plans[g]);
+    const int st = plan_job(*lj[g], bits, G, pairs, 0, &plans[g]);
     if (st != SQ_OK) return st;
   }
-  int st = balance_splits(lj, nlive, bits, G, sms, plans);
+  int st = balance_splits(lj, nlive, bits, G, pairs, plans);
   if (st != SQ_OK) return st;
   for (int g = 0; g < nlive; ++g)
     if ((st = prepare_job(*lj[g], &plans[g], bits, G, dev_status, &bt, g)) != SQ_OK) return st;
@@ -1189,8 +1267,19 @@ static int run_jobs(GemmJob* jobs, int njobs, int bits, int G, int32_t* dev_stat
     err = cudaMemsetAsync(zero_from, 0, static_cast<size_t>(zero_end - zero_from), s);
     if (err != cudaSuccess) return cuda_fail(err, "cudaMemsetAsync");
   }
-  int grid = units < sms ? units : sms;
-  if (max_ctas > 0 && grid > max_ctas) grid = max_ctas;
+  // two CTAs per pair; a cap on the CTAs leaves at least one pair
+  int npairs = units < pairs ? units : pairs;
+  if (max_ctas > 0 && npairs > max_ctas / 2) npairs = max_ctas / 2 > 0 ? max_ctas / 2 : 1;
+  const int grid = 2 * npairs;
+  // A pair holds up to about stages / K-blocks + 2 units of the last (shortest) GEMM at
+  // once: its operand ring and two TMEM buffers.  Over that many final waves it takes
+  // one unit at a time, so the pairs run out of work together.
+  {
+    const int kb = plans[nlive - 1].kb_per_split > 0 ? plans[nlive - 1].kb_per_split : 1;
+    const int depth = 2 + (Smem::stages + kb - 1) / kb;
+    const long long from = static_cast<long long>(units) - static_cast<long long>(depth) * npairs;
+    bt.lazy_from = from > 0 ? static_cast<int>(from) : 0;
+  }
   st = plans[0].elem_bytes == 1 ? launch_variant<1>(bt, grid, dev, s, multi)
                                 : launch_variant<0>(bt, grid, dev, s, multi);
   if (st != SQ_OK) return st;
@@ -1198,7 +1287,7 @@ static int run_jobs(GemmJob* jobs, int njobs, int bits, int G, int32_t* dev_stat
     if (!bt.p[g].ws) continue;
     const int64_t quads = static_cast<int64_t>(bt.p[g].M) * (bt.p[g].N / 4);
     int64_t blocks = (quads + 255) / 256;
-    if (blocks > static_cast<int64_t>(sms) * 16) blocks = static_cast<int64_t>(sms) * 16;
+    if (blocks > static_cast<int64_t>(pairs) * 32) blocks = static_cast<int64_t>(pairs) * 32;
     splitk_finalize_kernel<<<static_cast<unsigned>(blocks), 256, 0, s>>>(bt.p[g]);
     err = cudaGetLastError();
     if (err != cudaSuccess) return cuda_fail(err, "splitk_finalize_kernel launch");
@@ -1234,13 +1323,13 @@ static void layer_jobs(const sq_layer_gemms* a, GemmJob jobs[3], int mask) {
 
 // Bytes of split-K workspace each GEMM of the layer would use (0: it would not split),
 // a multiple of 256 bytes.
-static void layer_ws_need(const GemmJob jobs[3], int bits, int G, int sms, size_t need[3]) {
+static void layer_ws_need(const GemmJob jobs[3], int bits, int G, int pairs, size_t need[3]) {
   for (int i = 0; i < 3; ++i) {
     need[i] = 0;
     const GemmJob& j = jobs[i];
     if (j.M <= 0 || j.N <= 0 || j.K <= 0 || j.N % 4 != 0) continue;
     Plan pl;
-    if (make_plan(j.which, j.M, j.N, j.K, bits, G, sms, 0, &pl) != SQ_OK) continue;
+    if (make_plan(j.which, j.M, j.N, j.K, bits, G, pairs, 0, &pl) != SQ_OK) continue;
     if (pl.splits > 1) need[i] = split_ws_bytes(j.M, j.N);
   }
 }
@@ -1248,12 +1337,12 @@ static void layer_ws_need(const GemmJob jobs[3], int bits, int G, int sms, size_
 // The layer workspace: the unit counter, then a split-K region for each GEMM that would
 // split, as far as the workspace reaches.  Returns the counter (null without a usable
 // workspace: the launch then strides over its units and splits nothing).
-static int* assign_layer_ws(GemmJob jobs[3], int bits, int G, int sms, void* workspace,
+static int* assign_layer_ws(GemmJob jobs[3], int bits, int G, int pairs, void* workspace,
                             size_t workspace_bytes) {
   if (workspace == nullptr || workspace_bytes < kSchedBytes || !aligned16(workspace)) return nullptr;
-  if (sms > 0) {
+  if (pairs > 0) {
     size_t need[3];
-    layer_ws_need(jobs, bits, G, sms, need);
+    layer_ws_need(jobs, bits, G, pairs, need);
     size_t off = kSchedBytes;
     for (int i = 0; i < 3; ++i) {
       if (need[i] == 0 || off + need[i] > workspace_bytes) continue;
@@ -1340,10 +1429,10 @@ extern "C" size_t shiftquant_gemm_workspace_bytes(int which, int64_t M, int64_t 
   if (which < 0 || which > 2 || !bits_ok(bits) || !groups_ok(n_groups) || M <= 0 || N <= 0 ||
       K <= 0)
     return 0;
-  const int sms = device_sms(nullptr);
-  if (sms <= 0) return 0;
+  const int pairs = device_pairs(nullptr);
+  if (pairs <= 0) return 0;
   Plan pl;
-  if (make_plan(which, M, N, K, bits, n_groups, sms, 0, &pl) != SQ_OK) return 0;
+  if (make_plan(which, M, N, K, bits, n_groups, pairs, 0, &pl) != SQ_OK) return 0;
   return pl.splits > 1 ? split_ws_bytes(M, N) : 0;
 }
 
@@ -1380,16 +1469,16 @@ extern "C" sq_status shiftquant_gemm_layer(const sq_layer_gemms* args, void* wor
     return fail(SQ_EINVAL, "gemm_layer: gemm_mask must be in [0, 7] and max_ctas >= 0");
   GemmJob jobs[3];
   layer_jobs(args, jobs, args->gemm_mask);
-  const int sms = device_sms(nullptr);
-  int* sched = assign_layer_ws(jobs, args->bits, args->n_groups, sms, workspace, workspace_bytes);
+  const int pairs = device_pairs(nullptr);
+  int* sched = assign_layer_ws(jobs, args->bits, args->n_groups, pairs, workspace, workspace_bytes);
   return run_jobs(jobs, 3, args->bits, args->n_groups, dev_status, stream, sched, args->max_ctas);
 }
 
 extern "C" size_t shiftquant_gemm_layer_workspace_bytes(int64_t M, int64_t K, int64_t N, int bits,
                                                         int n_groups) {
   if (!bits_ok(bits) || !groups_ok(n_groups)) return 0;
-  const int sms = device_sms(nullptr);
-  if (sms <= 0) return 0;
+  const int pairs = device_pairs(nullptr);
+  if (pairs <= 0) return 0;
   sq_layer_gemms a;
   memset(&a, 0, sizeof(a));
   a.M = M;
@@ -1398,7 +1487,7 @@ extern "C" size_t shiftquant_gemm_layer_workspace_bytes(int64_t M, int64_t K, in
   GemmJob jobs[3];
   layer_jobs(&a, jobs, 0);
   size_t need[3];
-  layer_ws_need(jobs, bits, n_groups, sms, need);
+  layer_ws_need(jobs, bits, n_groups, pairs, need);
   return kSchedBytes + need[0] + need[1] + need[2];
 }
 
@@ -1408,8 +1497,8 @@ extern "C" int shiftquant_gemm_layer_kernel_launches(int64_t M, int64_t K, int64
   if (!bits_ok(bits) || !groups_ok(n_groups) || M < 0 || K < 0 || N < 0 || gemm_mask < 0 ||
       gemm_mask > 7)
     return -1;
-  const int sms = device_sms(nullptr);
-  if (sms <= 0) return -1;
+  const int pairs = device_pairs(nullptr);
+  if (pairs <= 0) return -1;
   sq_layer_gemms a;
   memset(&a, 0, sizeof(a));
   a.M = M;
@@ -1418,7 +1507,7 @@ extern "C" int shiftquant_gemm_layer_kernel_launches(int64_t M, int64_t K, int64
   GemmJob jobs[3];
   layer_jobs(&a, jobs, gemm_mask);
   // the plan looks at the workspace's size and alignment only: a stand-in address serves
-  assign_layer_ws(jobs, bits, n_groups, sms, workspace_bytes ? reinterpret_cast<void*>(4096) : nullptr,
+  assign_layer_ws(jobs, bits, n_groups, pairs, workspace_bytes ? reinterpret_cast<void*>(4096) : nullptr,
                   workspace_bytes);
   Plan plans[kMaxBatch];
   GemmJob* lj[kMaxBatch];
@@ -1426,11 +1515,11 @@ extern "C" int shiftquant_gemm_layer_kernel_launches(int64_t M, int64_t K, int64
   for (int i = 0; i < 3; ++i) {
     if (jobs[i].M == 0 || jobs[i].N == 0 || jobs[i].K == 0) continue;
     lj[n] = &jobs[i];
-    if (plan_job(jobs[i], bits, n_groups, sms, 0, &plans[n]) != SQ_OK) return -1;
+    if (plan_job(jobs[i], bits, n_groups, pairs, 0, &plans[n]) != SQ_OK) return -1;
     ++n;
   }
   if (n == 0) return 0;
-  if (balance_splits(lj, n, bits, n_groups, sms, plans) != SQ_OK) return -1;
+  if (balance_splits(lj, n, bits, n_groups, pairs, plans) != SQ_OK) return -1;
   int launches = 1;
   for (int g = 0; g < n; ++g) launches += plans[g].splits > 1;
   return launches;
