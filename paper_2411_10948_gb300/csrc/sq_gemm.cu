@@ -48,31 +48,39 @@ namespace sq {
 
 constexpr int kBM = 128;                      // output rows of a CTA (its TMEM lanes)
 constexpr int kBN = 256;                      // output columns of a tile
-constexpr int kTileM = 2 * kBM;               // output rows of a CTA pair's tile
-constexpr int kBHalf = kBN / 2;               // B rows (output columns) a CTA holds
 constexpr int kBKBytes = 128;                 // one 128-byte swizzle row of K per stage
 constexpr int kABytes = kBM * kBKBytes;       // 16 KB
-constexpr int kBBytes = kBHalf * kBKBytes;    // 16 KB
-constexpr int kStageBytes = kABytes + kBBytes;
 constexpr int kThreads = 384;
 constexpr int kEpiWarp0 = 4;
 constexpr int kNumEpiWarps = 8;
 constexpr int kFacWarp = 2;   // chunk plan, then the column factors
 constexpr uint32_t kTmemCols = 2 * kBN;       // two FP32 accumulator buffers
 constexpr int64_t kExactSum = int64_t(1) << 24;  // every partial sum of a chunk stays within this
-// Shared memory of a CTA: a 6-stage operand ring (a stage: 128 rows of A and 128 of B's
-// rows, 32 KB), one 32 x 32 output staging box per epilogue warp (the box turns the
-// lane-per-row TMEM layout into row-contiguous stores, or is the source of a TMA store), two
-// per-tile column-factor tables, the barriers and the unit ring.  Six stages hold about
-// 1.5 us of MMA work at the tensor cores' rate: an operand tile fetched while other SMs
-// stream outputs takes more than 1 us to land.
+// Two tile modes.  Single (kPair false): a CTA runs a 128 x 256 tile; a stage holds its
+// 128 A rows and all 256 B rows (48 KB).  Pair (kPair true): a 2-CTA cluster runs a
+// 256 x 256 tile with cta_group::2 MMAs issued by the leader; a stage holds a CTA's 128 A
+// rows and 128 of the 256 B rows (32 KB), so the operand bytes each SM's shared memory
+// takes in and hands to the tensor core drop by a third: a single CTA's 128 x 256 MMA
+// needs more shared-memory bandwidth than the SM has and runs at about 70% of the tensor
+// rate.  The epilogue of a pair is slower, though (about 20% per output box), so
+// launches whose K loops are short keep single tiles.
+//
+// Shared memory of a CTA: the operand ring (4 stages single, 6 pair: about 1.3-1.5 us of
+// MMA work, more than an operand tile takes to land while other SMs stream outputs), one
+// 32 x 32 output staging box per epilogue warp (the box turns the lane-per-row TMEM layout
+// into row-contiguous stores, or is the source of a TMA store), two per-tile column-factor
+// tables, the barriers and the unit ring.
 constexpr int kOutBox = 32;
 constexpr int kUnitRing = 8;  // work units published by the producer ahead of the consumers
 constexpr int kOutStageBytes = kOutBox * kOutBox * 4;
 
+template <bool kPair>
 struct Smem {
-  static constexpr int stages = 6;
-  static constexpr int out_offset = stages * kStageBytes;
+  static constexpr int b_rows = kPair ? kBN / 2 : kBN;    // B rows (output columns) held
+  static constexpr int tile_m = kPair ? 2 * kBM : kBM;    // output rows of a unit
+  static constexpr int stage_bytes = kABytes + b_rows * kBKBytes;
+  static constexpr int stages = kPair ? 6 : 4;
+  static constexpr int out_offset = stages * stage_bytes;
   static constexpr int fac_offset = out_offset + kNumEpiWarps * kOutStageBytes;
   static constexpr int bar_offset = fac_offset + 2 * kBN * 4;
   // full, empty, tfull, tempty, fac, drain, unit ring full / empty, fac free, chunk plan
@@ -273,9 +281,9 @@ struct Unit {
 // cover a compact block of the output, so the A rows of a group stay in L2 while every
 // column tile of B passes by, and neither operand is streamed from HBM more than once
 // per group.
-constexpr int kGroupM = 8;
-
+template <bool kPair>
 __device__ __forceinline__ Unit decode_unit(const GemmParams& p, int u) {
+  constexpr int kGroupM = kPair ? 8 : 16;  // 2048 output rows either way
   const int tiles = p.m_tiles * p.n_tiles;
   const int split = u / tiles;
   const int t = u - split * tiles;
@@ -302,13 +310,34 @@ __device__ __forceinline__ int batch_member(const GemmBatch& bt, int u, int* loc
   return g;
 }
 
+// Waits on the unit ring and the TMEM-release barriers, and arrivals on the leader's
+// barriers: at cluster scope in a pair (the other CTA arrives, or wrote the ring slot),
+// at CTA scope otherwise.
+template <bool kPair>
+__device__ __forceinline__ bool ring_wait(uint64_t* bar, uint32_t parity, volatile int* abort_flag) {
+  if constexpr (kPair)
+    return mbar_wait_cluster(bar, parity, abort_flag);
+  else
+    return mbar_wait(bar, parity, abort_flag);
+}
+
+template <bool kPair>
+__device__ __forceinline__ void leader_arrive(uint64_t* local_bar, uint32_t cluster_bar) {
+  if constexpr (kPair)
+    mbar_arrive_cluster(cluster_bar);
+  else
+    mbar_arrive(local_bar);
+}
+
 // The factor warp: the dequantizing factor of each of a tile's 256 columns, into one of
 // two tables ahead of the epilogue: s_A 2^-(G-1) s_B[n] (forward, loss propagation) or
 // s_X s_dY 2^-eY_n (weight gradient; the row's 2^-eX_m is the epilogue's).  It reads the
 // units from the same ring as the other roles; a table is refilled once every epilogue
 // warp has released it (facfree).  Kept out of line: its registers stay its own.
+template <bool kPair>
 __device__ __noinline__ void factor_warp(const GemmBatch& bt, int units, uint64_t* ufull,
-                                         uint32_t uempty_c, volatile int* unit_ring,
+                                         uint64_t* uempty, uint32_t uempty_c,
+                                         volatile int* unit_ring,
                                          uint64_t* facbar, uint64_t* facfree, float* fac_tab,
                                          volatile int* abort_flag, uint32_t peer_abort_c,
                                          int lane) {
@@ -316,13 +345,13 @@ __device__ __noinline__ void factor_warp(const GemmBatch& bt, int units, uint64_
   int us = 0;
   uint32_t uph = 0;
   for (int it = 0; ok; ++it) {
-    if (!__all_sync(0xFFFFFFFFu, mbar_wait_cluster(&ufull[us], uph, abort_flag))) {
+    if (!__all_sync(0xFFFFFFFFu, ring_wait<kPair>(&ufull[us], uph, abort_flag))) {
       ok = false;
       break;
     }
     const int u = unit_ring[us];
     __syncwarp();
-    if (lane == 0) mbar_arrive_cluster(uempty_c + us * 8);
+    if (lane == 0) leader_arrive<kPair>(&uempty[us], uempty_c + us * 8);
     if (++us == kUnitRing) {
       us = 0;
       uph ^= 1u;
@@ -332,7 +361,7 @@ __device__ __noinline__ void factor_warp(const GemmBatch& bt, int units, uint64_
     const int g = batch_member(bt, u, &lu);
     const GemmParams& p = bt.p[g];
     const float a_fac = epilogue_a_factor(p);
-    const int64_t n0 = static_cast<int64_t>(decode_unit(p, lu).nb) * kBN;
+    const int64_t n0 = static_cast<int64_t>(decode_unit<kPair>(p, lu).nb) * kBN;
     float f[kBN / 32];
 #pragma unroll
     for (int j = 0; j < kBN / 32; ++j) {
@@ -357,7 +386,7 @@ __device__ __noinline__ void factor_warp(const GemmBatch& bt, int units, uint64_
   if (!ok && lane == 0) {
     atomicOr(bt.status, kDevTimeout);
     *abort_flag = 1;
-    st_cluster_u32(peer_abort_c, 1);
+    if (peer_abort_c != 0) st_cluster_u32(peer_abort_c, 1);
   }
 }
 
@@ -428,10 +457,11 @@ __device__ __noinline__ void plan_chunks(const GemmBatch& bt, volatile int* out,
   }
 }
 
-template <int kF8, bool kMulti>
-__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
-    shiftmm_kernel(const __grid_constant__ GemmBatch bt) {
-  using L = Smem;
+// kPair: launched as 2-CTA clusters running 256-row tiles (the host sets the cluster shape)
+template <int kF8, bool kMulti, bool kPair>
+__global__ void __launch_bounds__(kThreads, 1) shiftmm_kernel(const __grid_constant__ GemmBatch bt) {
+  using L = Smem<kPair>;
+  constexpr int kCg = kPair ? 2 : 1;
   constexpr int kStages = L::stages;
   extern __shared__ __align__(1024) uint8_t smem[];
   if ((smem_u32(smem) & 1023u) != 0) {  // the swizzled layouts need 1 KB alignment
@@ -463,7 +493,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(&tfull[b], 1);
-      mbar_init(&tempty[b], 2 * kNumEpiWarps);  // the leader's: the epilogue warps of both CTAs
+      mbar_init(&tempty[b], kCg * kNumEpiWarps);  // the leader's: the epilogue warps of all CTAs
       mbar_init(&facbar[b], 1);                // the factor warp has filled table b
       mbar_init(&facfree[b], kNumEpiWarps);    // every epilogue warp is done with table b
     }
@@ -472,8 +502,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     for (int r = 0; r < kUnitRing; ++r) {
       mbar_init(&ufull[r], 1);
       // the leader's: its MMA thread, and the producer (peer) or factor warp and every
-      // epilogue warp of both CTAs
-      mbar_init(&uempty[r], 2 * (2 + kNumEpiWarps));
+      // epilogue warp of each CTA
+      mbar_init(&uempty[r], kCg * (2 + kNumEpiWarps));
     }
     *abort_flag = 0;
     fence_mbar_init();
@@ -485,32 +515,40 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     }
   }
   if (warp == 1) {
-    tmem_alloc_pair(smem_u32(tmem_slot), kTmemCols);
-    tmem_relinquish_pair();
+    tmem_alloc<kCg>(smem_u32(tmem_slot), kTmemCols);
+    tmem_relinquish<kCg>();
   }
   tc_fence_before();
-  cluster_sync();  // both CTAs' barriers exist and their TMEM is allocated
+  if constexpr (kPair)
+    cluster_sync();  // both CTAs' barriers exist and their TMEM is allocated
+  else
+    __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
   const int units = bt.unit_end[bt.count - 1];
   constexpr int kBKElems = kF8 ? kBKBytes : kBKBytes / 2;
-  const uint32_t rank = cluster_ctarank();  // 0: the leader, which issues the MMAs
-  const int pair = static_cast<int>(blockIdx.x >> 1);
-  const int npairs = static_cast<int>(gridDim.x >> 1);
-  // the leader's unit-ring and TMEM release barriers, the peer's ring, the other's flag
+  // rank 0: the CTA that takes the units and issues the MMAs (a pair's leader, or a single CTA)
+  const uint32_t rank = kPair ? cluster_ctarank() : 0u;
+  const int pair = static_cast<int>(blockIdx.x) / kCg;   // the CTA group's index
+  const int npairs = static_cast<int>(gridDim.x) / kCg;  // CTA groups in the launch
+  // the leader's unit-ring and TMEM release barriers and stage barriers; in a pair also
+  // the peer's ring and the other CTA's abort flag
   const uint32_t uempty_c = mapa_shared(smem_u32(uempty), 0);
   const uint32_t tempty_c = mapa_shared(smem_u32(tempty), 0);
   const uint32_t full_c = mapa_shared(smem_u32(full), 0);
-  const uint32_t peer_ring_c = mapa_shared(smem_u32(const_cast<int*>(unit_ring)), 1);
-  const uint32_t peer_ufull_c = mapa_shared(smem_u32(ufull), 1);
-  const uint32_t peer_abort_c = mapa_shared(smem_u32(const_cast<int*>(abort_flag)), rank ^ 1u);
+  uint32_t peer_ring_c = 0, peer_ufull_c = 0, peer_abort_c = 0;
+  if constexpr (kPair) {
+    peer_ring_c = mapa_shared(smem_u32(const_cast<int*>(unit_ring)), 1);
+    peer_ufull_c = mapa_shared(smem_u32(ufull), 1);
+    peer_abort_c = mapa_shared(smem_u32(const_cast<int*>(abort_flag)), rank ^ 1u);
+  }
 
   if (warp == 0 && lane == 0) {
     // ------------------------------------------------------------ TMA producer
-    // Both CTAs load their halves of every stage: A rows m0 + 128 rank, B rows (output
-    // columns) n0 + 128 rank.  The leader takes the units (from the counter, or striding),
-    // publishes each to both CTAs' rings, and arms each stage's barrier for the bytes of
-    // both halves; the peer's copies count their bytes on that barrier too.
+    // In a pair both CTAs load their halves of every stage: A rows m0 + 128 rank, B rows
+    // (output columns) n0 + 128 rank.  The leader takes the units (from the counter, or
+    // striding), publishes each to both CTAs' rings, and arms each stage's barrier for the
+    // bytes of both halves; the peer's copies count their bytes on that barrier too.
     int s = 0;
     uint32_t ph = 0;
     long long issued = 0;
@@ -523,14 +561,16 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       if (rank == 0) {
         // publish the unit (or, past the end, the stop mark) to the roles of both CTAs
         u = next;
-        if (!mbar_wait_cluster(&uempty[us], uph ^ 1u, abort_flag)) {
+        if (!ring_wait<kPair>(&uempty[us], uph ^ 1u, abort_flag)) {
           ok = false;
           break;
         }
         unit_ring[us] = u;
-        st_cluster_u32(peer_ring_c + us * 4, static_cast<uint32_t>(u));
         mbar_arrive(&ufull[us]);
-        mbar_arrive_cluster(peer_ufull_c + us * 8);
+        if constexpr (kPair) {
+          st_cluster_u32(peer_ring_c + us * 4, static_cast<uint32_t>(u));
+          mbar_arrive_cluster(peer_ufull_c + us * 8);
+        }
       } else {
         if (!mbar_wait_cluster(&ufull[us], uph, abort_flag)) {
           ok = false;
@@ -558,19 +598,24 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       }
       int lu;
       const int g = batch_member(bt, u, &lu);
-      const Unit w = decode_unit(bt.p[g], lu);
+      const Unit w = decode_unit<kPair>(bt.p[g], lu);
       // rows past M (and columns past N) are read as zeros and never stored
-      const int32_t ya = w.mb * kTileM + static_cast<int32_t>(rank) * kBM;
-      const int32_t yb = w.nb * kBN + static_cast<int32_t>(rank) * kBHalf;
+      const int32_t ya = w.mb * L::tile_m + static_cast<int32_t>(rank) * kBM;
+      const int32_t yb = w.nb * kBN + static_cast<int32_t>(rank) * L::b_rows;
       for (int kb = w.kb0; kb < w.kb1; ++kb) {
         if (!mbar_wait(&empty[s], ph ^ 1u, abort_flag)) {
           ok = false;
           break;
         }
-        const uint32_t sa = smem_u32(smem + s * kStageBytes);
-        if (rank == 0) mbar_arrive_expect_tx(&full[s], 2 * kStageBytes);
-        tma_load_2d_pair(sa, &bt.a[g], full_c + s * 8, kb * kBKElems, ya);
-        tma_load_2d_pair(sa + kABytes, &bt.b[g], full_c + s * 8, kb * kBKElems, yb);
+        const uint32_t sa = smem_u32(smem + s * L::stage_bytes);
+        if (rank == 0) mbar_arrive_expect_tx(&full[s], kCg * L::stage_bytes);
+        if constexpr (kPair) {
+          tma_load_2d_pair(sa, &bt.a[g], full_c + s * 8, kb * kBKElems, ya);
+          tma_load_2d_pair(sa + kABytes, &bt.b[g], full_c + s * 8, kb * kBKElems, yb);
+        } else {
+          tma_load_2d(sa, &bt.a[g], smem_u32(&full[s]), kb * kBKElems, ya);
+          tma_load_2d(sa + kABytes, &bt.b[g], smem_u32(&full[s]), kb * kBKElems, yb);
+        }
         ++issued;
         if (++s == kStages) {
           s = 0;
@@ -578,7 +623,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
         }
       }
       if (ok && lazy) {
-        if (!mbar_wait_cluster(&uempty[u_slot], u_par, abort_flag)) {
+        if (!ring_wait<kPair>(&uempty[u_slot], u_par, abort_flag)) {
           ok = false;
           break;
         }
@@ -588,7 +633,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     if (!ok) {
       atomicOr(bt.status, kDevTimeout);
       *abort_flag = 1;
-      st_cluster_u32(peer_abort_c, 1);
+      if constexpr (kPair) st_cluster_u32(peer_abort_c, 1);
     }
     // Every issued copy must have landed before the CTAs may exit.  The leader's stage
     // barriers count both CTAs' bytes; after a timeout the peer cannot tell its own copies
@@ -596,16 +641,16 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     if (rank == 0) {
       for (long long i = issued > kStages ? issued - kStages : 0; i < issued; ++i)
         mbar_wait(&full[i % kStages], static_cast<uint32_t>((i / kStages) & 1), nullptr);
-    } else if (!ok) {
+    } else if (kPair && !ok) {
       const uint64_t t0 = globaltimer_ns();
       while (globaltimer_ns() - t0 < 200000ull) {
       }
     }
   } else if (warp == 1 && lane == 0 && rank == 0) {
     // ------------------------------------------------- MMA issuer (the leader's)
-    // 256 x 256 pair MMAs; a stage is released in both CTAs, and a finished chunk is
+    // In a pair: 256 x 256 MMAs; a stage is released in both CTAs, and a finished chunk
     // announced to both CTAs' epilogues, by multicast commits.
-    constexpr uint32_t idesc = make_idesc(kF8 ? 0u : 1u, kTileM, kBN);
+    constexpr uint32_t idesc = make_idesc(kF8 ? 0u : 1u, L::tile_m, kBN);
     int s = 0;
     uint32_t ph = 0;
     uint32_t c = 0;
@@ -628,11 +673,11 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       const int g = batch_member(bt, u, &lu);
       const int chunk_kb =
           bt.planned ? reinterpret_cast<volatile int*>(smem + L::chunk_offset)[g] : bt.p[g].chunk_kb;
-      const Unit w = decode_unit(bt.p[g], lu);
+      const Unit w = decode_unit<kPair>(bt.p[g], lu);
       for (int kc = w.kb0; kc < w.kb1 && ok; kc += chunk_kb) {
         const int kce = min(w.kb1, kc + chunk_kb);
         const uint32_t b = c & 1u, tph = (c >> 1) & 1u;
-        if (!mbar_wait_cluster(&tempty[b], tph ^ 1u, abort_flag)) {  // both CTAs' epilogues
+        if (!ring_wait<kPair>(&tempty[b], tph ^ 1u, abort_flag)) {  // every CTA's epilogue
           ok = false;
           break;
         }
@@ -644,7 +689,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
             break;
           }
           tc_fence_after();
-          const uint32_t a0 = smem_u32(smem + s * kStageBytes);
+          const uint32_t a0 = smem_u32(smem + s * L::stage_bytes);
           const uint32_t b0 = a0 + kABytes;
 #pragma unroll
           for (int k = 0; k < kBKBytes / 32; ++k) {
@@ -652,27 +697,27 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
             const uint64_t bd = make_sdesc_k_sw128(b0 + k * 32);
             const uint32_t accumulate = (kb > kc || k > 0) ? 1u : 0u;
             if (kF8)
-              tc_mma_f8(d, ad, bd, idesc, accumulate);
+              tc_mma_f8<kCg>(d, ad, bd, idesc, accumulate);
             else
-              tc_mma_f16(d, ad, bd, idesc, accumulate);
+              tc_mma_f16<kCg>(d, ad, bd, idesc, accumulate);
           }
-          tc_commit_pair(smem_u32(&empty[s]), 0x3);  // frees the stage in both CTAs
+          tc_commit<kCg>(smem_u32(&empty[s]), 0x3);  // frees the stage (in both CTAs)
           if (++s == kStages) {
             s = 0;
             ph ^= 1u;
           }
         }
         if (!ok) break;
-        tc_commit_pair(smem_u32(&tfull[b]), 0x3);  // chunk complete in TMEM buffer b
+        tc_commit<kCg>(smem_u32(&tfull[b]), 0x3);  // chunk complete in TMEM buffer b
         ++c;
       }
     }
     if (!ok) {
       atomicOr(bt.status, kDevTimeout);
       *abort_flag = 1;
-      st_cluster_u32(peer_abort_c, 1);
+      if constexpr (kPair) st_cluster_u32(peer_abort_c, 1);
     }
-    tc_commit_pair(smem_u32(drain), 0x1);  // every MMA issued has completed
+    tc_commit<kCg>(smem_u32(drain), 0x1);  // every MMA issued has completed
     mbar_wait(drain, 0, nullptr);
   } else if (warp == kFacWarp) {
     // --------------------------------------------------- chunk plan, column factors
@@ -681,7 +726,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       __syncwarp();
       if (lane == 0) mbar_arrive(chunkbar);
     }
-    factor_warp(bt, units, ufull, uempty_c, unit_ring, facbar, facfree,
+    factor_warp<kPair>(bt, units, ufull, uempty, uempty_c, unit_ring, facbar, facfree,
                 reinterpret_cast<float*>(smem + L::fac_offset), abort_flag, peer_abort_c, lane);
   } else if (warp >= kEpiWarp0) {
     // --------------------------------------------------------------- epilogue
@@ -695,13 +740,13 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     int us = 0;
     uint32_t uph = 0;
     for (int it = 0; ok; ++it) {
-      if (!__all_sync(0xFFFFFFFFu, mbar_wait_cluster(&ufull[us], uph, abort_flag))) {
+      if (!__all_sync(0xFFFFFFFFu, ring_wait<kPair>(&ufull[us], uph, abort_flag))) {
         ok = false;
         break;
       }
       const int u = unit_ring[us];
       __syncwarp();
-      if (lane == 0) mbar_arrive_cluster(uempty_c + us * 8);
+      if (lane == 0) leader_arrive<kPair>(&uempty[us], uempty_c + us * 8);
       if (++us == kUnitRing) {
         us = 0;
         uph ^= 1u;
@@ -712,11 +757,11 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
       const GemmParams& p = bt.p[g];
       const CUtensorMap* tma_y = &bt.y[g];
       const CUtensorMap* tma_ws = &bt.ws[g];
-      const Unit w = decode_unit(p, lu);
+      const Unit w = decode_unit<kPair>(p, lu);
       const int ckb =
           bt.planned ? reinterpret_cast<volatile int*>(smem + L::chunk_offset)[g] : p.chunk_kb;
       const int nch = (w.kb1 - w.kb0 + ckb - 1) / ckb;
-      const int64_t m0 = static_cast<int64_t>(w.mb) * kTileM + rank * kBM;  // this CTA's rows
+      const int64_t m0 = static_cast<int64_t>(w.mb) * L::tile_m + rank * kBM;  // this CTA's rows
       const int64_t n0 = static_cast<int64_t>(w.nb) * kBN;
       float* fac = fac_tab + (it & 1) * kBN;
       const int64_t row0 = m0 + q * 32;
@@ -741,7 +786,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
           if (s == 3) {
             tc_fence_before();
             __syncwarp();
-            if (lane == 0) mbar_arrive_cluster(tempty_c + b * 8);  // buffer b may take the next tile
+            if (lane == 0) leader_arrive<kPair>(&tempty[b], tempty_c + b * 8);  // b may take the next tile
           }
           const int64_t col0 = n0 + h * 128 + s * 32;
           if (row0 >= p.M || col0 >= p.N) continue;  // warp-uniform: nothing of this box exists
@@ -794,7 +839,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
           }
           tc_fence_before();
           __syncwarp();
-          if (lane == 0) mbar_arrive_cluster(tempty_c + b * 8);  // buffer b may take the next chunk
+          if (lane == 0) leader_arrive<kPair>(&tempty[b], tempty_c + b * 8);  // b may take the next chunk
           ++c;
         }
         if (!ok) break;
@@ -820,17 +865,21 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
     if (!ok) {
       atomicOr(bt.status, kDevTimeout);
       *abort_flag = 1;
-      st_cluster_u32(peer_abort_c, 1);
+      if constexpr (kPair) st_cluster_u32(peer_abort_c, 1);
     }
     if (lane == 0) bulk_wait_read<0>();  // no store still reads shared memory at exit
   }
 
-  // neither CTA leaves while the other may still reach its barriers, shared memory or TMEM
+  // neither CTA of a pair leaves while the other may still reach its barriers, shared
+  // memory or TMEM
   tc_fence_before();
-  cluster_sync();
+  if constexpr (kPair)
+    cluster_sync();
+  else
+    __syncthreads();
   if (warp == 1) {
     tc_fence_after();
-    tmem_dealloc_pair(tmem_base, kTmemCols);
+    tmem_dealloc<kCg>(tmem_base, kTmemCols);
   }
 }
 
@@ -953,9 +1002,10 @@ static int check_exact_range(int which, int64_t K, int bits, int G) {
   return SQ_OK;
 }
 
-// max_splits: 1 never splits K; 0 lets the SM count alone decide
-static int make_plan(int which, int64_t M, int64_t N, int64_t K, int bits, int G, int pairs,
-                     int max_splits, Plan* pl) {
+// Tiles of 128 (pair: 256) x 256 outputs spread over `workers` (SMs, or CTA pairs).
+// max_splits: 1 never splits K; 0 lets the worker count alone decide.
+static int make_plan(int which, int64_t M, int64_t N, int64_t K, int bits, int G, int workers,
+                     int max_splits, bool pair, Plan* pl) {
   const int st = check_exact_range(which, K, bits, G);
   if (st != SQ_OK) return st;
   const int64_t P = max_product(which, bits, G);
@@ -963,13 +1013,14 @@ static int make_plan(int which, int64_t M, int64_t N, int64_t K, int bits, int G
   const int bk = kBKBytes / pl->elem_bytes;
   pl->chunk_kb = static_cast<int>((kExactSum / P) / bk);
   if (pl->chunk_kb > (1 << 20)) pl->chunk_kb = 1 << 20;
-  pl->m_tiles = static_cast<int>((M + kTileM - 1) / kTileM);
+  const int tile_m = pair ? 2 * kBM : kBM;
+  pl->m_tiles = static_cast<int>((M + tile_m - 1) / tile_m);
   pl->n_tiles = static_cast<int>((N + kBN - 1) / kBN);
   pl->kb_total = static_cast<int>((K + bk - 1) / bk);
   const int64_t tiles = static_cast<int64_t>(pl->m_tiles) * pl->n_tiles;
   int splits = 1;
-  if (max_splits != 1 && tiles < pairs && pl->kb_total >= 4) {
-    splits = static_cast<int>(pairs / tiles);
+  if (max_splits != 1 && tiles < workers && pl->kb_total >= 4) {
+    splits = static_cast<int>(workers / tiles);
     if (splits > pl->kb_total / 2) splits = pl->kb_total / 2;
     if (max_splits > 1 && splits > max_splits) splits = max_splits;
     if (splits < 1) splits = 1;
@@ -987,13 +1038,13 @@ static size_t split_ws_bytes(int64_t M, int64_t N) {
 // The layer launch's workspace starts with the unit counter of its dynamic schedule.
 constexpr size_t kSchedBytes = 256;
 
-template <int kF8, bool kMulti>
+template <int kF8, bool kMulti, bool kPair>
 static int configure_kernel(int dev) {
   static bool done[64] = {};
   if (dev >= 0 && dev < 64 && done[dev]) return SQ_OK;
-  const cudaError_t err = cudaFuncSetAttribute(shiftmm_kernel<kF8, kMulti>,
+  const cudaError_t err = cudaFuncSetAttribute(shiftmm_kernel<kF8, kMulti, kPair>,
                                                cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                               static_cast<int>(Smem::bytes));
+                                               static_cast<int>(Smem<kPair>::bytes));
   if (err != cudaSuccess) return cuda_fail(err, "cudaFuncSetAttribute");
   if (dev >= 0 && dev < 64) done[dev] = true;
   return SQ_OK;
@@ -1009,17 +1060,23 @@ static int device_pairs(int* dev_out) {
   if (dev_out) *dev_out = dev;
   if (dev >= 0 && dev < 64 && cached[dev] > 0) return cached[dev];
   int pairs = sms / 2;
-  if (configure_kernel<1, false>(dev) == SQ_OK) {
+  if (configure_kernel<1, false, true>(dev) == SQ_OK) {
+    cudaLaunchAttribute at[1];
+    at[0].id = cudaLaunchAttributeClusterDimension;
+    at[0].val.clusterDim.x = 2;
+    at[0].val.clusterDim.y = 1;
+    at[0].val.clusterDim.z = 1;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(2 * pairs);
     cfg.blockDim = dim3(kThreads);
-    cfg.dynamicSmemBytes = Smem::bytes;
+    cfg.dynamicSmemBytes = Smem<true>::bytes;
+    cfg.attrs = at;
+    cfg.numAttrs = 1;
     int n = 0;
-    if (cudaOccupancyMaxActiveClusters(&n, shiftmm_kernel<1, false>, &cfg) == cudaSuccess && n > 0 &&
-        n < pairs)
-      pairs = n;
-    else
+    if (cudaOccupancyMaxActiveClusters(&n, shiftmm_kernel<1, false, true>, &cfg) != cudaSuccess)
       cudaGetLastError();  // an unanswered query leaves no error behind
+    else if (n > 0 && n < pairs)
+      pairs = n;
   }
   if (pairs < 1) pairs = 1;
   if (dev >= 0 && dev < 64) cached[dev] = pairs;
@@ -1094,19 +1151,42 @@ static int check_job(const GemmJob& j, int bits, int G, int32_t* dev_status, cud
 // Tiles and K splits of one checked GEMM: the SM count decides the splits, up to
 // max_splits, and a split needs a workspace for the [M, N] int32 partial sums (added by TMA
 // into N-element rows, which must stay 16-byte aligned).
-static int plan_job(const GemmJob& j, int bits, int G, int pairs, int max_splits, Plan* pl) {
-  const int st = make_plan(j.which, j.M, j.N, j.K, bits, G, pairs, max_splits, pl);
+static int plan_job(const GemmJob& j, int bits, int G, int workers, int max_splits, bool pair,
+                    Plan* pl) {
+  const int st = make_plan(j.which, j.M, j.N, j.K, bits, G, workers, max_splits, pair, pl);
   if (st != SQ_OK || pl->splits <= 1) return st;
   if (j.ws == nullptr || j.ws_bytes < split_ws_bytes(j.M, j.N) || !aligned16(j.ws) || j.N % 4 != 0)
-    return make_plan(j.which, j.M, j.N, j.K, bits, G, pairs, 1, pl);
+    return make_plan(j.which, j.M, j.N, j.K, bits, G, workers, 1, pair, pl);
   return SQ_OK;
+}
+
+// Pair tiles where a launch's units run long K loops, so that the tensor core sets the
+// pace; with short K loops the epilogue does, and single tiles run it faster.  Decided
+// from single-tile plans: the average K blocks per unit.  Measured on layer launches:
+// pairs 18% faster at 118 K blocks (16384 x 4096 x 11008), 2% at 27 (12608 x 768 x 3072),
+// even at 25, 4% slower at 14.5 and 18% slower at 5 (12544 x 2304 x 256, E4M3).
+constexpr int kPairMinKb = 26;
+static bool pair_mode(const GemmJob* const* jobs, int n, int bits, int G, int sms, int pairs) {
+  if (pairs <= 0) return false;
+  double units = 0.0, kb = 0.0;
+  for (int i = 0; i < n; ++i) {
+    const GemmJob& j = *jobs[i];
+    if (j.M <= 0 || j.N <= 0 || j.K <= 0) continue;
+    Plan pl;
+    if (make_plan(j.which, j.M, j.N, j.K, bits, G, sms, 0, false, &pl) != SQ_OK) continue;
+    const double u = static_cast<double>(pl.m_tiles) * pl.n_tiles * pl.splits;
+    units += u;
+    kb += u * pl.kb_per_split;
+  }
+  return units > 0.0 && kb >= kPairMinKb * units;
 }
 
 // Sharing the launch with other GEMMs, a split GEMM needs fewer splits: just enough that
 // its units stay well inside the launch's expected length.  Every split adds the whole
 // output once more to the L2 reductions, whose throughput is far below a plain store's.
 // Unit cost model, in K-block times: the K loop plus about 8 for the epilogue.
-static int balance_splits(GemmJob* const* jobs, int n, int bits, int G, int pairs, Plan* plans) {
+static int balance_splits(GemmJob* const* jobs, int n, int bits, int G, int workers, bool pair,
+                          Plan* plans) {
   if (n <= 1) return SQ_OK;
   constexpr double kEpiKb = 8.0;
   double work = 0.0;  // the batch's total cost, with every split GEMM at its maximum
@@ -1121,10 +1201,10 @@ static int balance_splits(GemmJob* const* jobs, int n, int bits, int G, int pair
       const double kbs = static_cast<double>((plans[g].kb_total + s - 1) / s);
       const double w = work - tiles * plans[g].splits * (plans[g].kb_per_split + kEpiKb) +
                        tiles * s * (kbs + kEpiKb);
-      if (kbs + kEpiKb <= 0.8 * w / pairs) break;
+      if (kbs + kEpiKb <= 0.8 * w / workers) break;
     }
     if (s < plans[g].splits) {
-      const int st = plan_job(*jobs[g], bits, G, pairs, s, &plans[g]);
+      const int st = plan_job(*jobs[g], bits, G, workers, s, pair, &plans[g]);
       if (st != SQ_OK) return st;
     }
   }
@@ -1133,11 +1213,12 @@ static int balance_splits(GemmJob* const* jobs, int n, int bits, int G, int pair
 
 // Slot g of the batch for one planned GEMM: tensor maps and parameters.
 static int prepare_job(const GemmJob& j, const Plan* pl, int bits, int G, int32_t* dev_status,
-                       GemmBatch* bt, int g) {
+                       bool pair, GemmBatch* bt, int g) {
   int st;
   const int eb = pl->elem_bytes;
   if ((st = make_operand_map(&bt->a[g], j.a, j.M, j.K, j.lda, eb, kBM)) != SQ_OK) return st;
-  if ((st = make_operand_map(&bt->b[g], j.b, j.N, j.K, j.ldb, eb, kBHalf)) != SQ_OK) return st;
+  if ((st = make_operand_map(&bt->b[g], j.b, j.N, j.K, j.ldb, eb, pair ? kBN / 2 : kBN)) != SQ_OK)
+    return st;
   GemmParams& p = bt->p[g];
   p.M = static_cast<int>(j.M);
   p.N = static_cast<int>(j.N);
@@ -1174,18 +1255,41 @@ static int prepare_job(const GemmJob& j, const Plan* pl, int bits, int G, int32_
   return st;
 }
 
-template <int kF8, bool kMulti>
+template <int kF8, bool kMulti, bool kPair>
 static int launch_kernel(const GemmBatch& bt, int grid, int dev, cudaStream_t s) {
-  const int st = configure_kernel<kF8, kMulti>(dev);
+  const int st = configure_kernel<kF8, kMulti, kPair>(dev);
   if (st != SQ_OK) return st;
-  shiftmm_kernel<kF8, kMulti><<<grid, kThreads, Smem::bytes, s>>>(bt);
-  const cudaError_t err = cudaGetLastError();
+  cudaError_t err;
+  if constexpr (kPair) {
+    cudaLaunchAttribute at[1];
+    at[0].id = cudaLaunchAttributeClusterDimension;
+    at[0].val.clusterDim.x = 2;
+    at[0].val.clusterDim.y = 1;
+    at[0].val.clusterDim.z = 1;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(grid);
+    cfg.blockDim = dim3(kThreads);
+    cfg.dynamicSmemBytes = Smem<true>::bytes;
+    cfg.stream = s;
+    cfg.attrs = at;
+    cfg.numAttrs = 1;
+    err = cudaLaunchKernelEx(&cfg, shiftmm_kernel<kF8, kMulti, true>, bt);
+    if (err == cudaSuccess) err = cudaGetLastError();
+  } else {
+    shiftmm_kernel<kF8, kMulti, false><<<grid, kThreads, Smem<false>::bytes, s>>>(bt);
+    err = cudaGetLastError();
+  }
   return err == cudaSuccess ? SQ_OK : cuda_fail(err, "shiftmm_kernel launch");
 }
 
 template <int kF8>
-static int launch_variant(const GemmBatch& bt, int grid, int dev, cudaStream_t s, bool multi) {
-  return multi ? launch_kernel<kF8, true>(bt, grid, dev, s) : launch_kernel<kF8, false>(bt, grid, dev, s);
+static int launch_variant(const GemmBatch& bt, int grid, int dev, cudaStream_t s, bool multi,
+                          bool pair) {
+  if (pair)
+    return multi ? launch_kernel<kF8, true, true>(bt, grid, dev, s)
+                 : launch_kernel<kF8, false, true>(bt, grid, dev, s);
+  return multi ? launch_kernel<kF8, true, false>(bt, grid, dev, s)
+               : launch_kernel<kF8, false, false>(bt, grid, dev, s);
 }
 
 // Checks, plans and launches up to kMaxBatch GEMMs (all with the same bits / n_groups) as
@@ -1206,21 +1310,25 @@ static int run_jobs(GemmJob* jobs, int njobs, int bits, int G, int32_t* dev_stat
   }
   if (nlive == 0) return SQ_OK;
   int dev = 0;
-  const int pairs = device_pairs(&dev);
-  if (pairs <= 0) return fail(SQ_ECUDA, "%s: no current CUDA device", job_name(jobs[live[0]].which));
+  const int sms = device_sms(&dev);
+  if (sms <= 0) return fail(SQ_ECUDA, "%s: no current CUDA device", job_name(jobs[live[0]].which));
   GemmBatch bt;
   memset(&bt, 0, sizeof(bt));
   Plan plans[kMaxBatch];
   GemmJob* lj[kMaxBatch];
+  for (int g = 0; g < nlive; ++g) lj[g] = &jobs[live[g]];
+  const int pairs = device_pairs(nullptr);
+  const bool pair = pair_mode(lj, nlive, bits, G, sms, pairs);
+  const int workers = pair ? pairs : sms;  // CTA groups resident at once
   for (int g = 0; g < nlive; ++g) {
-    lj[g] = &jobs[live[g]];
-    const int st = plan_job(*lj[g], bits, G, pairs, 0, &plans[g]);
+    const int st = plan_job(*lj[g], bits, G, workers, 0, pair, &plans[g]);
     if (st != SQ_OK) return st;
   }
-  int st = balance_splits(lj, nlive, bits, G, pairs, plans);
+  int st = balance_splits(lj, nlive, bits, G, workers, pair, plans);
   if (st != SQ_OK) return st;
   for (int g = 0; g < nlive; ++g)
-    if ((st = prepare_job(*lj[g], &plans[g], bits, G, dev_status, &bt, g)) != SQ_OK) return st;
+    if ((st = prepare_job(*lj[g], &plans[g], bits, G, dev_status, pair, &bt, g)) != SQ_OK)
+      return st;
   // longest K loop per unit first: the short units then fill in behind the long ones
   for (int a = 0; a < nlive; ++a)
     for (int b = a + 1; b < nlive; ++b)
@@ -1267,27 +1375,29 @@ static int run_jobs(GemmJob* jobs, int njobs, int bits, int G, int32_t* dev_stat
     err = cudaMemsetAsync(zero_from, 0, static_cast<size_t>(zero_end - zero_from), s);
     if (err != cudaSuccess) return cuda_fail(err, "cudaMemsetAsync");
   }
-  // two CTAs per pair; a cap on the CTAs leaves at least one pair
-  int npairs = units < pairs ? units : pairs;
-  if (max_ctas > 0 && npairs > max_ctas / 2) npairs = max_ctas / 2 > 0 ? max_ctas / 2 : 1;
-  const int grid = 2 * npairs;
-  // A pair holds up to about stages / K-blocks + 2 units of the last (shortest) GEMM at
-  // once: its operand ring and two TMEM buffers.  Over that many final waves it takes
-  // one unit at a time, so the pairs run out of work together.
+  // CTA groups (pairs, or single CTAs); a cap on the CTAs leaves at least one group
+  const int cg = pair ? 2 : 1;
+  int ngroups = units < workers ? units : workers;
+  if (max_ctas > 0 && ngroups > max_ctas / cg) ngroups = max_ctas / cg > 0 ? max_ctas / cg : 1;
+  const int grid = cg * ngroups;
+  // A CTA group holds up to about stages / K-blocks + 2 units of the last (shortest) GEMM
+  // at once: its operand ring and two TMEM buffers.  Over that many final waves it takes
+  // one unit at a time, so the groups run out of work together.
   {
     const int kb = plans[nlive - 1].kb_per_split > 0 ? plans[nlive - 1].kb_per_split : 1;
-    const int depth = 2 + (Smem::stages + kb - 1) / kb;
-    const long long from = static_cast<long long>(units) - static_cast<long long>(depth) * npairs;
+    const int stages = pair ? Smem<true>::stages : Smem<false>::stages;
+    const int depth = 2 + (stages + kb - 1) / kb;
+    const long long from = static_cast<long long>(units) - static_cast<long long>(depth) * ngroups;
     bt.lazy_from = from > 0 ? static_cast<int>(from) : 0;
   }
-  st = plans[0].elem_bytes == 1 ? launch_variant<1>(bt, grid, dev, s, multi)
-                                : launch_variant<0>(bt, grid, dev, s, multi);
+  st = plans[0].elem_bytes == 1 ? launch_variant<1>(bt, grid, dev, s, multi, pair)
+                                : launch_variant<0>(bt, grid, dev, s, multi, pair);
   if (st != SQ_OK) return st;
   for (int g = 0; g < nlive; ++g) {
     if (!bt.p[g].ws) continue;
     const int64_t quads = static_cast<int64_t>(bt.p[g].M) * (bt.p[g].N / 4);
     int64_t blocks = (quads + 255) / 256;
-    if (blocks > static_cast<int64_t>(pairs) * 32) blocks = static_cast<int64_t>(pairs) * 32;
+    if (blocks > static_cast<int64_t>(sms) * 16) blocks = static_cast<int64_t>(sms) * 16;
     splitk_finalize_kernel<<<static_cast<unsigned>(blocks), 256, 0, s>>>(bt.p[g]);
     err = cudaGetLastError();
     if (err != cudaSuccess) return cuda_fail(err, "splitk_finalize_kernel launch");
@@ -1323,13 +1433,17 @@ static void layer_jobs(const sq_layer_gemms* a, GemmJob jobs[3], int mask) {
 
 // Bytes of split-K workspace each GEMM of the layer would use (0: it would not split),
 // a multiple of 256 bytes.
-static void layer_ws_need(const GemmJob jobs[3], int bits, int G, int pairs, size_t need[3]) {
+static void layer_ws_need(const GemmJob jobs[3], int bits, int G, int sms, int pairs,
+                          size_t need[3]) {
+  const GemmJob* jp[3] = {&jobs[0], &jobs[1], &jobs[2]};
+  const bool pair = pair_mode(jp, 3, bits, G, sms, pairs);
   for (int i = 0; i < 3; ++i) {
     need[i] = 0;
     const GemmJob& j = jobs[i];
     if (j.M <= 0 || j.N <= 0 || j.K <= 0 || j.N % 4 != 0) continue;
     Plan pl;
-    if (make_plan(j.which, j.M, j.N, j.K, bits, G, pairs, 0, &pl) != SQ_OK) continue;
+    if (make_plan(j.which, j.M, j.N, j.K, bits, G, pair ? pairs : sms, 0, pair, &pl) != SQ_OK)
+      continue;
     if (pl.splits > 1) need[i] = split_ws_bytes(j.M, j.N);
   }
 }
@@ -1337,12 +1451,12 @@ static void layer_ws_need(const GemmJob jobs[3], int bits, int G, int pairs, siz
 // The layer workspace: the unit counter, then a split-K region for each GEMM that would
 // split, as far as the workspace reaches.  Returns the counter (null without a usable
 // workspace: the launch then strides over its units and splits nothing).
-static int* assign_layer_ws(GemmJob jobs[3], int bits, int G, int pairs, void* workspace,
+static int* assign_layer_ws(GemmJob jobs[3], int bits, int G, int sms, int pairs, void* workspace,
                             size_t workspace_bytes) {
   if (workspace == nullptr || workspace_bytes < kSchedBytes || !aligned16(workspace)) return nullptr;
-  if (pairs > 0) {
+  if (sms > 0) {
     size_t need[3];
-    layer_ws_need(jobs, bits, G, pairs, need);
+    layer_ws_need(jobs, bits, G, sms, pairs, need);
     size_t off = kSchedBytes;
     for (int i = 0; i < 3; ++i) {
       if (need[i] == 0 || off + need[i] > workspace_bytes) continue;
@@ -1429,10 +1543,18 @@ extern "C" size_t shiftquant_gemm_workspace_bytes(int which, int64_t M, int64_t 
   if (which < 0 || which > 2 || !bits_ok(bits) || !groups_ok(n_groups) || M <= 0 || N <= 0 ||
       K <= 0)
     return 0;
+  const int sms = device_sms(nullptr);
+  if (sms <= 0) return 0;
   const int pairs = device_pairs(nullptr);
-  if (pairs <= 0) return 0;
+  GemmJob j{};
+  j.which = which;
+  j.M = M;
+  j.N = N;
+  j.K = K;
+  const GemmJob* jp = &j;
+  const bool pair = pair_mode(&jp, 1, bits, n_groups, sms, pairs);
   Plan pl;
-  if (make_plan(which, M, N, K, bits, n_groups, pairs, 0, &pl) != SQ_OK) return 0;
+  if (make_plan(which, M, N, K, bits, n_groups, pair ? pairs : sms, 0, pair, &pl) != SQ_OK) return 0;
   return pl.splits > 1 ? split_ws_bytes(M, N) : 0;
 }
 
@@ -1469,16 +1591,19 @@ extern "C" sq_status shiftquant_gemm_layer(const sq_layer_gemms* args, void* wor
     return fail(SQ_EINVAL, "gemm_layer: gemm_mask must be in [0, 7] and max_ctas >= 0");
   GemmJob jobs[3];
   layer_jobs(args, jobs, args->gemm_mask);
+  const int sms = device_sms(nullptr);
   const int pairs = device_pairs(nullptr);
-  int* sched = assign_layer_ws(jobs, args->bits, args->n_groups, pairs, workspace, workspace_bytes);
+  int* sched =
+      assign_layer_ws(jobs, args->bits, args->n_groups, sms, pairs, workspace, workspace_bytes);
   return run_jobs(jobs, 3, args->bits, args->n_groups, dev_status, stream, sched, args->max_ctas);
 }
 
 extern "C" size_t shiftquant_gemm_layer_workspace_bytes(int64_t M, int64_t K, int64_t N, int bits,
                                                         int n_groups) {
   if (!bits_ok(bits) || !groups_ok(n_groups)) return 0;
+  const int sms = device_sms(nullptr);
+  if (sms <= 0) return 0;
   const int pairs = device_pairs(nullptr);
-  if (pairs <= 0) return 0;
   sq_layer_gemms a;
   memset(&a, 0, sizeof(a));
   a.M = M;
@@ -1487,7 +1612,7 @@ extern "C" size_t shiftquant_gemm_layer_workspace_bytes(int64_t M, int64_t K, in
   GemmJob jobs[3];
   layer_jobs(&a, jobs, 0);
   size_t need[3];
-  layer_ws_need(jobs, bits, n_groups, pairs, need);
+  layer_ws_need(jobs, bits, n_groups, sms, pairs, need);
   return kSchedBytes + need[0] + need[1] + need[2];
 }
 
@@ -1497,8 +1622,9 @@ extern "C" int shiftquant_gemm_layer_kernel_launches(int64_t M, int64_t K, int64
   if (!bits_ok(bits) || !groups_ok(n_groups) || M < 0 || K < 0 || N < 0 || gemm_mask < 0 ||
       gemm_mask > 7)
     return -1;
+  const int sms = device_sms(nullptr);
+  if (sms <= 0) return -1;
   const int pairs = device_pairs(nullptr);
-  if (pairs <= 0) return -1;
   sq_layer_gemms a;
   memset(&a, 0, sizeof(a));
   a.M = M;
@@ -1507,19 +1633,19 @@ extern "C" int shiftquant_gemm_layer_kernel_launches(int64_t M, int64_t K, int64
   GemmJob jobs[3];
   layer_jobs(&a, jobs, gemm_mask);
   // the plan looks at the workspace's size and alignment only: a stand-in address serves
-  assign_layer_ws(jobs, bits, n_groups, pairs, workspace_bytes ? reinterpret_cast<void*>(4096) : nullptr,
+  assign_layer_ws(jobs, bits, n_groups, sms, pairs, workspace_bytes ? reinterpret_cast<void*>(4096) : nullptr,
                   workspace_bytes);
   Plan plans[kMaxBatch];
   GemmJob* lj[kMaxBatch];
   int n = 0;
-  for (int i = 0; i < 3; ++i) {
-    if (jobs[i].M == 0 || jobs[i].N == 0 || jobs[i].K == 0) continue;
-    lj[n] = &jobs[i];
-    if (plan_job(jobs[i], bits, n_groups, pairs, 0, &plans[n]) != SQ_OK) return -1;
-    ++n;
-  }
+  for (int i = 0; i < 3; ++i)
+    if (jobs[i].M != 0 && jobs[i].N != 0 && jobs[i].K != 0) lj[n++] = &jobs[i];
   if (n == 0) return 0;
-  if (balance_splits(lj, n, bits, n_groups, pairs, plans) != SQ_OK) return -1;
+  const bool pair = pair_mode(lj, n, bits, n_groups, sms, pairs);
+  const int workers = pair ? pairs : sms;
+  for (int g = 0; g < n; ++g)
+    if (plan_job(*lj[g], bits, n_groups, workers, 0, pair, &plans[g]) != SQ_OK) return -1;
+  if (balance_splits(lj, n, bits, n_groups, workers, pair, plans) != SQ_OK) return -1;
   int launches = 1;
   for (int g = 0; g < n; ++g) launches += plans[g].splits > 1;
   return launches;
