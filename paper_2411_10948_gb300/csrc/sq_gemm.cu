@@ -19,19 +19,22 @@
 // channels in the last group (the usual case: tau_0 set by a few outlier channels) an
 // 8-bit chunk grows from 2 K blocks to about 10.
 //
-// One CTA per SM, persistent over output tiles of 128 x 256:
+// Persistent over output tiles: one CTA per SM with 128 x 256 tiles, or (for launches
+// whose K loops are long) 2-CTA clusters with 256 x 256 tiles and cta_group::2 MMAs.
+// The roles of a CTA:
 //   warp 0      TMA producer: A and B tiles (128-byte rows, 128-byte swizzle) into a
-//               4-stage shared-memory ring
-//   warp 1      TMEM allocation and the MMA issuer (one thread)
+//               shared-memory ring of 4 (pair: 6) stages
+//   warp 1      TMEM allocation and the MMA issuer (one thread; a pair's leader only)
 //   warp 2      the chunk plan (see above); then the dequantizing column factors of each
 //               tile, ahead of the epilogue
 //   warps 4-11  epilogue: tcgen05.ld, int32 accumulation across chunks, dequantizing
 //               multiply, TMA stores of 32 x 32 boxes (or int32 TMA reductions into a
 //               split-K workspace; plain stores where the output rows are not 16-byte
 //               aligned)
-// Work units reach the three roles through a small shared-memory ring that the producer
-// fills: with a scheduling counter the producer takes each next unit from it (units are
-// handed out in list order as CTAs free up), without one it strides over the list.
+// Work units reach the roles through a small shared-memory ring that the producer of the
+// CTA (a pair's leader) fills: with a scheduling counter it takes each next unit from it
+// (units are handed out in list order as CTAs free up), without one it strides over the
+// list.
 // Every wait is bounded (about 1 s); on expiry the kernel records SQ_DEV_TIMEOUT,
 // drains its own copies and MMAs, frees TMEM and returns.
 #include <cuda.h>
