@@ -11,7 +11,8 @@ then reading another 256 MiB buffer, so the step starts with no input in L2 and 
 dirty flush data that the step would otherwise have to write back.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
-                  [--workload conv3x3|wgrad_small|vit_mlp|large_linear|large_linear_8bit|vit_block]
+                  [--workload conv3x3|wgrad_small|vit_mlp|large_linear|large_linear_8bit|vit_block|
+                              large_linear_t4096]
 
 Prints one JSON line (rank 0).  --impl reference times the plain CPU oracle of the
 same definitions on the host cores instead (a bounded sample of the same workload).

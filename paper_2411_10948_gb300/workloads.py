@@ -54,7 +54,9 @@ C3_GRAD = ("grad", "laplace", 2.0, 0.0, 1.0)
 
 
 def workload(name: str) -> Workload:
-    """The five workloads: wgrad_small, conv3x3, vit_mlp, large_linear(_8bit), vit_block."""
+    """The workloads: wgrad_small, conv3x3, vit_mlp, large_linear(_8bit), vit_block, and
+    large_linear_t4096 (large_linear's layers on 4096 tokens: a profiling-size case of the
+    same kernels)."""
     if name == "wgrad_small":
         g = ("grad", "normal", 1.5, 0.01, 100.0)
         return Workload(name, "4-bit wgrad/dgrad, dY and X [256, 512], W [512, 512]",
@@ -69,12 +71,13 @@ def workload(name: str) -> Workload:
         return Workload(name, "ViT-B MLP fc1 768->3072 and fc2 3072->768, 12608 tokens, 6-bit",
                         [LayerSpec("fc1", M, 768, 3072, 6, 4, C3_ACT, C3_GRAD),
                          LayerSpec("fc2", M, 3072, 768, 6, 4, C3_ACT, C3_GRAD)])
-    if name in ("large_linear", "large_linear_8bit"):
+    if name in ("large_linear", "large_linear_8bit", "large_linear_t4096"):
         bits = 8 if name.endswith("8bit") else 6
+        T = 4096 if name.endswith("t4096") else 16384
         g = ("grad", "laplace", 2.5, 0.001, 1.0e4)
-        return Workload(name, f"16384 tokens, 4096->11008 and 11008->4096, {bits}-bit",
-                        [LayerSpec("up", 16384, 4096, 11008, bits, 4, C3_ACT, g),
-                         LayerSpec("down", 16384, 11008, 4096, bits, 4, C3_ACT, g)])
+        return Workload(name, f"{T} tokens, 4096->11008 and 11008->4096, {bits}-bit",
+                        [LayerSpec("up", T, 4096, 11008, bits, 4, C3_ACT, g),
+                         LayerSpec("down", T, 11008, 4096, bits, 4, C3_ACT, g)])
     if name == "vit_block":
         M = 64 * 197
         return Workload(name, "ViT-B/16 block (QKV, proj, fc1, fc2), batch 64 x 197 tokens, 6-bit",
@@ -86,7 +89,7 @@ def workload(name: str) -> Workload:
 
 
 WORKLOADS = ("wgrad_small", "conv3x3", "vit_mlp", "large_linear", "large_linear_8bit",
-             "vit_block")
+             "vit_block", "large_linear_t4096")
 
 
 def tensor_seed(seed: int, layer_idx: int, which: str) -> int:
