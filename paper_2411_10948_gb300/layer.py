@@ -259,3 +259,74 @@ class CapturedStep:
 
     def replay(self) -> None:
         self.graph.replay()
+
+
+class HostPipeline:
+    """Training steps fed from pinned host memory and returned to it.  Each step copies
+    the inputs X, W and dY of every layer to the device, runs every layer's step
+    (`QuantLinear.step_concurrent`, replayed as one CUDA graph), and copies Y, dX and dW
+    back.  Two sets of device buffers alternate between steps.  Step i+1's inputs copy in
+    on one stream and step i-1's outputs copy out on another while step i computes, so the
+    host link's two directions, not the GPU, set the pace.
+
+    shapes: (M, K, N) per layer.  The stochastic-rounding seed of a slot is fixed when its
+    graph is captured (slot s uses seed + s)."""
+
+    def __init__(self, shapes, bits, n_groups, device="cuda", seed=0x5EED):
+        dev = torch.device(device)
+        self.shapes = list(shapes)
+        self.s_in = torch.cuda.Stream(device=dev)
+        self.s_comp = torch.cuda.Stream(device=dev)
+        self.s_out = torch.cuda.Stream(device=dev)
+        self.slots = []
+        for k in range(2):
+            layers = [QuantLinear(M, K, N_, bits, n_groups, dev) for (M, K, N_) in self.shapes]
+            inputs = [(torch.zeros((M, K), dtype=torch.float32, device=dev),
+                       torch.zeros((K, N_), dtype=torch.float32, device=dev),
+                       torch.zeros((M, N_), dtype=torch.float32, device=dev))
+                      for (M, K, N_) in self.shapes]
+            streams = [[torch.cuda.Stream(device=dev) for _ in range(4)] for _ in layers]
+
+            def step(layers=layers, inputs=inputs, streams=streams, sd=seed + k):
+                for lay, (x, w, dy), ss in zip(layers, inputs, streams):
+                    lay.step_concurrent(x, w, dy, sd, ss)
+
+            self.slots.append({"layers": layers, "inputs": inputs, "graph": CapturedStep(step),
+                               "in_ready": torch.cuda.Event(), "done": torch.cuda.Event(),
+                               "out_copied": torch.cuda.Event()})
+
+    def run(self, host_inputs, host_outputs) -> torch.cuda.Event:
+        """Queue one step per entry.  host_inputs[i]: (x, w, dy) per layer, pinned float32
+        host tensors; host_outputs[i]: (y, dx, dw) per layer, pinned float32 host tensors
+        that receive step i's results.  Returns an event recorded after the last copy back
+        (synchronize on it before reading the host outputs)."""
+        cur = torch.cuda.current_stream()
+        for s in (self.s_in, self.s_comp, self.s_out):
+            s.wait_stream(cur)
+        for i, (hin, hout) in enumerate(zip(host_inputs, host_outputs)):
+            sl = self.slots[i % 2]
+            self.s_in.wait_event(sl["done"])        # the slot's last step no longer reads them
+            with torch.cuda.stream(self.s_in):
+                for dev_in, host_in in zip(sl["inputs"], hin):
+                    for d, h in zip(dev_in, host_in):
+                        d.copy_(h, non_blocking=True)
+                sl["in_ready"].record(self.s_in)
+            self.s_comp.wait_event(sl["in_ready"])
+            self.s_comp.wait_event(sl["out_copied"])  # the slot's last outputs have left
+            with torch.cuda.stream(self.s_comp):
+                sl["graph"].replay()
+                sl["done"].record(self.s_comp)
+            self.s_out.wait_event(sl["done"])
+            with torch.cuda.stream(self.s_out):
+                for lay, host_out in zip(sl["layers"], hout):
+                    for h, d in zip(host_out, (lay.y, lay.dx, lay.dw)):
+                        h.copy_(d, non_blocking=True)
+                sl["out_copied"].record(self.s_out)
+        end = torch.cuda.Event(enable_timing=True)
+        end.record(self.s_out)
+        for s in (self.s_in, self.s_comp, self.s_out):
+            cur.wait_stream(s)
+        return end
+
+    def status_ok(self) -> bool:
+        return all(int(l.status.item()) == 0 for sl in self.slots for l in sl["layers"])

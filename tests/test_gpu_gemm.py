@@ -203,6 +203,34 @@ def test_concurrent_step_equals_serial_step():
         np.testing.assert_array_equal(a.cpu().numpy(), b.cpu().numpy())
 
 
+def test_host_pipeline_equals_device_steps():
+    # layer.HostPipeline (copies in, the captured step, copies back, on three streams with
+    # two alternating buffer sets): every step's host outputs equal a device-resident step
+    # on the same inputs and seed
+    shapes = [(3000, 640, 384), (3000, 384, 640)]
+    bits, G, seed, steps = 6, 4, 0x5EED, 5
+    pipe = L.HostPipeline(shapes, bits, G, "cuda", seed=seed)
+    host_in, host_out = [], []
+    for i in range(steps):
+        rng = np.random.default_rng(100 + i)
+        host_in.append([tuple(torch.from_numpy(a).pin_memory() for a in layer_inputs(rng, *sh))
+                        for sh in shapes])
+        host_out.append([tuple(torch.empty(shp, dtype=torch.float32).pin_memory()
+                               for shp in ((M, Nn), (M, K), (K, Nn)))
+                         for (M, K, Nn) in shapes])
+    pipe.run(host_in, host_out).synchronize()
+    assert pipe.status_ok()
+    ref = [L.QuantLinear(M, K, Nn, bits, G, "cuda") for (M, K, Nn) in shapes]
+    for i in range(steps):
+        for li, lay in enumerate(ref):
+            x, w, dy = (t.cuda() for t in host_in[i][li])
+            lay.step(x, w, dy, seed + i % 2)
+            torch.cuda.synchronize()
+            assert lay.status.item() == 0
+            for got, want in zip(host_out[i][li], (lay.y, lay.dx, lay.dw)):
+                np.testing.assert_array_equal(got.numpy(), want.cpu().numpy())
+
+
 @pytest.mark.parametrize("M,K,Nn", [(5, 3, 7), (300, 1000, 513), (4096, 64, 96), (2000, 700, 256)])
 @pytest.mark.parametrize("bits", [4, 6, 8])
 def test_layer_gemms_in_one_launch_match_oracle(M, K, Nn, bits):
