@@ -89,9 +89,10 @@ struct Smem {
   // full, empty, tfull, tempty, fac, drain, unit ring full / empty, fac free, chunk plan
   static constexpr int num_bars = 2 * stages + 2 + 2 + 2 + 1 + 2 * kUnitRing + 2 + 1;
   static constexpr int ring_offset = bar_offset + num_bars * 8 + 16;  // after TMEM slot, flag
-  static constexpr int chunk_offset = ring_offset + kUnitRing * 4;  // K blocks per chunk, per GEMM
+  static constexpr int chunk_offset = ring_offset + kUnitRing * 32;  // K blocks per chunk, per GEMM
   static constexpr size_t bytes = chunk_offset + 4 * 4;
   static_assert(bytes <= 232448, "shared memory beyond the 227 KB per-CTA limit");
+  static_assert(ring_offset % 16 == 0, "unit-ring slots are read as 16-byte vectors");
   static_assert(out_offset % 1024 == 0 && kOutStageBytes % 1024 == 0, "swizzle atoms need 1 KB");
 };
 
@@ -279,6 +280,39 @@ struct Unit {
   int mb, nb, kb0, kb1;
 };
 
+// A unit as the producer publishes it in the ring (one 32-byte slot): its GEMM g and its
+// decoded tile and K range, so that no consumer repeats the decode (integer divisions and
+// indexed parameter loads, about 0.5 us between two epilogue tiles).  g < 0: the end of
+// the list.
+struct RingUnit {
+  int g;
+  Unit w;
+};
+
+__device__ __forceinline__ void ring_put(volatile int* slot, const RingUnit& r) {
+  asm volatile("st.volatile.shared.v4.u32 [%0], {%1, %2, %3, %4};" ::"r"(smem_u32(const_cast<int*>(slot))),
+               "r"(r.g), "r"(r.w.mb), "r"(r.w.nb), "r"(r.w.kb0)
+               : "memory");
+  slot[4] = r.w.kb1;
+}
+
+__device__ __forceinline__ void ring_put_cluster(uint32_t cluster_slot, const RingUnit& r) {
+  asm volatile("st.shared::cluster.v4.u32 [%0], {%1, %2, %3, %4};" ::"r"(cluster_slot), "r"(r.g),
+               "r"(r.w.mb), "r"(r.w.nb), "r"(r.w.kb0)
+               : "memory");
+  st_cluster_u32(cluster_slot + 16, static_cast<uint32_t>(r.w.kb1));
+}
+
+__device__ __forceinline__ RingUnit ring_get(const volatile int* slot) {
+  RingUnit r;
+  asm volatile("ld.volatile.shared.v4.u32 {%0, %1, %2, %3}, [%4];"
+               : "=r"(r.g), "=r"(r.w.mb), "=r"(r.w.nb), "=r"(r.w.kb0)
+               : "r"(smem_u32(const_cast<int*>(slot)))
+               : "memory");
+  r.w.kb1 = slot[4];
+  return r;
+}
+
 // Work unit u -> (tile, K split).  Tiles go in groups of kGroupM row tiles: inside a group
 // the row tile changes fastest, then the column tile.  The CTAs running at one time then
 // cover a compact block of the output, so the A rows of a group stay in L2 while every
@@ -338,7 +372,7 @@ __device__ __forceinline__ void leader_arrive(uint64_t* local_bar, uint32_t clus
 // units from the same ring as the other roles; a table is refilled once every epilogue
 // warp has released it (facfree).  Kept out of line: its registers stay its own.
 template <bool kPair>
-__device__ __noinline__ void factor_warp(const GemmBatch& bt, int units, uint64_t* ufull,
+__device__ __noinline__ void factor_warp(const GemmBatch& bt, uint64_t* ufull,
                                          uint64_t* uempty, uint32_t uempty_c,
                                          volatile int* unit_ring,
                                          uint64_t* facbar, uint64_t* facfree, float* fac_tab,
@@ -352,19 +386,17 @@ __device__ __noinline__ void factor_warp(const GemmBatch& bt, int units, uint64_
       ok = false;
       break;
     }
-    const int u = unit_ring[us];
+    const RingUnit r = ring_get(unit_ring + us * 8);
     __syncwarp();
     if (lane == 0) leader_arrive<kPair>(&uempty[us], uempty_c + us * 8);
     if (++us == kUnitRing) {
       us = 0;
       uph ^= 1u;
     }
-    if (u >= units) break;
-    int lu;
-    const int g = batch_member(bt, u, &lu);
-    const GemmParams& p = bt.p[g];
+    if (r.g < 0) break;
+    const GemmParams& p = bt.p[r.g];
     const float a_fac = epilogue_a_factor(p);
-    const int64_t n0 = static_cast<int64_t>(decode_unit<kPair>(p, lu).nb) * kBN;
+    const int64_t n0 = static_cast<int64_t>(r.w.nb) * kBN;
     float f[kBN / 32];
 #pragma unroll
     for (int j = 0; j < kBN / 32; ++j) {
@@ -560,18 +592,25 @@ __global__ void __launch_bounds__(kThreads, 1) shiftmm_kernel(const __grid_const
     int us = 0;
     uint32_t uph = 0;
     while (ok) {
-      int u;
+      int u = next;
+      RingUnit r;
       if (rank == 0) {
-        // publish the unit (or, past the end, the stop mark) to the roles of both CTAs
-        u = next;
+        // decode the unit and publish it (or, past the end, the stop mark) to the roles
+        // of both CTAs
+        r.g = -1;
+        if (u < units) {
+          int lu;
+          r.g = batch_member(bt, u, &lu);
+          r.w = decode_unit<kPair>(bt.p[r.g], lu);
+        }
         if (!ring_wait<kPair>(&uempty[us], uph ^ 1u, abort_flag)) {
           ok = false;
           break;
         }
-        unit_ring[us] = u;
+        ring_put(unit_ring + us * 8, r);
         mbar_arrive(&ufull[us]);
         if constexpr (kPair) {
-          st_cluster_u32(peer_ring_c + us * 4, static_cast<uint32_t>(u));
+          ring_put_cluster(peer_ring_c + us * 32, r);
           mbar_arrive_cluster(peer_ufull_c + us * 8);
         }
       } else {
@@ -579,14 +618,14 @@ __global__ void __launch_bounds__(kThreads, 1) shiftmm_kernel(const __grid_const
           ok = false;
           break;
         }
-        u = unit_ring[us];
+        r = ring_get(unit_ring + us * 8);
         mbar_arrive_cluster(uempty_c + us * 8);
       }
       if (++us == kUnitRing) {
         us = 0;
         uph ^= 1u;
       }
-      if (u >= units) break;
+      if (r.g < 0) break;
       // Within the last waves of units a pair takes its next unit only once its epilogues
       // have started this one, so that no pair holds several queued units while others
       // run dry.
@@ -599,9 +638,8 @@ __global__ void __launch_bounds__(kThreads, 1) shiftmm_kernel(const __grid_const
         else if (!lazy)
           next = npairs + atomicAdd(bt.sched, 1);
       }
-      int lu;
-      const int g = batch_member(bt, u, &lu);
-      const Unit w = decode_unit<kPair>(bt.p[g], lu);
+      const int g = r.g;
+      const Unit w = r.w;
       // rows past M (and columns past N) are read as zeros and never stored
       const int32_t ya = w.mb * L::tile_m + static_cast<int32_t>(rank) * kBM;
       const int32_t yb = w.nb * kBN + static_cast<int32_t>(rank) * L::b_rows;
@@ -665,18 +703,17 @@ __global__ void __launch_bounds__(kThreads, 1) shiftmm_kernel(const __grid_const
         ok = false;
         break;
       }
-      const int u = unit_ring[us];
+      const RingUnit r = ring_get(unit_ring + us * 8);
       mbar_arrive(&uempty[us]);
       if (++us == kUnitRing) {
         us = 0;
         uph ^= 1u;
       }
-      if (u >= units) break;
-      int lu;
-      const int g = batch_member(bt, u, &lu);
+      if (r.g < 0) break;
+      const int g = r.g;
       const int chunk_kb =
           bt.planned ? reinterpret_cast<volatile int*>(smem + L::chunk_offset)[g] : bt.p[g].chunk_kb;
-      const Unit w = decode_unit<kPair>(bt.p[g], lu);
+      const Unit w = r.w;
       for (int kc = w.kb0; kc < w.kb1 && ok; kc += chunk_kb) {
         const int kce = min(w.kb1, kc + chunk_kb);
         const uint32_t b = c & 1u, tph = (c >> 1) & 1u;
@@ -729,7 +766,7 @@ __global__ void __launch_bounds__(kThreads, 1) shiftmm_kernel(const __grid_const
       __syncwarp();
       if (lane == 0) mbar_arrive(chunkbar);
     }
-    factor_warp<kPair>(bt, units, ufull, uempty, uempty_c, unit_ring, facbar, facfree,
+    factor_warp<kPair>(bt, ufull, uempty, uempty_c, unit_ring, facbar, facfree,
                 reinterpret_cast<float*>(smem + L::fac_offset), abort_flag, peer_abort_c, lane);
   } else if (warp >= kEpiWarp0) {
     // --------------------------------------------------------------- epilogue
@@ -747,20 +784,19 @@ __global__ void __launch_bounds__(kThreads, 1) shiftmm_kernel(const __grid_const
         ok = false;
         break;
       }
-      const int u = unit_ring[us];
+      const RingUnit r = ring_get(unit_ring + us * 8);
       __syncwarp();
       if (lane == 0) leader_arrive<kPair>(&uempty[us], uempty_c + us * 8);
       if (++us == kUnitRing) {
         us = 0;
         uph ^= 1u;
       }
-      if (u >= units) break;
-      int lu;
-      const int g = batch_member(bt, u, &lu);
+      if (r.g < 0) break;
+      const int g = r.g;
       const GemmParams& p = bt.p[g];
       const CUtensorMap* tma_y = &bt.y[g];
       const CUtensorMap* tma_ws = &bt.ws[g];
-      const Unit w = decode_unit<kPair>(p, lu);
+      const Unit w = r.w;
       const int ckb =
           bt.planned ? reinterpret_cast<volatile int*>(smem + L::chunk_offset)[g] : p.chunk_kb;
       const int nch = (w.kb1 - w.kb0 + ckb - 1) / ckb;
