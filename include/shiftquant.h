@@ -233,6 +233,14 @@ size_t shiftquant_gemm_layer_workspace_bytes(int64_t M, int64_t K, int64_t N, in
 int shiftquant_gemm_layer_kernel_launches(int64_t M, int64_t K, int64_t N, int bits,
                                           int n_groups, size_t workspace_bytes, int gemm_mask);
 
+/* Tile mode of one shiftquant_gemm_layer call with this shape and gemm_mask on the current
+ * device: 1 when it runs on 2-CTA clusters with 256 x 256 tiles (cta_group::2 MMAs; chosen
+ * when the launch's units average at least 26 K blocks), 0 when each CTA runs 128 x 256
+ * tiles, -1 for invalid arguments, an empty launch, a shape beyond the exact range, or no
+ * device.  Results do not depend on the mode. */
+int shiftquant_gemm_layer_cta_pairs(int64_t M, int64_t K, int64_t N, int bits, int n_groups,
+                                    int gemm_mask);
+
 /* Weight-gradient GEMM for callers that cannot allocate device memory -- for instance a
  * plug-in running inside a host framework that owns every device allocation, or a
  * deployment whose device memory is fixed when the library is loaded.  The paper has no

@@ -1689,3 +1689,29 @@ extern "C" int shiftquant_gemm_layer_kernel_launches(int64_t M, int64_t K, int64
   for (int g = 0; g < n; ++g) launches += plans[g].splits > 1;
   return launches;
 }
+
+extern "C" int shiftquant_gemm_layer_cta_pairs(int64_t M, int64_t K, int64_t N, int bits,
+                                               int n_groups, int gemm_mask) {
+  if (!bits_ok(bits) || !groups_ok(n_groups) || M < 0 || K < 0 || N < 0 || gemm_mask < 0 ||
+      gemm_mask > 7)
+    return -1;
+  const int sms = device_sms(nullptr);
+  if (sms <= 0) return -1;
+  const int pairs = device_pairs(nullptr);
+  sq_layer_gemms a;
+  memset(&a, 0, sizeof(a));
+  a.M = M;
+  a.K = K;
+  a.N = N;
+  GemmJob jobs[3];
+  layer_jobs(&a, jobs, gemm_mask);
+  const GemmJob* lj[3];
+  int n = 0;
+  for (int i = 0; i < 3; ++i) {
+    if (jobs[i].M == 0 || jobs[i].N == 0 || jobs[i].K == 0) continue;
+    if (check_exact_range(jobs[i].which, jobs[i].K, bits, n_groups) != SQ_OK) return -1;
+    lj[n++] = &jobs[i];
+  }
+  if (n == 0) return -1;
+  return pair_mode(lj, n, bits, n_groups, sms, pairs) ? 1 : 0;
+}

@@ -35,7 +35,8 @@ EXPORTS = (
     "shiftquant_quantize", "shiftquant_gemm_fwd", "shiftquant_gemm_dgrad",
     "shiftquant_gemm_wgrad", "shiftquant_gemm_wgrad_static", "shiftquant_gemm_workspace_bytes",
     "shiftquant_gemm_layer", "shiftquant_gemm_layer_workspace_bytes",
-    "shiftquant_gemm_layer_kernel_launches", "shiftquant_status_string", "shiftquant_last_error",
+    "shiftquant_gemm_layer_kernel_launches", "shiftquant_gemm_layer_cta_pairs",
+    "shiftquant_status_string", "shiftquant_last_error",
 )
 
 _lib = None
@@ -112,6 +113,8 @@ def load(path: str | None = None) -> ctypes.CDLL:
     lib.shiftquant_gemm_layer_workspace_bytes.restype = sz
     lib.shiftquant_gemm_layer_kernel_launches.argtypes = [i64, i64, i64, i32, i32, sz, i32]
     lib.shiftquant_gemm_layer_kernel_launches.restype = i32
+    lib.shiftquant_gemm_layer_cta_pairs.argtypes = [i64, i64, i64, i32, i32, i32]
+    lib.shiftquant_gemm_layer_cta_pairs.restype = i32
     lib.shiftquant_gemm_workspace_bytes.argtypes = [i32, i64, i64, i64, i32, i32]
     lib.shiftquant_gemm_workspace_bytes.restype = sz
     lib.shiftquant_status_string.argtypes = [i32]
@@ -270,3 +273,9 @@ def shiftquant_gemm_layer_kernel_launches(M: int, K: int, N: int, bits: int, n_g
                                           workspace_bytes: int, gemm_mask: int = 0) -> int:
     return int(load().shiftquant_gemm_layer_kernel_launches(M, K, N, bits, n_groups,
                                                             workspace_bytes, gemm_mask))
+
+
+def shiftquant_gemm_layer_cta_pairs(M: int, K: int, N: int, bits: int, n_groups: int,
+                                    gemm_mask: int = 0) -> int:
+    """1: the layer launch runs on 2-CTA clusters (256 x 256 tiles); 0: single-CTA tiles."""
+    return int(load().shiftquant_gemm_layer_cta_pairs(M, K, N, bits, n_groups, gemm_mask))

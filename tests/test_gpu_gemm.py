@@ -67,6 +67,25 @@ def test_layer_chain_matches_oracle(M, K, Nn, bits):
     run_and_compare(*layer_inputs(rng, M, K, Nn), bits, 4)
 
 
+@pytest.mark.parametrize("M,K,Nn,bits", [(1900, 1800, 1700, 6), (3300, 3500, 3400, 4),
+                                         (2000, 1800, 1700, 8)])
+def test_pair_tiles_with_ragged_tails_match_oracle(M, K, Nn, bits):
+    # layer launches that run on CTA pairs (256 x 256 tiles): M = 1900 leaves the second CTA
+    # of the last pair entirely past M, and the column tails (1700, 1800, 3400, 3500) end
+    # inside one CTA's half of B; 8-bit adds multi-chunk K loops sized from the exponents
+    assert N.shiftquant_gemm_layer_cta_pairs(M, K, Nn, bits, 4) == 1
+    rng = np.random.default_rng(M + K + Nn + bits)
+    run_and_compare(*layer_inputs(rng, M, K, Nn), bits, 4, fused=True)
+
+
+def test_tile_mode_query():
+    # conv3x3's short K loops stay on single tiles; the large linear layer runs on pairs
+    assert N.shiftquant_gemm_layer_cta_pairs(12544, 2304, 256, 4, 4) == 0
+    assert N.shiftquant_gemm_layer_cta_pairs(16384, 4096, 11008, 6, 4) == 1
+    assert N.shiftquant_gemm_layer_cta_pairs(0, 0, 0, 6, 4) == -1
+    assert N.shiftquant_gemm_layer_cta_pairs(16, 16, 16, 9, 4) == -1
+
+
 @pytest.mark.parametrize("bits,G", [(6, 4), (8, 4), (8, 5), (4, 7), (5, 5), (3, 8)])
 def test_multi_chunk_inner_dims(bits, G):
     # K long enough that the exact-FP32 chunking splits the K loop several times
