@@ -566,10 +566,10 @@ __global__ void __launch_bounds__(kThreads, 1) shiftmm_kernel(const __grid_const
   const uint32_t rank = kPair ? cluster_ctarank() : 0u;
   const int pair = static_cast<int>(blockIdx.x) / kCg;   // the CTA group's index
   const int npairs = static_cast<int>(gridDim.x) / kCg;  // CTA groups in the launch
-  // the leader's unit-ring and TMEM release barriers and stage barriers; in a pair also
-  // the peer's ring and the other CTA's abort flag
+  // the leader's unit-ring release and stage barriers; in a pair also the peer's ring and
+  // the other CTA's abort flag (the epilogue forms its cluster addresses where it uses
+  // them, which keeps them out of its registers)
   const uint32_t uempty_c = mapa_shared(smem_u32(uempty), 0);
-  const uint32_t tempty_c = mapa_shared(smem_u32(tempty), 0);
   const uint32_t full_c = mapa_shared(smem_u32(full), 0);
   uint32_t peer_ring_c = 0, peer_ufull_c = 0, peer_abort_c = 0;
   if constexpr (kPair) {
@@ -786,7 +786,7 @@ __global__ void __launch_bounds__(kThreads, 1) shiftmm_kernel(const __grid_const
       }
       const RingUnit r = ring_get(unit_ring + us * 8);
       __syncwarp();
-      if (lane == 0) leader_arrive<kPair>(&uempty[us], uempty_c + us * 8);
+      if (lane == 0) leader_arrive<kPair>(&uempty[us], kPair ? mapa_shared(smem_u32(&uempty[us]), 0) : 0u);
       if (++us == kUnitRing) {
         us = 0;
         uph ^= 1u;
@@ -825,7 +825,7 @@ __global__ void __launch_bounds__(kThreads, 1) shiftmm_kernel(const __grid_const
           if (s == 3) {
             tc_fence_before();
             __syncwarp();
-            if (lane == 0) leader_arrive<kPair>(&tempty[b], tempty_c + b * 8);  // b may take the next tile
+            if (lane == 0) leader_arrive<kPair>(&tempty[b], kPair ? mapa_shared(smem_u32(&tempty[b]), 0) : 0u);  // b may take the next tile
           }
           const int64_t col0 = n0 + h * 128 + s * 32;
           if (row0 >= p.M || col0 >= p.N) continue;  // warp-uniform: nothing of this box exists
@@ -878,7 +878,7 @@ __global__ void __launch_bounds__(kThreads, 1) shiftmm_kernel(const __grid_const
           }
           tc_fence_before();
           __syncwarp();
-          if (lane == 0) leader_arrive<kPair>(&tempty[b], tempty_c + b * 8);  // b may take the next chunk
+          if (lane == 0) leader_arrive<kPair>(&tempty[b], kPair ? mapa_shared(smem_u32(&tempty[b]), 0) : 0u);  // b may take the next chunk
           ++c;
         }
         if (!ok) break;
@@ -904,7 +904,7 @@ __global__ void __launch_bounds__(kThreads, 1) shiftmm_kernel(const __grid_const
     if (!ok) {
       atomicOr(bt.status, kDevTimeout);
       *abort_flag = 1;
-      if constexpr (kPair) st_cluster_u32(peer_abort_c, 1);
+      if constexpr (kPair) st_cluster_u32(mapa_shared(smem_u32(const_cast<int*>(abort_flag)), rank ^ 1u), 1);
     }
     if (lane == 0) bulk_wait_read<0>();  // no store still reads shared memory at exit
   }
