@@ -91,6 +91,24 @@ sq_status shiftquant_calibrate(const float *x, int64_t rows, int64_t cols, int64
                                int gran, int n_groups, float *range_out, float *tau0_out,
                                uint8_t *exp_out, int32_t *dev_status, void *stream);
 
+/* Grouping alone (Eq. 3) from a given per-channel range vector:
+ *   range[channels] fp32 (device, non-negative: max |x| per channel), *tau0_out = its
+ *   maximum, exp_out[channels] = e_c exactly as shiftquant_calibrate with SQ_GRAN_SHIFT.
+ *   A NaN/Inf range sets SQ_DEV_NONFINITE (tau0 NaN or Inf, every e_c 0).  channels == 0
+ *   gives tau0 = 0.
+ * Use: a tensor split by rows (tokens) across devices quantizes bit for bit as the whole
+ *   would when every shard
+ *   1. takes its per-column ranges (shiftquant_calibrate, SQ_GRAN_PER_COL),
+ *   2. replaces them by their element-wise maximum over the shards (an all-reduce(max):
+ *      exact, as a maximum of floats is),
+ *   3. calls shiftquant_group on the result, and
+ *   4. quantizes with SQ_GRAN_SHIFT; stochastic rounding draws the whole tensor's numbers
+ *      when a shard starting at row r0 passes seed + r0 * cols * 0x9E3779B97F4A7C15
+ *      (mod 2^64) as its seed, since the generator's state is linear in the index. */
+sq_status shiftquant_group(const float *range, int64_t channels, int n_groups,
+                           float *tau0_out, uint8_t *exp_out, int32_t *dev_status,
+                           void *stream);
+
 /* Quantization (App. D; stochastic rounding of App. B).
  *   x [rows, ld] fp32, bits in [2, 8], Q = 2^(bits-1) - 1.
  *   gran == SQ_GRAN_SHIFT: range_or_tau0 -> the device scalar tau_0 and exp[cols] from

@@ -69,6 +69,46 @@ __global__ void __launch_bounds__(256)
   if (counter != nullptr && blockIdx.x == 0 && threadIdx.x == 0) *counter = 0u;
 }
 
+// Grouping (Eq. 3) by one block of kGroupThreads threads from the per-channel range bits:
+// tau_0 = the largest range, then every channel's exponent; tau0_out receives tau_0 and the
+// status word the non-finite flag.  scratch: 33 words of shared memory.
+constexpr int kGroupThreads = 256;
+static_assert(kColTx * kColTy == kGroupThreads, "the range pass's last block does the grouping");
+
+__device__ void grouping_block(const unsigned* range_bits, int64_t C, int G, float* tau0_out,
+                               uint8_t* exp_out, int* status, unsigned* scratch, int tid) {
+  unsigned m = 0;
+  for (int64_t c = tid; c < C; c += kGroupThreads) m = max(m, __ldcg(range_bits + c));
+  m = __reduce_max_sync(0xFFFFFFFFu, m);
+  if ((tid & 31) == 0) scratch[tid >> 5] = m;
+  __syncthreads();
+  if (tid < 32) {
+    unsigned v = tid < kGroupThreads / 32 ? scratch[tid] : 0u;
+    v = __reduce_max_sync(0xFFFFFFFFu, v);
+    if (tid == 0) scratch[32] = v;
+  }
+  __syncthreads();
+  const unsigned tb = scratch[32];
+  const float tau = __uint_as_float(tb);
+  const bool nonfinite = tb >= 0x7F800000u;
+  for (int64_t c = tid; c < C; c += kGroupThreads)
+    exp_out[c] = static_cast<uint8_t>(nonfinite ? 0 : group_exponent(__uint_as_float(__ldcg(range_bits + c)), tau, G));
+  __syncthreads();
+  if (tid == 0) {
+    *tau0_out = tau;
+    if (nonfinite) atomicOr(status, kDevNonFinite);
+  }
+}
+
+// Grouping alone, from a given range vector (a sharded tensor's all-reduced ranges)
+__global__ void __launch_bounds__(kGroupThreads)
+    group_kernel(const unsigned* __restrict__ range_bits, int64_t C, int G,
+                 float* __restrict__ tau0_out, uint8_t* __restrict__ exp_out,
+                 int* __restrict__ status) {
+  __shared__ unsigned scratch[33];
+  grouping_block(range_bits, C, G, tau0_out, exp_out, status, scratch, threadIdx.x);
+}
+
 // Range pass: one wave of blocks, block (x, y) owning 128 columns and the 64-row tiles
 // y, y + gridDim.y, ... (so the blocks resident at one time read a contiguous band of whole
 // rows: long DRAM bursts).  Warp w reads rows 8w .. 8w+7 of a tile with all eight 16-byte
@@ -173,28 +213,7 @@ __global__ void __launch_bounds__(kColTx* kColTy)
   __syncthreads();
   if (!last_block) return;
   __threadfence();
-  unsigned m = 0;
-  for (int64_t c = tid; c < C; c += kColTx * kColTy) m = max(m, __ldcg(range_bits + c));
-  m = __reduce_max_sync(0xFFFFFFFFu, m);
-  unsigned* wmax = &red[0][0];
-  if ((tid & 31) == 0) wmax[tid >> 5] = m;
-  __syncthreads();
-  if (tid < 32) {
-    unsigned v = tid < (kColTx * kColTy) / 32 ? wmax[tid] : 0u;
-    v = __reduce_max_sync(0xFFFFFFFFu, v);
-    if (tid == 0) wmax[32] = v;
-  }
-  __syncthreads();
-  const unsigned tb = wmax[32];
-  const float tau = __uint_as_float(tb);
-  const bool nonfinite = tb >= 0x7F800000u;
-  for (int64_t c = tid; c < C; c += kColTx * kColTy)
-    exp_out[c] = static_cast<uint8_t>(nonfinite ? 0 : group_exponent(__uint_as_float(__ldcg(range_bits + c)), tau, G));
-  __syncthreads();
-  if (tid == 0) {
-    *tau0_out = tau;  // replaces the block counter
-    if (nonfinite) atomicOr(status, kDevNonFinite);
-  }
+  grouping_block(range_bits, C, G, tau0_out, exp_out, status, &red[0][0], tid);
 }
 
 // one warp per row: range[r] = max_c |x[r, c]|
@@ -670,6 +689,25 @@ extern "C" sq_status shiftquant_calibrate(const float* x, int64_t rows, int64_t 
                    tau0_out, exp_out);
   if (err == cudaSuccess) err = cudaGetLastError();
   return err == cudaSuccess ? SQ_OK : cuda_fail(err, "colmax_kernel launch");
+}
+
+extern "C" sq_status shiftquant_group(const float* range, int64_t channels, int n_groups,
+                                      float* tau0_out, uint8_t* exp_out, int32_t* dev_status,
+                                      void* stream) {
+  clear_error();
+  if (!groups_ok(n_groups)) return fail(SQ_EINVAL, "group: n_groups must be in [1, 8]");
+  if (channels < 0) return fail(SQ_EINVAL, "group: negative size");
+  if (tau0_out == nullptr || dev_status == nullptr || (channels > 0 && (range == nullptr || exp_out == nullptr)))
+    return fail(SQ_EINVAL, "group: range, tau0_out, exp_out and dev_status are required");
+  cudaStream_t s = as_stream(stream);
+  if (channels == 0) {
+    const cudaError_t err = cudaMemsetAsync(tau0_out, 0, sizeof(float), s);
+    return err == cudaSuccess ? SQ_OK : cuda_fail(err, "cudaMemsetAsync");
+  }
+  group_kernel<<<1, kGroupThreads, 0, s>>>(reinterpret_cast<const unsigned*>(range), channels,
+                                           n_groups, tau0_out, exp_out, dev_status);
+  const cudaError_t err = cudaGetLastError();
+  return err == cudaSuccess ? SQ_OK : cuda_fail(err, "group_kernel launch");
 }
 
 extern "C" sq_status shiftquant_quantize(const float* x, int64_t rows, int64_t cols, int64_t ld,

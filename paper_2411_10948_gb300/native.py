@@ -32,7 +32,7 @@ SQ_CODE_BF16 = 1
 # every symbol declared in include/shiftquant.h
 EXPORTS = (
     "shiftquant_code_type", "shiftquant_code_bytes", "shiftquant_calibrate",
-    "shiftquant_quantize", "shiftquant_gemm_fwd", "shiftquant_gemm_dgrad",
+    "shiftquant_group", "shiftquant_quantize", "shiftquant_gemm_fwd", "shiftquant_gemm_dgrad",
     "shiftquant_gemm_wgrad", "shiftquant_gemm_wgrad_static", "shiftquant_gemm_workspace_bytes",
     "shiftquant_gemm_layer", "shiftquant_gemm_layer_workspace_bytes",
     "shiftquant_gemm_layer_kernel_launches", "shiftquant_gemm_layer_cta_pairs",
@@ -93,6 +93,8 @@ def load(path: str | None = None) -> ctypes.CDLL:
     lib.shiftquant_code_bytes.restype = i32
     lib.shiftquant_calibrate.argtypes = [vp, i64, i64, i64, i32, i32, vp, vp, vp, vp, vp]
     lib.shiftquant_calibrate.restype = i32
+    lib.shiftquant_group.argtypes = [vp, i64, i32, vp, vp, vp, vp]
+    lib.shiftquant_group.restype = i32
     lib.shiftquant_quantize.argtypes = [vp, i64, i64, i64, i32, i32, i32, vp, vp, vp, i32, u64,
                                         vp, i64, vp, i64, vp, vp]
     lib.shiftquant_quantize.restype = i32
@@ -174,6 +176,12 @@ def shiftquant_calibrate(x, gran, n_groups, range_out, tau0_out, exp_out, dev_st
     _check(load().shiftquant_calibrate(_ptr(x), x.shape[0], x.shape[1], _ld(x), gran, n_groups,
                                        _ptr(range_out), _ptr(tau0_out), _ptr(exp_out),
                                        _ptr(dev_status), _stream(stream)))
+
+
+def shiftquant_group(range_, n_groups, tau0_out, exp_out, dev_status, stream=None) -> None:
+    """tau_0 and the group exponents from a given range vector (see the header)."""
+    _check(load().shiftquant_group(_ptr(range_), range_.numel(), n_groups, _ptr(tau0_out),
+                                   _ptr(exp_out), _ptr(dev_status), _stream(stream)))
 
 
 def shiftquant_quantize(x, gran, bits, n_groups, range_or_tau0, exp, fold_exp, mode, seed,

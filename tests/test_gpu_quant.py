@@ -153,3 +153,62 @@ def test_weight_quantization_with_fold(shape, bits, G):
     np.testing.assert_array_equal(f32_bits(d.range.cpu().numpy()), f32_bits(od["range"]))
     np.testing.assert_array_equal(f32_bits(d.scale.cpu().numpy()), f32_bits(od["scale"]))
     np.testing.assert_array_equal(decode(d.codes), folded(od["codes"], eg, G, axis=1))
+
+
+@pytest.mark.parametrize("mode", [N.SQ_ROUND_NEAREST_EVEN, N.SQ_ROUND_STOCHASTIC])
+@pytest.mark.parametrize("bits", [4, 6])
+def test_row_shards_quantize_as_the_whole_tensor(mode, bits):
+    # a tensor split by rows over two "ranks" (here two shards on one GPU, the all-reduce
+    # of their ranges an element-wise maximum): shard ranges, the exchange, the grouping
+    # alone (shiftquant_group) and the quantizer with the shifted generator give exactly the
+    # whole tensor's ranges, tau_0, exponents, scale, codes and transposed codes
+    rng = np.random.default_rng(bits * 10 + mode)
+    R, C, G, seed = 3000, 700, 4, 0x1234ABCD
+    x = to_gpu(gradient_like(rng, R, C))
+    st = torch.zeros(1, dtype=torch.int32, device="cuda")
+    whole = L.ShiftTensor.alloc(R, C, bits, G, "cuda")
+    L.shift_quantize(x, whole, bits, G, mode, seed, st)
+    bounds = [(0, 1201), (1201, R)]
+    shards = [L.ShiftTensor.alloc(r1 - r0, C, bits, G, "cuda") for r0, r1 in bounds]
+    parts = []
+    for (r0, r1), q in zip(bounds, shards):
+        N.shiftquant_calibrate(x[r0:r1], N.SQ_GRAN_PER_COL, G, q.range, None, None, st)
+        parts.append(q.range.clone())
+    both = torch.maximum(parts[0], parts[1])
+    for (r0, r1), q in zip(bounds, shards):
+        L.shard_shift_quantize(x[r0:r1], q, bits, G, mode, seed, r0, st, lambda t: t.copy_(both))
+    torch.cuda.synchronize()
+    assert st.item() == 0
+    want_codes, want_t = decode(whole.codes), decode(whole.codes_t)
+    for (r0, r1), q in zip(bounds, shards):
+        np.testing.assert_array_equal(f32_bits(q.range.cpu().numpy()), f32_bits(whole.range.cpu().numpy()))
+        assert f32_bits([q.tau0.item()])[0] == f32_bits([whole.tau0.item()])[0]
+        np.testing.assert_array_equal(q.exp.cpu().numpy(), whole.exp.cpu().numpy())
+        assert f32_bits([q.scale.item()])[0] == f32_bits([whole.scale.item()])[0]
+        np.testing.assert_array_equal(decode(q.codes), want_codes[r0:r1])
+        np.testing.assert_array_equal(decode(q.codes_t), want_t[:, r0:r1])
+
+
+def test_group_entry_matches_the_range_pass_grouping():
+    # shiftquant_group on the range pass's own output reproduces its tau_0 and exponents,
+    # including all-zero and outlier channels; zero channels alone give tau_0 = 0
+    rng = np.random.default_rng(5)
+    x = gradient_like(rng, 500, 333)
+    x[:, 7] = 0.0
+    xg = to_gpu(x)
+    st = torch.zeros(1, dtype=torch.int32, device="cuda")
+    for G in (1, 3, 4, 8):
+        q = L.ShiftTensor.alloc(500, 333, 4, G, "cuda")
+        N.shiftquant_calibrate(xg, N.SQ_GRAN_SHIFT, G, q.range, q.tau0, q.exp, st)
+        tau = torch.zeros(1, device="cuda")
+        e = torch.empty(333, dtype=torch.uint8, device="cuda")
+        N.shiftquant_group(q.range, G, tau, e, st)
+        torch.cuda.synchronize()
+        assert tau.item() == q.tau0.item()
+        np.testing.assert_array_equal(e.cpu().numpy(), q.exp.cpu().numpy())
+        t_o, e_o, _ = O.group(q.range.cpu().numpy(), G)
+        np.testing.assert_array_equal(e.cpu().numpy(), e_o)
+    z = torch.zeros(16, device="cuda")
+    N.shiftquant_group(z, 4, tau, e[:16], st)
+    torch.cuda.synchronize()
+    assert tau.item() == 0.0 and (e[:16].cpu().numpy() == 3).all() and st.item() == 0

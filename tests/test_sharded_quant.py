@@ -1,0 +1,91 @@
+"""The one exchange step of a tensor split by rows (tokens) across ranks, on CPU: two
+`gloo` ranks each hold a row shard, take its per-column ranges, all-reduce them with MAX,
+group, and quantize with the generator moved to the shard's first row
+(`layer.shard_seed`).  Every rank's ranges, tau_0, exponents, codes and scale must equal
+the whole tensor's, computed by the oracle (the CUDA path is exercised the same way by
+tests/test_gpu_quant.py on one GPU)."""
+import multiprocessing as mp
+import os
+import socket
+import sys
+
+import numpy as np
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def _free_port() -> int:
+    with socket.socket(socket.AF_INET, socket.SOCK_STREAM) as s:
+        s.bind(("127.0.0.1", 0))
+        return s.getsockname()[1]
+
+
+def _tensor():
+    rng = np.random.default_rng(7)
+    R, C = 300, 96
+    x = (rng.standard_normal((R, C)) * np.exp(rng.normal(0.0, 1.5, C))).astype(np.float32)
+    x[:, 5] *= 100.0
+    x[:, 9] = 0.0
+    return x
+
+
+def _shard_main(rank, world, port, bits, G, mode, seed, bounds, out):
+    sys.path.insert(0, ROOT)
+    os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port), RANK=str(rank),
+                      WORLD_SIZE=str(world))
+    import torch
+    import torch.distributed as dist
+    import oracle as O
+    from paper_2411_10948_gb300.layer import shard_seed
+    dist.init_process_group("gloo", rank=rank, world_size=world)
+    try:
+        x = _tensor()
+        r0, r1 = bounds[rank], bounds[rank + 1]
+        shard = x[r0:r1]
+        local, _ = O.range_cols(shard)
+        t = torch.from_numpy(local.copy())
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)   # the exchange
+        rng = t.numpy()
+        tau0, e, _ = O.group(rng, G)
+        q, s = O.quantize_shift(shard, bits, G, tau0, e, mode, shard_seed(seed, r0, x.shape[1]))
+        whole = O.shiftquant_tensor(x, bits, G, mode, seed)
+        ok = (np.array_equal(rng.view(np.uint32), whole["range"].view(np.uint32))
+              and np.float32(tau0).view(np.uint32) == np.float32(whole["tau0"]).view(np.uint32)
+              and np.array_equal(e, whole["exp"])
+              and np.array_equal(q, whole["codes"][r0:r1])
+              and np.float32(s).view(np.uint32) == np.float32(whole["scale"]).view(np.uint32))
+        out.put((rank, bool(ok)))
+        dist.barrier()
+    finally:
+        dist.destroy_process_group()
+
+
+@pytest.mark.parametrize("bits,mode", [(4, 0), (4, 1), (8, 1)])
+def test_two_gloo_ranks_quantize_their_shards_as_the_whole_tensor(bits, mode):
+    world, G, seed, bounds = 2, 4, 0xC0FFEE, [0, 131, 300]
+    ctx = mp.get_context("spawn")
+    out = ctx.Queue()
+    port = _free_port()
+    procs = [ctx.Process(target=_shard_main, args=(r, world, port, bits, G, mode, seed, bounds, out))
+             for r in range(world)]
+    for p in procs:
+        p.start()
+    got = sorted(out.get(timeout=180) for _ in range(world))
+    for p in procs:
+        p.join(timeout=60)
+        assert p.exitcode == 0
+    assert got == [(0, True), (1, True)]
+
+
+def test_shard_seed_moves_the_generator_exactly():
+    # the element (r, c) of a shard starting at row r0 draws what element (r0 + r, c) of the
+    # whole tensor draws
+    sys.path.insert(0, ROOT)
+    import oracle as O
+    from paper_2411_10948_gb300.layer import shard_seed
+    seed, C = 0xDEADBEEF12345678, 700
+    for r0 in (0, 1, 1201, 10**6):
+        s = shard_seed(seed, r0, C)
+        for r, c in ((0, 0), (3, 699), (17, 5)):
+            assert O.hash64(s, r * C + c) == O.hash64(seed, (r0 + r) * C + c)
