@@ -186,6 +186,30 @@ sq_status shiftquant_gemm_wgrad(const void *xt_codes, int64_t ldx, const float *
                                 void *workspace, size_t workspace_bytes,
                                 int32_t *dev_status, void *stream);
 
+/* The weight gradient over tokens split across ranks, exact: each rank sums its own tokens
+ * and the ranks add the integer sums before the one dequantizing multiply, so the result
+ * is bit for bit shiftquant_gemm_wgrad's over all tokens.
+ * shiftquant_gemm_wgrad_partial: the shard's raw sums
+ *   t_out[i, j] = sum over the shard's T tokens of q_X[t, i] q_dY[t, j]
+ *   (int32, dense [Ci, Co], 16-byte aligned, Co a multiple of 4), with the operands of
+ *   shiftquant_gemm_wgrad (xt_codes [Ci, ldx], gt_codes [Co, ldg], unshifted codes; the
+ *   scales and exponents are required as there, although the sums do not use them).  The
+ *   exact range is checked for total_tokens, the tokens of all shards together, so that
+ *   the all-reduce(sum) of the shards' t_out (int32) stays exact.
+ * shiftquant_gemm_wgrad_finish: dw[i, j] = float(T[i, j]) 2^-(eX_i + eY_j) (s_X s_dY) from
+ *   the summed T, and acc_out (may be NULL) = T << (2(G-1) - eX_i - eY_j) as int64. */
+sq_status shiftquant_gemm_wgrad_partial(const void *xt_codes, int64_t ldx, const float *x_scale,
+                                        const uint8_t *x_exp, const void *gt_codes, int64_t ldg,
+                                        const float *g_scale, const uint8_t *g_exp, int64_t Ci,
+                                        int64_t Co, int64_t T, int64_t total_tokens, int bits,
+                                        int n_groups, int32_t *t_out, int32_t *dev_status,
+                                        void *stream);
+sq_status shiftquant_gemm_wgrad_finish(const int32_t *t, int64_t Ci, int64_t Co, int bits,
+                                       int n_groups, const float *x_scale, const uint8_t *x_exp,
+                                       const float *g_scale, const uint8_t *g_exp, float *dw,
+                                       int64_t ld_dw, int64_t *acc_out, int64_t ld_acc,
+                                       int32_t *dev_status, void *stream);
+
 /* The three GEMMs of one quantized linear layer in ONE persistent launch.  They are
  * independent (each reads only codes produced before the call), so their output tiles share
  * the SMs: the work units of all three form one list, the GEMM with the longest K loop per

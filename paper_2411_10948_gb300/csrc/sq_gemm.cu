@@ -1142,6 +1142,7 @@ struct GemmJob {
   void* ws;
   size_t ws_bytes;
   const uint8_t* k_exp;  // exponents of the inner channels (forward, loss propagation), or null
+  int partial;  // weight gradient: int32 sums into ws (the caller's), no dequantizing pass
 };
 
 static const char* job_name(int which) {
@@ -1162,12 +1163,19 @@ static int check_job(const GemmJob& j, int bits, int G, int32_t* dev_status, cud
     return fail(SQ_EUNSUPPORTED, "%s: dimensions beyond 2^31", nm);
   if (dev_status == nullptr) return fail(SQ_EINVAL, "%s: dev_status is required", nm);
   if (j.M == 0 || j.N == 0) return SQ_OK;
-  if (j.y == nullptr || j.ldy < j.N) return fail(SQ_EINVAL, "%s: output is NULL or its ld < N", nm);
-  if (j.acc != nullptr && j.ld_acc < j.N) return fail(SQ_EINVAL, "%s: ld_acc < N", nm);
+  if (!j.partial) {  // a partial call writes int32 sums only, no fp32 output
+    if (j.y == nullptr || j.ldy < j.N) return fail(SQ_EINVAL, "%s: output is NULL or its ld < N", nm);
+    if (j.acc != nullptr && j.ld_acc < j.N) return fail(SQ_EINVAL, "%s: ld_acc < N", nm);
+  }
+  // the kernel reads the scales and exponents of every tile (a partial call too)
   if (j.a_scale == nullptr || j.b_scale == nullptr)
     return fail(SQ_EINVAL, "%s: scales are required", nm);
   if (j.which == 2 && (j.row_exp == nullptr || j.col_exp == nullptr))
     return fail(SQ_EINVAL, "%s: exponents are required", nm);
+  if (j.K == 0 && j.partial) {
+    const cudaError_t err = cudaMemsetAsync(j.ws, 0, static_cast<size_t>(j.M) * j.N * sizeof(int), s);
+    return err == cudaSuccess ? SQ_OK : cuda_fail(err, "cudaMemsetAsync");
+  }
   if (j.K == 0) {
     // an empty inner sum: T = 0 everywhere
     cudaError_t err = cudaMemset2DAsync(j.y, j.ldy * sizeof(float), 0, j.N * sizeof(float), j.M, s);
@@ -1193,7 +1201,7 @@ static int check_job(const GemmJob& j, int bits, int G, int32_t* dev_status, cud
 static int plan_job(const GemmJob& j, int bits, int G, int workers, int max_splits, bool pair,
                     Plan* pl) {
   const int st = make_plan(j.which, j.M, j.N, j.K, bits, G, workers, max_splits, pair, pl);
-  if (st != SQ_OK || pl->splits <= 1) return st;
+  if (st != SQ_OK || pl->splits <= 1 || j.partial) return st;  // partial: ws is the output
   if (j.ws == nullptr || j.ws_bytes < split_ws_bytes(j.M, j.N) || !aligned16(j.ws) || j.N % 4 != 0)
     return make_plan(j.which, j.M, j.N, j.K, bits, G, workers, 1, pair, pl);
   return SQ_OK;
@@ -1283,7 +1291,7 @@ static int prepare_job(const GemmJob& j, const Plan* pl, int bits, int G, int32_
   p.ldy = j.ldy;
   p.acc = reinterpret_cast<long long*>(j.acc);
   p.ld_acc = j.ld_acc;
-  p.ws = pl->splits > 1 ? static_cast<int*>(j.ws) : nullptr;
+  p.ws = (pl->splits > 1 || j.partial) ? static_cast<int*>(j.ws) : nullptr;
   p.status = dev_status;
   memset(&bt->y[g], 0, sizeof(CUtensorMap));
   memset(&bt->ws[g], 0, sizeof(CUtensorMap));
@@ -1356,6 +1364,7 @@ static int run_jobs(GemmJob* jobs, int njobs, int bits, int G, int32_t* dev_stat
   Plan plans[kMaxBatch];
   GemmJob* lj[kMaxBatch];
   for (int g = 0; g < nlive; ++g) lj[g] = &jobs[live[g]];
+  const bool partial = nlive == 1 && lj[0]->partial;  // only single-GEMM calls are partial
   const int pairs = device_pairs(nullptr);
   const bool pair = pair_mode(lj, nlive, bits, G, sms, pairs);
   const int workers = pair ? pairs : sms;  // CTA groups resident at once
@@ -1402,7 +1411,9 @@ static int run_jobs(GemmJob* jobs, int njobs, int bits, int G, int32_t* dev_stat
   for (int g = 0; g < nlive; ++g) {
     if (!bt.p[g].ws) continue;
     char* w = reinterpret_cast<char*>(bt.p[g].ws);
-    const size_t b = split_ws_bytes(bt.p[g].M, bt.p[g].N);
+    // a partial call's sums go to the caller's buffer of exactly M N words
+    const size_t b = partial ? static_cast<size_t>(bt.p[g].M) * bt.p[g].N * sizeof(int)
+                             : split_ws_bytes(bt.p[g].M, bt.p[g].N);
     if (zero_end != nullptr && w == zero_end) {
       zero_end = w + b;
       continue;
@@ -1433,7 +1444,7 @@ static int run_jobs(GemmJob* jobs, int njobs, int bits, int G, int32_t* dev_stat
                                 : launch_variant<0>(bt, grid, dev, s, multi, pair);
   if (st != SQ_OK) return st;
   for (int g = 0; g < nlive; ++g) {
-    if (!bt.p[g].ws) continue;
+    if (!bt.p[g].ws || partial) continue;
     const int64_t quads = static_cast<int64_t>(bt.p[g].M) * (bt.p[g].N / 4);
     int64_t blocks = (quads + 255) / 256;
     if (blocks > static_cast<int64_t>(sms) * 16) blocks = static_cast<int64_t>(sms) * 16;
@@ -1595,6 +1606,75 @@ extern "C" size_t shiftquant_gemm_workspace_bytes(int which, int64_t M, int64_t 
   Plan pl;
   if (make_plan(which, M, N, K, bits, n_groups, pair ? pairs : sms, 0, pair, &pl) != SQ_OK) return 0;
   return pl.splits > 1 ? split_ws_bytes(M, N) : 0;
+}
+
+extern "C" sq_status shiftquant_gemm_wgrad_partial(
+    const void* xt_codes, int64_t ldx, const float* x_scale, const uint8_t* x_exp,
+    const void* gt_codes, int64_t ldg, const float* g_scale, const uint8_t* g_exp, int64_t Ci,
+    int64_t Co, int64_t T, int64_t total_tokens, int bits, int n_groups, int32_t* t_out,
+    int32_t* dev_status, void* stream) {
+  fail(SQ_OK, "");
+  if (!bits_ok(bits) || !groups_ok(n_groups))
+    return fail(SQ_EINVAL, "gemm_wgrad_partial: bits must be in [2, 8] and n_groups in [1, 8]");
+  if (Ci < 0 || Co < 0 || T < 0 || total_tokens < T)
+    return fail(SQ_EINVAL, "gemm_wgrad_partial: negative size or total_tokens < T");
+  if (Ci == 0 || Co == 0) return SQ_OK;
+  if (t_out == nullptr || !aligned16(t_out) || Co % 4 != 0)
+    return fail(SQ_EALIGN, "gemm_wgrad_partial: t_out must be 16-byte aligned and Co a multiple of 4");
+  // the summed partials must stay in the exact int32 range for the whole token count
+  int st = check_exact_range(2, total_tokens, bits, n_groups);
+  if (st != SQ_OK) return st;
+  GemmJob j{2, xt_codes, ldx, gt_codes, ldg, Ci, Co, T, x_scale, g_scale, x_exp, g_exp,
+            nullptr, 0, nullptr, 0, t_out, static_cast<size_t>(Ci) * Co * sizeof(int32_t)};
+  j.partial = 1;
+  return run_jobs(&j, 1, bits, n_groups, dev_status, stream, nullptr);
+}
+
+extern "C" sq_status shiftquant_gemm_wgrad_finish(const int32_t* t, int64_t Ci, int64_t Co,
+                                                  int bits, int n_groups, const float* x_scale,
+                                                  const uint8_t* x_exp, const float* g_scale,
+                                                  const uint8_t* g_exp, float* dw, int64_t ld_dw,
+                                                  int64_t* acc_out, int64_t ld_acc,
+                                                  int32_t* dev_status, void* stream) {
+  fail(SQ_OK, "");
+  if (!bits_ok(bits) || !groups_ok(n_groups))
+    return fail(SQ_EINVAL, "gemm_wgrad_finish: bits must be in [2, 8] and n_groups in [1, 8]");
+  if (Ci < 0 || Co < 0) return fail(SQ_EINVAL, "gemm_wgrad_finish: negative size");
+  if (Ci == 0 || Co == 0) return SQ_OK;
+  if (t == nullptr || !aligned16(t) || Co % 4 != 0)
+    return fail(SQ_EALIGN, "gemm_wgrad_finish: t must be 16-byte aligned and Co a multiple of 4");
+  if (dw == nullptr || ld_dw < Co || x_scale == nullptr || g_scale == nullptr ||
+      x_exp == nullptr || g_exp == nullptr || dev_status == nullptr ||
+      (acc_out != nullptr && ld_acc < Co))
+    return fail(SQ_EINVAL, "gemm_wgrad_finish: NULL argument or ld < Co");
+  int dev = 0;
+  const int sms = device_sms(&dev);
+  if (sms <= 0) return fail(SQ_ECUDA, "gemm_wgrad_finish: no current CUDA device");
+  GemmParams p;
+  memset(&p, 0, sizeof(p));
+  p.M = static_cast<int>(Ci);
+  p.N = static_cast<int>(Co);
+  p.mode = 1;
+  p.G = n_groups;
+  p.vec_y = (ld_dw % 4 == 0) && aligned16(dw);
+  p.a_scale = x_scale;
+  p.b_scale = g_scale;
+  p.row_exp = x_exp;
+  p.col_exp = g_exp;
+  p.y = dw;
+  p.ldy = ld_dw;
+  p.acc = reinterpret_cast<long long*>(acc_out);
+  p.ld_acc = ld_acc;
+  p.ws = const_cast<int*>(t);
+  p.status = dev_status;
+  if (Ci > INT32_MAX || Co > INT32_MAX)
+    return fail(SQ_EUNSUPPORTED, "gemm_wgrad_finish: dimensions beyond 2^31");
+  const int64_t quads = Ci * (Co / 4);
+  int64_t blocks = (quads + 255) / 256;
+  if (blocks > static_cast<int64_t>(sms) * 16) blocks = static_cast<int64_t>(sms) * 16;
+  splitk_finalize_kernel<<<static_cast<unsigned>(blocks), 256, 0, as_stream(stream)>>>(p);
+  const cudaError_t err = cudaGetLastError();
+  return err == cudaSuccess ? SQ_OK : cuda_fail(err, "splitk_finalize_kernel launch");
 }
 
 extern "C" sq_status shiftquant_gemm_wgrad_static(

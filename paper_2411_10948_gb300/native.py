@@ -33,7 +33,8 @@ SQ_CODE_BF16 = 1
 EXPORTS = (
     "shiftquant_code_type", "shiftquant_code_bytes", "shiftquant_calibrate",
     "shiftquant_group", "shiftquant_quantize", "shiftquant_gemm_fwd", "shiftquant_gemm_dgrad",
-    "shiftquant_gemm_wgrad", "shiftquant_gemm_wgrad_static", "shiftquant_gemm_workspace_bytes",
+    "shiftquant_gemm_wgrad", "shiftquant_gemm_wgrad_partial", "shiftquant_gemm_wgrad_finish",
+    "shiftquant_gemm_wgrad_static", "shiftquant_gemm_workspace_bytes",
     "shiftquant_gemm_layer", "shiftquant_gemm_layer_workspace_bytes",
     "shiftquant_gemm_layer_kernel_launches", "shiftquant_gemm_layer_cta_pairs",
     "shiftquant_status_string", "shiftquant_last_error",
@@ -95,6 +96,12 @@ def load(path: str | None = None) -> ctypes.CDLL:
     lib.shiftquant_calibrate.restype = i32
     lib.shiftquant_group.argtypes = [vp, i64, i32, vp, vp, vp, vp]
     lib.shiftquant_group.restype = i32
+    lib.shiftquant_gemm_wgrad_partial.argtypes = [vp, i64, vp, vp, vp, i64, vp, vp, i64, i64, i64,
+                                                  i64, i32, i32, vp, vp, vp]
+    lib.shiftquant_gemm_wgrad_partial.restype = i32
+    lib.shiftquant_gemm_wgrad_finish.argtypes = [vp, i64, i64, i32, i32, vp, vp, vp, vp, vp, i64,
+                                                 vp, i64, vp, vp]
+    lib.shiftquant_gemm_wgrad_finish.restype = i32
     lib.shiftquant_quantize.argtypes = [vp, i64, i64, i64, i32, i32, i32, vp, vp, vp, i32, u64,
                                         vp, i64, vp, i64, vp, vp]
     lib.shiftquant_quantize.restype = i32
@@ -270,6 +277,25 @@ def shiftquant_gemm_layer(x_codes, xt_codes, x_scale, x_exp, g_codes, gt_codes, 
     _check(load().shiftquant_gemm_layer(
         ctypes.byref(a), _ptr(workspace),
         workspace.numel() * workspace.element_size() if workspace is not None else 0,
+        _ptr(dev_status), _stream(stream)))
+
+
+def shiftquant_gemm_wgrad_partial(xt_codes, x_scale, x_exp, gt_codes, g_scale, g_exp, Ci, Co, T,
+                                  total_tokens, bits, n_groups, t_out, dev_status,
+                                  stream=None) -> None:
+    """One token shard's int32 weight-gradient sums (see the header)."""
+    _check(load().shiftquant_gemm_wgrad_partial(
+        _ptr(xt_codes), _ld(xt_codes), _ptr(x_scale), _ptr(x_exp), _ptr(gt_codes),
+        _ld(gt_codes), _ptr(g_scale), _ptr(g_exp), Ci, Co, T, total_tokens, bits, n_groups,
+        _ptr(t_out), _ptr(dev_status), _stream(stream)))
+
+
+def shiftquant_gemm_wgrad_finish(t, Ci, Co, bits, n_groups, x_scale, x_exp, g_scale, g_exp, dw,
+                                 acc_out, dev_status, stream=None) -> None:
+    """dW from the summed int32 sums of every shard (see the header)."""
+    _check(load().shiftquant_gemm_wgrad_finish(
+        _ptr(t), Ci, Co, bits, n_groups, _ptr(x_scale), _ptr(x_exp), _ptr(g_scale), _ptr(g_exp),
+        _ptr(dw), _ld(dw), _ptr(acc_out), _ld(acc_out) if acc_out is not None else 0,
         _ptr(dev_status), _stream(stream)))
 
 

@@ -374,3 +374,48 @@ def test_layer_chunks_from_exponents_stay_exact(bits, G, K):
     T = A @ Bf.T
     np.testing.assert_array_equal(acc.cpu().numpy(), T)
     assert_close_f32(y.cpu().numpy(), T.astype(np.float64) * 2.0 ** -(G - 1), "Y")
+
+
+@pytest.mark.parametrize("bits", [4, 6, 8])
+def test_token_shards_weight_gradient_is_exact(bits):
+    # data parallel over tokens, exactly: two shards quantized with the range exchange
+    # (layer.shard_shift_quantize), each shard's int32 weight-gradient sums
+    # (shiftquant_gemm_wgrad_partial), their sum standing in for the all-reduce, and one
+    # dequantizing pass (shiftquant_gemm_wgrad_finish) give the whole batch's dW and T
+    rng = np.random.default_rng(40 + bits)
+    M, K, Nn, G, seed = 3000, 320, 256, 4, 77
+    x, w, dy = layer_inputs(rng, M, K, Nn)
+    xg, dyg = to_gpu(x), to_gpu(dy)
+    whole = L.QuantLinear(M, K, Nn, bits, G, "cuda", with_acc=True)
+    whole.quantize_activation(xg)
+    whole.quantize_gradient(dyg, seed)
+    whole.wgrad()
+    st = torch.zeros(1, dtype=torch.int32, device="cuda")
+    bounds = [(0, 1337), (1337, M)]
+    qx = [L.ShiftTensor.alloc(r1 - r0, K, bits, G, "cuda") for r0, r1 in bounds]
+    qg = [L.ShiftTensor.alloc(r1 - r0, Nn, bits, G, "cuda") for r0, r1 in bounds]
+    for t, qs in ((xg, qx), (dyg, qg)):
+        parts = []
+        for (r0, r1), q in zip(bounds, qs):
+            N.shiftquant_calibrate(t[r0:r1], N.SQ_GRAN_PER_COL, G, q.range, None, None, st)
+            parts.append(q.range.clone())
+        both = torch.maximum(parts[0], parts[1])
+        mode, sd = (N.SQ_ROUND_NEAREST_EVEN, 0) if t is xg else (N.SQ_ROUND_STOCHASTIC, seed)
+        for (r0, r1), q in zip(bounds, qs):
+            L.shard_shift_quantize(t[r0:r1], q, bits, G, mode, sd, r0, st,
+                                   lambda r, both=both: r.copy_(both))
+    sums = []
+    for (r0, r1), a, b in zip(bounds, qx, qg):
+        tt = torch.full((K, Nn), -1, dtype=torch.int32, device="cuda")
+        N.shiftquant_gemm_wgrad_partial(a.codes_t, a.scale, a.exp, b.codes_t, b.scale, b.exp, K, Nn,
+                                        r1 - r0, M, bits, G, tt, st)
+        sums.append(tt)
+    total = sums[0] + sums[1]
+    dw = torch.empty((K, Nn), dtype=torch.float32, device="cuda")
+    acc = torch.empty((K, Nn), dtype=torch.int64, device="cuda")
+    N.shiftquant_gemm_wgrad_finish(total, K, Nn, bits, G, qx[0].scale, qx[0].exp, qg[0].scale,
+                                   qg[0].exp, dw, acc, st)
+    torch.cuda.synchronize()
+    assert st.item() == 0 and whole.status.item() == 0
+    np.testing.assert_array_equal(acc.cpu().numpy(), whole.acc["wgrad"].cpu().numpy())
+    np.testing.assert_array_equal(f32_bits(dw.cpu().numpy()), f32_bits(whole.dw.cpu().numpy()))

@@ -1,9 +1,10 @@
-"""The one exchange step of a tensor split by rows (tokens) across ranks, on CPU: two
-`gloo` ranks each hold a row shard, take its per-column ranges, all-reduce them with MAX,
-group, and quantize with the generator moved to the shard's first row
-(`layer.shard_seed`).  Every rank's ranges, tau_0, exponents, codes and scale must equal
-the whole tensor's, computed by the oracle (the CUDA path is exercised the same way by
-tests/test_gpu_quant.py on one GPU)."""
+"""Tensors split by rows (tokens) across ranks, on CPU with two `gloo` ranks and the oracle as
+each rank's compute.  Quantization: each rank takes its shard's per-column ranges,
+all-reduces them with MAX, groups, and quantizes with the generator moved to the shard's
+first row (`layer.shard_seed`); every rank's ranges, tau_0, exponents, codes and scale must
+equal the whole tensor's.  Weight gradient: the ranks' integer sums, all-reduced with SUM
+and dequantized once, must equal the whole batch's.  The CUDA path is exercised the same
+way on one GPU by tests/test_gpu_quant.py and tests/test_gpu_gemm.py."""
 import multiprocessing as mp
 import os
 import socket
@@ -89,3 +90,60 @@ def test_shard_seed_moves_the_generator_exactly():
         s = shard_seed(seed, r0, C)
         for r, c in ((0, 0), (3, 699), (17, 5)):
             assert O.hash64(s, r * C + c) == O.hash64(seed, (r0 + r) * C + c)
+
+
+def _wgrad_main(rank, world, port, bits, G, seed, bounds, out):
+    sys.path.insert(0, ROOT)
+    os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port), RANK=str(rank),
+                      WORLD_SIZE=str(world))
+    import torch
+    import torch.distributed as dist
+    import oracle as O
+    from paper_2411_10948_gb300.layer import shard_seed
+    dist.init_process_group("gloo", rank=rank, world_size=world)
+    try:
+        x = _tensor()
+        dy = _tensor()[:, ::-1].copy() * np.float32(0.5)
+        r0, r1 = bounds[rank], bounds[rank + 1]
+        q = {}
+        for name, t, mode, sd in (("x", x, 0, 0), ("g", dy, 1, seed)):
+            local, _ = O.range_cols(t[r0:r1])
+            rt = torch.from_numpy(local.copy())
+            dist.all_reduce(rt, op=dist.ReduceOp.MAX)
+            tau0, e, _ = O.group(rt.numpy(), G)
+            codes, s = O.quantize_shift(t[r0:r1], bits, G, tau0, e, mode,
+                                        shard_seed(sd, r0, t.shape[1]))
+            q[name] = (codes, e, s)
+        # the shard's weight-gradient sums (canonical, int64), summed over the ranks
+        T = torch.from_numpy(O.gemm_wgrad(q["x"][0], q["x"][1], q["g"][0], q["g"][1], G))
+        dist.all_reduce(T, op=dist.ReduceOp.SUM)
+        dw = O.dequant(T.numpy(), q["x"][2], q["g"][2], 2 * (G - 1))
+        ox = O.shiftquant_tensor(x, bits, G, 0, 0)
+        og = O.shiftquant_tensor(dy, bits, G, 1, seed)
+        T_whole = O.gemm_wgrad(ox["codes"], ox["exp"], og["codes"], og["exp"], G)
+        dw_whole = O.dequant(T_whole, ox["scale"], og["scale"], 2 * (G - 1))
+        ok = np.array_equal(T.numpy(), T_whole) and np.array_equal(dw.view(np.uint32),
+                                                                   dw_whole.view(np.uint32))
+        out.put((rank, bool(ok)))
+        dist.barrier()
+    finally:
+        dist.destroy_process_group()
+
+
+@pytest.mark.parametrize("bits", [4, 8])
+def test_two_gloo_ranks_sum_the_weight_gradient_exactly(bits):
+    # each rank's integer weight-gradient sums over its own tokens, all-reduced with SUM and
+    # dequantized once, equal the whole batch's dW bit for bit
+    world, G, seed, bounds = 2, 4, 0xBEEF, [0, 131, 300]
+    ctx = mp.get_context("spawn")
+    out = ctx.Queue()
+    port = _free_port()
+    procs = [ctx.Process(target=_wgrad_main, args=(r, world, port, bits, G, seed, bounds, out))
+             for r in range(world)]
+    for p in procs:
+        p.start()
+    got = sorted(out.get(timeout=180) for _ in range(world))
+    for p in procs:
+        p.join(timeout=60)
+        assert p.exitcode == 0
+    assert got == [(0, True), (1, True)]
