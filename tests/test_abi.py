@@ -157,3 +157,32 @@ def test_layer_struct_layout_matches_the_binding(tmp_path):
                                           check=True).stdout.split()]
     assert out[0] == ctypes.sizeof(SqLayerGemms)
     assert out[1:] == [getattr(SqLayerGemms, f).offset for f in fields]
+
+
+def test_sharding_entries_reject_bad_arguments_before_launch(lib):
+    # shiftquant_group, shiftquant_gemm_wgrad_partial / _finish: host checks only, no device
+    st = ctypes.c_void_p(4096)          # stand-in device pointers: never dereferenced here
+    odd = ctypes.c_void_p(4096 + 4)     # not 16-byte aligned
+    g = lib.shiftquant_group
+    assert g(st, 16, 0, st, st, st, None) == native.SQ_EINVAL      # n_groups
+    assert g(st, -1, 4, st, st, st, None) == native.SQ_EINVAL      # channels
+    assert g(None, 16, 4, st, st, st, None) == native.SQ_EINVAL    # range
+    assert g(st, 16, 4, None, st, st, None) == native.SQ_EINVAL    # tau0_out
+    assert g(st, 16, 4, st, st, None, None) == native.SQ_EINVAL    # dev_status
+    p = lambda **k: lib.shiftquant_gemm_wgrad_partial(
+        st, 64, st, st, st, 64, st, st, k.get("Ci", 32), k.get("Co", 32), k.get("T", 64),
+        k.get("total", 128), k.get("bits", 4), 4, k.get("t", st), st, None)
+    assert p(bits=1) == native.SQ_EINVAL
+    assert p(T=-1) == native.SQ_EINVAL
+    assert p(total=32) == native.SQ_EINVAL                          # total_tokens < T
+    assert p(t=odd) == native.SQ_EALIGN
+    assert p(Co=30) == native.SQ_EALIGN                             # Co % 4
+    assert p(bits=8, total=1 << 20) == native.SQ_EUNSUPPORTED      # beyond exact int32
+    assert p(Ci=0) == native.SQ_OK and p(Co=0) == native.SQ_OK     # empty: nothing to do
+    f = lambda **k: lib.shiftquant_gemm_wgrad_finish(
+        k.get("t", st), 32, k.get("Co", 32), 4, 4, st, st, st, st, k.get("dw", st),
+        k.get("ld", 32), None, 0, st, None)
+    assert f(t=odd) == native.SQ_EALIGN
+    assert f(Co=30) == native.SQ_EALIGN
+    assert f(dw=None) == native.SQ_EINVAL
+    assert f(ld=16) == native.SQ_EINVAL
