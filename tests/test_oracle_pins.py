@@ -323,8 +323,14 @@ def test_wgrad_equals_dequantize_then_exact_matmul(bits, G):
                        Fraction(int(c["codes"][m, j])) * sc / 2 ** int(c["exp"][j])
                        for m in range(M)), Fraction(0))
             assert Fraction(int(T[i, j])) * sa * sc / 2 ** (2 * (G - 1)) == ref
+    # the two-scale dequantization (App. D with both operands ShiftQuant-ed): Y is the
+    # exact rational T s_X s_dY 2^-2(G-1) rounded to binary64 once (s_X s_dY is exact
+    # there) and then to binary32
     Y = O.dequant(T, a["scale"], c["scale"], 2 * (G - 1))
-    assert np.isfinite(Y).all()
+    for i in range(K):
+        for j in range(N):
+            exact = Fraction(int(T[i, j])) * sa * sc / 2 ** (2 * (G - 1))
+            assert float(Y[i, j]) == float(np.float32(float(exact))), (i, j)
 
 
 def test_int8_per_tensor_special_case_is_plain_integer_gemm():
@@ -384,3 +390,83 @@ def test_worked_ties_round_to_even():
     d = O.shiftquant_tensor(x, 4, 4, mode=0)
     np.testing.assert_array_equal(d["exp"], exp)
     np.testing.assert_array_equal(d["codes"], codes)
+
+
+def test_dequant_by_hand():
+    # Y = T s_a s_b 2^-shift col_scale[j]: 3 * 0.5 * 0.25 / 4 = 0.09375 and, with a column
+    # scale of 3, -5 * 0.5 * 0.25 / 4 * 3 = -0.46875 (all exact)
+    T = np.array([[3, -5]], np.int64)
+    Y = O.dequant(T, np.float32(0.5), np.float32(0.25), 2)
+    assert Y.tolist() == [[0.09375, -0.15625]]
+    Y = O.dequant(T, np.float32(0.5), np.float32(0.25), 2, np.array([1.0, 3.0], np.float32))
+    assert Y.tolist() == [[0.09375, -0.46875]]
+
+
+# ------------------------------------------------ per-channel weights (Sec. 5.1)
+def test_per_row_weight_worked_example():
+    toks = _read_golden("worked_example_per_row_b4.txt")
+    bits = int(toks[0].split()[1])
+    w = np.array([[float(v) for v in toks[2 + k].split()] for k in range(3)], np.float32)
+    rng = np.array([float(v) for v in toks[5].split()[1:]], np.float32)
+    num = [np.float32(float(v)) for v in toks[6].split()[1:]]
+    den = np.float32(float(toks[7].split()[1]))
+    codes = np.array([[int(v) for v in toks[9 + k].split()] for k in range(3)], np.int8)
+    d = O.channel_tensor(w, bits, axis=1)
+    assert d["status"] == 0
+    np.testing.assert_array_equal(d["range"], rng)
+    np.testing.assert_array_equal(d["codes"], codes)
+    # the scales are binary32 quotients range / Q (numpy's IEEE division)
+    np.testing.assert_array_equal(d["scale"], np.array([n / den for n in num], np.float32))
+
+
+@pytest.mark.parametrize("axis", [0, 1])
+@pytest.mark.parametrize("bits", [4, 6, 8])
+def test_rn_error_per_channel_weights(axis, bits):
+    # per channel (a column for axis 0, a row for axis 1): |w - q s| <= s (1/2 + 2^-15),
+    # s = range / Q, and the element of largest magnitude of a channel maps to +-Q
+    rng = np.random.default_rng(40 + 3 * bits + axis)
+    R, C = 23, 17
+    w = (rng.standard_normal((R, C)) * np.exp(rng.normal(0, 1, (R, 1)))
+         * np.exp(rng.normal(0, 1, (1, C)))).astype(np.float32)
+    w[4, :] = 0
+    w[:, 6] = 0
+    d = O.channel_tensor(w, bits, axis=axis)
+    Q = 2 ** (bits - 1) - 1
+    q = d["codes"].astype(np.int64)
+    assert np.abs(q).max() <= Q
+    wt = w if axis == 0 else w.T          # channels along the columns of wt
+    qt = q if axis == 0 else q.T
+    rg = np.abs(wt.astype(np.float64)).max(0)
+    np.testing.assert_array_equal(d["range"], rg.astype(np.float32))
+    s = d["scale"].astype(np.float64)
+    err = np.abs(wt.astype(np.float64) - qt * s[None, :])
+    assert (err <= s[None, :] * (0.5 + 2.0 ** -15) + 0.0).all()
+    for ch in range(wt.shape[1]):
+        if rg[ch] == 0:
+            assert s[ch] == 0 and (qt[:, ch] == 0).all()
+        else:
+            i = int(np.argmax(np.abs(wt[:, ch])))
+            assert abs(int(qt[i, ch])) == Q
+
+
+# ------------------------------------------------------- SR draw (App. B, R6)
+def _parse_sr_golden():
+    toks = _read_golden("sr_draws_seed0.txt")
+    cases = []
+    for i in range(0, len(toks), 3):
+        head, xs, cs = toks[i].split(), toks[i + 1].split(), toks[i + 2].split()
+        assert head[0] == "case" and xs[0] == "x24" and cs[0] == "codes"
+        x = np.array([int(v) * 2.0 ** -24 for v in xs[1:]], np.float64).reshape(2, 2)
+        assert (x.astype(np.float32).astype(np.float64) == x).all()   # exact in binary32
+        cases.append((head[1], int(head[2], 16), x.astype(np.float32),
+                      np.array([int(v) for v in cs[1:]], np.int8).reshape(2, 2)))
+    return cases
+
+
+def test_sr_draws_match_published_generator_outputs():
+    cases = _parse_sr_golden()
+    assert len(cases) == 6
+    for name, seed, x, codes in cases:
+        d = O.shiftquant_tensor(x, 4, 1, mode=1, seed=seed)
+        assert float(d["tau0"]) == 7.0 and (d["exp"] == 0).all()
+        np.testing.assert_array_equal(d["codes"], codes, err_msg=name)
