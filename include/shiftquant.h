@@ -102,9 +102,8 @@ sq_status shiftquant_calibrate(const float *x, int64_t rows, int64_t cols, int64
  *   2. replaces them by their element-wise maximum over the shards (an all-reduce(max):
  *      exact, as a maximum of floats is),
  *   3. calls shiftquant_group on the result, and
- *   4. quantizes with SQ_GRAN_SHIFT; stochastic rounding draws the whole tensor's numbers
- *      when a shard starting at row r0 passes seed + r0 * cols * 0x9E3779B97F4A7C15
- *      (mod 2^64) as its seed, since the generator's state is linear in the index. */
+ *   4. quantizes with SQ_GRAN_SHIFT, passing the shard's first row as row0 to
+ *      shiftquant_quantize, so that stochastic rounding draws the whole tensor's numbers. */
 sq_status shiftquant_group(const float *range, int64_t channels, int n_groups,
                            float *tau0_out, uint8_t *exp_out, int32_t *dev_status,
                            void *stream);
@@ -123,7 +122,10 @@ sq_status shiftquant_group(const float *range, int64_t channels, int n_groups,
  *     ShiftMM shift of Eq. 4 enters the contraction at no cost.
  *   mode: SQ_ROUND_NEAREST_EVEN (ties to even) or SQ_ROUND_STOCHASTIC: up with
  *     probability frac(v) using u = (SplitMix64(seed + (idx+1) 0x9E3779B97F4A7C15) >> 40)
- *     2^-24, idx = r * cols + c.
+ *     2^-24, idx = (row0 + r) * cols + c.
+ *   row0 (>= 0): the index of x's first row within the logical tensor.  0 for a whole
+ *     tensor; a row (token) shard starting at row r0 passes r0 and draws exactly the
+ *     numbers the whole tensor draws for those rows (see shiftquant_group).
  *   Outputs (codes in the type of shiftquant_code_type(bits, n_groups)):
  *     codes [rows, ld_codes] (may be NULL), codes_t [cols, ld_t], the transpose (may be
  *     NULL); at least one must be given.  tau_0 == 0 (or Q/tau_0 overflowing) gives
@@ -131,8 +133,8 @@ sq_status shiftquant_group(const float *range, int64_t channels, int n_groups,
 sq_status shiftquant_quantize(const float *x, int64_t rows, int64_t cols, int64_t ld,
                               int gran, int bits, int n_groups, const float *range_or_tau0,
                               const uint8_t *exp, const uint8_t *fold_exp, int mode,
-                              uint64_t seed, void *codes, int64_t ld_codes, void *codes_t,
-                              int64_t ld_t, float *scale_out, void *stream);
+                              uint64_t seed, int64_t row0, void *codes, int64_t ld_codes,
+                              void *codes_t, int64_t ld_t, float *scale_out, void *stream);
 
 /* Forward GEMM Y[M, N] = X[M, K] W[K, N] on quantized operands (Eq. 4 with the roles of
  * Sec. 5.1):
@@ -293,9 +295,11 @@ int shiftquant_gemm_layer_cta_pairs(int64_t M, int64_t K, int64_t N, int bits, i
  *     library until the process exits).  Ci * Co must not exceed 1048576; larger outputs
  *     return SQ_EUNSUPPORTED before anything is launched.
  *   Nothing is allocated: no cudaMalloc, no cudaFree, no allocating library routine.
- *   The first call on each device looks up the array's device address
- *     (cudaGetSymbolAddress) with that device current; make that first call before any
- *     stream capture begins.
+ *   Each call made outside stream capture looks up the array's device address
+ *     (cudaGetSymbolAddress) with the call's device current, so a device reset between
+ *     calls is harmless; a call made while its stream is being captured reuses the address
+ *     of the device's last such lookup.  The first call on each device must therefore come
+ *     before any stream capture begins (a first call during capture returns SQ_EINVAL).
  *   All calls on a device share the one array, and it keeps the last call's contents
  *     (each call clears the part it uses before use).  Two calls whose work overlaps on
  *     the GPU -- on different streams, or from different host threads -- race on it and

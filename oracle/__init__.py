@@ -58,7 +58,7 @@ def _load():
         lib.sqo_range_rows.argtypes = [vp, i64, i64, i64, vp]
         lib.sqo_group.argtypes = [vp, i64, i32, vp, vp]
         lib.sqo_quantize_shift.argtypes = [vp, i64, i64, i64, i32, i32, f32, vp, i32, u64,
-                                           vp, vp]
+                                           i64, vp, vp]
         lib.sqo_quantize_channel.argtypes = [vp, i64, i64, i64, i32, i32, vp, i32, u64, vp,
                                              vp]
         lib.sqo_gemm_fwd.argtypes = [vp, vp, vp, i64, i64, i64, i32, vp, i64, vp]
@@ -131,14 +131,15 @@ def group(ranges, n_groups: int) -> tuple[np.float32, np.ndarray, int]:
 
 # --------------------------------------------------------- App. D quantization
 def quantize_shift(x, bits: int, n_groups: int, tau0, exps, mode: int = 0,
-                   seed: int = 0) -> tuple[np.ndarray, np.float32]:
-    """ShiftQuant codes (int8 [R, C]) and the tensor scale s = tau_0 / Q."""
+                   seed: int = 0, row0: int = 0) -> tuple[np.ndarray, np.float32]:
+    """ShiftQuant codes (int8 [R, C]) and the tensor scale s = tau_0 / Q.  x holds rows
+    row0.. of the logical tensor (stochastic rounding draws by the logical index)."""
     x = _f32(x)
     e = np.ascontiguousarray(exps, dtype=np.uint8)
     q = np.empty(x.shape, np.int8)
     s = np.zeros(1, np.float32)
     _load().sqo_quantize_shift(_p(x), x.shape[0], x.shape[1], x.shape[1], bits, n_groups,
-                               np.float32(tau0), _p(e), mode, seed & (2**64 - 1), _p(q),
+                               np.float32(tau0), _p(e), mode, seed & (2**64 - 1), row0, _p(q),
                                _p(s))
     return q, np.float32(s[0])
 

@@ -172,10 +172,12 @@ static int32_t sqo_round(float v, int mode, uint64_t seed, uint64_t idx, int32_t
 
 /* ------------------------------------------- App. D (R3): group quantizer */
 /* code[r, c] = round(x[r, c] / ((tau_0 / Q) 2^-e_c)), computed as
- * fl(fl(x * 2^e_c) * fl(Q / tau_0)) then rounded; the first product is exact. */
+ * fl(fl(x * 2^e_c) * fl(Q / tau_0)) then rounded; the first product is exact.
+ * The R rows of x are rows row0 .. row0+R-1 of the logical tensor (a row shard of it):
+ * stochastic rounding draws with the logical index (row0 + r) * C + c (R6). */
 int sqo_quantize_shift(const float *x, int64_t R, int64_t C, int64_t ld, int bits, int G,
-                       float tau0, const uint8_t *exp, int mode, uint64_t seed, int8_t *q,
-                       float *scale_out) {
+                       float tau0, const uint8_t *exp, int mode, uint64_t seed, int64_t row0,
+                       int8_t *q, float *scale_out) {
     (void)G;
     const int32_t Q = (1 << (bits - 1)) - 1;
     float invS = (float)Q / tau0;
@@ -187,7 +189,7 @@ int sqo_quantize_shift(const float *x, int64_t R, int64_t C, int64_t ld, int bit
             if (!zero_mode) {
                 float xs = ldexpf(x[r * ld + c], (int)exp[c]);
                 float v = xs * invS;
-                code = sqo_round(v, mode, seed, (uint64_t)(r * C + c), Q);
+                code = sqo_round(v, mode, seed, (uint64_t)((row0 + r) * C + c), Q);
             }
             q[r * C + c] = (int8_t)code;
         }

@@ -1528,21 +1528,30 @@ constexpr size_t kStaticScratchBytes = size_t(4) << 20;   // the int32 sums of 2
 static __device__ __align__(256) int g_wgrad_scratch[kStaticScratchBytes / sizeof(int)];
 
 // Device address of g_wgrad_scratch on the current device.  In host code the array's
-// name only stands in for the symbol, so the address is looked up once per device with
-// that device current and cached.
-static int static_scratch_address(void** out) {
+// name only stands in for the symbol, so the address is looked up with the device
+// current: on every call made outside stream capture (a device reset re-creates the
+// array elsewhere, and the lookup is cheap), and the last address found is kept per device
+// for calls made while `s` is being captured, which must not make that lookup.
+static int static_scratch_address(void** out, cudaStream_t s) {
   static void* addr[64] = {};
   static std::mutex mu;
   int dev = 0;
   cudaError_t err = cudaGetDevice(&dev);
   if (err != cudaSuccess) return cuda_fail(err, "cudaGetDevice");
   if (dev < 0 || dev >= 64) return fail(SQ_EUNSUPPORTED, "device index %d beyond 63", dev);
+  cudaStreamCaptureStatus cap = cudaStreamCaptureStatusNone;
+  err = cudaStreamIsCapturing(s, &cap);
+  if (err != cudaSuccess) return cuda_fail(err, "cudaStreamIsCapturing");
   std::lock_guard<std::mutex> lock(mu);
-  if (addr[dev] == nullptr) {
+  if (cap == cudaStreamCaptureStatusNone) {
     void* p = nullptr;
     err = cudaGetSymbolAddress(&p, g_wgrad_scratch);
     if (err != cudaSuccess) return cuda_fail(err, "cudaGetSymbolAddress");
     addr[dev] = p;
+  } else if (addr[dev] == nullptr) {
+    return fail(SQ_EINVAL,
+                "gemm_wgrad_static: the first call on a device must come before any stream "
+                "capture (it looks up the scratch array's address)");
   }
   *out = addr[dev];
   return SQ_OK;
@@ -1683,15 +1692,16 @@ extern "C" sq_status shiftquant_gemm_wgrad_static(
     int64_t Co, int64_t T, int bits, int n_groups, float* dw, int64_t ld_dw, int64_t* acc_out,
     int64_t ld_acc, int32_t* dev_status, void* stream) {
   fail(SQ_OK, "");
-  if (Ci > 0 && Co > 0 && Ci * Co > kStaticMaxOutputs)
+  // compared by division, so that no product of huge sizes can overflow
+  if (Ci > 0 && Co > 0 && (Ci > kStaticMaxOutputs || Co > kStaticMaxOutputs / Ci))
     return fail(SQ_EUNSUPPORTED,
-                "gemm_wgrad_static: Ci * Co = %lld exceeds the %lld outputs of the library's "
-                "static scratch; use shiftquant_gemm_wgrad with a caller workspace",
-                static_cast<long long>(Ci) * static_cast<long long>(Co),
+                "gemm_wgrad_static: Ci = %lld, Co = %lld exceed the %lld outputs of the "
+                "library's static scratch; use shiftquant_gemm_wgrad with a caller workspace",
+                static_cast<long long>(Ci), static_cast<long long>(Co),
                 static_cast<long long>(kStaticMaxOutputs));
   void* scratch = nullptr;
   if (Ci > 0 && Co > 0 && T > 0) {
-    const int st = static_scratch_address(&scratch);
+    const int st = static_scratch_address(&scratch, as_stream(stream));
     if (st != SQ_OK) return st;
   }
   return run_gemm(2, xt_codes, ldx, gt_codes, ldg, Ci, Co, T, bits, n_groups, x_scale, g_scale,

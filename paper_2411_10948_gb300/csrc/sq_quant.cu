@@ -249,6 +249,7 @@ struct QuantArgs {
   int64_t R, C, ld;
   int gran, Q, G, mode;
   uint64_t seed;
+  int64_t row0;           // the tensor's first row within the logical tensor (SR index)
   const float* rt;        // &tau_0 (SHIFT) or range[] (PER_COL / PER_ROW)
   const uint8_t* exp;     // SHIFT: e_c
   const uint8_t* fold;    // optional: exponents of the other GEMM operand
@@ -414,7 +415,7 @@ __device__ __forceinline__ void quantize_tile(const QuantArgs& a, uint8_t* tile_
       } else {
         const float l = floorf(v);
         const float frac = __fsub_rn(v, l);
-        const uint64_t hsh = splitmix64_at(a.seed, static_cast<uint64_t>(r * a.C + cb + j));
+        const uint64_t hsh = splitmix64_at(a.seed, static_cast<uint64_t>((a.row0 + r) * a.C + cb + j));
         const float u = __fmul_rn(static_cast<float>(static_cast<uint32_t>(hsh >> 40)),
                                   5.9604644775390625e-08f);  // * 2^-24, exact
         q = (u < frac) ? __fadd_rn(l, 1.0f) : l;
@@ -714,12 +715,14 @@ extern "C" sq_status shiftquant_quantize(const float* x, int64_t rows, int64_t c
                                          int gran, int bits, int n_groups,
                                          const float* range_or_tau0, const uint8_t* exp,
                                          const uint8_t* fold_exp, int mode, uint64_t seed,
-                                         void* codes, int64_t ld_codes, void* codes_t,
-                                         int64_t ld_t, float* scale_out, void* stream) {
+                                         int64_t row0, void* codes, int64_t ld_codes,
+                                         void* codes_t, int64_t ld_t, float* scale_out,
+                                         void* stream) {
   clear_error();
   if (!bits_ok(bits) || !groups_ok(n_groups))
     return fail(SQ_EINVAL, "quantize: bits must be in [2, 8] and n_groups in [1, 8]");
   if (rows < 0 || cols < 0) return fail(SQ_EINVAL, "quantize: negative size");
+  if (row0 < 0) return fail(SQ_EINVAL, "quantize: negative row0");
   if (gran < SQ_GRAN_SHIFT || gran > SQ_GRAN_PER_ROW) return fail(SQ_EINVAL, "quantize: bad gran");
   if (mode != SQ_ROUND_NEAREST_EVEN && mode != SQ_ROUND_STOCHASTIC)
     return fail(SQ_EINVAL, "quantize: bad rounding mode");
@@ -755,6 +758,7 @@ extern "C" sq_status shiftquant_quantize(const float* x, int64_t rows, int64_t c
   a.G = n_groups;
   a.mode = mode;
   a.seed = seed;
+  a.row0 = row0;
   a.rt = range_or_tau0;
   a.exp = exp;
   a.fold = fold_exp;

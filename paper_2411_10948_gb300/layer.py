@@ -67,30 +67,19 @@ def shift_quantize(x, q: ShiftTensor, bits, n_groups, mode, seed, status, stream
                           q.codes, q.codes_t, q.scale, stream)
 
 
-# SplitMix64's increment: the stochastic-rounding generator's state is seed + (idx+1) * this
-SPLITMIX_GAMMA = 0x9E3779B97F4A7C15
-
-
-def shard_seed(seed: int, row0: int, cols: int) -> int:
-    """The seed under which a row shard starting at row `row0` of a [*, cols] tensor draws
-    the same stochastic-rounding numbers as the whole tensor does for those rows: the
-    generator's state, seed + (r cols + c + 1) gamma, is linear in the element index."""
-    return (seed + row0 * cols * SPLITMIX_GAMMA) % (1 << 64)
-
-
 def shard_shift_quantize(x, q: ShiftTensor, bits, n_groups, mode, seed, row0, status,
                          all_reduce_max, stream=None):
     """ShiftQuant of one row (token) shard x [R_local, C] of a tensor split across ranks,
     equal bit for bit to the whole tensor's rows: the shard's per-column ranges, their
     element-wise maximum over all shards (all_reduce_max(tensor) in place -- for instance
     torch.distributed.all_reduce with ReduceOp.MAX: the one exchange the path needs), the
-    grouping from that, and the quantizer with the generator moved to the shard's first
-    row (row0 in the whole tensor)."""
+    grouping from that, and the quantizer told the shard's first row (row0 in the whole
+    tensor), so that stochastic rounding draws the whole tensor's numbers."""
     N.shiftquant_calibrate(x, N.SQ_GRAN_PER_COL, n_groups, q.range, None, None, status, stream)
     all_reduce_max(q.range)
     N.shiftquant_group(q.range, n_groups, q.tau0, q.exp, status, stream)
     N.shiftquant_quantize(x, N.SQ_GRAN_SHIFT, bits, n_groups, q.tau0, q.exp, None, mode,
-                          shard_seed(seed, row0, x.shape[1]), q.codes, q.codes_t, q.scale, stream)
+                          seed, q.codes, q.codes_t, q.scale, stream, row0=row0)
 
 
 def weight_quantize_fwd(w, out: ChannelTensor, fold_exp, bits, n_groups, status, stream=None):

@@ -103,7 +103,7 @@ def load(path: str | None = None) -> ctypes.CDLL:
                                                  vp, i64, vp, vp]
     lib.shiftquant_gemm_wgrad_finish.restype = i32
     lib.shiftquant_quantize.argtypes = [vp, i64, i64, i64, i32, i32, i32, vp, vp, vp, i32, u64,
-                                        vp, i64, vp, i64, vp, vp]
+                                        i64, vp, i64, vp, i64, vp, vp]
     lib.shiftquant_quantize.restype = i32
     gemm = [vp, i64, vp, vp, i64, vp, i64, i64, i64, i32, i32, vp, i64, vp, i64, vp, sz, vp, vp]
     lib.shiftquant_gemm_fwd.argtypes = gemm
@@ -192,10 +192,10 @@ def shiftquant_group(range_, n_groups, tau0_out, exp_out, dev_status, stream=Non
 
 
 def shiftquant_quantize(x, gran, bits, n_groups, range_or_tau0, exp, fold_exp, mode, seed,
-                        codes, codes_t, scale_out, stream=None) -> None:
+                        codes, codes_t, scale_out, stream=None, row0=0) -> None:
     _check(load().shiftquant_quantize(
         _ptr(x), x.shape[0], x.shape[1], _ld(x), gran, bits, n_groups, _ptr(range_or_tau0),
-        _ptr(exp), _ptr(fold_exp), mode, seed & (2**64 - 1), _ptr(codes),
+        _ptr(exp), _ptr(fold_exp), mode, seed & (2**64 - 1), row0, _ptr(codes),
         _ld(codes) if codes is not None else 0, _ptr(codes_t),
         _ld(codes_t) if codes_t is not None else 0, _ptr(scale_out), _stream(stream)))
 

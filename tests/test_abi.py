@@ -76,19 +76,21 @@ def test_host_validation_rejects_before_launch(lib):
     assert lib.shiftquant_calibrate(st, 4, 8, 4, 0, 4, st, st, st, st, None) == native.SQ_EINVAL
     # quantize: bits, rounding mode, SHIFT with fold_exp, no outputs
     args = dict(x=st, rows=4, cols=4, ld=4, gran=0, bits=4, g=4, rt=st, exp=st, fold=None,
-                mode=0, seed=0, codes=st, ldc=16, codes_t=None, ldt=0, scale=st, s=None)
+                mode=0, seed=0, row0=0, codes=st, ldc=16, codes_t=None, ldt=0, scale=st,
+                s=None)
 
     def q(**kw):
         a = dict(args, **kw)
         return lib.shiftquant_quantize(a["x"], a["rows"], a["cols"], a["ld"], a["gran"],
                                        a["bits"], a["g"], a["rt"], a["exp"], a["fold"], a["mode"],
-                                       a["seed"], a["codes"], a["ldc"], a["codes_t"], a["ldt"],
-                                       a["scale"], a["s"])
+                                       a["seed"], a["row0"], a["codes"], a["ldc"], a["codes_t"],
+                                       a["ldt"], a["scale"], a["s"])
     assert q(bits=9) == native.SQ_EINVAL
     assert q(mode=5) == native.SQ_EINVAL
     assert q(fold=st) == native.SQ_EINVAL
     assert q(codes=None) == native.SQ_EINVAL
     assert q(ldc=2) == native.SQ_EINVAL
+    assert q(row0=-1) == native.SQ_EINVAL
     # gemm: misaligned operand and leading dimension (TMA needs 16-byte rows)
     a16, a_odd = ctypes.c_void_p(256), ctypes.c_void_p(257)
     g = lib.shiftquant_gemm_fwd
@@ -126,7 +128,7 @@ def test_empty_shapes_accept_null_pointers_of_empty_buffers(lib):
         ex = fake if C else None
         r = lib.shiftquant_calibrate(None, R, C, max(C, 1), 0, 4, rng, fake, ex, fake, None)
         assert r != native.SQ_EINVAL, (R, C, lib.shiftquant_last_error())
-        r = lib.shiftquant_quantize(None, R, C, max(C, 1), 0, 4, 4, fake, ex, None, 0, 0,
+        r = lib.shiftquant_quantize(None, R, C, max(C, 1), 0, 4, 4, fake, ex, None, 0, 0, 0,
                                     fake if R and C else None, 16, None, 0, fake, None)
         assert r != native.SQ_EINVAL, (R, C, lib.shiftquant_last_error())
         for gran in (1, 2):
@@ -135,8 +137,8 @@ def test_empty_shapes_accept_null_pointers_of_empty_buffers(lib):
                                          fake if ch else None, None, None, fake, None)
             assert r != native.SQ_EINVAL, (gran, R, C, lib.shiftquant_last_error())
             r = lib.shiftquant_quantize(None, R, C, max(C, 1), gran, 4, 4,
-                                        fake if ch else None, None, None, 0, 0, None, 0, None,
-                                        0, fake if ch else None, None)
+                                        fake if ch else None, None, None, 0, 0, 0, None, 0,
+                                        None, 0, fake if ch else None, None)
             assert r != native.SQ_EINVAL, (gran, R, C, lib.shiftquant_last_error())
 
 
@@ -186,3 +188,15 @@ def test_sharding_entries_reject_bad_arguments_before_launch(lib):
     assert f(Co=30) == native.SQ_EALIGN
     assert f(dw=None) == native.SQ_EINVAL
     assert f(ld=16) == native.SQ_EINVAL
+
+
+def test_static_weight_gradient_rejects_oversized_outputs_before_anything_else(lib):
+    # the 2^20-output limit of the library's static scratch is checked first and without
+    # forming Ci * Co (huge sizes must not wrap past it)
+    st = ctypes.c_void_p(16)
+    a16 = ctypes.c_void_p(256)
+    f = lib.shiftquant_gemm_wgrad_static
+    for ci, co in ((2**40, 2**40), (2**62, 4), (4, 2**62), ((1 << 20) + 1, 1), (1025, 1024)):
+        r = f(a16, 64, st, st, a16, 64, st, st, ci, co, 64, 4, 4, st, co, None, 0, st, None)
+        assert r == native.SQ_EUNSUPPORTED, (ci, co)
+        assert "static scratch" in lib.shiftquant_last_error().decode()

@@ -1,7 +1,7 @@
 """Tensors split by rows (tokens) across ranks, on CPU with two `gloo` ranks and the oracle as
 each rank's compute.  Quantization: each rank takes its shard's per-column ranges,
-all-reduces them with MAX, groups, and quantizes with the generator moved to the shard's
-first row (`layer.shard_seed`); every rank's ranges, tau_0, exponents, codes and scale must
+all-reduces them with MAX, groups, and quantizes telling the quantizer the shard's first
+row (row0: stochastic rounding draws by the logical index); every rank's ranges, tau_0, exponents, codes and scale must
 equal the whole tensor's.  Weight gradient: the ranks' integer sums, all-reduced with SUM
 and dequantized once, must equal the whole batch's.  The CUDA path is exercised the same
 way on one GPU by tests/test_gpu_quant.py and tests/test_gpu_gemm.py."""
@@ -38,7 +38,6 @@ def _shard_main(rank, world, port, bits, G, mode, seed, bounds, out):
     import torch
     import torch.distributed as dist
     import oracle as O
-    from paper_2411_10948_gb300.layer import shard_seed
     dist.init_process_group("gloo", rank=rank, world_size=world)
     try:
         x = _tensor()
@@ -49,7 +48,7 @@ def _shard_main(rank, world, port, bits, G, mode, seed, bounds, out):
         dist.all_reduce(t, op=dist.ReduceOp.MAX)   # the exchange
         rng = t.numpy()
         tau0, e, _ = O.group(rng, G)
-        q, s = O.quantize_shift(shard, bits, G, tau0, e, mode, shard_seed(seed, r0, x.shape[1]))
+        q, s = O.quantize_shift(shard, bits, G, tau0, e, mode, seed, row0=r0)
         whole = O.shiftquant_tensor(x, bits, G, mode, seed)
         ok = (np.array_equal(rng.view(np.uint32), whole["range"].view(np.uint32))
               and np.float32(tau0).view(np.uint32) == np.float32(whole["tau0"]).view(np.uint32)
@@ -79,17 +78,20 @@ def test_two_gloo_ranks_quantize_their_shards_as_the_whole_tensor(bits, mode):
     assert got == [(0, True), (1, True)]
 
 
-def test_shard_seed_moves_the_generator_exactly():
-    # the element (r, c) of a shard starting at row r0 draws what element (r0 + r, c) of the
-    # whole tensor draws
+def test_row_offset_draws_the_whole_tensors_numbers():
+    # rows row0.. of a tensor quantized alone with row0 draw what the whole tensor draws for
+    # them: the stochastic codes of every shard equal the whole tensor's rows, and without the
+    # offset they do not
     sys.path.insert(0, ROOT)
     import oracle as O
-    from paper_2411_10948_gb300.layer import shard_seed
-    seed, C = 0xDEADBEEF12345678, 700
-    for r0 in (0, 1, 1201, 10**6):
-        s = shard_seed(seed, r0, C)
-        for r, c in ((0, 0), (3, 699), (17, 5)):
-            assert O.hash64(s, r * C + c) == O.hash64(seed, (r0 + r) * C + c)
+    x = _tensor()
+    G, bits, seed = 4, 4, 0xDEADBEEF12345678
+    whole = O.shiftquant_tensor(x, bits, G, 1, seed)
+    for r0, r1 in ((0, 1), (1, 40), (131, 300), (299, 300)):
+        q, _ = O.quantize_shift(x[r0:r1], bits, G, whole["tau0"], whole["exp"], 1, seed, row0=r0)
+        np.testing.assert_array_equal(q, whole["codes"][r0:r1])
+    q, _ = O.quantize_shift(x[131:300], bits, G, whole["tau0"], whole["exp"], 1, seed)
+    assert (q != whole["codes"][131:300]).any()
 
 
 def _wgrad_main(rank, world, port, bits, G, seed, bounds, out):
@@ -99,7 +101,6 @@ def _wgrad_main(rank, world, port, bits, G, seed, bounds, out):
     import torch
     import torch.distributed as dist
     import oracle as O
-    from paper_2411_10948_gb300.layer import shard_seed
     dist.init_process_group("gloo", rank=rank, world_size=world)
     try:
         x = _tensor()
@@ -111,8 +112,7 @@ def _wgrad_main(rank, world, port, bits, G, seed, bounds, out):
             rt = torch.from_numpy(local.copy())
             dist.all_reduce(rt, op=dist.ReduceOp.MAX)
             tau0, e, _ = O.group(rt.numpy(), G)
-            codes, s = O.quantize_shift(t[r0:r1], bits, G, tau0, e, mode,
-                                        shard_seed(sd, r0, t.shape[1]))
+            codes, s = O.quantize_shift(t[r0:r1], bits, G, tau0, e, mode, sd, row0=r0)
             q[name] = (codes, e, s)
         # the shard's weight-gradient sums (canonical, int64), summed over the ranks
         T = torch.from_numpy(O.gemm_wgrad(q["x"][0], q["x"][1], q["g"][0], q["g"][1], G))
