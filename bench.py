@@ -37,9 +37,13 @@ sys.path.insert(0, ROOT)
 
 METRIC = "ShiftQuant GEMM TOPS & % dense-INT8 peak; quantizer GB/s & % HBM peak"
 UNIT = "TOPS"
-DEFAULT_WORKLOAD = "conv3x3"
+DEFAULT_WORKLOAD = "large_linear"
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 FP8_OVER_BF16 = 2.0    # nominal dense ratio (4.5 vs 2.25 PFLOP/s)
+# dense tensor-core operations per SM per clock (BF16; E4M3 is twice that): the clock-derived
+# peak at the sampled SM clock sits beside the measured cuBLAS peak, whose run was power-capped
+# at a lower clock than these short launches see
+BF16_OPS_PER_SM_CLOCK = 8192
 L2_FLUSH_BYTES = 256 << 20
 
 
@@ -53,7 +57,9 @@ def parse_args():
     ap.add_argument("--seed", type=int, default=0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
-    ap.add_argument("--also", default="large_linear",
+    ap.add_argument("--no-chain", action="store_true",
+                    help="skip the fused-range chain measurement")
+    ap.add_argument("--also", default="conv3x3",
                     help="second workload summarised in the same line ('none' for none)")
     return ap.parse_args()
 
@@ -392,32 +398,35 @@ def run_ours(args, rank, world, local_rank):
     total_ms = max_over_ranks(sum(step_ms), dev)
     ms_per_step = total_ms / args.steps
 
-    # e2e: the library's host pipeline (layer.HostPipeline): every step copies its inputs in
-    # from pinned host memory, runs, and copies Y, dX, dW back; step i+1's inputs and step
-    # i-1's outputs move while step i computes.  Timed from the first copy in to the last
-    # copy back.
+    # e2e: the C entry point shiftquant_layer_step_host (layer.HostSteps): every call copies a
+    # layer's X, W and dY in from pinned host memory, runs its whole step and copies Y, dX and
+    # dW back; two device buffer sets on two streams take the steps in turn.  Timed from the
+    # first copy in to the last copy back.
     e2e = None
     if not args.no_e2e:
         host_in = [[a.cpu().pin_memory() for a in inp] for inp in st.inputs]
-        host_out = [[torch.empty(o.shape, dtype=o.dtype, pin_memory=True) for o in (l.y, l.dx, l.dw)]
-                    for l in st.layers]
+        slots = 2
+        host_out = [[[torch.empty(o.shape, dtype=o.dtype, pin_memory=True)
+                      for o in (l.y, l.dx, l.dw)] for l in st.layers] for _ in range(slots)]
         h2d = sum(a.numel() * a.element_size() for inp in host_in for a in inp)
-        d2h = sum(a.numel() * a.element_size() for outs in host_out for a in outs)
-        pipe = L.HostPipeline([(s.M, s.K, s.N) for s in st.specs], st.specs[0].bits,
-                              st.specs[0].n_groups, dev)
-        pipe.run([host_in] * args.warmup, [host_out] * args.warmup).synchronize()
+        d2h = sum(a.numel() * a.element_size() for outs in host_out[0] for a in outs)
+        pipe = L.HostSteps([(s.M, s.K, s.N) for s in st.specs], st.specs[0].bits,
+                           st.specs[0].n_groups, dev, slots=slots)
+        outs = lambda n: [host_out[i % slots] for i in range(n)]
+        pipe.run([host_in] * args.warmup, outs(args.warmup)).synchronize()
         torch.cuda.synchronize()
         a = torch.cuda.Event(enable_timing=True)
-        a.record(pipe.s_in)
-        end = pipe.run([host_in] * args.steps, [host_out] * args.steps)
+        a.record(torch.cuda.current_stream())
+        end = pipe.run([host_in] * args.steps, outs(args.steps))
         end.synchronize()
         e_total = max_over_ranks(a.elapsed_time(end), dev)
         ok = ok and pipe.status_ok()
         e2e = {"value": job_throughput(st.gemm_ops(), world, args.steps, e_total),
                "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
                "ms_per_step": e_total / args.steps,
-               "pipeline": "two device buffer sets: step i+1's copy in and step i-1's copy back "
-                           "overlap step i",
+               "api": "shiftquant_layer_step_host (C ABI), one call per layer and step",
+               "pipeline": "two device buffer sets on two streams take the steps in turn: one "
+                           "step's copies overlap the other's compute",
                "l2": "not flushed: each step copies %.0f MB of inputs in from host memory "
                      "(L2 is 126 MB)" % (h2d / 1e6)}
         del pipe
@@ -458,8 +467,16 @@ def run_ours(args, rank, world, local_rank):
     kernel_name = ("shiftmm_kernel<%d, *> (one launch = forward + loss propagation + weight "
                    "gradient of a layer)" % (1 if fp8 else 0))
     tensor_src = f"{peak_src} bf16 burst" + (" x 2 (nominal FP8/BF16)" if fp8 else "")
+    sms = torch.cuda.get_device_properties(dev).multi_processor_count
+    clock_mhz = (clocks or {}).get("sm_mhz") or 0.0
+    clock_peak = (sms * BF16_OPS_PER_SM_CLOCK * (FP8_OVER_BF16 if fp8 else 1.0) * clock_mhz * 1e6
+                  / 1e12) if clock_mhz else None
     gemm_tensor = {"bound": "tensor", "achieved": gemm_tflops, "peak": tensor_peak,
                    "unit": "TFLOP/s", "frac": gemm_tflops / tensor_peak,
+                   "clock_peak": clock_peak,
+                   "frac_of_clock_peak": gemm_tflops / clock_peak if clock_peak else None,
+                   "clock_peak_source": "%d SMs x %d dense ops/clock x median sampled SM clock"
+                                        % (sms, BF16_OPS_PER_SM_CLOCK * (2 if fp8 else 1)),
                    "traffic": profiled_traffic(args.workload), "kernel": kernel_name,
                    "launch_time_source": gemm_src,
                    "peak_source": tensor_src}
@@ -536,6 +553,52 @@ def run_ours(args, rank, world, local_rank):
     return result, st
 
 
+def run_chain(args, dev, flush_steps=None):
+    """The range pass fused into the producer's epilogue, measured: vit_mlp's fc1 and fc2
+    trained as a chain (fc2's X = fc1's Y, fc1's dY = fc2's dX; nothing between the layers),
+    forward then backward, each variant captured as one CUDA graph and replayed after an L2
+    flush.  fused: the inner activation's and gradient's ranges come from the GEMM epilogues
+    (shiftquant_gemm_layer's y_range / dx_range); separate: the usual range passes."""
+    import torch
+    from paper_2411_10948_gb300 import layer as L
+    from paper_2411_10948_gb300 import workloads as W
+    wl = W.workload("vit_mlp")
+    s1, s2 = wl.layers
+    M, dims, bits, G = s1.M, (s1.K, s1.N, s2.N), s1.bits, s1.n_groups
+    x0, w1, _ = W.torch_layer_inputs(s1, args.seed, 0, dev)
+    _, w2, dy = W.torch_layer_inputs(s2, args.seed, 1, dev)
+    flush_w = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
+    flush_r = torch.zeros(L2_FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
+    sink = torch.zeros((), dtype=torch.float32, device=dev)
+    out = {}
+    steps = flush_steps or max(5, min(args.steps, 20))
+    for fused in (True, False):
+        ch = L.LinearChain(M, dims, bits, G, dev, fused_ranges=fused)
+        g = L.CapturedStep(lambda: ch.step(x0, [w1, w2], dy, 0x5EED))
+        for _ in range(3):
+            g.replay()
+        torch.cuda.synchronize()
+        ms = []
+        for _ in range(steps):
+            flush_w.zero_()
+            torch.sum(flush_r, dim=0, out=sink)
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record()
+            g.replay()
+            b.record()
+            b.synchronize()
+            ms.append(a.elapsed_time(b))
+        assert ch.status_ok(), "device status set in the chain"
+        out["fused_ms" if fused else "separate_ms"] = statistics.median(ms)
+        del g, ch
+    out.update({"workload": "vit_mlp fc1 -> fc2 as a chain (M=%d, %d -> %d -> %d, %d-bit), "
+                            "forward then backward, one graph per variant" % (M, *dims, bits),
+                "range_bytes_removed": 4 * M * dims[1] * 2,
+                "steps": steps, "statistic": "median of graph replays after an L2 flush"})
+    out["saved_frac"] = 1.0 - out["fused_ms"] / out["separate_ms"]
+    return out
+
+
 def oracle_sample_step(wl, rows_per_layer, seed):
     """One bounded oracle step: the quantizer chain and the three GEMMs on the first rows."""
     import oracle as O
@@ -577,10 +640,14 @@ def cpu_baseline(wl, seed, target_s=12.0):
     rows = choose_rows(wl, target_s, seed)
     run, ops = oracle_sample_step(wl, rows, seed)
     dt = run(0)
+    full_ops = sum(3 * 2 * s.M * s.N * s.K for s in wl.layers)
+    sampled = any(r < s.M for s, r in zip(wl.layers, rows))
     return {"value": ops / dt / 1e12, "unit": UNIT, "cores": O.max_threads(), "kind": "oracle",
             "sample": (f"first {rows} token rows of the {[s.M for s in wl.layers]} of each layer: "
                        "range+grouping+quantization of X, dY and W (both roles) and the three "
                        f"GEMMs over those rows, one step, {dt:.1f} s"),
+            "extrapolated": sampled,
+            "full_step_seconds_extrapolated": full_ops / (ops / dt) if sampled else dt,
             "seconds": dt}
 
 
@@ -629,16 +696,21 @@ def main():
     result, _ = run_ours(args, rank, world, local_rank)
     if rank == 0:
         if world == 1 and args.also not in ("", "none", args.workload):
-            # the large configuration the method's GEMM / quantizer targets are stated for
+            # a second workload (by default the 4-bit conv3x3 layer) summarised in the same line
             sub = argparse.Namespace(**vars(args))
             sub.workload, sub.no_e2e, sub.steps = args.also, True, max(3, min(args.steps, 10))
             other, _ = run_ours(sub, rank, world, local_rank)
             result["also"] = {k: other[k] for k in ("value", "unit", "ms_per_step", "dtype")}
             result["also"].update({"config": {"workload": args.also,
                                               "description": other["config"]["description"]},
-                                   "gemm": {k: other["gemm"][k] for k in ("achieved", "peak", "unit", "frac")},
+                                   "roofline": other["roofline"],
+                                   "gemm": {k: other["gemm"][k] for k in ("achieved", "peak", "unit", "frac",
+                                                                          "frac_of_clock_peak", "hbm_gbs",
+                                                                          "hbm_frac")},
                                    "quantizer": {k: other["quantizer"][k] for k in ("achieved", "peak", "unit", "frac")},
                                    "clocks": other["clocks"]})
+        if world == 1 and not args.no_chain:
+            result["fused_range_chain"] = run_chain(args, f"cuda:{local_rank}")
         if world == 1 and not args.no_cpu_baseline:
             from paper_2411_10948_gb300 import workloads as W
             result["cpu_baseline"] = cpu_baseline(W.workload(args.workload), args.seed)

@@ -145,12 +145,19 @@ sq_status shiftquant_quantize(const float *x, int64_t rows, int64_t cols, int64_
  *   Result: T[m, n] = sum_k q_X[m, k] q_W[k, n] 2^(G-1-e_k) exactly (int32, see the
  *     limits below), Y = float(T) * (s_X 2^-(G-1) * s_W[n]).
  *   acc_out [M, ld_acc] int64 (may be NULL): T itself, for exactness checks.
- *   workspace: optional int32 scratch of shiftquant_gemm_workspace_bytes() bytes; with
- *     it, a GEMM with too few output tiles splits K across SMs; NULL never splits.
+ *   workspace: optional scratch of shiftquant_gemm_workspace_bytes() bytes (16-byte
+ *     aligned); with it, a GEMM with too few output tiles splits K across SMs; NULL never
+ *     splits.
  *   Alignment: lda * code_bytes and ldb * code_bytes multiples of 16, code pointers
  *     16-byte aligned (the operands are read by TMA).
- *   Limits: max|q_X| max|q_W| 2^(G-1) K < 2^31 (the exact int32 range); larger K returns
- *     SQ_EUNSUPPORTED.  M, N or K == 0 is allowed. */
+ *   Exact range: T is exact for every K.  While max|q_X| max|q_W| 2^(G-1) K < 2^31 it is
+ *     summed in int32.  Beyond that (8 bits, N_G = 4: K > 16642) the K loop is split into
+ *     parts that each stay within int32 and the parts are added in int64 in the workspace,
+ *     which is then required (its size, M N 8 bytes rounded up, is what
+ *     shiftquant_gemm_workspace_bytes reports); without it the call returns
+ *     SQ_EUNSUPPORTED.  One K block (64 or 128 inner elements) of worst-case products must
+ *     stay within 2^24, the exact FP32 range of the tensor cores' sums (8 bits allows
+ *     N_G <= 5); otherwise SQ_EUNSUPPORTED.  M, N or K == 0 is allowed. */
 sq_status shiftquant_gemm_fwd(const void *a_codes, int64_t lda, const float *a_scale,
                               const void *b_codes, int64_t ldb, const float *b_scale,
                               int64_t M, int64_t N, int64_t K, int bits, int n_groups,
@@ -179,7 +186,8 @@ sq_status shiftquant_gemm_dgrad(const void *a_codes, int64_t lda, const float *a
  *   Both channel axes are outer dims here, so each group shift applies to the whole
  *   inner sum: T[i, j] = (sum_t q_X[t, i] q_dY[t, j]) 2^((G-1-eX_i) + (G-1-eY_j)) and
  *   dW = float(sum) * (s_X s_dY) 2^-(eX_i + eY_j).  acc_out receives T (int64).
- *   Limits: max|q_X| max|q_dY| T < 2^31. */
+ *   Exact range as for shiftquant_gemm_fwd with max|q_X| max|q_dY| T in place of the
+ *   forward bound (8 bits: int64 sums, with a workspace, beyond 133144 tokens). */
 sq_status shiftquant_gemm_wgrad(const void *xt_codes, int64_t ldx, const float *x_scale,
                                 const uint8_t *x_exp, const void *gt_codes, int64_t ldg,
                                 const float *g_scale, const uint8_t *g_exp, int64_t Ci,
@@ -254,6 +262,15 @@ typedef struct {
   /* At most this many CTAs (0: one per SM), for a launch that shares the GPU with work
    * running beside it on other streams. */
   int max_ctas;
+  /* Optional (NULL: not formed): the range pass of the next consumer of an output, formed in
+   * the GEMM's epilogue instead of a separate pass over the output (Sec. 3.1's channel
+   * ranges): y_range[N] = max_m |y[m, n]|, dx_range[K] = max_m |dx[m, k]|, equal bit for bit
+   * to shiftquant_calibrate(y or dx, SQ_GRAN_PER_COL).  The call zeroes them first.  When Y
+   * is the next layer's activation (or dX the previous layer's gradient), shiftquant_group
+   * on the range gives its tau_0 and exponents, and shiftquant_quantize follows without a
+   * range pass. */
+  float *y_range;
+  float *dx_range;
 } sq_layer_gemms;
 
 /* workspace: optional int32 scratch of shiftquant_gemm_layer_workspace_bytes() bytes,
@@ -285,6 +302,62 @@ int shiftquant_gemm_layer_kernel_launches(int64_t M, int64_t K, int64_t N, int b
 int shiftquant_gemm_layer_cta_pairs(int64_t M, int64_t K, int64_t N, int bits, int n_groups,
                                     int gemm_mask);
 
+/* One training step of one quantized linear layer X [M, K], W [K, N], dY [M, N], with the
+ * operand roles of the paper's setup (Sec. 5.1): every quantizer pass and the three GEMMs
+ * (Eq. 4 with the left-shift form of App. D), in stream order:
+ *   1. X:  range pass + grouping (Sec. 3.1, Eq. 3), codes and transposed codes, round to
+ *          nearest even (App. D);
+ *   2. dY: the same with stochastic rounding (App. B) drawn under `seed`;
+ *   3. W per out-channel (forward role): codes written transposed [N, K] with X's group
+ *      shifts folded in; W per in-channel (loss-propagation role): codes [K, N] with dY's
+ *      shifts folded in;
+ *   4. the forward, loss-propagation and weight-gradient GEMMs as one launch
+ *      (shiftquant_gemm_layer).
+ * Every buffer is a caller-owned DEVICE buffer; the layouts are those of the calls above:
+ *   x [M, K], w [K, N], dy [M, N], y [M, N], dx [M, K], dw [K, N]: fp32, dense row-major
+ *     (leading dimension = row length).  x, w and dy are written only by the host variant.
+ *   x_codes [M, ld_x], xt_codes [K, ld_xt], x_range[K], x_exp[K], x_tau0, x_scale (one
+ *     float each); g_codes [M, ld_g], gt_codes [N, ld_gt], g_range[N], g_exp[N], g_tau0,
+ *     g_scale; wf_codes [N, ld_wf], wf_range[N], wf_scale[N]; wd_codes [K, ld_wd],
+ *     wd_range[K], wd_scale[K].  Codes in the type of shiftquant_code_type(bits, n_groups),
+ *     rows 16-byte aligned (ld * code bytes a multiple of 16, pointers 16-byte aligned).
+ *   workspace: optional, as for shiftquant_gemm_layer (shiftquant_gemm_layer_workspace_bytes).
+ *   dev_status: the device status word (see the conventions above).
+ * The struct lives in host memory and is read during the call only.  The quantizer and GEMM
+ * launches run one after the other on `stream`; M, K or N == 0 does nothing. */
+typedef struct {
+  int64_t M, K, N;
+  int bits, n_groups;
+  float *x, *w, *dy;
+  void *x_codes;  int64_t ld_x;
+  void *xt_codes; int64_t ld_xt;
+  float *x_range, *x_tau0, *x_scale; uint8_t *x_exp;
+  void *g_codes;  int64_t ld_g;
+  void *gt_codes; int64_t ld_gt;
+  float *g_range, *g_tau0, *g_scale; uint8_t *g_exp;
+  void *wf_codes; int64_t ld_wf; float *wf_range, *wf_scale;
+  void *wd_codes; int64_t ld_wd; float *wd_range, *wd_scale;
+  float *y, *dx, *dw;
+  void *workspace; size_t workspace_bytes;
+  int32_t *dev_status;
+} sq_layer_step;
+
+sq_status shiftquant_layer_step(const sq_layer_step *args, uint64_t seed, void *stream);
+
+/* The same step fed from HOST memory and returned to it, all in the order of `stream`:
+ * copies x_host [M, K], w_host [K, N] and dy_host [M, N] (fp32, dense) into args->x, w, dy,
+ * runs shiftquant_layer_step, and copies y, dx, dw back into y_host [M, N], dx_host [M, K]
+ * and dw_host [K, N].  A NULL host pointer skips that copy (an input already on the device,
+ * an output left there).  The copies are cudaMemcpyAsync calls: with page-locked host memory
+ * (cudaHostAlloc / cudaHostRegister) they overlap work on other streams, so a caller that
+ * alternates two sets of device buffers on two streams overlaps one step's copies with the
+ * other's compute; with pageable memory they still give the right result but block the
+ * host.  The host outputs hold the results once the stream reaches the end of the call. */
+sq_status shiftquant_layer_step_host(const sq_layer_step *args, const float *x_host,
+                                     const float *w_host, const float *dy_host, float *y_host,
+                                     float *dx_host, float *dw_host, uint64_t seed,
+                                     void *stream);
+
 /* Weight-gradient GEMM for callers that cannot allocate device memory -- for instance a
  * plug-in running inside a host framework that owns every device allocation, or a
  * deployment whose device memory is fixed when the library is loaded.  The paper has no
@@ -293,7 +366,8 @@ int shiftquant_gemm_layer_cta_pairs(int64_t M, int64_t K, int64_t N, int bits, i
  *   Scratch: instead of a caller workspace, the split-K int32 partial sums live in a 4 MiB
  *     array inside the library (`static __device__`, held by every GPU that loads the
  *     library until the process exits).  Ci * Co must not exceed 1048576; larger outputs
- *     return SQ_EUNSUPPORTED before anything is launched.
+ *     return SQ_EUNSUPPORTED before anything is launched.  Past the int32 range (8 bits:
+ *     more than 133144 tokens) the sums are int64 and Ci * Co may not exceed 524288.
  *   Nothing is allocated: no cudaMalloc, no cudaFree, no allocating library routine.
  *   Each call made outside stream capture looks up the array's device address
  *     (cudaGetSymbolAddress) with the call's device current, so a device reset between
@@ -316,6 +390,20 @@ sq_status shiftquant_gemm_wgrad_static(const void *xt_codes, int64_t ldx, const 
  * 2 wgrad; M, N are the output dims and K the inner dim. */
 size_t shiftquant_gemm_workspace_bytes(int which, int64_t M, int64_t N, int64_t K,
                                        int bits, int n_groups);
+
+/* Failure-path self-test (for tests of the device-side timeout; the paper has no
+ * counterpart).  One GEMM launch with the operands and layout of shiftquant_gemm_fwd whose
+ * TMA producer arms every pipeline stage but issues no operand copy, so nothing is ever in
+ * flight and the tensor-core issuer's bounded wait on the first stage runs out after about
+ * 1 s.  The launch then records SQ_DEV_TIMEOUT in *dev_status, every role of every CTA
+ * leaves through the abort path (no copy or MMA outstanding, tensor memory freed) and the
+ * kernel returns; the CUDA context stays usable.  y is not written.  M, N and K must be in
+ * [1, 4096]; the checks and limits of shiftquant_gemm_fwd apply otherwise. */
+sq_status shiftquant_selftest_wait_timeout(const void *a_codes, int64_t lda, const float *a_scale,
+                                           const void *b_codes, int64_t ldb, const float *b_scale,
+                                           int64_t M, int64_t N, int64_t K, int bits,
+                                           int n_groups, float *y, int64_t ldy,
+                                           int32_t *dev_status, void *stream);
 
 /* Static description of a status code. */
 const char *shiftquant_status_string(sq_status status);

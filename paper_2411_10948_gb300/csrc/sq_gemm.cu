@@ -110,7 +110,11 @@ struct GemmParams {
   int64_t ldy;
   long long* acc;
   int64_t ld_acc;
-  int* ws;  // split-K int32 partial sums [M, N], or null
+  int* ws;  // split-K partial sums [M, N] (int32, or int64 when `wide`), or null
+  int wide;  // the K loop exceeds the exact int32 range: splits add int64 sums
+  // per-column max |output| (the next consumer's range pass, formed here), as the ordered
+  // bit patterns of non-negative floats, zeroed before the launch; or null
+  unsigned* colmax;
   int* status;
 };
 
@@ -134,6 +138,9 @@ struct GemmBatch {
   int planned;  // some GEMM sizes its chunks from exponents (warp 2 plans them)
   int* status;
   int lazy_from;  // with the counter: from this unit on, a pair takes one unit at a time
+  // failure-path self-test: the producer arms every stage but issues no copy, so the first
+  // consumer wait runs out (nothing is ever in flight) and the launch takes its abort path
+  int no_copies;
 };
 
 __device__ __forceinline__ float pow2_neg(int k) { return __int_as_float((127 - k) << 23); }
@@ -191,15 +198,18 @@ __device__ __noinline__ void write_acc_box(long long* acc, int64_t ld_acc, int64
 // only: the forward and loss-propagation outputs take the column factor alone).  The box is staged in shared
 // memory (128-byte swizzle) and leaves either as dequantized fp32 values through
 // row-contiguous 16-byte stores (eight lanes per 128-byte row, four rows per instruction),
-// or as int32 partial sums through a TMA reduce-add into the split-K workspace.  The
-// exactness-check integers are written when asked.
+// as int32 partial sums through a TMA reduce-add into the split-K workspace, or -- past the
+// int32 range -- as int64 additions (64-bit atomics, a row of 32 columns per instruction)
+// into the int64 workspace.  The exactness-check integers are written when asked.
 __device__ __forceinline__ void emit_box(const GemmParams& p, const CUtensorMap* tma_y,
                                          const CUtensorMap* tma_ws, const uint32_t (&vals)[32],
                                          bool as_float, uint32_t fac, float rfac, uint32_t buf,
                                          int64_t row0, int64_t col0, int lane) {
-  const bool tma_out = p.ws != nullptr || p.vec_y;
-  if (tma_out && lane == 0) {
-    bulk_wait_read<0>();  // the last TMA store has read the box
+  const bool tma_out = p.ws != nullptr ? !p.wide : p.vec_y != 0;
+  if (lane == 0) {
+    // the last TMA store has read the box (it may belong to another GEMM of the launch,
+    // whatever this box's own way out)
+    bulk_wait_read<0>();
   }
   __syncwarp();
   if (p.acc != nullptr && p.ws == nullptr) {
@@ -219,6 +229,11 @@ __device__ __forceinline__ void emit_box(const GemmParams& p, const CUtensorMap*
     __syncwarp();
   }
   const bool row_scaled = p.mode == 1;
+  // the column maxima of |output| over the box's 32 rows: one warp reduction per column
+  // (lanes are rows), lane j keeps column j's
+  const bool colmax = p.colmax != nullptr && p.ws == nullptr;
+  const bool row_in = row0 + lane < p.M;
+  uint32_t cmax = 0u;
 #pragma unroll
   for (int k = 0; k < 8; ++k) {
     uint32_t o[4];
@@ -234,8 +249,30 @@ __device__ __forceinline__ void emit_box(const GemmParams& p, const CUtensorMap*
         // x * 1 is x exactly, so skipping the row factor of 1 changes no result
         o[e] = __float_as_uint(__fmul_rn(row_scaled ? __fmul_rn(val, rfac) : val, f[e]));
       }
+      if (colmax) {
+        const uint32_t m = __reduce_max_sync(0xFFFFFFFFu, row_in ? (o[e] & 0x7FFFFFFFu) : 0u);
+        if (lane == k * 4 + e) cmax = m;
+      }
     }
     st_shared_v4(buf + lane * 128 + ((k ^ (lane & 7)) << 4), o[0], o[1], o[2], o[3]);
+  }
+  if (colmax && cmax != 0u && col0 + lane < p.N) atomicMax(p.colmax + col0 + lane, cmax);
+  if (p.ws != nullptr && p.wide) {
+    // a split of a K loop beyond the int32 range: its exact int32 sums are added into the
+    // int64 workspace, row by row (the lanes cover 32 consecutive columns of a row)
+    __syncwarp();
+    unsigned long long* w64 = reinterpret_cast<unsigned long long*>(p.ws);
+    const int64_t col = col0 + lane;
+    if (col < p.N) {
+      for (int rr = 0; rr < 32; ++rr) {
+        const int64_t row = row0 + rr;
+        if (row >= p.M) break;
+        const long long t = static_cast<int32_t>(staged(buf, rr, lane));
+        atomicAdd(w64 + row * p.N + col, static_cast<unsigned long long>(t));
+      }
+    }
+    __syncwarp();  // the staging box is free for the next one
+    return;
   }
   if (tma_out) {
     fence_proxy_async_smem();
@@ -650,14 +687,16 @@ __global__ void __launch_bounds__(kThreads, 1) shiftmm_kernel(const __grid_const
         }
         const uint32_t sa = smem_u32(smem + s * L::stage_bytes);
         if (rank == 0) mbar_arrive_expect_tx(&full[s], kCg * L::stage_bytes);
-        if constexpr (kPair) {
-          tma_load_2d_pair(sa, &bt.a[g], full_c + s * 8, kb * kBKElems, ya);
-          tma_load_2d_pair(sa + kABytes, &bt.b[g], full_c + s * 8, kb * kBKElems, yb);
-        } else {
-          tma_load_2d(sa, &bt.a[g], smem_u32(&full[s]), kb * kBKElems, ya);
-          tma_load_2d(sa + kABytes, &bt.b[g], smem_u32(&full[s]), kb * kBKElems, yb);
+        if (!bt.no_copies) {
+          if constexpr (kPair) {
+            tma_load_2d_pair(sa, &bt.a[g], full_c + s * 8, kb * kBKElems, ya);
+            tma_load_2d_pair(sa + kABytes, &bt.b[g], full_c + s * 8, kb * kBKElems, yb);
+          } else {
+            tma_load_2d(sa, &bt.a[g], smem_u32(&full[s]), kb * kBKElems, ya);
+            tma_load_2d(sa + kABytes, &bt.b[g], smem_u32(&full[s]), kb * kBKElems, yb);
+          }
+          ++issued;
         }
-        ++issued;
         if (++s == kStages) {
           s = 0;
           ph ^= 1u;
@@ -938,6 +977,13 @@ __global__ void __launch_bounds__(256) splitk_finalize_kernel(const GemmParams p
     long long t[4];
 #pragma unroll
     for (int e = 0; e < 4; ++e) epilogue_value(p, row, col + e, tv[e], a_fac, &o[e], &t[e]);
+    if (p.colmax) {
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const uint32_t b = __float_as_uint(o[e]) & 0x7FFFFFFFu;
+        if (b != 0u) atomicMax(p.colmax + col + e, b);
+      }
+    }
     float* dst = p.y + row * p.ldy + col;
     if (p.vec_y) {
       *reinterpret_cast<float4*>(dst) = make_float4(o[0], o[1], o[2], o[3]);
@@ -949,6 +995,36 @@ __global__ void __launch_bounds__(256) splitk_finalize_kernel(const GemmParams p
 #pragma unroll
       for (int e = 0; e < 4; ++e) p.acc[row * p.ld_acc + col + e] = t[e];
     }
+  }
+}
+
+// The same from int64 sums (a K loop beyond the int32 range), one output per thread: the one
+// dequantizing multiply of the epilogue with T converted to FP32 once (round to nearest).
+__global__ void __launch_bounds__(256) splitk_finalize_wide_kernel(const GemmParams p) {
+  const float a_fac = epilogue_a_factor(p);
+  const long long* ws = reinterpret_cast<const long long*>(p.ws);
+  const int64_t n = static_cast<int64_t>(p.M) * p.N;
+  for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < n;
+       i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+    const int64_t row = i / p.N;
+    const int64_t col = i - row * p.N;
+    const long long t = __ldcs(ws + i);
+    float y;
+    long long tc;
+    if (p.mode == 0) {
+      y = __fmul_rn(__ll2float_rn(t), __fmul_rn(a_fac, __ldg(p.b_scale + col)));
+      tc = t;
+    } else {
+      const int er = __ldg(p.row_exp + row), ec = __ldg(p.col_exp + col);
+      y = __fmul_rn(__fmul_rn(__ll2float_rn(t), pow2_neg(er + ec)), a_fac);
+      tc = t << (2 * (p.G - 1) - er - ec);
+    }
+    p.y[row * p.ldy + col] = y;
+    if (p.colmax) {
+      const uint32_t b = __float_as_uint(y) & 0x7FFFFFFFu;
+      if (b != 0u) atomicMax(p.colmax + col, b);
+    }
+    if (p.acc) p.acc[row * p.ld_acc + col] = tc;
   }
 }
 
@@ -1016,6 +1092,7 @@ static int device_sms(int* dev_out) {
 struct Plan {
   int m_tiles, n_tiles, kb_total, chunk_kb, splits, kb_per_split;
   int elem_bytes;
+  int wide;  // max|T| can pass 2^31: every split stays within int32, splits add in int64
 };
 
 // max |product| of one inner index: q_A q_B 2^(G-1) with the shift folded into B
@@ -1025,20 +1102,30 @@ static int64_t max_product(int which, int bits, int G) {
   return (which == 2) ? Q * Q : (Q * Q) << (G - 1);
 }
 
-// the exactness limits, checked before anything touches the device
+// The exactness limit of the FP32 accumulation, checked before anything touches the device:
+// one K block of worst-case products must stay within 2^24 (the chunks are whole K blocks).
+// K itself is not limited: past the int32 range the K loop is split (see make_plan).
 static int check_exact_range(int which, int64_t K, int bits, int G) {
+  (void)K;
   const int64_t P = max_product(which, bits, G);
-  if (P * K > INT32_MAX)
-    return fail(SQ_EUNSUPPORTED,
-                "inner dimension %lld exceeds the exact int32 range for bits=%d, n_groups=%d "
-                "(max |T| = %lld * K)",
-                static_cast<long long>(K), bits, G, static_cast<long long>(P));
   const int bk = kBKBytes / code_bytes(code_type(bits, G));
   if (kExactSum / P < bk)
     return fail(SQ_EUNSUPPORTED,
                 "bits=%d with n_groups=%d: one %d-wide K block can exceed the exact FP32 sum range",
                 bits, G, bk);
   return SQ_OK;
+}
+
+// The int32 limit of a sum that is added across ranks as int32 (the sharded weight
+// gradient): max|T| = max|product| K must stay below 2^31.
+static int check_int32_range(int which, int64_t K, int bits, int G) {
+  const int64_t P = max_product(which, bits, G);
+  if (P * K > INT32_MAX)
+    return fail(SQ_EUNSUPPORTED,
+                "inner dimension %lld exceeds the exact int32 range for bits=%d, n_groups=%d "
+                "(max |T| = %lld * K)",
+                static_cast<long long>(K), bits, G, static_cast<long long>(P));
+  return check_exact_range(which, K, bits, G);
 }
 
 // Tiles of 128 (pair: 256) x 256 outputs spread over `workers` (SMs, or CTA pairs).
@@ -1064,15 +1151,24 @@ static int make_plan(int which, int64_t M, int64_t N, int64_t K, int bits, int G
     if (max_splits > 1 && splits > max_splits) splits = max_splits;
     if (splits < 1) splits = 1;
   }
+  // Past the int32 range every split keeps its K loop within it (its int32 register sums
+  // stay exact) and the splits add in int64: at least this many, whatever max_splits says.
+  const int64_t kb_int32 = (INT32_MAX / P) / bk;  // >= 1: one K block stays within 2^24
+  pl->wide = pl->kb_total > kb_int32 ? 1 : 0;
+  if (pl->wide) {
+    const int need = static_cast<int>((pl->kb_total + kb_int32 - 1) / kb_int32);
+    if (splits < need) splits = need;
+  }
   pl->kb_per_split = (pl->kb_total + splits - 1) / splits;
   pl->splits = (pl->kb_total + pl->kb_per_split - 1) / pl->kb_per_split;
   return SQ_OK;
 }
 
-// Split-K workspace of one GEMM: the int32 partial sums [M, N], zeroed before every launch
-// that uses them, rounded up to 256 bytes.
-static size_t split_ws_bytes(int64_t M, int64_t N) {
-  return (static_cast<size_t>(M) * static_cast<size_t>(N) * sizeof(int) + 255) & ~size_t(255);
+// Split-K workspace of one GEMM: the partial sums [M, N] (int32, or int64 past the int32
+// range), zeroed before every launch that uses them, rounded up to 256 bytes.
+static size_t split_ws_bytes(int64_t M, int64_t N, bool wide = false) {
+  const size_t eb = wide ? sizeof(long long) : sizeof(int);
+  return (static_cast<size_t>(M) * static_cast<size_t>(N) * eb + 255) & ~size_t(255);
 }
 // The layer launch's workspace starts with the unit counter of its dynamic schedule.
 constexpr size_t kSchedBytes = 256;
@@ -1143,6 +1239,7 @@ struct GemmJob {
   size_t ws_bytes;
   const uint8_t* k_exp;  // exponents of the inner channels (forward, loss propagation), or null
   int partial;  // weight gradient: int32 sums into ws (the caller's), no dequantizing pass
+  float* colmax;  // per-column max |output| [N], formed by the epilogue, or null
 };
 
 static const char* job_name(int which) {
@@ -1202,6 +1299,17 @@ static int plan_job(const GemmJob& j, int bits, int G, int workers, int max_spli
                     Plan* pl) {
   const int st = make_plan(j.which, j.M, j.N, j.K, bits, G, workers, max_splits, pair, pl);
   if (st != SQ_OK || pl->splits <= 1 || j.partial) return st;  // partial: ws is the output
+  if (pl->wide) {
+    // int64 sums need their workspace; there is no unsplit way to stay exact
+    if (j.ws == nullptr || j.ws_bytes < split_ws_bytes(j.M, j.N, true) || !aligned16(j.ws))
+      return fail(SQ_EUNSUPPORTED,
+                  "%s: inner dimension %lld exceeds the exact int32 range for bits=%d, "
+                  "n_groups=%d; int64 accumulation needs a 16-byte aligned workspace of %zu bytes "
+                  "(shiftquant_gemm_workspace_bytes)",
+                  job_name(j.which), static_cast<long long>(j.K), bits, G,
+                  split_ws_bytes(j.M, j.N, true));
+    return SQ_OK;
+  }
   if (j.ws == nullptr || j.ws_bytes < split_ws_bytes(j.M, j.N) || !aligned16(j.ws) || j.N % 4 != 0)
     return make_plan(j.which, j.M, j.N, j.K, bits, G, workers, 1, pair, pl);
   return SQ_OK;
@@ -1292,10 +1400,12 @@ static int prepare_job(const GemmJob& j, const Plan* pl, int bits, int G, int32_
   p.acc = reinterpret_cast<long long*>(j.acc);
   p.ld_acc = j.ld_acc;
   p.ws = (pl->splits > 1 || j.partial) ? static_cast<int*>(j.ws) : nullptr;
+  p.wide = pl->wide;
+  p.colmax = reinterpret_cast<unsigned*>(j.colmax);
   p.status = dev_status;
   memset(&bt->y[g], 0, sizeof(CUtensorMap));
   memset(&bt->ws[g], 0, sizeof(CUtensorMap));
-  if (p.ws)
+  if (p.ws && !p.wide)
     st = make_output_map(&bt->ws[g], p.ws, j.M, j.N, j.N, CU_TENSOR_MAP_DATA_TYPE_INT32);
   else if (p.vec_y)
     st = make_output_map(&bt->y[g], j.y, j.M, j.N, j.ldy, CU_TENSOR_MAP_DATA_TYPE_FLOAT32);
@@ -1345,15 +1455,24 @@ static int launch_variant(const GemmBatch& bt, int grid, int dev, cudaStream_t s
 // CTAs take their units as they free up -- for batches whose units differ in length.
 // Without one each CTA strides over the unit list.
 static int run_jobs(GemmJob* jobs, int njobs, int bits, int G, int32_t* dev_status, void* stream,
-                    int* sched, int max_ctas = 0) {
+                    int* sched, int max_ctas = 0, bool no_copies = false) {
   cudaStream_t s = as_stream(stream);
   int live[kMaxBatch];
   int nlive = 0;
+  for (int i = 0; i < njobs; ++i)
+    if (jobs[i].colmax != nullptr && (reinterpret_cast<uintptr_t>(jobs[i].colmax) & 3u) != 0)
+      return fail(SQ_EALIGN, "%s: column-range output must be 4-byte aligned", job_name(jobs[i].which));
   for (int i = 0; i < njobs; ++i) {
     bool launch = false;
     const int st = check_job(jobs[i], bits, G, dev_status, s, &launch);
     if (st != SQ_OK) return st;
     if (launch) live[nlive++] = i;
+  }
+  // column ranges start at 0 (an output with no rows, or K == 0, keeps them there)
+  for (int i = 0; i < njobs; ++i) {
+    if (jobs[i].colmax == nullptr || jobs[i].N <= 0) continue;
+    const cudaError_t err = cudaMemsetAsync(jobs[i].colmax, 0, static_cast<size_t>(jobs[i].N) * sizeof(float), s);
+    if (err != cudaSuccess) return cuda_fail(err, "cudaMemsetAsync");
   }
   if (nlive == 0) return SQ_OK;
   int dev = 0;
@@ -1401,6 +1520,7 @@ static int run_jobs(GemmJob* jobs, int njobs, int bits, int G, int32_t* dev_stat
   bt.count = nlive;
   bt.status = dev_status;
   bt.sched = sched;
+  bt.no_copies = no_copies ? 1 : 0;
   bt.planned = 0;
   for (int g = 0; g < nlive; ++g) bt.planned |= bt.k_exp[g] != nullptr;
   // zero the counter and the partial sums, with one memset for the regions that follow the
@@ -1413,7 +1533,7 @@ static int run_jobs(GemmJob* jobs, int njobs, int bits, int G, int32_t* dev_stat
     char* w = reinterpret_cast<char*>(bt.p[g].ws);
     // a partial call's sums go to the caller's buffer of exactly M N words
     const size_t b = partial ? static_cast<size_t>(bt.p[g].M) * bt.p[g].N * sizeof(int)
-                             : split_ws_bytes(bt.p[g].M, bt.p[g].N);
+                             : split_ws_bytes(bt.p[g].M, bt.p[g].N, bt.p[g].wide != 0);
     if (zero_end != nullptr && w == zero_end) {
       zero_end = w + b;
       continue;
@@ -1445,10 +1565,13 @@ static int run_jobs(GemmJob* jobs, int njobs, int bits, int G, int32_t* dev_stat
   if (st != SQ_OK) return st;
   for (int g = 0; g < nlive; ++g) {
     if (!bt.p[g].ws || partial) continue;
-    const int64_t quads = static_cast<int64_t>(bt.p[g].M) * (bt.p[g].N / 4);
-    int64_t blocks = (quads + 255) / 256;
+    const int64_t items = static_cast<int64_t>(bt.p[g].M) * (bt.p[g].wide ? bt.p[g].N : bt.p[g].N / 4);
+    int64_t blocks = (items + 255) / 256;
     if (blocks > static_cast<int64_t>(sms) * 16) blocks = static_cast<int64_t>(sms) * 16;
-    splitk_finalize_kernel<<<static_cast<unsigned>(blocks), 256, 0, s>>>(bt.p[g]);
+    if (bt.p[g].wide)
+      splitk_finalize_wide_kernel<<<static_cast<unsigned>(blocks), 256, 0, s>>>(bt.p[g]);
+    else
+      splitk_finalize_kernel<<<static_cast<unsigned>(blocks), 256, 0, s>>>(bt.p[g]);
     err = cudaGetLastError();
     if (err != cudaSuccess) return cuda_fail(err, "splitk_finalize_kernel launch");
   }
@@ -1476,6 +1599,8 @@ static void layer_jobs(const sq_layer_gemms* a, GemmJob jobs[3], int mask) {
                     nullptr, 0};
   jobs[0].k_exp = a->x_exp;  // the forward GEMM's inner channels are X's
   jobs[1].k_exp = a->g_exp;  // loss propagation's are dY's
+  jobs[0].colmax = a->y_range;
+  jobs[1].colmax = a->dx_range;
   // a GEMM left out of the mask becomes empty: nothing of it is checked or launched
   for (int i = 0; i < 3; ++i)
     if (mask != 0 && !(mask & (1 << i))) jobs[i].M = 0;
@@ -1490,11 +1615,12 @@ static void layer_ws_need(const GemmJob jobs[3], int bits, int G, int sms, int p
   for (int i = 0; i < 3; ++i) {
     need[i] = 0;
     const GemmJob& j = jobs[i];
-    if (j.M <= 0 || j.N <= 0 || j.K <= 0 || j.N % 4 != 0) continue;
+    if (j.M <= 0 || j.N <= 0 || j.K <= 0) continue;
     Plan pl;
     if (make_plan(j.which, j.M, j.N, j.K, bits, G, pair ? pairs : sms, 0, pair, &pl) != SQ_OK)
       continue;
-    if (pl.splits > 1) need[i] = split_ws_bytes(j.M, j.N);
+    if (!pl.wide && j.N % 4 != 0) continue;  // int32 splits are added by 16-byte TMA rows
+    if (pl.splits > 1) need[i] = split_ws_bytes(j.M, j.N, pl.wide != 0);
   }
 }
 
@@ -1614,7 +1740,8 @@ extern "C" size_t shiftquant_gemm_workspace_bytes(int which, int64_t M, int64_t 
   const bool pair = pair_mode(&jp, 1, bits, n_groups, sms, pairs);
   Plan pl;
   if (make_plan(which, M, N, K, bits, n_groups, pair ? pairs : sms, 0, pair, &pl) != SQ_OK) return 0;
-  return pl.splits > 1 ? split_ws_bytes(M, N) : 0;
+  if (!pl.wide && N % 4 != 0) return 0;
+  return pl.splits > 1 ? split_ws_bytes(M, N, pl.wide != 0) : 0;
 }
 
 extern "C" sq_status shiftquant_gemm_wgrad_partial(
@@ -1631,7 +1758,7 @@ extern "C" sq_status shiftquant_gemm_wgrad_partial(
   if (t_out == nullptr || !aligned16(t_out) || Co % 4 != 0)
     return fail(SQ_EALIGN, "gemm_wgrad_partial: t_out must be 16-byte aligned and Co a multiple of 4");
   // the summed partials must stay in the exact int32 range for the whole token count
-  int st = check_exact_range(2, total_tokens, bits, n_groups);
+  int st = check_int32_range(2, total_tokens, bits, n_groups);
   if (st != SQ_OK) return st;
   GemmJob j{2, xt_codes, ldx, gt_codes, ldg, Ci, Co, T, x_scale, g_scale, x_exp, g_exp,
             nullptr, 0, nullptr, 0, t_out, static_cast<size_t>(Ci) * Co * sizeof(int32_t)};
@@ -1725,6 +1852,22 @@ extern "C" sq_status shiftquant_gemm_layer(const sq_layer_gemms* args, void* wor
   int* sched =
       assign_layer_ws(jobs, args->bits, args->n_groups, sms, pairs, workspace, workspace_bytes);
   return run_jobs(jobs, 3, args->bits, args->n_groups, dev_status, stream, sched, args->max_ctas);
+}
+
+extern "C" sq_status shiftquant_selftest_wait_timeout(const void* a_codes, int64_t lda,
+                                                      const float* a_scale, const void* b_codes,
+                                                      int64_t ldb, const float* b_scale, int64_t M,
+                                                      int64_t N, int64_t K, int bits, int n_groups,
+                                                      float* y, int64_t ldy, int32_t* dev_status,
+                                                      void* stream) {
+  fail(SQ_OK, "");
+  if (M <= 0 || N <= 0 || K <= 0)
+    return fail(SQ_EINVAL, "selftest_wait_timeout: the launch needs a non-empty GEMM");
+  if (M > 4096 || N > 4096 || K > 4096)
+    return fail(SQ_EINVAL, "selftest_wait_timeout: M, N and K must be at most 4096");
+  GemmJob j{0, a_codes, lda, b_codes, ldb, M, N, K, a_scale, b_scale, nullptr, nullptr,
+            y, ldy, nullptr, 0, nullptr, 0};
+  return run_jobs(&j, 1, bits, n_groups, dev_status, stream, nullptr, 0, true);
 }
 
 extern "C" size_t shiftquant_gemm_layer_workspace_bytes(int64_t M, int64_t K, int64_t N, int bits,

@@ -100,9 +100,15 @@ class QuantLinear:
     """Buffers and calls of one quantized linear layer: X [M, K], W [K, N], dY [M, N]."""
 
     def __init__(self, M, K, N_, bits, n_groups, device="cuda", with_acc=False,
-                 use_workspace=True):
+                 use_workspace=True, with_inputs=False):
         self.M, self.K, self.N, self.bits, self.G = M, K, N_, bits, n_groups
         dev = torch.device(device)
+        # device input buffers for shiftquant_layer_step(_host), when asked for
+        self.inputs = None
+        if with_inputs:
+            self.inputs = (torch.zeros((M, K), dtype=torch.float32, device=dev),
+                           torch.zeros((K, N_), dtype=torch.float32, device=dev),
+                           torch.zeros((M, N_), dtype=torch.float32, device=dev))
         self.status = torch.zeros(1, dtype=torch.int32, device=dev)
         self.x = ShiftTensor.alloc(M, K, bits, n_groups, dev)
         self.g = ShiftTensor.alloc(M, N_, bits, n_groups, dev)
@@ -168,7 +174,8 @@ class QuantLinear:
                                 self.G, self.dw, self.acc["wgrad"] if self.acc else None,
                                 self.ws_wgrad, self.status, stream)
 
-    def gemms(self, stream=None, gemm_mask=0, max_ctas=0, use_workspace=True):
+    def gemms(self, stream=None, gemm_mask=0, max_ctas=0, use_workspace=True, y_range=None,
+              dx_range=None):
         """The three GEMMs in one persistent launch (shiftquant_gemm_layer); gemm_mask picks
         a subset (bit 0 forward, 1 loss propagation, 2 weight gradient), max_ctas caps the
         CTAs.  A launch running beside another on a different stream must not share its
@@ -180,7 +187,8 @@ class QuantLinear:
                                 self.M, self.K, self.N, self.bits, self.G, self.y, self.dx,
                                 self.dw, acc.get("fwd"), acc.get("dgrad"), acc.get("wgrad"),
                                 self.ws_layer if use_workspace else None, self.status, stream,
-                                gemm_mask=gemm_mask, max_ctas=max_ctas)
+                                gemm_mask=gemm_mask, max_ctas=max_ctas, y_range=y_range,
+                                dx_range=dx_range)
 
     def step(self, x, w, dy, seed, stream=None):
         """One training step of the layer: every quantizer pass and all three GEMMs."""
@@ -249,9 +257,84 @@ class QuantLinear:
         if gemm_events is not None:
             gemm_events[1].record(main)
 
+    def step_args(self, x=None, w=None, dy=None):
+        """The C struct sq_layer_step over this layer's buffers, with x, w, dy (dense device
+        tensors) as the inputs, or the layer's own input buffers (with_inputs=True)."""
+        if x is None:
+            assert self.inputs is not None, "QuantLinear(with_inputs=True) or explicit inputs"
+            x, w, dy = self.inputs
+        return N.layer_step_args(
+            self.M, self.K, self.N, self.bits, self.G, x, w, dy, self.x.codes, self.x.codes_t,
+            self.x.range, self.x.tau0, self.x.scale, self.x.exp, self.g.codes, self.g.codes_t,
+            self.g.range, self.g.tau0, self.g.scale, self.g.exp, self.wf.codes, self.wf.range,
+            self.wf.scale, self.wd.codes, self.wd.range, self.wd.scale, self.y, self.dx, self.dw,
+            self.ws_layer, self.status)
+
     @property
     def gemm_ops(self) -> int:
         return 3 * 2 * self.M * self.N * self.K
+
+
+class LinearChain:
+    """Quantized linear layers applied one after another, X_{l+1} = Y_l (nothing between the
+    layers), trained by a forward pass over the layers and a backward pass in reverse with
+    dY_l = dX_{l+1}.  dims = (d_0, d_1, ..., d_L): layer l maps d_l to d_{l+1} over M tokens.
+
+    fused_ranges=True: the range pass of every inner activation Y_l and inner gradient dX_l
+    is formed in the epilogue of the GEMM that writes it (the y_range / dx_range outputs of
+    shiftquant_gemm_layer), and its consumer groups from that vector (shiftquant_group) and
+    quantizes: no pass over the tensor before its quantization.  fused_ranges=False runs the
+    usual range pass (shiftquant_calibrate) instead.  Both give the same bits."""
+
+    def __init__(self, M, dims, bits, n_groups, device="cuda", fused_ranges=True):
+        dev = torch.device(device)
+        self.M, self.dims, self.bits, self.G = M, list(dims), bits, n_groups
+        self.fused = fused_ranges
+        self.layers = [QuantLinear(M, dims[i], dims[i + 1], bits, n_groups, dev)
+                       for i in range(len(dims) - 1)]
+        self.y_range = [torch.zeros(d, dtype=torch.float32, device=dev) for d in dims[1:]]
+        self.dx_range = [torch.zeros(d, dtype=torch.float32, device=dev) for d in dims[:-1]]
+
+    def _quantize_input(self, t, q, range_vec, mode, seed, status, stream):
+        if range_vec is not None:
+            N.shiftquant_group(range_vec, self.G, q.tau0, q.exp, status, stream)
+        else:
+            N.shiftquant_calibrate(t, N.SQ_GRAN_SHIFT, self.G, q.range, q.tau0, q.exp, status,
+                                   stream)
+        N.shiftquant_quantize(t, N.SQ_GRAN_SHIFT, self.bits, self.G, q.tau0, q.exp, None, mode,
+                              seed, q.codes, q.codes_t, q.scale, stream)
+
+    def step(self, x0, weights, dy_last, seed, stream=None):
+        """One training step: forward through every layer from x0 [M, d_0], then backward
+        from dy_last [M, d_L]; weights[l] is W_l [d_l, d_{l+1}].  Layer l's gradient rounds
+        stochastically under seed + l."""
+        Lz = self.layers
+        last = len(Lz) - 1
+        for l, lay in enumerate(Lz):
+            x = x0 if l == 0 else Lz[l - 1].y
+            rng = self.y_range[l - 1] if (self.fused and l > 0) else None
+            self._quantize_input(x, lay.x, rng, N.SQ_ROUND_NEAREST_EVEN, 0, lay.status, stream)
+            weight_quantize_fwd(weights[l], lay.wf, lay.x.exp, self.bits, self.G, lay.status,
+                                stream)
+            lay.gemms(stream, gemm_mask=1,
+                      y_range=self.y_range[l] if (self.fused and l < last) else None)
+        for l in range(last, -1, -1):
+            lay = Lz[l]
+            dy = dy_last if l == last else Lz[l + 1].dx
+            rng = self.dx_range[l + 1] if (self.fused and l < last) else None
+            self._quantize_input(dy, lay.g, rng, N.SQ_ROUND_STOCHASTIC, seed + l, lay.status,
+                                 stream)
+            weight_quantize_dgrad(weights[l], lay.wd, lay.g.exp, self.bits, self.G, lay.status,
+                                  stream)
+            lay.gemms(stream, gemm_mask=6,
+                      dx_range=self.dx_range[l] if (self.fused and l > 0) else None)
+
+    def status_ok(self) -> bool:
+        return all(int(l.status.item()) == 0 for l in self.layers)
+
+    @property
+    def gemm_ops(self) -> int:
+        return sum(l.gemm_ops for l in self.layers)
 
 
 class CapturedStep:
@@ -276,71 +359,43 @@ class CapturedStep:
         self.graph.replay()
 
 
-class HostPipeline:
-    """Training steps fed from pinned host memory and returned to it.  Each step copies
-    the inputs X, W and dY of every layer to the device, runs every layer's step
-    (`QuantLinear.step_concurrent`, replayed as one CUDA graph), and copies Y, dX and dW
-    back.  Two sets of device buffers alternate between steps.  Step i+1's inputs copy in
-    on one stream and step i-1's outputs copy out on another while step i computes, so the
-    host link's two directions, not the GPU, set the pace.
+class HostSteps:
+    """Training steps fed from host memory and returned to it through the C entry point
+    shiftquant_layer_step_host: for every layer of a step, one call copies X, W and dY in,
+    runs the layer's whole step and copies Y, dX and dW back, all inside the library and in
+    the order of one stream.  Two sets of device buffers, each with its own stream, take
+    the steps in turn, so one step's copies overlap the other's compute and the host
+    link's two directions, not the GPU, set the pace.
 
-    shapes: (M, K, N) per layer.  The stochastic-rounding seed of a slot is fixed when its
-    graph is captured (slot s uses seed + s)."""
+    shapes: (M, K, N) per layer."""
 
-    def __init__(self, shapes, bits, n_groups, device="cuda", seed=0x5EED):
+    def __init__(self, shapes, bits, n_groups, device="cuda", slots=2):
         dev = torch.device(device)
         self.shapes = list(shapes)
-        self.s_in = torch.cuda.Stream(device=dev)
-        self.s_comp = torch.cuda.Stream(device=dev)
-        self.s_out = torch.cuda.Stream(device=dev)
         self.slots = []
-        for k in range(2):
-            layers = [QuantLinear(M, K, N_, bits, n_groups, dev) for (M, K, N_) in self.shapes]
-            inputs = [(torch.zeros((M, K), dtype=torch.float32, device=dev),
-                       torch.zeros((K, N_), dtype=torch.float32, device=dev),
-                       torch.zeros((M, N_), dtype=torch.float32, device=dev))
+        for _ in range(slots):
+            layers = [QuantLinear(M, K, N_, bits, n_groups, dev, with_inputs=True)
                       for (M, K, N_) in self.shapes]
-            streams = [[torch.cuda.Stream(device=dev) for _ in range(4)] for _ in layers]
+            self.slots.append({"layers": layers, "args": [l.step_args() for l in layers],
+                               "stream": torch.cuda.Stream(device=dev)})
 
-            def step(layers=layers, inputs=inputs, streams=streams, sd=seed + k):
-                for lay, (x, w, dy), ss in zip(layers, inputs, streams):
-                    lay.step_concurrent(x, w, dy, sd, ss)
-
-            self.slots.append({"layers": layers, "inputs": inputs, "graph": CapturedStep(step),
-                               "in_ready": torch.cuda.Event(), "done": torch.cuda.Event(),
-                               "out_copied": torch.cuda.Event()})
-
-    def run(self, host_inputs, host_outputs) -> torch.cuda.Event:
-        """Queue one step per entry.  host_inputs[i]: (x, w, dy) per layer, pinned float32
-        host tensors; host_outputs[i]: (y, dx, dw) per layer, pinned float32 host tensors
-        that receive step i's results.  Returns an event recorded after the last copy back
-        (synchronize on it before reading the host outputs)."""
+    def run(self, host_inputs, host_outputs, seed=0x5EED) -> torch.cuda.Event:
+        """Queue one step per entry: host_inputs[i] = (x, w, dy) per layer, host_outputs[i] =
+        (y, dx, dw) per layer, page-locked float32 host tensors (an entry may be None to
+        skip that copy).  Step i draws its stochastic rounding under seed + i.  Returns an
+        event on the current stream after the last copy back (synchronize on it before
+        reading the host outputs)."""
         cur = torch.cuda.current_stream()
-        for s in (self.s_in, self.s_comp, self.s_out):
-            s.wait_stream(cur)
+        for sl in self.slots:
+            sl["stream"].wait_stream(cur)
         for i, (hin, hout) in enumerate(zip(host_inputs, host_outputs)):
-            sl = self.slots[i % 2]
-            self.s_in.wait_event(sl["done"])        # the slot's last step no longer reads them
-            with torch.cuda.stream(self.s_in):
-                for dev_in, host_in in zip(sl["inputs"], hin):
-                    for d, h in zip(dev_in, host_in):
-                        d.copy_(h, non_blocking=True)
-                sl["in_ready"].record(self.s_in)
-            self.s_comp.wait_event(sl["in_ready"])
-            self.s_comp.wait_event(sl["out_copied"])  # the slot's last outputs have left
-            with torch.cuda.stream(self.s_comp):
-                sl["graph"].replay()
-                sl["done"].record(self.s_comp)
-            self.s_out.wait_event(sl["done"])
-            with torch.cuda.stream(self.s_out):
-                for lay, host_out in zip(sl["layers"], hout):
-                    for h, d in zip(host_out, (lay.y, lay.dx, lay.dw)):
-                        h.copy_(d, non_blocking=True)
-                sl["out_copied"].record(self.s_out)
+            sl = self.slots[i % len(self.slots)]
+            for args, (x, w, dy), (y, dx, dw) in zip(sl["args"], hin, hout):
+                N.shiftquant_layer_step_host(args, x, w, dy, y, dx, dw, seed + i, sl["stream"])
+        for sl in self.slots:
+            cur.wait_stream(sl["stream"])
         end = torch.cuda.Event(enable_timing=True)
-        end.record(self.s_out)
-        for s in (self.s_in, self.s_comp, self.s_out):
-            cur.wait_stream(s)
+        end.record(cur)
         return end
 
     def status_ok(self) -> bool:

@@ -37,6 +37,7 @@ EXPORTS = (
     "shiftquant_gemm_wgrad_static", "shiftquant_gemm_workspace_bytes",
     "shiftquant_gemm_layer", "shiftquant_gemm_layer_workspace_bytes",
     "shiftquant_gemm_layer_kernel_launches", "shiftquant_gemm_layer_cta_pairs",
+    "shiftquant_layer_step", "shiftquant_layer_step_host", "shiftquant_selftest_wait_timeout",
     "shiftquant_status_string", "shiftquant_last_error",
 )
 
@@ -63,6 +64,31 @@ class SqLayerGemms(ctypes.Structure):
         ("acc_dx", ctypes.c_void_p), ("ld_acc_dx", ctypes.c_int64),
         ("acc_dw", ctypes.c_void_p), ("ld_acc_dw", ctypes.c_int64),
         ("gemm_mask", ctypes.c_int), ("max_ctas", ctypes.c_int),
+        ("y_range", ctypes.c_void_p), ("dx_range", ctypes.c_void_p),
+    ]
+
+
+class SqLayerStep(ctypes.Structure):
+    """Mirror of the C struct sq_layer_step (include/shiftquant.h)."""
+    _fields_ = [
+        ("M", ctypes.c_int64), ("K", ctypes.c_int64), ("N", ctypes.c_int64),
+        ("bits", ctypes.c_int), ("n_groups", ctypes.c_int),
+        ("x", ctypes.c_void_p), ("w", ctypes.c_void_p), ("dy", ctypes.c_void_p),
+        ("x_codes", ctypes.c_void_p), ("ld_x", ctypes.c_int64),
+        ("xt_codes", ctypes.c_void_p), ("ld_xt", ctypes.c_int64),
+        ("x_range", ctypes.c_void_p), ("x_tau0", ctypes.c_void_p),
+        ("x_scale", ctypes.c_void_p), ("x_exp", ctypes.c_void_p),
+        ("g_codes", ctypes.c_void_p), ("ld_g", ctypes.c_int64),
+        ("gt_codes", ctypes.c_void_p), ("ld_gt", ctypes.c_int64),
+        ("g_range", ctypes.c_void_p), ("g_tau0", ctypes.c_void_p),
+        ("g_scale", ctypes.c_void_p), ("g_exp", ctypes.c_void_p),
+        ("wf_codes", ctypes.c_void_p), ("ld_wf", ctypes.c_int64),
+        ("wf_range", ctypes.c_void_p), ("wf_scale", ctypes.c_void_p),
+        ("wd_codes", ctypes.c_void_p), ("ld_wd", ctypes.c_int64),
+        ("wd_range", ctypes.c_void_p), ("wd_scale", ctypes.c_void_p),
+        ("y", ctypes.c_void_p), ("dx", ctypes.c_void_p), ("dw", ctypes.c_void_p),
+        ("workspace", ctypes.c_void_p), ("workspace_bytes", ctypes.c_size_t),
+        ("dev_status", ctypes.c_void_p),
     ]
 
 
@@ -126,6 +152,14 @@ def load(path: str | None = None) -> ctypes.CDLL:
     lib.shiftquant_gemm_layer_cta_pairs.restype = i32
     lib.shiftquant_gemm_workspace_bytes.argtypes = [i32, i64, i64, i64, i32, i32]
     lib.shiftquant_gemm_workspace_bytes.restype = sz
+    lib.shiftquant_layer_step.argtypes = [ctypes.POINTER(SqLayerStep), u64, vp]
+    lib.shiftquant_layer_step.restype = i32
+    lib.shiftquant_layer_step_host.argtypes = [ctypes.POINTER(SqLayerStep), vp, vp, vp, vp, vp,
+                                               vp, u64, vp]
+    lib.shiftquant_layer_step_host.restype = i32
+    lib.shiftquant_selftest_wait_timeout.argtypes = [vp, i64, vp, vp, i64, vp, i64, i64, i64,
+                                                     i32, i32, vp, i64, vp, vp]
+    lib.shiftquant_selftest_wait_timeout.restype = i32
     lib.shiftquant_status_string.argtypes = [i32]
     lib.shiftquant_status_string.restype = ctypes.c_char_p
     lib.shiftquant_last_error.argtypes = []
@@ -258,9 +292,11 @@ def _ld_opt(t) -> int:
 def shiftquant_gemm_layer(x_codes, xt_codes, x_scale, x_exp, g_codes, gt_codes, g_scale, g_exp,
                           wf_codes, wf_scale, wd_codes, wd_scale, M, K, N, bits, n_groups, y, dx,
                           dw, acc_y=None, acc_dx=None, acc_dw=None, workspace=None,
-                          dev_status=None, stream=None, gemm_mask=0, max_ctas=0) -> None:
+                          dev_status=None, stream=None, gemm_mask=0, max_ctas=0, y_range=None,
+                          dx_range=None) -> None:
     """Forward, loss-propagation and weight-gradient GEMMs of one layer in one launch
-    (gemm_mask: bit 0 forward, 1 loss propagation, 2 weight gradient; 0 = all)."""
+    (gemm_mask: bit 0 forward, 1 loss propagation, 2 weight gradient; 0 = all); y_range and
+    dx_range optionally receive the per-column max |Y| and max |dX| from the epilogue."""
     a = SqLayerGemms(
         x_codes=_addr(x_codes), ld_x=_ld_opt(x_codes), xt_codes=_addr(xt_codes),
         ld_xt=_ld_opt(xt_codes), x_scale=_addr(x_scale), x_exp=_addr(x_exp),
@@ -273,7 +309,8 @@ def shiftquant_gemm_layer(x_codes, xt_codes, x_scale, x_exp, g_codes, gt_codes, 
         ld_dw=_ld_opt(dw), acc_y=_addr(acc_y), ld_acc_y=_ld_opt(acc_y),
         acc_dx=_addr(acc_dx), ld_acc_dx=_ld_opt(acc_dx),
         acc_dw=_addr(acc_dw), ld_acc_dw=_ld_opt(acc_dw),
-        gemm_mask=gemm_mask, max_ctas=max_ctas)
+        gemm_mask=gemm_mask, max_ctas=max_ctas, y_range=_addr(y_range),
+        dx_range=_addr(dx_range))
     _check(load().shiftquant_gemm_layer(
         ctypes.byref(a), _ptr(workspace),
         workspace.numel() * workspace.element_size() if workspace is not None else 0,
@@ -313,3 +350,55 @@ def shiftquant_gemm_layer_cta_pairs(M: int, K: int, N: int, bits: int, n_groups:
                                     gemm_mask: int = 0) -> int:
     """1: the layer launch runs on 2-CTA clusters (256 x 256 tiles); 0: single-CTA tiles."""
     return int(load().shiftquant_gemm_layer_cta_pairs(M, K, N, bits, n_groups, gemm_mask))
+
+
+def layer_step_args(M, K, N, bits, n_groups, x, w, dy, x_codes, xt_codes, x_range, x_tau0,
+                    x_scale, x_exp, g_codes, gt_codes, g_range, g_tau0, g_scale, g_exp,
+                    wf_codes, wf_range, wf_scale, wd_codes, wd_range, wd_scale, y, dx, dw,
+                    workspace, dev_status) -> SqLayerStep:
+    """The C struct sq_layer_step over these device tensors (inputs and outputs dense)."""
+    for t, shape in ((x, (M, K)), (w, (K, N)), (dy, (M, N)), (y, (M, N)), (dx, (M, K)),
+                     (dw, (K, N))):
+        assert tuple(t.shape) == shape and t.is_contiguous(), "dense fp32 matrices expected"
+    return SqLayerStep(
+        M=M, K=K, N=N, bits=bits, n_groups=n_groups, x=_addr(x), w=_addr(w), dy=_addr(dy),
+        x_codes=_addr(x_codes), ld_x=_ld(x_codes), xt_codes=_addr(xt_codes), ld_xt=_ld(xt_codes),
+        x_range=_addr(x_range), x_tau0=_addr(x_tau0), x_scale=_addr(x_scale), x_exp=_addr(x_exp),
+        g_codes=_addr(g_codes), ld_g=_ld(g_codes), gt_codes=_addr(gt_codes), ld_gt=_ld(gt_codes),
+        g_range=_addr(g_range), g_tau0=_addr(g_tau0), g_scale=_addr(g_scale), g_exp=_addr(g_exp),
+        wf_codes=_addr(wf_codes), ld_wf=_ld(wf_codes), wf_range=_addr(wf_range),
+        wf_scale=_addr(wf_scale), wd_codes=_addr(wd_codes), ld_wd=_ld(wd_codes),
+        wd_range=_addr(wd_range), wd_scale=_addr(wd_scale), y=_addr(y), dx=_addr(dx),
+        dw=_addr(dw), workspace=_addr(workspace),
+        workspace_bytes=workspace.numel() * workspace.element_size() if workspace is not None else 0,
+        dev_status=_addr(dev_status))
+
+
+def shiftquant_layer_step(args: SqLayerStep, seed: int, stream=None) -> None:
+    """One layer's whole training step on the device (see the header)."""
+    _check(load().shiftquant_layer_step(ctypes.byref(args), seed & (2**64 - 1), _stream(stream)))
+
+
+def _host_ptr(t):
+    if t is None:
+        return None
+    assert t.device.type == "cpu" and t.is_contiguous() and t.dtype == torch.float32
+    return ctypes.c_void_p(t.data_ptr())
+
+
+def shiftquant_layer_step_host(args: SqLayerStep, x_host, w_host, dy_host, y_host, dx_host,
+                               dw_host, seed: int, stream=None) -> None:
+    """The step fed from host tensors and returned to them (pinned for asynchronous copies);
+    any of them may be None (see the header)."""
+    _check(load().shiftquant_layer_step_host(
+        ctypes.byref(args), _host_ptr(x_host), _host_ptr(w_host), _host_ptr(dy_host),
+        _host_ptr(y_host), _host_ptr(dx_host), _host_ptr(dw_host), seed & (2**64 - 1),
+        _stream(stream)))
+
+
+def shiftquant_selftest_wait_timeout(a_codes, a_scale, b_codes, b_scale, M, N, K, bits, n_groups,
+                                     y, dev_status, stream=None) -> None:
+    """A GEMM launch whose waits run out on purpose (see the header): SQ_DEV_TIMEOUT."""
+    _check(load().shiftquant_selftest_wait_timeout(
+        _ptr(a_codes), _ld(a_codes), _ptr(a_scale), _ptr(b_codes), _ld(b_codes), _ptr(b_scale),
+        M, N, K, bits, n_groups, _ptr(y), _ld(y), _ptr(dev_status), _stream(stream)))

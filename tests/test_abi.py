@@ -107,14 +107,21 @@ def test_host_validation_rejects_before_launch(lib):
              None) == native.SQ_EINVAL
 
 
-def test_exact_range_limits_reject_oversized_inner_dims(lib):
+def test_exact_range_limits_reject_before_launch(lib):
     st = ctypes.c_void_p(16)
     a16 = ctypes.c_void_p(256)
     g = lib.shiftquant_gemm_fwd
-    # 8-bit, N_G = 4: max |T| = 127 * 127 * 8 * K must stay below 2^31 -> K <= 16642
-    r = g(a16, 20000, st, a16, 20000, st, 8, 8, 20000, 8, 4, st, 8, None, 0, None, 0, st, None)
+    # 8-bit, N_G = 6: one 64-wide K block of products 127 * 127 * 32 can pass 2^24, the exact
+    # FP32 range of the tensor cores' sums, whatever K
+    r = g(a16, 64, st, a16, 64, st, 8, 8, 64, 8, 6, st, 8, None, 0, None, 0, st, None)
     assert r == native.SQ_EUNSUPPORTED
-    assert "exact" in lib.shiftquant_last_error().decode()
+    assert "exact FP32" in lib.shiftquant_last_error().decode()
+    # the sharded weight gradient adds int32 sums across ranks: 8 bits over more than 133144
+    # tokens in all is refused (a single-device call accumulates in int64 instead)
+    p = lib.shiftquant_gemm_wgrad_partial
+    r = p(a16, 140000, st, st, a16, 140000, st, st, 8, 8, 70000, 140000, 8, 4, a16, st, None)
+    assert r == native.SQ_EUNSUPPORTED
+    assert "int32" in lib.shiftquant_last_error().decode()
 
 
 @pytest.mark.skipif(__import__("torch").cuda.is_available(),
@@ -142,15 +149,18 @@ def test_empty_shapes_accept_null_pointers_of_empty_buffers(lib):
             assert r != native.SQ_EINVAL, (gran, R, C, lib.shiftquant_last_error())
 
 
-def test_layer_struct_layout_matches_the_binding(tmp_path):
-    # the ctypes mirror of sq_layer_gemms must have the C struct's size and field offsets
+@pytest.mark.parametrize("cname,pyname", [("sq_layer_gemms", "SqLayerGemms"),
+                                           ("sq_layer_step", "SqLayerStep")])
+def test_layer_struct_layout_matches_the_binding(tmp_path, cname, pyname):
+    # the ctypes mirrors of the C structs must have their size and field offsets
     import ctypes
-    from paper_2411_10948_gb300.native import SqLayerGemms
+    from paper_2411_10948_gb300 import native as nat
+    SqLayerGemms = getattr(nat, pyname)
     fields = [f for f, _ in SqLayerGemms._fields_]
     src = tmp_path / "layout.c"
     src.write_text('#include <stddef.h>\n#include <stdio.h>\n#include "shiftquant.h"\nint main(void) {\n'
-                   '  printf("%zu\\n", sizeof(sq_layer_gemms));\n' +
-                   "".join(f'  printf("%zu\\n", offsetof(sq_layer_gemms, {f}));\n' for f in fields) +
+                   f'  printf("%zu\\n", sizeof({cname}));\n' +
+                   "".join(f'  printf("%zu\\n", offsetof({cname}, {f}));\n' for f in fields) +
                    "  return 0;\n}\n")
     exe = tmp_path / "layout"
     subprocess.run(["gcc", "-std=c99", "-I", os.path.join(ROOT, "include"), str(src), "-o", str(exe)],
@@ -200,3 +210,25 @@ def test_static_weight_gradient_rejects_oversized_outputs_before_anything_else(l
         r = f(a16, 64, st, st, a16, 64, st, st, ci, co, 64, 4, 4, st, co, None, 0, st, None)
         assert r == native.SQ_EUNSUPPORTED, (ci, co)
         assert "static scratch" in lib.shiftquant_last_error().decode()
+
+
+def test_layer_step_validates_before_anything_runs(lib):
+    # a NULL struct, a missing status word, bad bits or a missing buffer fail on the host
+    from paper_2411_10948_gb300.native import SqLayerStep
+    assert lib.shiftquant_layer_step(None, 0, None) == native.SQ_EINVAL
+    fake = 4096
+    a = SqLayerStep(M=64, K=64, N=64, bits=4, n_groups=4, dev_status=None)
+    for f, _ in SqLayerStep._fields_:
+        if f not in ("M", "K", "N", "bits", "n_groups", "workspace", "workspace_bytes",
+                     "dev_status") and not f.startswith("ld_"):
+            setattr(a, f, fake)
+    assert lib.shiftquant_layer_step(ctypes.byref(a), 0, None) == native.SQ_EINVAL
+    a.dev_status = fake
+    a.bits = 9
+    assert lib.shiftquant_layer_step(ctypes.byref(a), 0, None) == native.SQ_EINVAL
+    a.bits = 4
+    a.dy = None
+    assert lib.shiftquant_layer_step(ctypes.byref(a), 0, None) == native.SQ_EINVAL
+    assert lib.shiftquant_layer_step_host(ctypes.byref(a), None, None, None, None, None, None, 0,
+                                          None) == native.SQ_EINVAL
+    assert "NULL" in lib.shiftquant_last_error().decode()

@@ -173,6 +173,86 @@ def test_worst_case_wgrad(bits, T):
                      "dW")
 
 
+@pytest.mark.parametrize("which,bits,G,K", [(0, 8, 4, 20000), (1, 8, 4, 21000), (0, 8, 5, 10000),
+                                            (1, 6, 4, 330000)])
+def test_int64_accumulation_beyond_the_int32_range(which, bits, G, K):
+    # max|T| = Q^2 2^(G-1) K passes 2^31: the K loop splits into int32-exact parts whose sums
+    # add in int64 in the workspace.  Same-sign worst-case products drive T past 2^31, odd
+    # products are mixed in, and T is compared with the exact integer product.
+    Q = 2 ** (bits - 1) - 1
+    M, Nn = 130, 260
+    rng = np.random.default_rng(K + which)
+    A = np.full((M, K), Q, np.int64)
+    A[1::2] *= -1
+    A[5] = rng.integers(-Q, Q + 1, K)
+    kk = np.arange(K)[None, :]
+    nn = np.arange(Nn)[:, None]
+    B = np.where((kk + nn) % 7 == 0, Q - 1, Q << (G - 1)).astype(np.int64)
+    B[7] = rng.integers(-Q, Q + 1, K) << rng.integers(0, G, K)
+    # the reference product in binary64 BLAS: every partial sum is an integer below 2^53,
+    # so it is exact whatever the summation order
+    T = np.rint(A.astype(np.float64) @ B.T.astype(np.float64)).astype(np.int64)
+    assert np.abs(T).max() > 2**31 and Q * Q * (1 << (G - 1)) * K > 2**31
+    a, b = _encode(A, bits, G), _encode(B, bits, G)
+    one = torch.ones(1, device="cuda")
+    ones = torch.ones(Nn, device="cuda")
+    y = torch.zeros((M, Nn), device="cuda")
+    acc = torch.zeros((M, Nn), dtype=torch.int64, device="cuda")
+    st = torch.zeros(1, dtype=torch.int32, device="cuda")
+    need = N.shiftquant_gemm_workspace_bytes(which, M, Nn, K, bits, G)
+    assert need >= M * Nn * 8
+    ws = torch.zeros(need // 4, dtype=torch.int32, device="cuda")
+    fn = N.shiftquant_gemm_fwd if which == 0 else N.shiftquant_gemm_dgrad
+    # without the workspace the call is refused before any launch
+    with pytest.raises(N.ShiftQuantError) as e:
+        fn(a, one, b, ones, M, Nn, K, bits, G, y, acc, None, st)
+    assert e.value.status == N.SQ_EUNSUPPORTED and "int64" in str(e.value)
+    fn(a, one, b, ones, M, Nn, K, bits, G, y, acc, ws, st)
+    torch.cuda.synchronize()
+    assert st.item() == 0
+    np.testing.assert_array_equal(acc.cpu().numpy(), T)
+    assert_close_f32(y.cpu().numpy(), T.astype(np.float64) * 2.0 ** -(G - 1), "Y")
+
+
+def test_int64_weight_gradient_beyond_the_int32_range():
+    # 8 bits over 160000 tokens: Q^2 T > 2^31, the token loop splits into int32-exact parts
+    bits, G, T = 8, 4, 160000
+    Q = 2 ** (bits - 1) - 1
+    Ci, Co = 96, 136
+    rng = np.random.default_rng(3)
+    X = np.full((Ci, T), Q, np.int64)
+    X[::5] = rng.integers(-Q, Q + 1, (len(X[::5]), T))
+    Y = np.full((Co, T), Q, np.int64)
+    Y[:, ::9] = 1
+    ex = rng.integers(0, G, Ci).astype(np.uint8)
+    ey = rng.integers(0, G, Co).astype(np.uint8)
+    a, b = _encode(X, bits, G), _encode(Y, bits, G)
+    raw = (torch.from_numpy(X).double() @ torch.from_numpy(Y).double().T).numpy()
+    raw = np.rint(raw).astype(np.int64)   # every partial sum is below 2^53: exact in binary64
+    assert np.abs(raw).max() > 2**31
+    one = torch.ones(1, device="cuda")
+    dw = torch.zeros((Ci, Co), device="cuda")
+    acc = torch.zeros((Ci, Co), dtype=torch.int64, device="cuda")
+    st = torch.zeros(1, dtype=torch.int32, device="cuda")
+    need = N.shiftquant_gemm_workspace_bytes(2, Ci, Co, T, bits, G)
+    ws = torch.zeros(need // 4, dtype=torch.int32, device="cuda")
+    N.shiftquant_gemm_wgrad(a, one, torch.from_numpy(ex).cuda(), b, one,
+                            torch.from_numpy(ey).cuda(), Ci, Co, T, bits, G, dw, acc, ws, st)
+    torch.cuda.synchronize()
+    assert st.item() == 0
+    sh = (2 * (G - 1) - ex.astype(np.int64)[:, None] - ey.astype(np.int64)[None, :])
+    np.testing.assert_array_equal(acc.cpu().numpy(), raw << sh)
+    assert_close_f32(dw.cpu().numpy(), raw * 2.0 ** -(ex[:, None] + ey[None, :]).astype(np.float64),
+                     "dW")
+
+
+def test_layer_launch_with_an_int64_gemm_matches_oracle():
+    # the layer launch mixes a forward GEMM past the int32 range (8 bits, K = 17000: int64
+    # splits) with the loss-propagation and weight-gradient GEMMs of ordinary ranges
+    rng = np.random.default_rng(17)
+    run_and_compare(*layer_inputs(rng, 256, 17000, 256), 8, 4, fused=True)
+
+
 def test_empty_and_zero_inner_dims():
     st = torch.zeros(1, dtype=torch.int32, device="cuda")
     one = torch.ones(1, device="cuda")
@@ -222,13 +302,13 @@ def test_concurrent_step_equals_serial_step():
         np.testing.assert_array_equal(a.cpu().numpy(), b.cpu().numpy())
 
 
-def test_host_pipeline_equals_device_steps():
-    # layer.HostPipeline (copies in, the captured step, copies back, on three streams with
-    # two alternating buffer sets): every step's host outputs equal a device-resident step
-    # on the same inputs and seed
+def test_c_host_steps_equal_device_steps():
+    # shiftquant_layer_step_host (copies in, the layer's whole step, copies back, inside one
+    # C call) driven by layer.HostSteps on two alternating buffer sets and streams: every
+    # step's host outputs equal a device-resident step on the same inputs and seed
     shapes = [(3000, 640, 384), (3000, 384, 640)]
     bits, G, seed, steps = 6, 4, 0x5EED, 5
-    pipe = L.HostPipeline(shapes, bits, G, "cuda", seed=seed)
+    pipe = L.HostSteps(shapes, bits, G, "cuda")
     host_in, host_out = [], []
     for i in range(steps):
         rng = np.random.default_rng(100 + i)
@@ -237,17 +317,40 @@ def test_host_pipeline_equals_device_steps():
         host_out.append([tuple(torch.empty(shp, dtype=torch.float32).pin_memory()
                                for shp in ((M, Nn), (M, K), (K, Nn)))
                          for (M, K, Nn) in shapes])
-    pipe.run(host_in, host_out).synchronize()
+    pipe.run(host_in, host_out, seed=seed).synchronize()
     assert pipe.status_ok()
     ref = [L.QuantLinear(M, K, Nn, bits, G, "cuda") for (M, K, Nn) in shapes]
     for i in range(steps):
         for li, lay in enumerate(ref):
             x, w, dy = (t.cuda() for t in host_in[i][li])
-            lay.step(x, w, dy, seed + i % 2)
+            lay.step(x, w, dy, seed + i)
             torch.cuda.synchronize()
             assert lay.status.item() == 0
             for got, want in zip(host_out[i][li], (lay.y, lay.dx, lay.dw)):
                 np.testing.assert_array_equal(got.numpy(), want.cpu().numpy())
+
+
+def test_c_layer_step_matches_oracle():
+    # shiftquant_layer_step on device inputs: the whole step against the oracle's layer
+    rng = np.random.default_rng(77)
+    M, K, Nn, bits, G, seed = 1000, 320, 288, 4, 4, 0xABC
+    x, w, dy = layer_inputs(rng, M, K, Nn)
+    lay = L.QuantLinear(M, K, Nn, bits, G, "cuda")
+    N.shiftquant_layer_step(lay.step_args(to_gpu(x), to_gpu(w), to_gpu(dy)), seed)
+    torch.cuda.synchronize()
+    assert lay.status.item() == 0
+    ox = O.shiftquant_tensor(x, bits, G, 0)
+    og = O.shiftquant_tensor(dy, bits, G, 1, seed)
+    wf = O.channel_tensor(w, bits, 0)
+    wd = O.channel_tensor(w, bits, 1)
+    want = (O.dequant(O.gemm_fwd(ox["codes"], ox["exp"], wf["codes"], G), ox["scale"], 1.0,
+                      G - 1, wf["scale"]),
+            O.dequant(O.gemm_dgrad(og["codes"], og["exp"], wd["codes"], G), og["scale"], 1.0,
+                      G - 1, wd["scale"]),
+            O.dequant(O.gemm_wgrad(ox["codes"], ox["exp"], og["codes"], og["exp"], G),
+                      ox["scale"], og["scale"], 2 * (G - 1)))
+    for got, ref, what in zip((lay.y, lay.dx, lay.dw), want, ("Y", "dX", "dW")):
+        assert_close_f32(got.cpu().numpy(), ref, what)
 
 
 @pytest.mark.parametrize("M,K,Nn", [(5, 3, 7), (300, 1000, 513), (4096, 64, 96), (2000, 700, 256)])
@@ -419,3 +522,58 @@ def test_token_shards_weight_gradient_is_exact(bits):
     assert st.item() == 0 and whole.status.item() == 0
     np.testing.assert_array_equal(acc.cpu().numpy(), whole.acc["wgrad"].cpu().numpy())
     np.testing.assert_array_equal(f32_bits(dw.cpu().numpy()), f32_bits(whole.dw.cpu().numpy()))
+
+
+@pytest.mark.parametrize("M,K,Nn,bits", [(4096, 512, 768, 6), (1000, 300, 250, 4),
+                                         (200, 2304, 256, 4), (3000, 4096, 1024, 6)])
+def test_fused_output_ranges_equal_a_range_pass_of_the_outputs(M, K, Nn, bits):
+    # y_range / dx_range of the layer launch (formed in the epilogue, or in the split-K output
+    # pass for a GEMM with few tiles) against the oracle's range pass over the GPU's own fp32
+    # Y and dX, bit for bit; ragged tiles, single and pair tile modes
+    rng = np.random.default_rng(M + K + Nn)
+    x, w, dy = layer_inputs(rng, M, K, Nn)
+    G = 4
+    lay = L.QuantLinear(M, K, Nn, bits, G, "cuda")
+    lay.quantize_activation(to_gpu(x))
+    lay.quantize_gradient(to_gpu(dy), 5)
+    lay.quantize_weights(to_gpu(w))
+    yr = torch.full((Nn,), 7.0, device="cuda")      # stale values: the call zeroes them first
+    dxr = torch.full((K,), 7.0, device="cuda")
+    lay.gemms(y_range=yr, dx_range=dxr)
+    torch.cuda.synchronize()
+    assert lay.status.item() == 0
+    for out, got, what in ((lay.y, yr, "Y"), (lay.dx, dxr, "dX")):
+        want, st = O.range_cols(out.cpu().numpy())
+        assert st == 0
+        np.testing.assert_array_equal(f32_bits(got.cpu().numpy()), f32_bits(want), err_msg=what)
+
+
+@pytest.mark.parametrize("bits", [4, 6])
+def test_chain_with_fused_ranges_equals_separate_range_passes(bits):
+    # a three-layer chain trained forward then backward: the fused range outputs replace the
+    # range passes of the inner activations and gradients and change no bit of any result
+    M, dims, G, seed = 1500, (320, 512, 384, 256), 4, 0x77
+    rng = np.random.default_rng(bits)
+    x0 = to_gpu(rng.standard_normal((M, dims[0])).astype(np.float32))
+    ws = [to_gpu((rng.standard_normal((dims[i], dims[i + 1])) * 0.05).astype(np.float32))
+          for i in range(3)]
+    dy = to_gpu((rng.laplace(0, 1, (M, dims[-1])) * np.exp(rng.normal(0, 2, dims[-1])))
+                .astype(np.float32))
+    out = []
+    for fused in (True, False):
+        ch = L.LinearChain(M, dims, bits, G, "cuda", fused_ranges=fused)
+        ch.step(x0, ws, dy, seed)
+        torch.cuda.synchronize()
+        assert ch.status_ok()
+        out.append(ch)
+    a, b = out
+    for la, lb in zip(a.layers, b.layers):
+        for t, u in ((la.y, lb.y), (la.dx, lb.dx), (la.dw, lb.dw), (la.x.exp, lb.x.exp),
+                     (la.g.exp, lb.g.exp), (la.x.tau0, lb.x.tau0), (la.g.tau0, lb.g.tau0)):
+            np.testing.assert_array_equal(t.cpu().numpy(), u.cpu().numpy())
+        np.testing.assert_array_equal(decode(la.x.codes), decode(lb.x.codes))
+        np.testing.assert_array_equal(decode(la.g.codes), decode(lb.g.codes))
+    # the inner tensors really were grouped from the fused ranges
+    for l in range(2):
+        want, _ = O.range_cols(a.layers[l].y.cpu().numpy())
+        np.testing.assert_array_equal(f32_bits(a.y_range[l].cpu().numpy()), f32_bits(want))
