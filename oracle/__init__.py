@@ -65,8 +65,11 @@ def _load():
         lib.sqo_gemm_dgrad.argtypes = [vp, vp, vp, i64, i64, i64, i32, vp, i64, vp]
         lib.sqo_gemm_wgrad.argtypes = [vp, vp, vp, vp, i64, i64, i64, i32, vp, i64, vp]
         lib.sqo_dequant.argtypes = [vp, i64, i64, f32, f32, i32, vp, vp]
+        lib.sqo_l1bn_forward.argtypes = [vp, i64, i64, i32, i32, vp, vp, vp, vp, vp, vp]
+        lib.sqo_l1bn_backward.argtypes = [vp, i64, i64, i32, i32, u64, vp, vp, vp, vp, vp, vp,
+                                          vp]
         for name in ("sqo_range_cols", "sqo_range_rows", "sqo_group", "sqo_quantize_shift",
-                     "sqo_quantize_channel"):
+                     "sqo_quantize_channel", "sqo_l1bn_forward", "sqo_l1bn_backward"):
             getattr(lib, name).restype = i32
         for name in ("sqo_gemm_fwd", "sqo_gemm_dgrad", "sqo_gemm_wgrad", "sqo_dequant"):
             getattr(lib, name).restype = None
@@ -223,3 +226,40 @@ def channel_tensor(w, bits: int, axis: int, mode: int = 0, seed: int = 0) -> dic
     rng, st = (range_cols(w) if axis == 0 else range_rows(w))
     q, s = quantize_channel(w, bits, axis, rng, mode, seed)
     return {"range": rng, "codes": q, "scale": s, "status": st}
+
+
+# --------------------------------------- Sec. 4, App. C: fully-quantized L1 BatchNorm
+def l1bn_forward(x, gamma, beta, bits: int = 8, n_groups: int = 4) -> dict:
+    """Forward of the fully-quantized L1 BatchNorm over x [R, C] (readings R12-R16 of the
+    C source): codes q, output y, integer stats (sum q, sum |q - m|, sum sign(q - m)) and
+    per-channel values (s, m, sigma, sigma^q, gamma^q, beta^q)."""
+    x = _f32(x)
+    R, C = x.shape
+    g = np.ascontiguousarray(gamma, np.float32)
+    b = np.ascontiguousarray(beta, np.float32)
+    q = np.empty((R, C), np.int8)
+    y = np.empty((R, C), np.float32)
+    stats = np.empty((3, C), np.int64)
+    chan = np.empty((6, C), np.float32)
+    st = _load().sqo_l1bn_forward(_p(x), R, C, bits, n_groups, _p(g), _p(b), _p(q), _p(y),
+                                  _p(stats), _p(chan))
+    names = ("s", "m", "sigma", "sigma_q", "gamma_q", "beta_q")
+    return {"q": q, "y": y, "S1": stats[0], "S": stats[1], "Z": stats[2], "stats": stats,
+            "chan": chan, **{k: chan[i] for i, k in enumerate(names)}, "status": int(st)}
+
+
+def l1bn_backward(gy, fwd: dict, bits: int = 8, n_groups: int = 4, seed: int = 0) -> dict:
+    """Backward of the fully-quantized L1 BatchNorm (R15) from gy [R, C] and the forward's
+    result: gradient codes p, dx, dgamma, dbeta."""
+    gy = _f32(gy)
+    R, C = gy.shape
+    p = np.empty((R, C), np.int8)
+    dx = np.empty((R, C), np.float32)
+    dg = np.empty(C, np.float32)
+    db = np.empty(C, np.float32)
+    st = _load().sqo_l1bn_backward(_p(gy), R, C, bits, n_groups, seed & (2**64 - 1),
+                                   _p(np.ascontiguousarray(fwd["q"])),
+                                   _p(np.ascontiguousarray(fwd["stats"])),
+                                   _p(np.ascontiguousarray(fwd["chan"])), _p(p), _p(dx), _p(dg),
+                                   _p(db))
+    return {"p": p, "dx": dx, "dgamma": dg, "dbeta": db, "status": int(st)}

@@ -34,6 +34,25 @@
  *       of both operands apply to the whole inner sum.
  *   R8  tau_0 == 0, or Q/tau_0 not finite: every code is 0 and the scale is 0.
  *       A NaN or Inf in the input sets the non-finite status; exponents are then 0.
+ *
+ * The fully-quantized L1 batch normalization (Sec. 4, App. C) takes these readings:
+ *   R12 sigma_1 of a channel is its mean absolute deviation (1/R) sum_r |x - mu| over the
+ *       channel's R elements (App. C writes the L1 norm |x - mu|_1; as a batch statistic it
+ *       is divided by the element count, as the L2 form is by its own).
+ *   R13 "all input features, statistics and parameters are quantized" (Sec. 4; 8 bits in
+ *       the paper's experiments): the input by ShiftQuant (round to nearest) to codes q with
+ *       per-channel steps s_c; the mean onto the channel's own code grid,
+ *       m_c = round-half-even(sum_r q / R), mu^q = m_c s_c, so that x^q - mu^q = (q - m) s_c
+ *       is an integer code difference; sigma to 8-bit codes on one per-tensor grid,
+ *       sigma^q = k_c (sigma_max / 127); gamma and beta to 8-bit symmetric per-tensor codes.
+ *   R14 a channel whose sigma^q is 0 outputs beta^q (x-hat = 0) and passes no gradient.
+ *   R15 backward: the incoming gradient by ShiftQuant with stochastic rounding, every
+ *       quantizer passed straight through, and the chain rule of L1 normalization
+ *       (sigma' = mean(sign(x - mu)) terms in place of L2's x-hat):
+ *       dx = (gamma / sigma)(g - mean g - mean(g xhat) (sign(d) - mean sign(d))),
+ *       dgamma = sum g xhat, dbeta = sum g.
+ *   R16 the binary32 order of every per-channel and per-element step, written out in
+ *       sqo_l1bn_forward / sqo_l1bn_backward; the sums over a channel are exact integers.
  */
 #include <math.h>
 #ifdef _OPENMP
@@ -331,4 +350,116 @@ void sqo_dequant(const int64_t *T, int64_t rows, int64_t cols, float s_a, float 
             double f = col_scale ? (double)col_scale[j] : 1.0;
             Y[i * cols + j] = (float)((double)T[i * cols + j] * base * f);
         }
+}
+
+/* ---------------------------------- Sec. 4, App. C: fully-quantized L1 BatchNorm */
+/* round-half-even of the rational a / b (b > 0), in integers */
+static int64_t sqo_rne_div(int64_t a, int64_t b) {
+    int64_t q = a / b, r = a % b;
+    if (r < 0) { q -= 1; r += b; }          /* floor division: 0 <= r < b */
+    if (2 * r > b || (2 * r == b && (q & 1))) q += 1;
+    return q;
+}
+
+/* symmetric 8-bit per-tensor quantization of a vector v[n] (R13): returns each v^q */
+static void sqo_quant8_tensor(const float *v, int64_t n, float *vq) {
+    float vmax = 0.0f;
+    for (int64_t i = 0; i < n; ++i) if (fabsf(v[i]) > vmax) vmax = fabsf(v[i]);
+    float inv = 127.0f / vmax, step = vmax / 127.0f;
+    int zero = !(vmax > 0.0f) || !sqo_finite(inv);
+    for (int64_t i = 0; i < n; ++i) {
+        float k = zero ? 0.0f : rintf(v[i] * inv);
+        if (k > 127.0f) k = 127.0f;
+        if (k < -127.0f) k = -127.0f;
+        vq[i] = k * step;
+    }
+}
+
+/* Forward of the fully-quantized L1 BatchNorm over x [R, C] (channels = columns, the R rows
+ * are the batch and spatial positions).  Outputs: q [R, C] the input's ShiftQuant codes,
+ * y [R, C], stats [3, C] = (sum q, sum |q - m|, sum sign(q - m)) and chan [6, C] =
+ * (s_c, m_c, sigma_c, sigma^q_c, gamma^q_c, beta^q_c).  Returns the input's status. */
+int sqo_l1bn_forward(const float *x, int64_t R, int64_t C, int bits, int G, const float *gamma,
+                     const float *beta, int8_t *q, float *y, int64_t *stats, float *chan) {
+    float *rng = (float *)malloc(sizeof(float) * (size_t)(C > 0 ? C : 1));
+    uint8_t *e = (uint8_t *)malloc((size_t)(C > 0 ? C : 1));
+    float tau0 = 0.0f, scale = 0.0f;
+    int st = sqo_range_cols(x, R, C, C, rng);
+    st |= sqo_group(rng, C, G, &tau0, e);
+    sqo_quantize_shift(x, R, C, C, bits, G, tau0, e, 0, 0, 0, q, &scale);
+    float *s_c = chan, *m_c = chan + C, *sig = chan + 2 * C, *sq = chan + 3 * C;
+    float *gq = chan + 4 * C, *bq = chan + 5 * C;
+    const float Rf = (float)R;
+    for (int64_t c = 0; c < C; ++c) {
+        int64_t S1 = 0, S = 0, Z = 0;
+        for (int64_t r = 0; r < R; ++r) S1 += q[r * C + c];
+        const int64_t m = R > 0 ? sqo_rne_div(S1, R) : 0;            /* mu^q = m s_c */
+        for (int64_t r = 0; r < R; ++r) {
+            const int64_t d = q[r * C + c] - m;
+            S += d < 0 ? -d : d;
+            Z += (d > 0) - (d < 0);
+        }
+        stats[c] = S1;
+        stats[C + c] = S;
+        stats[2 * C + c] = Z;
+        s_c[c] = ldexpf(scale, -(int)e[c]);                             /* step of channel c */
+        m_c[c] = (float)m;
+        sig[c] = ((float)S / Rf) * s_c[c];                              /* sigma_1 (R12) */
+    }
+    /* sigma^q on one 8-bit grid over the channels (sigma >= 0) */
+    sqo_quant8_tensor(sig, C, sq);
+    sqo_quant8_tensor(gamma, C, gq);
+    sqo_quant8_tensor(beta, C, bq);
+    for (int64_t r = 0; r < R; ++r) {
+        for (int64_t c = 0; c < C; ++c) {
+            const float xq = (float)q[r * C + c] * s_c[c];              /* x^q, exact */
+            const float mq = m_c[c] * s_c[c];                           /* mu^q, exact */
+            const float xhat = sq[c] > 0.0f ? (xq - mq) / sq[c] : 0.0f; /* R14 */
+            y[r * C + c] = gq[c] * xhat + bq[c];
+        }
+    }
+    free(rng);
+    free(e);
+    return st;
+}
+
+/* Backward (R15) from the incoming gradient gy [R, C], the forward's codes q, stats and
+ * chan.  Outputs: p [R, C] the gradient's ShiftQuant codes (stochastic rounding under
+ * `seed`), dx [R, C], dgamma [C], dbeta [C].  Returns the gradient's status. */
+int sqo_l1bn_backward(const float *gy, int64_t R, int64_t C, int bits, int G, uint64_t seed,
+                      const int8_t *q, const int64_t *stats, const float *chan, int8_t *p,
+                      float *dx, float *dgamma, float *dbeta) {
+    float *rng = (float *)malloc(sizeof(float) * (size_t)(C > 0 ? C : 1));
+    uint8_t *e = (uint8_t *)malloc((size_t)(C > 0 ? C : 1));
+    float tau0 = 0.0f, scale = 0.0f;
+    int st = sqo_range_cols(gy, R, C, C, rng);
+    st |= sqo_group(rng, C, G, &tau0, e);
+    sqo_quantize_shift(gy, R, C, C, bits, G, tau0, e, 1, seed, 0, p, &scale);
+    const float *s_c = chan, *m_c = chan + C, *sq = chan + 3 * C, *gq = chan + 4 * C;
+    const float Rf = (float)R;
+    for (int64_t c = 0; c < C; ++c) {
+        const int64_t m = (int64_t)m_c[c];
+        int64_t P = 0, D = 0;
+        for (int64_t r = 0; r < R; ++r) {
+            P += p[r * C + c];
+            D += (int64_t)p[r * C + c] * (q[r * C + c] - m);
+        }
+        const float t = ldexpf(scale, -(int)e[c]);                      /* step of g's channel */
+        const float u = sq[c] > 0.0f ? gq[c] / sq[c] : 0.0f;            /* gamma / sigma */
+        const float mg = ((float)P * t) / Rf;                           /* mean g */
+        const float dg = sq[c] > 0.0f ? (((float)D * t) * s_c[c]) / sq[c] : 0.0f;
+        const float mgx = dg / Rf;                                      /* mean(g xhat) */
+        const float zs = (float)stats[2 * C + c] / Rf;                  /* mean sign(d) */
+        dgamma[c] = dg;
+        dbeta[c] = (float)P * t;
+        for (int64_t r = 0; r < R; ++r) {
+            const int64_t d = q[r * C + c] - m;
+            const float g = (float)p[r * C + c] * t;
+            const float sg = (float)((d > 0) - (d < 0));
+            dx[r * C + c] = u * ((g - mg) - mgx * (sg - zs));
+        }
+    }
+    free(rng);
+    free(e);
+    return st;
 }
