@@ -59,6 +59,8 @@ def parse_args():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-chain", action="store_true",
                     help="skip the fused-range chain measurement")
+    ap.add_argument("--no-l1bn", action="store_true",
+                    help="skip the L1 batch normalization measurement")
     ap.add_argument("--also", default="conv3x3",
                     help="second workload summarised in the same line ('none' for none)")
     return ap.parse_args()
@@ -599,6 +601,61 @@ def run_chain(args, dev, flush_steps=None):
     return out
 
 
+L1BN_SHAPES = (("resnet_stage1", 64 * 56 * 56, 64), ("resnet_stage3", 64 * 14 * 14, 256))
+# HBM bytes per element of the passes (fp32 in / out, 1-byte codes): forward = range pass 4,
+# quantize + code sums 4 + 1, deviation sums 1, output 1 + 4; backward = range pass 4,
+# quantize + sums 4 + 1 (x codes) + 1 (gradient codes), output 1 + 1 + 4
+L1BN_FWD_BYTES, L1BN_BWD_BYTES = 15, 16
+
+
+def run_l1bn(args, dev):
+    """The fully-quantized L1 batch normalization (8-bit, N_G = 4) on ResNet-shaped
+    activations: forward and backward each timed with CUDA events after an L2 flush
+    (median), against HBM."""
+    import torch
+    from paper_2411_10948_gb300 import native as N
+    from paper_2411_10948_gb300 import workloads as W
+    peaks, src = load_peaks()
+    flush_w = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
+    out = []
+    steps = max(5, min(args.steps, 20))
+    for name, R, C in L1BN_SHAPES:
+        x = W.torch_tensor(("normal_outlier", 0.02, 50.0), R, C, args.seed + 1, dev)
+        dy = W.torch_tensor(("grad", "laplace", 2.0, 0.0, 1.0), R, C, args.seed + 2, dev)
+        gamma = torch.ones(C, device=dev) + 0.1 * torch.randn(C, device=dev)
+        beta = 0.1 * torch.randn(C, device=dev)
+        y, dx = torch.empty_like(x), torch.empty_like(x)
+        dg, db = torch.empty(C, device=dev), torch.empty(C, device=dev)
+        st = torch.zeros(1, dtype=torch.int32, device=dev)
+        state = torch.zeros(N.shiftquant_l1bn_state_bytes(R, C), dtype=torch.uint8, device=dev)
+        fwd = lambda: N.shiftquant_l1bn_forward(x, gamma, beta, 8, 4, y, state, st)
+        bwd = lambda: N.shiftquant_l1bn_backward(dy, 8, 4, 0x5EED, state, dx, dg, db, st)
+        for _ in range(3):
+            fwd()
+            bwd()
+        times = {"fwd": [], "bwd": []}
+        for _ in range(steps):
+            for k, fn in (("fwd", fwd), ("bwd", bwd)):
+                flush_w.zero_()
+                a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                a.record()
+                fn()
+                b.record()
+                b.synchronize()
+                times[k].append(a.elapsed_time(b))
+        assert st.item() == 0, "device status set in the L1 batch normalization"
+        fm, bm = statistics.median(times["fwd"]), statistics.median(times["bwd"])
+        fg = L1BN_FWD_BYTES * R * C / (fm * 1e-3) / 1e9
+        bg = L1BN_BWD_BYTES * R * C / (bm * 1e-3) / 1e9
+        out.append({"shape": name, "rows": R, "channels": C, "fwd_ms": fm, "bwd_ms": bm,
+                    "fwd_gbs": fg, "bwd_gbs": bg, "fwd_frac": fg / peaks["hbm_gbs"],
+                    "bwd_frac": bg / peaks["hbm_gbs"], "launches": {"fwd": 6, "bwd": 5}})
+    return {"bits": 8, "n_groups": 4, "bytes_per_element": {"fwd": L1BN_FWD_BYTES,
+                                                           "bwd": L1BN_BWD_BYTES},
+            "peak": peaks["hbm_gbs"], "peak_source": f"{src} copy bandwidth",
+            "statistic": "median over L2-flushed calls", "shapes": out}
+
+
 def oracle_sample_step(wl, rows_per_layer, seed):
     """One bounded oracle step: the quantizer chain and the three GEMMs on the first rows."""
     import oracle as O
@@ -711,6 +768,8 @@ def main():
                                    "clocks": other["clocks"]})
         if world == 1 and not args.no_chain:
             result["fused_range_chain"] = run_chain(args, f"cuda:{local_rank}")
+        if world == 1 and not args.no_l1bn:
+            result["l1bn"] = run_l1bn(args, f"cuda:{local_rank}")
         if world == 1 and not args.no_cpu_baseline:
             from paper_2411_10948_gb300 import workloads as W
             result["cpu_baseline"] = cpu_baseline(W.workload(args.workload), args.seed)

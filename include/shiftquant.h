@@ -352,11 +352,15 @@ sq_status shiftquant_layer_step(const sq_layer_step *args, uint64_t seed, void *
  * (cudaHostAlloc / cudaHostRegister) they overlap work on other streams, so a caller that
  * alternates two sets of device buffers on two streams overlaps one step's copies with the
  * other's compute; with pageable memory they still give the right result but block the
- * host.  The host outputs hold the results once the stream reaches the end of the call. */
+ * host.  The host outputs hold the results once the stream reaches the end of the call.
+ * inputs_queued (may be NULL): a cudaEvent_t the caller created; it is recorded on `stream`
+ * right after the input copies, so that the caller can queue the next call's copies behind
+ * this call's (another stream waiting on the event) while this call computes and copies
+ * back -- which keeps both directions of the host link busy. */
 sq_status shiftquant_layer_step_host(const sq_layer_step *args, const float *x_host,
                                      const float *w_host, const float *dy_host, float *y_host,
                                      float *dx_host, float *dw_host, uint64_t seed,
-                                     void *stream);
+                                     void *inputs_queued, void *stream);
 
 /* Weight-gradient GEMM for callers that cannot allocate device memory -- for instance a
  * plug-in running inside a host framework that owns every device allocation, or a
@@ -390,6 +394,45 @@ sq_status shiftquant_gemm_wgrad_static(const void *xt_codes, int64_t ldx, const 
  * 2 wgrad; M, N are the output dims and K the inner dim. */
 size_t shiftquant_gemm_workspace_bytes(int which, int64_t M, int64_t N, int64_t K,
                                        int bits, int n_groups);
+
+/* Fully-quantized L1 batch normalization (Sec. 4; App. C), training mode, over x [rows,
+ * channels] fp32 (row-major with leading dimension ld_x; the rows are a channel's batch
+ * and spatial positions, N H W).  With the readings this library takes of the paper:
+ *   - x quantized by ShiftQuant (bits, n_groups; round to nearest even) to int8 codes q,
+ *     step s_c = s 2^-e_c per channel;
+ *   - the mean onto the channel's code grid: m_c = round-half-even(sum_r q / rows),
+ *     mu^q = m_c s_c, so that x^q - mu^q = (q - m_c) s_c exactly;
+ *   - the L1 deviation sigma_c = (sum_r |q - m_c| / rows) s_c (mean absolute deviation);
+ *   - sigma, gamma[channels] and beta[channels] each quantized to 8-bit symmetric codes on
+ *     one per-tensor grid (step max / 127);
+ *   - y = gamma^q ((x^q - mu^q) / sigma^q) + beta^q, and beta^q where sigma^q is 0.
+ * Every channel sum is an exact integer and every other step one IEEE binary32 operation
+ * in a fixed order, so results do not depend on the launch configuration.
+ * state: a caller-owned device buffer of shiftquant_l1bn_state_bytes(rows, channels) bytes
+ *   (16-byte aligned) that the forward fills and the backward reads and extends: the int8
+ *   codes of x, row-major [rows, channels], at its start (kept for the backward, as a
+ *   quantized activation is), then the gradient's codes, the channel sums and values.
+ * rows >= 1 when channels >= 1; channels == 0 does nothing.  A NaN/Inf in x sets
+ * SQ_DEV_NONFINITE. */
+size_t shiftquant_l1bn_state_bytes(int64_t rows, int64_t channels);
+
+sq_status shiftquant_l1bn_forward(const float *x, int64_t rows, int64_t channels, int64_t ld_x,
+                                  const float *gamma, const float *beta, int bits,
+                                  int n_groups, float *y, int64_t ld_y, void *state,
+                                  size_t state_bytes, int32_t *dev_status, void *stream);
+
+/* Backward of the layer above from dy [rows, channels] (leading dimension ld_dy) and the
+ * state its forward left: dy quantized by ShiftQuant (bits, n_groups) with stochastic
+ * rounding drawn under `seed` (element index r * channels + c) to int8 codes p, g = p t_c;
+ * every quantizer passed straight through, the L1 normalization's chain rule
+ *   dx = (gamma^q / sigma^q) (g - mean g - mean(g xhat) (sign(q - m) - mean sign(q - m)))
+ * with xhat = (q - m) s_c / sigma^q, and dgamma[c] = sum_r g xhat, dbeta[c] = sum_r g (a
+ * channel with sigma^q = 0 passes dx = 0 and dgamma = 0).  dx [rows, ld_dx]. */
+sq_status shiftquant_l1bn_backward(const float *dy, int64_t rows, int64_t channels,
+                                   int64_t ld_dy, int bits, int n_groups, uint64_t seed,
+                                   void *state, size_t state_bytes, float *dx, int64_t ld_dx,
+                                   float *dgamma, float *dbeta, int32_t *dev_status,
+                                   void *stream);
 
 /* Failure-path self-test (for tests of the device-side timeout; the paper has no
  * counterpart).  One GEMM launch with the operands and layout of shiftquant_gemm_fwd whose

@@ -16,12 +16,13 @@ HERE = os.path.dirname(os.path.abspath(__file__))
 CSRC = os.path.join(HERE, "csrc")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libshiftquant.so")
-SOURCES = ["sq_quant.cu", "sq_gemm.cu", "sq_step.cu"]
+SOURCES = ["sq_quant.cu", "sq_gemm.cu", "sq_step.cu", "sq_l1bn.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 COMMON = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", "-Xcompiler", "-O2",
           "--expt-relaxed-constexpr"]
-# the quantizer rounds exactly as the method states: no multiply-add contraction anywhere
-PER_FILE = {"sq_quant.cu": ["-fmad=false"]}
+# the quantizer and the quantized normalization round exactly as the method states: no
+# multiply-add contraction anywhere in them
+PER_FILE = {"sq_quant.cu": ["-fmad=false"], "sq_l1bn.cu": ["-fmad=false"]}
 
 
 def nvcc() -> str:

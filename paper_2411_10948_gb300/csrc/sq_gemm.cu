@@ -229,11 +229,6 @@ __device__ __forceinline__ void emit_box(const GemmParams& p, const CUtensorMap*
     __syncwarp();
   }
   const bool row_scaled = p.mode == 1;
-  // the column maxima of |output| over the box's 32 rows: one warp reduction per column
-  // (lanes are rows), lane j keeps column j's
-  const bool colmax = p.colmax != nullptr && p.ws == nullptr;
-  const bool row_in = row0 + lane < p.M;
-  uint32_t cmax = 0u;
 #pragma unroll
   for (int k = 0; k < 8; ++k) {
     uint32_t o[4];
@@ -249,14 +244,42 @@ __device__ __forceinline__ void emit_box(const GemmParams& p, const CUtensorMap*
         // x * 1 is x exactly, so skipping the row factor of 1 changes no result
         o[e] = __float_as_uint(__fmul_rn(row_scaled ? __fmul_rn(val, rfac) : val, f[e]));
       }
-      if (colmax) {
-        const uint32_t m = __reduce_max_sync(0xFFFFFFFFu, row_in ? (o[e] & 0x7FFFFFFFu) : 0u);
-        if (lane == k * 4 + e) cmax = m;
-      }
     }
     st_shared_v4(buf + lane * 128 + ((k ^ (lane & 7)) << 4), o[0], o[1], o[2], o[3]);
   }
-  if (colmax && cmax != 0u && col0 + lane < p.N) atomicMax(p.colmax + col0 + lane, cmax);
+  if (p.colmax != nullptr && p.ws == nullptr) {
+    // The column maxima of |output| over the box's 32 rows, from the staged box: lane l
+    // reads the four columns 4 (l & 7) .. +3 of the eight rows 8 (l >> 3) .. +7 (16-byte
+    // loads), the four row groups combine by two exchanges, and lanes 0-7 add each column's
+    // maximum to the output range (ordered bit patterns of |y|).
+    __syncwarp();
+    const int cq = lane & 7, rg = lane >> 3;
+    uint32_t m[4] = {0u, 0u, 0u, 0u};
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      const int rr = rg * 8 + i;
+      if (row0 + rr < p.M) {
+        uint32_t v[4];
+        asm volatile("ld.shared.v4.b32 {%0, %1, %2, %3}, [%4];"
+                     : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3])
+                     : "r"(buf + rr * 128 + ((cq ^ (rr & 7)) << 4)));
+#pragma unroll
+        for (int e = 0; e < 4; ++e) m[e] = max(m[e], v[e] & 0x7FFFFFFFu);
+      }
+    }
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      m[e] = max(m[e], __shfl_xor_sync(0xFFFFFFFFu, m[e], 8));
+      m[e] = max(m[e], __shfl_xor_sync(0xFFFFFFFFu, m[e], 16));
+    }
+    if (rg == 0) {
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const int64_t col = col0 + cq * 4 + e;
+        if (m[e] != 0u && col < p.N) atomicMax(p.colmax + col, m[e]);
+      }
+    }
+  }
   if (p.ws != nullptr && p.wide) {
     // a split of a K loop beyond the int32 range: its exact int32 sums are added into the
     // int64 workspace, row by row (the lanes cover 32 consecutive columns of a row)

@@ -21,6 +21,7 @@
 
 #include "sq_device.cuh"
 #include "sq_host.h"
+#include "sq_quant_dev.cuh"
 
 namespace sq {
 
@@ -261,16 +262,6 @@ struct QuantArgs {
   int vec_in, vec_out, vec_t;
 };
 
-// SplitMix64 (Steele, Lea, Flood 2014): the (idx+1)-th output of the generator whose
-// state starts at `seed`.
-__device__ __forceinline__ uint64_t splitmix64_at(uint64_t seed, uint64_t idx) {
-  uint64_t z = seed + (idx + 1ull) * 0x9E3779B97F4A7C15ull;
-  z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
-  z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
-  return z ^ (z >> 31);
-}
-
-__device__ __forceinline__ float pow2f(int k) { return __int_as_float((127 + k) << 23); }
 
 template <typename CodeT>
 __device__ __forceinline__ CodeT encode_code(float v);

@@ -106,7 +106,8 @@ extern "C" sq_status shiftquant_layer_step(const sq_layer_step* args, uint64_t s
 extern "C" sq_status shiftquant_layer_step_host(const sq_layer_step* args, const float* x_host,
                                                 const float* w_host, const float* dy_host,
                                                 float* y_host, float* dx_host, float* dw_host,
-                                                uint64_t seed, void* stream) {
+                                                uint64_t seed, void* inputs_queued,
+                                                void* stream) {
   fail(SQ_OK, "");
   int st = check_step(args);
   if (st != SQ_OK || args->M == 0 || args->K == 0 || args->N == 0) return st;
@@ -115,6 +116,10 @@ extern "C" sq_status shiftquant_layer_step_host(const sq_layer_step* args, const
   if ((st = copy(args->x, x_host, M * K, cudaMemcpyHostToDevice, s)) != SQ_OK) return st;
   if ((st = copy(args->w, w_host, K * N, cudaMemcpyHostToDevice, s)) != SQ_OK) return st;
   if ((st = copy(args->dy, dy_host, M * N, cudaMemcpyHostToDevice, s)) != SQ_OK) return st;
+  if (inputs_queued != nullptr) {
+    const cudaError_t err = cudaEventRecord(static_cast<cudaEvent_t>(inputs_queued), s);
+    if (err != cudaSuccess) return cuda_fail(err, "cudaEventRecord");
+  }
   if ((st = run_step(args, seed, stream)) != SQ_OK) return st;
   if ((st = copy(y_host, args->y, M * N, cudaMemcpyDeviceToHost, s)) != SQ_OK) return st;
   if ((st = copy(dx_host, args->dx, M * K, cudaMemcpyDeviceToHost, s)) != SQ_OK) return st;

@@ -364,8 +364,10 @@ class HostSteps:
     shiftquant_layer_step_host: for every layer of a step, one call copies X, W and dY in,
     runs the layer's whole step and copies Y, dX and dW back, all inside the library and in
     the order of one stream.  Two sets of device buffers, each with its own stream, take
-    the steps in turn, so one step's copies overlap the other's compute and the host
-    link's two directions, not the GPU, set the pace.
+    the steps in turn; every call's input copies queue behind the previous call's (an event
+    the library records after them), so the copies in run back to back while the other
+    slot computes and copies back, and the host link's two directions, not the GPU, set
+    the pace.
 
     shapes: (M, K, N) per layer."""
 
@@ -378,6 +380,11 @@ class HostSteps:
                       for (M, K, N_) in self.shapes]
             self.slots.append({"layers": layers, "args": [l.step_args() for l in layers],
                                "stream": torch.cuda.Stream(device=dev)})
+        # a ring of events marking each call's queued input copies (recorded once here so
+        # that the CUDA events exist before the library records them)
+        self.events = [torch.cuda.Event() for _ in range(2 * slots * max(1, len(self.shapes)))]
+        for ev in self.events:
+            ev.record()
 
     def run(self, host_inputs, host_outputs, seed=0x5EED) -> torch.cuda.Event:
         """Queue one step per entry: host_inputs[i] = (x, w, dy) per layer, host_outputs[i] =
@@ -388,10 +395,16 @@ class HostSteps:
         cur = torch.cuda.current_stream()
         for sl in self.slots:
             sl["stream"].wait_stream(cur)
+        prev, k = None, 0
         for i, (hin, hout) in enumerate(zip(host_inputs, host_outputs)):
             sl = self.slots[i % len(self.slots)]
             for args, (x, w, dy), (y, dx, dw) in zip(sl["args"], hin, hout):
-                N.shiftquant_layer_step_host(args, x, w, dy, y, dx, dw, seed + i, sl["stream"])
+                if prev is not None:
+                    sl["stream"].wait_event(prev)
+                ev = self.events[k % len(self.events)]
+                N.shiftquant_layer_step_host(args, x, w, dy, y, dx, dw, seed + i, sl["stream"],
+                                             inputs_queued=ev)
+                prev, k = ev, k + 1
         for sl in self.slots:
             cur.wait_stream(sl["stream"])
         end = torch.cuda.Event(enable_timing=True)

@@ -38,6 +38,7 @@ EXPORTS = (
     "shiftquant_gemm_layer", "shiftquant_gemm_layer_workspace_bytes",
     "shiftquant_gemm_layer_kernel_launches", "shiftquant_gemm_layer_cta_pairs",
     "shiftquant_layer_step", "shiftquant_layer_step_host", "shiftquant_selftest_wait_timeout",
+    "shiftquant_l1bn_state_bytes", "shiftquant_l1bn_forward", "shiftquant_l1bn_backward",
     "shiftquant_status_string", "shiftquant_last_error",
 )
 
@@ -155,11 +156,19 @@ def load(path: str | None = None) -> ctypes.CDLL:
     lib.shiftquant_layer_step.argtypes = [ctypes.POINTER(SqLayerStep), u64, vp]
     lib.shiftquant_layer_step.restype = i32
     lib.shiftquant_layer_step_host.argtypes = [ctypes.POINTER(SqLayerStep), vp, vp, vp, vp, vp,
-                                               vp, u64, vp]
+                                               vp, u64, vp, vp]
     lib.shiftquant_layer_step_host.restype = i32
     lib.shiftquant_selftest_wait_timeout.argtypes = [vp, i64, vp, vp, i64, vp, i64, i64, i64,
                                                      i32, i32, vp, i64, vp, vp]
     lib.shiftquant_selftest_wait_timeout.restype = i32
+    lib.shiftquant_l1bn_state_bytes.argtypes = [i64, i64]
+    lib.shiftquant_l1bn_state_bytes.restype = sz
+    lib.shiftquant_l1bn_forward.argtypes = [vp, i64, i64, i64, vp, vp, i32, i32, vp, i64, vp, sz,
+                                            vp, vp]
+    lib.shiftquant_l1bn_forward.restype = i32
+    lib.shiftquant_l1bn_backward.argtypes = [vp, i64, i64, i64, i32, i32, u64, vp, sz, vp, i64,
+                                             vp, vp, vp, vp]
+    lib.shiftquant_l1bn_backward.restype = i32
     lib.shiftquant_status_string.argtypes = [i32]
     lib.shiftquant_status_string.restype = ctypes.c_char_p
     lib.shiftquant_last_error.argtypes = []
@@ -387,12 +396,14 @@ def _host_ptr(t):
 
 
 def shiftquant_layer_step_host(args: SqLayerStep, x_host, w_host, dy_host, y_host, dx_host,
-                               dw_host, seed: int, stream=None) -> None:
+                               dw_host, seed: int, stream=None, inputs_queued=None) -> None:
     """The step fed from host tensors and returned to them (pinned for asynchronous copies);
-    any of them may be None (see the header)."""
+    any of them may be None.  inputs_queued: an optional torch.cuda.Event (already created)
+    recorded after the input copies (see the header)."""
+    ev = ctypes.c_void_p(inputs_queued.cuda_event) if inputs_queued is not None else None
     _check(load().shiftquant_layer_step_host(
         ctypes.byref(args), _host_ptr(x_host), _host_ptr(w_host), _host_ptr(dy_host),
-        _host_ptr(y_host), _host_ptr(dx_host), _host_ptr(dw_host), seed & (2**64 - 1),
+        _host_ptr(y_host), _host_ptr(dx_host), _host_ptr(dw_host), seed & (2**64 - 1), ev,
         _stream(stream)))
 
 
@@ -402,3 +413,25 @@ def shiftquant_selftest_wait_timeout(a_codes, a_scale, b_codes, b_scale, M, N, K
     _check(load().shiftquant_selftest_wait_timeout(
         _ptr(a_codes), _ld(a_codes), _ptr(a_scale), _ptr(b_codes), _ld(b_codes), _ptr(b_scale),
         M, N, K, bits, n_groups, _ptr(y), _ld(y), _ptr(dev_status), _stream(stream)))
+
+
+def shiftquant_l1bn_state_bytes(rows: int, channels: int) -> int:
+    return int(load().shiftquant_l1bn_state_bytes(rows, channels))
+
+
+def shiftquant_l1bn_forward(x, gamma, beta, bits, n_groups, y, state, dev_status,
+                            stream=None) -> None:
+    """Fully-quantized L1 batch normalization, forward (see the header)."""
+    _check(load().shiftquant_l1bn_forward(
+        _ptr(x), x.shape[0], x.shape[1], _ld(x), _ptr(gamma), _ptr(beta), bits, n_groups,
+        _ptr(y), _ld(y), _ptr(state), state.numel() * state.element_size(), _ptr(dev_status),
+        _stream(stream)))
+
+
+def shiftquant_l1bn_backward(dy, bits, n_groups, seed, state, dx, dgamma, dbeta, dev_status,
+                             stream=None) -> None:
+    """Fully-quantized L1 batch normalization, backward (see the header)."""
+    _check(load().shiftquant_l1bn_backward(
+        _ptr(dy), dy.shape[0], dy.shape[1], _ld(dy), bits, n_groups, seed & (2**64 - 1),
+        _ptr(state), state.numel() * state.element_size(), _ptr(dx), _ld(dx), _ptr(dgamma),
+        _ptr(dbeta), _ptr(dev_status), _stream(stream)))

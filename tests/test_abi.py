@@ -230,5 +230,5 @@ def test_layer_step_validates_before_anything_runs(lib):
     a.dy = None
     assert lib.shiftquant_layer_step(ctypes.byref(a), 0, None) == native.SQ_EINVAL
     assert lib.shiftquant_layer_step_host(ctypes.byref(a), None, None, None, None, None, None, 0,
-                                          None) == native.SQ_EINVAL
+                                          None, None) == native.SQ_EINVAL
     assert "NULL" in lib.shiftquant_last_error().decode()
