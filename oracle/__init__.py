@@ -65,6 +65,12 @@ def _load():
         lib.sqo_gemm_dgrad.argtypes = [vp, vp, vp, i64, i64, i64, i32, vp, i64, vp]
         lib.sqo_gemm_wgrad.argtypes = [vp, vp, vp, vp, i64, i64, i64, i32, vp, i64, vp]
         lib.sqo_dequant.argtypes = [vp, i64, i64, f32, f32, i32, vp, vp]
+        lib.sqo_pack4.argtypes = [vp, i64, i64, vp]
+        lib.sqo_unpack4.argtypes = [vp, i64, i64, vp]
+        lib.sqo_pack_groups.argtypes = [vp, i64, i32, vp]
+        lib.sqo_unpack_groups.argtypes = [vp, i64, i32, vp]
+        for name in ("sqo_pack4", "sqo_unpack4", "sqo_pack_groups", "sqo_unpack_groups"):
+            getattr(lib, name).restype = None
         lib.sqo_l1bn_forward.argtypes = [vp, i64, i64, i32, i32, vp, vp, vp, vp, vp, vp]
         lib.sqo_l1bn_backward.argtypes = [vp, i64, i64, i32, i32, u64, vp, vp, vp, vp, vp, vp,
                                           vp]
@@ -263,3 +269,41 @@ def l1bn_backward(gy, fwd: dict, bits: int = 8, n_groups: int = 4, seed: int = 0
                                    _p(np.ascontiguousarray(fwd["chan"])), _p(p), _p(dx), _p(dg),
                                    _p(db))
     return {"p": p, "dx": dx, "dgamma": dg, "dbeta": db, "status": int(st)}
+
+
+# ------------------------------------------- Sec. 5.2: packed sub-byte storage (R17, R18)
+def pack4(q) -> np.ndarray:
+    """Codes of at most 4 bits [R, C] -> bytes [R, ceil(C/2)], two's-complement nibbles,
+    element 2b in the low nibble of byte b."""
+    q = np.ascontiguousarray(q, np.int8)
+    R, C = q.shape
+    out = np.empty((R, (C + 1) // 2), np.uint8)
+    _load().sqo_pack4(_p(q), R, C, _p(out))
+    return out
+
+
+def unpack4(b, cols: int) -> np.ndarray:
+    b = np.ascontiguousarray(b, np.uint8)
+    q = np.empty((b.shape[0], cols), np.int8)
+    _load().sqo_unpack4(_p(b), b.shape[0], cols, _p(q))
+    return q
+
+
+def group_field_bits(n_groups: int) -> int:
+    return 1 if n_groups <= 2 else (2 if n_groups <= 4 else 4)
+
+
+def pack_groups(e, n_groups: int) -> np.ndarray:
+    """The grouping map in 1/2/4-bit fields, 8/w channels per byte (low bits first)."""
+    e = np.ascontiguousarray(e, np.uint8)
+    per = 8 // group_field_bits(n_groups)
+    out = np.empty((e.size + per - 1) // per, np.uint8)
+    _load().sqo_pack_groups(_p(e), e.size, n_groups, _p(out))
+    return out
+
+
+def unpack_groups(b, channels: int, n_groups: int) -> np.ndarray:
+    b = np.ascontiguousarray(b, np.uint8)
+    e = np.empty(channels, np.uint8)
+    _load().sqo_unpack_groups(_p(b), channels, n_groups, _p(e))
+    return e

@@ -53,6 +53,15 @@
  *       dgamma = sum g xhat, dbeta = sum g.
  *   R16 the binary32 order of every per-channel and per-element step, written out in
  *       sqo_l1bn_forward / sqo_l1bn_backward; the sums over a channel are exact integers.
+ *
+ * Packed sub-byte storage (Sec. 5.2: with N_G = 4 the grouping map takes exactly 2 bits):
+ *   R17 codes of at most 4 bits are stored two per byte as 4-bit two's complement: element c
+ *       of a row in byte c / 2, the low nibble for even c and the high nibble for odd c; a
+ *       row of C codes takes ceil(C / 2) bytes, an odd row's last high nibble is 0.
+ *   R18 the grouping map stores each channel's exponent in w = 1, 2 or 4 bits (N_G <= 2,
+ *       <= 4, <= 8: the smallest power-of-two field that holds N_G - 1, so that no field
+ *       straddles a byte), 8 / w channels per byte, channel c at bit (c mod (8 / w)) w of
+ *       byte c / (8 / w).
  */
 #include <math.h>
 #ifdef _OPENMP
@@ -462,4 +471,40 @@ int sqo_l1bn_backward(const float *gy, int64_t R, int64_t C, int bits, int G, ui
     free(rng);
     free(e);
     return st;
+}
+
+/* ------------------------------- Sec. 5.2 (R17, R18): packed sub-byte storage */
+void sqo_pack4(const int8_t *q, int64_t R, int64_t C, uint8_t *out) {
+    const int64_t W = (C + 1) / 2;
+    for (int64_t r = 0; r < R; ++r)
+        for (int64_t b = 0; b < W; ++b) {
+            const int lo = q[r * C + 2 * b];
+            const int hi = 2 * b + 1 < C ? q[r * C + 2 * b + 1] : 0;
+            out[r * W + b] = (uint8_t)((lo & 0xF) | ((hi & 0xF) << 4));
+        }
+}
+
+void sqo_unpack4(const uint8_t *in, int64_t R, int64_t C, int8_t *q) {
+    const int64_t W = (C + 1) / 2;
+    for (int64_t r = 0; r < R; ++r)
+        for (int64_t c = 0; c < C; ++c) {
+            const int nib = (in[r * W + c / 2] >> (4 * (c & 1))) & 0xF;
+            q[r * C + c] = (int8_t)(nib >= 8 ? nib - 16 : nib);     /* two's complement */
+        }
+}
+
+static int sqo_group_bits(int G) { return G <= 2 ? 1 : (G <= 4 ? 2 : 4); }
+
+void sqo_pack_groups(const uint8_t *e, int64_t C, int G, uint8_t *out) {
+    const int w = sqo_group_bits(G), per = 8 / w;
+    const int64_t W = (C + per - 1) / per;
+    for (int64_t b = 0; b < W; ++b) out[b] = 0;
+    for (int64_t c = 0; c < C; ++c)
+        out[c / per] |= (uint8_t)((e[c] & ((1 << w) - 1)) << ((c % per) * w));
+}
+
+void sqo_unpack_groups(const uint8_t *in, int64_t C, int G, uint8_t *e) {
+    const int w = sqo_group_bits(G), per = 8 / w;
+    for (int64_t c = 0; c < C; ++c)
+        e[c] = (uint8_t)((in[c / per] >> ((c % per) * w)) & ((1 << w) - 1));
 }

@@ -470,3 +470,40 @@ def test_sr_draws_match_published_generator_outputs():
         d = O.shiftquant_tensor(x, 4, 1, mode=1, seed=seed)
         assert float(d["tau0"]) == 7.0 and (d["exp"] == 0).all()
         np.testing.assert_array_equal(d["codes"], codes, err_msg=name)
+
+
+# --------------------------------- packed sub-byte storage (Sec. 5.2; R17, R18)
+def _golden_packed():
+    d = {}
+    for line in _read_golden("packed_storage.txt"):
+        k, *v = line.split()
+        d[k] = v
+    return d
+
+
+def test_packed_codes_and_group_maps_by_hand():
+    d = _golden_packed()
+    q = np.array([[int(v) for v in d["codes0"]], [int(v) for v in d["codes1"]]], np.int8)
+    want = np.array([[int(v, 16) for v in d["packed0"]], [int(v, 16) for v in d["packed1"]]],
+                    np.uint8)
+    np.testing.assert_array_equal(O.pack4(q), want)
+    np.testing.assert_array_equal(O.unpack4(want, 7), q)
+    for G, key in ((4, "map4"), (8, "map8"), (2, "map2")):
+        e = np.array([int(v) for v in d[key]], np.uint8)
+        b = np.array([int(v, 16) for v in d[key + "_bytes"]], np.uint8)
+        np.testing.assert_array_equal(O.pack_groups(e, G), b)
+        np.testing.assert_array_equal(O.unpack_groups(b, e.size, G), e)
+
+
+@pytest.mark.parametrize("C", [1, 2, 7, 64, 129])
+def test_packing_round_trips_and_halves_the_bytes(C):
+    rng = np.random.default_rng(C)
+    q = rng.integers(-8, 8, (5, C)).astype(np.int8)
+    b = O.pack4(q)
+    assert b.shape == (5, (C + 1) // 2)
+    np.testing.assert_array_equal(O.unpack4(b, C), q)
+    for G in (1, 2, 3, 4, 5, 8):
+        e = rng.integers(0, G, C).astype(np.uint8)
+        np.testing.assert_array_equal(O.unpack_groups(O.pack_groups(e, G), C, G), e)
+    # the 2-bit map of N_G = 4 (Sec. 5.2): four channels per byte
+    assert O.pack_groups(np.zeros(C, np.uint8), 4).size == (C + 3) // 4
