@@ -61,6 +61,10 @@ def parse_args():
                     help="skip the fused-range chain measurement")
     ap.add_argument("--no-l1bn", action="store_true",
                     help="skip the L1 batch normalization measurement")
+    ap.add_argument("--no-group-order", action="store_true",
+                    help="skip the group-ordered contraction measurement")
+    ap.add_argument("--no-pack", action="store_true",
+                    help="skip the packed-storage measurement")
     ap.add_argument("--also", default="conv3x3",
                     help="second workload summarised in the same line ('none' for none)")
     return ap.parse_args()
@@ -656,6 +660,106 @@ def run_l1bn(args, dev):
             "statistic": "median over L2-flushed calls", "shapes": out}
 
 
+def run_group_order(args, dev):
+    """The group-ordered contraction against the folded layout, on the 8-bit large_linear
+    layers (16384 tokens, 4096 <-> 11008): each layer's GEMM launch timed alone (median of
+    CUDA-event timings after an L2 flush), on the workload's own data and on 'flat' data whose
+    channels all fall in the top group (N(0,1) activations and gradients: every range within a
+    factor 2 of the largest), where the folded layout's chunks are shortest."""
+    import torch
+    from paper_2411_10948_gb300 import layer as L
+    from paper_2411_10948_gb300 import workloads as W
+    peaks, src = load_peaks()
+    wl = W.workload("large_linear_8bit")
+    flush_w = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
+    steps = max(3, min(args.steps, 10))
+    rows = []
+    for data in ("workload", "flat"):
+        for grouped in (False, True):
+            ms_tot, flops = 0.0, 0
+            for li, spec in enumerate(wl.layers):
+                x, w, dy = W.torch_layer_inputs(spec, args.seed, li, dev)
+                if data == "flat":
+                    x = torch.randn_like(x)
+                    dy = torch.randn_like(dy)
+                lay = L.QuantLinear(spec.M, spec.K, spec.N, spec.bits, spec.n_groups, dev,
+                                    grouped=grouped)
+                lay.quantize_activation(x)
+                lay.quantize_gradient(dy, 7)
+                lay.quantize_weights(w)
+                for _ in range(2):
+                    lay.gemms()
+                ts = []
+                for _ in range(steps):
+                    flush_w.zero_()
+                    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                    a.record()
+                    lay.gemms()
+                    b.record()
+                    b.synchronize()
+                    ts.append(a.elapsed_time(b))
+                assert lay.status.item() == 0, "device status set"
+                hist = [int(v) for v in torch.bincount(lay.x.exp.long(), minlength=spec.n_groups).cpu()]
+                ms_tot += statistics.median(ts)
+                flops += lay.gemm_ops
+                del lay, x, w, dy
+            tf = flops / (ms_tot * 1e-3) / 1e12
+            rows.append({"data": data, "layout": "group-ordered" if grouped else "folded",
+                         "gemm_ms": ms_tot, "tflops": tf, "frac": tf / peaks["bf16_tflops"],
+                         "x_group_histogram_last_layer": hist})
+    return {"workload": "large_linear_8bit layers (16384 x 4096 x 11008, 16384 x 11008 x 4096)",
+            "peak": peaks["bf16_tflops"], "peak_source": f"{src} bf16 burst",
+            "statistic": "sum over the two layers of the median layer-launch time", "rows": rows}
+
+
+def run_pack(args, dev):
+    """Packed sub-byte storage of the 4-bit conv3x3 activation codes (X [12544, 2304] and the
+    transposed copy the weight gradient keeps): pack (1 byte read + 0.5 written per code) and
+    unpack (0.5 + 1), each timed with CUDA events after an L2 flush (median), against HBM."""
+    import torch
+    from paper_2411_10948_gb300 import layer as L
+    from paper_2411_10948_gb300 import native as N
+    from paper_2411_10948_gb300 import workloads as W
+    peaks, src = load_peaks()
+    spec = W.workload("conv3x3").layers[0]
+    bits, G = spec.bits, spec.n_groups
+    x = W.torch_tensor(spec.act, spec.M, spec.K, args.seed + 3, dev)
+    q = L.ShiftTensor.alloc(spec.M, spec.K, bits, G, dev)
+    st = torch.zeros(1, dtype=torch.int32, device=dev)
+    L.shift_quantize(x, q, bits, G, N.SQ_ROUND_NEAREST_EVEN, 0, st)
+    flush_w = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
+    steps = max(5, min(args.steps, 20))
+    out = []
+    for name, codes in (("X codes", q.codes), ("X codes transposed", q.codes_t)):
+        R, C = codes.shape
+        packed = torch.zeros((R, (C + 15) // 16 * 8), dtype=torch.uint8, device=dev)
+        back = L.empty_codes(R, C, bits, G, dev)
+        fns = {"pack": lambda: N.shiftquant_pack_codes(codes, bits, G, packed, st),
+               "unpack": lambda: N.shiftquant_unpack_codes(packed, C, bits, G, back)}
+        row = {"tensor": name, "rows": R, "cols": C, "bytes_codes": R * C,
+               "bytes_packed": R * ((C + 1) // 2)}
+        for k, fn in fns.items():
+            fn()
+            ts = []
+            for _ in range(steps):
+                flush_w.zero_()
+                a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                a.record()
+                fn()
+                b.record()
+                b.synchronize()
+                ts.append(a.elapsed_time(b))
+            ms = statistics.median(ts)
+            gbs = 1.5 * R * C / (ms * 1e-3) / 1e9
+            row.update({f"{k}_ms": ms, f"{k}_gbs": gbs, f"{k}_frac": gbs / peaks["hbm_gbs"]})
+        assert torch.equal(back.view(torch.uint8), codes.view(torch.uint8)), "round trip"
+        out.append(row)
+    assert st.item() == 0
+    return {"bits": bits, "n_groups": G, "bytes_per_code": 1.5, "peak": peaks["hbm_gbs"],
+            "peak_source": f"{src} copy bandwidth", "statistic": "median over L2-flushed calls",
+            "tensors": out}
+
+
 def oracle_sample_step(wl, rows_per_layer, seed):
     """One bounded oracle step: the quantizer chain and the three GEMMs on the first rows."""
     import oracle as O
@@ -770,6 +874,10 @@ def main():
             result["fused_range_chain"] = run_chain(args, f"cuda:{local_rank}")
         if world == 1 and not args.no_l1bn:
             result["l1bn"] = run_l1bn(args, f"cuda:{local_rank}")
+        if world == 1 and not args.no_group_order:
+            result["group_order"] = run_group_order(args, f"cuda:{local_rank}")
+        if world == 1 and not args.no_pack:
+            result["packed_storage"] = run_pack(args, f"cuda:{local_rank}")
         if world == 1 and not args.no_cpu_baseline:
             from paper_2411_10948_gb300 import workloads as W
             result["cpu_baseline"] = cpu_baseline(W.workload(args.workload), args.seed)

@@ -136,6 +136,42 @@ sq_status shiftquant_quantize(const float *x, int64_t rows, int64_t cols, int64_
                               uint64_t seed, int64_t row0, void *codes, int64_t ld_codes,
                               void *codes_t, int64_t ld_t, float *scale_out, void *stream);
 
+/* Group order of a GEMM inner index (Sec. 3.2's per-group GEMMs, done as one launch):
+ * from exp[channels] (the exponents of shiftquant_calibrate / shiftquant_group), a stable
+ * order with every group's channels contiguous and each group's segment starting on a
+ * K-block boundary (128 bytes of codes: 64 BF16 or 128 E4M3 codes).
+ *   pos_out[channels]: the position of each channel (int32, device);
+ *   seg_out[2 n_groups + 1]: the segment starts seg[0..n_groups] in elements (seg[n_groups]
+ *     = the padded width used) then the channel count of each group (int32, device).
+ * In this layout each group of the contraction accumulates without a shift and its exact
+ * sum is shifted once (shiftquant_gemm_layer with x_seg / g_seg): the per-chunk exact range
+ * is that of unshifted products, so 8-bit codes work with any n_groups <= 8. */
+sq_status shiftquant_group_order(const uint8_t *exp, int64_t channels, int bits, int n_groups,
+                                 int32_t *pos_out, int32_t *seg_out, void *stream);
+
+/* The largest padded width of a group order of `channels` channels (elements): the code
+ * buffers of a group-ordered operand need at least this leading dimension.  -1 for
+ * invalid arguments. */
+int64_t shiftquant_group_order_width(int64_t channels, int bits, int n_groups);
+
+/* shiftquant_quantize writing the codes of the GEMM inner index in a group order
+ * (pos, seg of shiftquant_group_order over that index), the padding between segments set to
+ * zero, and no folded shift (fold_exp is not taken):
+ *   SQ_GRAN_SHIFT   codes [rows, ld_codes]: column c at pos[c] (the channels are the inner
+ *                   index of the forward / loss-propagation GEMM); codes_t unchanged
+ *   SQ_GRAN_PER_COL codes_t [cols, ld_t]: its column r (x's row) at pos[r] (W [K, N] in the
+ *                   forward role, ordered by X's channels k); codes unchanged
+ *   SQ_GRAN_PER_ROW codes [rows, ld_codes]: column n at pos[n] (W in the loss-propagation
+ *                   role, ordered by dY's channels n); codes_t unchanged
+ * The ordered output is required, with a leading dimension of at least
+ * shiftquant_group_order_width(); every other argument is shiftquant_quantize's. */
+sq_status shiftquant_quantize_ordered(const float *x, int64_t rows, int64_t cols, int64_t ld,
+                                      int gran, int bits, int n_groups, const float *range_or_tau0,
+                                      const uint8_t *exp, int mode, uint64_t seed, int64_t row0,
+                                      const int32_t *pos, const int32_t *seg, void *codes,
+                                      int64_t ld_codes, void *codes_t, int64_t ld_t,
+                                      float *scale_out, void *stream);
+
 /* Forward GEMM Y[M, N] = X[M, K] W[K, N] on quantized operands (Eq. 4 with the roles of
  * Sec. 5.1):
  *   a_codes [M, lda]: ShiftQuant codes of X (SQ_GRAN_SHIFT, unshifted), a_scale: device
@@ -271,6 +307,16 @@ typedef struct {
    * range pass. */
   float *y_range;
   float *dx_range;
+  /* Optional (NULL: the folded layout above): the group order of the forward GEMM's inner
+   * index (X's channels, x_seg) and of the loss-propagation GEMM's (dY's channels, g_seg):
+   * the seg tables of shiftquant_group_order.  With x_seg, x_codes [M, ld_x] and wf_codes
+   * [N, ld_wf] hold their K channels in that order over the padded width
+   * shiftquant_group_order_width(K, bits, n_groups) (ld_x, ld_wf at least that), as
+   * shiftquant_quantize_ordered writes them, and wf_codes carry NO folded shifts; each
+   * group accumulates unshifted and its exact sum is shifted once.  g_seg likewise for
+   * g_codes [M, ld_g] and wd_codes [K, ld_wd] over dY's N channels. */
+  const int32_t *x_seg;
+  const int32_t *g_seg;
 } sq_layer_gemms;
 
 /* workspace: optional int32 scratch of shiftquant_gemm_layer_workspace_bytes() bytes,
@@ -283,9 +329,14 @@ sq_status shiftquant_gemm_layer(const sq_layer_gemms *args, void *workspace,
                                 size_t workspace_bytes, int32_t *dev_status, void *stream);
 
 /* Bytes of workspace that let shiftquant_gemm_layer schedule its units dynamically and
- * split every GEMM that would benefit on the current device (at least 256). */
+ * split every GEMM that would benefit on the current device (at least 256), and hold the
+ * int64 sums of a GEMM past the int32 range.  The _grouped form sizes a launch whose
+ * forward and loss-propagation inner indices are both group-ordered (x_seg and g_seg;
+ * K and N are the channel counts). */
 size_t shiftquant_gemm_layer_workspace_bytes(int64_t M, int64_t K, int64_t N, int bits,
                                              int n_groups);
+size_t shiftquant_gemm_layer_workspace_bytes_grouped(int64_t M, int64_t K, int64_t N, int bits,
+                                                     int n_groups);
 
 /* Number of kernels one shiftquant_gemm_layer call with this shape, workspace size and
  * gemm_mask launches on the current device: the GEMM launch, plus one output pass per GEMM
@@ -433,6 +484,34 @@ sq_status shiftquant_l1bn_backward(const float *dy, int64_t rows, int64_t channe
                                    void *state, size_t state_bytes, float *dx, int64_t ld_dx,
                                    float *dgamma, float *dbeta, int32_t *dev_status,
                                    void *stream);
+
+/* Packed sub-byte storage (Sec. 5.2: with N_G = 4 the grouping map takes exactly 2 bits).
+ * The tensor cores read codes as E4M3 / BF16 (there is no integer MMA on sm_103a, and the
+ * 4-bit float E2M1 lacks the integers 5 and 7), so the packed form is the storage of a
+ * quantized tensor between its quantization and its use -- for instance the activation
+ * codes kept for the backward pass, at half the bytes -- expanded before the GEMM.
+ * shiftquant_pack_codes: codes [rows, ld] of bits <= 4 (the library's storage type for
+ *   bits / n_groups; unshifted ShiftQuant codes, |q| <= 7) -> packed [rows, ld_packed]
+ *   bytes, ld_packed >= ceil(cols / 2): element c of a row in byte c / 2, the low nibble
+ *   for even c, as a 4-bit two's complement; an odd row's last high nibble is 0.  A code
+ *   outside [-8, 7] (a shifted weight code) sets SQ_DEV_INTERNAL.
+ * shiftquant_unpack_codes: the inverse, into codes [rows, ld] of the storage type. */
+sq_status shiftquant_pack_codes(const void *codes, int64_t rows, int64_t cols, int64_t ld,
+                                int bits, int n_groups, uint8_t *packed, int64_t ld_packed,
+                                int32_t *dev_status, void *stream);
+sq_status shiftquant_unpack_codes(const uint8_t *packed, int64_t ld_packed, int64_t rows,
+                                  int64_t cols, int bits, int n_groups, void *codes, int64_t ld,
+                                  void *stream);
+
+/* The grouping map (each channel's exponent) in w-bit fields, w = 1, 2 or 4 for n_groups
+ * <= 2, <= 4, <= 8 (2 bits at the default N_G = 4): channel c at bit (c mod (8 / w)) w of byte
+ * c / (8 / w).  shiftquant_packed_groups_bytes gives the packed size (-1 for bad
+ * arguments). */
+int64_t shiftquant_packed_groups_bytes(int64_t channels, int n_groups);
+sq_status shiftquant_pack_groups(const uint8_t *exp, int64_t channels, int n_groups,
+                                 uint8_t *packed, void *stream);
+sq_status shiftquant_unpack_groups(const uint8_t *packed, int64_t channels, int n_groups,
+                                   uint8_t *exp, void *stream);
 
 /* Failure-path self-test (for tests of the device-side timeout; the paper has no
  * counterpart).  One GEMM launch with the operands and layout of shiftquant_gemm_fwd whose

@@ -16,7 +16,7 @@ HERE = os.path.dirname(os.path.abspath(__file__))
 CSRC = os.path.join(HERE, "csrc")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libshiftquant.so")
-SOURCES = ["sq_quant.cu", "sq_gemm.cu", "sq_step.cu", "sq_l1bn.cu"]
+SOURCES = ["sq_quant.cu", "sq_gemm.cu", "sq_step.cu", "sq_l1bn.cu", "sq_pack.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 COMMON = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", "-Xcompiler", "-O2",
           "--expt-relaxed-constexpr"]

@@ -75,6 +75,8 @@ constexpr int64_t kExactSum = int64_t(1) << 24;  // every partial sum of a chunk
 // tables, the barriers and the unit ring.
 constexpr int kOutBox = 32;
 constexpr int kUnitRing = 8;  // work units published by the producer ahead of the consumers
+constexpr int kMaxSegGemms = 3;  // a launch holds at most three GEMMs
+constexpr int kSegSlots = 12;    // segment starts of up to 8 groups (9 used)
 constexpr int kOutStageBytes = kOutBox * kOutBox * 4;
 
 template <bool kPair>
@@ -90,7 +92,9 @@ struct Smem {
   static constexpr int num_bars = 2 * stages + 2 + 2 + 2 + 1 + 2 * kUnitRing + 2 + 1;
   static constexpr int ring_offset = bar_offset + num_bars * 8 + 16;  // after TMEM slot, flag
   static constexpr int chunk_offset = ring_offset + kUnitRing * 32;  // K blocks per chunk, per GEMM
-  static constexpr size_t bytes = chunk_offset + 4 * 4;
+  // group-ordered GEMMs: segment starts in K blocks (G + 1 of them), per GEMM
+  static constexpr int seg_offset = chunk_offset + 4 * 4;
+  static constexpr size_t bytes = seg_offset + kMaxSegGemms * kSegSlots * 4;
   static_assert(bytes <= 232448, "shared memory beyond the 227 KB per-CTA limit");
   static_assert(ring_offset % 16 == 0, "unit-ring slots are read as 16-byte vectors");
   static_assert(out_offset % 1024 == 0 && kOutStageBytes % 1024 == 0, "swizzle atoms need 1 KB");
@@ -141,6 +145,12 @@ struct GemmBatch {
   // failure-path self-test: the producer arms every stage but issues no copy, so the first
   // consumer wait runs out (nothing is ever in flight) and the launch takes its abort path
   int no_copies;
+  // per GEMM: the group order of its inner index (segment starts in elements, then the
+  // channel counts; a device table), or null.  A group-ordered GEMM's operands hold each
+  // group's inner channels contiguously and unshifted; its chunks end at segment boundaries
+  // and each chunk's sum is multiplied by the segment's shift 2^(G-1-g) in the epilogue.
+  const int* seg[kMaxBatch];
+  int segmented;  // some GEMM is group-ordered (every role waits for the table)
 };
 
 __device__ __forceinline__ float pow2_neg(int k) { return __int_as_float((127 - k) << 23); }
@@ -426,6 +436,24 @@ __device__ __forceinline__ void leader_arrive(uint64_t* local_bar, uint32_t clus
     mbar_arrive(local_bar);
 }
 
+// The chunk that starts at K block kc of a unit whose K loop ends at kend: its end and its
+// shift exponent.  Without a segment table chunks are chunk_kb blocks; with one (segkb =
+// the G + 1 segment starts in K blocks) a chunk also ends at its segment's end and carries
+// the segment's shift G-1-g.  The producer, the MMA issuer and the epilogue walk the same
+// sequence.
+__device__ __forceinline__ int chunk_end(const volatile int* segkb, int G, int kc, int kend,
+                                         int chunk_kb, int* shift) {
+  int e = min(kend, kc + chunk_kb);
+  *shift = 0;
+  if (segkb != nullptr) {
+    int s = 0;
+    while (s + 1 < G && kc >= segkb[s + 1]) ++s;
+    *shift = G - 1 - s;
+    e = min(e, segkb[s + 1]);
+  }
+  return e;
+}
+
 // The factor warp: the dequantizing factor of each of a tile's 256 columns, into one of
 // two tables ahead of the epilogue: s_A 2^-(G-1) s_B[n] (forward, loss propagation) or
 // s_X s_dY 2^-eY_n (weight gradient; the row's 2^-eX_m is the epilogue's).  It reads the
@@ -651,6 +679,7 @@ __global__ void __launch_bounds__(kThreads, 1) shiftmm_kernel(const __grid_const
     int next = pair;  // a pair's first unit is its own index
     int us = 0;
     uint32_t uph = 0;
+    if (bt.segmented && !mbar_wait(chunkbar, 0, abort_flag)) ok = false;  // the segment table
     while (ok) {
       int u = next;
       RingUnit r;
@@ -703,7 +732,11 @@ __global__ void __launch_bounds__(kThreads, 1) shiftmm_kernel(const __grid_const
       // rows past M (and columns past N) are read as zeros and never stored
       const int32_t ya = w.mb * L::tile_m + static_cast<int32_t>(rank) * kBM;
       const int32_t yb = w.nb * kBN + static_cast<int32_t>(rank) * L::b_rows;
-      for (int kb = w.kb0; kb < w.kb1; ++kb) {
+      // a group-ordered GEMM's K loop stops at its padded width (the segment table's end)
+      const int kend = bt.seg[g] != nullptr
+                           ? min(w.kb1, reinterpret_cast<volatile int*>(smem + L::seg_offset)[g * kSegSlots + bt.p[g].G])
+                           : w.kb1;
+      for (int kb = w.kb0; kb < kend; ++kb) {
         if (!mbar_wait(&empty[s], ph ^ 1u, abort_flag)) {
           ok = false;
           break;
@@ -776,8 +809,13 @@ __global__ void __launch_bounds__(kThreads, 1) shiftmm_kernel(const __grid_const
       const int chunk_kb =
           bt.planned ? reinterpret_cast<volatile int*>(smem + L::chunk_offset)[g] : bt.p[g].chunk_kb;
       const Unit w = r.w;
-      for (int kc = w.kb0; kc < w.kb1 && ok; kc += chunk_kb) {
-        const int kce = min(w.kb1, kc + chunk_kb);
+      const volatile int* segkb =
+          bt.seg[g] != nullptr ? reinterpret_cast<volatile int*>(smem + L::seg_offset) + g * kSegSlots : nullptr;
+      const int kend = segkb != nullptr ? min(w.kb1, segkb[bt.p[g].G]) : w.kb1;
+      int kce;
+      for (int kc = w.kb0; kc < kend && ok; kc = kce) {
+        int sh_unused;
+        kce = chunk_end(segkb, bt.p[g].G, kc, kend, chunk_kb, &sh_unused);
         const uint32_t b = c & 1u, tph = (c >> 1) & 1u;
         if (!ring_wait<kPair>(&tempty[b], tph ^ 1u, abort_flag)) {  // every CTA's epilogue
           ok = false;
@@ -825,6 +863,10 @@ __global__ void __launch_bounds__(kThreads, 1) shiftmm_kernel(const __grid_const
     // --------------------------------------------------- chunk plan, column factors
     if (bt.planned) {
       plan_chunks(bt, reinterpret_cast<volatile int*>(smem + L::chunk_offset), lane, kBKElems);
+      volatile int* segkb = reinterpret_cast<volatile int*>(smem + L::seg_offset);
+      for (int g = 0; g < bt.count; ++g)
+        if (bt.seg[g] != nullptr && lane <= bt.p[g].G)
+          segkb[g * kSegSlots + lane] = __ldg(bt.seg[g] + lane) / kBKElems;
       __syncwarp();
       if (lane == 0) mbar_arrive(chunkbar);
     }
@@ -861,7 +903,9 @@ __global__ void __launch_bounds__(kThreads, 1) shiftmm_kernel(const __grid_const
       const Unit w = r.w;
       const int ckb =
           bt.planned ? reinterpret_cast<volatile int*>(smem + L::chunk_offset)[g] : p.chunk_kb;
-      const int nch = (w.kb1 - w.kb0 + ckb - 1) / ckb;
+      const volatile int* segkb =
+          bt.seg[g] != nullptr ? reinterpret_cast<volatile int*>(smem + L::seg_offset) + g * kSegSlots : nullptr;
+      const int kend = segkb != nullptr ? min(w.kb1, segkb[p.G]) : w.kb1;
       const int64_t m0 = static_cast<int64_t>(w.mb) * L::tile_m + rank * kBM;  // this CTA's rows
       const int64_t n0 = static_cast<int64_t>(w.nb) * kBN;
       float* fac = fac_tab + (it & 1) * kBN;
@@ -900,7 +944,16 @@ __global__ void __launch_bounds__(kThreads, 1) shiftmm_kernel(const __grid_const
         ++c;
       } else {
         uint32_t acc[128];  // int32 sums of the chunks
-        for (int ch = 0; ch < nch; ++ch) {
+        if (kend <= w.kb0) {
+          // a split of a group-ordered GEMM that lies past its padded width: no chunk
+#pragma unroll
+          for (int i = 0; i < 128; ++i) acc[i] = 0u;
+        }
+        int kce;
+        for (int kc = w.kb0, ch = 0; kc < kend; kc = kce, ++ch) {
+          int sh;
+          kce = chunk_end(segkb, p.G, kc, kend, ckb, &sh);
+          const int32_t mul = 1 << sh;  // the segment's shift (1 without a segment table)
           const uint32_t b = c & 1u, tph = (c >> 1) & 1u;
           if (!__all_sync(0xFFFFFFFFu, mbar_wait(&tfull[b], tph, abort_flag))) {
             ok = false;
@@ -925,14 +978,14 @@ __global__ void __launch_bounds__(kThreads, 1) shiftmm_kernel(const __grid_const
 #pragma unroll
               for (int i = 0; i < 16; ++i) {
                 const int32_t t =
-                    __float_as_int(__fadd_rn(__uint_as_float(v[i]), 12582912.0f)) - 0x4B400000;
+                    (__float_as_int(__fadd_rn(__uint_as_float(v[i]), 12582912.0f)) - 0x4B400000) * mul;
                 acc[j * 16 + i] =
                     static_cast<uint32_t>(ch == 0 ? t : static_cast<int32_t>(acc[j * 16 + i]) + t);
               }
             } else {
 #pragma unroll
               for (int i = 0; i < 16; ++i) {
-                const int32_t t = __float2int_rn(__uint_as_float(v[i]));
+                const int32_t t = __float2int_rn(__uint_as_float(v[i])) * mul;
                 acc[j * 16 + i] =
                     static_cast<uint32_t>(ch == 0 ? t : static_cast<int32_t>(acc[j * 16 + i]) + t);
               }
@@ -1118,19 +1171,23 @@ struct Plan {
   int wide;  // max|T| can pass 2^31: every split stays within int32, splits add in int64
 };
 
-// max |product| of one inner index: q_A q_B 2^(G-1) with the shift folded into B
-// (forward, loss propagation) or q_A q_B with the shifts applied after the sum (wgrad)
-static int64_t max_product(int which, int bits, int G) {
+// max |product| of one inner index as the tensor core sees it: q_A q_B 2^(G-1) with the
+// shift folded into B (forward, loss propagation), or q_A q_B with the shifts applied
+// after the sum (the weight gradient; a group-ordered GEMM, whose chunks are shifted whole)
+static int64_t max_product(int which, int bits, int G, bool seg = false) {
   const int64_t Q = q_of_bits(bits);
-  return (which == 2) ? Q * Q : (Q * Q) << (G - 1);
+  return (which == 2 || seg) ? Q * Q : (Q * Q) << (G - 1);
 }
+
+// max |T| per inner index: the shifted product, however the shift is applied
+static int64_t max_total_product(int which, int bits, int G) { return max_product(which, bits, G); }
 
 // The exactness limit of the FP32 accumulation, checked before anything touches the device:
 // one K block of worst-case products must stay within 2^24 (the chunks are whole K blocks).
 // K itself is not limited: past the int32 range the K loop is split (see make_plan).
-static int check_exact_range(int which, int64_t K, int bits, int G) {
+static int check_exact_range(int which, int64_t K, int bits, int G, bool seg = false) {
   (void)K;
-  const int64_t P = max_product(which, bits, G);
+  const int64_t P = max_product(which, bits, G, seg);
   const int bk = kBKBytes / code_bytes(code_type(bits, G));
   if (kExactSum / P < bk)
     return fail(SQ_EUNSUPPORTED,
@@ -1154,10 +1211,10 @@ static int check_int32_range(int which, int64_t K, int bits, int G) {
 // Tiles of 128 (pair: 256) x 256 outputs spread over `workers` (SMs, or CTA pairs).
 // max_splits: 1 never splits K; 0 lets the worker count alone decide.
 static int make_plan(int which, int64_t M, int64_t N, int64_t K, int bits, int G, int workers,
-                     int max_splits, bool pair, Plan* pl) {
-  const int st = check_exact_range(which, K, bits, G);
+                     int max_splits, bool pair, Plan* pl, bool seg = false) {
+  const int st = check_exact_range(which, K, bits, G, seg);
   if (st != SQ_OK) return st;
-  const int64_t P = max_product(which, bits, G);
+  const int64_t P = max_product(which, bits, G, seg);
   pl->elem_bytes = code_bytes(code_type(bits, G));
   const int bk = kBKBytes / pl->elem_bytes;
   pl->chunk_kb = static_cast<int>((kExactSum / P) / bk);
@@ -1176,7 +1233,7 @@ static int make_plan(int which, int64_t M, int64_t N, int64_t K, int bits, int G
   }
   // Past the int32 range every split keeps its K loop within it (its int32 register sums
   // stay exact) and the splits add in int64: at least this many, whatever max_splits says.
-  const int64_t kb_int32 = (INT32_MAX / P) / bk;  // >= 1: one K block stays within 2^24
+  const int64_t kb_int32 = (INT32_MAX / max_total_product(which, bits, G)) / bk;  // >= 1
   pl->wide = pl->kb_total > kb_int32 ? 1 : 0;
   if (pl->wide) {
     const int need = static_cast<int>((pl->kb_total + kb_int32 - 1) / kb_int32);
@@ -1263,6 +1320,7 @@ struct GemmJob {
   const uint8_t* k_exp;  // exponents of the inner channels (forward, loss propagation), or null
   int partial;  // weight gradient: int32 sums into ws (the caller's), no dequantizing pass
   float* colmax;  // per-column max |output| [N], formed by the epilogue, or null
+  const int* seg;  // group order of the inner index (device table), or null
 };
 
 static const char* job_name(int which) {
@@ -1309,7 +1367,7 @@ static int check_job(const GemmJob& j, int bits, int G, int32_t* dev_status, cud
   if (!aligned16(j.a) || !aligned16(j.b) || (j.lda * eb) % 16 != 0 || (j.ldb * eb) % 16 != 0)
     return fail(SQ_EALIGN, "%s: operand pointers must be 16-byte aligned and ld * %d bytes a "
                 "multiple of 16", nm, eb);
-  const int st = check_exact_range(j.which, j.K, bits, G);
+  const int st = check_exact_range(j.which, j.K, bits, G, j.seg != nullptr);
   if (st != SQ_OK) return st;
   *launch = true;
   return SQ_OK;
@@ -1320,7 +1378,8 @@ static int check_job(const GemmJob& j, int bits, int G, int32_t* dev_status, cud
 // into N-element rows, which must stay 16-byte aligned).
 static int plan_job(const GemmJob& j, int bits, int G, int workers, int max_splits, bool pair,
                     Plan* pl) {
-  const int st = make_plan(j.which, j.M, j.N, j.K, bits, G, workers, max_splits, pair, pl);
+  const bool sg = j.seg != nullptr;
+  const int st = make_plan(j.which, j.M, j.N, j.K, bits, G, workers, max_splits, pair, pl, sg);
   if (st != SQ_OK || pl->splits <= 1 || j.partial) return st;  // partial: ws is the output
   if (pl->wide) {
     // int64 sums need their workspace; there is no unsplit way to stay exact
@@ -1334,7 +1393,7 @@ static int plan_job(const GemmJob& j, int bits, int G, int workers, int max_spli
     return SQ_OK;
   }
   if (j.ws == nullptr || j.ws_bytes < split_ws_bytes(j.M, j.N) || !aligned16(j.ws) || j.N % 4 != 0)
-    return make_plan(j.which, j.M, j.N, j.K, bits, G, workers, 1, pair, pl);
+    return make_plan(j.which, j.M, j.N, j.K, bits, G, workers, 1, pair, pl, sg);
   return SQ_OK;
 }
 
@@ -1351,7 +1410,8 @@ static bool pair_mode(const GemmJob* const* jobs, int n, int bits, int G, int sm
     const GemmJob& j = *jobs[i];
     if (j.M <= 0 || j.N <= 0 || j.K <= 0) continue;
     Plan pl;
-    if (make_plan(j.which, j.M, j.N, j.K, bits, G, sms, 0, false, &pl) != SQ_OK) continue;
+    if (make_plan(j.which, j.M, j.N, j.K, bits, G, sms, 0, false, &pl, j.seg != nullptr) != SQ_OK)
+      continue;
     const double u = static_cast<double>(pl.m_tiles) * pl.n_tiles * pl.splits;
     units += u;
     kb += u * pl.kb_per_split;
@@ -1409,7 +1469,10 @@ static int prepare_job(const GemmJob& j, const Plan* pl, int bits, int G, int32_
   p.chunk_kb = pl->chunk_kb;
   // exponent-sized chunks pay where worst-case chunks would split a unit three ways or more
   // (8-bit); elsewhere the planning only costs time
-  bt->k_exp[g] = (j.which == 2 || pl->kb_per_split <= 2 * pl->chunk_kb) ? nullptr : j.k_exp;
+  bt->k_exp[g] = (j.which == 2 || j.seg != nullptr || pl->kb_per_split <= 2 * pl->chunk_kb)
+                    ? nullptr
+                    : j.k_exp;
+  bt->seg[g] = j.seg;
   bt->raw_prod[g] = q_of_bits(bits) * q_of_bits(bits);
   p.mode = j.which == 2 ? 1 : 0;
   p.G = G;
@@ -1531,6 +1594,7 @@ static int run_jobs(GemmJob* jobs, int njobs, int bits, int G, int32_t* dev_stat
         t = bt.y[a]; bt.y[a] = bt.y[b]; bt.y[b] = t;
         t = bt.ws[a]; bt.ws[a] = bt.ws[b]; bt.ws[b] = t;
         const uint8_t* te = bt.k_exp[a]; bt.k_exp[a] = bt.k_exp[b]; bt.k_exp[b] = te;
+        const int* ts = bt.seg[a]; bt.seg[a] = bt.seg[b]; bt.seg[b] = ts;
         const int tr = bt.raw_prod[a]; bt.raw_prod[a] = bt.raw_prod[b]; bt.raw_prod[b] = tr;
       }
   int units = 0;
@@ -1539,13 +1603,18 @@ static int run_jobs(GemmJob* jobs, int njobs, int bits, int G, int32_t* dev_stat
     units += plans[g].m_tiles * plans[g].n_tiles * plans[g].splits;
     bt.unit_end[g] = units;
     multi |= plans[g].kb_per_split > plans[g].chunk_kb;  // a unit spans several exact chunks
+    multi |= bt.seg[g] != nullptr;  // chunks end at segment boundaries and carry their shifts
   }
   bt.count = nlive;
   bt.status = dev_status;
   bt.sched = sched;
   bt.no_copies = no_copies ? 1 : 0;
   bt.planned = 0;
-  for (int g = 0; g < nlive; ++g) bt.planned |= bt.k_exp[g] != nullptr;
+  bt.segmented = 0;
+  for (int g = 0; g < nlive; ++g) {
+    bt.planned |= bt.k_exp[g] != nullptr || bt.seg[g] != nullptr;
+    bt.segmented |= bt.seg[g] != nullptr;
+  }
   // zero the counter and the partial sums, with one memset for the regions that follow the
   // counter back to back
   char* zero_from = reinterpret_cast<char*>(sched);
@@ -1624,6 +1693,15 @@ static void layer_jobs(const sq_layer_gemms* a, GemmJob jobs[3], int mask) {
   jobs[1].k_exp = a->g_exp;  // loss propagation's are dY's
   jobs[0].colmax = a->y_range;
   jobs[1].colmax = a->dx_range;
+  // group-ordered inner indices: the operands span the padded width of the order
+  if (a->x_seg != nullptr) {
+    jobs[0].seg = a->x_seg;
+    jobs[0].K = shiftquant_group_order_width(a->K, a->bits, a->n_groups);
+  }
+  if (a->g_seg != nullptr) {
+    jobs[1].seg = a->g_seg;
+    jobs[1].K = shiftquant_group_order_width(a->N, a->bits, a->n_groups);
+  }
   // a GEMM left out of the mask becomes empty: nothing of it is checked or launched
   for (int i = 0; i < 3; ++i)
     if (mask != 0 && !(mask & (1 << i))) jobs[i].M = 0;
@@ -1640,7 +1718,8 @@ static void layer_ws_need(const GemmJob jobs[3], int bits, int G, int sms, int p
     const GemmJob& j = jobs[i];
     if (j.M <= 0 || j.N <= 0 || j.K <= 0) continue;
     Plan pl;
-    if (make_plan(j.which, j.M, j.N, j.K, bits, G, pair ? pairs : sms, 0, pair, &pl) != SQ_OK)
+    if (make_plan(j.which, j.M, j.N, j.K, bits, G, pair ? pairs : sms, 0, pair, &pl,
+                  j.seg != nullptr) != SQ_OK)
       continue;
     if (!pl.wide && j.N % 4 != 0) continue;  // int32 splits are added by 16-byte TMA rows
     if (pl.splits > 1) need[i] = split_ws_bytes(j.M, j.N, pl.wide != 0);
@@ -1893,8 +1972,8 @@ extern "C" sq_status shiftquant_selftest_wait_timeout(const void* a_codes, int64
   return run_jobs(&j, 1, bits, n_groups, dev_status, stream, nullptr, 0, true);
 }
 
-extern "C" size_t shiftquant_gemm_layer_workspace_bytes(int64_t M, int64_t K, int64_t N, int bits,
-                                                        int n_groups) {
+static size_t layer_workspace_bytes(int64_t M, int64_t K, int64_t N, int bits, int n_groups,
+                                    bool grouped) {
   if (!bits_ok(bits) || !groups_ok(n_groups)) return 0;
   const int sms = device_sms(nullptr);
   if (sms <= 0) return 0;
@@ -1904,11 +1983,27 @@ extern "C" size_t shiftquant_gemm_layer_workspace_bytes(int64_t M, int64_t K, in
   a.M = M;
   a.K = K;
   a.N = N;
+  a.bits = bits;
+  a.n_groups = n_groups;
+  if (grouped) {  // the plan reads only whether a table exists: a stand-in address serves
+    a.x_seg = reinterpret_cast<const int32_t*>(static_cast<uintptr_t>(256));
+    a.g_seg = a.x_seg;
+  }
   GemmJob jobs[3];
   layer_jobs(&a, jobs, 0);
   size_t need[3];
   layer_ws_need(jobs, bits, n_groups, sms, pairs, need);
   return kSchedBytes + need[0] + need[1] + need[2];
+}
+
+extern "C" size_t shiftquant_gemm_layer_workspace_bytes(int64_t M, int64_t K, int64_t N, int bits,
+                                                        int n_groups) {
+  return layer_workspace_bytes(M, K, N, bits, n_groups, false);
+}
+
+extern "C" size_t shiftquant_gemm_layer_workspace_bytes_grouped(int64_t M, int64_t K, int64_t N,
+                                                                int bits, int n_groups) {
+  return layer_workspace_bytes(M, K, N, bits, n_groups, true);
 }
 
 extern "C" int shiftquant_gemm_layer_kernel_launches(int64_t M, int64_t K, int64_t N, int bits,

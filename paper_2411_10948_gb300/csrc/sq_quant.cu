@@ -37,6 +37,11 @@ int fail(int status, const char* fmt, ...) {
 
 static void clear_error() { g_last_error[0] = 0; }
 
+// the group order a shiftquant_quantize_ordered call hands to the quantizer launch it makes
+// (per host thread; null outside such a call)
+static thread_local const int* g_order_cols = nullptr;
+static thread_local const int* g_order_rows = nullptr;
+
 // ===================================================================== range pass
 constexpr int kColTx = 32;  // threads along columns, 4 columns each: 128 columns per block
 constexpr int kColTy = 8;   // threads along rows
@@ -260,6 +265,10 @@ struct QuantArgs {
   int64_t ldt;
   float* scale_out;
   int vec_in, vec_out, vec_t;
+  // group order of the GEMM inner index (or null): codes column c goes to pos_cols[c]
+  // (ShiftQuant and per-row grans), codes_t column r to pos_rows[r] (per-column gran)
+  const int* pos_cols;
+  const int* pos_rows;
 };
 
 
@@ -420,7 +429,12 @@ __device__ __forceinline__ void quantize_tile(const QuantArgs& a, uint8_t* tile_
       out[j] = encode_code<CodeT>(__fadd_rn(q, 0.0f));  // +0 for a zero code
       packed[j][i / kPerWord] |= static_cast<uint32_t>(out[j]) << (8 * sizeof(CodeT) * (i % kPerWord));
     }
-    if (a.codes && row_in) {
+    if (a.codes && row_in && a.pos_cols != nullptr) {
+      CodeT* dst = static_cast<CodeT*>(a.codes) + r * a.ldc;
+#pragma unroll
+      for (int j = 0; j < 4; ++j)
+        if (FULL || cb + j < a.C) dst[__ldg(a.pos_cols + cb + j)] = out[j];
+    } else if (a.codes && row_in) {
       CodeT* dst = static_cast<CodeT*>(a.codes) + r * a.ldc + cb;
       if (FULL || (a.vec_out && cb + 3 < a.C)) {
         if constexpr (sizeof(CodeT) == 2) {
@@ -455,6 +469,19 @@ __device__ __forceinline__ void quantize_tile(const QuantArgs& a, uint8_t* tile_
                      "r"(packed[j][1]) : "memory");
     }
     __syncthreads();
+    if (a.pos_rows != nullptr) {
+      // group-ordered transposed copy: element (column c, row r) goes to pos_rows[r]
+      CodeT* ctp = static_cast<CodeT*>(a.codes_t);
+      for (int idx = tid; idx < kQC * kQR; idx += 256) {
+        const int lc = idx / kQR, rr = idx % kQR;
+        const int64_t c = c0 + lc, r = r0 + rr;
+        if (!FULL && (c >= a.C || r >= a.R)) continue;
+        const CodeT v = reinterpret_cast<const CodeT*>(tile_t + chunk_slot(lc, rr >> 3) * kChunkBytes)[rr & 7];
+        ctp[c * a.ldt + __ldg(a.pos_rows + r)] = v;
+      }
+      goto scales;
+    }
+    {
     // each transposed row (one tile column) holds 64 codes = 8 chunks; 16-byte stores
     constexpr int kChunksPerStore = 16 / kChunkBytes;            // 1 (BF16) or 2 (E4M3)
     constexpr int kStoresPerRow = 8 / kChunksPerStore;
@@ -484,8 +511,9 @@ __device__ __forceinline__ void quantize_tile(const QuantArgs& a, uint8_t* tile_
             dst[e * sizeof(CodeT) + b] = vb[e * sizeof(CodeT) + b];
       }
     }
+    }
   }
-
+scales:
   // scales: s = tau_0 / Q, or range / Q per channel (0 for an all-zero channel)
   if (GRAN == SQ_GRAN_SHIFT) {
     if (blockIdx.x == 0 && blockIdx.y == 0 && tid == 0) {
@@ -572,6 +600,93 @@ static void launch_quantize(const QuantArgs& a, dim3 grid, cudaStream_t s) {
     } else {
       if (fold) launch_pdl(quantize_kernel<CodeT, SQ_GRAN_PER_ROW, SQ_ROUND_STOCHASTIC, true>, grid, dim3(256), s, a);
       else launch_pdl(quantize_kernel<CodeT, SQ_GRAN_PER_ROW, SQ_ROUND_STOCHASTIC, false>, grid, dim3(256), s, a);
+    }
+  }
+}
+
+// ============================================================ group order (Sec. 3.2)
+// The inner index of a forward or loss-propagation GEMM in group order: every group's
+// channels contiguous (stable: in channel order within a group), each group's segment
+// starting on a K-block boundary (bk elements), so that the contraction can accumulate a
+// group unshifted and apply its shift once per segment.  seg[0..G] = segment starts (seg[G]
+// = the padded width), seg[G+1..2G] = channels per group; pos[c] = the position of channel
+// c.  One block: counts per group, then stable ranks chunk by chunk with warp ballots.
+constexpr int kOrderThreads = 1024;
+
+__global__ void __launch_bounds__(kOrderThreads)
+    group_order_kernel(const uint8_t* __restrict__ exp, int64_t C, int G, int bk,
+                       int* __restrict__ pos, int* __restrict__ seg) {
+  __shared__ int cnt[8];
+  __shared__ int start[9];
+  __shared__ int base[8];
+  __shared__ int wtot[kOrderThreads / 32][8];
+  const int tid = threadIdx.x, lane = tid & 31, w = tid >> 5;
+  if (tid < 8) cnt[tid] = 0;
+  __syncthreads();
+  int mine[8] = {0, 0, 0, 0, 0, 0, 0, 0};
+  for (int64_t c = tid; c < C; c += kOrderThreads) {
+    const int e = min(static_cast<int>(exp[c]), G - 1);
+#pragma unroll
+    for (int g = 0; g < 8; ++g) mine[g] += (e == g);
+  }
+#pragma unroll
+  for (int g = 0; g < 8; ++g) {
+    const int v = __reduce_add_sync(0xFFFFFFFFu, mine[g]);
+    if (lane == 0 && v) atomicAdd(&cnt[g], v);
+  }
+  __syncthreads();
+  if (tid == 0) {
+    int o = 0;
+    for (int g = 0; g < G; ++g) {
+      start[g] = o;
+      o += (cnt[g] + bk - 1) / bk * bk;
+      base[g] = 0;
+    }
+    start[G] = o;
+    for (int g = 0; g <= G; ++g) seg[g] = start[g];
+    for (int g = 0; g < G; ++g) seg[G + 1 + g] = cnt[g];
+  }
+  __syncthreads();
+  for (int64_t c0 = 0; c0 < C; c0 += kOrderThreads) {
+    const int64_t c = c0 + tid;
+    const int e = c < C ? min(static_cast<int>(exp[c]), G - 1) : -1;
+    const unsigned below = (1u << lane) - 1u;
+    int rank = 0;
+#pragma unroll
+    for (int g = 0; g < 8; ++g) {
+      const unsigned b = __ballot_sync(0xFFFFFFFFu, e == g);
+      if (e == g) rank = __popc(b & below);
+      if (lane == 0) wtot[w][g] = __popc(b);
+    }
+    __syncthreads();
+    if (e >= 0) {
+      int before = 0;
+      for (int k = 0; k < w; ++k) before += wtot[k][e];
+      pos[c] = start[e] + base[e] + before + rank;
+    }
+    __syncthreads();
+    if (tid < G) {
+      int t = 0;
+      for (int k = 0; k < kOrderThreads / 32; ++k) t += wtot[k][tid];
+      base[tid] += t;
+    }
+    __syncthreads();
+  }
+}
+
+// zero the padding positions of a group-ordered code buffer [rows, ld]: the tail
+// [seg[g] + count_g, seg[g+1]) of every segment, one warp per row
+template <typename CodeT>
+__global__ void __launch_bounds__(256)
+    order_pad_kernel(CodeT* __restrict__ codes, int64_t rows, int64_t ld, const int* __restrict__ seg,
+                     int G) {
+  const int lane = threadIdx.x & 31;
+  for (int64_t r = (static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x) / 32; r < rows;
+       r += static_cast<int64_t>(gridDim.x) * blockDim.x / 32) {
+    CodeT* row = codes + r * ld;
+    for (int g = 0; g < G; ++g) {
+      const int from = seg[g] + seg[G + 1 + g], to = seg[g + 1];
+      for (int i = from + lane; i < to; i += 32) row[i] = CodeT(0);
     }
   }
 }
@@ -762,6 +877,8 @@ extern "C" sq_status shiftquant_quantize(const float* x, int64_t rows, int64_t c
   a.vec_out = codes != nullptr && ((ld_codes * cbytes) % (4 * cbytes) == 0) &&
               (reinterpret_cast<uintptr_t>(codes) % (4 * cbytes) == 0);
   a.vec_t = codes_t != nullptr && ((ld_t * cbytes) % 16 == 0) && aligned16(codes_t);
+  a.pos_cols = g_order_cols;
+  a.pos_rows = g_order_rows;
   const int64_t gx = (cols + kQC - 1) / kQC, gy = (rows + kQR - 1) / kQR;
   if (gx > 0x7FFFFFFF || gy > 65535)
     return fail(SQ_EUNSUPPORTED, "quantize: tensor too large for one launch (%lld x %lld)",
@@ -773,4 +890,73 @@ extern "C" sq_status shiftquant_quantize(const float* x, int64_t rows, int64_t c
     launch_quantize<uint16_t>(a, grid, s);
   const cudaError_t err = cudaGetLastError();
   return err == cudaSuccess ? SQ_OK : cuda_fail(err, "quantize_kernel launch");
+}
+
+// ------------------------------------------------------------------ group order
+extern "C" int64_t shiftquant_group_order_width(int64_t channels, int bits, int n_groups) {
+  if (channels < 0 || !bits_ok(bits) || !groups_ok(n_groups)) return -1;
+  const int64_t bk = 128 / code_bytes(code_type(bits, n_groups));
+  return (channels + bk - 1) / bk * bk + (n_groups - 1) * bk;
+}
+
+extern "C" sq_status shiftquant_group_order(const uint8_t* exp, int64_t channels, int bits,
+                                            int n_groups, int32_t* pos_out, int32_t* seg_out,
+                                            void* stream) {
+  clear_error();
+  if (!bits_ok(bits) || !groups_ok(n_groups))
+    return fail(SQ_EINVAL, "group_order: bits must be in [2, 8] and n_groups in [1, 8]");
+  if (channels < 0 || channels > INT32_MAX / 2) return fail(SQ_EINVAL, "group_order: bad channel count");
+  if (seg_out == nullptr || (channels > 0 && (exp == nullptr || pos_out == nullptr)))
+    return fail(SQ_EINVAL, "group_order: exp, pos_out and seg_out are required");
+  const int bk = 128 / code_bytes(code_type(bits, n_groups));
+  group_order_kernel<<<1, kOrderThreads, 0, as_stream(stream)>>>(exp, channels, n_groups, bk,
+                                                                   pos_out, seg_out);
+  const cudaError_t err = cudaGetLastError();
+  return err == cudaSuccess ? SQ_OK : cuda_fail(err, "group_order_kernel launch");
+}
+
+extern "C" sq_status shiftquant_quantize_ordered(const float* x, int64_t rows, int64_t cols,
+                                                 int64_t ld, int gran, int bits, int n_groups,
+                                                 const float* range_or_tau0, const uint8_t* exp,
+                                                 int mode, uint64_t seed, int64_t row0,
+                                                 const int32_t* pos, const int32_t* seg,
+                                                 void* codes, int64_t ld_codes, void* codes_t,
+                                                 int64_t ld_t, float* scale_out, void* stream) {
+  clear_error();
+  if (pos == nullptr || seg == nullptr) return fail(SQ_EINVAL, "quantize_ordered: pos and seg are required");
+  if (!bits_ok(bits) || !groups_ok(n_groups))
+    return fail(SQ_EINVAL, "quantize_ordered: bits must be in [2, 8] and n_groups in [1, 8]");
+  // the ordered output: codes for ShiftQuant and per-row grans, codes_t for per-column
+  const bool on_t = gran == SQ_GRAN_PER_COL;
+  void* ordered = on_t ? codes_t : codes;
+  const int64_t ord_rows = on_t ? cols : rows;       // rows of the ordered buffer
+  const int64_t ord_ld = on_t ? ld_t : ld_codes;
+  const int64_t chans = on_t ? rows : cols;          // the ordered (inner) index
+  if (ordered == nullptr)
+    return fail(SQ_EINVAL, "quantize_ordered: the group-ordered output (%s) is required",
+                on_t ? "codes_t" : "codes");
+  const int64_t width = shiftquant_group_order_width(chans, bits, n_groups);
+  if (ord_ld < width)
+    return fail(SQ_EINVAL, "quantize_ordered: the ordered output needs a leading dimension of "
+                "at least %lld (shiftquant_group_order_width)", static_cast<long long>(width));
+  // the other output (if any) keeps the natural order; a leading dimension >= the natural
+  // width is checked by the plain quantizer below
+  g_order_cols = on_t ? nullptr : pos;
+  g_order_rows = on_t ? pos : nullptr;
+  const sq_status st = shiftquant_quantize(x, rows, cols, ld, gran, bits, n_groups, range_or_tau0,
+                                           exp, nullptr, mode, seed, row0, codes, ld_codes, codes_t,
+                                           ld_t, scale_out, stream);
+  g_order_cols = g_order_rows = nullptr;
+  if (st != SQ_OK || ord_rows == 0) return st;
+  cudaStream_t s = as_stream(stream);
+  int64_t blocks = (ord_rows + 7) / 8;
+  if (blocks > 4096) blocks = 4096;
+  if (code_type(bits, n_groups) == SQ_CODE_E4M3)
+    order_pad_kernel<uint8_t><<<static_cast<unsigned>(blocks), 256, 0, s>>>(
+        static_cast<uint8_t*>(ordered), ord_rows, ord_ld, seg, n_groups);
+  else
+    order_pad_kernel<uint16_t><<<static_cast<unsigned>(blocks), 256, 0, s>>>(
+        static_cast<uint16_t*>(ordered), ord_rows, ord_ld, seg, n_groups);
+  const cudaError_t err = cudaGetLastError();
+  return err == cudaSuccess ? SQ_OK : cuda_fail(err, "order_pad_kernel launch");
 }

@@ -100,8 +100,9 @@ class QuantLinear:
     """Buffers and calls of one quantized linear layer: X [M, K], W [K, N], dY [M, N]."""
 
     def __init__(self, M, K, N_, bits, n_groups, device="cuda", with_acc=False,
-                 use_workspace=True, with_inputs=False):
+                 use_workspace=True, with_inputs=False, grouped=False):
         self.M, self.K, self.N, self.bits, self.G = M, K, N_, bits, n_groups
+        self.grouped = grouped
         dev = torch.device(device)
         # device input buffers for shiftquant_layer_step(_host), when asked for
         self.inputs = None
@@ -112,10 +113,22 @@ class QuantLinear:
         self.status = torch.zeros(1, dtype=torch.int32, device=dev)
         self.x = ShiftTensor.alloc(M, K, bits, n_groups, dev)
         self.g = ShiftTensor.alloc(M, N_, bits, n_groups, dev)
-        self.wf = ChannelTensor(empty_codes(N_, K, bits, n_groups, dev),
+        # grouped: the forward and loss-propagation operands hold their inner index in group
+        # order (Sec. 3.2's per-group products as one launch) over the padded width
+        self.x_pos = self.x_seg = self.g_pos = self.g_seg = None
+        kw = N.shiftquant_group_order_width(K, bits, n_groups) if grouped else K
+        nw = N.shiftquant_group_order_width(N_, bits, n_groups) if grouped else N_
+        if grouped:
+            self.x.codes = empty_codes(M, kw, bits, n_groups, dev)
+            self.g.codes = empty_codes(M, nw, bits, n_groups, dev)
+            self.x_pos = torch.zeros(max(K, 1), dtype=torch.int32, device=dev)[:K]
+            self.g_pos = torch.zeros(max(N_, 1), dtype=torch.int32, device=dev)[:N_]
+            self.x_seg = torch.zeros(2 * n_groups + 1, dtype=torch.int32, device=dev)
+            self.g_seg = torch.zeros(2 * n_groups + 1, dtype=torch.int32, device=dev)
+        self.wf = ChannelTensor(empty_codes(N_, kw, bits, n_groups, dev),
                                 torch.zeros(N_, dtype=torch.float32, device=dev),
                                 torch.zeros(N_, dtype=torch.float32, device=dev))
-        self.wd = ChannelTensor(empty_codes(K, N_, bits, n_groups, dev),
+        self.wd = ChannelTensor(empty_codes(K, nw, bits, n_groups, dev),
                                 torch.zeros(K, dtype=torch.float32, device=dev),
                                 torch.zeros(K, dtype=torch.float32, device=dev))
         self.y = torch.zeros((M, N_), dtype=torch.float32, device=dev)
@@ -139,22 +152,45 @@ class QuantLinear:
             self.ws_dgrad if self.ws_dgrad is not None else self.ws_wgrad)
         self.ws_layer = None
         if use_workspace:
-            need = N.shiftquant_gemm_layer_workspace_bytes(M, K, N_, bits, n_groups)
+            need = N.shiftquant_gemm_layer_workspace_bytes(M, K, N_, bits, n_groups,
+                                                           grouped=grouped)
             if need:
                 self.ws_layer = torch.zeros(need // 4, dtype=torch.int32, device=dev)
 
     # --- the hot path, step by step --------------------------------------------------
+    def _shift_quantize(self, t, q, pos, seg, mode, seed, stream):
+        if not self.grouped:
+            shift_quantize(t, q, self.bits, self.G, mode, seed, self.status, stream)
+            return
+        N.shiftquant_calibrate(t, N.SQ_GRAN_SHIFT, self.G, q.range, q.tau0, q.exp, self.status,
+                               stream)
+        N.shiftquant_group_order(q.exp, self.bits, self.G, pos, seg, stream)
+        N.shiftquant_quantize_ordered(t, N.SQ_GRAN_SHIFT, self.bits, self.G, q.tau0, q.exp, mode,
+                                      seed, pos, seg, q.codes, q.codes_t, q.scale, stream)
+
     def quantize_activation(self, x, stream=None):
-        shift_quantize(x, self.x, self.bits, self.G, N.SQ_ROUND_NEAREST_EVEN, 0, self.status,
-                       stream)
+        self._shift_quantize(x, self.x, self.x_pos, self.x_seg, N.SQ_ROUND_NEAREST_EVEN, 0,
+                             stream)
 
     def quantize_gradient(self, dy, seed, stream=None):
-        shift_quantize(dy, self.g, self.bits, self.G, N.SQ_ROUND_STOCHASTIC, seed, self.status,
-                       stream)
+        self._shift_quantize(dy, self.g, self.g_pos, self.g_seg, N.SQ_ROUND_STOCHASTIC, seed,
+                             stream)
 
     def quantize_weights(self, w, stream=None):
-        weight_quantize_fwd(w, self.wf, self.x.exp, self.bits, self.G, self.status, stream)
-        weight_quantize_dgrad(w, self.wd, self.g.exp, self.bits, self.G, self.status, stream)
+        if not self.grouped:
+            weight_quantize_fwd(w, self.wf, self.x.exp, self.bits, self.G, self.status, stream)
+            weight_quantize_dgrad(w, self.wd, self.g.exp, self.bits, self.G, self.status, stream)
+            return
+        # group-ordered weights carry no folded shift: each segment is shifted whole
+        st, b, G = self.status, self.bits, self.G
+        N.shiftquant_calibrate(w, N.SQ_GRAN_PER_COL, G, self.wf.range, None, None, st, stream)
+        N.shiftquant_quantize_ordered(w, N.SQ_GRAN_PER_COL, b, G, self.wf.range, None,
+                                      N.SQ_ROUND_NEAREST_EVEN, 0, self.x_pos, self.x_seg, None,
+                                      self.wf.codes, self.wf.scale, stream)
+        N.shiftquant_calibrate(w, N.SQ_GRAN_PER_ROW, G, self.wd.range, None, None, st, stream)
+        N.shiftquant_quantize_ordered(w, N.SQ_GRAN_PER_ROW, b, G, self.wd.range, None,
+                                      N.SQ_ROUND_NEAREST_EVEN, 0, self.g_pos, self.g_seg,
+                                      self.wd.codes, None, self.wd.scale, stream)
 
     def forward(self, stream=None):
         N.shiftquant_gemm_fwd(self.x.codes, self.x.scale, self.wf.codes, self.wf.scale, self.M,
@@ -188,13 +224,16 @@ class QuantLinear:
                                 self.dw, acc.get("fwd"), acc.get("dgrad"), acc.get("wgrad"),
                                 self.ws_layer if use_workspace else None, self.status, stream,
                                 gemm_mask=gemm_mask, max_ctas=max_ctas, y_range=y_range,
-                                dx_range=dx_range)
+                                dx_range=dx_range, x_seg=self.x_seg, g_seg=self.g_seg)
 
     def step(self, x, w, dy, seed, stream=None):
         """One training step of the layer: every quantizer pass and all three GEMMs."""
         self.quantize_activation(x, stream)
         self.quantize_gradient(dy, seed, stream)
         self.quantize_weights(w, stream)
+        if self.grouped:   # group-ordered operands: the layer launch carries the segment tables
+            self.gemms(stream)
+            return
         self.forward(stream)
         self.dgrad(stream)
         self.wgrad(stream)

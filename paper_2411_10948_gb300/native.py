@@ -36,9 +36,13 @@ EXPORTS = (
     "shiftquant_gemm_wgrad", "shiftquant_gemm_wgrad_partial", "shiftquant_gemm_wgrad_finish",
     "shiftquant_gemm_wgrad_static", "shiftquant_gemm_workspace_bytes",
     "shiftquant_gemm_layer", "shiftquant_gemm_layer_workspace_bytes",
+    "shiftquant_gemm_layer_workspace_bytes_grouped",
     "shiftquant_gemm_layer_kernel_launches", "shiftquant_gemm_layer_cta_pairs",
     "shiftquant_layer_step", "shiftquant_layer_step_host", "shiftquant_selftest_wait_timeout",
     "shiftquant_l1bn_state_bytes", "shiftquant_l1bn_forward", "shiftquant_l1bn_backward",
+    "shiftquant_group_order", "shiftquant_group_order_width", "shiftquant_quantize_ordered",
+    "shiftquant_pack_codes", "shiftquant_unpack_codes", "shiftquant_packed_groups_bytes",
+    "shiftquant_pack_groups", "shiftquant_unpack_groups",
     "shiftquant_status_string", "shiftquant_last_error",
 )
 
@@ -66,6 +70,7 @@ class SqLayerGemms(ctypes.Structure):
         ("acc_dw", ctypes.c_void_p), ("ld_acc_dw", ctypes.c_int64),
         ("gemm_mask", ctypes.c_int), ("max_ctas", ctypes.c_int),
         ("y_range", ctypes.c_void_p), ("dx_range", ctypes.c_void_p),
+        ("x_seg", ctypes.c_void_p), ("g_seg", ctypes.c_void_p),
     ]
 
 
@@ -147,6 +152,8 @@ def load(path: str | None = None) -> ctypes.CDLL:
     lib.shiftquant_gemm_layer.restype = i32
     lib.shiftquant_gemm_layer_workspace_bytes.argtypes = [i64, i64, i64, i32, i32]
     lib.shiftquant_gemm_layer_workspace_bytes.restype = sz
+    lib.shiftquant_gemm_layer_workspace_bytes_grouped.argtypes = [i64, i64, i64, i32, i32]
+    lib.shiftquant_gemm_layer_workspace_bytes_grouped.restype = sz
     lib.shiftquant_gemm_layer_kernel_launches.argtypes = [i64, i64, i64, i32, i32, sz, i32]
     lib.shiftquant_gemm_layer_kernel_launches.restype = i32
     lib.shiftquant_gemm_layer_cta_pairs.argtypes = [i64, i64, i64, i32, i32, i32]
@@ -169,6 +176,23 @@ def load(path: str | None = None) -> ctypes.CDLL:
     lib.shiftquant_l1bn_backward.argtypes = [vp, i64, i64, i64, i32, i32, u64, vp, sz, vp, i64,
                                              vp, vp, vp, vp]
     lib.shiftquant_l1bn_backward.restype = i32
+    lib.shiftquant_group_order.argtypes = [vp, i64, i32, i32, vp, vp, vp]
+    lib.shiftquant_group_order.restype = i32
+    lib.shiftquant_group_order_width.argtypes = [i64, i32, i32]
+    lib.shiftquant_group_order_width.restype = i64
+    lib.shiftquant_quantize_ordered.argtypes = [vp, i64, i64, i64, i32, i32, i32, vp, vp, i32, u64,
+                                                i64, vp, vp, vp, i64, vp, i64, vp, vp]
+    lib.shiftquant_quantize_ordered.restype = i32
+    lib.shiftquant_pack_codes.argtypes = [vp, i64, i64, i64, i32, i32, vp, i64, vp, vp]
+    lib.shiftquant_pack_codes.restype = i32
+    lib.shiftquant_unpack_codes.argtypes = [vp, i64, i64, i64, i32, i32, vp, i64, vp]
+    lib.shiftquant_unpack_codes.restype = i32
+    lib.shiftquant_packed_groups_bytes.argtypes = [i64, i32]
+    lib.shiftquant_packed_groups_bytes.restype = i64
+    lib.shiftquant_pack_groups.argtypes = [vp, i64, i32, vp, vp]
+    lib.shiftquant_pack_groups.restype = i32
+    lib.shiftquant_unpack_groups.argtypes = [vp, i64, i32, vp, vp]
+    lib.shiftquant_unpack_groups.restype = i32
     lib.shiftquant_status_string.argtypes = [i32]
     lib.shiftquant_status_string.restype = ctypes.c_char_p
     lib.shiftquant_last_error.argtypes = []
@@ -302,7 +326,7 @@ def shiftquant_gemm_layer(x_codes, xt_codes, x_scale, x_exp, g_codes, gt_codes, 
                           wf_codes, wf_scale, wd_codes, wd_scale, M, K, N, bits, n_groups, y, dx,
                           dw, acc_y=None, acc_dx=None, acc_dw=None, workspace=None,
                           dev_status=None, stream=None, gemm_mask=0, max_ctas=0, y_range=None,
-                          dx_range=None) -> None:
+                          dx_range=None, x_seg=None, g_seg=None) -> None:
     """Forward, loss-propagation and weight-gradient GEMMs of one layer in one launch
     (gemm_mask: bit 0 forward, 1 loss propagation, 2 weight gradient; 0 = all); y_range and
     dx_range optionally receive the per-column max |Y| and max |dX| from the epilogue."""
@@ -319,7 +343,7 @@ def shiftquant_gemm_layer(x_codes, xt_codes, x_scale, x_exp, g_codes, gt_codes, 
         acc_dx=_addr(acc_dx), ld_acc_dx=_ld_opt(acc_dx),
         acc_dw=_addr(acc_dw), ld_acc_dw=_ld_opt(acc_dw),
         gemm_mask=gemm_mask, max_ctas=max_ctas, y_range=_addr(y_range),
-        dx_range=_addr(dx_range))
+        dx_range=_addr(dx_range), x_seg=_addr(x_seg), g_seg=_addr(g_seg))
     _check(load().shiftquant_gemm_layer(
         ctypes.byref(a), _ptr(workspace),
         workspace.numel() * workspace.element_size() if workspace is not None else 0,
@@ -345,8 +369,11 @@ def shiftquant_gemm_wgrad_finish(t, Ci, Co, bits, n_groups, x_scale, x_exp, g_sc
         _ptr(dev_status), _stream(stream)))
 
 
-def shiftquant_gemm_layer_workspace_bytes(M: int, K: int, N: int, bits: int, n_groups: int) -> int:
-    return int(load().shiftquant_gemm_layer_workspace_bytes(M, K, N, bits, n_groups))
+def shiftquant_gemm_layer_workspace_bytes(M: int, K: int, N: int, bits: int, n_groups: int,
+                                          grouped: bool = False) -> int:
+    fn = (load().shiftquant_gemm_layer_workspace_bytes_grouped if grouped
+          else load().shiftquant_gemm_layer_workspace_bytes)
+    return int(fn(M, K, N, bits, n_groups))
 
 
 def shiftquant_gemm_layer_kernel_launches(M: int, K: int, N: int, bits: int, n_groups: int,
@@ -435,3 +462,49 @@ def shiftquant_l1bn_backward(dy, bits, n_groups, seed, state, dx, dgamma, dbeta,
         _ptr(dy), dy.shape[0], dy.shape[1], _ld(dy), bits, n_groups, seed & (2**64 - 1),
         _ptr(state), state.numel() * state.element_size(), _ptr(dx), _ld(dx), _ptr(dgamma),
         _ptr(dbeta), _ptr(dev_status), _stream(stream)))
+
+
+def shiftquant_group_order_width(channels: int, bits: int, n_groups: int) -> int:
+    return int(load().shiftquant_group_order_width(channels, bits, n_groups))
+
+
+def shiftquant_group_order(exp, bits, n_groups, pos_out, seg_out, stream=None) -> None:
+    """Stable group order of a GEMM inner index from its exponents (see the header)."""
+    _check(load().shiftquant_group_order(_ptr(exp), exp.numel(), bits, n_groups, _ptr(pos_out),
+                                         _ptr(seg_out), _stream(stream)))
+
+
+def shiftquant_quantize_ordered(x, gran, bits, n_groups, range_or_tau0, exp, mode, seed, pos, seg,
+                                codes, codes_t, scale_out, stream=None, row0=0) -> None:
+    """shiftquant_quantize writing the GEMM inner index in group order (see the header)."""
+    _check(load().shiftquant_quantize_ordered(
+        _ptr(x), x.shape[0], x.shape[1], _ld(x), gran, bits, n_groups, _ptr(range_or_tau0),
+        _ptr(exp), mode, seed & (2**64 - 1), row0, _ptr(pos), _ptr(seg), _ptr(codes),
+        _ld(codes) if codes is not None else 0, _ptr(codes_t),
+        _ld(codes_t) if codes_t is not None else 0, _ptr(scale_out), _stream(stream)))
+
+
+def shiftquant_pack_codes(codes, bits, n_groups, packed, dev_status, stream=None) -> None:
+    """4-bit codes [R, C] -> packed bytes [R, >= ceil(C/2)] (see the header)."""
+    _check(load().shiftquant_pack_codes(_ptr(codes), codes.shape[0], codes.shape[1], _ld(codes),
+                                        bits, n_groups, _ptr(packed), _ld(packed),
+                                        _ptr(dev_status), _stream(stream)))
+
+
+def shiftquant_unpack_codes(packed, cols, bits, n_groups, codes, stream=None) -> None:
+    _check(load().shiftquant_unpack_codes(_ptr(packed), _ld(packed), packed.shape[0], cols, bits,
+                                          n_groups, _ptr(codes), _ld(codes), _stream(stream)))
+
+
+def shiftquant_packed_groups_bytes(channels: int, n_groups: int) -> int:
+    return int(load().shiftquant_packed_groups_bytes(channels, n_groups))
+
+
+def shiftquant_pack_groups(exp, n_groups, packed, stream=None) -> None:
+    _check(load().shiftquant_pack_groups(_ptr(exp), exp.numel(), n_groups, _ptr(packed),
+                                         _stream(stream)))
+
+
+def shiftquant_unpack_groups(packed, channels, n_groups, exp, stream=None) -> None:
+    _check(load().shiftquant_unpack_groups(_ptr(packed), channels, n_groups, _ptr(exp),
+                                           _stream(stream)))
