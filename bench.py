@@ -206,7 +206,7 @@ class Step:
         n = 0
         N = self.N
         for lay in self.layers:
-            n += 2 + 1 + 2 + 1          # X and dY: range init + range/grouping, quantize
+            n += 3 + 1 + 3 + 1          # X and dY: range init, range, grouping; quantize
             n += 2 + 1 + 1 + 1          # weights: range init + range, quantize (out-channel);
                                         # row range, quantize (in-channel)
             # the three GEMMs: one launch, plus the output pass of each GEMM that splits K
@@ -404,6 +404,46 @@ def run_ours(args, rank, world, local_rank):
     total_ms = max_over_ranks(sum(step_ms), dev)
     ms_per_step = total_ms / args.steps
 
+    # the quantizer passes as the step runs them, in a CUDA graph: the step's range and
+    # quantize calls serial on one stream, captured once and replayed after an L2 flush,
+    # timed with events around the replay (no per-launch host gap)
+    qcalls = [(n, fn) for n, fn in st.calls(args.warmup) if n != "gemm"]
+    q_graph = L.CapturedStep(lambda: [fn() for _, fn in qcalls])
+    q_graph_ms = 0.0
+    for i in range(args.warmup + args.steps):
+        flush_l2()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        q_graph.replay()
+        b.record(stream)
+        torch.cuda.synchronize()
+        if i >= args.warmup:
+            q_graph_ms += a.elapsed_time(b)
+    q_graph_ms = max_over_ranks(q_graph_ms, dev)
+    # per tensor: a graph of its range call and one of its range and quantize calls, each
+    # timed the same way (event nodes inside a graph cost microseconds each, so the calls
+    # are not split by events); the quantize time is the difference
+    def graph_ms(fns):
+        g = L.CapturedStep(lambda: [fn() for fn in fns])
+        tot = 0.0
+        for i in range(args.warmup + args.steps):
+            flush_l2()
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record(stream)
+            g.replay()
+            b.record(stream)
+            torch.cuda.synchronize()
+            if i >= args.warmup:
+                tot += a.elapsed_time(b)
+        del g
+        return tot
+    q_call_graph_ms = []
+    for j in range(0, len(qcalls), 2):
+        r_ms = graph_ms([qcalls[j][1]])
+        both_ms = graph_ms([qcalls[j][1], qcalls[j + 1][1]])
+        q_call_graph_ms += [r_ms, max(both_ms - r_ms, 1e-6)]
+    del q_graph
+
     # e2e: the C entry point shiftquant_layer_step_host (layer.HostSteps): every call copies a
     # layer's X, W and dY in from pinned host memory, runs its whole step and copies Y, dX and
     # dW back; two device buffer sets on two streams take the steps in turn.  Timed from the
@@ -438,17 +478,22 @@ def run_ours(args, rank, world, local_rank):
         del pipe
     clocks = sampler.stop()
 
-    # quantizer throughput per tensor: range pass, quantize pass and both, from the breakdown
+    # quantizer throughput per tensor: range pass, quantize pass and both, from the calls
+    # inside the quantizer graph (else from the un-graphed breakdown)
     per_tensor = []
     cbytes = st.call_bytes()
-    for j in range(0, len(names), 9):
-        for k in range(4):
-            (lname, tname, rb), (_, _, qb) = cbytes[j + 2 * k], cbytes[j + 2 * k + 1]
-            rms, qms = call_ms[j + 2 * k] / args.steps, call_ms[j + 2 * k + 1] / args.steps
-            per_tensor.append({"layer": lname, "tensor": tname,
-                               "range_gbs": round(rb / (rms * 1e-3) / 1e9, 1),
-                               "quantize_gbs": round(qb / (qms * 1e-3) / 1e9, 1),
-                               "both_gbs": round((rb + qb) / ((rms + qms) * 1e-3) / 1e9, 1)})
+    qcbytes = [c for c, n in zip(cbytes, names) if n != "gemm"]
+    q_per_call = q_call_graph_ms
+    per_tensor_src = ("per tensor, one graph of its range call and one of its range and quantize "
+                      "calls, each replayed after an L2 flush; quantize = the difference")
+    for j in range(0, len(qcbytes), 2):
+        (lname, tname, rb), (_, _, qb) = qcbytes[j], qcbytes[j + 1]
+        rms, qms = q_per_call[j] / args.steps, q_per_call[j + 1] / args.steps
+        per_tensor.append({"layer": lname, "tensor": tname,
+                           "range_us": round(rms * 1e3, 2), "quantize_us": round(qms * 1e3, 2),
+                           "range_gbs": round(rb / (rms * 1e-3) / 1e9, 1),
+                           "quantize_gbs": round(qb / (qms * 1e-3) / 1e9, 1),
+                           "both_gbs": round((rb + qb) / ((rms + qms) * 1e-3) / 1e9, 1)})
     peaks, peak_src = load_peaks()
     spec0 = wl.layers[0]
     fp8 = native.shiftquant_code_type(spec0.bits, spec0.n_groups) == native.SQ_CODE_E4M3
@@ -461,7 +506,9 @@ def run_ours(args, rank, world, local_rank):
         gemm_launch_ms = graph_gemm_ms
     gemm_tflops = sum(flops) / (sum(gemm_launch_ms) * 1e-3) / 1e12
     q_bytes = st.quantizer_bytes() * args.steps
-    q_ms = kind_ms["calibrate"] + kind_ms["quantize"]
+    q_ms_ungraphed = kind_ms["calibrate"] + kind_ms["quantize"]
+    q_gbs_ungraphed = q_bytes / (q_ms_ungraphed * 1e-3) / 1e9
+    q_ms = q_graph_ms
     q_gbs = q_bytes / (q_ms * 1e-3) / 1e9
     # The layer GEMM launch is bound by the tensor cores or by HBM depending on its
     # arithmetic intensity (operations per algorithmic byte) against the ridge point
@@ -496,7 +543,15 @@ def run_ours(args, rank, world, local_rank):
                      intensity_ops_per_byte=intensity, ridge_ops_per_byte=ridge)
     quant_roof = {"bound": "hbm", "achieved": q_gbs, "peak": peaks["hbm_gbs"], "unit": "GB/s",
                   "frac": q_gbs / peaks["hbm_gbs"], "kernel": "calibrate + quantize",
-                  "peak_source": f"{peak_src} copy bandwidth"}
+                  "peak_source": f"{peak_src} copy bandwidth",
+                  "timing": "every range and quantize call of a step, serial on one stream, "
+                            "in one CUDA-graph replay after an L2 flush",
+                  "ms_per_step": q_ms / args.steps,
+                  "ungraphed": {"achieved": q_gbs_ungraphed,
+                                "frac": q_gbs_ungraphed / peaks["hbm_gbs"],
+                                "ms_per_step": q_ms_ungraphed / args.steps,
+                                "timing": "the same calls launched one by one from the host, "
+                                          "queued behind a sleep kernel, events between them"}}
     # the dominant kernel: the kernel class (range pass, quantize, layer GEMM launch) of the
     # single launch with the most device time in the step
     def hbm_roof(nbytes, ms, name):
@@ -545,6 +600,7 @@ def run_ours(args, rank, world, local_rank):
         "breakdown_ms_per_step": {k: v / args.steps for k, v in kind_ms.items()},
         "calls_ms_per_step": [[f"{n}", round(v / args.steps, 5)] for n, v in zip(names, call_ms)],
         "quantizer_per_tensor": per_tensor,
+        "quantizer_per_tensor_source": per_tensor_src,
         "group_histograms": st.group_histograms(),
         "timing": "CUDA events around one CUDA-graph replay of the whole step (per layer: "
                   "activation chain, gradient chain and both weight roles on four streams, "

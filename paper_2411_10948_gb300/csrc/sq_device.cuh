@@ -38,6 +38,16 @@ __device__ __forceinline__ float4 ld_stream_v4(const float* p) {
   return v;
 }
 
+// the same load as a pure function of the address (no volatile): the compiler may batch
+// a run of them ahead of their uses, keeping all of them in flight together
+__device__ __forceinline__ float4 ld_nc_v4(const float* p) {
+  float4 v;
+  asm("ld.global.nc.L1::no_allocate.L2::256B.v4.f32 {%0, %1, %2, %3}, [%4];"
+      : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
+      : "l"(p));
+  return v;
+}
+
 // ----------------------------------------------------- programmatic dependent launch
 // Wait until the preceding kernel of the stream has completed and its writes are visible
 // (a no-op for a kernel launched without programmatic stream serialization).
@@ -161,6 +171,20 @@ __device__ __forceinline__ bool mbar_wait_cluster(uint64_t* bar, uint32_t parity
 // every thread of both CTAs: writes before it are visible to the other CTA after it
 __device__ __forceinline__ void cluster_sync() {
   asm volatile("barrier.cluster.arrive.release;\n\tbarrier.cluster.wait.acquire;" ::: "memory");
+}
+
+// the two halves of cluster_sync, for work placed between them
+__device__ __forceinline__ void cluster_arrive_release() {
+  asm volatile("barrier.cluster.arrive.release;" ::: "memory");
+}
+__device__ __forceinline__ void cluster_wait_acquire() {
+  asm volatile("barrier.cluster.wait.acquire;" ::: "memory");
+}
+
+// atomic max into a shared::cluster address (another CTA's shared memory)
+__device__ __forceinline__ void red_max_cluster_u32(uint32_t cluster_addr, uint32_t v) {
+  asm volatile("red.relaxed.cluster.shared::cluster.max.u32 [%0], %1;" ::"r"(cluster_addr), "r"(v)
+               : "memory");
 }
 
 // ----------------------------------------------------------------------- TMA

@@ -75,103 +75,106 @@ __global__ void __launch_bounds__(256)
   if (counter != nullptr && blockIdx.x == 0 && threadIdx.x == 0) *counter = 0u;
 }
 
-// Grouping (Eq. 3) by one block of kGroupThreads threads from the per-channel range bits:
-// tau_0 = the largest range, then every channel's exponent; tau0_out receives tau_0 and the
-// status word the non-finite flag.  scratch: 33 words of shared memory.
-constexpr int kGroupThreads = 256;
-static_assert(kColTx * kColTy == kGroupThreads, "the range pass's last block does the grouping");
+// Grouping (Eq. 3) by one block of THREADS threads from the per-channel range bits:
+// tau_0 = the largest range, then every channel's exponent; tau0_out receives tau_0 and
+// the status word the non-finite flag.  Thread t holds channels t, t + THREADS, ... (up to
+// kGroupPerThread of them in registers, so all its loads are in flight together; wider
+// tensors read the rest twice).  Small blocks start faster, large ones take wide tensors
+// in one round of loads.  Launched behind the range pass with programmatic stream
+// serialization, it waits for the range pass before reading anything.
+constexpr int kGroupPerThread = 16;
+constexpr int kGroupSmallThreads = 256;
+constexpr int kGroupLargeThreads = 1024;
 
-__device__ void grouping_block(const unsigned* range_bits, int64_t C, int G, float* tau0_out,
-                               uint8_t* exp_out, int* status, unsigned* scratch, int tid) {
+template <int THREADS>
+__global__ void __launch_bounds__(THREADS)
+    group_kernel(const unsigned* __restrict__ range_bits, int64_t C, int G,
+                 float* __restrict__ tau0_out, uint8_t* __restrict__ exp_out,
+                 int* __restrict__ status) {
+  __shared__ unsigned wmax[THREADS / 32];
+  __shared__ unsigned tau_bits;
+  griddep_wait();
+  griddep_launch_dependents();
+  const int tid = threadIdx.x;
+  unsigned v[kGroupPerThread];
   unsigned m = 0;
-  for (int64_t c = tid; c < C; c += kGroupThreads) m = max(m, __ldcg(range_bits + c));
+#pragma unroll
+  for (int k = 0; k < kGroupPerThread; ++k) {
+    const int64_t c = tid + static_cast<int64_t>(k) * THREADS;
+    v[k] = c < C ? __ldcg(range_bits + c) : 0u;
+    m = max(m, v[k]);
+  }
+  constexpr int64_t kHeld = static_cast<int64_t>(THREADS) * kGroupPerThread;
+  for (int64_t c = kHeld + tid; c < C; c += THREADS) m = max(m, __ldcg(range_bits + c));
   m = __reduce_max_sync(0xFFFFFFFFu, m);
-  if ((tid & 31) == 0) scratch[tid >> 5] = m;
+  if ((tid & 31) == 0) wmax[tid >> 5] = m;
   __syncthreads();
   if (tid < 32) {
-    unsigned v = tid < kGroupThreads / 32 ? scratch[tid] : 0u;
-    v = __reduce_max_sync(0xFFFFFFFFu, v);
-    if (tid == 0) scratch[32] = v;
+    const unsigned w = __reduce_max_sync(0xFFFFFFFFu, tid < THREADS / 32 ? wmax[tid] : 0u);
+    if (tid == 0) tau_bits = w;
   }
   __syncthreads();
-  const unsigned tb = scratch[32];
+  const unsigned tb = tau_bits;
   const float tau = __uint_as_float(tb);
   const bool nonfinite = tb >= 0x7F800000u;
-  for (int64_t c = tid; c < C; c += kGroupThreads)
+#pragma unroll
+  for (int k = 0; k < kGroupPerThread; ++k) {
+    const int64_t c = tid + static_cast<int64_t>(k) * THREADS;
+    if (c < C) exp_out[c] = static_cast<uint8_t>(nonfinite ? 0 : group_exponent(__uint_as_float(v[k]), tau, G));
+  }
+  for (int64_t c = kHeld + tid; c < C; c += THREADS)
     exp_out[c] = static_cast<uint8_t>(nonfinite ? 0 : group_exponent(__uint_as_float(__ldcg(range_bits + c)), tau, G));
-  __syncthreads();
   if (tid == 0) {
     *tau0_out = tau;
     if (nonfinite) atomicOr(status, kDevNonFinite);
   }
 }
 
-// Grouping alone, from a given range vector (a sharded tensor's all-reduced ranges)
-__global__ void __launch_bounds__(kGroupThreads)
-    group_kernel(const unsigned* __restrict__ range_bits, int64_t C, int G,
-                 float* __restrict__ tau0_out, uint8_t* __restrict__ exp_out,
-                 int* __restrict__ status) {
-  __shared__ unsigned scratch[33];
-  grouping_block(range_bits, C, G, tau0_out, exp_out, status, scratch, threadIdx.x);
-}
-
-// Range pass: one wave of blocks, block (x, y) owning 128 columns and the 64-row tiles
-// y, y + gridDim.y, ... (so the blocks resident at one time read a contiguous band of whole
-// rows: long DRAM bursts).  Warp w reads rows 8w .. 8w+7 of a tile with all eight 16-byte
-// loads in flight; lane l owns columns 4l .. 4l+3.  The block's per-column maxima go to
-// range_bits with one atomic max each, on the ordered bit pattern of the non-negative
-// floats (NaN sorts above Inf).
-// G > 0: the block that finishes last also performs the grouping (Eq. 3): tau_0 and the
-// exponents.  Until then tau0_out holds the count of finished blocks.
+// Range pass: block (x, y) reads the 64 x 128 tile (y, x) -- warp w rows 8w .. 8w+7 with
+// all eight 16-byte loads in flight, lane l columns 4l .. 4l+3 -- and takes its per-column
+// maxima as ordered bit patterns of the non-negative floats (NaN sorts above Inf), sent to
+// range_bits with one atomic max per column.  Same-address atomics from hundreds of tiles
+// of a narrow tensor serialise in L2, so narrow tensors (CL = kRangeCluster) run in
+// clusters of CL blocks along the rows: each block merges its maxima into the first block
+// of its cluster with atomic maxima on that block's shared memory, and only that block
+// sends them on.  Wide tensors (CL = 1) spread their atomics over many addresses and run
+// without clusters, which schedule more slowly.  Grids taller than the 65535-block limit
+// walk the extra tiles in steps of gridDim.y.
 constexpr int kRangeRows = 64;
+constexpr int kRangeCluster = 8;
+constexpr int64_t kRangeClusterMaxCols = 4 * kColTx * 4;   // clusters up to 4 column blocks
 
+template <int CL>
 __global__ void __launch_bounds__(kColTx* kColTy)
     colmax_kernel(const float* __restrict__ x, int64_t R, int64_t C, int64_t ld, int vec,
-                  unsigned* __restrict__ range_bits, int* __restrict__ status, int G,
-                  float* __restrict__ tau0_out, uint8_t* __restrict__ exp_out) {
+                  unsigned* __restrict__ range_bits, int* __restrict__ status) {
   __shared__ unsigned red[kColTy][kColTx * 4];
-  __shared__ unsigned last_block;
+  __shared__ unsigned cmax[CL > 1 ? kColTx * 4 : 1];   // the cluster's maxima (first block)
   const int tx = threadIdx.x, ty = threadIdx.y;   // tx: lane (columns), ty: warp (rows)
+  const int tid = ty * kColTx + tx;
   const int64_t c0 = (static_cast<int64_t>(blockIdx.x) * kColTx + tx) * 4;
+  const int64_t tiles = (R + kRangeRows - 1) / kRangeRows;
+  if (CL > 1) {
+    if (tid < kColTx * 4) cmax[tid] = 0u;
+    cluster_arrive_release();   // the zeroed cmax is visible to the cluster after the wait
+  }
   unsigned m0 = 0, m1 = 0, m2 = 0, m3 = 0;
-  // grid-stride over row tiles: the blocks resident together cover consecutive row tiles
-  if (vec && c0 + 3 < C) {
-    // software-pipelined: the next tile's eight loads leave before this tile is reduced.
-    // Rows past the end re-read the last row, which leaves a maximum unchanged.
-    auto load_tile = [&](int64_t t, float4 (&v)[8]) {
-      const int64_t r0 = t * kRangeRows + ty * 8;
+#pragma unroll 1
+  for (int64_t t = blockIdx.y; t < tiles; t += gridDim.y) {
+    const int64_t r0 = t * kRangeRows + ty * 8;
+    if (vec && c0 + 3 < C) {
+      // rows past the end re-read the last row, which leaves a maximum unchanged
+      float4 v[8];
+#pragma unroll
+      for (int u = 0; u < 8; ++u) v[u] = ld_stream_v4(x + min(r0 + u, R - 1) * ld + c0);
 #pragma unroll
       for (int u = 0; u < 8; ++u) {
-        const int64_t r = min(r0 + u, R - 1);
-        v[u] = ld_stream_v4(x + r * ld + c0);
+        m0 = max(m0, abs_bits(v[u].x));
+        m1 = max(m1, abs_bits(v[u].y));
+        m2 = max(m2, abs_bits(v[u].z));
+        m3 = max(m3, abs_bits(v[u].w));
       }
-    };
-    float4 cur[8], nxt[8];
-    int64_t t = blockIdx.y;
-    if (t * kRangeRows < R) {
-      load_tile(t, cur);
-#pragma unroll 1
-      while (true) {
-        const int64_t tn = t + gridDim.y;
-        const bool more = tn * kRangeRows < R;
-        if (more) load_tile(tn, nxt);
-#pragma unroll
-        for (int u = 0; u < 8; ++u) {
-          m0 = max(m0, abs_bits(cur[u].x));
-          m1 = max(m1, abs_bits(cur[u].y));
-          m2 = max(m2, abs_bits(cur[u].z));
-          m3 = max(m3, abs_bits(cur[u].w));
-        }
-        if (!more) break;
-#pragma unroll
-        for (int u = 0; u < 8; ++u) cur[u] = nxt[u];
-        t = tn;
-      }
-    }
-  } else {
-#pragma unroll 1
-    for (int64_t t = blockIdx.y; t * kRangeRows < R; t += gridDim.y) {
-      const int64_t r0 = t * kRangeRows + ty * 8;
+    } else {
 #pragma unroll 1
       for (int u = 0; u < 8; ++u) {
         const int64_t r = r0 + u;
@@ -184,42 +187,50 @@ __global__ void __launch_bounds__(kColTx* kColTy)
       }
     }
   }
-  // x has been read: the next kernel (the quantizer) may start launching; the
-  // accumulators below are zeroed by the preceding kernel, which must have completed
+  // x has been read: the next kernel (the grouping) may start launching
   griddep_launch_dependents();
-  griddep_wait();
   red[ty][tx * 4 + 0] = m0;
   red[ty][tx * 4 + 1] = m1;
   red[ty][tx * 4 + 2] = m2;
   red[ty][tx * 4 + 3] = m3;
   __syncthreads();
+  unsigned m[4];
   if (ty == 0) {
-    bool bad = false;
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
-      unsigned m = 0;
+      m[i] = 0;
 #pragma unroll
-      for (int y = 0; y < kColTy; ++y) m = max(m, red[y][tx * 4 + i]);
-      if (c0 + i < C && m != 0) {
-        atomicMax(range_bits + c0 + i, m);
-        bad |= m >= 0x7F800000u;
-      }
+      for (int y = 0; y < kColTy; ++y) m[i] = max(m[i], red[y][tx * 4 + i]);
     }
-    if (bad) atomicOr(status, kDevNonFinite);
   }
-  if (G == 0) return;
-  // grouping by the last block to finish (the classic fence-then-count pattern)
-  __threadfence();
-  __syncthreads();
-  const int tid = ty * kColTx + tx;
-  if (tid == 0) {
-    const unsigned total = gridDim.x * gridDim.y;
-    last_block = atomicAdd(reinterpret_cast<unsigned*>(tau0_out), 1u) == total - 1u;
+  if (CL > 1) {
+    cluster_wait_acquire();
+    if (ty == 0) {
+      const uint32_t lead = mapa_shared(smem_u32(cmax), 0);
+#pragma unroll
+      for (int i = 0; i < 4; ++i)
+        if (m[i] != 0) red_max_cluster_u32(lead + (tx * 4 + i) * 4, m[i]);
+    }
+    cluster_arrive_release();
+    cluster_wait_acquire();   // every block's maxima are in the first block's cmax
+    if (cluster_ctarank() != 0) return;
+    if (ty == 0) {
+#pragma unroll
+      for (int i = 0; i < 4; ++i) m[i] = cmax[tx * 4 + i];
+    }
   }
-  __syncthreads();
-  if (!last_block) return;
-  __threadfence();
-  grouping_block(range_bits, C, G, tau0_out, exp_out, status, &red[0][0], tid);
+  if (ty != 0) return;
+  // the accumulators are zeroed by the preceding kernel, which must have completed
+  griddep_wait();
+  bool bad = false;
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    if (c0 + i < C && m[i] != 0) {
+      atomicMax(range_bits + c0 + i, m[i]);
+      bad |= m[i] >= 0x7F800000u;
+    }
+  }
+  if (bad) atomicOr(status, kDevNonFinite);
 }
 
 // one warp per row: range[r] = max_c |x[r, c]|
@@ -376,6 +387,14 @@ __device__ __forceinline__ void quantize_tile(const QuantArgs& a, uint8_t* tile_
 #pragma unroll
     for (int k = 0; k < kWords; ++k) packed[j][k] = 0u;
 
+  // stochastic rounding: the generator state of element (r, c) is seed + (idx+1) gamma with
+  // idx = (row0 + r) C + c; it advances by gamma per column and by C gamma per row
+  uint64_t sr_state = 0;
+  if (MODE == SQ_ROUND_STOCHASTIC)
+    sr_state = a.seed + (static_cast<uint64_t>(a.row0 + r0 + wq * 8) * static_cast<uint64_t>(a.C) +
+                         static_cast<uint64_t>(cb) + 1ull) * kSplitMixGamma;
+  const uint64_t sr_row_step = static_cast<uint64_t>(a.C) * kSplitMixGamma;
+
 #pragma unroll
   for (int i = 0; i < kQRowsPerWarp; ++i) {
     const int64_t r = r0 + wq * 8 + i;
@@ -415,9 +434,9 @@ __device__ __forceinline__ void quantize_tile(const QuantArgs& a, uint8_t* tile_
       } else {
         const float l = floorf(v);
         const float frac = __fsub_rn(v, l);
-        const uint64_t hsh = splitmix64_at(a.seed, static_cast<uint64_t>((a.row0 + r) * a.C + cb + j));
-        const float u = __fmul_rn(static_cast<float>(static_cast<uint32_t>(hsh >> 40)),
-                                  5.9604644775390625e-08f);  // * 2^-24, exact
+        const uint32_t h24 = splitmix64_top24(sr_state + static_cast<uint64_t>(j) * kSplitMixGamma +
+                                              static_cast<uint64_t>(i) * sr_row_step);
+        const float u = __fmul_rn(static_cast<float>(h24), 5.9604644775390625e-08f);  // * 2^-24, exact
         q = (u < frac) ? __fadd_rn(l, 1.0f) : l;
         q = fminf(fmaxf(q, -Qf), Qf);
       }
@@ -770,32 +789,47 @@ extern "C" sq_status shiftquant_calibrate(const float* x, int64_t rows, int64_t 
   {
     const int64_t iblocks = (cols + 255) / 256;
     calib_init_kernel<<<static_cast<unsigned>(iblocks < 1024 ? iblocks : 1024), 256, 0, s>>>(
-        reinterpret_cast<unsigned*>(range_out), cols,
-        shift ? reinterpret_cast<unsigned*>(tau0_out) : nullptr);
+        reinterpret_cast<unsigned*>(range_out), cols, nullptr);
     err = cudaGetLastError();
     if (err != cudaSuccess) return cuda_fail(err, "calib_init_kernel launch");
   }
   const int64_t cblocks = (cols + kColTx * 4 - 1) / (kColTx * 4);
   const int64_t tiles = (rows + kRangeRows - 1) / kRangeRows;
-  // one wave of resident blocks (never a partial second wave)
-  int per_sm = 0, dev = 0, sms = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess ||
-      cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || sms < 1)
-    sms = 148;
-  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, colmax_kernel, kColTx * kColTy, 0) !=
-          cudaSuccess || per_sm < 1)
-    per_sm = 4;
-  int64_t rblocks = static_cast<int64_t>(sms) * per_sm / cblocks;
-  if (rblocks > tiles) rblocks = tiles;
-  if (rblocks > 65535) rblocks = 65535;
-  if (rblocks < 1) rblocks = 1;
+  if (cblocks > 0x7FFFFFFF) return fail(SQ_EINVAL, "calibrate: too many columns");
+  // one block per 64 x 128 tile; narrow tensors in whole clusters along the rows
+  const int cl = cols <= kRangeClusterMaxCols ? kRangeCluster : 1;
+  const int64_t max_rblocks = 65535 / cl * cl;
+  int64_t rblocks = (tiles + cl - 1) / cl * cl;
+  if (rblocks > max_rblocks) rblocks = max_rblocks;
   const int vec = (ld % 4 == 0) && aligned16(x);
-  dim3 grid(static_cast<unsigned>(cblocks), static_cast<unsigned>(rblocks));
-  err = launch_pdl(colmax_kernel, grid, dim3(kColTx, kColTy), s, x, rows, cols, ld, vec,
-                   reinterpret_cast<unsigned*>(range_out), dev_status, shift ? n_groups : 0,
-                   tau0_out, exp_out);
+  cudaLaunchConfig_t cfg;
+  memset(&cfg, 0, sizeof(cfg));
+  cfg.gridDim = dim3(static_cast<unsigned>(cblocks), static_cast<unsigned>(rblocks));
+  cfg.blockDim = dim3(kColTx, kColTy);
+  cfg.stream = s;
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  attr[1].id = cudaLaunchAttributeClusterDimension;
+  attr[1].val.clusterDim.x = 1;
+  attr[1].val.clusterDim.y = cl;
+  attr[1].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = cl > 1 ? 2 : 1;
+  unsigned* bits = reinterpret_cast<unsigned*>(range_out);
+  err = cl > 1 ? cudaLaunchKernelEx(&cfg, colmax_kernel<kRangeCluster>, x, rows, cols, ld, vec, bits, dev_status)
+               : cudaLaunchKernelEx(&cfg, colmax_kernel<1>, x, rows, cols, ld, vec, bits, dev_status);
   if (err == cudaSuccess) err = cudaGetLastError();
-  return err == cudaSuccess ? SQ_OK : cuda_fail(err, "colmax_kernel launch");
+  if (err != cudaSuccess) return cuda_fail(err, "colmax_kernel launch");
+  if (!shift) return SQ_OK;
+  // grouping (Eq. 3) by one block behind the range pass
+  err = cols <= static_cast<int64_t>(kGroupSmallThreads) * kGroupPerThread
+            ? launch_pdl(group_kernel<kGroupSmallThreads>, dim3(1), dim3(kGroupSmallThreads), s,
+                         static_cast<const unsigned*>(bits), cols, n_groups, tau0_out, exp_out, dev_status)
+            : launch_pdl(group_kernel<kGroupLargeThreads>, dim3(1), dim3(kGroupLargeThreads), s,
+                         static_cast<const unsigned*>(bits), cols, n_groups, tau0_out, exp_out, dev_status);
+  if (err == cudaSuccess) err = cudaGetLastError();
+  return err == cudaSuccess ? SQ_OK : cuda_fail(err, "group_kernel launch");
 }
 
 extern "C" sq_status shiftquant_group(const float* range, int64_t channels, int n_groups,
@@ -811,8 +845,13 @@ extern "C" sq_status shiftquant_group(const float* range, int64_t channels, int 
     const cudaError_t err = cudaMemsetAsync(tau0_out, 0, sizeof(float), s);
     return err == cudaSuccess ? SQ_OK : cuda_fail(err, "cudaMemsetAsync");
   }
-  group_kernel<<<1, kGroupThreads, 0, s>>>(reinterpret_cast<const unsigned*>(range), channels,
-                                           n_groups, tau0_out, exp_out, dev_status);
+  const unsigned* rb = reinterpret_cast<const unsigned*>(range);
+  if (channels <= static_cast<int64_t>(kGroupSmallThreads) * kGroupPerThread)
+    group_kernel<kGroupSmallThreads><<<1, kGroupSmallThreads, 0, s>>>(rb, channels, n_groups, tau0_out,
+                                                                     exp_out, dev_status);
+  else
+    group_kernel<kGroupLargeThreads><<<1, kGroupLargeThreads, 0, s>>>(rb, channels, n_groups, tau0_out,
+                                                                     exp_out, dev_status);
   const cudaError_t err = cudaGetLastError();
   return err == cudaSuccess ? SQ_OK : cuda_fail(err, "group_kernel launch");
 }

@@ -8,12 +8,24 @@
 namespace sq {
 
 // SplitMix64 (Steele, Lea, Flood 2014): the (idx+1)-th output of the generator whose
-// state starts at `seed`.
+// state starts at `seed` is the output function applied to the state
+// seed + (idx+1) * gamma (mod 2^64).
+constexpr uint64_t kSplitMixGamma = 0x9E3779B97F4A7C15ull;
+
 __device__ __forceinline__ uint64_t splitmix64_at(uint64_t seed, uint64_t idx) {
-  uint64_t z = seed + (idx + 1ull) * 0x9E3779B97F4A7C15ull;
+  uint64_t z = seed + (idx + 1ull) * kSplitMixGamma;
   z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
   z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
   return z ^ (z >> 31);
+}
+
+// bits 40..63 of the output for the state z (= seed + (idx+1) gamma).  The final step
+// z ^ (z >> 31) leaves those bits as they are ((z >> 31) is zero above bit 32), so it is
+// skipped; the result equals splitmix64_at(seed, idx) >> 40.
+__device__ __forceinline__ uint32_t splitmix64_top24(uint64_t z) {
+  z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
+  z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+  return static_cast<uint32_t>(z >> 40);
 }
 
 __device__ __forceinline__ float pow2f(int k) { return __int_as_float((127 + k) << 23); }
