@@ -166,16 +166,11 @@ class Step:
                 ("quantize", lambda lay=lay, dy=dy, seed=seed: N.shiftquant_quantize(
                     dy, N.SQ_GRAN_SHIFT, lay.bits, lay.G, lay.g.tau0, lay.g.exp, None,
                     N.SQ_ROUND_STOCHASTIC, seed, lay.g.codes, lay.g.codes_t, lay.g.scale)),
-                ("calibrate", lambda lay=lay, w=w: N.shiftquant_calibrate(
-                    w, N.SQ_GRAN_PER_COL, lay.G, lay.wf.range, None, None, lay.status)),
-                ("quantize", lambda lay=lay, w=w: N.shiftquant_quantize(
-                    w, N.SQ_GRAN_PER_COL, lay.bits, lay.G, lay.wf.range, None, lay.x.exp,
-                    N.SQ_ROUND_NEAREST_EVEN, 0, None, lay.wf.codes, lay.wf.scale)),
-                ("calibrate", lambda lay=lay, w=w: N.shiftquant_calibrate(
-                    w, N.SQ_GRAN_PER_ROW, lay.G, lay.wd.range, None, None, lay.status)),
-                ("quantize", lambda lay=lay, w=w: N.shiftquant_quantize(
-                    w, N.SQ_GRAN_PER_ROW, lay.bits, lay.G, lay.wd.range, None, lay.g.exp,
-                    N.SQ_ROUND_NEAREST_EVEN, 0, lay.wd.codes, None, lay.wd.scale)),
+                ("calibrate", lambda lay=lay, w=w: N.shiftquant_calibrate_weight(
+                    w, lay.wf.range, lay.wd.range, lay.status)),
+                ("quantize", lambda lay=lay, w=w: N.shiftquant_quantize_weight(
+                    w, lay.bits, lay.G, lay.wf.range, lay.wd.range, lay.x.exp, lay.g.exp,
+                    lay.wf.codes, lay.wf.scale, lay.wd.codes, lay.wd.scale)),
                 ("gemm", lay.gemms),   # forward, loss propagation, weight gradient: one launch
             ]
         return out
@@ -188,8 +183,7 @@ class Step:
             MK, MN, KN = s.M * s.K, s.M * s.N, s.K * s.N
             out += [(s.name, "X", 4 * MK), (s.name, "X", 4 * MK + 2 * cb * MK),
                     (s.name, "dY", 4 * MN), (s.name, "dY", 4 * MN + 2 * cb * MN),
-                    (s.name, "W per out-channel", 4 * KN), (s.name, "W per out-channel", 4 * KN + cb * KN),
-                    (s.name, "W per in-channel", 4 * KN), (s.name, "W per in-channel", 4 * KN + cb * KN),
+                    (s.name, "W (both roles)", 4 * KN), (s.name, "W (both roles)", 4 * KN + 2 * cb * KN),
                     (s.name, "GEMMs", gb)]
         return out
 
@@ -207,8 +201,7 @@ class Step:
         N = self.N
         for lay in self.layers:
             n += 3 + 1 + 3 + 1          # X and dY: range init, range, grouping; quantize
-            n += 2 + 1 + 1 + 1          # weights: range init + range, quantize (out-channel);
-                                        # row range, quantize (in-channel)
+            n += 2 + 1                  # weight: range init, both ranges; both roles' codes
             # the three GEMMs: one launch, plus the output pass of each GEMM that splits K
             n += N.shiftquant_gemm_layer_kernel_launches(
                 lay.M, lay.K, lay.N, lay.bits, lay.G,
@@ -234,7 +227,7 @@ class Step:
 
     def range_bytes(self) -> int:
         """Algorithmic HBM bytes of the range passes of one step (4 B read per element)."""
-        return sum(4 * (s.M * s.K + s.M * s.N + 2 * s.K * s.N) for s in self.specs)
+        return sum(4 * (s.M * s.K + s.M * s.N + s.K * s.N) for s in self.specs)
 
     def quantize_bytes(self) -> int:
         """Algorithmic HBM bytes of the quantize passes of one step."""
@@ -243,7 +236,7 @@ class Step:
             cb = self.N.shiftquant_code_bytes(s.bits, s.n_groups)
             for R, C in ((s.M, s.K), (s.M, s.N)):        # X and dY: read, codes + transposed
                 tot += 4 * R * C + 2 * cb * R * C
-            tot += 2 * (4 * s.K * s.N + cb * s.K * s.N)   # W, two roles
+            tot += 4 * s.K * s.N + 2 * cb * s.K * s.N    # W: one read, both roles' codes
         return tot
 
     def quantizer_bytes(self) -> int:
@@ -328,9 +321,9 @@ def run_ours(args, rank, world, local_rank):
     assert st.status_ok(), "device status set during warm-up"
 
     # the timed step is the whole step captured in one CUDA graph: per layer, the activation
-    # chain, the gradient chain and the two weight roles on their own streams, then the
+    # chain, the gradient chain and the weight (both roles) each on its own stream, then the
     # layer's three GEMMs as one launch
-    streams = [[torch.cuda.Stream(device=dev) for _ in range(4)] for _ in st.layers]
+    streams = [[torch.cuda.Stream(device=dev) for _ in range(3)] for _ in st.layers]
 
     # A second capture of the same step with events around each layer's GEMM call (external
     # events are recorded as graph nodes) times the GEMM launches in graph replays; the
@@ -603,7 +596,7 @@ def run_ours(args, rank, world, local_rank):
         "quantizer_per_tensor_source": per_tensor_src,
         "group_histograms": st.group_histograms(),
         "timing": "CUDA events around one CUDA-graph replay of the whole step (per layer: "
-                  "activation chain, gradient chain and both weight roles on four streams, "
+                  "activation chain, gradient chain and the weight (both roles) on three streams, "
                   "then the three GEMMs as one launch); breakdown from un-graphed serial "
                   "calls (one launch per GEMM) queued behind a sleep kernel",
         "gpu_launches": st.launches_per_step() * args.steps,

@@ -136,6 +136,35 @@ sq_status shiftquant_quantize(const float *x, int64_t rows, int64_t cols, int64_
                               uint64_t seed, int64_t row0, void *codes, int64_t ld_codes,
                               void *codes_t, int64_t ld_t, float *scale_out, void *stream);
 
+/* Both weight roles of a layer (Sec. 5.1) in two passes over W instead of four: the
+ * range pass of the forward GEMM's per-out-channel scales and of loss propagation's
+ * per-in-channel scales (Sec. 3.1 channel ranges) from one read of W.
+ *   w [rows = K, ld] fp32 (rows: in-channels, cols: out-channels).
+ *   range_out_ch[cols] = max_r |w[r, c]|, range_in_ch[rows] = max_c |w[r, c]|: bit for bit
+ *     shiftquant_calibrate with SQ_GRAN_PER_COL and with SQ_GRAN_PER_ROW.
+ *   A NaN/Inf sets SQ_DEV_NONFINITE.  rows or cols == 0 gives zero ranges. */
+sq_status shiftquant_calibrate_weight(const float *w, int64_t rows, int64_t cols, int64_t ld,
+                                      float *range_out_ch, float *range_in_ch,
+                                      int32_t *dev_status, void *stream);
+
+/* Both weight roles quantized from one read of W (App. D quantizer, round to nearest even;
+ * Sec. 5.1 roles), with the ranges of shiftquant_calibrate_weight:
+ *   codes_fwd [cols, ld_fwd], scale_fwd[cols]: the forward GEMM's per-out-channel codes,
+ *     TRANSPOSED, with fold_fwd[rows] (the activation's exponents, or NULL) folded in --
+ *     bit for bit shiftquant_quantize(w, SQ_GRAN_PER_COL, ..., fold_exp = fold_fwd,
+ *     codes = NULL, codes_t = codes_fwd, ...).
+ *   codes_dgrad [rows, ld_dgrad], scale_dgrad[rows]: loss propagation's per-in-channel
+ *     codes with fold_dgrad[cols] (the gradient's exponents, or NULL) folded in -- bit for
+ *     bit shiftquant_quantize(w, SQ_GRAN_PER_ROW, ..., fold_exp = fold_dgrad,
+ *     codes = codes_dgrad, codes_t = NULL, ...).
+ *   rows or cols == 0 gives zero scales and writes no code. */
+sq_status shiftquant_quantize_weight(const float *w, int64_t rows, int64_t cols, int64_t ld,
+                                     int bits, int n_groups, const float *range_out_ch,
+                                     const float *range_in_ch, const uint8_t *fold_fwd,
+                                     const uint8_t *fold_dgrad, void *codes_fwd, int64_t ld_fwd,
+                                     float *scale_fwd, void *codes_dgrad, int64_t ld_dgrad,
+                                     float *scale_dgrad, void *stream);
+
 /* Group order of a GEMM inner index (Sec. 3.2's per-group GEMMs, done as one launch):
  * from exp[channels] (the exponents of shiftquant_calibrate / shiftquant_group), a stable
  * order with every group's channels contiguous and each group's segment starting on a
@@ -361,7 +390,8 @@ int shiftquant_gemm_layer_cta_pairs(int64_t M, int64_t K, int64_t N, int bits, i
  *   2. dY: the same with stochastic rounding (App. B) drawn under `seed`;
  *   3. W per out-channel (forward role): codes written transposed [N, K] with X's group
  *      shifts folded in; W per in-channel (loss-propagation role): codes [K, N] with dY's
- *      shifts folded in;
+ *      shifts folded in -- both roles by shiftquant_calibrate_weight and
+ *      shiftquant_quantize_weight;
  *   4. the forward, loss-propagation and weight-gradient GEMMs as one launch
  *      (shiftquant_gemm_layer).
  * Every buffer is a caller-owned DEVICE buffer; the layouts are those of the calls above:

@@ -406,9 +406,6 @@ __device__ __forceinline__ Unit decode_unit(const GemmParams& p, int u) {
   return r;
 }
 
-// kMulti: the K loop of a tile spans several exact chunks, whose int32 sums the epilogue
-// keeps in registers; otherwise every output streams from TMEM once.
-// the GEMM of global unit u, and u's index inside that GEMM
 // the GEMM of global unit u, and u's index inside that GEMM
 __device__ __forceinline__ int batch_member(const GemmBatch& bt, int u, int* local) {
   int g = 0;
@@ -580,6 +577,8 @@ __device__ __noinline__ void plan_chunks(const GemmBatch& bt, volatile int* out,
   }
 }
 
+// kMulti: the K loop of a tile spans several exact chunks, whose int32 sums the epilogue
+// keeps in registers; otherwise every output streams from TMEM once.
 // kPair: launched as 2-CTA clusters running 256-row tiles (the host sets the cluster shape)
 template <int kF8, bool kMulti, bool kPair>
 __global__ void __launch_bounds__(kThreads, 1) shiftmm_kernel(const __grid_constant__ GemmBatch bt) {

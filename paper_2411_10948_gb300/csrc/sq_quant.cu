@@ -64,15 +64,17 @@ __device__ __forceinline__ int group_exponent(float r, float tau, int G) {
   return e;
 }
 
-// zero the range accumulators (and the completion counter of the grouping step); the range
-// pass that follows may launch at once: it reads x first and these only after its wait
+// zero the range accumulators a[na] and b[nb] (b may be null); the range pass that follows
+// may launch at once: it reads x first and these only after its wait
 __global__ void __launch_bounds__(256)
-    calib_init_kernel(unsigned* __restrict__ range_bits, int64_t C, unsigned* __restrict__ counter) {
+    calib_init_kernel(unsigned* __restrict__ a, int64_t na, unsigned* __restrict__ b, int64_t nb) {
   griddep_launch_dependents();
-  for (int64_t c = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; c < C;
-       c += static_cast<int64_t>(gridDim.x) * blockDim.x)
-    range_bits[c] = 0u;
-  if (counter != nullptr && blockIdx.x == 0 && threadIdx.x == 0) *counter = 0u;
+  const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
+  for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < na; i += stride)
+    a[i] = 0u;
+  if (b != nullptr)
+    for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < nb; i += stride)
+      b[i] = 0u;
 }
 
 // Grouping (Eq. 3) by one block of THREADS threads from the per-channel range bits:
@@ -140,14 +142,18 @@ __global__ void __launch_bounds__(THREADS)
 // sends them on.  Wide tensors (CL = 1) spread their atomics over many addresses and run
 // without clusters, which schedule more slowly.  Grids taller than the 65535-block limit
 // walk the extra tiles in steps of gridDim.y.
+// ROWS: the range pass of a weight for both of its roles -- also every row's max|x| over
+// all columns (the per-in-channel ranges), each warp's eight rows of a tile reduced across
+// its lanes and sent to row_bits with one atomic max per row and column block.
 constexpr int kRangeRows = 64;
 constexpr int kRangeCluster = 8;
 constexpr int64_t kRangeClusterMaxCols = 4 * kColTx * 4;   // clusters up to 4 column blocks
 
-template <int CL>
+template <int CL, bool ROWS>
 __global__ void __launch_bounds__(kColTx* kColTy)
     colmax_kernel(const float* __restrict__ x, int64_t R, int64_t C, int64_t ld, int vec,
-                  unsigned* __restrict__ range_bits, int* __restrict__ status) {
+                  unsigned* __restrict__ range_bits, unsigned* __restrict__ row_bits,
+                  int* __restrict__ status) {
   __shared__ unsigned red[kColTy][kColTx * 4];
   __shared__ unsigned cmax[CL > 1 ? kColTx * 4 : 1];   // the cluster's maxima (first block)
   const int tx = threadIdx.x, ty = threadIdx.y;   // tx: lane (columns), ty: warp (rows)
@@ -159,9 +165,11 @@ __global__ void __launch_bounds__(kColTx* kColTy)
     cluster_arrive_release();   // the zeroed cmax is visible to the cluster after the wait
   }
   unsigned m0 = 0, m1 = 0, m2 = 0, m3 = 0;
+  bool row_bad = false;
 #pragma unroll 1
   for (int64_t t = blockIdx.y; t < tiles; t += gridDim.y) {
     const int64_t r0 = t * kRangeRows + ty * 8;
+    unsigned rm[8];   // ROWS: this thread's four columns of each of its rows
     if (vec && c0 + 3 < C) {
       // rows past the end re-read the last row, which leaves a maximum unchanged
       float4 v[8];
@@ -169,24 +177,51 @@ __global__ void __launch_bounds__(kColTx* kColTy)
       for (int u = 0; u < 8; ++u) v[u] = ld_stream_v4(x + min(r0 + u, R - 1) * ld + c0);
 #pragma unroll
       for (int u = 0; u < 8; ++u) {
-        m0 = max(m0, abs_bits(v[u].x));
-        m1 = max(m1, abs_bits(v[u].y));
-        m2 = max(m2, abs_bits(v[u].z));
-        m3 = max(m3, abs_bits(v[u].w));
+        const unsigned a0 = abs_bits(v[u].x), a1 = abs_bits(v[u].y);
+        const unsigned a2 = abs_bits(v[u].z), a3 = abs_bits(v[u].w);
+        m0 = max(m0, a0);
+        m1 = max(m1, a1);
+        m2 = max(m2, a2);
+        m3 = max(m3, a3);
+        if (ROWS) rm[u] = max(max(a0, a1), max(a2, a3));
       }
     } else {
+#pragma unroll
+      for (int u = 0; u < 8; ++u) rm[u] = 0u;
 #pragma unroll 1
       for (int u = 0; u < 8; ++u) {
         const int64_t r = r0 + u;
         if (r >= R) break;
         const float* row = x + r * ld;
-        if (c0 + 0 < C) m0 = max(m0, abs_bits(__ldg(row + c0 + 0)));
-        if (c0 + 1 < C) m1 = max(m1, abs_bits(__ldg(row + c0 + 1)));
-        if (c0 + 2 < C) m2 = max(m2, abs_bits(__ldg(row + c0 + 2)));
-        if (c0 + 3 < C) m3 = max(m3, abs_bits(__ldg(row + c0 + 3)));
+        unsigned a[4] = {0u, 0u, 0u, 0u};
+#pragma unroll
+        for (int k = 0; k < 4; ++k)
+          if (c0 + k < C) a[k] = abs_bits(__ldg(row + c0 + k));
+        m0 = max(m0, a[0]);
+        m1 = max(m1, a[1]);
+        m2 = max(m2, a[2]);
+        m3 = max(m3, a[3]);
+        if (ROWS) {
+#pragma unroll
+          for (int k = 0; k < 8; ++k)  // rm stays in registers: no run-time index
+            if (k == u) rm[k] = max(max(a[0], a[1]), max(a[2], a[3]));
+        }
+      }
+    }
+    if (ROWS) {
+      // the row accumulators are zeroed by the preceding kernel, which must have completed
+      griddep_wait();
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        const unsigned m = __reduce_max_sync(0xFFFFFFFFu, rm[u]);
+        if (tx == 0 && r0 + u < R && m != 0u) {
+          atomicMax(row_bits + r0 + u, m);
+          row_bad |= m >= 0x7F800000u;
+        }
       }
     }
   }
+  if (ROWS && row_bad) atomicOr(status, kDevNonFinite);
   // x has been read: the next kernel (the grouping) may start launching
   griddep_launch_dependents();
   red[ty][tx * 4 + 0] = m0;
@@ -623,6 +658,37 @@ static void launch_quantize(const QuantArgs& a, dim3 grid, cudaStream_t s) {
   }
 }
 
+// Both roles of a weight from one pass over it (Sec. 5.1): the forward GEMM's
+// per-out-channel codes (gran PER_COL, written transposed, the fold indexed by row) and loss
+// propagation's per-in-channel codes (gran PER_ROW, natural layout, the fold indexed by
+// column).  The second role re-reads the block's tile, which the first has just brought
+// into L2, so HBM sees one read of the weight.
+template <typename CodeT, bool FF, bool FD>
+__global__ void __launch_bounds__(256) quantize_weight_kernel(const QuantArgs af, const QuantArgs ad) {
+  __shared__ __align__(16) uint8_t tile_t[kQC * 8 * 8 * sizeof(CodeT)];
+  griddep_wait();
+  const bool inside = (static_cast<int64_t>(blockIdx.y) + 1) * kQR <= af.R &&
+                      (static_cast<int64_t>(blockIdx.x) + 1) * kQC <= af.C && af.vec_in;
+  if (inside && af.vec_t)
+    quantize_tile<CodeT, SQ_GRAN_PER_COL, SQ_ROUND_NEAREST_EVEN, FF, true>(af, tile_t);
+  else
+    quantize_tile<CodeT, SQ_GRAN_PER_COL, SQ_ROUND_NEAREST_EVEN, FF, false>(af, tile_t);
+  if (inside && ad.vec_out)
+    quantize_tile<CodeT, SQ_GRAN_PER_ROW, SQ_ROUND_NEAREST_EVEN, FD, true>(ad, tile_t);
+  else
+    quantize_tile<CodeT, SQ_GRAN_PER_ROW, SQ_ROUND_NEAREST_EVEN, FD, false>(ad, tile_t);
+}
+
+template <typename CodeT>
+static void launch_quantize_weight(const QuantArgs& af, const QuantArgs& ad, dim3 grid,
+                                   cudaStream_t s) {
+  const bool ff = af.fold != nullptr, fd = ad.fold != nullptr;
+  if (ff && fd) launch_pdl(quantize_weight_kernel<CodeT, true, true>, grid, dim3(256), s, af, ad);
+  else if (ff) launch_pdl(quantize_weight_kernel<CodeT, true, false>, grid, dim3(256), s, af, ad);
+  else if (fd) launch_pdl(quantize_weight_kernel<CodeT, false, true>, grid, dim3(256), s, af, ad);
+  else launch_pdl(quantize_weight_kernel<CodeT, false, false>, grid, dim3(256), s, af, ad);
+}
+
 // ============================================================ group order (Sec. 3.2)
 // The inner index of a forward or loss-propagation GEMM in group order: every group's
 // channels contiguous (stable: in channel order within a group), each group's segment
@@ -710,6 +776,48 @@ __global__ void __launch_bounds__(256)
   }
 }
 
+// The range pass of x [rows, cols] (0 < rows, 0 < cols < 2^36, checked by the callers):
+// one block per 64 x 128 tile, narrow tensors in whole clusters along the rows; with
+// row_bits also the per-row maxima.
+static cudaError_t launch_range(const float* x, int64_t rows, int64_t cols, int64_t ld,
+                                unsigned* col_bits, unsigned* row_bits, int* status,
+                                cudaStream_t s) {
+  const int64_t cblocks = (cols + kColTx * 4 - 1) / (kColTx * 4);   // <= 2^29: cols < 2^36
+  const int64_t tiles = (rows + kRangeRows - 1) / kRangeRows;
+  const int cl = cols <= kRangeClusterMaxCols ? kRangeCluster : 1;
+  const int64_t max_rblocks = 65535 / cl * cl;
+  int64_t rblocks = (tiles + cl - 1) / cl * cl;
+  if (rblocks > max_rblocks) rblocks = max_rblocks;
+  const int vec = (ld % 4 == 0) && aligned16(x);
+  cudaLaunchConfig_t cfg;
+  memset(&cfg, 0, sizeof(cfg));
+  cfg.gridDim = dim3(static_cast<unsigned>(cblocks), static_cast<unsigned>(rblocks));
+  cfg.blockDim = dim3(kColTx, kColTy);
+  cfg.stream = s;
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  attr[1].id = cudaLaunchAttributeClusterDimension;
+  attr[1].val.clusterDim.x = 1;
+  attr[1].val.clusterDim.y = cl;
+  attr[1].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = cl > 1 ? 2 : 1;
+  cudaError_t err;
+  if (row_bits != nullptr)
+    err = cl > 1 ? cudaLaunchKernelEx(&cfg, colmax_kernel<kRangeCluster, true>, x, rows, cols, ld, vec,
+                                      col_bits, row_bits, status)
+                 : cudaLaunchKernelEx(&cfg, colmax_kernel<1, true>, x, rows, cols, ld, vec, col_bits,
+                                      row_bits, status);
+  else
+    err = cl > 1 ? cudaLaunchKernelEx(&cfg, colmax_kernel<kRangeCluster, false>, x, rows, cols, ld, vec,
+                                      col_bits, row_bits, status)
+                 : cudaLaunchKernelEx(&cfg, colmax_kernel<1, false>, x, rows, cols, ld, vec, col_bits,
+                                      row_bits, status);
+  if (err == cudaSuccess) err = cudaGetLastError();
+  return err;
+}
+
 }  // namespace sq
 
 using namespace sq;
@@ -746,6 +854,7 @@ extern "C" sq_status shiftquant_calibrate(const float* x, int64_t rows, int64_t 
                                           int32_t* dev_status, void* stream) {
   clear_error();
   if (rows < 0 || cols < 0) return fail(SQ_EINVAL, "calibrate: negative size");
+  if (cols >= (int64_t(1) << 36)) return fail(SQ_EINVAL, "calibrate: too many columns");
   if (gran < SQ_GRAN_SHIFT || gran > SQ_GRAN_PER_ROW) return fail(SQ_EINVAL, "calibrate: bad gran %d", gran);
   if (gran == SQ_GRAN_SHIFT && !groups_ok(n_groups))
     return fail(SQ_EINVAL, "calibrate: n_groups must be in [1, 8]");
@@ -789,37 +898,12 @@ extern "C" sq_status shiftquant_calibrate(const float* x, int64_t rows, int64_t 
   {
     const int64_t iblocks = (cols + 255) / 256;
     calib_init_kernel<<<static_cast<unsigned>(iblocks < 1024 ? iblocks : 1024), 256, 0, s>>>(
-        reinterpret_cast<unsigned*>(range_out), cols, nullptr);
+        reinterpret_cast<unsigned*>(range_out), cols, nullptr, 0);
     err = cudaGetLastError();
     if (err != cudaSuccess) return cuda_fail(err, "calib_init_kernel launch");
   }
-  const int64_t cblocks = (cols + kColTx * 4 - 1) / (kColTx * 4);
-  const int64_t tiles = (rows + kRangeRows - 1) / kRangeRows;
-  if (cblocks > 0x7FFFFFFF) return fail(SQ_EINVAL, "calibrate: too many columns");
-  // one block per 64 x 128 tile; narrow tensors in whole clusters along the rows
-  const int cl = cols <= kRangeClusterMaxCols ? kRangeCluster : 1;
-  const int64_t max_rblocks = 65535 / cl * cl;
-  int64_t rblocks = (tiles + cl - 1) / cl * cl;
-  if (rblocks > max_rblocks) rblocks = max_rblocks;
-  const int vec = (ld % 4 == 0) && aligned16(x);
-  cudaLaunchConfig_t cfg;
-  memset(&cfg, 0, sizeof(cfg));
-  cfg.gridDim = dim3(static_cast<unsigned>(cblocks), static_cast<unsigned>(rblocks));
-  cfg.blockDim = dim3(kColTx, kColTy);
-  cfg.stream = s;
-  cudaLaunchAttribute attr[2];
-  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  attr[0].val.programmaticStreamSerializationAllowed = 1;
-  attr[1].id = cudaLaunchAttributeClusterDimension;
-  attr[1].val.clusterDim.x = 1;
-  attr[1].val.clusterDim.y = cl;
-  attr[1].val.clusterDim.z = 1;
-  cfg.attrs = attr;
-  cfg.numAttrs = cl > 1 ? 2 : 1;
   unsigned* bits = reinterpret_cast<unsigned*>(range_out);
-  err = cl > 1 ? cudaLaunchKernelEx(&cfg, colmax_kernel<kRangeCluster>, x, rows, cols, ld, vec, bits, dev_status)
-               : cudaLaunchKernelEx(&cfg, colmax_kernel<1>, x, rows, cols, ld, vec, bits, dev_status);
-  if (err == cudaSuccess) err = cudaGetLastError();
+  err = launch_range(x, rows, cols, ld, bits, nullptr, dev_status, s);
   if (err != cudaSuccess) return cuda_fail(err, "colmax_kernel launch");
   if (!shift) return SQ_OK;
   // grouping (Eq. 3) by one block behind the range pass
@@ -998,4 +1082,116 @@ extern "C" sq_status shiftquant_quantize_ordered(const float* x, int64_t rows, i
         static_cast<uint16_t*>(ordered), ord_rows, ord_ld, seg, n_groups);
   const cudaError_t err = cudaGetLastError();
   return err == cudaSuccess ? SQ_OK : cuda_fail(err, "order_pad_kernel launch");
+}
+
+extern "C" sq_status shiftquant_calibrate_weight(const float* w, int64_t rows, int64_t cols,
+                                                 int64_t ld, float* range_out_ch,
+                                                 float* range_in_ch, int32_t* dev_status,
+                                                 void* stream) {
+  clear_error();
+  if (rows < 0 || cols < 0) return fail(SQ_EINVAL, "calibrate_weight: negative size");
+  if (cols >= (int64_t(1) << 36)) return fail(SQ_EINVAL, "calibrate_weight: too many columns");
+  if (rows > 0 && cols > 0 && (w == nullptr || ld < cols))
+    return fail(SQ_EINVAL, "calibrate_weight: w is NULL or ld < cols");
+  if (dev_status == nullptr || (cols > 0 && range_out_ch == nullptr) ||
+      (rows > 0 && range_in_ch == nullptr))
+    return fail(SQ_EINVAL, "calibrate_weight: range_out_ch, range_in_ch and dev_status are required");
+  cudaStream_t s = as_stream(stream);
+  cudaError_t err;
+  if (rows == 0 || cols == 0) {
+    // every range is 0
+    if (cols > 0 && (err = cudaMemsetAsync(range_out_ch, 0, sizeof(float) * cols, s)) != cudaSuccess)
+      return cuda_fail(err, "cudaMemsetAsync");
+    if (rows > 0 && (err = cudaMemsetAsync(range_in_ch, 0, sizeof(float) * rows, s)) != cudaSuccess)
+      return cuda_fail(err, "cudaMemsetAsync");
+    return SQ_OK;
+  }
+  unsigned* cb = reinterpret_cast<unsigned*>(range_out_ch);
+  unsigned* rb = reinterpret_cast<unsigned*>(range_in_ch);
+  // Both ranges from one read.  On wide weights the blocks of one row tile run together and
+  // their per-row atomics (one per 128 columns) partly serialise; measured on a
+  // [4096, 11008] weight this pass (58 us) still beats a column pass plus a one-warp-per-row
+  // pass (34 + 30 us).
+  const int64_t n = rows > cols ? rows : cols;
+  const int64_t iblocks = (n + 255) / 256;
+  calib_init_kernel<<<static_cast<unsigned>(iblocks < 1024 ? iblocks : 1024), 256, 0, s>>>(
+      cb, cols, rb, rows);
+  err = cudaGetLastError();
+  if (err != cudaSuccess) return cuda_fail(err, "calib_init_kernel launch");
+  err = launch_range(w, rows, cols, ld, cb, rb, dev_status, s);
+  return err == cudaSuccess ? SQ_OK : cuda_fail(err, "colmax_kernel launch");
+}
+
+extern "C" sq_status shiftquant_quantize_weight(const float* w, int64_t rows, int64_t cols,
+                                                int64_t ld, int bits, int n_groups,
+                                                const float* range_out_ch, const float* range_in_ch,
+                                                const uint8_t* fold_fwd, const uint8_t* fold_dgrad,
+                                                void* codes_fwd, int64_t ld_fwd, float* scale_fwd,
+                                                void* codes_dgrad, int64_t ld_dgrad,
+                                                float* scale_dgrad, void* stream) {
+  clear_error();
+  if (!bits_ok(bits) || !groups_ok(n_groups))
+    return fail(SQ_EINVAL, "quantize_weight: bits must be in [2, 8] and n_groups in [1, 8]");
+  if (rows < 0 || cols < 0) return fail(SQ_EINVAL, "quantize_weight: negative size");
+  cudaStream_t s = as_stream(stream);
+  const int type = code_type(bits, n_groups);
+  const int cbytes = code_bytes(type);
+  if (rows == 0 || cols == 0) {
+    // every range is 0: the scales are 0 and there is no code to write
+    cudaError_t err;
+    if (cols > 0) {
+      if (scale_fwd == nullptr) return fail(SQ_EINVAL, "quantize_weight: scale_fwd is required");
+      if ((err = cudaMemsetAsync(scale_fwd, 0, sizeof(float) * cols, s)) != cudaSuccess)
+        return cuda_fail(err, "cudaMemsetAsync");
+    }
+    if (rows > 0) {
+      if (scale_dgrad == nullptr) return fail(SQ_EINVAL, "quantize_weight: scale_dgrad is required");
+      if ((err = cudaMemsetAsync(scale_dgrad, 0, sizeof(float) * rows, s)) != cudaSuccess)
+        return cuda_fail(err, "cudaMemsetAsync");
+    }
+    return SQ_OK;
+  }
+  if (w == nullptr || ld < cols) return fail(SQ_EINVAL, "quantize_weight: w is NULL or ld < cols");
+  if (range_out_ch == nullptr || range_in_ch == nullptr || scale_fwd == nullptr ||
+      scale_dgrad == nullptr || codes_fwd == nullptr || codes_dgrad == nullptr)
+    return fail(SQ_EINVAL, "quantize_weight: ranges, codes and scales of both roles are required");
+  if (ld_fwd < rows) return fail(SQ_EINVAL, "quantize_weight: ld_fwd < rows");
+  if (ld_dgrad < cols) return fail(SQ_EINVAL, "quantize_weight: ld_dgrad < cols");
+  QuantArgs af;
+  memset(&af, 0, sizeof(af));
+  af.x = w;
+  af.R = rows;
+  af.C = cols;
+  af.ld = ld;
+  af.gran = SQ_GRAN_PER_COL;
+  af.Q = q_of_bits(bits);
+  af.G = n_groups;
+  af.mode = SQ_ROUND_NEAREST_EVEN;
+  af.vec_in = (ld % 4 == 0) && aligned16(w);
+  QuantArgs ad = af;
+  af.rt = range_out_ch;
+  af.fold = fold_fwd;
+  af.codes_t = codes_fwd;
+  af.ldt = ld_fwd;
+  af.scale_out = scale_fwd;
+  af.vec_t = ((ld_fwd * cbytes) % 16 == 0) && aligned16(codes_fwd);
+  ad.gran = SQ_GRAN_PER_ROW;
+  ad.rt = range_in_ch;
+  ad.fold = fold_dgrad;
+  ad.codes = codes_dgrad;
+  ad.ldc = ld_dgrad;
+  ad.scale_out = scale_dgrad;
+  ad.vec_out = ((ld_dgrad * cbytes) % (4 * cbytes) == 0) &&
+               (reinterpret_cast<uintptr_t>(codes_dgrad) % (4 * cbytes) == 0);
+  const int64_t gx = (cols + kQC - 1) / kQC, gy = (rows + kQR - 1) / kQR;
+  if (gx > 0x7FFFFFFF || gy > 65535)
+    return fail(SQ_EUNSUPPORTED, "quantize_weight: tensor too large for one launch (%lld x %lld)",
+                static_cast<long long>(rows), static_cast<long long>(cols));
+  const dim3 grid(static_cast<unsigned>(gx), static_cast<unsigned>(gy));
+  if (type == SQ_CODE_E4M3)
+    launch_quantize_weight<uint8_t>(af, ad, grid, s);
+  else
+    launch_quantize_weight<uint16_t>(af, ad, grid, s);
+  const cudaError_t err = cudaGetLastError();
+  return err == cudaSuccess ? SQ_OK : cuda_fail(err, "quantize_weight_kernel launch");
 }

@@ -51,21 +51,15 @@ static int run_step(const sq_layer_step* L, uint64_t seed, void* s) {
                                 SQ_ROUND_STOCHASTIC, seed, 0, L->g_codes, L->ld_g, L->gt_codes,
                                 L->ld_gt, L->g_scale, s)) != SQ_OK)
     return st;
-  // weight, forward role: per out-channel (column), written transposed [N, K], X's shifts in
-  if ((st = shiftquant_calibrate(L->w, K, N, N, SQ_GRAN_PER_COL, G, L->wf_range, nullptr, nullptr,
-                                 L->dev_status, s)) != SQ_OK)
+  // weight, both roles from two passes over it: forward per out-channel (column), written
+  // transposed [N, K], X's shifts in; loss propagation per in-channel (row), natural layout,
+  // dY's shifts in
+  if ((st = shiftquant_calibrate_weight(L->w, K, N, N, L->wf_range, L->wd_range, L->dev_status,
+                                        s)) != SQ_OK)
     return st;
-  if ((st = shiftquant_quantize(L->w, K, N, N, SQ_GRAN_PER_COL, b, G, L->wf_range, nullptr,
-                                L->x_exp, SQ_ROUND_NEAREST_EVEN, 0, 0, nullptr, 0, L->wf_codes,
-                                L->ld_wf, L->wf_scale, s)) != SQ_OK)
-    return st;
-  // weight, loss-propagation role: per in-channel (row), natural layout, dY's shifts in
-  if ((st = shiftquant_calibrate(L->w, K, N, N, SQ_GRAN_PER_ROW, G, L->wd_range, nullptr, nullptr,
-                                 L->dev_status, s)) != SQ_OK)
-    return st;
-  if ((st = shiftquant_quantize(L->w, K, N, N, SQ_GRAN_PER_ROW, b, G, L->wd_range, nullptr,
-                                L->g_exp, SQ_ROUND_NEAREST_EVEN, 0, 0, L->wd_codes, L->ld_wd,
-                                nullptr, 0, L->wd_scale, s)) != SQ_OK)
+  if ((st = shiftquant_quantize_weight(L->w, K, N, N, b, G, L->wf_range, L->wd_range, L->x_exp,
+                                       L->g_exp, L->wf_codes, L->ld_wf, L->wf_scale, L->wd_codes,
+                                       L->ld_wd, L->wd_scale, s)) != SQ_OK)
     return st;
   // the three GEMMs, one persistent launch
   sq_layer_gemms g = {};

@@ -96,6 +96,15 @@ def weight_quantize_dgrad(w, out: ChannelTensor, fold_exp, bits, n_groups, statu
                           N.SQ_ROUND_NEAREST_EVEN, 0, out.codes, None, out.scale, stream)
 
 
+def weight_quantize_both(w, wf: ChannelTensor, wd: ChannelTensor, x_exp, g_exp, bits, n_groups,
+                         status, stream=None):
+    """Both roles of W [K, N] in two passes over it: the ranges of both from one read, then
+    both code sets from one read (the same codes as weight_quantize_fwd and _dgrad)."""
+    N.shiftquant_calibrate_weight(w, wf.range, wd.range, status, stream)
+    N.shiftquant_quantize_weight(w, bits, n_groups, wf.range, wd.range, x_exp, g_exp, wf.codes,
+                                 wf.scale, wd.codes, wd.scale, stream)
+
+
 class QuantLinear:
     """Buffers and calls of one quantized linear layer: X [M, K], W [K, N], dY [M, N]."""
 
@@ -178,8 +187,8 @@ class QuantLinear:
 
     def quantize_weights(self, w, stream=None):
         if not self.grouped:
-            weight_quantize_fwd(w, self.wf, self.x.exp, self.bits, self.G, self.status, stream)
-            weight_quantize_dgrad(w, self.wd, self.g.exp, self.bits, self.G, self.status, stream)
+            weight_quantize_both(w, self.wf, self.wd, self.x.exp, self.g.exp, self.bits, self.G,
+                                 self.status, stream)
             return
         # group-ordered weights carry no folded shift: each segment is shifted whole
         st, b, G = self.status, self.bits, self.G
@@ -239,10 +248,11 @@ class QuantLinear:
         self.wgrad(stream)
 
     def step_concurrent(self, x, w, dy, seed, streams, gemm_events=None, dgrad_ctas=0):
-        """The same step with its independent quantizer work on four streams forked from the
-        current one -- the activation chain, the gradient chain and each weight role (its
-        range pass right away, its quantization once the other operand's exponents exist) --
-        joined back before the three GEMMs run as one launch on the current stream.
+        """The same step with its independent quantizer work on three streams forked from the
+        current one -- the activation chain, the gradient chain and the weight (its range
+        pass right away, its quantization for both roles once both other operands'
+        exponents exist) -- joined back before the three GEMMs run as one launch on the
+        current stream.
         Capturable in a CUDA graph, which then runs the independent work concurrently.
         gemm_events: optional (start, end) CUDA events recorded around the GEMM call (for
         timing inside a captured graph they must be created with external=True).
@@ -251,8 +261,8 @@ class QuantLinear:
         operands exist, beside the activation chain; the forward and weight-gradient GEMMs
         follow as one launch."""
         main = torch.cuda.current_stream()
-        s_x, s_g, s_wf, s_wd = streams[:4]
-        for s in (s_x, s_g, s_wf, s_wd):
+        s_x, s_g, s_w = streams[:3]
+        for s in (s_x, s_g, s_w):
             s.wait_stream(main)
         ev = {k: torch.cuda.Event() for k in ("x_cal", "g_cal")}
         b, G, st = self.bits, self.G, self.status
@@ -263,23 +273,18 @@ class QuantLinear:
                 ev[cal].record(s_)
                 N.shiftquant_quantize(t, N.SQ_GRAN_SHIFT, b, G, q.tau0, q.exp, None, mode, sd,
                                       q.codes, q.codes_t, q.scale, s_)
-        with torch.cuda.stream(s_wf):
-            N.shiftquant_calibrate(w, N.SQ_GRAN_PER_COL, G, self.wf.range, None, None, st, s_wf)
-            s_wf.wait_event(ev["x_cal"])
-            N.shiftquant_quantize(w, N.SQ_GRAN_PER_COL, b, G, self.wf.range, None, self.x.exp,
-                                  N.SQ_ROUND_NEAREST_EVEN, 0, None, self.wf.codes, self.wf.scale,
-                                  s_wf)
-        with torch.cuda.stream(s_wd):
-            N.shiftquant_calibrate(w, N.SQ_GRAN_PER_ROW, G, self.wd.range, None, None, st, s_wd)
-            s_wd.wait_event(ev["g_cal"])
-            N.shiftquant_quantize(w, N.SQ_GRAN_PER_ROW, b, G, self.wd.range, None, self.g.exp,
-                                  N.SQ_ROUND_NEAREST_EVEN, 0, self.wd.codes, None, self.wd.scale,
-                                  s_wd)
+        with torch.cuda.stream(s_w):
+            N.shiftquant_calibrate_weight(w, self.wf.range, self.wd.range, st, s_w)
+            s_w.wait_event(ev["x_cal"])
+            s_w.wait_event(ev["g_cal"])
+            N.shiftquant_quantize_weight(w, b, G, self.wf.range, self.wd.range, self.x.exp,
+                                         self.g.exp, self.wf.codes, self.wf.scale, self.wd.codes,
+                                         self.wd.scale, s_w)
         if dgrad_ctas > 0:
             with torch.cuda.stream(s_g):
-                s_g.wait_stream(s_wd)
+                s_g.wait_stream(s_w)
                 self.gemms(s_g, gemm_mask=2, max_ctas=dgrad_ctas, use_workspace=False)
-            for s in (s_x, s_wf, s_wd):
+            for s in (s_x, s_w):
                 main.wait_stream(s)
             if gemm_events is not None:
                 gemm_events[0].record(main)
@@ -288,7 +293,7 @@ class QuantLinear:
                 gemm_events[1].record(main)
             main.wait_stream(s_g)
             return
-        for s in (s_x, s_g, s_wf, s_wd):
+        for s in (s_x, s_g, s_w):
             main.wait_stream(s)
         if gemm_events is not None:
             gemm_events[0].record(main)

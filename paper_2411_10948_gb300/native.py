@@ -32,7 +32,8 @@ SQ_CODE_BF16 = 1
 # every symbol declared in include/shiftquant.h
 EXPORTS = (
     "shiftquant_code_type", "shiftquant_code_bytes", "shiftquant_calibrate",
-    "shiftquant_group", "shiftquant_quantize", "shiftquant_gemm_fwd", "shiftquant_gemm_dgrad",
+    "shiftquant_group", "shiftquant_quantize", "shiftquant_calibrate_weight",
+    "shiftquant_quantize_weight", "shiftquant_gemm_fwd", "shiftquant_gemm_dgrad",
     "shiftquant_gemm_wgrad", "shiftquant_gemm_wgrad_partial", "shiftquant_gemm_wgrad_finish",
     "shiftquant_gemm_wgrad_static", "shiftquant_gemm_workspace_bytes",
     "shiftquant_gemm_layer", "shiftquant_gemm_layer_workspace_bytes",
@@ -128,6 +129,11 @@ def load(path: str | None = None) -> ctypes.CDLL:
     lib.shiftquant_calibrate.restype = i32
     lib.shiftquant_group.argtypes = [vp, i64, i32, vp, vp, vp, vp]
     lib.shiftquant_group.restype = i32
+    lib.shiftquant_calibrate_weight.argtypes = [vp, i64, i64, i64, vp, vp, vp, vp]
+    lib.shiftquant_calibrate_weight.restype = i32
+    lib.shiftquant_quantize_weight.argtypes = [vp, i64, i64, i64, i32, i32, vp, vp, vp, vp, vp,
+                                               i64, vp, vp, i64, vp, vp]
+    lib.shiftquant_quantize_weight.restype = i32
     lib.shiftquant_gemm_wgrad_partial.argtypes = [vp, i64, vp, vp, vp, i64, vp, vp, i64, i64, i64,
                                                   i64, i32, i32, vp, vp, vp]
     lib.shiftquant_gemm_wgrad_partial.restype = i32
@@ -265,6 +271,26 @@ def shiftquant_quantize(x, gran, bits, n_groups, range_or_tau0, exp, fold_exp, m
         _ptr(exp), _ptr(fold_exp), mode, seed & (2**64 - 1), row0, _ptr(codes),
         _ld(codes) if codes is not None else 0, _ptr(codes_t),
         _ld(codes_t) if codes_t is not None else 0, _ptr(scale_out), _stream(stream)))
+
+
+def shiftquant_calibrate_weight(w, range_out_ch, range_in_ch, dev_status, stream=None) -> None:
+    """Both weight ranges (per out-channel and per in-channel) from one read of w [K, N]."""
+    _check(load().shiftquant_calibrate_weight(_ptr(w), w.shape[0], w.shape[1], _ld(w),
+                                              _ptr(range_out_ch), _ptr(range_in_ch),
+                                              _ptr(dev_status), _stream(stream)))
+
+
+def shiftquant_quantize_weight(w, bits, n_groups, range_out_ch, range_in_ch, fold_fwd,
+                               fold_dgrad, codes_fwd, scale_fwd, codes_dgrad, scale_dgrad,
+                               stream=None) -> None:
+    """Both weight roles from one read of w [K, N]: codes_fwd [N, K] (per out-channel,
+    transposed) and codes_dgrad [K, N] (per in-channel)."""
+    _check(load().shiftquant_quantize_weight(
+        _ptr(w), w.shape[0], w.shape[1], _ld(w), bits, n_groups, _ptr(range_out_ch),
+        _ptr(range_in_ch), _ptr(fold_fwd), _ptr(fold_dgrad), _ptr(codes_fwd),
+        _ld(codes_fwd) if codes_fwd is not None else 0, _ptr(scale_fwd), _ptr(codes_dgrad),
+        _ld(codes_dgrad) if codes_dgrad is not None else 0, _ptr(scale_dgrad),
+        _stream(stream)))
 
 
 def _gemm(fn, a, a_scale, b, b_scale, M, N, K, bits, n_groups, y, acc, workspace, dev_status,

@@ -74,6 +74,21 @@ def test_host_validation_rejects_before_launch(lib):
     assert lib.shiftquant_calibrate(st, 4, 4, 4, 0, 4, st, None, st, st, None) == native.SQ_EINVAL
     # ld < cols
     assert lib.shiftquant_calibrate(st, 4, 8, 4, 0, 4, st, st, st, st, None) == native.SQ_EINVAL
+    # both weight roles: negative sizes, ld < cols, missing outputs, bad bits
+    assert lib.shiftquant_calibrate_weight(st, -1, 4, 4, st, st, st, None) == native.SQ_EINVAL
+    assert lib.shiftquant_calibrate_weight(st, 4, 8, 4, st, st, st, None) == native.SQ_EINVAL
+    assert lib.shiftquant_calibrate_weight(st, 4, 4, 4, st, None, st, None) == native.SQ_EINVAL
+    assert lib.shiftquant_calibrate_weight(st, 4, 4, 4, st, st, None, None) == native.SQ_EINVAL
+    assert lib.shiftquant_quantize_weight(st, 4, 4, 4, 9, 4, st, st, None, None, st, 16, st, st,
+                                          16, st, None) == native.SQ_EINVAL
+    assert lib.shiftquant_quantize_weight(st, 4, 4, 4, 4, 4, st, st, None, None, None, 16, st,
+                                          st, 16, st, None) == native.SQ_EINVAL
+    assert lib.shiftquant_quantize_weight(st, 4, 4, 4, 4, 4, st, st, None, None, st, 2, st, st,
+                                          16, st, None) == native.SQ_EINVAL   # ld_fwd < rows
+    assert lib.shiftquant_quantize_weight(st, 4, 4, 4, 4, 4, st, st, None, None, st, 16, st, st,
+                                          2, st, None) == native.SQ_EINVAL    # ld_dgrad < cols
+    assert lib.shiftquant_quantize_weight(st, -4, 4, 4, 4, 4, st, st, None, None, st, 16, st, st,
+                                          16, st, None) == native.SQ_EINVAL
     # quantize: bits, rounding mode, SHIFT with fold_exp, no outputs
     args = dict(x=st, rows=4, cols=4, ld=4, gran=0, bits=4, g=4, rt=st, exp=st, fold=None,
                 mode=0, seed=0, row0=0, codes=st, ldc=16, codes_t=None, ldt=0, scale=st,

@@ -155,6 +155,69 @@ def test_weight_quantization_with_fold(shape, bits, G):
     np.testing.assert_array_equal(decode(d.codes), folded(od["codes"], eg, G, axis=1))
 
 
+def both_roles(w_np, bits, G, ex, eg, ld=None):
+    """Both weight roles by shiftquant_calibrate_weight + shiftquant_quantize_weight."""
+    K, Nn = w_np.shape
+    wg = to_gpu(w_np, ld) if w_np.size else torch.zeros((K, Nn), device="cuda")
+    status = torch.zeros(1, dtype=torch.int32, device="cuda")
+    f = L.ChannelTensor(L.empty_codes(Nn, K, bits, G, "cuda"), torch.zeros(max(Nn, 1), device="cuda")[:Nn],
+                        torch.full((max(Nn, 1),), 7.0, device="cuda")[:Nn])
+    d = L.ChannelTensor(L.empty_codes(K, Nn, bits, G, "cuda"), torch.zeros(max(K, 1), device="cuda")[:K],
+                        torch.full((max(K, 1),), 7.0, device="cuda")[:K])
+    L.weight_quantize_both(wg, f, d, None if ex is None else torch.from_numpy(ex).cuda(),
+                           None if eg is None else torch.from_numpy(eg).cuda(), bits, G, status)
+    torch.cuda.synchronize()
+    return f, d, int(status.item())
+
+
+@pytest.mark.parametrize("shape", [(1, 1), (70, 33), (300, 257), (2304, 256), (129, 1031),
+                                   (64, 600), (1000, 96)])
+@pytest.mark.parametrize("bits,G", [(4, 4), (6, 4), (8, 4), (4, 7)])
+@pytest.mark.parametrize("fold", [True, False])
+def test_weight_both_roles_from_one_pass(shape, bits, G, fold):
+    """The fused weight quantizer (one range pass, one quantize pass for both roles) gives
+    the oracle's per-column and per-row ranges, scales and folded codes bit for bit."""
+    rng = np.random.default_rng(shape[0] * 7 + shape[1] + bits)
+    K, Nn = shape
+    w = (rng.standard_normal((K, Nn)) * np.exp(rng.normal(0, 1, Nn)) * 0.02).astype(np.float32)
+    w[:, 0] = 0                      # a zero out-channel
+    w[K // 2, :] = 0                 # a zero in-channel
+    ex = rng.integers(0, G, K).astype(np.uint8) if fold else None
+    eg = rng.integers(0, G, Nn).astype(np.uint8) if fold else None
+    # with the fold: dense rows; without: rows padded to an odd length (scalar loads)
+    f, d, st = both_roles(w, bits, G, ex, eg, ld=None if fold else Nn + 1)
+    assert st == 0
+    of = O.channel_tensor(w, bits, axis=0)
+    od = O.channel_tensor(w, bits, axis=1)
+    zx = np.full(K, G - 1, np.uint8) if ex is None else ex    # no fold: shift 2^0
+    zg = np.full(Nn, G - 1, np.uint8) if eg is None else eg
+    np.testing.assert_array_equal(f32_bits(f.range.cpu().numpy()), f32_bits(of["range"]))
+    np.testing.assert_array_equal(f32_bits(f.scale.cpu().numpy()), f32_bits(of["scale"]))
+    np.testing.assert_array_equal(decode(f.codes), folded(of["codes"], zx, G, axis=0).T)
+    np.testing.assert_array_equal(f32_bits(d.range.cpu().numpy()), f32_bits(od["range"]))
+    np.testing.assert_array_equal(f32_bits(d.scale.cpu().numpy()), f32_bits(od["scale"]))
+    np.testing.assert_array_equal(decode(d.codes), folded(od["codes"], zg, G, axis=1))
+
+
+@pytest.mark.parametrize("bad", [np.nan, np.inf])
+def test_weight_both_roles_nonfinite(bad):
+    w = np.full((40, 300), 0.01, np.float32)
+    w[13, 200] = bad
+    f, d, st = both_roles(w, 4, 4, None, None)
+    assert st & N.SQ_DEV_NONFINITE
+    fr, dr = f.range.cpu().numpy(), d.range.cpu().numpy()
+    assert not np.isfinite(fr[200]) and not np.isfinite(dr[13])
+    assert np.isfinite(np.delete(fr, 200)).all() and np.isfinite(np.delete(dr, 13)).all()
+
+
+def test_weight_both_roles_empty():
+    for K, Nn in ((0, 5), (5, 0)):
+        f, d, st = both_roles(np.zeros((K, Nn), np.float32), 4, 4, None, None)
+        assert st == 0
+        assert (f.range.cpu().numpy() == 0).all() and (f.scale.cpu().numpy() == 0).all()
+        assert (d.range.cpu().numpy() == 0).all() and (d.scale.cpu().numpy() == 0).all()
+
+
 @pytest.mark.parametrize("mode", [N.SQ_ROUND_NEAREST_EVEN, N.SQ_ROUND_STOCHASTIC])
 @pytest.mark.parametrize("bits", [4, 6])
 def test_row_shards_quantize_as_the_whole_tensor(mode, bits):
