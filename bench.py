@@ -663,9 +663,10 @@ L1BN_FWD_BYTES, L1BN_BWD_BYTES = 15, 16
 
 def run_l1bn(args, dev):
     """The fully-quantized L1 batch normalization (8-bit, N_G = 4) on ResNet-shaped
-    activations: forward and backward each timed with CUDA events after an L2 flush
-    (median), against HBM."""
+    activations: forward and backward each captured in a CUDA graph and timed with CUDA
+    events around a replay after an L2 flush (median), against HBM."""
     import torch
+    from paper_2411_10948_gb300 import layer as L
     from paper_2411_10948_gb300 import native as N
     from paper_2411_10948_gb300 import workloads as W
     peaks, src = load_peaks()
@@ -681,8 +682,10 @@ def run_l1bn(args, dev):
         dg, db = torch.empty(C, device=dev), torch.empty(C, device=dev)
         st = torch.zeros(1, dtype=torch.int32, device=dev)
         state = torch.zeros(N.shiftquant_l1bn_state_bytes(R, C), dtype=torch.uint8, device=dev)
-        fwd = lambda: N.shiftquant_l1bn_forward(x, gamma, beta, 8, 4, y, state, st)
-        bwd = lambda: N.shiftquant_l1bn_backward(dy, 8, 4, 0x5EED, state, dx, dg, db, st)
+        fwd_call = lambda: N.shiftquant_l1bn_forward(x, gamma, beta, 8, 4, y, state, st)
+        bwd_call = lambda: N.shiftquant_l1bn_backward(dy, 8, 4, 0x5EED, state, dx, dg, db, st)
+        fwd_graph, bwd_graph = L.CapturedStep(fwd_call), L.CapturedStep(bwd_call)
+        fwd, bwd = fwd_graph.replay, bwd_graph.replay
         for _ in range(3):
             fwd()
             bwd()
@@ -702,11 +705,11 @@ def run_l1bn(args, dev):
         bg = L1BN_BWD_BYTES * R * C / (bm * 1e-3) / 1e9
         out.append({"shape": name, "rows": R, "channels": C, "fwd_ms": fm, "bwd_ms": bm,
                     "fwd_gbs": fg, "bwd_gbs": bg, "fwd_frac": fg / peaks["hbm_gbs"],
-                    "bwd_frac": bg / peaks["hbm_gbs"], "launches": {"fwd": 6, "bwd": 5}})
+                    "bwd_frac": bg / peaks["hbm_gbs"], "launches": {"fwd": 7, "bwd": 6}})
     return {"bits": 8, "n_groups": 4, "bytes_per_element": {"fwd": L1BN_FWD_BYTES,
                                                            "bwd": L1BN_BWD_BYTES},
             "peak": peaks["hbm_gbs"], "peak_source": f"{src} copy bandwidth",
-            "statistic": "median over L2-flushed calls", "shapes": out}
+            "statistic": "median over graph replays after an L2 flush", "shapes": out}
 
 
 def run_group_order(args, dev):

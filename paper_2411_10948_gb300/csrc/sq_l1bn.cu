@@ -15,11 +15,16 @@
 // p (q - m)); each binary32 step is one IEEE operation in a fixed order (this file compiles
 // with -fmad=false), so the results are reproducible bit for bit.
 //
-// Kernels, all streaming HBM passes: a column-reduction pass that quantizes and sums
-// (128 columns x a slab of rows per block, four columns per thread with 16-byte loads,
-// sums combined across warps in shared memory and across blocks with 64-bit atomics), a
-// second reduction over the 1-byte codes for the deviation sums, a one-block pass for the
-// per-channel values, and an elementwise output pass (four outputs per thread).
+// Kernels, all streaming HBM passes over a tile of TC columns (the channel count rounded
+// up to a power of two, at most 128) whose 256 threads each own one four-column quad and
+// every (1024 / TC)-th row, with 8 (fp32) or 16 (code) loads in flight: a column-reduction
+// pass that quantizes and sums, a second reduction over the 1-byte codes for the deviation
+// sums, a one-block pass for the per-channel values, and an elementwise output pass whose
+// threads keep their quad's per-channel constants in registers.  Channel sums go from
+// shared memory to global 64-bit atomics into one of kSpread slots per sum (the block row
+// modulo kSpread), so that same-address atomics from hundreds of blocks do not serialise;
+// readers add the slots.  Every kernel after the range pass is launched behind the one
+// before it (programmatic stream serialization).
 #include <cuda_runtime.h>
 
 #include <cstring>
@@ -35,14 +40,20 @@ enum {
   kChXRange, kChGRange, kChS, kChM, kChSig, kChSq, kChGq, kChBq, kChT, kChU, kChMg, kChMgx,
   kChZs, kNumChan
 };
-// per-channel int64 sums of the state
+// per-channel int64 sums of the state, each kept in kSpread slots (block row y adds to slot
+// y mod kSpread, so that same-address atomics from many blocks do not serialise; a reader
+// adds the slots)
 enum { kStS1, kStS, kStZ, kStP, kStD, kNumStats };
+constexpr int kSpread = 8;
 // scalars of the state
 enum { kScXTau, kScXScale, kScGTau, kScGScale, kNumScal };
 
 struct L1bnLayout {
-  size_t xq, gq, stats, chan, exps, scal, total;
+  size_t xq, gq, stats, chan, lut, exps, scal, total;
 };
+
+// the forward output of every code value per channel: lut[c][q + 127]
+constexpr int kLutStride = 256;
 
 static L1bnLayout l1bn_layout(int64_t R, int64_t C) {
   auto up = [](size_t n) { return (n + 255) & ~size_t(255); };
@@ -51,8 +62,9 @@ static L1bnLayout l1bn_layout(int64_t R, int64_t C) {
   size_t o = 0;
   L.xq = o;    o += up(n);
   L.gq = o;    o += up(n);
-  L.stats = o; o += up(kNumStats * static_cast<size_t>(C) * sizeof(long long));
+  L.stats = o; o += up(kNumStats * kSpread * static_cast<size_t>(C) * sizeof(long long));
   L.chan = o;  o += up(kNumChan * static_cast<size_t>(C) * sizeof(float));
+  L.lut = o;   o += up(kLutStride * static_cast<size_t>(C) * sizeof(float));
   L.exps = o;  o += up(2 * static_cast<size_t>(C));
   L.scal = o;  o += 256;
   L.total = o;
@@ -67,8 +79,9 @@ struct L1bnArgs {
   float* out;       // y or dx
   int8_t* xq;
   int8_t* gq;
-  long long* st;  // [kNumStats][C]
+  long long* st;  // [kNumStats][kSpread][C]
   float* ch;      // [kNumChan][C]
+  float* lut;     // [C][kLutStride]
   uint8_t* xe;
   uint8_t* ge;
   float* scal;
@@ -79,8 +92,10 @@ struct L1bnArgs {
   int vec_in, vec_out;  // 16-byte rows: four elements per load / store
 };
 
-constexpr int kL1Cols = 128;  // columns of a reduction block (four per lane)
 constexpr int kL1Threads = 256;
+constexpr int kL1MaxCols = 128;   // widest tile: 32 quads
+constexpr int kL1PassesF32 = 4;    // rows in flight per thread in the passes that read fp32
+constexpr int kL1PassesCodes = 8;  // ... and in those that read only codes
 
 __device__ __forceinline__ long long rne_div(long long a, long long b) {
   long long q = a / b, r = a % b;
@@ -92,134 +107,244 @@ __device__ __forceinline__ long long rne_div(long long a, long long b) {
   return q;
 }
 
-// four consecutive elements of row r from column c (zeros past C)
-__device__ __forceinline__ void load4(const float* row, int64_t c, int64_t C, bool vec, float v[4]) {
+// channel sum k of column c: its slots added
+__device__ __forceinline__ long long stat_sum(const long long* st, int k, int64_t C, int64_t c) {
+  long long v = 0;
+#pragma unroll
+  for (int i = 0; i < kSpread; ++i) v += st[(static_cast<int64_t>(k) * kSpread + i) * C + c];
+  return v;
+}
+
+// the slot row of statistic k that block row y adds to
+__device__ __forceinline__ long long* stat_slot(long long* st, int k, int64_t C) {
+  return st + (static_cast<int64_t>(k) * kSpread + blockIdx.y % kSpread) * C;
+}
+
+// The thread's place in a tile: its quad (four consecutive columns) and its first row.
+struct TilePos {
+  int tc;        // tile columns: 4 << lg
+  int rpp;       // rows per pass: 256 / (tc / 4)
+  int qc, ro;    // this thread's quad and row offset
+  int64_t c;     // its first column
+};
+
+__device__ __forceinline__ TilePos tile_pos(int lg) {
+  TilePos t;
+  t.tc = 4 << lg;
+  t.rpp = kL1Threads >> lg;
+  t.qc = threadIdx.x & ((1 << lg) - 1);
+  t.ro = threadIdx.x >> lg;
+  t.c = static_cast<int64_t>(blockIdx.x) * t.tc + 4 * t.qc;
+  return t;
+}
+
+// the four elements of a quad at p (its first column c; zeros past C)
+__device__ __forceinline__ void load4(const float* p, int64_t c, int64_t C, bool vec, float v[4]) {
   if (vec && c + 3 < C) {
-    const float4 t = __ldg(reinterpret_cast<const float4*>(row + c));
+    const float4 t = ld_stream_v4(p);
     v[0] = t.x; v[1] = t.y; v[2] = t.z; v[3] = t.w;
   } else {
 #pragma unroll
-    for (int j = 0; j < 4; ++j) v[j] = c + j < C ? __ldg(row + c + j) : 0.0f;
+    for (int j = 0; j < 4; ++j) v[j] = c + j < C ? __ldg(p + j) : 0.0f;
   }
 }
 
-__device__ __forceinline__ void load_codes4(const int8_t* codes, int64_t off, int64_t c, int64_t C,
-                                            int q[4]) {
-  if ((C & 3) == 0) {
-    const char4 t = *reinterpret_cast<const char4*>(codes + off);
-    q[0] = t.x; q[1] = t.y; q[2] = t.z; q[3] = t.w;
-  } else {
+// the four codes of a quad at p packed in one word, byte j = column c + j (zeros past C)
+__device__ __forceinline__ uint32_t load_codes_w(const int8_t* p, int64_t c, int64_t C) {
+  if ((C & 3) == 0) return __ldg(reinterpret_cast<const unsigned int*>(p));
+  uint32_t w = 0;
 #pragma unroll
-    for (int j = 0; j < 4; ++j) q[j] = c + j < C ? codes[off + j] : 0;
-  }
+  for (int j = 0; j < 4; ++j)
+    if (c + j < C) w |= static_cast<uint32_t>(static_cast<uint8_t>(p[j])) << (8 * j);
+  return w;
 }
 
-__device__ __forceinline__ void store_codes4(int8_t* codes, int64_t off, int64_t c, int64_t C,
-                                             const int q[4]) {
+__device__ __forceinline__ int code_at(uint32_t w, int j) {
+  return static_cast<int>(static_cast<int8_t>(static_cast<uint8_t>(w >> (8 * j))));
+}
+
+__device__ __forceinline__ void store_codes4(int8_t* p, int64_t c, int64_t C, const int q[4]) {
   if ((C & 3) == 0) {
-    *reinterpret_cast<char4*>(codes + off) = make_char4(static_cast<signed char>(q[0]),
-                                                        static_cast<signed char>(q[1]),
-                                                        static_cast<signed char>(q[2]),
-                                                        static_cast<signed char>(q[3]));
+    *reinterpret_cast<char4*>(p) = make_char4(static_cast<signed char>(q[0]), static_cast<signed char>(q[1]),
+                                              static_cast<signed char>(q[2]), static_cast<signed char>(q[3]));
   } else {
 #pragma unroll
     for (int j = 0; j < 4; ++j)
-      if (c + j < C) codes[off + j] = static_cast<int8_t>(q[j]);
+      if (c + j < C) p[j] = static_cast<int8_t>(q[j]);
   }
 }
 
-// Per-block column sums -> global: each thread holds sums of its four columns over its
-// rows; the eight warps combine in shared memory and 128 threads add one column each.
-template <typename T>
-__device__ __forceinline__ void add_columns(const T (&acc)[4], long long* dst, int64_t c0,
-                                            int64_t C, T* red) {
-  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+__device__ __forceinline__ void store4(float* p, int64_t c, int64_t C, bool vec, const float y[4]) {
+  if (vec && c + 3 < C) {
+    *reinterpret_cast<float4*>(p) = make_float4(y[0], y[1], y[2], y[3]);
+  } else {
 #pragma unroll
-  for (int j = 0; j < 4; ++j) red[w * kL1Cols + lane * 4 + j] = acc[j];
+    for (int j = 0; j < 4; ++j)
+      if (c + j < C) p[j] = y[j];
+  }
+}
+
+// The rows of a thread: block row y takes rows y rpp + ro, then every S = gridDim.y rpp-th
+// row after it; U of them are in flight per step (their loads first, then their work).
+struct RowWalk {
+  int64_t r, S;
+};
+
+__device__ __forceinline__ RowWalk row_walk(const TilePos& t) {
+  RowWalk w;
+  w.r = static_cast<int64_t>(blockIdx.y) * t.rpp + t.ro;
+  w.S = static_cast<int64_t>(gridDim.y) * t.rpp;
+  return w;
+}
+
+// Shared memory of a reduction block: every thread's NS x 4 partial sums.
+template <int NS>
+struct RedSmem {
+  long long part[NS][kL1Threads * 4];
+};
+
+// The block's column sums of NS statistics -> global (dst[k]: the block's slot row of
+// statistic k): acc[k][j] is this thread's sum over its rows for column t.c + j.
+template <int NS>
+__device__ __forceinline__ void red_end(const long long (&acc)[NS][4], long long* const (&dst)[NS],
+                                        const TilePos& t, int64_t C, RedSmem<NS>& sm) {
+#pragma unroll
+  for (int k = 0; k < NS; ++k)
+#pragma unroll
+    for (int j = 0; j < 4; ++j) sm.part[k][t.ro * t.tc + t.qc * 4 + j] = acc[k][j];
   __syncthreads();
-  if (threadIdx.x < kL1Cols) {
-    long long s = 0;
+  const int tid = threadIdx.x;
+  long long tot[NS];
 #pragma unroll
-    for (int k = 0; k < kL1Threads / 32; ++k) s += static_cast<long long>(red[k * kL1Cols + threadIdx.x]);
-    const int64_t c = c0 + threadIdx.x;
-    if (c < C && s != 0)
-      atomicAdd(reinterpret_cast<unsigned long long*>(dst + c), static_cast<unsigned long long>(s));
+  for (int k = 0; k < NS; ++k) {
+    tot[k] = 0;
+    if (tid < t.tc)
+      for (int r = 0; r < t.rpp; ++r) tot[k] += sm.part[k][r * t.tc + tid];
   }
-}
-
-// rows of this block: [r0, r1); the block's warps take rows r0 + w, r0 + w + 8, ...
-__device__ __forceinline__ void block_rows(int64_t R, int64_t* r0, int64_t* r1) {
-  const int64_t per = (R + gridDim.y - 1) / gridDim.y;
-  *r0 = static_cast<int64_t>(blockIdx.y) * per;
-  *r1 = min(R, *r0 + per);
+  const int64_t c = static_cast<int64_t>(blockIdx.x) * t.tc + tid;
+  if (tid < t.tc && c < C) {
+#pragma unroll
+    for (int k = 0; k < NS; ++k)
+      if (tot[k] != 0)
+        atomicAdd(reinterpret_cast<unsigned long long*>(dst[k] + c), static_cast<unsigned long long>(tot[k]));
+  }
 }
 
 // Forward pass 1: x -> int8 ShiftQuant codes (round to nearest), sum of codes per channel.
-__global__ void __launch_bounds__(kL1Threads) l1bn_fwd_quant_kernel(const L1bnArgs a) {
-  __shared__ int red[kL1Threads / 32 * kL1Cols];
-  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
-  const int64_t c0 = static_cast<int64_t>(blockIdx.x) * kL1Cols;
-  const int64_t c = c0 + lane * 4;
+__global__ void __launch_bounds__(kL1Threads, 3) l1bn_fwd_quant_kernel(const L1bnArgs a, int lg) {
+  // launched behind the previous kernel (programmatic stream serialization): wait for it
+  // before reading anything it wrote, and let the next kernel start launching
+  griddep_wait();
+  griddep_launch_dependents();
+  __shared__ RedSmem<1> sm;
+  const TilePos t = tile_pos(lg);
   const float tau = a.scal[kScXTau];
   const float Qf = static_cast<float>(a.Q);
   const float invS = __fdiv_rn(Qf, tau);
   const bool zero = !(tau > 0.0f) || !isfinite(tau) || !isfinite(invS);
   int e[4];
 #pragma unroll
-  for (int j = 0; j < 4; ++j) e[j] = c + j < a.C ? a.xe[c + j] : 0;
-  int acc[4] = {0, 0, 0, 0};
-  int64_t r0, r1;
-  block_rows(a.R, &r0, &r1);
-  if (c < a.C) {
-#pragma unroll 4
-    for (int64_t r = r0 + w; r < r1; r += kL1Threads / 32) {
-      float v[4];
-      load4(a.in + r * a.ld_in, c, a.C, a.vec_in, v);
-      int q[4];
+  for (int j = 0; j < 4; ++j) e[j] = t.c + j < a.C ? a.xe[t.c + j] : 0;
+  long long acc[1][4] = {{0, 0, 0, 0}};
+  constexpr int U = kL1PassesF32;
+  if (t.c < a.C) {
+    RowWalk w = row_walk(t);
+    const float* px = a.in + w.r * a.ld_in + t.c;
+    int8_t* pq = a.xq + w.r * a.C + t.c;
+    const int64_t sx = w.S * a.ld_in, sq = w.S * a.C;
+    for (; w.r < a.R; w.r += U * w.S, px += U * sx, pq += U * sq) {
+      float v[U][4];
 #pragma unroll
-      for (int j = 0; j < 4; ++j) {
-        q[j] = c + j < a.C ? shift_code(v[j], e[j], invS, zero, Qf, false, 0, 0) : 0;
-        acc[j] += q[j];
+      for (int u = 0; u < U; ++u)
+        if (w.r + u * w.S < a.R) load4(px + u * sx, t.c, a.C, a.vec_in, v[u]);
+#pragma unroll
+      for (int u = 0; u < U; ++u) {
+        if (w.r + u * w.S >= a.R) break;
+        int q[4];
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          q[j] = t.c + j < a.C ? shift_code(v[u][j], e[j], invS, zero, Qf, false, 0, 0) : 0;
+          acc[0][j] += q[j];
+        }
+        store_codes4(pq + u * sq, t.c, a.C, q);
       }
-      store_codes4(a.xq, r * a.C + c, c, a.C, q);
     }
   }
-  add_columns(acc, a.st + kStS1 * a.C, c0, a.C, red);
+  long long* const dst[1] = {stat_slot(a.st, kStS1, a.C)};
+  red_end<1>(acc, dst, t, a.C, sm);
   if (blockIdx.x == 0 && blockIdx.y == 0 && threadIdx.x == 0)
     a.scal[kScXScale] = zero ? 0.0f : __fdiv_rn(tau, Qf);
 }
 
 // Forward pass 2: over the codes, sum |q - m| and sum sign(q - m) per channel, with
 // m = round-half-even(sum q / R).
-__global__ void __launch_bounds__(kL1Threads) l1bn_fwd_dev_kernel(const L1bnArgs a) {
-  __shared__ int red[kL1Threads / 32 * kL1Cols];
-  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
-  const int64_t c0 = static_cast<int64_t>(blockIdx.x) * kL1Cols;
-  const int64_t c = c0 + lane * 4;
+__global__ void __launch_bounds__(kL1Threads, 3) l1bn_fwd_dev_kernel(const L1bnArgs a, int lg) {
+  griddep_wait();
+  griddep_launch_dependents();
+  __shared__ RedSmem<2> sm;
+  const TilePos t = tile_pos(lg);
+  // the block's columns' means, from their sum slots, once per block
+  __shared__ int mean[kL1MaxCols];
+  {
+    long long* fold = &sm.part[0][0];   // free until the block's reduction at the end
+    const int64_t cb = static_cast<int64_t>(blockIdx.x) * t.tc;
+    for (int i = threadIdx.x; i < kSpread * t.tc; i += kL1Threads) {
+      const int slot = i / t.tc, col = i - slot * t.tc;
+      fold[i] = cb + col < a.C ? a.st[(static_cast<int64_t>(kStS1) * kSpread + slot) * a.C + cb + col] : 0;
+    }
+    __syncthreads();
+    if (threadIdx.x < t.tc) {
+      long long v = 0;
+#pragma unroll
+      for (int k = 0; k < kSpread; ++k) v += fold[k * t.tc + threadIdx.x];
+      mean[threadIdx.x] = static_cast<int>(rne_div(v, a.R));
+    }
+    __syncthreads();
+  }
   int m[4];
 #pragma unroll
-  for (int j = 0; j < 4; ++j)
-    m[j] = c + j < a.C ? static_cast<int>(rne_div(a.st[kStS1 * a.C + c + j], a.R)) : 0;
-  int sabs[4] = {0, 0, 0, 0}, ssgn[4] = {0, 0, 0, 0};
-  int64_t r0, r1;
-  block_rows(a.R, &r0, &r1);
-  if (c < a.C) {
-#pragma unroll 4
-    for (int64_t r = r0 + w; r < r1; r += kL1Threads / 32) {
-      int q[4];
-      load_codes4(a.xq, r * a.C + c, c, a.C, q);
+  for (int j = 0; j < 4; ++j) m[j] = t.c + j < a.C ? mean[4 * t.qc + j] : 0;
+  long long acc[2][4] = {{0, 0, 0, 0}, {0, 0, 0, 0}};
+  constexpr int U = kL1PassesCodes;
+  if (t.c < a.C) {
+    RowWalk w = row_walk(t);
+    const int8_t* pq = a.xq + w.r * a.C + t.c;
+    const int64_t sq = w.S * a.C;
+    int sabs[4] = {0, 0, 0, 0}, ssgn[4] = {0, 0, 0, 0};
+    int n = 0;
+    for (; w.r < a.R; w.r += U * w.S, pq += U * sq) {
+      uint32_t q[U];
 #pragma unroll
-      for (int j = 0; j < 4; ++j) {
-        if (c + j >= a.C) continue;
-        const int d = q[j] - m[j];
-        sabs[j] += d < 0 ? -d : d;
-        ssgn[j] += (d > 0) - (d < 0);
+      for (int u = 0; u < U; ++u) q[u] = w.r + u * w.S < a.R ? load_codes_w(pq + u * sq, t.c, a.C) : 0u;
+#pragma unroll
+      for (int u = 0; u < U; ++u) {
+        if (w.r + u * w.S >= a.R) break;
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          const int d = code_at(q[u], j) - m[j];
+          sabs[j] += abs(d);
+          ssgn[j] += (d > 0) - (d < 0);
+        }
+      }
+      // |d| <= 255: int sums of up to 2^23 rows stay exact; fold them into 64 bits by then
+      if (++n == (1 << 20) / U) {
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          acc[0][j] += sabs[j];
+          acc[1][j] += ssgn[j];
+          sabs[j] = ssgn[j] = 0;
+        }
+        n = 0;
       }
     }
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {   // columns past C: zero codes and m = 0, so d = 0
+      acc[0][j] += sabs[j];
+      acc[1][j] += ssgn[j];
+    }
   }
-  add_columns(sabs, a.st + kStS * a.C, c0, a.C, red);
-  __syncthreads();
-  add_columns(ssgn, a.st + kStZ * a.C, c0, a.C, red);
+  long long* const dst[2] = {stat_slot(a.st, kStS, a.C), stat_slot(a.st, kStZ, a.C)};
+  red_end<2>(acc, dst, t, a.C, sm);
 }
 
 // max over the block of non-negative values given as bit patterns
@@ -245,6 +370,8 @@ __device__ __forceinline__ float quant8(float v, float vmax) {
 
 // Forward pass 3 (one block): s_c, m_c, sigma_c, then sigma^q, gamma^q, beta^q.
 __global__ void __launch_bounds__(1024) l1bn_fwd_chan_kernel(const L1bnArgs a) {
+  griddep_wait();
+  griddep_launch_dependents();
   __shared__ uint32_t red[32];
   const float Rf = __ll2float_rn(a.R);
   const float scale = a.scal[kScXScale];
@@ -253,8 +380,8 @@ __global__ void __launch_bounds__(1024) l1bn_fwd_chan_kernel(const L1bnArgs a) {
   uint32_t ms = 0, mg = 0, mb = 0;
   for (int64_t c = threadIdx.x; c < C; c += blockDim.x) {
     const float s = __fmul_rn(scale, pow2f(-static_cast<int>(a.xe[c])));
-    const long long m = rne_div(a.st[kStS1 * C + c], a.R);
-    const float sig = __fmul_rn(__fdiv_rn(__ll2float_rn(a.st[kStS * C + c]), Rf), s);
+    const long long m = rne_div(stat_sum(a.st, kStS1, C, c), a.R);
+    const float sig = __fmul_rn(__fdiv_rn(__ll2float_rn(stat_sum(a.st, kStS, C, c)), Rf), s);
     ch[kChS * C + c] = s;
     ch[kChM * C + c] = static_cast<float>(m);
     ch[kChSig * C + c] = sig;
@@ -272,47 +399,71 @@ __global__ void __launch_bounds__(1024) l1bn_fwd_chan_kernel(const L1bnArgs a) {
   }
 }
 
-// Forward pass 4: y = gamma^q ((x^q - mu^q) / sigma^q) + beta^q, four outputs per thread.
-__global__ void __launch_bounds__(256) l1bn_fwd_out_kernel(const L1bnArgs a) {
-  const int64_t nq = (a.C + 3) / 4;
-  const int64_t quads = a.R * nq;
+// Forward pass 3b (one block per channel): the output of every code value q in [-127, 127]
+// in the output pass's operations and order.  A code takes at most 255 values, so the
+// output pass looks its result up instead of dividing per element.
+__global__ void __launch_bounds__(kLutStride) l1bn_fwd_lut_kernel(const L1bnArgs a) {
+  griddep_wait();
+  griddep_launch_dependents();
+  const int64_t C = a.C, c = blockIdx.x;
   const float* ch = a.ch;
+  const int q = static_cast<int>(threadIdx.x) - 127;
+  const float s = ch[kChS * C + c], sq = ch[kChSq * C + c];
+  const float xq = __fmul_rn(static_cast<float>(q), s);
+  const float mq = __fmul_rn(ch[kChM * C + c], s);
+  const float xhat = sq > 0.0f ? __fdiv_rn(__fsub_rn(xq, mq), sq) : 0.0f;
+  a.lut[c * kLutStride + threadIdx.x] = __fadd_rn(__fmul_rn(ch[kChGq * C + c], xhat), ch[kChBq * C + c]);
+}
+
+// zero n 64-bit channel sums (the first kernel of a call: nothing before it in the call)
+__global__ void __launch_bounds__(256) l1bn_zero_kernel(long long* __restrict__ p, int64_t n) {
+  for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < n;
+       i += static_cast<int64_t>(gridDim.x) * blockDim.x)
+    p[i] = 0;
+}
+
+// Forward pass 4: y = gamma^q ((x^q - mu^q) / sigma^q) + beta^q, looked up per code from
+// the table the channel pass built (copied to shared memory for the block's columns).
+__global__ void __launch_bounds__(kL1Threads, 3) l1bn_fwd_out_kernel(const L1bnArgs a, int lg) {
+  griddep_wait();
+  griddep_launch_dependents();
+  extern __shared__ float lut[];   // [tile columns][kLutStride]
+  const TilePos t = tile_pos(lg);
   const int64_t C = a.C;
-  for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < quads;
-       i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
-    const int64_t r = i / nq;
-    const int64_t c = (i - r * nq) * 4;
-    int q[4];
-    load_codes4(a.xq, r * C + c, c, C, q);
-    float y[4];
+  const int64_t cbase = static_cast<int64_t>(blockIdx.x) * t.tc;
+  const int ncol = static_cast<int>(min(static_cast<int64_t>(t.tc), C - cbase));
+  for (int i = threadIdx.x; i < ncol * kLutStride; i += kL1Threads)
+    lut[i] = a.lut[cbase * kLutStride + i];
+  __syncthreads();
+  if (t.c >= C) return;
+  constexpr int U = kL1PassesCodes;
+  RowWalk w = row_walk(t);
+  const int8_t* pq = a.xq + w.r * C + t.c;
+  float* py = a.out + w.r * a.ld_out + t.c;
+  const int64_t sq = w.S * C, sy = w.S * a.ld_out;
+  const int col0 = 4 * t.qc * kLutStride + 127;
+  for (; w.r < a.R; w.r += U * w.S, pq += U * sq, py += U * sy) {
+    uint32_t q[U];
 #pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      y[j] = 0.0f;
-      if (c + j >= C) continue;
-      const float s = ch[kChS * C + c + j], sq = ch[kChSq * C + c + j];
-      const float xq = __fmul_rn(static_cast<float>(q[j]), s);
-      const float mq = __fmul_rn(ch[kChM * C + c + j], s);
-      const float xhat = sq > 0.0f ? __fdiv_rn(__fsub_rn(xq, mq), sq) : 0.0f;
-      y[j] = __fadd_rn(__fmul_rn(ch[kChGq * C + c + j], xhat), ch[kChBq * C + c + j]);
-    }
-    float* dst = a.out + r * a.ld_out + c;
-    if (a.vec_out && c + 3 < C) {
-      *reinterpret_cast<float4*>(dst) = make_float4(y[0], y[1], y[2], y[3]);
-    } else {
+    for (int u = 0; u < U; ++u) q[u] = w.r + u * w.S < a.R ? load_codes_w(pq + u * sq, t.c, C) : 0u;
 #pragma unroll
-      for (int j = 0; j < 4; ++j)
-        if (c + j < C) dst[j] = y[j];
+    for (int u = 0; u < U; ++u) {
+      if (w.r + u * w.S >= a.R) break;
+      float y[4];
+#pragma unroll
+      for (int j = 0; j < 4; ++j) y[j] = t.c + j < C ? lut[col0 + j * kLutStride + code_at(q[u], j)] : 0.0f;
+      store4(py + u * sy, t.c, C, a.vec_out, y);
     }
   }
 }
 
 // Backward pass 1: dy -> int8 ShiftQuant codes p (stochastic rounding of element r C + c),
 // sums of p and of p (q - m) per channel.
-__global__ void __launch_bounds__(kL1Threads) l1bn_bwd_quant_kernel(const L1bnArgs a) {
-  __shared__ long long red[kL1Threads / 32 * kL1Cols];
-  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
-  const int64_t c0 = static_cast<int64_t>(blockIdx.x) * kL1Cols;
-  const int64_t c = c0 + lane * 4;
+__global__ void __launch_bounds__(kL1Threads, 3) l1bn_bwd_quant_kernel(const L1bnArgs a, int lg) {
+  griddep_wait();
+  griddep_launch_dependents();
+  __shared__ RedSmem<2> sm;
+  const TilePos t = tile_pos(lg);
   const float tau = a.scal[kScGTau];
   const float Qf = static_cast<float>(a.Q);
   const float invS = __fdiv_rn(Qf, tau);
@@ -320,40 +471,55 @@ __global__ void __launch_bounds__(kL1Threads) l1bn_bwd_quant_kernel(const L1bnAr
   int e[4], m[4];
 #pragma unroll
   for (int j = 0; j < 4; ++j) {
-    e[j] = c + j < a.C ? a.ge[c + j] : 0;
-    m[j] = c + j < a.C ? static_cast<int>(a.ch[kChM * a.C + c + j]) : 0;
+    e[j] = t.c + j < a.C ? a.ge[t.c + j] : 0;
+    m[j] = t.c + j < a.C ? static_cast<int>(a.ch[kChM * a.C + t.c + j]) : 0;
   }
-  long long sp[4] = {0, 0, 0, 0}, spd[4] = {0, 0, 0, 0};
-  int64_t r0, r1;
-  block_rows(a.R, &r0, &r1);
-  if (c < a.C) {
-#pragma unroll 4
-    for (int64_t r = r0 + w; r < r1; r += kL1Threads / 32) {
-      float v[4];
-      load4(a.in + r * a.ld_in, c, a.C, a.vec_in, v);
-      int qx[4];
-      load_codes4(a.xq, r * a.C + c, c, a.C, qx);
-      int p[4];
+  long long acc[2][4] = {{0, 0, 0, 0}, {0, 0, 0, 0}};
+  constexpr int U = kL1PassesF32;
+  if (t.c < a.C) {
+    RowWalk w = row_walk(t);
+    const float* pg = a.in + w.r * a.ld_in + t.c;
+    const int8_t* px = a.xq + w.r * a.C + t.c;
+    int8_t* pp = a.gq + w.r * a.C + t.c;
+    const int64_t sg = w.S * a.ld_in, sc = w.S * a.C;
+    for (; w.r < a.R; w.r += U * w.S, pg += U * sg, px += U * sc, pp += U * sc) {
+      float v[U][4];
+      uint32_t qx[U];
 #pragma unroll
-      for (int j = 0; j < 4; ++j) {
-        p[j] = c + j < a.C ? shift_code(v[j], e[j], invS, zero, Qf, true, a.seed,
-                                        static_cast<uint64_t>(r * a.C + c + j))
-                           : 0;
-        sp[j] += p[j];
-        spd[j] += static_cast<long long>(p[j]) * (qx[j] - m[j]);
+      for (int u = 0; u < U; ++u) {
+        qx[u] = 0u;
+        if (w.r + u * w.S < a.R) {
+          load4(pg + u * sg, t.c, a.C, a.vec_in, v[u]);
+          qx[u] = load_codes_w(px + u * sc, t.c, a.C);
+        }
       }
-      store_codes4(a.gq, r * a.C + c, c, a.C, p);
+#pragma unroll
+      for (int u = 0; u < U; ++u) {
+        const int64_t r = w.r + u * w.S;
+        if (r >= a.R) break;
+        int pc[4];
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          pc[j] = t.c + j < a.C ? shift_code(v[u][j], e[j], invS, zero, Qf, true, a.seed,
+                                             static_cast<uint64_t>(r * a.C + t.c + j))
+                                : 0;
+          acc[0][j] += pc[j];
+          acc[1][j] += pc[j] * (code_at(qx[u], j) - m[j]);
+        }
+        store_codes4(pp + u * sc, t.c, a.C, pc);
+      }
     }
   }
-  add_columns(sp, a.st + kStP * a.C, c0, a.C, red);
-  __syncthreads();
-  add_columns(spd, a.st + kStD * a.C, c0, a.C, red);
+  long long* const dst[2] = {stat_slot(a.st, kStP, a.C), stat_slot(a.st, kStD, a.C)};
+  red_end<2>(acc, dst, t, a.C, sm);
   if (blockIdx.x == 0 && blockIdx.y == 0 && threadIdx.x == 0)
     a.scal[kScGScale] = zero ? 0.0f : __fdiv_rn(tau, Qf);
 }
 
 // Backward pass 2: the per-channel constants of the input gradient, dgamma and dbeta.
 __global__ void __launch_bounds__(256) l1bn_bwd_chan_kernel(const L1bnArgs a) {
+  griddep_wait();
+  griddep_launch_dependents();
   const float Rf = __ll2float_rn(a.R);
   const float gscale = a.scal[kScGScale];
   const int64_t C = a.C;
@@ -362,53 +528,70 @@ __global__ void __launch_bounds__(256) l1bn_bwd_chan_kernel(const L1bnArgs a) {
        c += static_cast<int64_t>(gridDim.x) * blockDim.x) {
     const float t = __fmul_rn(gscale, pow2f(-static_cast<int>(a.ge[c])));
     const float sq = ch[kChSq * C + c], s = ch[kChS * C + c];
-    const float P = __ll2float_rn(a.st[kStP * C + c]);
+    const float P = __ll2float_rn(stat_sum(a.st, kStP, C, c));
     const float u = sq > 0.0f ? __fdiv_rn(ch[kChGq * C + c], sq) : 0.0f;
     const float mg = __fdiv_rn(__fmul_rn(P, t), Rf);
     const float dg =
-        sq > 0.0f ? __fdiv_rn(__fmul_rn(__fmul_rn(__ll2float_rn(a.st[kStD * C + c]), t), s), sq) : 0.0f;
+        sq > 0.0f ? __fdiv_rn(__fmul_rn(__fmul_rn(__ll2float_rn(stat_sum(a.st, kStD, C, c)), t), s), sq) : 0.0f;
     ch[kChT * C + c] = t;
     ch[kChU * C + c] = u;
     ch[kChMg * C + c] = mg;
     ch[kChMgx * C + c] = __fdiv_rn(dg, Rf);
-    ch[kChZs * C + c] = __fdiv_rn(__ll2float_rn(a.st[kStZ * C + c]), Rf);
+    ch[kChZs * C + c] = __fdiv_rn(__ll2float_rn(stat_sum(a.st, kStZ, C, c)), Rf);
     a.dgamma[c] = dg;
     a.dbeta[c] = __fmul_rn(P, t);
   }
 }
 
-// Backward pass 3: dx = u ((g - mean g) - mean(g xhat) (sign(q - m) - mean sign)).
-__global__ void __launch_bounds__(256) l1bn_bwd_out_kernel(const L1bnArgs a) {
-  const int64_t nq = (a.C + 3) / 4;
-  const int64_t quads = a.R * nq;
+// Backward pass 3: dx = u ((g - mean g) - mean(g xhat) (sign(q - m) - mean sign)), the
+// per-channel values of each thread's quad in registers; mean(g xhat) (sign - mean sign)
+// takes one of three values per channel, formed once.
+__global__ void __launch_bounds__(kL1Threads, 3) l1bn_bwd_out_kernel(const L1bnArgs a, int lg) {
+  griddep_wait();
+  griddep_launch_dependents();
+  const TilePos t = tile_pos(lg);
+  if (t.c >= a.C) return;
   const float* ch = a.ch;
   const int64_t C = a.C;
-  for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < quads;
-       i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
-    const int64_t r = i / nq;
-    const int64_t c = (i - r * nq) * 4;
-    int q[4], p[4];
-    load_codes4(a.xq, r * C + c, c, C, q);
-    load_codes4(a.gq, r * C + c, c, C, p);
-    float dx[4];
+  int m[4];
+  float tt[4], mg[4], u4[4], k[4][3];
 #pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      dx[j] = 0.0f;
-      if (c + j >= C) continue;
-      const int d = q[j] - static_cast<int>(ch[kChM * C + c + j]);
-      const float g = __fmul_rn(static_cast<float>(p[j]), ch[kChT * C + c + j]);
-      const float sg = static_cast<float>((d > 0) - (d < 0));
-      const float inner = __fsub_rn(__fsub_rn(g, ch[kChMg * C + c + j]),
-                                    __fmul_rn(ch[kChMgx * C + c + j], __fsub_rn(sg, ch[kChZs * C + c + j])));
-      dx[j] = __fmul_rn(ch[kChU * C + c + j], inner);
+  for (int j = 0; j < 4; ++j) {
+    const int64_t c = t.c + j < C ? t.c + j : C - 1;
+    m[j] = static_cast<int>(ch[kChM * C + c]);
+    tt[j] = ch[kChT * C + c];
+    mg[j] = ch[kChMg * C + c];
+    u4[j] = ch[kChU * C + c];
+    const float mgx = ch[kChMgx * C + c], zs = ch[kChZs * C + c];
+#pragma unroll
+    for (int sgn = -1; sgn <= 1; ++sgn) k[j][sgn + 1] = __fmul_rn(mgx, __fsub_rn(static_cast<float>(sgn), zs));
+  }
+  constexpr int U = kL1PassesCodes;
+  RowWalk w = row_walk(t);
+  const int8_t* pq = a.xq + w.r * C + t.c;
+  const int8_t* pp = a.gq + w.r * C + t.c;
+  float* pd = a.out + w.r * a.ld_out + t.c;
+  const int64_t sc = w.S * C, sd = w.S * a.ld_out;
+  for (; w.r < a.R; w.r += U * w.S, pq += U * sc, pp += U * sc, pd += U * sd) {
+    uint32_t q[U], p[U];
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      const bool in = w.r + u * w.S < a.R;
+      q[u] = in ? load_codes_w(pq + u * sc, t.c, C) : 0u;
+      p[u] = in ? load_codes_w(pp + u * sc, t.c, C) : 0u;
     }
-    float* dst = a.out + r * a.ld_out + c;
-    if (a.vec_out && c + 3 < C) {
-      *reinterpret_cast<float4*>(dst) = make_float4(dx[0], dx[1], dx[2], dx[3]);
-    } else {
 #pragma unroll
-      for (int j = 0; j < 4; ++j)
-        if (c + j < C) dst[j] = dx[j];
+    for (int u = 0; u < U; ++u) {
+      if (w.r + u * w.S >= a.R) break;
+      float dx[4];
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        const int d = code_at(q[u], j) - m[j];
+        const float g = __fmul_rn(static_cast<float>(code_at(p[u], j)), tt[j]);
+        const float kj = d > 0 ? k[j][2] : (d < 0 ? k[j][0] : k[j][1]);
+        dx[j] = __fmul_rn(u4[j], __fsub_rn(__fsub_rn(g, mg[j]), kj));
+      }
+      store4(pd + u * sd, t.c, C, a.vec_out, dx);
     }
   }
 }
@@ -434,6 +617,7 @@ static L1bnArgs l1bn_args(int64_t R, int64_t C, int bits, void* state) {
   a.gq = reinterpret_cast<int8_t*>(b + L.gq);
   a.st = reinterpret_cast<long long*>(b + L.stats);
   a.ch = reinterpret_cast<float*>(b + L.chan);
+  a.lut = reinterpret_cast<float*>(b + L.lut);
   a.xe = reinterpret_cast<uint8_t*>(b + L.exps);
   a.ge = a.xe + C;
   a.scal = reinterpret_cast<float*>(b + L.scal);
@@ -448,7 +632,7 @@ static int l1bn_check(const char* nm, int64_t R, int64_t C, int64_t ld_in, int64
   if (R < 0 || C < 0) return fail(SQ_EINVAL, "%s: negative size", nm);
   if (C > 0 && R == 0) return fail(SQ_EINVAL, "%s: a channel needs at least one element", nm);
   if (C == 0) return SQ_OK;
-  if (R > (int64_t(1) << 40) || C > (int64_t(1) << 31) || R * C > (int64_t(1) << 40))
+  if (R > (int64_t(1) << 40) || C >= (int64_t(1) << 31) || R * C > (int64_t(1) << 40))
     return fail(SQ_EUNSUPPORTED, "%s: tensor too large", nm);
   if (in == nullptr || out == nullptr || state == nullptr || dev_status == nullptr)
     return fail(SQ_EINVAL, "%s: NULL argument", nm);
@@ -459,21 +643,59 @@ static int l1bn_check(const char* nm, int64_t R, int64_t C, int64_t ld_in, int64
   return SQ_OK;
 }
 
-static dim3 reduction_grid(int64_t R, int64_t C, int sms) {
-  const int64_t gx = (C + kL1Cols - 1) / kL1Cols;
-  int64_t gy = (4 * static_cast<int64_t>(sms) + gx - 1) / gx;  // about four blocks per SM
-  const int64_t max_gy = (R + 7) / 8;                          // at least eight rows a block
-  if (gy > max_gy) gy = max_gy;
+// The tile of a tensor with C channels: TC = 4 << lg columns, the channel count rounded up
+// to a power of two (at least 4, at most 128).
+static int tile_lg(int64_t C) {
+  int lg = 0;
+  while (lg < 5 && (int64_t(4) << lg) < C) ++lg;
+  return lg;
+}
+
+// A reduction launch: the column tiles by about three blocks per SM (one resident wave),
+// each block taking every gridDim.y-th tile of `rows_per_tile` rows.
+static dim3 reduction_grid(int64_t R, int64_t C, int lg, int rows_per_tile, int sms) {
+  const int64_t gx = (C + (int64_t(4) << lg) - 1) / (int64_t(4) << lg);
+  const int64_t tiles = (R + rows_per_tile - 1) / rows_per_tile;
+  int64_t gy = (3 * static_cast<int64_t>(sms) + gx - 1) / gx;   // one wave at three blocks per SM
+  if (gy > tiles) gy = tiles;
   if (gy > 65535) gy = 65535;
   if (gy < 1) gy = 1;
   return dim3(static_cast<unsigned>(gx), static_cast<unsigned>(gy));
 }
 
-static unsigned elementwise_blocks(int64_t R, int64_t C, int sms) {
-  const int64_t quads = R * ((C + 3) / 4);
-  int64_t b = (quads + 255) / 256;
-  if (b > static_cast<int64_t>(sms) * 16) b = static_cast<int64_t>(sms) * 16;
-  return static_cast<unsigned>(b < 1 ? 1 : b);
+// An elementwise launch: the column tiles by about three blocks per SM, each block walking
+// its rows (at most one step of kL1PassesCodes rows per thread when there are few rows).
+static dim3 elementwise_grid(int64_t R, int64_t C, int lg, int sms) {
+  const int64_t gx = (C + (int64_t(4) << lg) - 1) / (int64_t(4) << lg);
+  const int64_t rows_per_step = kL1PassesCodes * (int64_t(kL1Threads) >> lg);
+  int64_t gy = (R + rows_per_step - 1) / rows_per_step;
+  const int64_t want = (3 * static_cast<int64_t>(sms) + gx - 1) / gx;
+  if (gy > want) gy = want;
+  if (gy > 65535) gy = 65535;
+  return dim3(static_cast<unsigned>(gx), static_cast<unsigned>(gy < 1 ? 1 : gy));
+}
+
+// The output pass's tile: at most 32 columns, so that the table it keeps in shared memory
+// (32 KB) leaves room for three blocks per SM.
+constexpr int kL1OutMaxLg = 3;
+
+// Launch a kernel behind the previous one of the stream with programmatic stream
+// serialization (it waits for that kernel before reading its results).
+template <typename... Params, typename... Args>
+static cudaError_t launch_behind(void (*kernel)(Params...), dim3 grid, dim3 block, size_t smem,
+                                 cudaStream_t s, Args... args) {
+  cudaLaunchConfig_t cfg;
+  memset(&cfg, 0, sizeof(cfg));
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kernel, args...);
 }
 
 static int launched(const char* what) {
@@ -512,21 +734,34 @@ extern "C" sq_status shiftquant_l1bn_forward(const float* x, int64_t rows, int64
   a.beta = beta;
   a.vec_in = (ld_x % 4 == 0) && aligned16(x);
   a.vec_out = (ld_y % 4 == 0) && aligned16(y);
+  // the channel sums start at zero (a kernel, not a memset, so that the launches after the
+  // range pass stay a chain of kernels, each launched behind the one before)
+  const int64_t nz = 3 * kSpread * channels;
+  l1bn_zero_kernel<<<static_cast<unsigned>((nz + 255) / 256 < 1024 ? (nz + 255) / 256 : 1024), 256, 0, s>>>(a.st, nz);
+  if ((st = launched("l1bn_zero_kernel launch")) != SQ_OK) return st;
   // range pass and grouping of x (the library's own), into the state
   st = shiftquant_calibrate(x, rows, channels, ld_x, SQ_GRAN_SHIFT, n_groups,
                             a.ch + kChXRange * channels, a.scal + kScXTau, a.xe, dev_status, stream);
   if (st != SQ_OK) return st;
-  cudaError_t err = cudaMemsetAsync(a.st, 0, 3 * static_cast<size_t>(channels) * sizeof(long long), s);
-  if (err != cudaSuccess) return cuda_fail(err, "cudaMemsetAsync");
-  const dim3 rg = reduction_grid(rows, channels, sms);
-  l1bn_fwd_quant_kernel<<<rg, kL1Threads, 0, s>>>(a);
-  if ((st = launched("l1bn_fwd_quant_kernel launch")) != SQ_OK) return st;
-  l1bn_fwd_dev_kernel<<<rg, kL1Threads, 0, s>>>(a);
-  if ((st = launched("l1bn_fwd_dev_kernel launch")) != SQ_OK) return st;
-  l1bn_fwd_chan_kernel<<<1, 1024, 0, s>>>(a);
-  if ((st = launched("l1bn_fwd_chan_kernel launch")) != SQ_OK) return st;
-  l1bn_fwd_out_kernel<<<elementwise_blocks(rows, channels, sms), 256, 0, s>>>(a);
-  return launched("l1bn_fwd_out_kernel launch");
+  cudaError_t err;
+  const int lg = tile_lg(channels);
+  const int rpp = kL1Threads >> lg;
+  err = launch_behind(l1bn_fwd_quant_kernel, reduction_grid(rows, channels, lg, kL1PassesF32 * rpp, sms),
+                      dim3(kL1Threads), 0, s, a, lg);
+  if (err != cudaSuccess) return cuda_fail(err, "l1bn_fwd_quant_kernel launch");
+  err = launch_behind(l1bn_fwd_dev_kernel, reduction_grid(rows, channels, lg, kL1PassesCodes * rpp, sms),
+                      dim3(kL1Threads), 0, s, a, lg);
+  if (err != cudaSuccess) return cuda_fail(err, "l1bn_fwd_dev_kernel launch");
+  if ((err = launch_behind(l1bn_fwd_chan_kernel, dim3(1), dim3(1024), 0, s, a)) != cudaSuccess)
+    return cuda_fail(err, "l1bn_fwd_chan_kernel launch");
+  if ((err = launch_behind(l1bn_fwd_lut_kernel, dim3(static_cast<unsigned>(channels)), dim3(kLutStride),
+                           0, s, a)) != cudaSuccess)
+    return cuda_fail(err, "l1bn_fwd_lut_kernel launch");
+  const int lgo = lg < kL1OutMaxLg ? lg : kL1OutMaxLg;
+  const size_t lut_bytes = (size_t(4) << lgo) * kLutStride * sizeof(float);
+  err = launch_behind(l1bn_fwd_out_kernel, elementwise_grid(rows, channels, lgo, sms), dim3(kL1Threads),
+                      lut_bytes, s, a, lgo);
+  return err == cudaSuccess ? SQ_OK : cuda_fail(err, "l1bn_fwd_out_kernel launch");
 }
 
 extern "C" sq_status shiftquant_l1bn_backward(const float* dy, int64_t rows, int64_t channels,
@@ -553,18 +788,23 @@ extern "C" sq_status shiftquant_l1bn_backward(const float* dy, int64_t rows, int
   a.dbeta = dbeta;
   a.vec_in = (ld_dy % 4 == 0) && aligned16(dy);
   a.vec_out = (ld_dx % 4 == 0) && aligned16(dx);
+  const int64_t nz = 2 * kSpread * channels;
+  l1bn_zero_kernel<<<static_cast<unsigned>((nz + 255) / 256 < 1024 ? (nz + 255) / 256 : 1024), 256, 0, s>>>(
+      a.st + kStP * kSpread * channels, nz);
+  if ((st = launched("l1bn_zero_kernel launch")) != SQ_OK) return st;
   st = shiftquant_calibrate(dy, rows, channels, ld_dy, SQ_GRAN_SHIFT, n_groups,
                             a.ch + kChGRange * channels, a.scal + kScGTau, a.ge, dev_status, stream);
   if (st != SQ_OK) return st;
-  cudaError_t err = cudaMemsetAsync(a.st + kStP * channels, 0,
-                                    2 * static_cast<size_t>(channels) * sizeof(long long), s);
-  if (err != cudaSuccess) return cuda_fail(err, "cudaMemsetAsync");
-  const dim3 rg = reduction_grid(rows, channels, sms);
-  l1bn_bwd_quant_kernel<<<rg, kL1Threads, 0, s>>>(a);
-  if ((st = launched("l1bn_bwd_quant_kernel launch")) != SQ_OK) return st;
+  cudaError_t err;
+  const int lg = tile_lg(channels);
+  const int rpp = kL1Threads >> lg;
+  err = launch_behind(l1bn_bwd_quant_kernel, reduction_grid(rows, channels, lg, kL1PassesF32 * rpp, sms),
+                      dim3(kL1Threads), 0, s, a, lg);
+  if (err != cudaSuccess) return cuda_fail(err, "l1bn_bwd_quant_kernel launch");
   const unsigned cb = static_cast<unsigned>((channels + 255) / 256);
-  l1bn_bwd_chan_kernel<<<cb, 256, 0, s>>>(a);
-  if ((st = launched("l1bn_bwd_chan_kernel launch")) != SQ_OK) return st;
-  l1bn_bwd_out_kernel<<<elementwise_blocks(rows, channels, sms), 256, 0, s>>>(a);
-  return launched("l1bn_bwd_out_kernel launch");
+  if ((err = launch_behind(l1bn_bwd_chan_kernel, dim3(cb), dim3(256), 0, s, a)) != cudaSuccess)
+    return cuda_fail(err, "l1bn_bwd_chan_kernel launch");
+  err = launch_behind(l1bn_bwd_out_kernel, elementwise_grid(rows, channels, lg, sms), dim3(kL1Threads), 0,
+                      s, a, lg);
+  return err == cudaSuccess ? SQ_OK : cuda_fail(err, "l1bn_bwd_out_kernel launch");
 }

@@ -49,7 +49,9 @@ def _run(x, gamma, beta, dy, bits, G, seed):
 
 
 @pytest.mark.parametrize("R,C,bits,G", [(12544, 256, 8, 4), (1000, 77, 8, 4), (3000, 130, 6, 3),
-                                        (1, 9, 8, 4), (64, 4, 4, 1), (200, 1000, 8, 8)])
+                                        (1, 9, 8, 4), (64, 4, 4, 1), (200, 1000, 8, 8),
+                                        (20000, 64, 8, 4), (3001, 16, 8, 4), (777, 3, 8, 4),
+                                        (5000, 600, 8, 4)])
 def test_l1bn_matches_oracle_bit_for_bit(R, C, bits, G):
     rng = np.random.default_rng(R + C)
     x, gamma, beta, dy = _inputs(rng, R, C)
