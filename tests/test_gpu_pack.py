@@ -24,7 +24,8 @@ def _lib():
 
 @pytest.mark.parametrize("R,C,bits,G,ldp_extra", [(12544, 2304, 4, 4, 0), (300, 77, 4, 4, 3),
                                                   (64, 33, 3, 2, 0), (129, 1000, 4, 8, 0),
-                                                  (5, 1, 2, 1, 0)])
+                                                  (5, 1, 2, 1, 0), (2304, 12544, 4, 4, 0),
+                                                  (40, 528, 4, 4, 8)])
 def test_packed_codes_match_oracle_and_round_trip(R, C, bits, G, ldp_extra):
     rng = np.random.default_rng(R + C)
     x = (rng.standard_normal((R, C)) * np.exp(rng.normal(0, 1.5, C))).astype(np.float32)
