@@ -451,10 +451,11 @@ def run_ours(args, rank, world, local_rank):
         q_call_graph_ms += [r_ms, max(both_ms - r_ms, 1e-6)]
     del q_graph
 
-    # e2e: the C entry point shiftquant_layer_step_host (layer.HostSteps): every call copies a
-    # layer's X, W and dY in from pinned host memory, runs its whole step and copies Y, dX and
-    # dW back; two device buffer sets on two streams take the steps in turn.  Timed from the
-    # first copy in to the last copy back.
+    # e2e: the C entry point shiftquant_layer_step_host_split (layer.HostSteps): every call
+    # copies a layer's X, W and dY in from pinned host memory on the copy-in stream, runs its
+    # whole step on the layer's stream and copies Y, dX and dW back on the copy-out stream;
+    # two device buffer sets take the steps in turn.  Timed from the first copy in to the last
+    # copy back.
     e2e = None
     if not args.no_e2e:
         host_in = [[a.cpu().pin_memory() for a in inp] for inp in st.inputs]
@@ -477,9 +478,11 @@ def run_ours(args, rank, world, local_rank):
         e2e = {"value": job_throughput(st.gemm_ops(), world, args.steps, e_total),
                "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
                "ms_per_step": e_total / args.steps,
-               "api": "shiftquant_layer_step_host (C ABI), one call per layer and step",
-               "pipeline": "two device buffer sets on two streams take the steps in turn: one "
-                           "step's copies overlap the other's compute",
+               "api": "shiftquant_layer_step_host_split (C ABI), one call per layer and step",
+               "pipeline": "one copy-in and one copy-out stream for all calls, a stream per "
+                           "layer for the steps, two device buffer sets taking the steps in "
+                           "turn: copies in, compute and copies back of successive steps "
+                           "overlap",
                "l2": "not flushed: each step copies %.0f MB of inputs in from host memory "
                      "(L2 is 126 MB)" % (h2d / 1e6)}
         del pipe

@@ -443,6 +443,29 @@ sq_status shiftquant_layer_step_host(const sq_layer_step *args, const float *x_h
                                      float *dx_host, float *dw_host, uint64_t seed,
                                      void *inputs_queued, void *stream);
 
+/* The same step with its copies on their own streams: the input copies on copy_in_stream,
+ * the step (shiftquant_layer_step) on `stream`, the copies back on copy_out_stream, joined
+ * by caller-created cudaEvent_t handles:
+ *   buffers_free (may be NULL): copy_in_stream waits for it before copying in -- the event
+ *     of the previous call's copies back from these device buffers;
+ *   inputs_in:   recorded on copy_in_stream after the input copies; `stream` waits for it;
+ *   step_done:   recorded on `stream` after the step; copy_out_stream waits for it;
+ *   outputs_out: recorded on copy_out_stream after the copies back (the host outputs hold
+ *     the results, and the device buffers are free, once it completes).
+ * A copy engine serves its copies in the order they were queued, so copies in queued on
+ * one stream behind another call's copies back wait for them; with one stream for all
+ * copies in and one for all copies back, a caller that alternates device buffer sets keeps
+ * both directions of the host link busy while earlier steps compute.  Host pointers as in
+ * shiftquant_layer_step_host (page-locked memory for overlap; NULL skips a copy); the three
+ * streams may be the same stream. */
+sq_status shiftquant_layer_step_host_split(const sq_layer_step *args, const float *x_host,
+                                           const float *w_host, const float *dy_host,
+                                           float *y_host, float *dx_host, float *dw_host,
+                                           uint64_t seed, void *copy_in_stream, void *stream,
+                                           void *copy_out_stream, void *buffers_free,
+                                           void *inputs_in, void *step_done,
+                                           void *outputs_out);
+
 /* Weight-gradient GEMM for callers that cannot allocate device memory -- for instance a
  * plug-in running inside a host framework that owns every device allocation, or a
  * deployment whose device memory is fixed when the library is loaded.  The paper has no

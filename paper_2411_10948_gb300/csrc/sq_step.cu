@@ -119,3 +119,45 @@ extern "C" sq_status shiftquant_layer_step_host(const sq_layer_step* args, const
   if ((st = copy(dx_host, args->dx, M * K, cudaMemcpyDeviceToHost, s)) != SQ_OK) return st;
   return copy(dw_host, args->dw, K * N, cudaMemcpyDeviceToHost, s);
 }
+
+extern "C" sq_status shiftquant_layer_step_host_split(const sq_layer_step* args, const float* x_host,
+                                                      const float* w_host, const float* dy_host,
+                                                      float* y_host, float* dx_host, float* dw_host,
+                                                      uint64_t seed, void* copy_in_stream,
+                                                      void* stream, void* copy_out_stream,
+                                                      void* buffers_free, void* inputs_in,
+                                                      void* step_done, void* outputs_out) {
+  fail(SQ_OK, "");
+  int st = check_step(args);
+  if (st != SQ_OK) return st;
+  if (inputs_in == nullptr || step_done == nullptr || outputs_out == nullptr)
+    return fail(SQ_EINVAL, "layer_step_host_split: inputs_in, step_done and outputs_out are required");
+  const int64_t M = args->M, K = args->K, N = args->N;
+  const bool empty = M == 0 || K == 0 || N == 0;
+  cudaStream_t si = as_stream(copy_in_stream), sc = as_stream(stream), so = as_stream(copy_out_stream);
+  cudaEvent_t ev_in = static_cast<cudaEvent_t>(inputs_in);
+  cudaEvent_t ev_done = static_cast<cudaEvent_t>(step_done);
+  cudaEvent_t ev_out = static_cast<cudaEvent_t>(outputs_out);
+  cudaError_t err;
+  if (buffers_free != nullptr &&
+      (err = cudaStreamWaitEvent(si, static_cast<cudaEvent_t>(buffers_free), 0)) != cudaSuccess)
+    return cuda_fail(err, "cudaStreamWaitEvent");
+  if (!empty) {
+    if ((st = copy(args->x, x_host, M * K, cudaMemcpyHostToDevice, si)) != SQ_OK) return st;
+    if ((st = copy(args->w, w_host, K * N, cudaMemcpyHostToDevice, si)) != SQ_OK) return st;
+    if ((st = copy(args->dy, dy_host, M * N, cudaMemcpyHostToDevice, si)) != SQ_OK) return st;
+  }
+  if ((err = cudaEventRecord(ev_in, si)) != cudaSuccess) return cuda_fail(err, "cudaEventRecord");
+  if ((err = cudaStreamWaitEvent(sc, ev_in, 0)) != cudaSuccess) return cuda_fail(err, "cudaStreamWaitEvent");
+  if (!empty && (st = run_step(args, seed, stream)) != SQ_OK) return st;
+  if ((err = cudaEventRecord(ev_done, sc)) != cudaSuccess) return cuda_fail(err, "cudaEventRecord");
+  if ((err = cudaStreamWaitEvent(so, ev_done, 0)) != cudaSuccess)
+    return cuda_fail(err, "cudaStreamWaitEvent");
+  if (!empty) {
+    if ((st = copy(y_host, args->y, M * N, cudaMemcpyDeviceToHost, so)) != SQ_OK) return st;
+    if ((st = copy(dx_host, args->dx, M * K, cudaMemcpyDeviceToHost, so)) != SQ_OK) return st;
+    if ((st = copy(dw_host, args->dw, K * N, cudaMemcpyDeviceToHost, so)) != SQ_OK) return st;
+  }
+  if ((err = cudaEventRecord(ev_out, so)) != cudaSuccess) return cuda_fail(err, "cudaEventRecord");
+  return SQ_OK;
+}

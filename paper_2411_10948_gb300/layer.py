@@ -405,30 +405,35 @@ class CapturedStep:
 
 class HostSteps:
     """Training steps fed from host memory and returned to it through the C entry point
-    shiftquant_layer_step_host: for every layer of a step, one call copies X, W and dY in,
-    runs the layer's whole step and copies Y, dX and dW back, all inside the library and in
-    the order of one stream.  Two sets of device buffers, each with its own stream, take
-    the steps in turn; every call's input copies queue behind the previous call's (an event
-    the library records after them), so the copies in run back to back while the other
-    slot computes and copies back, and the host link's two directions, not the GPU, set
-    the pace.
+    shiftquant_layer_step_host_split: for every layer of a step, one call copies X, W and
+    dY in on the copy-in stream, runs the layer's whole step on the layer's own stream and
+    copies Y, dX and dW back on the copy-out stream, the three joined by events.  Two sets
+    of device buffers take the steps in turn; a set's copies in wait for its previous
+    copies back.  With one stream for every copy in and one for every copy back, each
+    direction of the host link works through its copies in step order while earlier steps
+    compute, so the link, not the GPU, sets the pace (a copy engine serves its copies in
+    queue order: copies in queued behind another call's copies back would wait for them).
 
     shapes: (M, K, N) per layer."""
 
     def __init__(self, shapes, bits, n_groups, device="cuda", slots=2):
         dev = torch.device(device)
         self.shapes = list(shapes)
+        self.copy_in = torch.cuda.Stream(device=dev)
+        self.copy_out = torch.cuda.Stream(device=dev)
         self.slots = []
         for _ in range(slots):
             layers = [QuantLinear(M, K, N_, bits, n_groups, dev, with_inputs=True)
                       for (M, K, N_) in self.shapes]
+            # per layer: inputs in, step done, outputs out (recorded once here so that the
+            # CUDA events exist before the library records them)
+            events = [{k: torch.cuda.Event() for k in ("in", "done", "out")} for _ in layers]
+            for evs in events:
+                for ev in evs.values():
+                    ev.record()
             self.slots.append({"layers": layers, "args": [l.step_args() for l in layers],
-                               "stream": torch.cuda.Stream(device=dev)})
-        # a ring of events marking each call's queued input copies (recorded once here so
-        # that the CUDA events exist before the library records them)
-        self.events = [torch.cuda.Event() for _ in range(2 * slots * max(1, len(self.shapes)))]
-        for ev in self.events:
-            ev.record()
+                               "streams": [torch.cuda.Stream(device=dev) for _ in layers],
+                               "events": events})
 
     def run(self, host_inputs, host_outputs, seed=0x5EED) -> torch.cuda.Event:
         """Queue one step per entry: host_inputs[i] = (x, w, dy) per layer, host_outputs[i] =
@@ -437,20 +442,19 @@ class HostSteps:
         event on the current stream after the last copy back (synchronize on it before
         reading the host outputs)."""
         cur = torch.cuda.current_stream()
-        for sl in self.slots:
-            sl["stream"].wait_stream(cur)
-        prev, k = None, 0
+        streams = [self.copy_in, self.copy_out] + [st for sl in self.slots for st in sl["streams"]]
+        for st in streams:
+            st.wait_stream(cur)
         for i, (hin, hout) in enumerate(zip(host_inputs, host_outputs)):
             sl = self.slots[i % len(self.slots)]
-            for args, (x, w, dy), (y, dx, dw) in zip(sl["args"], hin, hout):
-                if prev is not None:
-                    sl["stream"].wait_event(prev)
-                ev = self.events[k % len(self.events)]
-                N.shiftquant_layer_step_host(args, x, w, dy, y, dx, dw, seed + i, sl["stream"],
-                                             inputs_queued=ev)
-                prev, k = ev, k + 1
-        for sl in self.slots:
-            cur.wait_stream(sl["stream"])
+            for args, st, ev, (x, w, dy), (y, dx, dw) in zip(sl["args"], sl["streams"],
+                                                             sl["events"], hin, hout):
+                N.shiftquant_layer_step_host_split(args, x, w, dy, y, dx, dw, seed + i,
+                                                   self.copy_in, st, self.copy_out,
+                                                   buffers_free=ev["out"], inputs_in=ev["in"],
+                                                   step_done=ev["done"], outputs_out=ev["out"])
+        for st in streams:
+            cur.wait_stream(st)
         end = torch.cuda.Event(enable_timing=True)
         end.record(cur)
         return end

@@ -39,7 +39,8 @@ EXPORTS = (
     "shiftquant_gemm_layer", "shiftquant_gemm_layer_workspace_bytes",
     "shiftquant_gemm_layer_workspace_bytes_grouped",
     "shiftquant_gemm_layer_kernel_launches", "shiftquant_gemm_layer_cta_pairs",
-    "shiftquant_layer_step", "shiftquant_layer_step_host", "shiftquant_selftest_wait_timeout",
+    "shiftquant_layer_step", "shiftquant_layer_step_host", "shiftquant_layer_step_host_split",
+    "shiftquant_selftest_wait_timeout",
     "shiftquant_l1bn_state_bytes", "shiftquant_l1bn_forward", "shiftquant_l1bn_backward",
     "shiftquant_group_order", "shiftquant_group_order_width", "shiftquant_quantize_ordered",
     "shiftquant_pack_codes", "shiftquant_unpack_codes", "shiftquant_packed_groups_bytes",
@@ -171,6 +172,9 @@ def load(path: str | None = None) -> ctypes.CDLL:
     lib.shiftquant_layer_step_host.argtypes = [ctypes.POINTER(SqLayerStep), vp, vp, vp, vp, vp,
                                                vp, u64, vp, vp]
     lib.shiftquant_layer_step_host.restype = i32
+    lib.shiftquant_layer_step_host_split.argtypes = [ctypes.POINTER(SqLayerStep), vp, vp, vp, vp,
+                                                     vp, vp, u64, vp, vp, vp, vp, vp, vp, vp]
+    lib.shiftquant_layer_step_host_split.restype = i32
     lib.shiftquant_selftest_wait_timeout.argtypes = [vp, i64, vp, vp, i64, vp, i64, i64, i64,
                                                      i32, i32, vp, i64, vp, vp]
     lib.shiftquant_selftest_wait_timeout.restype = i32
@@ -458,6 +462,23 @@ def shiftquant_layer_step_host(args: SqLayerStep, x_host, w_host, dy_host, y_hos
         ctypes.byref(args), _host_ptr(x_host), _host_ptr(w_host), _host_ptr(dy_host),
         _host_ptr(y_host), _host_ptr(dx_host), _host_ptr(dw_host), seed & (2**64 - 1), ev,
         _stream(stream)))
+
+
+def _event(ev):
+    return ctypes.c_void_p(ev.cuda_event) if ev is not None else None
+
+
+def shiftquant_layer_step_host_split(args: SqLayerStep, x_host, w_host, dy_host, y_host,
+                                     dx_host, dw_host, seed: int, copy_in_stream, stream,
+                                     copy_out_stream, buffers_free, inputs_in, step_done,
+                                     outputs_out) -> None:
+    """The host-fed step with its copies on their own streams (see the header); the events
+    are torch.cuda.Event objects that already exist (buffers_free may be None)."""
+    _check(load().shiftquant_layer_step_host_split(
+        ctypes.byref(args), _host_ptr(x_host), _host_ptr(w_host), _host_ptr(dy_host),
+        _host_ptr(y_host), _host_ptr(dx_host), _host_ptr(dw_host), seed & (2**64 - 1),
+        _stream(copy_in_stream), _stream(stream), _stream(copy_out_stream), _event(buffers_free),
+        _event(inputs_in), _event(step_done), _event(outputs_out)))
 
 
 def shiftquant_selftest_wait_timeout(a_codes, a_scale, b_codes, b_scale, M, N, K, bits, n_groups,

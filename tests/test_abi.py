@@ -247,3 +247,12 @@ def test_layer_step_validates_before_anything_runs(lib):
     assert lib.shiftquant_layer_step_host(ctypes.byref(a), None, None, None, None, None, None, 0,
                                           None, None) == native.SQ_EINVAL
     assert "NULL" in lib.shiftquant_last_error().decode()
+    assert lib.shiftquant_layer_step_host_split(ctypes.byref(a), None, None, None, None, None,
+                                                None, 0, None, None, None, None, fake, fake,
+                                                fake) == native.SQ_EINVAL
+    a.dy = fake
+    # every buffer given: the three events are still required
+    assert lib.shiftquant_layer_step_host_split(ctypes.byref(a), None, None, None, None, None,
+                                                None, 0, None, None, None, None, None, fake,
+                                                fake) == native.SQ_EINVAL
+    assert "inputs_in" in lib.shiftquant_last_error().decode()

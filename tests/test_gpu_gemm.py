@@ -303,9 +303,10 @@ def test_concurrent_step_equals_serial_step():
 
 
 def test_c_host_steps_equal_device_steps():
-    # shiftquant_layer_step_host (copies in, the layer's whole step, copies back, inside one
-    # C call) driven by layer.HostSteps on two alternating buffer sets and streams: every
-    # step's host outputs equal a device-resident step on the same inputs and seed
+    # shiftquant_layer_step_host_split (copies in on a copy-in stream, the layer's whole step
+    # on the layer's stream, copies back on a copy-out stream, inside one C call) driven by
+    # layer.HostSteps on two alternating buffer sets: every step's host outputs equal a
+    # device-resident step on the same inputs and seed
     shapes = [(3000, 640, 384), (3000, 384, 640)]
     bits, G, seed, steps = 6, 4, 0x5EED, 5
     pipe = L.HostSteps(shapes, bits, G, "cuda")
@@ -577,3 +578,23 @@ def test_chain_with_fused_ranges_equals_separate_range_passes(bits):
     for l in range(2):
         want, _ = O.range_cols(a.layers[l].y.cpu().numpy())
         np.testing.assert_array_equal(f32_bits(a.y_range[l].cpu().numpy()), f32_bits(want))
+
+
+def test_c_host_step_on_one_stream_equals_device_step():
+    # shiftquant_layer_step_host: copies in, the step and copies back in one stream's order
+    M, K, Nn = 1000, 384, 640
+    bits, G, seed = 4, 4, 0xBEEF
+    rng = np.random.default_rng(7)
+    x, w, dy = (torch.from_numpy(a).pin_memory() for a in layer_inputs(rng, M, K, Nn))
+    outs = [torch.empty(shp, dtype=torch.float32).pin_memory() for shp in ((M, Nn), (M, K), (K, Nn))]
+    lay = L.QuantLinear(M, K, Nn, bits, G, "cuda", with_inputs=True)
+    ev = torch.cuda.Event()
+    ev.record()
+    N.shiftquant_layer_step_host(lay.step_args(), x, w, dy, *outs, seed, inputs_queued=ev)
+    torch.cuda.synchronize()
+    assert lay.status.item() == 0
+    ref = L.QuantLinear(M, K, Nn, bits, G, "cuda")
+    ref.step(x.cuda(), w.cuda(), dy.cuda(), seed)
+    torch.cuda.synchronize()
+    for got, want in zip(outs, (ref.y, ref.dx, ref.dw)):
+        np.testing.assert_array_equal(got.numpy(), want.cpu().numpy())
