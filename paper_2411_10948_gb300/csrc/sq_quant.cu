@@ -132,34 +132,38 @@ __global__ void __launch_bounds__(THREADS)
   }
 }
 
-// Range pass: block (x, y) reads the 64 x 128 tile (y, x) -- warp w rows 8w .. 8w+7 with
-// all eight 16-byte loads in flight, lane l columns 4l .. 4l+3 -- and takes its per-column
-// maxima as ordered bit patterns of the non-negative floats (NaN sorts above Inf), sent to
-// range_bits with one atomic max per column.  Same-address atomics from hundreds of tiles
-// of a narrow tensor serialise in L2, so narrow tensors (CL = kRangeCluster) run in
-// clusters of CL blocks along the rows: each block merges its maxima into the first block
-// of its cluster with atomic maxima on that block's shared memory, and only that block
-// sends them on.  Wide tensors (CL = 1) spread their atomics over many addresses and run
-// without clusters, which schedule more slowly.  Grids taller than the 65535-block limit
+// Range pass: block (x, y) reads tile (y, x) of TC = 4 << lg columns (the column count
+// rounded up to a power of two, 4 to 128) by 8 passes of 1024 / TC rows -- thread t owns
+// the four-column quad t mod (TC / 4) and the rows t / (TC / 4) + k 1024 / TC, with all
+// eight 16-byte loads in flight -- and takes its per-column maxima as ordered bit patterns
+// of the non-negative floats (NaN sorts above Inf), sent to range_bits with one atomic max
+// per column.  Same-address atomics from hundreds of tiles of a narrow tensor serialise in
+// L2, so narrow tensors (CL = kRangeCluster) run in clusters of CL blocks along the rows:
+// each block merges its maxima into the first block of its cluster with atomic maxima on
+// that block's shared memory, and only that block sends them on.  Wide tensors (CL = 1)
+// spread their atomics over many addresses and run without clusters, which schedule more
+// slowly.  Grids taller than the 65535-block limit
 // walk the extra tiles in steps of gridDim.y.
 // ROWS: the range pass of a weight for both of its roles -- also every row's max|x| over
 // all columns (the per-in-channel ranges), each warp's eight rows of a tile reduced across
 // its lanes and sent to row_bits with one atomic max per row and column block.
-constexpr int kRangeRows = 64;
 constexpr int kRangeCluster = 8;
-constexpr int64_t kRangeClusterMaxCols = 4 * kColTx * 4;   // clusters up to 4 column blocks
+constexpr int64_t kRangeClusterMaxCols = 512;   // clusters for tensors of at most 512 columns
 
 template <int CL, bool ROWS>
 __global__ void __launch_bounds__(kColTx* kColTy)
-    colmax_kernel(const float* __restrict__ x, int64_t R, int64_t C, int64_t ld, int vec,
+    colmax_kernel(const float* __restrict__ x, int64_t R, int64_t C, int64_t ld, int vec, int lg,
                   unsigned* __restrict__ range_bits, unsigned* __restrict__ row_bits,
                   int* __restrict__ status) {
-  __shared__ unsigned red[kColTy][kColTx * 4];
+  __shared__ unsigned red[kColTy * kColTx * 4];
   __shared__ unsigned cmax[CL > 1 ? kColTx * 4 : 1];   // the cluster's maxima (first block)
-  const int tx = threadIdx.x, ty = threadIdx.y;   // tx: lane (columns), ty: warp (rows)
-  const int tid = ty * kColTx + tx;
-  const int64_t c0 = (static_cast<int64_t>(blockIdx.x) * kColTx + tx) * 4;
-  const int64_t tiles = (R + kRangeRows - 1) / kRangeRows;
+  const int tid = threadIdx.y * kColTx + threadIdx.x;
+  // the tile: tc = 4 << lg columns (one four-column quad per thread) by 8 passes of rpp rows
+  const int tc = 4 << lg, rpp = (kColTx * kColTy) >> lg;
+  const int qc = tid & ((1 << lg) - 1), ro = tid >> lg;
+  const int64_t c0 = static_cast<int64_t>(blockIdx.x) * tc + 4 * qc;
+  const int64_t tile_rows = 8 * static_cast<int64_t>(rpp);
+  const int64_t tiles = (R + tile_rows - 1) / tile_rows;
   if (CL > 1) {
     if (tid < kColTx * 4) cmax[tid] = 0u;
     cluster_arrive_release();   // the zeroed cmax is visible to the cluster after the wait
@@ -168,13 +172,13 @@ __global__ void __launch_bounds__(kColTx* kColTy)
   bool row_bad = false;
 #pragma unroll 1
   for (int64_t t = blockIdx.y; t < tiles; t += gridDim.y) {
-    const int64_t r0 = t * kRangeRows + ty * 8;
+    const int64_t r0 = t * tile_rows + ro;   // this thread's rows: r0 + u rpp
     unsigned rm[8];   // ROWS: this thread's four columns of each of its rows
     if (vec && c0 + 3 < C) {
       // rows past the end re-read the last row, which leaves a maximum unchanged
       float4 v[8];
 #pragma unroll
-      for (int u = 0; u < 8; ++u) v[u] = ld_stream_v4(x + min(r0 + u, R - 1) * ld + c0);
+      for (int u = 0; u < 8; ++u) v[u] = ld_stream_v4(x + min(r0 + u * rpp, R - 1) * ld + c0);
 #pragma unroll
       for (int u = 0; u < 8; ++u) {
         const unsigned a0 = abs_bits(v[u].x), a1 = abs_bits(v[u].y);
@@ -190,7 +194,7 @@ __global__ void __launch_bounds__(kColTx* kColTy)
       for (int u = 0; u < 8; ++u) rm[u] = 0u;
 #pragma unroll 1
       for (int u = 0; u < 8; ++u) {
-        const int64_t r = r0 + u;
+        const int64_t r = r0 + u * rpp;
         if (r >= R) break;
         const float* row = x + r * ld;
         unsigned a[4] = {0u, 0u, 0u, 0u};
@@ -209,13 +213,15 @@ __global__ void __launch_bounds__(kColTx* kColTy)
       }
     }
     if (ROWS) {
+      // (lg = 5: a warp's 32 quads are one row of the tile, a warp row per pass)
       // the row accumulators are zeroed by the preceding kernel, which must have completed
       griddep_wait();
 #pragma unroll
       for (int u = 0; u < 8; ++u) {
         const unsigned m = __reduce_max_sync(0xFFFFFFFFu, rm[u]);
-        if (tx == 0 && r0 + u < R && m != 0u) {
-          atomicMax(row_bits + r0 + u, m);
+        const int64_t r = r0 + u * rpp;
+        if (threadIdx.x == 0 && r < R && m != 0u) {
+          atomicMax(row_bits + r, m);
           row_bad |= m >= 0x7F800000u;
         }
       }
@@ -224,48 +230,31 @@ __global__ void __launch_bounds__(kColTx* kColTy)
   if (ROWS && row_bad) atomicOr(status, kDevNonFinite);
   // x has been read: the next kernel (the grouping) may start launching
   griddep_launch_dependents();
-  red[ty][tx * 4 + 0] = m0;
-  red[ty][tx * 4 + 1] = m1;
-  red[ty][tx * 4 + 2] = m2;
-  red[ty][tx * 4 + 3] = m3;
+  red[ro * tc + 4 * qc + 0] = m0;
+  red[ro * tc + 4 * qc + 1] = m1;
+  red[ro * tc + 4 * qc + 2] = m2;
+  red[ro * tc + 4 * qc + 3] = m3;
   __syncthreads();
-  unsigned m[4];
-  if (ty == 0) {
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      m[i] = 0;
-#pragma unroll
-      for (int y = 0; y < kColTy; ++y) m[i] = max(m[i], red[y][tx * 4 + i]);
-    }
-  }
+  // thread t < tc: column t of the tile
+  unsigned m = 0;
+  if (tid < tc)
+    for (int y = 0; y < rpp; ++y) m = max(m, red[y * tc + tid]);
   if (CL > 1) {
     cluster_wait_acquire();
-    if (ty == 0) {
-      const uint32_t lead = mapa_shared(smem_u32(cmax), 0);
-#pragma unroll
-      for (int i = 0; i < 4; ++i)
-        if (m[i] != 0) red_max_cluster_u32(lead + (tx * 4 + i) * 4, m[i]);
-    }
+    if (tid < tc && m != 0) red_max_cluster_u32(mapa_shared(smem_u32(cmax), 0) + tid * 4, m);
     cluster_arrive_release();
     cluster_wait_acquire();   // every block's maxima are in the first block's cmax
     if (cluster_ctarank() != 0) return;
-    if (ty == 0) {
-#pragma unroll
-      for (int i = 0; i < 4; ++i) m[i] = cmax[tx * 4 + i];
-    }
+    if (tid < tc) m = cmax[tid];
   }
-  if (ty != 0) return;
+  if (tid >= tc) return;
   // the accumulators are zeroed by the preceding kernel, which must have completed
   griddep_wait();
-  bool bad = false;
-#pragma unroll
-  for (int i = 0; i < 4; ++i) {
-    if (c0 + i < C && m[i] != 0) {
-      atomicMax(range_bits + c0 + i, m[i]);
-      bad |= m[i] >= 0x7F800000u;
-    }
+  const int64_t c = static_cast<int64_t>(blockIdx.x) * tc + tid;
+  if (c < C && m != 0) {
+    atomicMax(range_bits + c, m);
+    if (m >= 0x7F800000u) atomicOr(status, kDevNonFinite);
   }
-  if (bad) atomicOr(status, kDevNonFinite);
 }
 
 // one warp per row: range[r] = max_c |x[r, c]|
@@ -777,13 +766,20 @@ __global__ void __launch_bounds__(256)
 }
 
 // The range pass of x [rows, cols] (0 < rows, 0 < cols < 2^36, checked by the callers):
-// one block per 64 x 128 tile, narrow tensors in whole clusters along the rows; with
+// one block per tile, narrow tensors in whole clusters along the rows; with
 // row_bits also the per-row maxima.
 static cudaError_t launch_range(const float* x, int64_t rows, int64_t cols, int64_t ld,
                                 unsigned* col_bits, unsigned* row_bits, int* status,
                                 cudaStream_t s) {
-  const int64_t cblocks = (cols + kColTx * 4 - 1) / (kColTx * 4);   // <= 2^29: cols < 2^36
-  const int64_t tiles = (rows + kRangeRows - 1) / kRangeRows;
+  // the tile: the column count rounded up to a power of two (4 .. 128) wide, 1024 elements;
+  // a weight's row ranges need whole 128-column warp rows
+  int lg = 5;
+  if (row_bits == nullptr)
+    for (lg = 0; lg < 5 && (int64_t(4) << lg) < cols; ++lg) {
+    }
+  const int64_t tc = int64_t(4) << lg;
+  const int64_t cblocks = (cols + tc - 1) / tc;   // < 2^29: cols < 2^36, tc = 128 past 64
+  const int64_t tiles = (rows + 8 * (256 >> lg) - 1) / (8 * (256 >> lg));
   const int cl = cols <= kRangeClusterMaxCols ? kRangeCluster : 1;
   const int64_t max_rblocks = 65535 / cl * cl;
   int64_t rblocks = (tiles + cl - 1) / cl * cl;
@@ -806,13 +802,13 @@ static cudaError_t launch_range(const float* x, int64_t rows, int64_t cols, int6
   cudaError_t err;
   if (row_bits != nullptr)
     err = cl > 1 ? cudaLaunchKernelEx(&cfg, colmax_kernel<kRangeCluster, true>, x, rows, cols, ld, vec,
-                                      col_bits, row_bits, status)
-                 : cudaLaunchKernelEx(&cfg, colmax_kernel<1, true>, x, rows, cols, ld, vec, col_bits,
+                                      lg, col_bits, row_bits, status)
+                 : cudaLaunchKernelEx(&cfg, colmax_kernel<1, true>, x, rows, cols, ld, vec, lg, col_bits,
                                       row_bits, status);
   else
     err = cl > 1 ? cudaLaunchKernelEx(&cfg, colmax_kernel<kRangeCluster, false>, x, rows, cols, ld, vec,
-                                      col_bits, row_bits, status)
-                 : cudaLaunchKernelEx(&cfg, colmax_kernel<1, false>, x, rows, cols, ld, vec, col_bits,
+                                      lg, col_bits, row_bits, status)
+                 : cudaLaunchKernelEx(&cfg, colmax_kernel<1, false>, x, rows, cols, ld, vec, lg, col_bits,
                                       row_bits, status);
   if (err == cudaSuccess) err = cudaGetLastError();
   return err;
