@@ -144,8 +144,11 @@ class Step:
         self.layers, self.inputs = [], []
         for i, spec in enumerate(wl.layers):
             self.inputs.append(W.torch_layer_inputs(spec, seed, i, device))
+            # transposed code copies only where the library advises them (the weight
+            # gradient otherwise reads X's and dY's codes in place)
             self.layers.append(L.QuantLinear(spec.M, spec.K, spec.N, spec.bits, spec.n_groups,
-                                             device, with_acc=False, use_workspace=True))
+                                             device, with_acc=False, use_workspace=True,
+                                             transposed=None))
         self.specs = list(wl.layers)
 
     # (name, callable) for every library call of one step, in order
@@ -181,11 +184,18 @@ class Step:
         for s, lay, gb in zip(self.specs, self.layers, self.gemm_bytes_per_launch()):
             cb = self.N.shiftquant_code_bytes(s.bits, s.n_groups)
             MK, MN, KN = s.M * s.K, s.M * s.N, s.K * s.N
-            out += [(s.name, "X", 4 * MK), (s.name, "X", 4 * MK + 2 * cb * MK),
-                    (s.name, "dY", 4 * MN), (s.name, "dY", 4 * MN + 2 * cb * MN),
+            cx, cg = self.code_copies(lay)
+            out += [(s.name, "X", 4 * MK), (s.name, "X", 4 * MK + cx * cb * MK),
+                    (s.name, "dY", 4 * MN), (s.name, "dY", 4 * MN + cg * cb * MN),
                     (s.name, "W (both roles)", 4 * KN), (s.name, "W (both roles)", 4 * KN + 2 * cb * KN),
                     (s.name, "GEMMs", gb)]
         return out
+
+    @staticmethod
+    def code_copies(lay):
+        """Code sets the quantizer writes for X and dY: the codes, plus the transposed copy
+        where the layer keeps one."""
+        return (1 + (lay.x.codes_t is not None), 1 + (lay.g.codes_t is not None))
 
     def group_histograms(self):
         """Channels per group of every grouped tensor (after the last step)."""
@@ -215,12 +225,14 @@ class Step:
         return [3 * 2 * l.M * l.N * l.K for l in self.layers]
 
     def gemm_bytes_per_launch(self):
-        """Algorithmic HBM bytes of each layer's GEMM launch: every operand code read once,
-        every fp32 output written once."""
+        """Algorithmic HBM bytes of each layer's GEMM launch: every GEMM's operand codes read
+        once, every fp32 output written once."""
         out = []
         for s, lay in zip(self.specs, self.layers):
             cb = self.N.shiftquant_code_bytes(s.bits, s.n_groups)
-            codes = cb * (2 * s.M * s.K + 2 * s.M * s.N + 2 * s.K * s.N)  # X, X^T, dY, dY^T, W x2
+            # X and dY codes twice each (forward / loss propagation, and the weight gradient,
+            # in place or from the transposed copy), both weight roles
+            codes = cb * (2 * s.M * s.K + 2 * s.M * s.N + 2 * s.K * s.N)
             outs = 4 * (s.M * s.N + s.M * s.K + s.K * s.N)
             out.append(codes + outs)
         return out
@@ -232,10 +244,11 @@ class Step:
     def quantize_bytes(self) -> int:
         """Algorithmic HBM bytes of the quantize passes of one step."""
         tot = 0
-        for s in self.specs:
+        for s, lay in zip(self.specs, self.layers):
             cb = self.N.shiftquant_code_bytes(s.bits, s.n_groups)
-            for R, C in ((s.M, s.K), (s.M, s.N)):        # X and dY: read, codes + transposed
-                tot += 4 * R * C + 2 * cb * R * C
+            # X and dY: read, codes (+ the transposed copy where kept)
+            for (R, C), n in zip(((s.M, s.K), (s.M, s.N)), self.code_copies(lay)):
+                tot += 4 * R * C + n * cb * R * C
             tot += 4 * s.K * s.N + 2 * cb * s.K * s.N    # W: one read, both roles' codes
         return tot
 
@@ -606,7 +619,9 @@ def run_ours(args, rank, world, local_rank):
                      int8_peak="none: sm_103a has no integer MMA (tcgen05 kind::i8 does not "
                                "assemble); exact integers run on the E4M3/BF16 tensor cores"),
         "quantizer": dict(quant_roof, bytes_per_step=st.quantizer_bytes(),
-                          nominal_hbm_gbs=7900.0, frac_nominal=q_gbs / 7900.0),
+                          nominal_hbm_gbs=7900.0, frac_nominal=q_gbs / 7900.0,
+                          transposed_copies={s.name: lay.x.codes_t is not None
+                                             for s, lay in zip(st.specs, st.layers)}),
         "breakdown_ms_per_step": {k: v / args.steps for k, v in kind_ms.items()},
         "calls_ms_per_step": [[f"{n}", round(v / args.steps, 5)] for n, v in zip(names, call_ms)],
         "quantizer_per_tensor": per_tensor,
@@ -782,8 +797,9 @@ def run_group_order(args, dev):
 
 
 def run_pack(args, dev):
-    """Packed sub-byte storage of the 4-bit conv3x3 activation codes (X [12544, 2304] and the
-    transposed copy the weight gradient keeps): pack (1 byte read + 0.5 written per code) and
+    """Packed sub-byte storage of the 4-bit conv3x3 activation codes (X [12544, 2304], and its
+    transposed copy [2304, 12544], the layout a group-ordered layer's weight gradient reads):
+    pack (1 byte read + 0.5 written per code) and
     unpack (0.5 + 1), each captured in a CUDA graph and timed with CUDA events around a
     replay after an L2 flush (median), against HBM."""
     import torch

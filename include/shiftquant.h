@@ -296,7 +296,11 @@ sq_status shiftquant_gemm_wgrad_finish(const int32_t *t, int64_t Ci, int64_t Co,
  *   loss propagation   dx [M, K] from g_codes [M, N] and wd_codes [K, N] (per-in-channel W
  *                      codes, dY's shifts folded in), scales g_scale, wd_scale[K]
  *   weight gradient    dw [K, N] from xt_codes [K, M] and gt_codes [N, M] with the exponents
- *                      x_exp[K], g_exp[N] and the scales x_scale, g_scale
+ *                      x_exp[K], g_exp[N] and the scales x_scale, g_scale.  xt_codes NULL:
+ *                      it reads x_codes [M, ld_x] in place (the tensor core takes the
+ *                      operand MN-major), so X needs no transposed copy; gt_codes NULL
+ *                      likewise reads g_codes.  Not with x_seg (g_seg): a group-ordered
+ *                      operand's channels are permuted, and the call returns SQ_EINVAL.
  * acc_* are the optional int64 exactness-check outputs.  The struct lives in host memory and
  * is read during the call only.
  * The launch sizes the exact FP32 accumulation chunks of the forward and loss-propagation
@@ -382,12 +386,24 @@ int shiftquant_gemm_layer_kernel_launches(int64_t M, int64_t K, int64_t N, int b
 int shiftquant_gemm_layer_cta_pairs(int64_t M, int64_t K, int64_t N, int bits, int n_groups,
                                     int gemm_mask);
 
+/* Layout advice for a layer's X and dY codes on the current device: 1 when the weight
+ * gradient of shiftquant_gemm_layer (all three GEMMs, this shape) is expected to run as fast
+ * on the codes in place (xt_codes / gt_codes NULL) as on transposed copies -- so the
+ * quantizer can skip writing the copies; 0 when transposed copies are faster (an MN-major
+ * operand slows the tensor core where it sets the launch's pace: CTA pairs, unsplit units
+ * filling at least half the pairs, K loops of 64 blocks or more); -1 for invalid arguments,
+ * a shape beyond the exact range, or no device.  Results do not depend on the choice. */
+int shiftquant_gemm_layer_wgrad_in_place(int64_t M, int64_t K, int64_t N, int bits,
+                                         int n_groups);
+
 /* One training step of one quantized linear layer X [M, K], W [K, N], dY [M, N], with the
  * operand roles of the paper's setup (Sec. 5.1): every quantizer pass and the three GEMMs
  * (Eq. 4 with the left-shift form of App. D), in stream order:
  *   1. X:  range pass + grouping (Sec. 3.1, Eq. 3), codes and transposed codes, round to
- *          nearest even (App. D);
- *   2. dY: the same with stochastic rounding (App. B) drawn under `seed`;
+ *          nearest even (App. D); xt_codes NULL writes no transposed copy, and the weight
+ *          gradient reads x_codes in place (see sq_layer_gemms);
+ *   2. dY: the same with stochastic rounding (App. B) drawn under `seed` (gt_codes NULL:
+ *          likewise);
  *   3. W per out-channel (forward role): codes written transposed [N, K] with X's group
  *      shifts folded in; W per in-channel (loss-propagation role): codes [K, N] with dY's
  *      shifts folded in -- both roles by shiftquant_calibrate_weight and
@@ -397,8 +413,9 @@ int shiftquant_gemm_layer_cta_pairs(int64_t M, int64_t K, int64_t N, int bits, i
  * Every buffer is a caller-owned DEVICE buffer; the layouts are those of the calls above:
  *   x [M, K], w [K, N], dy [M, N], y [M, N], dx [M, K], dw [K, N]: fp32, dense row-major
  *     (leading dimension = row length).  x, w and dy are written only by the host variant.
- *   x_codes [M, ld_x], xt_codes [K, ld_xt], x_range[K], x_exp[K], x_tau0, x_scale (one
- *     float each); g_codes [M, ld_g], gt_codes [N, ld_gt], g_range[N], g_exp[N], g_tau0,
+ *   x_codes [M, ld_x], xt_codes [K, ld_xt] (or NULL), x_range[K], x_exp[K], x_tau0,
+ *     x_scale (one float each); g_codes [M, ld_g], gt_codes [N, ld_gt] (or NULL), g_range[N],
+ *     g_exp[N], g_tau0,
  *     g_scale; wf_codes [N, ld_wf], wf_range[N], wf_scale[N]; wd_codes [K, ld_wd],
  *     wd_range[K], wd_scale[K].  Codes in the type of shiftquant_code_type(bits, n_groups),
  *     rows 16-byte aligned (ld * code bytes a multiple of 16, pointers 16-byte aligned).

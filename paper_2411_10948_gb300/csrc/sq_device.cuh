@@ -384,6 +384,12 @@ __host__ __device__ constexpr uint32_t make_idesc(uint32_t fmt, uint32_t M, uint
          | ((M >> 4) << 24);       // M / 16
 }
 
+// The operand-major bits of an instruction descriptor: A (bit 15) and B (bit 16) read from
+// MN-major tiles instead of K-major ones.
+__host__ __device__ constexpr uint32_t idesc_mn_major(bool a_mn, bool b_mn) {
+  return (a_mn ? 1u << 15 : 0u) | (b_mn ? 1u << 16 : 0u);
+}
+
 // Shared-memory matrix descriptor for a K-major operand tile written by TMA with
 // 128-byte swizzle: rows of 128 bytes, 8-row (1024-byte) swizzle atoms stacked along
 // M/N, so the stride between atoms is 1024 bytes.  The tile base is 1024-byte aligned;
@@ -392,6 +398,21 @@ __device__ __forceinline__ uint64_t make_sdesc_k_sw128(uint32_t saddr) {
   uint64_t d = 0;
   d |= static_cast<uint64_t>((saddr & 0x3FFFFu) >> 4);   // start address
   d |= static_cast<uint64_t>(1) << 16;                    // leading byte offset (unused)
+  d |= static_cast<uint64_t>(1024 >> 4) << 32;            // stride byte offset
+  d |= static_cast<uint64_t>(1) << 46;                    // descriptor version (sm_100+)
+  d |= static_cast<uint64_t>(2) << 61;                    // swizzle: 128 bytes
+  return d;
+}
+
+// Shared-memory matrix descriptor for an MN-major operand tile written by TMA with 128-byte
+// swizzle: a 128-byte row holds consecutive M (or N) elements at one k, 8 consecutive k rows
+// form a 1024-byte swizzle atom, so the stride between atoms along K (stride byte offset) is
+// 1024 bytes; `mn_stride` bytes separate the 128-byte-wide column blocks along M/N (leading
+// byte offset).  A K step inside the tile moves the start address by whole rows.
+__device__ __forceinline__ uint64_t make_sdesc_mn_sw128(uint32_t saddr, uint32_t mn_stride) {
+  uint64_t d = 0;
+  d |= static_cast<uint64_t>((saddr & 0x3FFFFu) >> 4);   // start address
+  d |= static_cast<uint64_t>(mn_stride >> 4) << 16;       // leading byte offset
   d |= static_cast<uint64_t>(1024 >> 4) << 32;            // stride byte offset
   d |= static_cast<uint64_t>(1) << 46;                    // descriptor version (sm_100+)
   d |= static_cast<uint64_t>(2) << 61;                    // swizzle: 128 bytes

@@ -151,6 +151,10 @@ struct GemmBatch {
   // and each chunk's sum is multiplied by the segment's shift 2^(G-1-g) in the epilogue.
   const int* seg[kMaxBatch];
   int segmented;  // some GEMM is group-ordered (every role waits for the table)
+  // per GEMM: bit 0 set when A, bit 1 when B is stored MN-major ([K, ld] with the M or N
+  // index contiguous: the weight gradient reading the activation and gradient codes in
+  // their own layout instead of transposed copies); clear: K-major ([M or N, ld])
+  int mn[kMaxBatch];
 };
 
 __device__ __forceinline__ float pow2_neg(int k) { return __int_as_float((127 - k) << 23); }
@@ -577,10 +581,69 @@ __device__ __noinline__ void plan_chunks(const GemmBatch& bt, volatile int* out,
   }
 }
 
+// One operand tile of a pipeline stage: kRows rows of the M (or N) index from r0, one K
+// block from k0, landing at dst (1 KB aligned) with its bytes counted on `bar`.
+//   K-major: one box of kRows rows x 128 bytes of K.
+//   MN-major: one box per 128 bytes of M (64 BF16 or 128 E4M3 elements) x the K block's
+//   rows, placed one after another; each is a column of whole 1 KB swizzle atoms (8 K rows
+//   of 128 bytes), which is the layout make_sdesc_mn_sw128 describes.
+template <int kF8, bool kPair, int kRows>
+__device__ __forceinline__ void load_operand(uint32_t dst, const CUtensorMap* map, uint32_t bar,
+                                             int32_t k0, int32_t r0, bool mn) {
+  constexpr int kBKElems = kF8 ? kBKBytes : kBKBytes / 2;
+  constexpr int kMnElems = kF8 ? 128 : 64;
+  if (!mn) {
+    if constexpr (kPair)
+      tma_load_2d_pair(dst, map, bar, k0, r0);
+    else
+      tma_load_2d(dst, map, bar, k0, r0);
+    return;
+  }
+#pragma unroll
+  for (int j = 0; j < kRows / kMnElems; ++j) {
+    if constexpr (kPair)
+      tma_load_2d_pair(dst + j * kBKElems * 128, map, bar, r0 + j * kMnElems, k0);
+    else
+      tma_load_2d(dst + j * kBKElems * 128, map, bar, r0 + j * kMnElems, k0);
+  }
+}
+
+// The MMAs of one K block of a stage at a0 (A tile, then the B tile kABytes on), into the
+// TMEM accumulator d (cleared by the block's first MMA when `first`).  An MMA takes 32
+// bytes of K: 32 bytes along a K-major row, or that many 128-byte rows of an MN-major tile,
+// whose 128-byte column blocks of M (N) lie a whole K block apart (a tile one block wide
+// never steps to a second one, and its stride is given as one atom).
+template <int kF8, int kCg, int kBRows, bool kAMn, bool kBMn>
+__device__ __forceinline__ void mma_kblock(uint32_t d, uint32_t a0, bool first) {
+  constexpr int kBKElems = kF8 ? kBKBytes : kBKBytes / 2;
+  constexpr uint32_t kMnKStep = (kF8 ? 32 : 16) * 128;
+  constexpr uint32_t kMnBlock = kBKElems * 128;
+  constexpr uint32_t kStrideA = kBM * (kF8 ? 1 : 2) > 128 ? kMnBlock : 1024;
+  constexpr uint32_t kStrideB = kBRows * (kF8 ? 1 : 2) > 128 ? kMnBlock : 1024;
+  constexpr uint32_t idesc =
+      make_idesc(kF8 ? 0u : 1u, kCg * kBM, kBN) | idesc_mn_major(kAMn, kBMn);
+  const uint32_t b0 = a0 + kABytes;
+#pragma unroll
+  for (int k = 0; k < kBKBytes / 32; ++k) {
+    const uint64_t ad = kAMn ? make_sdesc_mn_sw128(a0 + k * kMnKStep, kStrideA)
+                             : make_sdesc_k_sw128(a0 + k * 32);
+    const uint64_t bd = kBMn ? make_sdesc_mn_sw128(b0 + k * kMnKStep, kStrideB)
+                             : make_sdesc_k_sw128(b0 + k * 32);
+    const uint32_t accumulate = (!first || k > 0) ? 1u : 0u;
+    if (kF8)
+      tc_mma_f8<kCg>(d, ad, bd, idesc, accumulate);
+    else
+      tc_mma_f16<kCg>(d, ad, bd, idesc, accumulate);
+  }
+}
+
 // kMulti: the K loop of a tile spans several exact chunks, whose int32 sums the epilogue
 // keeps in registers; otherwise every output streams from TMEM once.
 // kPair: launched as 2-CTA clusters running 256-row tiles (the host sets the cluster shape)
-template <int kF8, bool kMulti, bool kPair>
+// kMn: some GEMM of the launch reads an operand MN-major (bt.mn); without it the copy and
+// MMA loops hold the K-major form alone (measured: the MN branches in them, never taken,
+// cost K-major launches 8-10%)
+template <int kF8, bool kMulti, bool kPair, bool kMn>
 __global__ void __launch_bounds__(kThreads, 1) shiftmm_kernel(const __grid_constant__ GemmBatch bt) {
   using L = Smem<kPair>;
   constexpr int kCg = kPair ? 2 : 1;
@@ -728,6 +791,7 @@ __global__ void __launch_bounds__(kThreads, 1) shiftmm_kernel(const __grid_const
       }
       const int g = r.g;
       const Unit w = r.w;
+      const int mn = kMn ? bt.mn[g] : 0;
       // rows past M (and columns past N) are read as zeros and never stored
       const int32_t ya = w.mb * L::tile_m + static_cast<int32_t>(rank) * kBM;
       const int32_t yb = w.nb * kBN + static_cast<int32_t>(rank) * L::b_rows;
@@ -743,12 +807,19 @@ __global__ void __launch_bounds__(kThreads, 1) shiftmm_kernel(const __grid_const
         const uint32_t sa = smem_u32(smem + s * L::stage_bytes);
         if (rank == 0) mbar_arrive_expect_tx(&full[s], kCg * L::stage_bytes);
         if (!bt.no_copies) {
-          if constexpr (kPair) {
-            tma_load_2d_pair(sa, &bt.a[g], full_c + s * 8, kb * kBKElems, ya);
-            tma_load_2d_pair(sa + kABytes, &bt.b[g], full_c + s * 8, kb * kBKElems, yb);
+          if (!kMn || mn == 0) {
+            if constexpr (kPair) {
+              tma_load_2d_pair(sa, &bt.a[g], full_c + s * 8, kb * kBKElems, ya);
+              tma_load_2d_pair(sa + kABytes, &bt.b[g], full_c + s * 8, kb * kBKElems, yb);
+            } else {
+              tma_load_2d(sa, &bt.a[g], smem_u32(&full[s]), kb * kBKElems, ya);
+              tma_load_2d(sa + kABytes, &bt.b[g], smem_u32(&full[s]), kb * kBKElems, yb);
+            }
           } else {
-            tma_load_2d(sa, &bt.a[g], smem_u32(&full[s]), kb * kBKElems, ya);
-            tma_load_2d(sa + kABytes, &bt.b[g], smem_u32(&full[s]), kb * kBKElems, yb);
+            const uint32_t bar = kPair ? full_c + s * 8 : smem_u32(&full[s]);
+            load_operand<kF8, kPair, kBM>(sa, &bt.a[g], bar, kb * kBKElems, ya, mn & 1);
+            load_operand<kF8, kPair, L::b_rows>(sa + kABytes, &bt.b[g], bar, kb * kBKElems, yb,
+                                                mn & 2);
           }
           ++issued;
         }
@@ -785,7 +856,6 @@ __global__ void __launch_bounds__(kThreads, 1) shiftmm_kernel(const __grid_const
     // ------------------------------------------------- MMA issuer (the leader's)
     // In a pair: 256 x 256 MMAs; a stage is released in both CTAs, and a finished chunk
     // announced to both CTAs' epilogues, by multicast commits.
-    constexpr uint32_t idesc = make_idesc(kF8 ? 0u : 1u, L::tile_m, kBN);
     int s = 0;
     uint32_t ph = 0;
     uint32_t c = 0;
@@ -811,6 +881,7 @@ __global__ void __launch_bounds__(kThreads, 1) shiftmm_kernel(const __grid_const
       const volatile int* segkb =
           bt.seg[g] != nullptr ? reinterpret_cast<volatile int*>(smem + L::seg_offset) + g * kSegSlots : nullptr;
       const int kend = segkb != nullptr ? min(w.kb1, segkb[bt.p[g].G]) : w.kb1;
+      const int mn = kMn ? bt.mn[g] : 0;
       int kce;
       for (int kc = w.kb0; kc < kend && ok; kc = kce) {
         int sh_unused;
@@ -829,16 +900,16 @@ __global__ void __launch_bounds__(kThreads, 1) shiftmm_kernel(const __grid_const
           }
           tc_fence_after();
           const uint32_t a0 = smem_u32(smem + s * L::stage_bytes);
-          const uint32_t b0 = a0 + kABytes;
-#pragma unroll
-          for (int k = 0; k < kBKBytes / 32; ++k) {
-            const uint64_t ad = make_sdesc_k_sw128(a0 + k * 32);
-            const uint64_t bd = make_sdesc_k_sw128(b0 + k * 32);
-            const uint32_t accumulate = (kb > kc || k > 0) ? 1u : 0u;
-            if (kF8)
-              tc_mma_f8<kCg>(d, ad, bd, idesc, accumulate);
-            else
-              tc_mma_f16<kCg>(d, ad, bd, idesc, accumulate);
+          const bool first = kb == kc;
+          if constexpr (!kMn) {
+            mma_kblock<kF8, kCg, L::b_rows, false, false>(d, a0, first);
+          } else {
+            switch (mn) {  // the operand layouts as compile-time descriptor steps
+              case 0: mma_kblock<kF8, kCg, L::b_rows, false, false>(d, a0, first); break;
+              case 1: mma_kblock<kF8, kCg, L::b_rows, true, false>(d, a0, first); break;
+              case 2: mma_kblock<kF8, kCg, L::b_rows, false, true>(d, a0, first); break;
+              default: mma_kblock<kF8, kCg, L::b_rows, true, true>(d, a0, first); break;
+            }
           }
           tc_commit<kCg>(smem_u32(&empty[s]), 0x3);  // frees the stage (in both CTAs)
           if (++s == kStages) {
@@ -1138,6 +1209,27 @@ static int make_operand_map(CUtensorMap* map, const void* base, int64_t rows, in
   return SQ_OK;
 }
 
+// MN-major operand: K rows of `mn` elements, leading dimension ld (elements), the M (or N)
+// index contiguous: boxes of 128 bytes of M x one K block of rows, 128-byte swizzle, zero
+// fill outside the tensor
+static int make_operand_map_mn(CUtensorMap* map, const void* base, int64_t mn, int64_t K,
+                               int64_t ld, int elem_bytes) {
+  auto fn = encode_fn();
+  if (!fn) return fail(SQ_ECUDA, "cuTensorMapEncodeTiled is not available from the driver");
+  const CUtensorMapDataType dt =
+      elem_bytes == 2 ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_UINT8;
+  cuuint64_t gdim[2] = {static_cast<cuuint64_t>(mn), static_cast<cuuint64_t>(K)};
+  cuuint64_t gstride[1] = {static_cast<cuuint64_t>(ld * elem_bytes)};
+  cuuint32_t box[2] = {static_cast<cuuint32_t>(kBKBytes / elem_bytes),
+                       static_cast<cuuint32_t>(kBKBytes / elem_bytes)};
+  cuuint32_t estride[2] = {1, 1};
+  const CUresult r = fn(map, dt, 2, const_cast<void*>(base), gdim, gstride, box, estride,
+                        CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                        CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) return fail(SQ_ECUDA, "cuTensorMapEncodeTiled (MN-major) failed (%d)", static_cast<int>(r));
+  return SQ_OK;
+}
+
 // fp32 output or int32 split-K workspace [rows, cols] (leading dimension ld elements):
 // 32 x 32 boxes with 128-byte swizzle, matching the epilogue's staging layout
 static int make_output_map(CUtensorMap* map, void* base, int64_t rows, int64_t cols, int64_t ld,
@@ -1252,11 +1344,11 @@ static size_t split_ws_bytes(int64_t M, int64_t N, bool wide = false) {
 // The layer launch's workspace starts with the unit counter of its dynamic schedule.
 constexpr size_t kSchedBytes = 256;
 
-template <int kF8, bool kMulti, bool kPair>
+template <int kF8, bool kMulti, bool kPair, bool kMn>
 static int configure_kernel(int dev) {
   static bool done[64] = {};
   if (dev >= 0 && dev < 64 && done[dev]) return SQ_OK;
-  const cudaError_t err = cudaFuncSetAttribute(shiftmm_kernel<kF8, kMulti, kPair>,
+  const cudaError_t err = cudaFuncSetAttribute(shiftmm_kernel<kF8, kMulti, kPair, kMn>,
                                                cudaFuncAttributeMaxDynamicSharedMemorySize,
                                                static_cast<int>(Smem<kPair>::bytes));
   if (err != cudaSuccess) return cuda_fail(err, "cudaFuncSetAttribute");
@@ -1274,7 +1366,7 @@ static int device_pairs(int* dev_out) {
   if (dev_out) *dev_out = dev;
   if (dev >= 0 && dev < 64 && cached[dev] > 0) return cached[dev];
   int pairs = sms / 2;
-  if (configure_kernel<1, false, true>(dev) == SQ_OK) {
+  if (configure_kernel<1, false, true, false>(dev) == SQ_OK) {
     cudaLaunchAttribute at[1];
     at[0].id = cudaLaunchAttributeClusterDimension;
     at[0].val.clusterDim.x = 2;
@@ -1287,7 +1379,8 @@ static int device_pairs(int* dev_out) {
     cfg.attrs = at;
     cfg.numAttrs = 1;
     int n = 0;
-    if (cudaOccupancyMaxActiveClusters(&n, shiftmm_kernel<1, false, true>, &cfg) != cudaSuccess)
+    if (cudaOccupancyMaxActiveClusters(&n, shiftmm_kernel<1, false, true, false>, &cfg) !=
+        cudaSuccess)
       cudaGetLastError();  // an unanswered query leaves no error behind
     else if (n > 0 && n < pairs)
       pairs = n;
@@ -1320,6 +1413,9 @@ struct GemmJob {
   int partial;  // weight gradient: int32 sums into ws (the caller's), no dequantizing pass
   float* colmax;  // per-column max |output| [N], formed by the epilogue, or null
   const int* seg;  // group order of the inner index (device table), or null
+  // operands stored MN-major: a as [K, lda] with M contiguous, b as [K, ldb] with N
+  // contiguous (the weight gradient on the codes' own layout); else K-major
+  int a_mn, b_mn;
 };
 
 static const char* job_name(int which) {
@@ -1361,7 +1457,8 @@ static int check_job(const GemmJob& j, int bits, int G, int32_t* dev_status, cud
     return err == cudaSuccess ? SQ_OK : cuda_fail(err, "cudaMemset2DAsync");
   }
   if (j.a == nullptr || j.b == nullptr) return fail(SQ_EINVAL, "%s: codes are NULL", nm);
-  if (j.lda < j.K || j.ldb < j.K) return fail(SQ_EINVAL, "%s: operand ld smaller than K", nm);
+  if (j.lda < (j.a_mn ? j.M : j.K) || j.ldb < (j.b_mn ? j.N : j.K))
+    return fail(SQ_EINVAL, "%s: operand ld smaller than its row", nm);
   const int eb = code_bytes(code_type(bits, G));
   if (!aligned16(j.a) || !aligned16(j.b) || (j.lda * eb) % 16 != 0 || (j.ldb * eb) % 16 != 0)
     return fail(SQ_EALIGN, "%s: operand pointers must be 16-byte aligned and ld * %d bytes a "
@@ -1453,9 +1550,13 @@ static int prepare_job(const GemmJob& j, const Plan* pl, int bits, int G, int32_
                        bool pair, GemmBatch* bt, int g) {
   int st;
   const int eb = pl->elem_bytes;
-  if ((st = make_operand_map(&bt->a[g], j.a, j.M, j.K, j.lda, eb, kBM)) != SQ_OK) return st;
-  if ((st = make_operand_map(&bt->b[g], j.b, j.N, j.K, j.ldb, eb, pair ? kBN / 2 : kBN)) != SQ_OK)
-    return st;
+  st = j.a_mn ? make_operand_map_mn(&bt->a[g], j.a, j.M, j.K, j.lda, eb)
+              : make_operand_map(&bt->a[g], j.a, j.M, j.K, j.lda, eb, kBM);
+  if (st != SQ_OK) return st;
+  st = j.b_mn ? make_operand_map_mn(&bt->b[g], j.b, j.N, j.K, j.ldb, eb)
+              : make_operand_map(&bt->b[g], j.b, j.N, j.K, j.ldb, eb, pair ? kBN / 2 : kBN);
+  if (st != SQ_OK) return st;
+  bt->mn[g] = (j.a_mn ? 1 : 0) | (j.b_mn ? 2 : 0);
   GemmParams& p = bt->p[g];
   p.M = static_cast<int>(j.M);
   p.N = static_cast<int>(j.N);
@@ -1497,9 +1598,9 @@ static int prepare_job(const GemmJob& j, const Plan* pl, int bits, int G, int32_
   return st;
 }
 
-template <int kF8, bool kMulti, bool kPair>
+template <int kF8, bool kMulti, bool kPair, bool kMn>
 static int launch_kernel(const GemmBatch& bt, int grid, int dev, cudaStream_t s) {
-  const int st = configure_kernel<kF8, kMulti, kPair>(dev);
+  const int st = configure_kernel<kF8, kMulti, kPair, kMn>(dev);
   if (st != SQ_OK) return st;
   cudaError_t err;
   if constexpr (kPair) {
@@ -1515,23 +1616,23 @@ static int launch_kernel(const GemmBatch& bt, int grid, int dev, cudaStream_t s)
     cfg.stream = s;
     cfg.attrs = at;
     cfg.numAttrs = 1;
-    err = cudaLaunchKernelEx(&cfg, shiftmm_kernel<kF8, kMulti, true>, bt);
+    err = cudaLaunchKernelEx(&cfg, shiftmm_kernel<kF8, kMulti, true, kMn>, bt);
     if (err == cudaSuccess) err = cudaGetLastError();
   } else {
-    shiftmm_kernel<kF8, kMulti, false><<<grid, kThreads, Smem<false>::bytes, s>>>(bt);
+    shiftmm_kernel<kF8, kMulti, false, kMn><<<grid, kThreads, Smem<false>::bytes, s>>>(bt);
     err = cudaGetLastError();
   }
   return err == cudaSuccess ? SQ_OK : cuda_fail(err, "shiftmm_kernel launch");
 }
 
-template <int kF8>
+template <int kF8, bool kMn>
 static int launch_variant(const GemmBatch& bt, int grid, int dev, cudaStream_t s, bool multi,
                           bool pair) {
   if (pair)
-    return multi ? launch_kernel<kF8, true, true>(bt, grid, dev, s)
-                 : launch_kernel<kF8, false, true>(bt, grid, dev, s);
-  return multi ? launch_kernel<kF8, true, false>(bt, grid, dev, s)
-               : launch_kernel<kF8, false, false>(bt, grid, dev, s);
+    return multi ? launch_kernel<kF8, true, true, kMn>(bt, grid, dev, s)
+                 : launch_kernel<kF8, false, true, kMn>(bt, grid, dev, s);
+  return multi ? launch_kernel<kF8, true, false, kMn>(bt, grid, dev, s)
+               : launch_kernel<kF8, false, false, kMn>(bt, grid, dev, s);
 }
 
 // Checks, plans and launches up to kMaxBatch GEMMs (all with the same bits / n_groups) as
@@ -1595,6 +1696,7 @@ static int run_jobs(GemmJob* jobs, int njobs, int bits, int G, int32_t* dev_stat
         const uint8_t* te = bt.k_exp[a]; bt.k_exp[a] = bt.k_exp[b]; bt.k_exp[b] = te;
         const int* ts = bt.seg[a]; bt.seg[a] = bt.seg[b]; bt.seg[b] = ts;
         const int tr = bt.raw_prod[a]; bt.raw_prod[a] = bt.raw_prod[b]; bt.raw_prod[b] = tr;
+        const int tm = bt.mn[a]; bt.mn[a] = bt.mn[b]; bt.mn[b] = tm;
       }
   int units = 0;
   bool multi = false;
@@ -1651,8 +1753,14 @@ static int run_jobs(GemmJob* jobs, int njobs, int bits, int G, int32_t* dev_stat
     const long long from = static_cast<long long>(units) - static_cast<long long>(depth) * ngroups;
     bt.lazy_from = from > 0 ? static_cast<int>(from) : 0;
   }
-  st = plans[0].elem_bytes == 1 ? launch_variant<1>(bt, grid, dev, s, multi, pair)
-                                : launch_variant<0>(bt, grid, dev, s, multi, pair);
+  bool mn = false;
+  for (int g = 0; g < nlive; ++g) mn |= bt.mn[g] != 0;
+  if (plans[0].elem_bytes == 1)
+    st = mn ? launch_variant<1, true>(bt, grid, dev, s, multi, pair)
+            : launch_variant<1, false>(bt, grid, dev, s, multi, pair);
+  else
+    st = mn ? launch_variant<0, true>(bt, grid, dev, s, multi, pair)
+            : launch_variant<0, false>(bt, grid, dev, s, multi, pair);
   if (st != SQ_OK) return st;
   for (int g = 0; g < nlive; ++g) {
     if (!bt.p[g].ws || partial) continue;
@@ -1685,9 +1793,14 @@ static void layer_jobs(const sq_layer_gemms* a, GemmJob jobs[3], int mask) {
                     a->wf_scale, nullptr, nullptr, a->y, a->ld_y, a->acc_y, a->ld_acc_y, nullptr, 0};
   jobs[1] = GemmJob{1, a->g_codes, a->ld_g, a->wd_codes, a->ld_wd, a->M, a->K, a->N, a->g_scale,
                     a->wd_scale, nullptr, nullptr, a->dx, a->ld_dx, a->acc_dx, a->ld_acc_dx, nullptr, 0};
-  jobs[2] = GemmJob{2, a->xt_codes, a->ld_xt, a->gt_codes, a->ld_gt, a->K, a->N, a->M, a->x_scale,
-                    a->g_scale, a->x_exp, a->g_exp, a->dw, a->ld_dw, a->acc_dw, a->ld_acc_dw,
-                    nullptr, 0};
+  // without a transposed copy the weight gradient reads X's (dY's) codes MN-major
+  const bool x_mn = a->xt_codes == nullptr, g_mn = a->gt_codes == nullptr;
+  jobs[2] = GemmJob{2, x_mn ? a->x_codes : a->xt_codes, x_mn ? a->ld_x : a->ld_xt,
+                    g_mn ? a->g_codes : a->gt_codes, g_mn ? a->ld_g : a->ld_gt, a->K, a->N, a->M,
+                    a->x_scale, a->g_scale, a->x_exp, a->g_exp, a->dw, a->ld_dw, a->acc_dw,
+                    a->ld_acc_dw, nullptr, 0};
+  jobs[2].a_mn = x_mn;
+  jobs[2].b_mn = g_mn;
   jobs[0].k_exp = a->x_exp;  // the forward GEMM's inner channels are X's
   jobs[1].k_exp = a->g_exp;  // loss propagation's are dY's
   jobs[0].colmax = a->y_range;
@@ -1946,6 +2059,11 @@ extern "C" sq_status shiftquant_gemm_layer(const sq_layer_gemms* args, void* wor
     return fail(SQ_EINVAL, "gemm_layer: bits must be in [2, 8] and n_groups in [1, 8]");
   if (args->gemm_mask < 0 || args->gemm_mask > 7 || args->max_ctas < 0)
     return fail(SQ_EINVAL, "gemm_layer: gemm_mask must be in [0, 7] and max_ctas >= 0");
+  const bool wgrad = args->gemm_mask == 0 || (args->gemm_mask & 4);
+  if (wgrad && ((args->xt_codes == nullptr && args->x_seg != nullptr) ||
+                (args->gt_codes == nullptr && args->g_seg != nullptr)))
+    return fail(SQ_EINVAL, "gemm_layer: a group-ordered operand needs its transposed copy "
+                "(xt_codes / gt_codes) for the weight gradient");
   GemmJob jobs[3];
   layer_jobs(args, jobs, args->gemm_mask);
   const int sms = device_sms(nullptr);
@@ -2038,6 +2156,26 @@ extern "C" int shiftquant_gemm_layer_kernel_launches(int64_t M, int64_t K, int64
   int launches = 1;
   for (int g = 0; g < n; ++g) launches += plans[g].splits > 1;
   return launches;
+}
+
+// Whether the weight gradient of a layer launch should read X's and dY's codes in place
+// (MN-major operands) rather than transposed copies.  Measured on GB300: an MMA with an
+// MN-major operand (either or both) runs 8% (E4M3) to 16-20% (BF16) slower than the K-major
+// form once the tensor core sets the pace -- pair tiles, a full wave of unsplit units with
+// long K loops (16384 x 4096 x 11008: 729 -> 924 us; 4096^3: 95 -> 113 us) -- and within
+// 2-4% where the launch is bound by split-K reductions or epilogues (12608 x 3072 x 768,
+// 12544 x 2304 x 256), where dropping the copies' quantizer writes wins.
+extern "C" int shiftquant_gemm_layer_wgrad_in_place(int64_t M, int64_t K, int64_t N, int bits,
+                                                    int n_groups) {
+  const int pair = shiftquant_gemm_layer_cta_pairs(M, K, N, bits, n_groups, 0);
+  if (pair < 0) return -1;
+  if (pair == 0) return 1;
+  const int pairs = device_pairs(nullptr);
+  Plan pl;
+  if (make_plan(2, K, N, M, bits, n_groups, pairs, 0, true, &pl) != SQ_OK) return -1;
+  const int64_t units = static_cast<int64_t>(pl.m_tiles) * pl.n_tiles * pl.splits;
+  const bool mma_bound = pl.splits == 1 && 2 * units >= pairs && pl.kb_per_split >= 64;
+  return mma_bound ? 0 : 1;
 }
 
 extern "C" int shiftquant_gemm_layer_cta_pairs(int64_t M, int64_t K, int64_t N, int bits,

@@ -21,8 +21,8 @@ static int check_step(const sq_layer_step* L) {
   if (L->M < 0 || L->K < 0 || L->N < 0) return fail(SQ_EINVAL, "layer_step: negative size");
   if (L->dev_status == nullptr) return fail(SQ_EINVAL, "layer_step: dev_status is required");
   if (L->M == 0 || L->K == 0 || L->N == 0) return SQ_OK;
-  const void* need[] = {L->x, L->w, L->dy, L->x_codes, L->xt_codes, L->x_range, L->x_tau0,
-                        L->x_scale, L->x_exp, L->g_codes, L->gt_codes, L->g_range, L->g_tau0,
+  const void* need[] = {L->x, L->w, L->dy, L->x_codes, L->x_range, L->x_tau0,
+                        L->x_scale, L->x_exp, L->g_codes, L->g_range, L->g_tau0,
                         L->g_scale, L->g_exp, L->wf_codes, L->wf_range, L->wf_scale,
                         L->wd_codes, L->wd_range, L->wd_scale, L->y, L->dx, L->dw};
   for (const void* p : need)
@@ -35,7 +35,8 @@ static int run_step(const sq_layer_step* L, uint64_t seed, void* s) {
   const int64_t M = L->M, K = L->K, N = L->N;
   const int b = L->bits, G = L->n_groups;
   int st;
-  // activation: range pass + grouping, then codes and the transposed copy (RN)
+  // activation: range pass + grouping, then codes and (if asked for) the transposed copy
+  // (RN); without the copy the weight gradient reads the codes MN-major
   if ((st = shiftquant_calibrate(L->x, M, K, K, SQ_GRAN_SHIFT, G, L->x_range, L->x_tau0,
                                  L->x_exp, L->dev_status, s)) != SQ_OK)
     return st;

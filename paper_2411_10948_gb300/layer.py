@@ -109,7 +109,16 @@ class QuantLinear:
     """Buffers and calls of one quantized linear layer: X [M, K], W [K, N], dY [M, N]."""
 
     def __init__(self, M, K, N_, bits, n_groups, device="cuda", with_acc=False,
-                 use_workspace=True, with_inputs=False, grouped=False):
+                 use_workspace=True, with_inputs=False, grouped=False, transposed=True):
+        """transposed=False: X and dY keep no transposed code copies; the weight gradient
+        reads their codes in place (MN-major operands of the layer launch).  None: the
+        library's advice for this shape (shiftquant_gemm_layer_wgrad_in_place).  A grouped
+        layer needs the copies (its forward operands are channel-permuted)."""
+        if grouped and transposed is False:
+            raise ValueError("a group-ordered layer needs the transposed code copies")
+        if transposed is None:
+            transposed = grouped or N.shiftquant_gemm_layer_wgrad_in_place(
+                M, K, N_, bits, n_groups) != 1
         self.M, self.K, self.N, self.bits, self.G = M, K, N_, bits, n_groups
         self.grouped = grouped
         dev = torch.device(device)
@@ -120,8 +129,8 @@ class QuantLinear:
                            torch.zeros((K, N_), dtype=torch.float32, device=dev),
                            torch.zeros((M, N_), dtype=torch.float32, device=dev))
         self.status = torch.zeros(1, dtype=torch.int32, device=dev)
-        self.x = ShiftTensor.alloc(M, K, bits, n_groups, dev)
-        self.g = ShiftTensor.alloc(M, N_, bits, n_groups, dev)
+        self.x = ShiftTensor.alloc(M, K, bits, n_groups, dev, transposed)
+        self.g = ShiftTensor.alloc(M, N_, bits, n_groups, dev, transposed)
         # grouped: the forward and loss-propagation operands hold their inner index in group
         # order (Sec. 3.2's per-group products as one launch) over the padded width
         self.x_pos = self.x_seg = self.g_pos = self.g_seg = None
@@ -214,6 +223,10 @@ class QuantLinear:
                                 self.status, stream)
 
     def wgrad(self, stream=None):
+        if self.x.codes_t is None or self.g.codes_t is None:
+            # codes in place: the layer launch with the weight gradient alone
+            self.gemms(stream, gemm_mask=4)
+            return
         N.shiftquant_gemm_wgrad(self.x.codes_t, self.x.scale, self.x.exp, self.g.codes_t,
                                 self.g.scale, self.g.exp, self.K, self.N, self.M, self.bits,
                                 self.G, self.dw, self.acc["wgrad"] if self.acc else None,
@@ -334,7 +347,8 @@ class LinearChain:
         dev = torch.device(device)
         self.M, self.dims, self.bits, self.G = M, list(dims), bits, n_groups
         self.fused = fused_ranges
-        self.layers = [QuantLinear(M, dims[i], dims[i + 1], bits, n_groups, dev)
+        self.layers = [QuantLinear(M, dims[i], dims[i + 1], bits, n_groups, dev,
+                                   transposed=None)
                        for i in range(len(dims) - 1)]
         self.y_range = [torch.zeros(d, dtype=torch.float32, device=dev) for d in dims[1:]]
         self.dx_range = [torch.zeros(d, dtype=torch.float32, device=dev) for d in dims[:-1]]
@@ -423,7 +437,8 @@ class HostSteps:
         self.copy_out = torch.cuda.Stream(device=dev)
         self.slots = []
         for _ in range(slots):
-            layers = [QuantLinear(M, K, N_, bits, n_groups, dev, with_inputs=True)
+            layers = [QuantLinear(M, K, N_, bits, n_groups, dev, with_inputs=True,
+                                  transposed=None)
                       for (M, K, N_) in self.shapes]
             # per layer: inputs in, step done, outputs out (recorded once here so that the
             # CUDA events exist before the library records them)

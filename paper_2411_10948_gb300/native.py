@@ -39,6 +39,7 @@ EXPORTS = (
     "shiftquant_gemm_layer", "shiftquant_gemm_layer_workspace_bytes",
     "shiftquant_gemm_layer_workspace_bytes_grouped",
     "shiftquant_gemm_layer_kernel_launches", "shiftquant_gemm_layer_cta_pairs",
+    "shiftquant_gemm_layer_wgrad_in_place",
     "shiftquant_layer_step", "shiftquant_layer_step_host", "shiftquant_layer_step_host_split",
     "shiftquant_selftest_wait_timeout",
     "shiftquant_l1bn_state_bytes", "shiftquant_l1bn_forward", "shiftquant_l1bn_backward",
@@ -165,6 +166,8 @@ def load(path: str | None = None) -> ctypes.CDLL:
     lib.shiftquant_gemm_layer_kernel_launches.restype = i32
     lib.shiftquant_gemm_layer_cta_pairs.argtypes = [i64, i64, i64, i32, i32, i32]
     lib.shiftquant_gemm_layer_cta_pairs.restype = i32
+    lib.shiftquant_gemm_layer_wgrad_in_place.argtypes = [i64, i64, i64, i32, i32]
+    lib.shiftquant_gemm_layer_wgrad_in_place.restype = i32
     lib.shiftquant_gemm_workspace_bytes.argtypes = [i32, i64, i64, i64, i32, i32]
     lib.shiftquant_gemm_workspace_bytes.restype = sz
     lib.shiftquant_layer_step.argtypes = [ctypes.POINTER(SqLayerStep), u64, vp]
@@ -418,6 +421,13 @@ def shiftquant_gemm_layer_cta_pairs(M: int, K: int, N: int, bits: int, n_groups:
     return int(load().shiftquant_gemm_layer_cta_pairs(M, K, N, bits, n_groups, gemm_mask))
 
 
+def shiftquant_gemm_layer_wgrad_in_place(M: int, K: int, N: int, bits: int,
+                                         n_groups: int) -> int:
+    """1: the layer launch's weight gradient reads X's and dY's codes in place as fast as
+    transposed copies (skip the copies); 0: keep the copies; -1: invalid or no device."""
+    return int(load().shiftquant_gemm_layer_wgrad_in_place(M, K, N, bits, n_groups))
+
+
 def layer_step_args(M, K, N, bits, n_groups, x, w, dy, x_codes, xt_codes, x_range, x_tau0,
                     x_scale, x_exp, g_codes, gt_codes, g_range, g_tau0, g_scale, g_exp,
                     wf_codes, wf_range, wf_scale, wd_codes, wd_range, wd_scale, y, dx, dw,
@@ -428,9 +438,11 @@ def layer_step_args(M, K, N, bits, n_groups, x, w, dy, x_codes, xt_codes, x_rang
         assert tuple(t.shape) == shape and t.is_contiguous(), "dense fp32 matrices expected"
     return SqLayerStep(
         M=M, K=K, N=N, bits=bits, n_groups=n_groups, x=_addr(x), w=_addr(w), dy=_addr(dy),
-        x_codes=_addr(x_codes), ld_x=_ld(x_codes), xt_codes=_addr(xt_codes), ld_xt=_ld(xt_codes),
+        x_codes=_addr(x_codes), ld_x=_ld(x_codes), xt_codes=_addr(xt_codes),
+        ld_xt=_ld_opt(xt_codes),
         x_range=_addr(x_range), x_tau0=_addr(x_tau0), x_scale=_addr(x_scale), x_exp=_addr(x_exp),
-        g_codes=_addr(g_codes), ld_g=_ld(g_codes), gt_codes=_addr(gt_codes), ld_gt=_ld(gt_codes),
+        g_codes=_addr(g_codes), ld_g=_ld(g_codes), gt_codes=_addr(gt_codes),
+        ld_gt=_ld_opt(gt_codes),
         g_range=_addr(g_range), g_tau0=_addr(g_tau0), g_scale=_addr(g_scale), g_exp=_addr(g_exp),
         wf_codes=_addr(wf_codes), ld_wf=_ld(wf_codes), wf_range=_addr(wf_range),
         wf_scale=_addr(wf_scale), wd_codes=_addr(wd_codes), ld_wd=_ld(wd_codes),

@@ -256,3 +256,18 @@ def test_layer_step_validates_before_anything_runs(lib):
                                                 None, 0, None, None, None, None, None, fake,
                                                 fake) == native.SQ_EINVAL
     assert "inputs_in" in lib.shiftquant_last_error().decode()
+
+
+def test_layer_launch_refuses_in_place_weight_gradient_on_group_ordered_codes(lib):
+    # without a transposed copy the weight gradient reads the codes in place, which a
+    # group-ordered operand (channels permuted) cannot serve: refused on the host
+    from paper_2411_10948_gb300.native import SqLayerGemms
+    fake = 4096
+    a = SqLayerGemms(M=64, K=64, N=64, bits=8, n_groups=4, x_codes=fake, ld_x=64,
+                     xt_codes=None, g_codes=fake, ld_g=64, gt_codes=fake, ld_gt=64,
+                     x_seg=fake)
+    st = ctypes.c_void_p(fake)
+    assert lib.shiftquant_gemm_layer(ctypes.byref(a), None, 0, st, None) == native.SQ_EINVAL
+    assert "transposed copy" in lib.shiftquant_last_error().decode()
+    a.x_seg, a.g_seg, a.xt_codes, a.gt_codes = None, fake, fake, None
+    assert lib.shiftquant_gemm_layer(ctypes.byref(a), None, 0, st, None) == native.SQ_EINVAL

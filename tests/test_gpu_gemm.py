@@ -32,10 +32,12 @@ def layer_inputs(rng, M, K, Nn):
     return x, w, dy
 
 
-def run_and_compare(x, w, dy, bits, G, seed=11, use_workspace=True, fused=False):
+def run_and_compare(x, w, dy, bits, G, seed=11, use_workspace=True, fused=False,
+                    transposed=True):
     M, K = x.shape
     Nn = w.shape[1]
-    lay = L.QuantLinear(M, K, Nn, bits, G, "cuda", with_acc=True, use_workspace=use_workspace)
+    lay = L.QuantLinear(M, K, Nn, bits, G, "cuda", with_acc=True, use_workspace=use_workspace,
+                        transposed=transposed)
     if fused:
         lay.quantize_activation(to_gpu(x))
         lay.quantize_gradient(to_gpu(dy), seed)
@@ -76,6 +78,47 @@ def test_pair_tiles_with_ragged_tails_match_oracle(M, K, Nn, bits):
     assert N.shiftquant_gemm_layer_cta_pairs(M, K, Nn, bits, 4) == 1
     rng = np.random.default_rng(M + K + Nn + bits)
     run_and_compare(*layer_inputs(rng, M, K, Nn), bits, 4, fused=True)
+
+
+@pytest.mark.parametrize("M,K,Nn", [(1, 1, 1), (5, 3, 7), (130, 70, 300), (300, 1000, 513),
+                                    (4096, 64, 96), (2000, 700, 256), (1900, 1800, 1700)])
+@pytest.mark.parametrize("bits", [6, 8, 4])
+def test_weight_gradient_reads_the_codes_in_place(M, K, Nn, bits):
+    # no transposed copies: the weight gradient of the layer launch reads X's [M, K] and dY's
+    # [M, N] codes as MN-major operands (the tensor core transposes them from shared memory);
+    # ragged tails in both the output (K, N) and the inner (token) index, single tiles and
+    # CTA pairs (1900 x 1800 x 1700)
+    rng = np.random.default_rng(M + 3 * K + Nn + bits)
+    lay = run_and_compare(*layer_inputs(rng, M, K, Nn), bits, 4, fused=True, transposed=False)
+    assert lay.x.codes_t is None and lay.g.codes_t is None
+
+
+def test_layout_advice_keeps_copies_only_where_the_tensor_core_sets_the_pace():
+    # shiftquant_gemm_layer_wgrad_in_place: in place where the launch is bound by split-K
+    # reductions or epilogues, transposed copies for full waves of long pair-tile units
+    adv = N.shiftquant_gemm_layer_wgrad_in_place
+    assert adv(12544, 2304, 256, 4, 4) == 1        # single tiles
+    assert adv(12608, 768, 3072, 6, 4) == 1        # split-K weight gradient
+    assert adv(16384, 4096, 11008, 6, 4) == 0      # 688 unsplit units of 256 K blocks
+    assert adv(4096, 4096, 4096, 6, 4) == 0
+    assert adv(16, 16, 16, 9, 4) == -1
+    lay = L.QuantLinear(12544, 2304, 256, 4, 4, "cuda", transposed=None)
+    assert lay.x.codes_t is None and lay.g.codes_t is None
+    lay = L.QuantLinear(4096, 4096, 4096, 6, 4, "cuda", transposed=None)
+    assert lay.x.codes_t is not None and lay.g.codes_t is not None
+
+
+@pytest.mark.parametrize("bits", [6, 4])
+def test_weight_gradient_in_place_equals_the_transposed_copies(bits):
+    # the same launch on the codes in place and on transposed copies: equal dW bit for bit,
+    # through the separate-GEMM step as well (its weight gradient becomes a layer launch)
+    rng = np.random.default_rng(60 + bits)
+    x, w, dy = layer_inputs(rng, 3000, 640, 384)
+    a = run_and_compare(x, w, dy, bits, 4, fused=True, transposed=False)
+    b = run_and_compare(x, w, dy, bits, 4, fused=True, transposed=True)
+    c = run_and_compare(x, w, dy, bits, 4, fused=False, transposed=False)
+    for t in (b, c):
+        np.testing.assert_array_equal(a.dw.cpu().numpy(), t.dw.cpu().numpy())
 
 
 def test_tile_mode_query():
@@ -331,12 +374,14 @@ def test_c_host_steps_equal_device_steps():
                 np.testing.assert_array_equal(got.numpy(), want.cpu().numpy())
 
 
-def test_c_layer_step_matches_oracle():
-    # shiftquant_layer_step on device inputs: the whole step against the oracle's layer
-    rng = np.random.default_rng(77)
-    M, K, Nn, bits, G, seed = 1000, 320, 288, 4, 4, 0xABC
+@pytest.mark.parametrize("bits,transposed", [(4, True), (4, False), (6, False)])
+def test_c_layer_step_matches_oracle(bits, transposed):
+    # shiftquant_layer_step on device inputs: the whole step against the oracle's layer; with
+    # transposed=False the step writes no transposed copies and dW reads the codes in place
+    rng = np.random.default_rng(77 + bits)
+    M, K, Nn, G, seed = 1000, 320, 288, 4, 0xABC
     x, w, dy = layer_inputs(rng, M, K, Nn)
-    lay = L.QuantLinear(M, K, Nn, bits, G, "cuda")
+    lay = L.QuantLinear(M, K, Nn, bits, G, "cuda", transposed=transposed)
     N.shiftquant_layer_step(lay.step_args(to_gpu(x), to_gpu(w), to_gpu(dy)), seed)
     torch.cuda.synchronize()
     assert lay.status.item() == 0
