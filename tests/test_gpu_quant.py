@@ -171,7 +171,7 @@ def both_roles(w_np, bits, G, ex, eg, ld=None):
 
 
 @pytest.mark.parametrize("shape", [(1, 1), (70, 33), (300, 257), (2304, 256), (129, 1031),
-                                   (64, 600), (1000, 96)])
+                                   (64, 600), (1000, 96), (700, 4100), (3, 2049)])
 @pytest.mark.parametrize("bits,G", [(4, 4), (6, 4), (8, 4), (4, 7)])
 @pytest.mark.parametrize("fold", [True, False])
 def test_weight_both_roles_from_one_pass(shape, bits, G, fold):
@@ -200,14 +200,15 @@ def test_weight_both_roles_from_one_pass(shape, bits, G, fold):
 
 
 @pytest.mark.parametrize("bad", [np.nan, np.inf])
-def test_weight_both_roles_nonfinite(bad):
-    w = np.full((40, 300), 0.01, np.float32)
-    w[13, 200] = bad
+@pytest.mark.parametrize("C,col", [(300, 200), (1300, 1200)])   # narrow and wide range passes
+def test_weight_both_roles_nonfinite(bad, C, col):
+    w = np.full((40, C), 0.01, np.float32)
+    w[13, col] = bad
     f, d, st = both_roles(w, 4, 4, None, None)
     assert st & N.SQ_DEV_NONFINITE
     fr, dr = f.range.cpu().numpy(), d.range.cpu().numpy()
-    assert not np.isfinite(fr[200]) and not np.isfinite(dr[13])
-    assert np.isfinite(np.delete(fr, 200)).all() and np.isfinite(np.delete(dr, 13)).all()
+    assert not np.isfinite(fr[col]) and not np.isfinite(dr[13])
+    assert np.isfinite(np.delete(fr, col)).all() and np.isfinite(np.delete(dr, 13)).all()
 
 
 def test_weight_both_roles_empty():
