@@ -434,11 +434,46 @@ __device__ __forceinline__ int chunk_slot(int col, int chunk) {
   return col * 8 + (chunk ^ ((col >> 2) & 7));
 }
 
+// The thread's eight input rows of the block's 64 x 128 tile (four columns each), all
+// loads in flight together; outside the tensor the values are 0.  FULL: the tile lies
+// inside the tensor and its rows are 16-byte aligned.
+template <bool FULL>
+__device__ __forceinline__ void load_quant_tile(const QuantArgs& a, float4 (&xin)[kQRowsPerWarp]) {
+  const int tid = threadIdx.x;
+  const int lane = tid & 31;
+  const int wq = tid >> 5;
+  const int64_t r0 = static_cast<int64_t>(blockIdx.y) * kQR;
+  const int64_t cb = static_cast<int64_t>(blockIdx.x) * kQC + lane * 4;
+#pragma unroll
+  for (int i = 0; i < kQRowsPerWarp; ++i) {
+    const int64_t r = r0 + wq * 8 + i;
+    const float* row = a.x + r * a.ld;
+    if (FULL) {
+      xin[i] = ld_stream_v4(row + cb);
+    } else {
+      xin[i] = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+      if (r < a.R) {
+        if (a.vec_in && cb + 3 < a.C) {
+          xin[i] = __ldg(reinterpret_cast<const float4*>(row + cb));
+        } else {
+          if (cb + 0 < a.C) xin[i].x = __ldg(row + cb + 0);
+          if (cb + 1 < a.C) xin[i].y = __ldg(row + cb + 1);
+          if (cb + 2 < a.C) xin[i].z = __ldg(row + cb + 2);
+          if (cb + 3 < a.C) xin[i].w = __ldg(row + cb + 3);
+        }
+      }
+    }
+  }
+}
+
 // One 64 x 128 tile.  GRAN: SQ_GRAN_*; MODE: SQ_ROUND_*; FOLD: weight codes carry the
 // ShiftMM shift 2^(G-1-fold[i]); FULL: the tile lies inside the tensor and every access
-// is vector-aligned, so no element needs a bounds check.
-template <typename CodeT, int GRAN, int MODE, bool FOLD, bool FULL>
-__device__ __forceinline__ void quantize_tile(const QuantArgs& a, uint8_t* tile_t) {
+// is vector-aligned, so no element needs a bounds check.  LOAD: the tile's loads are
+// issued here; otherwise `pre` holds the thread's eight rows, loaded by the caller
+// (load_quant_tile) -- the weight kernel quantizes one load for both roles.
+template <typename CodeT, int GRAN, int MODE, bool FOLD, bool FULL, bool LOAD = true>
+__device__ __forceinline__ void quantize_tile(const QuantArgs& a, uint8_t* tile_t,
+                                              const float4* pre = nullptr) {
   constexpr int kChunkBytes = 8 * sizeof(CodeT);  // eight codes of one column
   constexpr int kWords = kChunkBytes / 4;         // 32-bit words per packed column chunk
   constexpr int kPerWord = 4 / sizeof(CodeT);
@@ -454,6 +489,10 @@ __device__ __forceinline__ void quantize_tile(const QuantArgs& a, uint8_t* tile_
   float4 xin[kQRowsPerWarp];
 #pragma unroll
   for (int i = 0; i < kQRowsPerWarp; ++i) {
+    if (!LOAD) {
+      xin[i] = pre[i];
+      continue;
+    }
     const int64_t r = r0 + wq * 8 + i;
     const float* row = a.x + r * a.ld;
     if (FULL) {
@@ -747,22 +786,30 @@ static void launch_quantize(const QuantArgs& a, dim3 grid, cudaStream_t s) {
 // Both roles of a weight from one pass over it (Sec. 5.1): the forward GEMM's
 // per-out-channel codes (gran PER_COL, written transposed, the fold indexed by row) and loss
 // propagation's per-in-channel codes (gran PER_ROW, natural layout, the fold indexed by
-// column).  The second role re-reads the block's tile, which the first has just brought
-// into L2, so HBM sees one read of the weight.
+// column), both from the one load of the block's tile held in registers.  Re-reading the
+// tile for the second role (from L2) put a second load latency in every block: 87 us for
+// large_linear's [4096, 11008] weight against 76 us now.  The tile held across both roles
+// needs about 98 registers; three blocks per SM (80, a few bytes spilled) measured 76 us, two (98) 93 us,
+// four (64, spilling) 73 us on the wide weights but slower on small ones.
 template <typename CodeT, bool FF, bool FD>
-__global__ void __launch_bounds__(256) quantize_weight_kernel(const QuantArgs af, const QuantArgs ad) {
+__global__ void __launch_bounds__(256, 3) quantize_weight_kernel(const QuantArgs af, const QuantArgs ad) {
   __shared__ __align__(16) uint8_t tile_t[kQC * 8 * 8 * sizeof(CodeT)];
   griddep_wait();
   const bool inside = (static_cast<int64_t>(blockIdx.y) + 1) * kQR <= af.R &&
                       (static_cast<int64_t>(blockIdx.x) + 1) * kQC <= af.C && af.vec_in;
+  float4 xin[kQRowsPerWarp];   // both roles read the same tensor: af and ad share x, R, C, ld
+  if (inside)
+    load_quant_tile<true>(af, xin);
+  else
+    load_quant_tile<false>(af, xin);
   if (inside && af.vec_t)
-    quantize_tile<CodeT, SQ_GRAN_PER_COL, SQ_ROUND_NEAREST_EVEN, FF, true>(af, tile_t);
+    quantize_tile<CodeT, SQ_GRAN_PER_COL, SQ_ROUND_NEAREST_EVEN, FF, true, false>(af, tile_t, xin);
   else
-    quantize_tile<CodeT, SQ_GRAN_PER_COL, SQ_ROUND_NEAREST_EVEN, FF, false>(af, tile_t);
+    quantize_tile<CodeT, SQ_GRAN_PER_COL, SQ_ROUND_NEAREST_EVEN, FF, false, false>(af, tile_t, xin);
   if (inside && ad.vec_out)
-    quantize_tile<CodeT, SQ_GRAN_PER_ROW, SQ_ROUND_NEAREST_EVEN, FD, true>(ad, tile_t);
+    quantize_tile<CodeT, SQ_GRAN_PER_ROW, SQ_ROUND_NEAREST_EVEN, FD, true, false>(ad, tile_t, xin);
   else
-    quantize_tile<CodeT, SQ_GRAN_PER_ROW, SQ_ROUND_NEAREST_EVEN, FD, false>(ad, tile_t);
+    quantize_tile<CodeT, SQ_GRAN_PER_ROW, SQ_ROUND_NEAREST_EVEN, FD, false, false>(ad, tile_t, xin);
 }
 
 template <typename CodeT>
