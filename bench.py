@@ -735,9 +735,11 @@ def run_l1bn(args, dev):
         fm, bm = statistics.median(times["fwd"]), statistics.median(times["bwd"])
         fg = L1BN_FWD_BYTES * R * C / (fm * 1e-3) / 1e9
         bg = L1BN_BWD_BYTES * R * C / (bm * 1e-3) / 1e9
+        launches = {"fwd": N.shiftquant_l1bn_kernel_launches(C),
+                    "bwd": N.shiftquant_l1bn_kernel_launches(C, True)}
         out.append({"shape": name, "rows": R, "channels": C, "fwd_ms": fm, "bwd_ms": bm,
                     "fwd_gbs": fg, "bwd_gbs": bg, "fwd_frac": fg / peaks["hbm_gbs"],
-                    "bwd_frac": bg / peaks["hbm_gbs"], "launches": {"fwd": 7, "bwd": 6}})
+                    "bwd_frac": bg / peaks["hbm_gbs"], "launches": launches})
     return {"bits": 8, "n_groups": 4, "bytes_per_element": {"fwd": L1BN_FWD_BYTES,
                                                            "bwd": L1BN_BWD_BYTES},
             "peak": peaks["hbm_gbs"], "peak_source": f"{src} copy bandwidth",

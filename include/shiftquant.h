@@ -555,6 +555,14 @@ sq_status shiftquant_l1bn_backward(const float *dy, int64_t rows, int64_t channe
                                    float *dgamma, float *dbeta, int32_t *dev_status,
                                    void *stream);
 
+/* Kernels one shiftquant_l1bn_forward (backward = 0) or _backward (1) call launches on the
+ * current device: 1 for at most 1024 channels on a device that runs cooperative launches
+ * (the passes then run as phases of one launch, separated by bounded grid barriers, after
+ * one memset of the state's counter and range slots), else the chain of 9 (forward) or 7
+ * (backward) kernels; 0 for no channels, -1 for a negative count or no device.  Results do
+ * not depend on the form. */
+int shiftquant_l1bn_kernel_launches(int64_t channels, int backward);
+
 /* Packed sub-byte storage (Sec. 5.2: with N_G = 4 the grouping map takes exactly 2 bits).
  * The tensor cores read codes as E4M3 / BF16 (there is no integer MMA on sm_103a, and the
  * 4-bit float E2M1 lacks the integers 5 and 7), so the packed form is the storage of a

@@ -49,7 +49,7 @@ constexpr int kSpread = 8;
 enum { kScXTau, kScXScale, kScGTau, kScGScale, kNumScal };
 
 struct L1bnLayout {
-  size_t xq, gq, stats, chan, lut, exps, scal, total;
+  size_t xq, gq, stats, chan, lut, exps, scal, sync, total;
 };
 
 // the forward output of every code value per channel: lut[c][q + 127]
@@ -67,6 +67,9 @@ static L1bnLayout l1bn_layout(int64_t R, int64_t C) {
   L.lut = o;   o += up(kLutStride * static_cast<size_t>(C) * sizeof(float));
   L.exps = o;  o += up(2 * static_cast<size_t>(C));
   L.scal = o;  o += 256;
+  // the single-launch form's barrier counter (first 256 bytes) and the range pass's
+  // per-column maxima in kSpread slot rows, zeroed before each call
+  L.sync = o;  o += up(256 + kSpread * static_cast<size_t>(C) * sizeof(unsigned));
   L.total = o;
   return L;
 }
@@ -90,6 +93,7 @@ struct L1bnArgs {
   float* dgamma;
   float* dbeta;
   int vec_in, vec_out;  // 16-byte rows: four elements per load / store
+  unsigned* sync;       // single-launch form: barrier counter, then range slots [kSpread][C]
 };
 
 constexpr int kL1Threads = 256;
@@ -111,13 +115,23 @@ __device__ __forceinline__ long long rne_div(long long a, long long b) {
 __device__ __forceinline__ long long stat_sum(const long long* st, int k, int64_t C, int64_t c) {
   long long v = 0;
 #pragma unroll
-  for (int i = 0; i < kSpread; ++i) v += st[(static_cast<int64_t>(k) * kSpread + i) * C + c];
+  for (int i = 0; i < kSpread; ++i) v += __ldcg(st + (static_cast<int64_t>(k) * kSpread + i) * C + c);
   return v;
 }
 
 // the slot row of statistic k that block row y adds to
-__device__ __forceinline__ long long* stat_slot(long long* st, int k, int64_t C) {
-  return st + (static_cast<int64_t>(k) * kSpread + blockIdx.y % kSpread) * C;
+__device__ __forceinline__ long long* stat_slot(long long* st, int k, int64_t C, int64_t y) {
+  return st + (static_cast<int64_t>(k) * kSpread + y % kSpread) * C;
+}
+
+// A pass's block: its column tile x and row slab y of a gx x gy grid (the launch's own
+// grid, or the part of a cooperative launch's blocks that runs the pass).
+struct Blk {
+  int64_t x, y, gx, gy;
+};
+
+__device__ __forceinline__ Blk launch_blk() {
+  return Blk{blockIdx.x, blockIdx.y, gridDim.x, gridDim.y};
 }
 
 // The thread's place in a tile: its quad (four consecutive columns) and its first row.
@@ -128,13 +142,13 @@ struct TilePos {
   int64_t c;     // its first column
 };
 
-__device__ __forceinline__ TilePos tile_pos(int lg) {
+__device__ __forceinline__ TilePos tile_pos(int lg, const Blk& b) {
   TilePos t;
   t.tc = 4 << lg;
   t.rpp = kL1Threads >> lg;
   t.qc = threadIdx.x & ((1 << lg) - 1);
   t.ro = threadIdx.x >> lg;
-  t.c = static_cast<int64_t>(blockIdx.x) * t.tc + 4 * t.qc;
+  t.c = b.x * t.tc + 4 * t.qc;
   return t;
 }
 
@@ -149,13 +163,20 @@ __device__ __forceinline__ void load4(const float* p, int64_t c, int64_t C, bool
   }
 }
 
-// the four codes of a quad at p packed in one word, byte j = column c + j (zeros past C)
+// the four codes of a quad at p packed in one word, byte j = column c + j (zeros past C).
+// COH: codes written earlier in the same launch (the single-launch form): coherent loads
+// through L2, not the read-only path, which holds only data no part of the launch writes.
+template <bool COH = false>
 __device__ __forceinline__ uint32_t load_codes_w(const int8_t* p, int64_t c, int64_t C) {
-  if ((C & 3) == 0) return __ldg(reinterpret_cast<const unsigned int*>(p));
+  if ((C & 3) == 0)
+    return COH ? __ldcg(reinterpret_cast<const unsigned int*>(p)) : __ldg(reinterpret_cast<const unsigned int*>(p));
   uint32_t w = 0;
 #pragma unroll
   for (int j = 0; j < 4; ++j)
-    if (c + j < C) w |= static_cast<uint32_t>(static_cast<uint8_t>(p[j])) << (8 * j);
+    if (c + j < C) {
+      const int8_t v = COH ? __ldcg(p + j) : p[j];
+      w |= static_cast<uint32_t>(static_cast<uint8_t>(v)) << (8 * j);
+    }
   return w;
 }
 
@@ -190,10 +211,10 @@ struct RowWalk {
   int64_t r, S;
 };
 
-__device__ __forceinline__ RowWalk row_walk(const TilePos& t) {
+__device__ __forceinline__ RowWalk row_walk(const TilePos& t, const Blk& b) {
   RowWalk w;
-  w.r = static_cast<int64_t>(blockIdx.y) * t.rpp + t.ro;
-  w.S = static_cast<int64_t>(gridDim.y) * t.rpp;
+  w.r = b.y * t.rpp + t.ro;
+  w.S = b.gy * t.rpp;
   return w;
 }
 
@@ -207,7 +228,7 @@ struct RedSmem {
 // statistic k): acc[k][j] is this thread's sum over its rows for column t.c + j.
 template <int NS>
 __device__ __forceinline__ void red_end(const long long (&acc)[NS][4], long long* const (&dst)[NS],
-                                        const TilePos& t, int64_t C, RedSmem<NS>& sm) {
+                                        const TilePos& t, int64_t C, RedSmem<NS>& sm, const Blk& b) {
 #pragma unroll
   for (int k = 0; k < NS; ++k)
 #pragma unroll
@@ -221,7 +242,7 @@ __device__ __forceinline__ void red_end(const long long (&acc)[NS][4], long long
     if (tid < t.tc)
       for (int r = 0; r < t.rpp; ++r) tot[k] += sm.part[k][r * t.tc + tid];
   }
-  const int64_t c = static_cast<int64_t>(blockIdx.x) * t.tc + tid;
+  const int64_t c = b.x * t.tc + tid;
   if (tid < t.tc && c < C) {
 #pragma unroll
     for (int k = 0; k < NS; ++k)
@@ -231,24 +252,20 @@ __device__ __forceinline__ void red_end(const long long (&acc)[NS][4], long long
 }
 
 // Forward pass 1: x -> int8 ShiftQuant codes (round to nearest), sum of codes per channel.
-__global__ void __launch_bounds__(kL1Threads, 3) l1bn_fwd_quant_kernel(const L1bnArgs a, int lg) {
-  // launched behind the previous kernel (programmatic stream serialization): wait for it
-  // before reading anything it wrote, and let the next kernel start launching
-  griddep_wait();
-  griddep_launch_dependents();
-  __shared__ RedSmem<1> sm;
-  const TilePos t = tile_pos(lg);
-  const float tau = a.scal[kScXTau];
+// tau: tau_0; the exponent of column c is ex[c - ex0].
+__device__ __forceinline__ void fwd_quant_pass(const L1bnArgs& a, int lg, const Blk& b, float tau,
+                                               const uint8_t* ex, int64_t ex0, RedSmem<1>& sm) {
+  const TilePos t = tile_pos(lg, b);
   const float Qf = static_cast<float>(a.Q);
   const float invS = __fdiv_rn(Qf, tau);
   const bool zero = !(tau > 0.0f) || !isfinite(tau) || !isfinite(invS);
   int e[4];
 #pragma unroll
-  for (int j = 0; j < 4; ++j) e[j] = t.c + j < a.C ? a.xe[t.c + j] : 0;
+  for (int j = 0; j < 4; ++j) e[j] = t.c + j < a.C ? ex[t.c + j - ex0] : 0;
   long long acc[1][4] = {{0, 0, 0, 0}};
   constexpr int U = kL1PassesF32;
   if (t.c < a.C) {
-    RowWalk w = row_walk(t);
+    RowWalk w = row_walk(t, b);
     const float* px = a.in + w.r * a.ld_in + t.c;
     int8_t* pq = a.xq + w.r * a.C + t.c;
     const int64_t sx = w.S * a.ld_in, sq = w.S * a.C;
@@ -270,27 +287,33 @@ __global__ void __launch_bounds__(kL1Threads, 3) l1bn_fwd_quant_kernel(const L1b
       }
     }
   }
-  long long* const dst[1] = {stat_slot(a.st, kStS1, a.C)};
-  red_end<1>(acc, dst, t, a.C, sm);
-  if (blockIdx.x == 0 && blockIdx.y == 0 && threadIdx.x == 0)
-    a.scal[kScXScale] = zero ? 0.0f : __fdiv_rn(tau, Qf);
+  long long* const dst[1] = {stat_slot(a.st, kStS1, a.C, b.y)};
+  red_end<1>(acc, dst, t, a.C, sm, b);
+  if (b.x == 0 && b.y == 0 && threadIdx.x == 0) a.scal[kScXScale] = zero ? 0.0f : __fdiv_rn(tau, Qf);
+}
+
+__global__ void __launch_bounds__(kL1Threads, 3) l1bn_fwd_quant_kernel(const L1bnArgs a, int lg) {
+  // launched behind the previous kernel (programmatic stream serialization): wait for it
+  // before reading anything it wrote, and let the next kernel start launching
+  griddep_wait();
+  griddep_launch_dependents();
+  __shared__ RedSmem<1> sm;
+  fwd_quant_pass(a, lg, launch_blk(), a.scal[kScXTau], a.xe, 0, sm);
 }
 
 // Forward pass 2: over the codes, sum |q - m| and sum sign(q - m) per channel, with
-// m = round-half-even(sum q / R).
-__global__ void __launch_bounds__(kL1Threads, 3) l1bn_fwd_dev_kernel(const L1bnArgs a, int lg) {
-  griddep_wait();
-  griddep_launch_dependents();
-  __shared__ RedSmem<2> sm;
-  const TilePos t = tile_pos(lg);
+// m = round-half-even(sum q / R).  mean: shared scratch for the block's columns.
+template <bool COH>
+__device__ __forceinline__ void fwd_dev_pass(const L1bnArgs& a, int lg, const Blk& b, RedSmem<2>& sm,
+                                             int* mean) {
+  const TilePos t = tile_pos(lg, b);
   // the block's columns' means, from their sum slots, once per block
-  __shared__ int mean[kL1MaxCols];
   {
     long long* fold = &sm.part[0][0];   // free until the block's reduction at the end
-    const int64_t cb = static_cast<int64_t>(blockIdx.x) * t.tc;
+    const int64_t cb = b.x * t.tc;
     for (int i = threadIdx.x; i < kSpread * t.tc; i += kL1Threads) {
       const int slot = i / t.tc, col = i - slot * t.tc;
-      fold[i] = cb + col < a.C ? a.st[(static_cast<int64_t>(kStS1) * kSpread + slot) * a.C + cb + col] : 0;
+      fold[i] = cb + col < a.C ? __ldcg(a.st + (static_cast<int64_t>(kStS1) * kSpread + slot) * a.C + cb + col) : 0;
     }
     __syncthreads();
     if (threadIdx.x < t.tc) {
@@ -307,7 +330,7 @@ __global__ void __launch_bounds__(kL1Threads, 3) l1bn_fwd_dev_kernel(const L1bnA
   long long acc[2][4] = {{0, 0, 0, 0}, {0, 0, 0, 0}};
   constexpr int U = kL1PassesCodes;
   if (t.c < a.C) {
-    RowWalk w = row_walk(t);
+    RowWalk w = row_walk(t, b);
     const int8_t* pq = a.xq + w.r * a.C + t.c;
     const int64_t sq = w.S * a.C;
     int sabs[4] = {0, 0, 0, 0}, ssgn[4] = {0, 0, 0, 0};
@@ -315,7 +338,7 @@ __global__ void __launch_bounds__(kL1Threads, 3) l1bn_fwd_dev_kernel(const L1bnA
     for (; w.r < a.R; w.r += U * w.S, pq += U * sq) {
       uint32_t q[U];
 #pragma unroll
-      for (int u = 0; u < U; ++u) q[u] = w.r + u * w.S < a.R ? load_codes_w(pq + u * sq, t.c, a.C) : 0u;
+      for (int u = 0; u < U; ++u) q[u] = w.r + u * w.S < a.R ? load_codes_w<COH>(pq + u * sq, t.c, a.C) : 0u;
 #pragma unroll
       for (int u = 0; u < U; ++u) {
         if (w.r + u * w.S >= a.R) break;
@@ -343,8 +366,16 @@ __global__ void __launch_bounds__(kL1Threads, 3) l1bn_fwd_dev_kernel(const L1bnA
       acc[1][j] += ssgn[j];
     }
   }
-  long long* const dst[2] = {stat_slot(a.st, kStS, a.C), stat_slot(a.st, kStZ, a.C)};
-  red_end<2>(acc, dst, t, a.C, sm);
+  long long* const dst[2] = {stat_slot(a.st, kStS, a.C, b.y), stat_slot(a.st, kStZ, a.C, b.y)};
+  red_end<2>(acc, dst, t, a.C, sm, b);
+}
+
+__global__ void __launch_bounds__(kL1Threads, 3) l1bn_fwd_dev_kernel(const L1bnArgs a, int lg) {
+  griddep_wait();
+  griddep_launch_dependents();
+  __shared__ RedSmem<2> sm;
+  __shared__ int mean[kL1MaxCols];
+  fwd_dev_pass<false>(a, lg, launch_blk(), sm, mean);
 }
 
 // max over the block of non-negative values given as bit patterns
@@ -368,6 +399,29 @@ __device__ __forceinline__ float quant8(float v, float vmax) {
   return __fmul_rn(k, step);
 }
 
+// The forward statistics of channel c: its step s_c = s 2^-e_c, mean code m_c =
+// round-half-even(sum q / R) and sigma_c = (sum |q - m| / R) s_c.
+struct FwdChan {
+  float s, m, sig;
+};
+
+__device__ __forceinline__ FwdChan fwd_chan_of(const L1bnArgs& a, int64_t c, float scale, float Rf) {
+  FwdChan f;
+  f.s = __fmul_rn(scale, pow2f(-static_cast<int>(__ldcg(a.xe + c))));
+  f.m = static_cast<float>(rne_div(stat_sum(a.st, kStS1, a.C, c), a.R));
+  f.sig = __fmul_rn(__fdiv_rn(__ll2float_rn(stat_sum(a.st, kStS, a.C, c)), Rf), f.s);
+  return f;
+}
+
+// The output for code q of a channel with step s, mean code m and quantized sigma^q,
+// gamma^q, beta^q: y = gamma^q (q s - m s) / sigma^q + beta^q (beta^q where sigma^q = 0).
+__device__ __forceinline__ float l1bn_out_of(int q, float s, float m, float sq, float gq, float bq) {
+  const float xq = __fmul_rn(static_cast<float>(q), s);
+  const float mq = __fmul_rn(m, s);
+  const float xhat = sq > 0.0f ? __fdiv_rn(__fsub_rn(xq, mq), sq) : 0.0f;
+  return __fadd_rn(__fmul_rn(gq, xhat), bq);
+}
+
 // Forward pass 3 (one block): s_c, m_c, sigma_c, then sigma^q, gamma^q, beta^q.
 __global__ void __launch_bounds__(1024) l1bn_fwd_chan_kernel(const L1bnArgs a) {
   griddep_wait();
@@ -379,13 +433,11 @@ __global__ void __launch_bounds__(1024) l1bn_fwd_chan_kernel(const L1bnArgs a) {
   const int64_t C = a.C;
   uint32_t ms = 0, mg = 0, mb = 0;
   for (int64_t c = threadIdx.x; c < C; c += blockDim.x) {
-    const float s = __fmul_rn(scale, pow2f(-static_cast<int>(a.xe[c])));
-    const long long m = rne_div(stat_sum(a.st, kStS1, C, c), a.R);
-    const float sig = __fmul_rn(__fdiv_rn(__ll2float_rn(stat_sum(a.st, kStS, C, c)), Rf), s);
-    ch[kChS * C + c] = s;
-    ch[kChM * C + c] = static_cast<float>(m);
-    ch[kChSig * C + c] = sig;
-    ms = max(ms, __float_as_uint(sig) & 0x7FFFFFFFu);
+    const FwdChan f = fwd_chan_of(a, c, scale, Rf);
+    ch[kChS * C + c] = f.s;
+    ch[kChM * C + c] = f.m;
+    ch[kChSig * C + c] = f.sig;
+    ms = max(ms, __float_as_uint(f.sig) & 0x7FFFFFFFu);
     mg = max(mg, __float_as_uint(a.gamma[c]) & 0x7FFFFFFFu);
     mb = max(mb, __float_as_uint(a.beta[c]) & 0x7FFFFFFFu);
   }
@@ -408,11 +460,9 @@ __global__ void __launch_bounds__(kLutStride) l1bn_fwd_lut_kernel(const L1bnArgs
   const int64_t C = a.C, c = blockIdx.x;
   const float* ch = a.ch;
   const int q = static_cast<int>(threadIdx.x) - 127;
-  const float s = ch[kChS * C + c], sq = ch[kChSq * C + c];
-  const float xq = __fmul_rn(static_cast<float>(q), s);
-  const float mq = __fmul_rn(ch[kChM * C + c], s);
-  const float xhat = sq > 0.0f ? __fdiv_rn(__fsub_rn(xq, mq), sq) : 0.0f;
-  a.lut[c * kLutStride + threadIdx.x] = __fadd_rn(__fmul_rn(ch[kChGq * C + c], xhat), ch[kChBq * C + c]);
+  a.lut[c * kLutStride + threadIdx.x] = l1bn_out_of(q, ch[kChS * C + c], ch[kChM * C + c],
+                                                    ch[kChSq * C + c], ch[kChGq * C + c],
+                                                    ch[kChBq * C + c]);
 }
 
 // zero n 64-bit channel sums (the first kernel of a call: nothing before it in the call)
@@ -423,21 +473,14 @@ __global__ void __launch_bounds__(256) l1bn_zero_kernel(long long* __restrict__ 
 }
 
 // Forward pass 4: y = gamma^q ((x^q - mu^q) / sigma^q) + beta^q, looked up per code from
-// the table the channel pass built (copied to shared memory for the block's columns).
-__global__ void __launch_bounds__(kL1Threads, 3) l1bn_fwd_out_kernel(const L1bnArgs a, int lg) {
-  griddep_wait();
-  griddep_launch_dependents();
-  extern __shared__ float lut[];   // [tile columns][kLutStride]
-  const TilePos t = tile_pos(lg);
+// lut, the block's columns' tables in shared memory.
+template <bool COH>
+__device__ __forceinline__ void fwd_out_pass(const L1bnArgs& a, int lg, const Blk& b, const float* lut) {
+  const TilePos t = tile_pos(lg, b);
   const int64_t C = a.C;
-  const int64_t cbase = static_cast<int64_t>(blockIdx.x) * t.tc;
-  const int ncol = static_cast<int>(min(static_cast<int64_t>(t.tc), C - cbase));
-  for (int i = threadIdx.x; i < ncol * kLutStride; i += kL1Threads)
-    lut[i] = a.lut[cbase * kLutStride + i];
-  __syncthreads();
   if (t.c >= C) return;
   constexpr int U = kL1PassesCodes;
-  RowWalk w = row_walk(t);
+  RowWalk w = row_walk(t, b);
   const int8_t* pq = a.xq + w.r * C + t.c;
   float* py = a.out + w.r * a.ld_out + t.c;
   const int64_t sq = w.S * C, sy = w.S * a.ld_out;
@@ -445,7 +488,7 @@ __global__ void __launch_bounds__(kL1Threads, 3) l1bn_fwd_out_kernel(const L1bnA
   for (; w.r < a.R; w.r += U * w.S, pq += U * sq, py += U * sy) {
     uint32_t q[U];
 #pragma unroll
-    for (int u = 0; u < U; ++u) q[u] = w.r + u * w.S < a.R ? load_codes_w(pq + u * sq, t.c, C) : 0u;
+    for (int u = 0; u < U; ++u) q[u] = w.r + u * w.S < a.R ? load_codes_w<COH>(pq + u * sq, t.c, C) : 0u;
 #pragma unroll
     for (int u = 0; u < U; ++u) {
       if (w.r + u * w.S >= a.R) break;
@@ -457,27 +500,37 @@ __global__ void __launch_bounds__(kL1Threads, 3) l1bn_fwd_out_kernel(const L1bnA
   }
 }
 
-// Backward pass 1: dy -> int8 ShiftQuant codes p (stochastic rounding of element r C + c),
-// sums of p and of p (q - m) per channel.
-__global__ void __launch_bounds__(kL1Threads, 3) l1bn_bwd_quant_kernel(const L1bnArgs a, int lg) {
+__global__ void __launch_bounds__(kL1Threads, 3) l1bn_fwd_out_kernel(const L1bnArgs a, int lg) {
   griddep_wait();
   griddep_launch_dependents();
-  __shared__ RedSmem<2> sm;
-  const TilePos t = tile_pos(lg);
-  const float tau = a.scal[kScGTau];
+  extern __shared__ float lut[];   // [tile columns][kLutStride]
+  const int64_t cbase = static_cast<int64_t>(blockIdx.x) * (int64_t(4) << lg);
+  const int ncol = static_cast<int>(min(int64_t(4) << lg, a.C - cbase));
+  for (int i = threadIdx.x; i < ncol * kLutStride; i += kL1Threads)
+    lut[i] = a.lut[cbase * kLutStride + i];
+  __syncthreads();
+  fwd_out_pass<false>(a, lg, launch_blk(), lut);
+}
+
+// Backward pass 1: dy -> int8 ShiftQuant codes p (stochastic rounding of element r C + c),
+// sums of p and of p (q - m) per channel.  tau: dy's tau_0; the exponent of column c is
+// ex[c - ex0].
+__device__ __forceinline__ void bwd_quant_pass(const L1bnArgs& a, int lg, const Blk& b, float tau,
+                                               const uint8_t* ex, int64_t ex0, RedSmem<2>& sm) {
+  const TilePos t = tile_pos(lg, b);
   const float Qf = static_cast<float>(a.Q);
   const float invS = __fdiv_rn(Qf, tau);
   const bool zero = !(tau > 0.0f) || !isfinite(tau) || !isfinite(invS);
   int e[4], m[4];
 #pragma unroll
   for (int j = 0; j < 4; ++j) {
-    e[j] = t.c + j < a.C ? a.ge[t.c + j] : 0;
+    e[j] = t.c + j < a.C ? ex[t.c + j - ex0] : 0;
     m[j] = t.c + j < a.C ? static_cast<int>(a.ch[kChM * a.C + t.c + j]) : 0;
   }
   long long acc[2][4] = {{0, 0, 0, 0}, {0, 0, 0, 0}};
   constexpr int U = kL1PassesF32;
   if (t.c < a.C) {
-    RowWalk w = row_walk(t);
+    RowWalk w = row_walk(t, b);
     const float* pg = a.in + w.r * a.ld_in + t.c;
     const int8_t* px = a.xq + w.r * a.C + t.c;
     int8_t* pp = a.gq + w.r * a.C + t.c;
@@ -510,10 +563,52 @@ __global__ void __launch_bounds__(kL1Threads, 3) l1bn_bwd_quant_kernel(const L1b
       }
     }
   }
-  long long* const dst[2] = {stat_slot(a.st, kStP, a.C), stat_slot(a.st, kStD, a.C)};
-  red_end<2>(acc, dst, t, a.C, sm);
-  if (blockIdx.x == 0 && blockIdx.y == 0 && threadIdx.x == 0)
-    a.scal[kScGScale] = zero ? 0.0f : __fdiv_rn(tau, Qf);
+  long long* const dst[2] = {stat_slot(a.st, kStP, a.C, b.y), stat_slot(a.st, kStD, a.C, b.y)};
+  red_end<2>(acc, dst, t, a.C, sm, b);
+  if (b.x == 0 && b.y == 0 && threadIdx.x == 0) a.scal[kScGScale] = zero ? 0.0f : __fdiv_rn(tau, Qf);
+}
+
+__global__ void __launch_bounds__(kL1Threads, 3) l1bn_bwd_quant_kernel(const L1bnArgs a, int lg) {
+  griddep_wait();
+  griddep_launch_dependents();
+  __shared__ RedSmem<2> sm;
+  bwd_quant_pass(a, lg, launch_blk(), a.scal[kScGTau], a.ge, 0, sm);
+}
+
+// The backward constants of channel c: dy's step t_c, u = gamma^q / sigma^q, mean g,
+// mean(g xhat), mean sign(q - m), dgamma and dbeta.
+struct BwdChan {
+  float t, u, mg, mgx, zs, dg, db;
+};
+
+__device__ __forceinline__ BwdChan bwd_chan_of(const L1bnArgs& a, int64_t c, float gscale, float Rf) {
+  const int64_t C = a.C;
+  const float* ch = a.ch;
+  BwdChan k;
+  k.t = __fmul_rn(gscale, pow2f(-static_cast<int>(__ldcg(a.ge + c))));
+  const float sq = ch[kChSq * C + c], s = ch[kChS * C + c];
+  const float P = __ll2float_rn(stat_sum(a.st, kStP, C, c));
+  k.u = sq > 0.0f ? __fdiv_rn(ch[kChGq * C + c], sq) : 0.0f;
+  k.mg = __fdiv_rn(__fmul_rn(P, k.t), Rf);
+  k.dg = sq > 0.0f ? __fdiv_rn(__fmul_rn(__fmul_rn(__ll2float_rn(stat_sum(a.st, kStD, C, c)), k.t), s), sq)
+                   : 0.0f;
+  k.mgx = __fdiv_rn(k.dg, Rf);
+  k.zs = __fdiv_rn(__ll2float_rn(stat_sum(a.st, kStZ, C, c)), Rf);
+  k.db = __fmul_rn(P, k.t);
+  return k;
+}
+
+// channel c's backward constants into the state (for the output pass), dgamma and dbeta
+__device__ __forceinline__ void put_bwd_chan(const L1bnArgs& a, int64_t c, const BwdChan& k) {
+  const int64_t C = a.C;
+  float* ch = a.ch;
+  ch[kChT * C + c] = k.t;
+  ch[kChU * C + c] = k.u;
+  ch[kChMg * C + c] = k.mg;
+  ch[kChMgx * C + c] = k.mgx;
+  ch[kChZs * C + c] = k.zs;
+  a.dgamma[c] = k.dg;
+  a.dbeta[c] = k.db;
 }
 
 // Backward pass 2: the per-channel constants of the input gradient, dgamma and dbeta.
@@ -522,34 +617,20 @@ __global__ void __launch_bounds__(256) l1bn_bwd_chan_kernel(const L1bnArgs a) {
   griddep_launch_dependents();
   const float Rf = __ll2float_rn(a.R);
   const float gscale = a.scal[kScGScale];
-  const int64_t C = a.C;
-  float* ch = a.ch;
-  for (int64_t c = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; c < C;
-       c += static_cast<int64_t>(gridDim.x) * blockDim.x) {
-    const float t = __fmul_rn(gscale, pow2f(-static_cast<int>(a.ge[c])));
-    const float sq = ch[kChSq * C + c], s = ch[kChS * C + c];
-    const float P = __ll2float_rn(stat_sum(a.st, kStP, C, c));
-    const float u = sq > 0.0f ? __fdiv_rn(ch[kChGq * C + c], sq) : 0.0f;
-    const float mg = __fdiv_rn(__fmul_rn(P, t), Rf);
-    const float dg =
-        sq > 0.0f ? __fdiv_rn(__fmul_rn(__fmul_rn(__ll2float_rn(stat_sum(a.st, kStD, C, c)), t), s), sq) : 0.0f;
-    ch[kChT * C + c] = t;
-    ch[kChU * C + c] = u;
-    ch[kChMg * C + c] = mg;
-    ch[kChMgx * C + c] = __fdiv_rn(dg, Rf);
-    ch[kChZs * C + c] = __fdiv_rn(__ll2float_rn(stat_sum(a.st, kStZ, C, c)), Rf);
-    a.dgamma[c] = dg;
-    a.dbeta[c] = __fmul_rn(P, t);
-  }
+  for (int64_t c = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; c < a.C;
+       c += static_cast<int64_t>(gridDim.x) * blockDim.x)
+    put_bwd_chan(a, c, bwd_chan_of(a, c, gscale, Rf));
 }
 
 // Backward pass 3: dx = u ((g - mean g) - mean(g xhat) (sign(q - m) - mean sign)), the
 // per-channel values of each thread's quad in registers; mean(g xhat) (sign - mean sign)
-// takes one of three values per channel, formed once.
-__global__ void __launch_bounds__(kL1Threads, 3) l1bn_bwd_out_kernel(const L1bnArgs a, int lg) {
-  griddep_wait();
-  griddep_launch_dependents();
-  const TilePos t = tile_pos(lg);
+// takes one of three values per channel, formed once.  FROM_STATE: the constants come
+// from the state (the channel pass wrote them); otherwise from kc[c - first column of the
+// block's tile], formed by the caller with bwd_chan_of (the same operations), and the codes
+// are read coherently (the single-launch form writes them in the same launch).
+template <bool FROM_STATE>
+__device__ __forceinline__ void bwd_out_pass(const L1bnArgs& a, int lg, const Blk& b, const BwdChan* kc) {
+  const TilePos t = tile_pos(lg, b);
   if (t.c >= a.C) return;
   const float* ch = a.ch;
   const int64_t C = a.C;
@@ -559,15 +640,26 @@ __global__ void __launch_bounds__(kL1Threads, 3) l1bn_bwd_out_kernel(const L1bnA
   for (int j = 0; j < 4; ++j) {
     const int64_t c = t.c + j < C ? t.c + j : C - 1;
     m[j] = static_cast<int>(ch[kChM * C + c]);
-    tt[j] = ch[kChT * C + c];
-    mg[j] = ch[kChMg * C + c];
-    u4[j] = ch[kChU * C + c];
-    const float mgx = ch[kChMgx * C + c], zs = ch[kChZs * C + c];
+    float mgx, zs;
+    if (FROM_STATE) {
+      tt[j] = ch[kChT * C + c];
+      mg[j] = ch[kChMg * C + c];
+      u4[j] = ch[kChU * C + c];
+      mgx = ch[kChMgx * C + c];
+      zs = ch[kChZs * C + c];
+    } else {
+      const BwdChan& v = kc[c - b.x * t.tc];
+      tt[j] = v.t;
+      mg[j] = v.mg;
+      u4[j] = v.u;
+      mgx = v.mgx;
+      zs = v.zs;
+    }
 #pragma unroll
     for (int sgn = -1; sgn <= 1; ++sgn) k[j][sgn + 1] = __fmul_rn(mgx, __fsub_rn(static_cast<float>(sgn), zs));
   }
   constexpr int U = kL1PassesCodes;
-  RowWalk w = row_walk(t);
+  RowWalk w = row_walk(t, b);
   const int8_t* pq = a.xq + w.r * C + t.c;
   const int8_t* pp = a.gq + w.r * C + t.c;
   float* pd = a.out + w.r * a.ld_out + t.c;
@@ -577,8 +669,8 @@ __global__ void __launch_bounds__(kL1Threads, 3) l1bn_bwd_out_kernel(const L1bnA
 #pragma unroll
     for (int u = 0; u < U; ++u) {
       const bool in = w.r + u * w.S < a.R;
-      q[u] = in ? load_codes_w(pq + u * sc, t.c, C) : 0u;
-      p[u] = in ? load_codes_w(pp + u * sc, t.c, C) : 0u;
+      q[u] = in ? load_codes_w<!FROM_STATE>(pq + u * sc, t.c, C) : 0u;
+      p[u] = in ? load_codes_w<!FROM_STATE>(pp + u * sc, t.c, C) : 0u;
     }
 #pragma unroll
     for (int u = 0; u < U; ++u) {
@@ -594,6 +686,268 @@ __global__ void __launch_bounds__(kL1Threads, 3) l1bn_bwd_out_kernel(const L1bnA
       store4(pd + u * sd, t.c, C, a.vec_out, dx);
     }
   }
+}
+
+__global__ void __launch_bounds__(kL1Threads, 3) l1bn_bwd_out_kernel(const L1bnArgs a, int lg) {
+  griddep_wait();
+  griddep_launch_dependents();
+  bwd_out_pass<true>(a, lg, launch_blk(), nullptr);
+}
+
+// ------------------------------------------------------------- single-launch form
+// For up to kCoopMaxChannels channels the passes of a call run as the phases of one
+// cooperative launch (every block resident), separated by grid barriers: on the ResNet
+// shapes the launch-to-launch gaps of the chain of kernels cost more than its HBM traffic.
+// Each phase runs the same pass body as the multi-kernel form (the same operations in the
+// same order, so the results are bit for bit the same); what the multi-kernel form reads
+// back from the state between launches (tau_0, exponents, channel constants) each block
+// forms here from the channel sums itself, for the columns it needs.
+constexpr int kCoopMaxChannels = 1024;
+constexpr int kCoopOutLg = 3;   // output-pass tiles of 32 columns (a 32 KB table per block)
+
+// Grid barrier of a cooperative launch: the k-th barrier of a call waits until the
+// counter (zeroed before the launch) reaches k gridDim.x.  A block's writes are ordered
+// before its arrival by the block barrier and the arrival's release; the acquire load that
+// sees the count orders the other blocks' writes before what the block reads next.
+// (Measured with 456 blocks: 1.6 us a barrier; with full fences around a relaxed atomic,
+// 2.0-2.2 us, also with the arrivals spread over up to 32 counters.)  Bounded: after
+// kWaitBudgetNs the block records SQ_DEV_TIMEOUT and the call's blocks unwind (each gives
+// up at its own next barrier).
+__device__ __forceinline__ bool grid_barrier(unsigned* ctr, unsigned target, int* status) {
+  __shared__ int ok;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    asm volatile("red.release.gpu.global.add.u32 [%0], 1;" ::"l"(ctr) : "memory");
+    int good = 1;
+    const uint64_t t0 = globaltimer_ns();
+    while (true) {
+      unsigned v;
+      asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(ctr) : "memory");
+      if (v >= target) break;
+      if (globaltimer_ns() - t0 > kWaitBudgetNs) {
+        atomicOr(status, kDevTimeout);
+        good = 0;
+        break;
+      }
+      __nanosleep(32);
+    }
+    ok = good;
+  }
+  __syncthreads();
+  return ok != 0;
+}
+
+// zero n 64-bit channel sums, spread over the launch's blocks
+__device__ __forceinline__ void zero_sums(long long* p, int64_t n) {
+  for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < n;
+       i += static_cast<int64_t>(gridDim.x) * blockDim.x)
+    p[i] = 0;
+}
+
+// Range pass of x (or dy): the per-column max |x| of the block's rows into slot row
+// b.y mod kSpread of `slots` (ordered bit patterns), as shiftquant_calibrate forms them.
+__device__ __forceinline__ void range_pass(const L1bnArgs& a, int lg, const Blk& b, unsigned* slots,
+                                           RedSmem<1>& sm, int* status) {
+  const TilePos t = tile_pos(lg, b);
+  unsigned mx[4] = {0u, 0u, 0u, 0u};
+  constexpr int U = kL1PassesF32;
+  if (t.c < a.C) {
+    RowWalk w = row_walk(t, b);
+    const float* px = a.in + w.r * a.ld_in + t.c;
+    const int64_t sx = w.S * a.ld_in;
+    for (; w.r < a.R; w.r += U * w.S, px += U * sx) {
+      float v[U][4];
+#pragma unroll
+      for (int u = 0; u < U; ++u)
+        if (w.r + u * w.S < a.R) load4(px + u * sx, t.c, a.C, a.vec_in, v[u]);
+#pragma unroll
+      for (int u = 0; u < U; ++u) {
+        if (w.r + u * w.S >= a.R) break;
+#pragma unroll
+        for (int j = 0; j < 4; ++j) mx[j] = max(mx[j], __float_as_uint(v[u][j]) & 0x7FFFFFFFu);
+      }
+    }
+  }
+#pragma unroll
+  for (int j = 0; j < 4; ++j) sm.part[0][t.ro * t.tc + t.qc * 4 + j] = mx[j];
+  __syncthreads();
+  const int tid = threadIdx.x;
+  const int64_t c = b.x * t.tc + tid;
+  if (tid < t.tc && c < a.C) {
+    unsigned m = 0;
+    for (int r = 0; r < t.rpp; ++r) m = max(m, static_cast<unsigned>(sm.part[0][r * t.tc + tid]));
+    if (m != 0u) atomicMax(slots + (b.y % kSpread) * a.C + c, m);
+    if (m >= 0x7F800000u) atomicOr(status, kDevNonFinite);
+  }
+  __syncthreads();   // sm is reused by the next phase
+}
+
+// range of column c: its slot rows' maximum (bit pattern)
+__device__ __forceinline__ unsigned slot_range(const unsigned* slots, int64_t C, int64_t c) {
+  unsigned m = 0;
+#pragma unroll
+  for (int i = 0; i < kSpread; ++i) m = max(m, __ldcg(slots + i * C + c));
+  return m;
+}
+
+// After the range pass: tau_0 (the largest range) and the exponents of the block's tile
+// columns (Eq. 3, as group_kernel forms them) into sexp; block 0 also stores the ranges,
+// tau_0 and every exponent in the state.  Returns tau_0.
+__device__ __forceinline__ float coop_group(const L1bnArgs& a, int lg, const Blk& b, int G,
+                                            const unsigned* slots, float* range_out, float* tau_out,
+                                            uint8_t* exp_out, uint8_t* sexp, uint32_t* red,
+                                            int* status) {
+  unsigned m = 0;
+  for (int64_t c = threadIdx.x; c < a.C; c += kL1Threads) m = max(m, slot_range(slots, a.C, c));
+  const unsigned tb = block_max(m, red);
+  const float tau = __uint_as_float(tb);
+  const bool nonfinite = tb >= 0x7F800000u;
+  const int tc = 4 << lg;
+  const int64_t c0 = b.x * tc;
+  if (threadIdx.x < tc && c0 + threadIdx.x < a.C) {
+    const unsigned r = slot_range(slots, a.C, c0 + threadIdx.x);
+    sexp[threadIdx.x] = static_cast<uint8_t>(nonfinite ? 0 : group_exponent(__uint_as_float(r), tau, G));
+  }
+  if (blockIdx.x == 0) {
+    for (int64_t c = threadIdx.x; c < a.C; c += kL1Threads) {
+      const unsigned r = slot_range(slots, a.C, c);
+      range_out[c] = __uint_as_float(r);
+      exp_out[c] = static_cast<uint8_t>(nonfinite ? 0 : group_exponent(__uint_as_float(r), tau, G));
+    }
+    if (threadIdx.x == 0) {
+      *tau_out = tau;
+      if (nonfinite) atomicOr(status, kDevNonFinite);
+    }
+  }
+  __syncthreads();
+  return tau;
+}
+
+struct CoopGeom {
+  int lg, gx, gy;     // reduction passes: tile columns 4 << lg, gx x gy blocks
+  int lgo, gxo, gyo;  // output pass: tile columns 4 << lgo, gxo x gyo blocks
+  int G;
+  int* status;
+};
+
+__device__ __forceinline__ Blk red_blk(const CoopGeom& g) {
+  return Blk{blockIdx.x % g.gx, blockIdx.x / g.gx, g.gx, g.gy};
+}
+__device__ __forceinline__ Blk out_blk(const CoopGeom& g) {
+  return Blk{blockIdx.x % g.gxo, blockIdx.x / g.gxo, g.gxo, g.gyo};
+}
+
+// The forward as one launch: range pass -> tau_0, exponents, codes and code sums -> the
+// deviation sums -> channel constants and output tables, spread over the blocks by channel
+// -> output.  (Each block building the tables of its own output columns instead -- 8192
+// entries, a division each -- took 8.7 us of a 29 us call on [12544, 256].)
+__global__ void __launch_bounds__(kL1Threads, 3) l1bn_fwd_coop_kernel(const L1bnArgs a, const CoopGeom g) {
+  extern __shared__ __align__(16) unsigned char dyn[];   // reductions, then the output table
+  __shared__ uint8_t sexp[kL1MaxCols];
+  __shared__ int mean[kL1MaxCols];
+  __shared__ uint32_t red[32];
+  __shared__ float cs[1], cm[1], csq[1], cgq[1], cbq[1];
+  RedSmem<2>& sm2 = *reinterpret_cast<RedSmem<2>*>(dyn);
+  RedSmem<1>& sm1 = *reinterpret_cast<RedSmem<1>*>(dyn);
+  unsigned* ctr = a.sync;
+  unsigned* slots = a.sync + 64;
+  const unsigned nb = gridDim.x;
+  const bool red_on = blockIdx.x < static_cast<unsigned>(g.gx * g.gy);
+  const Blk b = red_blk(g);
+  // 1. range pass; the sums the later phases add into start at zero
+  zero_sums(a.st, 3 * kSpread * a.C);   // kStS1, kStS, kStZ
+  if (red_on) range_pass(a, g.lg, b, slots, sm1, g.status);
+  if (!grid_barrier(ctr, nb, g.status)) return;
+  // 2. tau_0, exponents; codes and their sums
+  if (red_on) {
+    const float tau = coop_group(a, g.lg, b, g.G, slots, a.ch + kChXRange * a.C, a.scal + kScXTau,
+                                 a.xe, sexp, red, g.status);
+    fwd_quant_pass(a, g.lg, b, tau, sexp, b.x * (int64_t(4) << g.lg), sm1);
+  }
+  if (!grid_barrier(ctr, 2 * nb, g.status)) return;
+  // 3. deviation sums
+  if (red_on) fwd_dev_pass<true>(a, g.lg, b, sm2, mean);
+  if (!grid_barrier(ctr, 3 * nb, g.status)) return;
+  // 4. per-tensor maxima of sigma, |gamma|, |beta| over all channels
+  const float Rf = __ll2float_rn(a.R);
+  const float scale = __ldcg(a.scal + kScXScale);
+  uint32_t ms = 0, mg = 0, mb = 0;
+  for (int64_t c = threadIdx.x; c < a.C; c += kL1Threads) {
+    ms = max(ms, __float_as_uint(fwd_chan_of(a, c, scale, Rf).sig) & 0x7FFFFFFFu);
+    mg = max(mg, __float_as_uint(a.gamma[c]) & 0x7FFFFFFFu);
+    mb = max(mb, __float_as_uint(a.beta[c]) & 0x7FFFFFFFu);
+  }
+  const float smax = __uint_as_float(block_max(ms, red));
+  const float gmax = __uint_as_float(block_max(mg, red));
+  const float bmax = __uint_as_float(block_max(mb, red));
+  // 5. block b: the constants of channels b, b + gridDim.x, ... into the state (the
+  // backward reads them) and their output tables (one entry per thread)
+  for (int64_t c = blockIdx.x; c < a.C; c += gridDim.x) {
+    if (threadIdx.x == 0) {
+      const int64_t C = a.C;
+      const FwdChan f = fwd_chan_of(a, c, scale, Rf);
+      cs[0] = f.s;
+      cm[0] = f.m;
+      csq[0] = quant8(f.sig, smax);
+      cgq[0] = quant8(a.gamma[c], gmax);
+      cbq[0] = quant8(a.beta[c], bmax);
+      a.ch[kChS * C + c] = f.s;
+      a.ch[kChM * C + c] = f.m;
+      a.ch[kChSig * C + c] = f.sig;
+      a.ch[kChSq * C + c] = csq[0];
+      a.ch[kChGq * C + c] = cgq[0];
+      a.ch[kChBq * C + c] = cbq[0];
+    }
+    __syncthreads();
+    a.lut[c * kLutStride + threadIdx.x] =
+        l1bn_out_of(static_cast<int>(threadIdx.x) - 127, cs[0], cm[0], csq[0], cgq[0], cbq[0]);
+    __syncthreads();
+  }
+  if (!grid_barrier(ctr, 4 * nb, g.status)) return;
+  // 6. output: the block's columns' tables into shared memory, then y
+  if (blockIdx.x >= static_cast<unsigned>(g.gxo * g.gyo)) return;
+  const Blk bo = out_blk(g);
+  const int64_t cbase = bo.x * (int64_t(4) << g.lgo);
+  const int ncol = static_cast<int>(min(int64_t(4) << g.lgo, a.C - cbase));
+  float* lut = reinterpret_cast<float*>(dyn);
+  for (int i = threadIdx.x; i < ncol * kLutStride; i += kL1Threads) lut[i] = __ldcg(a.lut + cbase * kLutStride + i);
+  __syncthreads();
+  fwd_out_pass<true>(a, g.lgo, bo, lut);
+}
+
+// The backward as one launch: range pass of dy -> its tau_0, exponents, codes and the sums
+// of p and p (q - m) -> channel constants (dgamma, dbeta) and the input gradient.
+__global__ void __launch_bounds__(kL1Threads, 2) l1bn_bwd_coop_kernel(const L1bnArgs a, const CoopGeom g) {
+  __shared__ RedSmem<2> sm2;
+  __shared__ uint8_t sexp[kL1MaxCols];
+  __shared__ uint32_t red[32];
+  __shared__ BwdChan sc[4 << kCoopOutLg];
+  RedSmem<1>& sm1 = *reinterpret_cast<RedSmem<1>*>(&sm2);
+  unsigned* ctr = a.sync;
+  unsigned* slots = a.sync + 64;
+  const unsigned nb = gridDim.x;
+  const bool red_on = blockIdx.x < static_cast<unsigned>(g.gx * g.gy);
+  const Blk b = red_blk(g);
+  zero_sums(a.st + kStP * kSpread * a.C, 2 * kSpread * a.C);   // kStP, kStD
+  if (red_on) range_pass(a, g.lg, b, slots, sm1, g.status);
+  if (!grid_barrier(ctr, nb, g.status)) return;
+  if (red_on) {
+    const float tau = coop_group(a, g.lg, b, g.G, slots, a.ch + kChGRange * a.C, a.scal + kScGTau,
+                                 a.ge, sexp, red, g.status);
+    bwd_quant_pass(a, g.lg, b, tau, sexp, b.x * (int64_t(4) << g.lg), sm2);
+  }
+  if (!grid_barrier(ctr, 2 * nb, g.status)) return;
+  if (blockIdx.x >= static_cast<unsigned>(g.gxo * g.gyo)) return;
+  const Blk bo = out_blk(g);
+  const float gscale = __ldcg(a.scal + kScGScale);
+  const float Rf = __ll2float_rn(a.R);
+  const int64_t c = bo.x * (int64_t(4) << g.lgo) + threadIdx.x;
+  if (threadIdx.x < (4 << g.lgo) && c < a.C) {
+    sc[threadIdx.x] = bwd_chan_of(a, c, gscale, Rf);
+    if (bo.y == 0) put_bwd_chan(a, c, sc[threadIdx.x]);   // dgamma, dbeta, the state: once per column
+  }
+  __syncthreads();
+  bwd_out_pass<false>(a, g.lgo, bo, sc);
 }
 
 // ------------------------------------------------------------------ host side
@@ -621,6 +975,7 @@ static L1bnArgs l1bn_args(int64_t R, int64_t C, int bits, void* state) {
   a.xe = reinterpret_cast<uint8_t*>(b + L.exps);
   a.ge = a.xe + C;
   a.scal = reinterpret_cast<float*>(b + L.scal);
+  a.sync = reinterpret_cast<unsigned*>(b + L.sync);
   return a;
 }
 
@@ -703,6 +1058,75 @@ static int launched(const char* what) {
   return err == cudaSuccess ? SQ_OK : cuda_fail(err, what);
 }
 
+// The single-launch form's block count on the current device (one resident wave: every
+// block of a cooperative launch must be resident at once), 0 where it cannot run.
+template <bool FWD>
+static int coop_blocks() {
+  static int cached[64][2];   // [device][fwd]: blocks + 1, 0 = not asked yet
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 0;
+  int& slot = cached[dev][FWD ? 1 : 0];
+  if (slot == 0) {
+    int coop = 0, sms = 0, per_sm = 0;
+    cudaDeviceGetAttribute(&coop, cudaDevAttrCooperativeLaunch, dev);
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    const size_t dyn = FWD ? size_t(4 << kCoopOutLg) * kLutStride * sizeof(float) : 0;
+    if (coop && sms > 0 &&
+        cudaOccupancyMaxActiveBlocksPerMultiprocessor(
+            &per_sm, FWD ? l1bn_fwd_coop_kernel : l1bn_bwd_coop_kernel, kL1Threads, dyn) == cudaSuccess)
+      slot = 1 + (per_sm > 3 ? 3 : per_sm) * sms;
+    else
+      slot = 1;
+    cudaGetLastError();
+  }
+  return slot - 1;
+}
+
+// The single-launch form of a call: the counter and range slots zeroed, then one
+// cooperative launch of `blocks` blocks.
+template <bool FWD>
+static int launch_coop(const L1bnArgs& a, int G, int blocks, int32_t* dev_status, cudaStream_t s) {
+  cudaError_t err = cudaMemsetAsync(a.sync, 0, 256 + kSpread * static_cast<size_t>(a.C) * sizeof(unsigned), s);
+  if (err != cudaSuccess) return cuda_fail(err, "cudaMemsetAsync (l1bn sync)");
+  CoopGeom g;
+  g.lg = tile_lg(a.C);
+  g.gx = static_cast<int>((a.C + (int64_t(4) << g.lg) - 1) / (int64_t(4) << g.lg));
+  g.gy = blocks / g.gx;
+  g.lgo = g.lg < kCoopOutLg ? g.lg : kCoopOutLg;
+  g.gxo = static_cast<int>((a.C + (int64_t(4) << g.lgo) - 1) / (int64_t(4) << g.lgo));
+  g.gyo = blocks / g.gxo;
+  g.G = G;
+  g.status = dev_status;
+  cudaLaunchConfig_t cfg;
+  memset(&cfg, 0, sizeof(cfg));
+  cfg.gridDim = dim3(static_cast<unsigned>(blocks));
+  cfg.blockDim = dim3(kL1Threads);
+  cfg.dynamicSmemBytes = FWD ? size_t(4 << g.lgo) * kLutStride * sizeof(float) : 0;
+  if (FWD && cfg.dynamicSmemBytes < sizeof(RedSmem<2>)) cfg.dynamicSmemBytes = sizeof(RedSmem<2>);
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeCooperative;
+  attr[0].val.cooperative = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  err = FWD ? cudaLaunchKernelEx(&cfg, l1bn_fwd_coop_kernel, a, g)
+            : cudaLaunchKernelEx(&cfg, l1bn_bwd_coop_kernel, a, g);
+  if (err == cudaSuccess) err = cudaGetLastError();
+  return err == cudaSuccess ? SQ_OK : cuda_fail(err, FWD ? "l1bn_fwd_coop_kernel launch" : "l1bn_bwd_coop_kernel launch");
+}
+
+// the single-launch form serves this call: few enough channels for every block to form
+// the per-tensor maxima over all of them, and a device that runs cooperative launches
+// with at least one block per output column tile
+template <bool FWD>
+static int coop_use(int64_t C) {
+  if (C > kCoopMaxChannels) return 0;
+  const int blocks = coop_blocks<FWD>();
+  const int lgo = tile_lg(C) < kCoopOutLg ? tile_lg(C) : kCoopOutLg;
+  const int64_t gxo = (C + (int64_t(4) << lgo) - 1) / (int64_t(4) << lgo);
+  return blocks >= gxo && blocks >= 8 ? blocks : 0;
+}
+
 }  // namespace sq
 
 using namespace sq;
@@ -710,6 +1134,15 @@ using namespace sq;
 extern "C" size_t shiftquant_l1bn_state_bytes(int64_t rows, int64_t channels) {
   if (rows < 0 || channels < 0) return 0;
   return l1bn_layout(rows, channels).total;
+}
+
+extern "C" int shiftquant_l1bn_kernel_launches(int64_t channels, int backward) {
+  if (channels < 0 || channels >= (int64_t(1) << 31)) return -1;
+  if (channels == 0) return 0;
+  if (l1bn_sms() <= 0) return -1;
+  if (backward ? coop_use<false>(channels) : coop_use<true>(channels)) return 1;
+  // zeroing, the range pass (zeroing, range, grouping), then the passes
+  return backward ? 1 + 3 + 3 : 1 + 3 + 5;
 }
 
 extern "C" sq_status shiftquant_l1bn_forward(const float* x, int64_t rows, int64_t channels,
@@ -734,6 +1167,7 @@ extern "C" sq_status shiftquant_l1bn_forward(const float* x, int64_t rows, int64
   a.beta = beta;
   a.vec_in = (ld_x % 4 == 0) && aligned16(x);
   a.vec_out = (ld_y % 4 == 0) && aligned16(y);
+  if (const int blocks = coop_use<true>(channels)) return launch_coop<true>(a, n_groups, blocks, dev_status, s);
   // the channel sums start at zero (a kernel, not a memset, so that the launches after the
   // range pass stay a chain of kernels, each launched behind the one before)
   const int64_t nz = 3 * kSpread * channels;
@@ -788,6 +1222,7 @@ extern "C" sq_status shiftquant_l1bn_backward(const float* dy, int64_t rows, int
   a.dbeta = dbeta;
   a.vec_in = (ld_dy % 4 == 0) && aligned16(dy);
   a.vec_out = (ld_dx % 4 == 0) && aligned16(dx);
+  if (const int blocks = coop_use<false>(channels)) return launch_coop<false>(a, n_groups, blocks, dev_status, s);
   const int64_t nz = 2 * kSpread * channels;
   l1bn_zero_kernel<<<static_cast<unsigned>((nz + 255) / 256 < 1024 ? (nz + 255) / 256 : 1024), 256, 0, s>>>(
       a.st + kStP * kSpread * channels, nz);

@@ -50,20 +50,6 @@ __device__ __forceinline__ uint32_t abs_bits(float v) { return __float_as_uint(v
 
 // range_bits[c] = max over this block's rows of |x[r, c]| as an ordered bit pattern
 // (for non-negative floats, larger value <=> larger unsigned pattern; NaN sorts above Inf).
-// exponent of one channel: max{e in [0, G-1] : r 2^e <= tau}; the product by 2^e is exact
-// (no rounding) for every finite r <= tau, so the comparison is exact
-__device__ __forceinline__ int group_exponent(float r, float tau, int G) {
-  if (r == 0.0f) return G - 1;
-  int e = 0;
-#pragma unroll 1
-  for (int k = 1; k < G; ++k) {
-    const float scaled = __fmul_rn(r, __int_as_float((127 + k) << 23));  // r 2^k
-    if (scaled <= tau) e = k;
-    else break;
-  }
-  return e;
-}
-
 // zero the range accumulators a[na] and b[nb] (b may be null); the range pass that follows
 // may launch at once: it reads x first and these only after its wait
 __global__ void __launch_bounds__(256)

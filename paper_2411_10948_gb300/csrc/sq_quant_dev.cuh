@@ -30,6 +30,20 @@ __device__ __forceinline__ uint32_t splitmix64_top24(uint64_t z) {
 
 __device__ __forceinline__ float pow2f(int k) { return __int_as_float((127 + k) << 23); }
 
+// The grouping of Eq. 3 for one channel: max{e in [0, G-1] : r 2^e <= tau}; the product by
+// 2^e is exact (no rounding) for every finite r <= tau, so the comparison is exact.
+__device__ __forceinline__ int group_exponent(float r, float tau, int G) {
+  if (r == 0.0f) return G - 1;
+  int e = 0;
+#pragma unroll 1
+  for (int k = 1; k < G; ++k) {
+    const float scaled = __fmul_rn(r, __int_as_float((127 + k) << 23));  // r 2^k
+    if (scaled <= tau) e = k;
+    else break;
+  }
+  return e;
+}
+
 // The ShiftQuant code of one element (App. D; stochastic rounding of App. B): the scaled
 // value v = fl(fl(x 2^e) invS) with invS = fl(Q / tau_0), rounded to nearest even
 // (stochastic == false) or up with probability frac(v) on the draw of element `idx`,

@@ -43,6 +43,7 @@ EXPORTS = (
     "shiftquant_layer_step", "shiftquant_layer_step_host", "shiftquant_layer_step_host_split",
     "shiftquant_selftest_wait_timeout",
     "shiftquant_l1bn_state_bytes", "shiftquant_l1bn_forward", "shiftquant_l1bn_backward",
+    "shiftquant_l1bn_kernel_launches",
     "shiftquant_group_order", "shiftquant_group_order_width", "shiftquant_quantize_ordered",
     "shiftquant_pack_codes", "shiftquant_unpack_codes", "shiftquant_packed_groups_bytes",
     "shiftquant_pack_groups", "shiftquant_unpack_groups",
@@ -183,6 +184,8 @@ def load(path: str | None = None) -> ctypes.CDLL:
     lib.shiftquant_selftest_wait_timeout.restype = i32
     lib.shiftquant_l1bn_state_bytes.argtypes = [i64, i64]
     lib.shiftquant_l1bn_state_bytes.restype = sz
+    lib.shiftquant_l1bn_kernel_launches.argtypes = [i64, i32]
+    lib.shiftquant_l1bn_kernel_launches.restype = i32
     lib.shiftquant_l1bn_forward.argtypes = [vp, i64, i64, i64, vp, vp, i32, i32, vp, i64, vp, sz,
                                             vp, vp]
     lib.shiftquant_l1bn_forward.restype = i32
@@ -503,6 +506,11 @@ def shiftquant_selftest_wait_timeout(a_codes, a_scale, b_codes, b_scale, M, N, K
 
 def shiftquant_l1bn_state_bytes(rows: int, channels: int) -> int:
     return int(load().shiftquant_l1bn_state_bytes(rows, channels))
+
+
+def shiftquant_l1bn_kernel_launches(channels: int, backward: bool = False) -> int:
+    """Kernels one L1 batch-norm call launches: 1 in the single-launch form, else 9 / 7."""
+    return int(load().shiftquant_l1bn_kernel_launches(channels, 1 if backward else 0))
 
 
 def shiftquant_l1bn_forward(x, gamma, beta, bits, n_groups, y, state, dev_status,

@@ -51,7 +51,8 @@ def _run(x, gamma, beta, dy, bits, G, seed):
 @pytest.mark.parametrize("R,C,bits,G", [(12544, 256, 8, 4), (1000, 77, 8, 4), (3000, 130, 6, 3),
                                         (1, 9, 8, 4), (64, 4, 4, 1), (200, 1000, 8, 8),
                                         (20000, 64, 8, 4), (3001, 16, 8, 4), (777, 3, 8, 4),
-                                        (5000, 600, 8, 4)])
+                                        (5000, 600, 8, 4), (300, 1100, 8, 4), (1500, 1027, 6, 4),
+                                        (200704, 64, 8, 4)])
 def test_l1bn_matches_oracle_bit_for_bit(R, C, bits, G):
     rng = np.random.default_rng(R + C)
     x, gamma, beta, dy = _inputs(rng, R, C)
@@ -67,6 +68,46 @@ def test_l1bn_matches_oracle_bit_for_bit(R, C, bits, G):
     np.testing.assert_array_equal(f32_bits(dg), f32_bits(b["dgamma"]), err_msg="dgamma")
     np.testing.assert_array_equal(f32_bits(db), f32_bits(b["dbeta"]), err_msg="dbeta")
     np.testing.assert_array_equal(f32_bits(dx), f32_bits(b["dx"]), err_msg="dx")
+
+
+def test_l1bn_launch_forms():
+    # at most 1024 channels: one cooperative launch per call; wider: the chain of kernels
+    # (the shapes above cover both, and both must match the oracle bit for bit)
+    for C in (3, 64, 256, 1024):
+        assert N.shiftquant_l1bn_kernel_launches(C) == 1
+        assert N.shiftquant_l1bn_kernel_launches(C, True) == 1
+    assert N.shiftquant_l1bn_kernel_launches(1025) == 9
+    assert N.shiftquant_l1bn_kernel_launches(1100, True) == 7
+    assert N.shiftquant_l1bn_kernel_launches(0) == 0
+
+
+def test_l1bn_repeated_calls_on_one_state_stay_exact():
+    # the single-launch form zeroes its barrier counter and range slots per call: a second
+    # forward and backward on the same state (a training loop) give the same bits
+    rng = np.random.default_rng(11)
+    x, gamma, beta, dy = _inputs(rng, 4000, 96)
+    R, C = x.shape
+    st = torch.zeros(1, dtype=torch.int32, device="cuda")
+    state = torch.full((N.shiftquant_l1bn_state_bytes(R, C),), 0x5A, dtype=torch.uint8, device="cuda")
+    outs = []
+    for _ in range(2):
+        y = torch.empty((R, C), device="cuda")
+        dx = torch.empty((R, C), device="cuda")
+        dg = torch.empty(C, device="cuda")
+        db = torch.empty(C, device="cuda")
+        N.shiftquant_l1bn_forward(to_gpu(x), torch.from_numpy(gamma).cuda(), torch.from_numpy(beta).cuda(),
+                                  8, 4, y, state, st)
+        N.shiftquant_l1bn_backward(to_gpu(dy), 8, 4, 9, state, dx, dg, db, st)
+        torch.cuda.synchronize()
+        outs.append([t.cpu().numpy() for t in (y, dx, dg, db)])
+    assert st.item() == 0
+    f = O.l1bn_forward(x, gamma, beta, 8, 4)
+    b = O.l1bn_backward(dy, f, 8, 4, 9)
+    for got in outs:
+        np.testing.assert_array_equal(f32_bits(got[0]), f32_bits(f["y"]))
+        np.testing.assert_array_equal(f32_bits(got[1]), f32_bits(b["dx"]))
+        np.testing.assert_array_equal(f32_bits(got[2]), f32_bits(b["dgamma"]))
+        np.testing.assert_array_equal(f32_bits(got[3]), f32_bits(b["dbeta"]))
 
 
 def test_l1bn_nonfinite_input_sets_status():
