@@ -563,6 +563,14 @@ sq_status shiftquant_l1bn_backward(const float *dy, int64_t rows, int64_t channe
  * not depend on the form. */
 int shiftquant_l1bn_kernel_launches(int64_t channels, int backward);
 
+/* Self-test of the single-launch L1 batch normalization's grid barrier (failure path):
+ * a cooperative launch of 8 blocks in which one block never arrives, so every block's
+ * bounded wait runs out after about 1 s, ORs SQ_DEV_TIMEOUT into dev_status and returns;
+ * the context stays usable.  scratch: 256 bytes of device memory (16-byte aligned), zeroed
+ * here.  For tests of the failure path only. */
+sq_status shiftquant_selftest_grid_barrier_timeout(void *scratch, int32_t *dev_status,
+                                                   void *stream);
+
 /* Packed sub-byte storage (Sec. 5.2: with N_G = 4 the grouping map takes exactly 2 bits).
  * The tensor cores read codes as E4M3 / BF16 (there is no integer MMA on sm_103a, and the
  * 4-bit float E2M1 lacks the integers 5 and 7), so the packed form is the storage of a

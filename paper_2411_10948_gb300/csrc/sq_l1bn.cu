@@ -713,11 +713,13 @@ constexpr int kCoopOutLg = 3;   // output-pass tiles of 32 columns (a 32 KB tabl
 // 2.0-2.2 us, also with the arrivals spread over up to 32 counters.)  Bounded: after
 // kWaitBudgetNs the block records SQ_DEV_TIMEOUT and the call's blocks unwind (each gives
 // up at its own next barrier).
-__device__ __forceinline__ bool grid_barrier(unsigned* ctr, unsigned target, int* status) {
+// (arrive = false: the block waits without arriving -- the self-test of the expiry path.)
+__device__ __forceinline__ bool grid_barrier(unsigned* ctr, unsigned target, int* status,
+                                             bool arrive = true) {
   __shared__ int ok;
   __syncthreads();
   if (threadIdx.x == 0) {
-    asm volatile("red.release.gpu.global.add.u32 [%0], 1;" ::"l"(ctr) : "memory");
+    if (arrive) asm volatile("red.release.gpu.global.add.u32 [%0], 1;" ::"l"(ctr) : "memory");
     int good = 1;
     const uint64_t t0 = globaltimer_ns();
     while (true) {
@@ -950,6 +952,12 @@ __global__ void __launch_bounds__(kL1Threads, 2) l1bn_bwd_coop_kernel(const L1bn
   bwd_out_pass<false>(a, g.lgo, bo, sc);
 }
 
+// Self-test of the grid barrier's expiry path: block 0 never arrives, so every block's
+// bounded wait runs out (about 1 s), records SQ_DEV_TIMEOUT and returns.
+__global__ void __launch_bounds__(kL1Threads) l1bn_selftest_barrier_kernel(unsigned* ctr, int* status) {
+  grid_barrier(ctr, gridDim.x, status, blockIdx.x != 0);
+}
+
 // ------------------------------------------------------------------ host side
 static int l1bn_sms() {
   int dev = 0, n = 0;
@@ -1134,6 +1142,30 @@ using namespace sq;
 extern "C" size_t shiftquant_l1bn_state_bytes(int64_t rows, int64_t channels) {
   if (rows < 0 || channels < 0) return 0;
   return l1bn_layout(rows, channels).total;
+}
+
+extern "C" sq_status shiftquant_selftest_grid_barrier_timeout(void* scratch, int32_t* dev_status,
+                                                              void* stream) {
+  fail(SQ_OK, "");
+  if (scratch == nullptr || dev_status == nullptr || !aligned16(scratch))
+    return fail(SQ_EINVAL, "selftest_grid_barrier_timeout: scratch (16-byte aligned) and dev_status are required");
+  cudaStream_t s = as_stream(stream);
+  cudaError_t err = cudaMemsetAsync(scratch, 0, 256, s);
+  if (err != cudaSuccess) return cuda_fail(err, "cudaMemsetAsync");
+  cudaLaunchConfig_t cfg;
+  memset(&cfg, 0, sizeof(cfg));
+  cfg.gridDim = dim3(8);
+  cfg.blockDim = dim3(kL1Threads);
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeCooperative;
+  attr[0].val.cooperative = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  err = cudaLaunchKernelEx(&cfg, l1bn_selftest_barrier_kernel, static_cast<unsigned*>(scratch),
+                           reinterpret_cast<int*>(dev_status));
+  if (err == cudaSuccess) err = cudaGetLastError();
+  return err == cudaSuccess ? SQ_OK : cuda_fail(err, "l1bn_selftest_barrier_kernel launch");
 }
 
 extern "C" int shiftquant_l1bn_kernel_launches(int64_t channels, int backward) {

@@ -43,7 +43,7 @@ EXPORTS = (
     "shiftquant_layer_step", "shiftquant_layer_step_host", "shiftquant_layer_step_host_split",
     "shiftquant_selftest_wait_timeout",
     "shiftquant_l1bn_state_bytes", "shiftquant_l1bn_forward", "shiftquant_l1bn_backward",
-    "shiftquant_l1bn_kernel_launches",
+    "shiftquant_l1bn_kernel_launches", "shiftquant_selftest_grid_barrier_timeout",
     "shiftquant_group_order", "shiftquant_group_order_width", "shiftquant_quantize_ordered",
     "shiftquant_pack_codes", "shiftquant_unpack_codes", "shiftquant_packed_groups_bytes",
     "shiftquant_pack_groups", "shiftquant_unpack_groups",
@@ -186,6 +186,8 @@ def load(path: str | None = None) -> ctypes.CDLL:
     lib.shiftquant_l1bn_state_bytes.restype = sz
     lib.shiftquant_l1bn_kernel_launches.argtypes = [i64, i32]
     lib.shiftquant_l1bn_kernel_launches.restype = i32
+    lib.shiftquant_selftest_grid_barrier_timeout.argtypes = [vp, vp, vp]
+    lib.shiftquant_selftest_grid_barrier_timeout.restype = i32
     lib.shiftquant_l1bn_forward.argtypes = [vp, i64, i64, i64, vp, vp, i32, i32, vp, i64, vp, sz,
                                             vp, vp]
     lib.shiftquant_l1bn_forward.restype = i32
@@ -506,6 +508,12 @@ def shiftquant_selftest_wait_timeout(a_codes, a_scale, b_codes, b_scale, M, N, K
 
 def shiftquant_l1bn_state_bytes(rows: int, channels: int) -> int:
     return int(load().shiftquant_l1bn_state_bytes(rows, channels))
+
+
+def shiftquant_selftest_grid_barrier_timeout(scratch, dev_status, stream=None) -> None:
+    """Failure-path self-test: a grid barrier whose bounded waits run out (about 1 s)."""
+    _check(load().shiftquant_selftest_grid_barrier_timeout(_ptr(scratch), _ptr(dev_status),
+                                                           _stream(stream)))
 
 
 def shiftquant_l1bn_kernel_launches(channels: int, backward: bool = False) -> int:

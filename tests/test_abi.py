@@ -271,3 +271,10 @@ def test_layer_launch_refuses_in_place_weight_gradient_on_group_ordered_codes(li
     assert "transposed copy" in lib.shiftquant_last_error().decode()
     a.x_seg, a.g_seg, a.xt_codes, a.gt_codes = None, fake, fake, None
     assert lib.shiftquant_gemm_layer(ctypes.byref(a), None, 0, st, None) == native.SQ_EINVAL
+
+
+def test_grid_barrier_selftest_validates_before_launch(lib):
+    st = ctypes.c_void_p(4096)
+    assert lib.shiftquant_selftest_grid_barrier_timeout(None, st, None) == native.SQ_EINVAL
+    assert lib.shiftquant_selftest_grid_barrier_timeout(ctypes.c_void_p(4100), st, None) == native.SQ_EINVAL
+    assert lib.shiftquant_selftest_grid_barrier_timeout(ctypes.c_void_p(4096), None, None) == native.SQ_EINVAL

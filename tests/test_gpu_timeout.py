@@ -63,3 +63,32 @@ def test_selftest_refuses_empty_or_large_launches():
     for M, Nn, K in ((0, 8, 64), (8, 8, 0), (5000, 8, 64)):
         with pytest.raises(N.ShiftQuantError):
             N.shiftquant_selftest_wait_timeout(a, one, a, one, M, Nn, K, 4, 4, y, st)
+
+
+def test_a_grid_barrier_that_runs_out_reports_timeout_and_the_context_stays_usable():
+    # the single-launch L1 batch normalization's grid barrier: one block never arrives, so
+    # every block's bounded wait runs out (about 1 s), records SQ_DEV_TIMEOUT and returns;
+    # an L1 batch normalization right after matches the oracle
+    scratch = torch.zeros(64, dtype=torch.int32, device="cuda")
+    st = torch.zeros(1, dtype=torch.int32, device="cuda")
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    N.shiftquant_selftest_grid_barrier_timeout(scratch, st)
+    torch.cuda.synchronize()
+    dt = time.perf_counter() - t0
+    assert st.item() & N.SQ_DEV_TIMEOUT, st.item()
+    assert dt < 30.0, dt
+    rng = np.random.default_rng(5)
+    R, C = 500, 48
+    x = rng.standard_normal((R, C)).astype(np.float32)
+    gamma = np.ones(C, np.float32)
+    beta = np.zeros(C, np.float32)
+    st2 = torch.zeros(1, dtype=torch.int32, device="cuda")
+    state = torch.zeros(N.shiftquant_l1bn_state_bytes(R, C), dtype=torch.uint8, device="cuda")
+    y = torch.empty((R, C), device="cuda")
+    N.shiftquant_l1bn_forward(to_gpu(x), torch.from_numpy(gamma).cuda(), torch.from_numpy(beta).cuda(),
+                              8, 4, y, state, st2)
+    torch.cuda.synchronize()
+    assert st2.item() == 0
+    f = O.l1bn_forward(x, gamma, beta, 8, 4)
+    np.testing.assert_array_equal(y.cpu().numpy().view(np.uint32), f["y"].view(np.uint32))
