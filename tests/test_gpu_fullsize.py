@@ -1,8 +1,10 @@
 """Parity at the benchmark's full sizes, in the launch configuration the benchmark times
-(the five-stream step captured in a CUDA graph), for every workload: the quantizer outputs
-of every tensor compared in full (ranges, tau_0, exponents, scales, codes and transposed
-codes, bit-exact), and the three GEMMs on sampled output rows (integer accumulators
-bit-exact, fp32 outputs within 1e-6 relative)."""
+(the five-stream step captured in a CUDA graph, each layer's X and dY codes with or
+without transposed copies as the library advises, as the benchmark builds them), for every
+workload: the quantizer outputs of every tensor compared in full (ranges, tau_0,
+exponents, scales, codes and, where kept, transposed codes, bit-exact), and the three GEMMs
+on sampled output rows (integer accumulators bit-exact, fp32 outputs within 1e-6
+relative)."""
 import numpy as np
 import pytest
 import torch
@@ -44,7 +46,8 @@ def _compare_shift(q, o, what):
     np.testing.assert_array_equal(q.exp.cpu().numpy(), o["exp"], what)
     assert f32_bits([q.scale.item()])[0] == f32_bits([o["scale"]])[0], what
     _compare_codes_chunked(q.codes, o["codes"], what + " codes")
-    _compare_codes_chunked(q.codes_t, o["codes"], what + " transposed codes", transpose=True)
+    if q.codes_t is not None:
+        _compare_codes_chunked(q.codes_t, o["codes"], what + " transposed codes", transpose=True)
 
 
 @pytest.mark.parametrize("name", ["wgrad_small", "conv3x3", "vit_mlp", "vit_block",
@@ -55,7 +58,9 @@ def test_workload_full_size(name):
     for li, spec in enumerate(wl.layers):
         x, w, dy = W.np_layer_inputs(spec, SEED, li)
         G, bits = spec.n_groups, spec.bits
-        lay = L.QuantLinear(spec.M, spec.K, spec.N, bits, G, "cuda", with_acc=True)
+        lay = L.QuantLinear(spec.M, spec.K, spec.N, bits, G, "cuda", with_acc=True, transposed=None)
+        want_t = N.shiftquant_gemm_layer_wgrad_in_place(spec.M, spec.K, spec.N, bits, G) != 1
+        assert (lay.x.codes_t is not None) == want_t
         xg, wg, dyg = (torch.from_numpy(a).cuda() for a in (x, w, dy))
         streams = [torch.cuda.Stream() for _ in range(5)]
         graph = L.CapturedStep(lambda: lay.step_concurrent(xg, wg, dyg, SR_SEED, streams))
