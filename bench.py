@@ -355,16 +355,20 @@ def run_ours(args, rank, world, local_rank):
     # A second capture of the same step with events around each layer's GEMM call (external
     # events are recorded as graph nodes) times the GEMM launches in graph replays; the
     # headline replays run the graph without them.
+    # (and an event at the start of each layer's step: the quantizer phase, as the step runs
+    # its three quantizer chains side by side, is the time from it to the GEMM call)
     try:
         gemm_ev = [(torch.cuda.Event(enable_timing=True, external=True),
                     torch.cuda.Event(enable_timing=True, external=True)) for _ in st.layers]
+        phase_ev = [torch.cuda.Event(enable_timing=True, external=True) for _ in st.layers]
     except TypeError:
-        gemm_ev = None
+        gemm_ev = phase_ev = None
 
     def run_step_concurrent(i, events=None):
         for li, (lay, (x, w, dy), ss) in enumerate(zip(st.layers, st.inputs, streams)):
             lay.step_concurrent(x, w, dy, 0x5EED + i, ss,
-                                gemm_events=events[li] if events else None)
+                                gemm_events=events[li] if events else None,
+                                start_event=phase_ev[li] if events else None)
 
     graph = L.CapturedStep(lambda: run_step_concurrent(args.warmup))
     for i in range(args.warmup):
@@ -392,6 +396,7 @@ def run_ours(args, rank, world, local_rank):
     ok = st.status_ok()
 
     graph_gemm_ms = []   # per layer and replay: the GEMM call inside a graph replay
+    graph_quant_ms = []  # per replay: the layers' quantizer phases (step start to GEMM call)
     if gemm_ev:
         graph_ev = L.CapturedStep(lambda: run_step_concurrent(args.warmup, gemm_ev))
         for i in range(args.steps):
@@ -399,6 +404,7 @@ def run_ours(args, rank, world, local_rank):
             graph_ev.replay()
             torch.cuda.synchronize()   # the events are recorded again by the next replay
             graph_gemm_ms += [e0.elapsed_time(e1) for e0, e1 in gemm_ev]
+            graph_quant_ms.append(sum(p.elapsed_time(e0) for p, (e0, _) in zip(phase_ev, gemm_ev)))
         del graph_ev
 
     # per-call breakdown: the same calls un-graphed, queued behind a sleep kernel so the
@@ -575,6 +581,15 @@ def run_ours(args, rank, world, local_rank):
                                 "ms_per_step": q_ms_ungraphed / args.steps,
                                 "timing": "the same calls launched one by one from the host, "
                                           "queued behind a sleep kernel, events between them"}}
+    if graph_quant_ms:
+        qs_ms = statistics.median(graph_quant_ms)
+        qs_gbs = st.quantizer_bytes() / (qs_ms * 1e-3) / 1e9
+        quant_roof["in_step"] = {
+            "achieved": qs_gbs, "frac": qs_gbs / peaks["hbm_gbs"], "ms_per_step": qs_ms,
+            "timing": "the quantizer phases of the step as it runs them (each layer's "
+                      "activation, gradient and weight chains side by side on their own "
+                      "streams): event nodes from the start of each layer's step to its "
+                      "GEMM call, in a graph replay after an L2 flush, median over replays"}
     # the dominant kernel: the kernel class (range pass, quantize, layer GEMM launch) of the
     # single launch with the most device time in the step
     def hbm_roof(nbytes, ms, name):
@@ -957,7 +972,8 @@ def main():
                                    "gemm": {k: other["gemm"][k] for k in ("achieved", "peak", "unit", "frac",
                                                                           "frac_of_clock_peak", "hbm_gbs",
                                                                           "hbm_frac")},
-                                   "quantizer": {k: other["quantizer"][k] for k in ("achieved", "peak", "unit", "frac")},
+                                   "quantizer": {k: other["quantizer"][k] for k in ("achieved", "peak", "unit", "frac", "in_step")
+                                                 if k in other["quantizer"]},
                                    "clocks": other["clocks"]})
         if world == 1 and not args.no_chain:
             result["fused_range_chain"] = run_chain(args, f"cuda:{local_rank}")

@@ -260,7 +260,8 @@ class QuantLinear:
         self.dgrad(stream)
         self.wgrad(stream)
 
-    def step_concurrent(self, x, w, dy, seed, streams, gemm_events=None, dgrad_ctas=0):
+    def step_concurrent(self, x, w, dy, seed, streams, gemm_events=None, dgrad_ctas=0,
+                        start_event=None):
         """The same step with its independent quantizer work on three streams forked from the
         current one -- the activation chain, the gradient chain and the weight (its range
         pass right away, its quantization for both roles once both other operands'
@@ -268,12 +269,16 @@ class QuantLinear:
         current stream.
         Capturable in a CUDA graph, which then runs the independent work concurrently.
         gemm_events: optional (start, end) CUDA events recorded around the GEMM call (for
-        timing inside a captured graph they must be created with external=True).
+        timing inside a captured graph they must be created with external=True);
+        start_event: optional event recorded on the current stream before anything else
+        (with gemm_events[0]: the quantizer phase of the step).
         dgrad_ctas > 0: the loss-propagation GEMM (which needs only dY's and W's codes) runs
         as its own launch of at most that many CTAs on the gradient stream as soon as its
         operands exist, beside the activation chain; the forward and weight-gradient GEMMs
         follow as one launch."""
         main = torch.cuda.current_stream()
+        if start_event is not None:
+            start_event.record(main)
         s_x, s_g, s_w = streams[:3]
         for s in (s_x, s_g, s_w):
             s.wait_stream(main)
